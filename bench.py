@@ -1,0 +1,357 @@
+"""Benchmark of the heterogeneous data-parallel SGD step (arXiv 2110.08941) on GB300.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--impl ours|reference]
+
+A step is one synchronous SGD step of the whole hot path through libhs: per-worker forward and
+backward over M = 16 compute-proportional segments of a 16384-sample batch (MLP
+4096 -> 8192 -> 8192 -> 1000, bf16 tensor cores), softmax cross-entropy, per-worker gradient
+slabs, and the fused reduce + update.  Inputs are seeded synthetic data already resident in
+HBM; the working set (activations and 7 GB of gradient slabs) is far larger than L2, so no
+explicit L2 flush is needed between steps.
+
+Prints ONE JSON line (rank 0).  With --gpus N > 1 (launched by torch.distributed.run) every rank
+runs an independent replica of the workload (the one-GPU method has no cross-GPU exchange in
+this build): weak scaling, value = all ranks' samples / max-over-ranks time.
+
+--impl reference times the fp64 CPU oracle on the host cores (bounded samples of the same
+workload), the reference arm of this build.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import synth  # noqa: E402
+
+METRIC = "samples/sec per synchronous SGD step on 1 GB300"
+UNIT = "samples/s"
+DEFAULT_WORKLOAD = synth.CFG5
+
+
+def _peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        d = json.load(open(path))
+        return dict(hbm=d["hbm_gbs"], bf16=d["bf16_tflops"], bf16_sust=d.get("bf16_tflops_sustained", d["bf16_tflops"]),
+                    src="measured")
+    return dict(hbm=6800.0, bf16=1900.0, bf16_sust=1700.0, src="fallback")
+
+
+# ------------------------------------------------------------------------------ clocks
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.lines = []
+        self.thread = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits", "-lms", "200",
+                 "-i", str(self.gpu)], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except (FileNotFoundError, OSError):
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        if self.thread:
+            self.thread.join(timeout=2)
+        sm, smax, reasons = [], [], set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for ln in self.lines:
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                smax.append(float(parts[2]))
+            except ValueError:
+                continue
+            for nm, val in zip(names, parts[5:9]):
+                if val.lower() == "active":
+                    reasons.add(nm)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(smax), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ------------------------------------------------------------------------------ workload math
+def gemm_flops(wl):
+    dims = wl.dims
+    sw = sum(dims[l] * dims[l - 1] for l in range(1, len(dims)))
+    sw_dgrad = sum(dims[l] * dims[l - 1] for l in range(2, len(dims)))
+    n = wl.global_batch
+    return dict(forward=2.0 * n * sw, wgrad=2.0 * n * sw, dgrad=2.0 * n * sw_dgrad)
+
+
+def update_bytes(wl, P):
+    # M slab reads + theta read, theta write + bf16 shadow write
+    return (wl.workers + 2) * P * 4 + 2 * P
+
+
+# ------------------------------------------------------------------------------ CPU oracle baseline
+def oracle_sample(wl, seconds_target=12.0, max_workers=None):
+    """Time the oracle (as it stands) on whole worker segments of the workload: the smallest
+    workers first, adding workers until about `seconds_target` of CPU time.  Returns
+    (samples/s, description, cores)."""
+    from oracle import mlp, sgd
+    from oracle import partition as P
+
+    try:
+        from threadpoolctl import threadpool_info
+        threads = max([i.get("num_threads", 1) for i in threadpool_info()] or [1])
+    except Exception:
+        threads = os.cpu_count()
+    x, y = synth.make_batch(wl)
+    theta = synth.make_params(wl).astype(np.float64)
+    sizes = P.partition_sizes(list(synth.initial_weights(wl)), wl.global_batch)
+    off = P.offsets(sizes)
+    order = sorted(range(wl.workers), key=lambda m: sizes[m])
+    if max_workers:
+        order = order[:max_workers]
+    done_samples, elapsed, used = 0, 0.0, []
+    for m in order:
+        xs, ys = x[off[m]:off[m + 1]], y[off[m]:off[m + 1]]
+        t0 = time.perf_counter()
+        sgd.step(mlp.worker_loss_grad, theta, wl.dims, xs, ys, [sizes[m]], wl.lr, sgd.SYNC_CP_WEIGHTED)
+        elapsed += time.perf_counter() - t0
+        done_samples += sizes[m]
+        used.append(m)
+        if elapsed >= seconds_target:
+            break
+    desc = (f"oracle fp64 step (forward, backward, weighted accumulation, update) over the whole segments "
+            f"of workers {used} ({done_samples} samples) of {wl.name}")
+    return done_samples / elapsed, desc, threads
+
+
+# ------------------------------------------------------------------------------ arms
+def run_reference(args, wl, rank, world):
+    if rank != 0:
+        return
+    from oracle import mlp, sgd
+    from oracle import partition as P
+    try:
+        from threadpoolctl import threadpool_info
+        cores = max([i.get("num_threads", 1) for i in threadpool_info()] or [1])
+    except Exception:
+        cores = os.cpu_count()
+    x, y = synth.make_batch(wl)
+    theta = synth.make_params(wl).astype(np.float64)
+    sizes = P.partition_sizes(list(synth.initial_weights(wl)), wl.global_batch)
+    off = P.offsets(sizes)
+    m = min(range(wl.workers), key=lambda k: sizes[k])      # smallest worker segment per step
+    xs, ys = x[off[m]:off[m + 1]], y[off[m]:off[m + 1]]
+
+    def one():
+        nonlocal theta
+        theta, _, _, _, _ = sgd.step(mlp.worker_loss_grad, theta, wl.dims, xs, ys, [sizes[m]], wl.lr,
+                                     sgd.SYNC_CP_WEIGHTED)
+
+    for _ in range(args.warmup):
+        one()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        one()
+    dt = time.perf_counter() - t0
+    value = sizes[m] * args.steps / dt
+    sample = (f"each step: oracle fp64 step over worker {m}'s whole segment ({sizes[m]} samples) of {wl.name}")
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * dt / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": {"workload": wl.name, "global_batch": wl.global_batch,
+                                            "workers": wl.workers},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": sample},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def run_ours(args, wl, rank, world, local_rank):
+    import torch
+    import paper_2110_08941_gb300 as hs
+
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist_mod
+        dist = dist_mod
+
+    def barrier():
+        if dist is not None:
+            dist.barrier()
+
+    precision = hs.HS_BF16 if args.precision == "bf16" else hs.HS_FP32_CHECK
+    x, y = synth.make_batch(wl)
+    theta0 = synth.make_params(wl)
+    w = synth.initial_weights(wl)
+    ctx = hs.hs_init(wl.arch, wl.dims, wl.workers, wl.global_batch, compute_weights=w, precision=precision,
+                     sync=hs.HS_SYNC_CP_WEIGHTED)
+    params = torch.from_numpy(theta0).to(dev)
+    xd = torch.from_numpy(x).to(dev)
+    yd = torch.from_numpy(y).to(dev)
+    stream = torch.cuda.current_stream(dev)
+    part = ctx.partition
+
+    for _ in range(args.warmup):
+        hs.hs_step(ctx, params, xd, yd, part, wl.lr, stream=stream, want_loss=False)
+    torch.cuda.synchronize()
+    hs.hs_read_profile(ctx)                 # discard warm-up counts
+    hs.hs_set_profiling(ctx, True)
+
+    clocks = ClockSampler(local_rank)
+    clocks.start()
+    time.sleep(0.3)
+    barrier()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        hs.hs_step(ctx, params, xd, yd, part, wl.lr, stream=stream, want_loss=False)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    clk = clocks.stop()
+    ms = e0.elapsed_time(e1)
+    prof = hs.hs_read_profile(ctx)
+    hs.hs_set_profiling(ctx, False)
+    if dist is not None:
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    loss = hs.hs_step(ctx, params, xd, yd, part, 0.0, stream=stream, want_loss=True)   # finite-loss check
+
+    # end to end through the public API: host (pinned) inputs, loss read back every step
+    xh = torch.from_numpy(x).pin_memory()
+    yh = torch.from_numpy(y).pin_memory()
+    k_e2e = max(3, min(args.steps, 10))
+    hs.hs_step(ctx, params, xh, yh, part, wl.lr, stream=stream, want_loss=True)
+    barrier()
+    t0 = time.perf_counter()
+    for _ in range(k_e2e):
+        hs.hs_step(ctx, params, xh, yh, part, wl.lr, stream=stream, want_loss=True)
+    e2e_s = time.perf_counter() - t0
+    if dist is not None:
+        t = torch.tensor([e2e_s], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_s = float(t.item())
+
+    P = ctx.P
+    peaks = _peaks()
+    flops = gemm_flops(wl)
+    per_step = {k: v[0] / args.steps for k, v in prof.items()}
+    launches = sum(v[1] for v in prof.values())
+    gemm_phase = max(("forward", "wgrad", "dgrad"), key=lambda k: per_step[k])
+    upd_bytes = update_bytes(wl, P)
+    candidates = {k: per_step[k] for k in ("forward", "wgrad", "dgrad", "update")}
+    dominant = max(candidates, key=candidates.get)
+
+    def gemm_roof(name):
+        ach = flops[name] / (per_step[name] * 1e-3) / 1e12
+        return {"kernel": f"tc_gemm ({name})", "bound": "tensor", "achieved": ach, "peak": peaks["bf16_sust"],
+                "unit": "TFLOP/s", "frac": ach / peaks["bf16_sust"], "traffic": None,
+                "peak_kind": f"{peaks['src']} bf16 sustained"}
+
+    upd_ach = upd_bytes / (per_step["update"] * 1e-3) / 1e9
+    roof_update = {"kernel": "reduce_update", "bound": "hbm", "achieved": upd_ach, "peak": peaks["hbm"],
+                   "unit": "GB/s", "frac": upd_ach / peaks["hbm"], "traffic": None,
+                   "peak_kind": f"{peaks['src']} copy bandwidth", "algorithmic_bytes": upd_bytes}
+    roofline = roof_update if dominant == "update" else gemm_roof(dominant)
+    gemm_ms = per_step["forward"] + per_step["wgrad"] + per_step["dgrad"]
+    gemm_total = sum(flops.values())
+    out = None
+    if rank == 0:
+        cpu = None
+        if world == 1 and not args.no_cpu_baseline:
+            v, desc, cores = oracle_sample(wl)
+            cpu = {"value": v, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": desc}
+        value = world * wl.global_batch * args.steps / (ms * 1e-3)
+        out = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16" if precision == hs.HS_BF16 else "f32", "data": "synthetic",
+            "config": {"workload": wl.name, "global_batch": wl.global_batch, "workers": wl.workers,
+                       "dims": list(wl.dims), "sync": "cp_weighted", "parallelism": f"replicas{world}",
+                       "l2": "working set > L2 (7 GB slabs, 0.9 GB activations per step), no flush"},
+            "roofline": roofline,
+            "roofline_gemm_phase": {"bound": "tensor", "achieved": gemm_total / (gemm_ms * 1e-3) / 1e12,
+                                    "peak": peaks["bf16_sust"], "unit": "TFLOP/s",
+                                    "frac": gemm_total / (gemm_ms * 1e-3) / 1e12 / peaks["bf16_sust"],
+                                    "flops_per_step": gemm_total},
+            "roofline_reduce_update": roof_update,
+            "phases_ms_per_step": per_step,
+            "gpu_launches": int(launches),
+            "cpu_baseline": cpu,
+            "e2e": {"value": world * wl.global_batch * k_e2e / e2e_s, "unit": UNIT,
+                    "h2d_bytes_per_step": int(x.nbytes + y.nbytes), "d2h_bytes_per_step": 12},
+            "clocks": clk,
+            "loss_after": loss,
+        }
+        print(json.dumps(out), flush=True)
+    ctx.close()
+    return out
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(synth.WORKLOADS))
+    ap.add_argument("--impl", default="ours", choices=("ours", "reference"))
+    ap.add_argument("--precision", default="bf16", choices=("bf16", "fp32"))
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3 and args.impl == "ours":
+        args.warmup = 3
+    wl = synth.WORKLOADS[args.workload]
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        run_reference(args, wl, rank, world)
+        return
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+        torch.cuda.set_device(local_rank)
+        dist.init_process_group("nccl")
+    try:
+        run_ours(args, wl, rank, world, local_rank)
+    finally:
+        if world > 1:
+            import torch.distributed as dist
+            dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

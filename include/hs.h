@@ -1,0 +1,205 @@
+/*
+ * hs.h - C ABI of libhs: one synchronous data-parallel SGD step over M logical
+ * workers whose partitions follow their compute power (arXiv 2110.08941).
+ *
+ * The paper's method in the terms used here:
+ *   - Section 1: M workers each compute a stochastic gradient g^m_t of their
+ *     local objective f_m (Eq. 1, the mean loss over the worker's data); the
+ *     gradients are averaged, g_t = (1/M) sum_m g^m_t, and the model is updated
+ *     theta_{t+1} = theta_t - eta_t g_t.
+ *   - Section 4, Eq. 2: compute power CP_m = |D_m| / X_m (samples per second).
+ *   - Section 4.1, Algorithm 1 (Dynamic Partitioning): normalise the CPs and
+ *     size worker m's partition as CP_m * |D|; the first partition is even.
+ *   - Section 4.2 (Enhanced Dynamic Partitioning): weight each g^m by the
+ *     normalised compute power before the gradient exchange.
+ *
+ * On one GPU the M workers are contiguous segments of one global minibatch:
+ * worker m owns samples [off_m, off_m + n_m).  Each segment gets its own
+ * forward and backward pass (the per-worker gradient slab G_m), then one fused
+ * pass reduces sum_m w_m G_m and applies the update.
+ *
+ * Conventions for every entry point:
+ *   - Pointers marked "device" are CUDA device pointers on the device that was
+ *     current at hs_init; "host" pointers are ordinary CPU memory.  The library
+ *     never takes ownership of caller memory.
+ *   - `stream` is a cudaStream_t (NULL = legacy default stream).  Work is
+ *     enqueued on it; calls return before the GPU finishes unless stated.
+ *   - Every call returns an hs_status and never throws or aborts.  Invalid
+ *     arguments are rejected on the host before any GPU work is enqueued; the
+ *     message is available from hs_last_error(ctx).
+ *   - A context is not thread-safe and is meant for one stream at a time.
+ */
+#ifndef HS_H_
+#define HS_H_
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct hs_ctx hs_ctx;
+
+typedef enum {
+  HS_OK = 0,
+  HS_ERR_INVALID_ARG = 1,   /* bad pointer, size, enum or numeric value; nothing was enqueued */
+  HS_ERR_CUDA = 2,          /* a CUDA runtime call failed (message has the CUDA error string) */
+  HS_ERR_OOM = 3,           /* device workspace allocation failed */
+  HS_ERR_UNSUPPORTED = 4,   /* valid request outside what this build implements */
+  HS_ERR_DEVICE_CHECK = 5   /* a kernel's own check failed (bounded wait timed out); results invalid */
+} hs_status;
+
+typedef enum { HS_MLP = 0, HS_CNN = 1 } hs_arch;
+
+/* HS_BF16: bf16 tensor-core operands (tcgen05), fp32 accumulation, fp32 master
+ * parameters and fp32 gradient slabs.  HS_FP32_CHECK: the same step with every
+ * contraction in fp32 on the CUDA cores (a check path for tight parity). */
+typedef enum { HS_BF16 = 0, HS_FP32_CHECK = 1 } hs_precision;
+
+/* Gradient synchronisation weights w_m in g = sum_m w_m g^m:
+ *   HS_SYNC_MEAN        w_m = 1/M                  (Section 1, Sync-SGD / DP-SGD)
+ *   HS_SYNC_CP_WEIGHTED w_m = n_m / N              (Section 4.2, EDP-SGD: the normalised
+ *                                                   compute power as realised by the integer
+ *                                                   partition; weights sum to 1)
+ *   HS_SYNC_CP_LITERAL  w_m = (CP_m / sum CP) / M  (Section 4.2 read literally: weight, then
+ *                                                   the averaging exchange of Section 1) */
+typedef enum { HS_SYNC_MEAN = 0, HS_SYNC_CP_WEIGHTED = 1, HS_SYNC_CP_LITERAL = 2 } hs_sync;
+
+/* Model description (all fields 32-bit for a stable ABI).
+ *   MLP: dims[0..n_layers] = d0 (input features), hidden widths, d_L = classes.
+ *        Layer l: A_l = H_{l-1} W_l^T + b_l, ReLU on every layer but the last.
+ *        HS_BF16 needs d0..d_{L-1} to be multiples of 8 (16-byte rows for TMA).
+ *   CNN: dims[0..6] = Cin, H, W, c1, c2, c3, classes: three 3x3 convs with
+ *        padding 1 and strides 1, 2, 2 (ReLU after each), global average pool,
+ *        one fully connected layer.  n_layers is ignored.
+ * Parameter layout (flat fp32): [W1, b1, W2, b2, ...]; linear W row-major
+ * [out, in]; conv W [Cout, Cin, 3, 3]; fc W [classes, c3]. */
+typedef struct {
+  int32_t arch;        /* hs_arch */
+  int32_t n_layers;
+  const int32_t* dims; /* host; copied by hs_init */
+  int32_t precision;   /* hs_precision */
+  int32_t sync;        /* hs_sync */
+} hs_model_desc;
+
+/* A partition as produced by hs_partition (Algorithm 1).  All pointers are
+ * owned by the context and stay valid until the next hs_partition call on it
+ * or hs_destroy. */
+typedef struct {
+  int32_t M, N;
+  const int32_t* counts_host;   /* host [M]: n_m, sum = N, each >= 1 */
+  const int32_t* offsets_host;  /* host [M+1]: exclusive prefix sum, offsets[M] = N */
+  const int32_t* index_map_dev; /* device [N]: index_map[i] = m for offsets[m] <= i < offsets[m+1] */
+  const double* weights_host;   /* host [M]: synchronisation weights w_m of the context's hs_sync */
+  const double* cp_host;        /* host [M]: normalised compute power the sizes were drawn from */
+  uint64_t version;             /* increments on every hs_partition call that changes the sizes */
+} hs_partition_t;
+
+/* Algorithm 1's sizing rule on the host, no GPU involved (Section 4.1,
+ * Algorithm 1; Eq. 2 gives the CPs).  counts_out[m] = n_m from compute powers
+ * cp[0..M-1] (any positive scale) over a batch of N samples:
+ *   S = sum cp (fp64, left to right); q_m = (cp_m / S) * N; n_m = floor(q_m),
+ *   then N - sum floor(q) extra samples to the largest remainders q_m - floor(q_m)
+ *   (ties: lower m); finally every worker with 0 samples takes one from the
+ *   largest worker (ties: lower m).
+ * Errors: HS_ERR_INVALID_ARG if M < 1, N < M, a null pointer, or any cp not
+ * finite and > 0.  counts_out is host [M], caller-owned. */
+hs_status hs_partition_sizes(int32_t M, int32_t N, const double* cp, int32_t* counts_out);
+
+/* Number of fp32 parameters P of a model (layout above).  Host only. */
+hs_status hs_param_count(const hs_model_desc* model, int64_t* P);
+
+/* Create a context on the current CUDA device for global batch N = global_batch
+ * split over M workers.  compute_weights: host [M] initial compute powers, or
+ * NULL for the even split of Algorithm 1's first epoch (t = 0).  Allocates all
+ * device workspace (per-worker gradient slabs M x P fp32, activations for N
+ * rows, the bf16 parameter shadow) and computes the initial partition
+ * synchronously.  Errors: HS_ERR_INVALID_ARG (bad model/M/N/weights),
+ * HS_ERR_UNSUPPORTED (shape constraint of the precision), HS_ERR_OOM,
+ * HS_ERR_CUDA.  On error *out is NULL. */
+hs_status hs_init(const hs_model_desc* model, int32_t M, const double* compute_weights,
+                  int32_t global_batch, hs_ctx** out);
+
+/* Dynamic Partitioning (Section 4.1, Algorithm 1; Eq. 2).  measured_throughputs:
+ * host [M], CP_m = |D_m| / X_m in samples per second measured by the caller over
+ * the last epoch (or window); NULL keeps the current partition.  The new sizes
+ * follow hs_partition_sizes; the sample->worker map is rebuilt on the device
+ * (contiguous segments in worker order) on `stream`.
+ * Outputs (each may be NULL): counts_out host [M]; index_map_out device [N]
+ * int32 (written on `stream`); out receives the partition view.
+ * Errors: HS_ERR_INVALID_ARG (non-finite or <= 0 throughput); nothing changes. */
+hs_status hs_partition(hs_ctx* ctx, const double* measured_throughputs, int32_t* counts_out,
+                       int32_t* index_map_out, void* stream, hs_partition_t* out);
+
+/* One synchronous SGD step (Section 1; Eq. 1; Section 4.2 for the weights).
+ *   params: device fp32 [P], updated in place: theta <- theta - lr * sum_m w_m G_m,
+ *           where G_m is the gradient of worker m's mean cross-entropy over its segment.
+ *   x:      fp32 [N, features] (MLP) or [N, Cin, H, W] (CNN, NCHW), row-major.
+ *   y:      int32 [N], class labels in [0, classes).
+ *           x and y may be device pointers or host pointers (pinned or pageable);
+ *           host inputs are copied to a context-owned device buffer on `stream`.
+ *   part:   the context's current partition (from hs_init/hs_partition), or NULL
+ *           for the same; a stale version is rejected.
+ *   loss_out: host float, or NULL.  When non-NULL the call waits for the step and
+ *           returns loss = sum_m w_m L_m at the parameters before the update; it
+ *           also reports HS_ERR_DEVICE_CHECK if a kernel's bounded wait expired.
+ *           When NULL the call is fully asynchronous.
+ * Labels outside [0, classes) are clamped by the loss kernel and counted as an
+ * error reported through HS_ERR_DEVICE_CHECK at the next synchronising call. */
+hs_status hs_step(hs_ctx* ctx, float* params, const void* x, const int32_t* y,
+                  const hs_partition_t* part, float lr, void* stream, float* loss_out);
+
+/* The bf16 parameter shadow is refreshed by every hs_step for the params
+ * pointer it updated.  A caller that writes params in place between steps
+ * (checkpoint restore, manual edits) calls this to re-derive the shadow. */
+hs_status hs_sync_params(hs_ctx* ctx, const float* params, void* stream);
+
+/* Keep a copy of the synchronised gradient g from each hs_step (costs one
+ * extra P x 4 byte write per step).  Off by default. */
+hs_status hs_set_debug(hs_ctx* ctx, int32_t enable);
+
+/* Copy the last step's synchronised gradient g (device fp32 [P]; needs
+ * hs_set_debug(ctx, 1) before that step, else HS_ERR_INVALID_ARG) and/or the
+ * per-worker gradient slabs G_m (device fp32 [M, P], row m = worker m).  Either
+ * pointer may be NULL.  Copies are enqueued on `stream`. */
+hs_status hs_debug_grads(hs_ctx* ctx, float* g_out, float* slabs_out, void* stream);
+
+/* Per-worker losses L_m of the last step (host float [M]); synchronises. */
+hs_status hs_worker_losses(hs_ctx* ctx, float* losses_out);
+
+/* Phases of hs_step for device-side timing (CUDA events recorded on the step's stream). */
+typedef enum {
+  HS_PHASE_CAST = 0,      /* fp32 -> bf16 casts of the inputs (and of params after an external change) */
+  HS_PHASE_FORWARD = 1,   /* per-worker forward products, bias + ReLU fused (Eq. 1 f_m) */
+  HS_PHASE_LOSS = 2,      /* softmax cross-entropy, loss gradient, per-worker mean losses L_m */
+  HS_PHASE_WGRAD = 3,     /* per-worker weight gradients G_m (grouped over the worker segments) */
+  HS_PHASE_BIASGRAD = 4,  /* per-worker bias gradients */
+  HS_PHASE_DGRAD = 5,     /* input gradients with the ReLU derivative fused */
+  HS_PHASE_UPDATE = 6,    /* g = sum_m w_m G_m fused with theta <- theta - lr g (Section 1) */
+  HS_PHASE_COUNT = 7
+} hs_phase;
+
+/* Record CUDA events around every phase of each hs_step while enabled (adds two event
+ * records per phase on the step's stream; off by default). */
+hs_status hs_set_profiling(hs_ctx* ctx, int32_t enable);
+
+/* Sum of device time (ms) and kernel launches per phase over the steps since the last read,
+ * then reset.  ms_out and launches_out are host [HS_PHASE_COUNT] (either may be NULL).
+ * Waits for the recorded events.  Launch counts are kept whether or not profiling is on. */
+hs_status hs_read_profile(hs_ctx* ctx, double* ms_out, int64_t* launches_out);
+
+/* Free the context and all its device memory (synchronises the device first).
+ * NULL is a no-op. */
+void hs_destroy(hs_ctx* ctx);
+
+const char* hs_status_string(hs_status s);
+/* Last error message of the context ("" if none).  For hs_init failures use
+ * hs_last_init_error().  The string is owned by the library. */
+const char* hs_last_error(const hs_ctx* ctx);
+const char* hs_last_init_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* HS_H_ */

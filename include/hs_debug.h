@@ -1,0 +1,44 @@
+/*
+ * hs_debug.h - test hook into libhs's tensor-core GEMM.
+ *
+ * Not part of the training API.  It runs one product through the same
+ * tcgen05/TMA kernel that hs_step uses for the per-worker forward and backward
+ * passes (Eq. 1's per-worker gradients g^m, Section 1), so tests can check that
+ * kernel in isolation against a plain reference.  All matrix pointers are
+ * device pointers, row-major, with leading dimensions in elements; the call is
+ * synchronous (it waits for the kernel and reports launch/runtime errors).
+ */
+#ifndef HS_DEBUG_H_
+#define HS_DEBUG_H_
+
+#include <stdint.h>
+
+#include "hs.h"
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+enum {
+  HS_GEMM_FWD_RELU = 0,   /* D bf16 [M,N] = relu(A[M,K] B[N,K]^T + bias[N])           */
+  HS_GEMM_FWD_LOGITS = 1, /* D fp32 [M,N] = A[M,K] B[N,K]^T + bias[N]                  */
+  HS_GEMM_DGRAD = 2,      /* D bf16 [M,N] = (A[M,K] B[K,N]) * (Z[M,N] > 0)              */
+  HS_GEMM_WGRAD = 3       /* D_g fp32 [M,N] = A[k_g, M]^T B[k_g, N] for each group g:   */
+                          /*   rows k of A [K,M] and B [K,N] in [k_off[g], k_off[g+1]), */
+                          /*   D_g at D + g * d_gstride                                  */
+};
+
+/* A, B, Z: bf16; bias: fp32 [N]; k_offsets_host: host int32 [groups+1] (HS_GEMM_WGRAD only,
+ * else NULL with groups = 1).  Returns HS_ERR_INVALID_ARG for shapes the kernel cannot take
+ * (leading dimensions must be multiples of 8 elements, pointers 16-byte aligned),
+ * HS_ERR_CUDA on a launch or runtime error. */
+hs_status hs_debug_gemm_bf16(int32_t mode, int32_t M, int32_t N, int32_t K, const void* A, int64_t lda,
+                             const void* B, int64_t ldb, void* D, int64_t ldd, const float* bias,
+                             const void* Z, int64_t ldz, const int32_t* k_offsets_host, int32_t groups,
+                             int64_t d_gstride, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* HS_DEBUG_H_ */

@@ -1,0 +1,252 @@
+"""Python binding of libhs (include/hs.h): argument marshalling only.
+
+Every function keeps the C name.  Tensors are torch tensors; the binding passes
+their data pointers and the current CUDA stream to the library and does no
+arithmetic of its own.  The shared library is built in-tree by
+``python -m paper_2110_08941_gb300.build``; importing this package when it is
+missing raises ImportError - there is no fallback path.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from ctypes import POINTER, c_double, c_float, c_int32, c_int64, c_uint64, c_void_p
+from typing import List, Optional, Sequence
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libhs.so")
+
+HS_OK, HS_ERR_INVALID_ARG, HS_ERR_CUDA, HS_ERR_OOM, HS_ERR_UNSUPPORTED, HS_ERR_DEVICE_CHECK = range(6)
+HS_MLP, HS_CNN = 0, 1
+HS_BF16, HS_FP32_CHECK = 0, 1
+HS_SYNC_MEAN, HS_SYNC_CP_WEIGHTED, HS_SYNC_CP_LITERAL = 0, 1, 2
+HS_GEMM_FWD_RELU, HS_GEMM_FWD_LOGITS, HS_GEMM_DGRAD, HS_GEMM_WGRAD = 0, 1, 2, 3
+
+EXPORTED = ("hs_partition_sizes", "hs_param_count", "hs_init", "hs_partition", "hs_step", "hs_sync_params",
+            "hs_set_debug", "hs_debug_grads", "hs_worker_losses", "hs_destroy", "hs_status_string",
+            "hs_last_error", "hs_last_init_error", "hs_debug_gemm_bf16", "hs_set_profiling", "hs_read_profile")
+PHASES = ("cast", "forward", "loss", "wgrad", "biasgrad", "dgrad", "update")
+
+
+class HsError(RuntimeError):
+    def __init__(self, status: int, msg: str):
+        self.status = status
+        super().__init__(f"{_status_name(status)}: {msg}")
+
+
+class hs_model_desc(ctypes.Structure):
+    _fields_ = [("arch", c_int32), ("n_layers", c_int32), ("dims", POINTER(c_int32)),
+                ("precision", c_int32), ("sync", c_int32)]
+
+
+class hs_partition_t(ctypes.Structure):
+    _fields_ = [("M", c_int32), ("N", c_int32), ("counts_host", POINTER(c_int32)),
+                ("offsets_host", POINTER(c_int32)), ("index_map_dev", c_void_p),
+                ("weights_host", POINTER(c_double)), ("cp_host", POINTER(c_double)), ("version", c_uint64)]
+
+
+def _load() -> ctypes.CDLL:
+    if not os.path.exists(LIB_PATH):
+        raise ImportError(f"libhs.so not built at {LIB_PATH}; run `python -m paper_2110_08941_gb300.build`")
+    lib = ctypes.CDLL(LIB_PATH)
+    S = c_int32
+    sig = {
+        "hs_partition_sizes": (S, [c_int32, c_int32, POINTER(c_double), POINTER(c_int32)]),
+        "hs_param_count": (S, [POINTER(hs_model_desc), POINTER(c_int64)]),
+        "hs_init": (S, [POINTER(hs_model_desc), c_int32, POINTER(c_double), c_int32, POINTER(c_void_p)]),
+        "hs_partition": (S, [c_void_p, POINTER(c_double), POINTER(c_int32), c_void_p, c_void_p,
+                             POINTER(hs_partition_t)]),
+        "hs_step": (S, [c_void_p, c_void_p, c_void_p, c_void_p, POINTER(hs_partition_t), c_float, c_void_p,
+                        POINTER(c_float)]),
+        "hs_sync_params": (S, [c_void_p, c_void_p, c_void_p]),
+        "hs_set_debug": (S, [c_void_p, c_int32]),
+        "hs_set_profiling": (S, [c_void_p, c_int32]),
+        "hs_read_profile": (S, [c_void_p, POINTER(c_double), POINTER(c_int64)]),
+        "hs_debug_grads": (S, [c_void_p, c_void_p, c_void_p, c_void_p]),
+        "hs_worker_losses": (S, [c_void_p, POINTER(c_float)]),
+        "hs_destroy": (None, [c_void_p]),
+        "hs_status_string": (ctypes.c_char_p, [c_int32]),
+        "hs_last_error": (ctypes.c_char_p, [c_void_p]),
+        "hs_last_init_error": (ctypes.c_char_p, []),
+        "hs_debug_gemm_bf16": (S, [c_int32, c_int32, c_int32, c_int32, c_void_p, c_int64, c_void_p, c_int64,
+                                   c_void_p, c_int64, c_void_p, c_void_p, c_int64, POINTER(c_int32), c_int32,
+                                   c_int64, c_void_p]),
+    }
+    for name, (res, args) in sig.items():
+        fn = getattr(lib, name)
+        fn.restype = res
+        fn.argtypes = args
+    return lib
+
+
+_lib = _load()
+
+
+def _status_name(s: int) -> str:
+    return _lib.hs_status_string(s).decode()
+
+
+def _check(status: int, ctx_ptr=None, init: bool = False):
+    if status == HS_OK:
+        return
+    if init or ctx_ptr is None:
+        msg = _lib.hs_last_init_error().decode()
+    else:
+        msg = _lib.hs_last_error(ctx_ptr).decode()
+    raise HsError(status, msg)
+
+
+def _stream_ptr(stream) -> int:
+    import torch
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return int(stream.cuda_stream) if hasattr(stream, "cuda_stream") else int(stream)
+
+
+def _desc(arch: int, dims: Sequence[int], precision: int, sync: int):
+    arr = (c_int32 * len(dims))(*[int(d) for d in dims])
+    n_layers = len(dims) - 1 if arch == HS_MLP else 0
+    return hs_model_desc(arch, n_layers, ctypes.cast(arr, POINTER(c_int32)), precision, sync), arr
+
+
+# ------------------------------------------------------------------------------- host-only calls
+def hs_partition_sizes(cp: Sequence[float], n: int) -> List[int]:
+    m = len(cp)
+    cpa = (c_double * max(m, 1))(*[float(v) for v in cp])
+    out = (c_int32 * max(m, 1))()
+    _check(_lib.hs_partition_sizes(m, int(n), cpa, out))
+    return list(out[:m])
+
+
+def hs_param_count(arch: int, dims: Sequence[int]) -> int:
+    d, keep = _desc(arch, dims, HS_BF16, HS_SYNC_MEAN)
+    p = c_int64()
+    _check(_lib.hs_param_count(ctypes.byref(d), ctypes.byref(p)))
+    return p.value
+
+
+# ------------------------------------------------------------------------------- context
+class Partition:
+    """Snapshot of hs_partition_t (host arrays copied out)."""
+
+    def __init__(self, raw: hs_partition_t):
+        self.raw = raw
+        self.M, self.N, self.version = raw.M, raw.N, raw.version
+        self.counts = [raw.counts_host[i] for i in range(raw.M)]
+        self.offsets = [raw.offsets_host[i] for i in range(raw.M + 1)]
+        self.weights = [raw.weights_host[i] for i in range(raw.M)]
+        self.cp = [raw.cp_host[i] for i in range(raw.M)]
+        self.index_map_dev = raw.index_map_dev
+
+
+class Context:
+    def __init__(self, ptr: int, arch: int, dims, M: int, N: int, P: int, precision: int, sync: int):
+        self.ptr = c_void_p(ptr)
+        self.arch, self.dims, self.M, self.N, self.P = arch, tuple(dims), M, N, P
+        self.precision, self.sync = precision, sync
+        self.partition: Optional[Partition] = None
+
+    def close(self):
+        if self.ptr and self.ptr.value:
+            _lib.hs_destroy(self.ptr)
+            self.ptr = c_void_p(0)
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+def hs_init(arch: int, dims: Sequence[int], M: int, global_batch: int, compute_weights=None,
+            precision: int = HS_BF16, sync: int = HS_SYNC_CP_WEIGHTED) -> Context:
+    d, keep = _desc(arch, dims, precision, sync)
+    cw = None
+    if compute_weights is not None:
+        cw = (c_double * M)(*[float(v) for v in compute_weights])
+    out = c_void_p()
+    _check(_lib.hs_init(ctypes.byref(d), int(M), cw, int(global_batch), ctypes.byref(out)), init=True)
+    ctx = Context(out.value, arch, dims, M, global_batch, hs_param_count(arch, dims), precision, sync)
+    ctx.partition = hs_partition(ctx)
+    return ctx
+
+
+def hs_partition(ctx: Context, measured_throughputs=None, index_map_out=None, stream=None) -> Partition:
+    tp = None
+    if measured_throughputs is not None:
+        tp = (c_double * ctx.M)(*[float(v) for v in measured_throughputs])
+    raw = hs_partition_t()
+    im = None
+    if index_map_out is not None:
+        import torch
+        assert index_map_out.is_cuda and index_map_out.dtype == torch.int32 and index_map_out.numel() == ctx.N
+        im = c_void_p(index_map_out.data_ptr())
+    s = c_void_p(_stream_ptr(stream)) if (tp is not None or im is not None) else c_void_p(0)
+    _check(_lib.hs_partition(ctx.ptr, tp, None, im, s, ctypes.byref(raw)), ctx.ptr)
+    ctx.partition = Partition(raw)
+    return ctx.partition
+
+
+def hs_step(ctx: Context, params, x, y, part: Optional[Partition] = None, lr: float = 0.01, stream=None,
+            want_loss: bool = True) -> Optional[float]:
+    import torch
+    assert params.dtype == torch.float32 and params.is_contiguous() and params.is_cuda
+    assert x.dtype == torch.float32 and x.is_contiguous()
+    assert y.dtype == torch.int32 and y.is_contiguous()
+    loss = c_float()
+    raw = ctypes.byref(part.raw) if part is not None else None
+    _check(_lib.hs_step(ctx.ptr, c_void_p(params.data_ptr()), c_void_p(x.data_ptr()), c_void_p(y.data_ptr()),
+                        raw, float(lr), c_void_p(_stream_ptr(stream)), ctypes.byref(loss) if want_loss else None),
+           ctx.ptr)
+    return loss.value if want_loss else None
+
+
+def hs_sync_params(ctx: Context, params, stream=None):
+    _check(_lib.hs_sync_params(ctx.ptr, c_void_p(params.data_ptr()), c_void_p(_stream_ptr(stream))), ctx.ptr)
+
+
+def hs_set_debug(ctx: Context, enable: bool = True):
+    _check(_lib.hs_set_debug(ctx.ptr, 1 if enable else 0), ctx.ptr)
+
+
+def hs_set_profiling(ctx: Context, enable: bool = True):
+    _check(_lib.hs_set_profiling(ctx.ptr, 1 if enable else 0), ctx.ptr)
+
+
+def hs_read_profile(ctx: Context):
+    """{phase: (ms, launches)} summed since the last read (waits for the recorded events)."""
+    ms = (c_double * len(PHASES))()
+    n = (c_int64 * len(PHASES))()
+    _check(_lib.hs_read_profile(ctx.ptr, ms, n), ctx.ptr)
+    return {name: (ms[i], n[i]) for i, name in enumerate(PHASES)}
+
+
+def hs_debug_grads(ctx: Context, g_out=None, slabs_out=None, stream=None):
+    _check(_lib.hs_debug_grads(ctx.ptr, c_void_p(g_out.data_ptr() if g_out is not None else 0),
+                               c_void_p(slabs_out.data_ptr() if slabs_out is not None else 0),
+                               c_void_p(_stream_ptr(stream))), ctx.ptr)
+
+
+def hs_worker_losses(ctx: Context) -> List[float]:
+    out = (c_float * ctx.M)()
+    _check(_lib.hs_worker_losses(ctx.ptr, out), ctx.ptr)
+    return list(out)
+
+
+def hs_destroy(ctx: Context):
+    ctx.close()
+
+
+def hs_debug_gemm_bf16(mode: int, M: int, N: int, K: int, A, B, D, bias=None, Z=None, k_offsets=None,
+                       d_gstride: int = 0, stream=None):
+    """Run one product through the tensor-core kernel (test hook, include/hs_debug.h)."""
+    ko = None
+    groups = 1
+    if k_offsets is not None:
+        groups = len(k_offsets) - 1
+        ko = (c_int32 * len(k_offsets))(*[int(v) for v in k_offsets])
+    _check(_lib.hs_debug_gemm_bf16(
+        int(mode), int(M), int(N), int(K), c_void_p(A.data_ptr()), int(A.stride(0)), c_void_p(B.data_ptr()),
+        int(B.stride(0)), c_void_p(D.data_ptr()), int(D.stride(0)),
+        c_void_p(bias.data_ptr() if bias is not None else 0), c_void_p(Z.data_ptr() if Z is not None else 0),
+        int(Z.stride(0)) if Z is not None else 0, ko, groups, int(d_gstride), c_void_p(_stream_ptr(stream))))

@@ -1,0 +1,73 @@
+// Internal declarations shared by the translation units of libhs (not part of the ABI).
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/hs.h"
+
+namespace hs {
+
+constexpr int kMaxWorkers = 1024;
+
+// Device-side error codes written to the context's status word (first error wins).
+enum DevErr : int32_t {
+  kDevOk = 0,
+  kDevWaitTimeout = 1,   // a bounded mbarrier wait in a tensor-core kernel expired
+  kDevBadLabel = 2,      // a label outside [0, classes) reached the loss kernel
+};
+
+struct DevStatus {
+  float loss;         // sum_m w_m L_m of the last step
+  int32_t err;        // DevErr
+  int32_t err_info;   // kernel-specific detail (which wait / which row)
+};
+
+hs_status partition_sizes_impl(int32_t M, int32_t N, const double* cp, int32_t* sizes,
+                               double* cp_norm, const char** why);
+
+// ---------------------------------------------------------------- elementwise / reduction kernels
+void launch_cast_f32_bf16(const float* x, __nv_bfloat16* y, int64_t n, cudaStream_t s);
+void launch_partition_scatter(const int32_t* d_offsets, int M, int N, int32_t* index_map,
+                              float* scale, int32_t* index_map_out, cudaStream_t s);
+// logits [N, ldl] fp32 -> ce[N], delta [N, ldd] (bf16 if delta_bf16 else fp32, columns >= C zeroed)
+void launch_softmax_xent(const float* logits, int ldl, const int32_t* y, const float* scale, int N,
+                         int C, void* delta, int ldd, bool delta_bf16, float* ce, DevStatus* st,
+                         cudaStream_t s);
+void launch_loss_reduce(const float* ce, const int32_t* d_offsets, int M, const float* d_w,
+                        float* lm, DevStatus* st, cudaStream_t s);
+// slabs[m*Ps + b_off + j] = sum_{i in seg_m} delta[i*ld + j], j < width
+void launch_bias_grad(const void* delta, bool delta_bf16, int ld, int width, const int32_t* d_offsets,
+                      int M, float* slabs, int64_t Ps, int64_t b_off, cudaStream_t s);
+// theta[j] -= lr * sum_m w[m] * slabs[m*Ps + j]; shadow[j] = bf16(theta[j]); gdebug[j] = g (optional)
+void launch_reduce_update(float* theta, const float* slabs, int64_t Ps, int M, const float* d_w,
+                          float lr, int64_t P, __nv_bfloat16* shadow, float* gdebug, int num_sms,
+                          cudaStream_t s);
+
+// ---------------------------------------------------------------- fp32 CUDA-core GEMM (check path)
+// C(m, n) = sum_k A(m, k) B(k, n) with A(m,k) = A[m*a_sm + k*a_sk], B(k,n) = B[k*b_sk + n*b_sn],
+// C[m*ldc + n].  Grouped form: blockIdx.z = g runs k over [k_offsets[g], k_offsets[g+1]) and writes
+// C + g*c_gstride.  Epilogues below.
+enum Epi : int32_t {
+  kEpiStore = 0,      // C = acc
+  kEpiBias = 1,       // C = acc + bias[n]
+  kEpiBiasRelu = 2,   // C = max(acc + bias[n], 0)
+  kEpiMask = 3,       // C = acc * (Z(m, n) > 0)
+};
+
+struct GemmF32Args {
+  const float* A; int64_t a_sm, a_sk;
+  const float* B; int64_t b_sk, b_sn;
+  float* C; int64_t ldc;
+  int Mdim, Ndim, Kdim;
+  int epi;
+  const float* bias;
+  const float* Z; int64_t ldz;
+  const int32_t* k_offsets;   // grouped if non-null
+  int groups;
+  int64_t c_gstride;
+};
+void launch_gemm_f32(const GemmF32Args& a, cudaStream_t s);
+
+}  // namespace hs

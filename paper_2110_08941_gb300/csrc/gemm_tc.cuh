@@ -1,0 +1,63 @@
+// Tensor-core (tcgen05) GEMM used by every bf16 contraction of the step.
+#pragma once
+
+#include <cuda.h>
+
+#include "common.cuh"
+
+namespace hs {
+
+constexpr int kTcMaxGroups = 32;   // groups (workers) per launch; more are split over launches
+
+// Epilogue variants of the tensor-core GEMM.
+enum TcEpi : int32_t {
+  kTcEpiBiasReluBf16 = 0,   // D bf16 = bf16(max(acc + bias[n], 0))        (hidden-layer forward)
+  kTcEpiBiasF32 = 1,        // D fp32 = acc + bias[n] (n < Ndim), 0 beyond   (logits)
+  kTcEpiMaskBf16 = 2,       // D bf16 = bf16(acc * (Z(m, n) > 0))            (input gradient + ReLU')
+  kTcEpiStoreF32 = 3,       // D fp32 = acc                                  (per-worker weight gradient)
+};
+
+// D[Mdim x n_store] (row-major, leading dimension ldd) = A[Mdim x K] * B[K x Ndim] + epilogue.
+// Operands are bf16 in global memory and are described by TMA tensor maps:
+//   K-major   ("row-major with K contiguous"): A as [M rows][K], B as [N rows][K]
+//   MN-major  ("K rows, M or N contiguous"):   A as [K rows][M], B as [K rows][N]
+// Grouped launches run `groups` independent products that share Mdim/Ndim but each has its own
+// A/B maps (a worker's row segment) and K extent; group g writes D + g * d_gstride.
+struct TcGemmParams {
+  CUtensorMap tmA[kTcMaxGroups];
+  CUtensorMap tmB[kTcMaxGroups];
+  int32_t num_kb[kTcMaxGroups];
+  int32_t groups;
+  int32_t Mdim, Ndim, n_store;
+  int32_t tiles_m, tiles_n;
+  int32_t epi;
+  int32_t a_mn, b_mn;
+  void* D;
+  int64_t ldd;
+  int64_t d_gstride;
+  const float* bias;
+  const __nv_bfloat16* Z;
+  int64_t ldz;
+  DevStatus* st;
+};
+
+// Operand view for building tensor maps.  `rows` x `cols` bf16 matrix, row stride `ld` elements.
+struct TcOperand {
+  const __nv_bfloat16* base;
+  int64_t rows, cols, ld;
+};
+
+// Host helpers.  Return false (and set *why) if the driver entry point or the encoding fails.
+bool tc_init_driver(const char** why);
+// K-major operand: matrix [rows][K] with K contiguous; box = 64 (K) x box_rows.
+bool tc_make_kmajor_map(CUtensorMap* tm, const TcOperand& op, int box_rows, const char** why);
+// MN-major operand: matrix [K rows][MN] with MN contiguous; box = 64 (MN) x 64 (K).
+bool tc_make_mnmajor_map(CUtensorMap* tm, const TcOperand& op, const char** why);
+
+constexpr int kTcBM = 128, kTcBN = 256, kTcBK = 64, kTcStages = 4;
+constexpr int kTcSmemBytes = kTcStages * (kTcBM + kTcBN) * kTcBK * 2 + 1024 /*align*/ + 256 /*barriers*/;
+
+// Launch on `num_sms` persistent CTAs (capped by the tile count).
+cudaError_t launch_tc_gemm(const TcGemmParams& p, int num_sms, cudaStream_t s);
+
+}  // namespace hs

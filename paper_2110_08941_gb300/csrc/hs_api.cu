@@ -1,0 +1,872 @@
+// C-ABI of libhs: context, Dynamic Partitioning (Algorithm 1) and the synchronous SGD step
+// (Section 1, Eq. 1, Section 4.2) over M logical workers on one GPU.
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "../../include/hs.h"
+#include "../../include/hs_debug.h"
+#include "common.cuh"
+#include "gemm_tc.cuh"
+
+using hs::DevStatus;
+
+namespace {
+
+thread_local std::string g_init_error;
+
+struct Layer {
+  int in, out;
+  int64_t w_off, b_off;
+};
+
+int64_t round_up(int64_t v, int64_t m) { return (v + m - 1) / m * m; }
+
+}  // namespace
+
+struct hs_ctx {
+  int device = 0;
+  int num_sms = 0;
+  int arch = HS_MLP, precision = HS_BF16, sync = HS_SYNC_MEAN;
+  std::vector<int32_t> dims;
+  std::vector<Layer> layers;
+  int L = 0;
+  int M = 0, N = 0;
+  int64_t P = 0, Ps = 0;
+  int C = 0, Cp = 0, maxw = 0;
+
+  // partition state (host mirror + device copies)
+  std::vector<int32_t> counts, offsets;
+  std::vector<double> weights, cp_norm;
+  uint64_t version = 0;
+  int32_t* d_offsets = nullptr;
+  int32_t* d_index_map = nullptr;
+  float* d_scale = nullptr;
+  float* d_w = nullptr;
+
+  // workspace
+  std::vector<void*> d_act;        // H_0 .. H_{L-1}
+  float* d_logits = nullptr;       // [N, Cp]
+  void* d_delta[2] = {nullptr, nullptr};
+  float* d_ce = nullptr;
+  float* d_lm = nullptr;
+  DevStatus* d_status = nullptr;
+  DevStatus* h_status = nullptr;   // pinned
+  float* d_slabs = nullptr;        // [M, Ps]
+  __nv_bfloat16* d_shadow = nullptr;
+  float* d_gdebug = nullptr;
+  void* d_xstage = nullptr;
+  int32_t* d_ystage = nullptr;
+  const float* shadow_src = nullptr;
+  bool shadow_valid = false;
+  bool debug = false;
+  bool gdebug_valid = false;
+  std::string err;
+
+  // profiling: per-phase event pairs recorded on the step's stream, summed on read
+  bool profiling = false;
+  struct Rec { int phase; cudaEvent_t a, b; };
+  std::vector<Rec> pending;
+  std::vector<cudaEvent_t> event_pool;
+  int64_t launches[HS_PHASE_COUNT] = {0};
+
+  cudaEvent_t take_event() {
+    if (!event_pool.empty()) {
+      cudaEvent_t e = event_pool.back();
+      event_pool.pop_back();
+      return e;
+    }
+    cudaEvent_t e = nullptr;
+    if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+    return e;
+  }
+
+  // tensor-core launch parameters (bf16 precision)
+  std::vector<hs::TcGemmParams> tc_fwd;                // per layer
+  std::vector<hs::TcGemmParams> tc_dgrad;              // per layer (index 0 unused)
+  std::vector<std::vector<hs::TcGemmParams>> tc_wgrad; // per layer, per chunk of <= 32 workers
+
+  size_t act_elem() const { return precision == HS_BF16 ? 2 : 4; }
+  int delta_ld(int l) const { return l == L - 1 ? Cp : layers[l].out; }     // l: 0-based layer
+  void* delta_buf(int l) const { return d_delta[(L - 1 - l) & 1]; }
+};
+
+namespace {
+
+// Brackets one phase of the step with CUDA events when profiling is on.
+class PhaseScope {
+ public:
+  PhaseScope(hs_ctx* c, int phase, cudaStream_t s) : c_(c), phase_(phase), s_(s) {
+    if (c_->profiling) {
+      a_ = c_->take_event();
+      if (a_) cudaEventRecord(a_, s_);
+    }
+  }
+  ~PhaseScope() {
+    if (c_->profiling && a_) {
+      cudaEvent_t b = c_->take_event();
+      if (b) {
+        cudaEventRecord(b, s_);
+        c_->pending.push_back({phase_, a_, b});
+      }
+    }
+  }
+  void launched(int n = 1) { c_->launches[phase_] += n; }
+
+ private:
+  hs_ctx* c_;
+  int phase_;
+  cudaStream_t s_;
+  cudaEvent_t a_ = nullptr;
+};
+
+hs_status fail(hs_ctx* c, hs_status s, const std::string& msg) {
+  if (c) c->err = msg; else g_init_error = msg;
+  return s;
+}
+
+hs_status cuda_fail(hs_ctx* c, cudaError_t e, const char* what) {
+  return fail(c, e == cudaErrorMemoryAllocation ? HS_ERR_OOM : HS_ERR_CUDA,
+              std::string(what) + ": " + cudaGetErrorString(e));
+}
+
+#define HS_CUDA(ctx, call)                                   \
+  do {                                                       \
+    cudaError_t e_ = (call);                                 \
+    if (e_ != cudaSuccess) return cuda_fail(ctx, e_, #call); \
+  } while (0)
+
+hs_status validate_model(const hs_model_desc* m, std::vector<int32_t>* dims, std::string* why) {
+  if (!m || !m->dims) { *why = "model or model->dims is NULL"; return HS_ERR_INVALID_ARG; }
+  if (m->precision != HS_BF16 && m->precision != HS_FP32_CHECK) { *why = "unknown precision"; return HS_ERR_INVALID_ARG; }
+  if (m->sync < HS_SYNC_MEAN || m->sync > HS_SYNC_CP_LITERAL) { *why = "unknown sync mode"; return HS_ERR_INVALID_ARG; }
+  if (m->arch == HS_MLP) {
+    if (m->n_layers < 1 || m->n_layers > 64) { *why = "n_layers must be in [1, 64]"; return HS_ERR_INVALID_ARG; }
+    dims->assign(m->dims, m->dims + m->n_layers + 1);
+    for (int32_t d : *dims)
+      if (d < 1 || d > (1 << 20)) { *why = "layer widths must be in [1, 2^20]"; return HS_ERR_INVALID_ARG; }
+    return HS_OK;
+  }
+  if (m->arch == HS_CNN) {
+    dims->assign(m->dims, m->dims + 7);
+    for (int32_t d : *dims)
+      if (d < 1 || d > (1 << 16)) { *why = "CNN dims must be in [1, 65536]"; return HS_ERR_INVALID_ARG; }
+    return HS_OK;
+  }
+  *why = "unknown arch";
+  return HS_ERR_INVALID_ARG;
+}
+
+int64_t mlp_param_count(const std::vector<int32_t>& d) {
+  int64_t p = 0;
+  for (size_t l = 1; l < d.size(); ++l) p += (int64_t)d[l] * d[l - 1] + d[l];
+  return p;
+}
+
+int64_t cnn_param_count(const std::vector<int32_t>& d) {
+  int64_t p = 0, prev = d[0];
+  for (int k = 3; k < 6; ++k) {
+    p += (int64_t)d[k] * prev * 9 + d[k];
+    prev = d[k];
+  }
+  p += (int64_t)d[6] * prev + d[6];
+  return p;
+}
+
+// ------------------------------------------------------------------ tensor-core plans
+hs_status build_tc_static(hs_ctx* c) {
+  const char* why = nullptr;
+  if (!hs::tc_init_driver(&why)) return fail(c, HS_ERR_CUDA, why);
+  c->tc_fwd.assign(c->L, hs::TcGemmParams{});
+  c->tc_dgrad.assign(c->L, hs::TcGemmParams{});
+  for (int l = 0; l < c->L; ++l) {
+    const Layer& ly = c->layers[l];
+    const bool last = (l == c->L - 1);
+    // forward: A = H_l [N, in] (K-major), B = W_l [out, in] (K-major)
+    hs::TcGemmParams& f = c->tc_fwd[l];
+    std::memset(&f, 0, sizeof(f));
+    hs::TcOperand a{reinterpret_cast<const __nv_bfloat16*>(c->d_act[l]), c->N, ly.in, ly.in};
+    hs::TcOperand b{c->d_shadow + ly.w_off, ly.out, ly.in, ly.in};
+    if (!hs::tc_make_kmajor_map(&f.tmA[0], a, hs::kTcBM, &why) ||
+        !hs::tc_make_kmajor_map(&f.tmB[0], b, hs::kTcBN, &why))
+      return fail(c, HS_ERR_CUDA, why);
+    f.num_kb[0] = (ly.in + hs::kTcBK - 1) / hs::kTcBK;
+    f.groups = 1;
+    f.Mdim = c->N;
+    f.Ndim = ly.out;
+    f.n_store = last ? c->Cp : ly.out;
+    f.tiles_m = (c->N + hs::kTcBM - 1) / hs::kTcBM;
+    f.tiles_n = (f.n_store + hs::kTcBN - 1) / hs::kTcBN;
+    f.epi = last ? hs::kTcEpiBiasF32 : hs::kTcEpiBiasReluBf16;
+    f.D = last ? static_cast<void*>(c->d_logits) : c->d_act[l + 1];
+    f.ldd = last ? c->Cp : ly.out;
+    f.st = c->d_status;
+    if (l == 0) continue;
+    // input gradient of layer l: A = delta_l [N, out] (K-major), B = W_l [out, in] (MN-major)
+    hs::TcGemmParams& d = c->tc_dgrad[l];
+    std::memset(&d, 0, sizeof(d));
+    hs::TcOperand da{reinterpret_cast<const __nv_bfloat16*>(c->delta_buf(l)), c->N, ly.out, c->delta_ld(l)};
+    hs::TcOperand db{c->d_shadow + ly.w_off, ly.out, ly.in, ly.in};
+    if (!hs::tc_make_kmajor_map(&d.tmA[0], da, hs::kTcBM, &why) || !hs::tc_make_mnmajor_map(&d.tmB[0], db, &why))
+      return fail(c, HS_ERR_CUDA, why);
+    d.num_kb[0] = (ly.out + hs::kTcBK - 1) / hs::kTcBK;
+    d.groups = 1;
+    d.Mdim = c->N;
+    d.Ndim = ly.in;
+    d.n_store = ly.in;
+    d.tiles_m = (c->N + hs::kTcBM - 1) / hs::kTcBM;
+    d.tiles_n = (ly.in + hs::kTcBN - 1) / hs::kTcBN;
+    d.epi = hs::kTcEpiMaskBf16;
+    d.a_mn = 0;
+    d.b_mn = 1;
+    d.D = c->delta_buf(l - 1);
+    d.ldd = c->delta_ld(l - 1);
+    d.Z = reinterpret_cast<const __nv_bfloat16*>(c->d_act[l]);
+    d.ldz = ly.in;
+    d.st = c->d_status;
+  }
+  return HS_OK;
+}
+
+// Per-worker weight gradients depend on the segments, so they are rebuilt on repartition.
+hs_status build_tc_wgrad(hs_ctx* c) {
+  const char* why = nullptr;
+  c->tc_wgrad.assign(c->L, {});
+  for (int l = 0; l < c->L; ++l) {
+    const Layer& ly = c->layers[l];
+    const int ldd_delta = c->delta_ld(l);
+    const int out_cols = (l == c->L - 1) ? c->C : ly.out;
+    for (int g0 = 0; g0 < c->M; g0 += hs::kTcMaxGroups) {
+      const int ng = std::min(hs::kTcMaxGroups, c->M - g0);
+      c->tc_wgrad[l].emplace_back();
+      hs::TcGemmParams& w = c->tc_wgrad[l].back();
+      std::memset(&w, 0, sizeof(w));
+      for (int g = 0; g < ng; ++g) {
+        const int m = g0 + g;
+        const int64_t off = c->offsets[m], n = c->counts[m];
+        // A^T: delta_l rows of worker m as [n rows][out cols] (MN-major: out contiguous)
+        hs::TcOperand a{reinterpret_cast<const __nv_bfloat16*>(c->delta_buf(l)) + off * ldd_delta, n, out_cols,
+                        ldd_delta};
+        // B: H_{l-1} rows of worker m as [n rows][in cols] (MN-major: in contiguous)
+        hs::TcOperand b{reinterpret_cast<const __nv_bfloat16*>(c->d_act[l]) + off * ly.in, n, ly.in, ly.in};
+        if (!hs::tc_make_mnmajor_map(&w.tmA[g], a, &why) || !hs::tc_make_mnmajor_map(&w.tmB[g], b, &why))
+          return fail(c, HS_ERR_CUDA, why);
+        w.num_kb[g] = (int32_t)((n + hs::kTcBK - 1) / hs::kTcBK);
+      }
+      w.groups = ng;
+      w.Mdim = out_cols;
+      w.Ndim = ly.in;
+      w.n_store = ly.in;
+      w.tiles_m = (out_cols + hs::kTcBM - 1) / hs::kTcBM;
+      w.tiles_n = (ly.in + hs::kTcBN - 1) / hs::kTcBN;
+      w.epi = hs::kTcEpiStoreF32;
+      w.a_mn = 1;
+      w.b_mn = 1;
+      w.D = c->d_slabs + (int64_t)g0 * c->Ps + ly.w_off;
+      w.ldd = ly.in;
+      w.d_gstride = c->Ps;
+      w.st = c->d_status;
+    }
+  }
+  return HS_OK;
+}
+
+void compute_weights(hs_ctx* c) {
+  c->weights.assign(c->M, 0.0);
+  for (int m = 0; m < c->M; ++m) {
+    if (c->sync == HS_SYNC_MEAN) c->weights[m] = 1.0 / c->M;
+    else if (c->sync == HS_SYNC_CP_WEIGHTED) c->weights[m] = (double)c->counts[m] / (double)c->N;
+    else c->weights[m] = c->cp_norm[m] / c->M;
+  }
+}
+
+// Apply a new partition (sizes already validated) and push it to the device on `s`.
+hs_status apply_partition(hs_ctx* c, const std::vector<int32_t>& sizes, const std::vector<double>& cpn,
+                          int32_t* index_map_out, cudaStream_t s) {
+  const bool changed = (sizes != c->counts);
+  c->cp_norm = cpn;
+  if (changed) {
+    c->counts = sizes;
+    c->offsets.assign(c->M + 1, 0);
+    for (int m = 0; m < c->M; ++m) c->offsets[m + 1] = c->offsets[m] + sizes[m];
+    ++c->version;
+  }
+  compute_weights(c);
+  std::vector<float> wf(c->weights.begin(), c->weights.end());
+  HS_CUDA(c, cudaMemcpyAsync(c->d_w, wf.data(), sizeof(float) * c->M, cudaMemcpyHostToDevice, s));
+  if (changed) {
+    HS_CUDA(c, cudaMemcpyAsync(c->d_offsets, c->offsets.data(), sizeof(int32_t) * (c->M + 1),
+                               cudaMemcpyHostToDevice, s));
+  }
+  if (changed || index_map_out) {
+    hs::launch_partition_scatter(c->d_offsets, c->M, c->N, c->d_index_map, c->d_scale, index_map_out, s);
+    HS_CUDA(c, cudaGetLastError());
+  }
+  // the host vectors above are pageable: make sure the copies consumed them before they change
+  HS_CUDA(c, cudaStreamSynchronize(s));
+  if (changed && c->arch == HS_MLP && c->precision == HS_BF16) {
+    hs_status st = build_tc_wgrad(c);
+    if (st != HS_OK) return st;
+  }
+  return HS_OK;
+}
+
+void fill_partition_view(const hs_ctx* c, hs_partition_t* out) {
+  if (!out) return;
+  out->M = c->M;
+  out->N = c->N;
+  out->counts_host = c->counts.data();
+  out->offsets_host = c->offsets.data();
+  out->index_map_dev = c->d_index_map;
+  out->weights_host = c->weights.data();
+  out->cp_host = c->cp_norm.data();
+  out->version = c->version;
+}
+
+template <typename T>
+hs_status dalloc(hs_ctx* c, T** p, size_t bytes) {
+  *p = nullptr;
+  if (bytes == 0) bytes = 16;
+  cudaError_t e = cudaMalloc(reinterpret_cast<void**>(p), bytes);
+  if (e != cudaSuccess) return cuda_fail(c, e, "cudaMalloc");
+  return HS_OK;
+}
+
+void free_all(hs_ctx* c) {
+  auto f = [](void* p) { if (p) cudaFree(p); };
+  f(c->d_offsets); f(c->d_index_map); f(c->d_scale); f(c->d_w);
+  for (void* p : c->d_act) f(p);
+  f(c->d_logits); f(c->d_delta[0]); f(c->d_delta[1]); f(c->d_ce); f(c->d_lm); f(c->d_status);
+  f(c->d_slabs); f(c->d_shadow); f(c->d_gdebug); f(c->d_xstage); f(c->d_ystage);
+  if (c->h_status) cudaFreeHost(c->h_status);
+  for (auto& r : c->pending) {
+    cudaEventDestroy(r.a);
+    cudaEventDestroy(r.b);
+  }
+  for (cudaEvent_t e : c->event_pool) cudaEventDestroy(e);
+}
+
+bool is_device_ptr(const void* p) {
+  cudaPointerAttributes a;
+  if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged;
+}
+
+// ------------------------------------------------------------------ the MLP step
+hs_status mlp_step_fp32(hs_ctx* c, float* params, const float* x, const int32_t* y, cudaStream_t s) {
+  const int L = c->L;
+  std::vector<const float*> act(L);
+  act[0] = x;
+  for (int l = 1; l < L; ++l) act[l] = reinterpret_cast<const float*>(c->d_act[l]);
+  {
+    // per-worker forward: the segments share theta, so all rows go through one product per layer
+    PhaseScope ph(c, HS_PHASE_FORWARD, s);
+    for (int l = 0; l < L; ++l) {
+      const Layer& ly = c->layers[l];
+      const bool last = (l == L - 1);
+      hs::GemmF32Args g{};
+      g.A = act[l]; g.a_sm = ly.in; g.a_sk = 1;
+      g.B = params + ly.w_off; g.b_sk = 1; g.b_sn = ly.in;
+      g.C = last ? c->d_logits : reinterpret_cast<float*>(c->d_act[l + 1]);
+      g.ldc = last ? c->Cp : ly.out;
+      g.Mdim = c->N; g.Ndim = ly.out; g.Kdim = ly.in;
+      g.epi = last ? hs::kEpiBias : hs::kEpiBiasRelu;
+      g.bias = params + ly.b_off;
+      hs::launch_gemm_f32(g, s);
+      ph.launched();
+    }
+  }
+  {
+    PhaseScope ph(c, HS_PHASE_LOSS, s);
+    hs::launch_softmax_xent(c->d_logits, c->Cp, y, c->d_scale, c->N, c->C, c->delta_buf(L - 1), c->Cp, false,
+                            c->d_ce, c->d_status, s);
+    hs::launch_loss_reduce(c->d_ce, c->d_offsets, c->M, c->d_w, c->d_lm, c->d_status, s);
+    ph.launched(2);
+  }
+  for (int l = L - 1; l >= 0; --l) {
+    const Layer& ly = c->layers[l];
+    const int ldd = c->delta_ld(l);
+    const float* delta = reinterpret_cast<const float*>(c->delta_buf(l));
+    const int out_cols = (l == L - 1) ? c->C : ly.out;
+    {
+      // per-worker weight gradient G_m[W_l] = delta_l[seg_m]^T H_{l-1}[seg_m]
+      PhaseScope ph(c, HS_PHASE_WGRAD, s);
+      hs::GemmF32Args w{};
+      w.A = delta; w.a_sm = 1; w.a_sk = ldd;
+      w.B = act[l]; w.b_sk = ly.in; w.b_sn = 1;
+      w.C = c->d_slabs + ly.w_off; w.ldc = ly.in;
+      w.Mdim = out_cols; w.Ndim = ly.in; w.Kdim = 0;
+      w.epi = hs::kEpiStore;
+      w.k_offsets = c->d_offsets; w.groups = c->M; w.c_gstride = c->Ps;
+      hs::launch_gemm_f32(w, s);
+      ph.launched();
+    }
+    {
+      PhaseScope ph(c, HS_PHASE_BIASGRAD, s);
+      hs::launch_bias_grad(delta, false, ldd, out_cols, c->d_offsets, c->M, c->d_slabs, c->Ps, ly.b_off, s);
+      ph.launched();
+    }
+    if (l > 0) {
+      PhaseScope ph(c, HS_PHASE_DGRAD, s);
+      hs::GemmF32Args d{};
+      d.A = delta; d.a_sm = ldd; d.a_sk = 1;
+      d.B = params + ly.w_off; d.b_sk = ly.in; d.b_sn = 1;
+      d.C = reinterpret_cast<float*>(c->delta_buf(l - 1)); d.ldc = c->delta_ld(l - 1);
+      d.Mdim = c->N; d.Ndim = ly.in; d.Kdim = out_cols;
+      d.epi = hs::kEpiMask; d.Z = act[l]; d.ldz = ly.in;
+      hs::launch_gemm_f32(d, s);
+      ph.launched();
+    }
+  }
+  return HS_OK;
+}
+
+hs_status mlp_step_bf16(hs_ctx* c, float* params, const float* x, const int32_t* y, cudaStream_t s) {
+  const int L = c->L;
+  {
+    PhaseScope ph(c, HS_PHASE_CAST, s);
+    hs::launch_cast_f32_bf16(x, reinterpret_cast<__nv_bfloat16*>(c->d_act[0]), (int64_t)c->N * c->layers[0].in, s);
+    ph.launched();
+  }
+  {
+    PhaseScope ph(c, HS_PHASE_FORWARD, s);
+    for (int l = 0; l < L; ++l) {
+      hs::TcGemmParams& f = c->tc_fwd[l];
+      f.bias = params + c->layers[l].b_off;
+      cudaError_t e = hs::launch_tc_gemm(f, c->num_sms, s);
+      if (e != cudaSuccess) return cuda_fail(c, e, "forward GEMM launch");
+      ph.launched();
+    }
+  }
+  {
+    PhaseScope ph(c, HS_PHASE_LOSS, s);
+    hs::launch_softmax_xent(c->d_logits, c->Cp, y, c->d_scale, c->N, c->C, c->delta_buf(L - 1), c->Cp, true,
+                            c->d_ce, c->d_status, s);
+    hs::launch_loss_reduce(c->d_ce, c->d_offsets, c->M, c->d_w, c->d_lm, c->d_status, s);
+    ph.launched(2);
+  }
+  for (int l = L - 1; l >= 0; --l) {
+    const Layer& ly = c->layers[l];
+    {
+      PhaseScope ph(c, HS_PHASE_WGRAD, s);
+      for (const hs::TcGemmParams& w : c->tc_wgrad[l]) {
+        cudaError_t e = hs::launch_tc_gemm(w, c->num_sms, s);
+        if (e != cudaSuccess) return cuda_fail(c, e, "weight-gradient GEMM launch");
+        ph.launched();
+      }
+    }
+    {
+      PhaseScope ph(c, HS_PHASE_BIASGRAD, s);
+      const int out_cols = (l == L - 1) ? c->C : ly.out;
+      hs::launch_bias_grad(c->delta_buf(l), true, c->delta_ld(l), out_cols, c->d_offsets, c->M, c->d_slabs, c->Ps,
+                           ly.b_off, s);
+      ph.launched();
+    }
+    if (l > 0) {
+      PhaseScope ph(c, HS_PHASE_DGRAD, s);
+      cudaError_t e = hs::launch_tc_gemm(c->tc_dgrad[l], c->num_sms, s);
+      if (e != cudaSuccess) return cuda_fail(c, e, "input-gradient GEMM launch");
+      ph.launched();
+    }
+  }
+  return HS_OK;
+}
+
+}  // namespace
+
+// ====================================================================== C ABI
+extern "C" {
+
+const char* hs_status_string(hs_status s) {
+  switch (s) {
+    case HS_OK: return "HS_OK";
+    case HS_ERR_INVALID_ARG: return "HS_ERR_INVALID_ARG";
+    case HS_ERR_CUDA: return "HS_ERR_CUDA";
+    case HS_ERR_OOM: return "HS_ERR_OOM";
+    case HS_ERR_UNSUPPORTED: return "HS_ERR_UNSUPPORTED";
+    case HS_ERR_DEVICE_CHECK: return "HS_ERR_DEVICE_CHECK";
+  }
+  return "HS_ERR_UNKNOWN";
+}
+
+const char* hs_last_error(const hs_ctx* ctx) { return ctx ? ctx->err.c_str() : ""; }
+const char* hs_last_init_error(void) { return g_init_error.c_str(); }
+
+hs_status hs_param_count(const hs_model_desc* model, int64_t* P) {
+  std::vector<int32_t> dims;
+  std::string why;
+  if (!P) return HS_ERR_INVALID_ARG;
+  hs_status st = validate_model(model, &dims, &why);
+  if (st != HS_OK) return st;
+  *P = model->arch == HS_MLP ? mlp_param_count(dims) : cnn_param_count(dims);
+  return HS_OK;
+}
+
+hs_status hs_init(const hs_model_desc* model, int32_t M, const double* compute_weights, int32_t global_batch,
+                  hs_ctx** out) {
+  g_init_error.clear();
+  if (!out) return fail(nullptr, HS_ERR_INVALID_ARG, "out is NULL");
+  *out = nullptr;
+  std::vector<int32_t> dims;
+  std::string why;
+  hs_status st = validate_model(model, &dims, &why);
+  if (st != HS_OK) return fail(nullptr, st, why);
+  if (M < 1 || M > hs::kMaxWorkers) return fail(nullptr, HS_ERR_INVALID_ARG, "M must be in [1, 1024]");
+  if (global_batch < M) return fail(nullptr, HS_ERR_INVALID_ARG, "global_batch must be >= M");
+  if (model->arch == HS_CNN) return fail(nullptr, HS_ERR_UNSUPPORTED, "CNN workloads are not built yet");
+
+  std::vector<double> cp(M, 1.0);
+  if (compute_weights) cp.assign(compute_weights, compute_weights + M);
+  std::vector<int32_t> sizes(M);
+  std::vector<double> cpn(M);
+  const char* pwhy = nullptr;
+  st = hs::partition_sizes_impl(M, global_batch, cp.data(), sizes.data(), cpn.data(), &pwhy);
+  if (st != HS_OK) return fail(nullptr, st, std::string("compute_weights: ") + pwhy);
+
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return fail(nullptr, HS_ERR_CUDA, std::string("no CUDA device: ") + cudaGetErrorString(e));
+  cudaDeviceProp prop;
+  e = cudaGetDeviceProperties(&prop, dev);
+  if (e != cudaSuccess) return fail(nullptr, HS_ERR_CUDA, cudaGetErrorString(e));
+  if (!(prop.major == 10 && prop.minor == 3))
+    return fail(nullptr, HS_ERR_UNSUPPORTED, "libhs is built for sm_103a (compute capability 10.3) only");
+
+  hs_ctx* c = new hs_ctx();
+  c->device = dev;
+  c->num_sms = prop.multiProcessorCount;
+  c->arch = model->arch;
+  c->precision = model->precision;
+  c->sync = model->sync;
+  c->dims = dims;
+  c->M = M;
+  c->N = global_batch;
+  c->L = model->n_layers;
+  if (c->precision == HS_BF16) {
+    for (int l = 0; l < c->L; ++l)
+      if (dims[l] % 8 != 0) {
+        delete c;
+        return fail(nullptr, HS_ERR_UNSUPPORTED, "bf16 precision needs input and hidden widths divisible by 8");
+      }
+  }
+  int64_t off = 0;
+  for (int l = 0; l < c->L; ++l) {
+    Layer ly{dims[l], dims[l + 1], 0, 0};
+    ly.w_off = off;
+    off += (int64_t)ly.in * ly.out;
+    ly.b_off = off;
+    off += ly.out;
+    c->layers.push_back(ly);
+  }
+  c->P = off;
+  c->Ps = round_up(c->P, 64);
+  c->C = dims[c->L];
+  c->Cp = (int)round_up(c->C, 8);
+  c->maxw = c->Cp;
+  for (int l = 1; l < c->L; ++l) c->maxw = std::max(c->maxw, dims[l]);
+
+  const size_t N = (size_t)c->N;
+  const size_t es = c->act_elem();
+  hs_status s2 = HS_OK;
+  auto chk = [&](hs_status r) { if (r != HS_OK && s2 == HS_OK) s2 = r; };
+  chk(dalloc(c, &c->d_offsets, sizeof(int32_t) * (M + 1)));
+  chk(dalloc(c, &c->d_index_map, sizeof(int32_t) * N));
+  chk(dalloc(c, &c->d_scale, sizeof(float) * N));
+  chk(dalloc(c, &c->d_w, sizeof(float) * M));
+  c->d_act.assign(c->L, nullptr);
+  for (int l = 0; l < c->L; ++l) {
+    if (l == 0 && c->precision == HS_FP32_CHECK) continue;   // fp32 reads x in place
+    chk(dalloc(c, &c->d_act[l], es * N * (size_t)dims[l]));
+  }
+  chk(dalloc(c, &c->d_logits, sizeof(float) * N * c->Cp));
+  chk(dalloc(c, &c->d_delta[0], es * N * c->maxw));
+  chk(dalloc(c, &c->d_delta[1], es * N * c->maxw));
+  chk(dalloc(c, &c->d_ce, sizeof(float) * N));
+  chk(dalloc(c, &c->d_lm, sizeof(float) * M));
+  chk(dalloc(c, &c->d_status, sizeof(DevStatus)));
+  chk(dalloc(c, &c->d_slabs, sizeof(float) * (size_t)M * (size_t)c->Ps));
+  if (c->precision == HS_BF16) chk(dalloc(c, &c->d_shadow, sizeof(__nv_bfloat16) * (size_t)c->Ps));
+  if (s2 == HS_OK) {
+    e = cudaMallocHost(reinterpret_cast<void**>(&c->h_status), sizeof(DevStatus));
+    if (e != cudaSuccess) s2 = cuda_fail(c, e, "cudaMallocHost");
+  }
+  if (s2 == HS_OK) {
+    e = cudaMemset(c->d_status, 0, sizeof(DevStatus));
+    if (e == cudaSuccess) e = cudaMemset(c->d_slabs, 0, sizeof(float) * (size_t)M * (size_t)c->Ps);
+    if (e == cudaSuccess && c->d_shadow) e = cudaMemset(c->d_shadow, 0, sizeof(__nv_bfloat16) * (size_t)c->Ps);
+    if (e == cudaSuccess) e = cudaMemset(c->d_delta[0], 0, es * N * c->maxw);
+    if (e == cudaSuccess) e = cudaMemset(c->d_delta[1], 0, es * N * c->maxw);
+    if (e != cudaSuccess) s2 = cuda_fail(c, e, "cudaMemset");
+  }
+  if (s2 == HS_OK && c->precision == HS_BF16) s2 = build_tc_static(c);
+  if (s2 == HS_OK) s2 = apply_partition(c, sizes, cpn, nullptr, 0);
+  if (s2 == HS_OK) {
+    e = cudaDeviceSynchronize();
+    if (e != cudaSuccess) s2 = cuda_fail(c, e, "initial partition");
+  }
+  if (s2 != HS_OK) {
+    g_init_error = c->err;
+    free_all(c);
+    delete c;
+    return s2;
+  }
+  *out = c;
+  return HS_OK;
+}
+
+hs_status hs_partition(hs_ctx* c, const double* measured_throughputs, int32_t* counts_out, int32_t* index_map_out,
+                       void* stream, hs_partition_t* out) {
+  if (!c) return HS_ERR_INVALID_ARG;
+  c->err.clear();
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (measured_throughputs) {
+    std::vector<int32_t> sizes(c->M);
+    std::vector<double> cpn(c->M);
+    const char* why = nullptr;
+    hs_status st = hs::partition_sizes_impl(c->M, c->N, measured_throughputs, sizes.data(), cpn.data(), &why);
+    if (st != HS_OK) return fail(c, st, std::string("measured_throughputs: ") + why);
+    st = apply_partition(c, sizes, cpn, index_map_out, s);
+    if (st != HS_OK) return st;
+  } else if (index_map_out) {
+    hs::launch_partition_scatter(c->d_offsets, c->M, c->N, c->d_index_map, c->d_scale, index_map_out, s);
+    HS_CUDA(c, cudaGetLastError());
+  }
+  if (counts_out) std::memcpy(counts_out, c->counts.data(), sizeof(int32_t) * c->M);
+  fill_partition_view(c, out);
+  return HS_OK;
+}
+
+hs_status hs_sync_params(hs_ctx* c, const float* params, void* stream) {
+  if (!c || !params) return c ? fail(c, HS_ERR_INVALID_ARG, "params is NULL") : HS_ERR_INVALID_ARG;
+  c->err.clear();
+  if (c->precision != HS_BF16) return HS_OK;
+  hs::launch_cast_f32_bf16(params, c->d_shadow, c->P, reinterpret_cast<cudaStream_t>(stream));
+  HS_CUDA(c, cudaGetLastError());
+  c->shadow_src = params;
+  c->shadow_valid = true;
+  return HS_OK;
+}
+
+hs_status hs_step(hs_ctx* c, float* params, const void* x, const int32_t* y, const hs_partition_t* part, float lr,
+                  void* stream, float* loss_out) {
+  if (!c) return HS_ERR_INVALID_ARG;
+  c->err.clear();
+  if (!params || !x || !y) return fail(c, HS_ERR_INVALID_ARG, "params, x and y must be non-NULL");
+  if ((reinterpret_cast<uintptr_t>(params) & 15u) != 0) return fail(c, HS_ERR_INVALID_ARG, "params must be 16-byte aligned");
+  if (!std::isfinite(lr)) return fail(c, HS_ERR_INVALID_ARG, "lr must be finite");
+  if (part && (part->version != c->version || part->M != c->M || part->N != c->N))
+    return fail(c, HS_ERR_INVALID_ARG, "partition does not match the context's current partition");
+  if (!is_device_ptr(params)) return fail(c, HS_ERR_INVALID_ARG, "params must be a device pointer");
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  const size_t in_feat = (size_t)c->layers[0].in;
+  const float* xd = reinterpret_cast<const float*>(x);
+  const int32_t* yd = y;
+  if (!is_device_ptr(x)) {
+    if (!c->d_xstage) {
+      hs_status r = dalloc(c, &c->d_xstage, sizeof(float) * c->N * in_feat);
+      if (r != HS_OK) return r;
+    }
+    HS_CUDA(c, cudaMemcpyAsync(c->d_xstage, x, sizeof(float) * c->N * in_feat, cudaMemcpyHostToDevice, s));
+    xd = reinterpret_cast<const float*>(c->d_xstage);
+  }
+  if (!is_device_ptr(y)) {
+    if (!c->d_ystage) {
+      hs_status r = dalloc(c, &c->d_ystage, sizeof(int32_t) * c->N);
+      if (r != HS_OK) return r;
+    }
+    HS_CUDA(c, cudaMemcpyAsync(c->d_ystage, y, sizeof(int32_t) * c->N, cudaMemcpyHostToDevice, s));
+    yd = c->d_ystage;
+  }
+  if (c->precision == HS_BF16 && (!c->shadow_valid || c->shadow_src != params)) {
+    PhaseScope ph(c, HS_PHASE_CAST, s);
+    hs::launch_cast_f32_bf16(params, c->d_shadow, c->P, s);
+    ph.launched();
+  }
+  if (c->debug && !c->d_gdebug) {
+    hs_status r = dalloc(c, &c->d_gdebug, sizeof(float) * c->Ps);
+    if (r != HS_OK) return r;
+  }
+  hs_status st = c->precision == HS_BF16 ? mlp_step_bf16(c, params, xd, yd, s) : mlp_step_fp32(c, params, xd, yd, s);
+  if (st != HS_OK) return st;
+  {
+    PhaseScope ph(c, HS_PHASE_UPDATE, s);
+    hs::launch_reduce_update(params, c->d_slabs, c->Ps, c->M, c->d_w, lr, c->P,
+                             c->precision == HS_BF16 ? c->d_shadow : nullptr, c->debug ? c->d_gdebug : nullptr,
+                             c->num_sms, s);
+    ph.launched();
+  }
+  HS_CUDA(c, cudaGetLastError());
+  c->shadow_src = params;
+  c->shadow_valid = (c->precision == HS_BF16);
+  c->gdebug_valid = c->debug;
+  if (loss_out) {
+    HS_CUDA(c, cudaMemcpyAsync(c->h_status, c->d_status, sizeof(DevStatus), cudaMemcpyDeviceToHost, s));
+    HS_CUDA(c, cudaStreamSynchronize(s));
+    *loss_out = c->h_status->loss;
+    if (c->h_status->err != hs::kDevOk) {
+      const int code = c->h_status->err, info = c->h_status->err_info;
+      cudaMemsetAsync(c->d_status, 0, sizeof(DevStatus), s);
+      cudaStreamSynchronize(s);
+      char buf[160];
+      std::snprintf(buf, sizeof(buf), "device check failed: code %d (%s), detail %d", code,
+                    code == hs::kDevWaitTimeout ? "bounded wait expired" : "label out of range", info);
+      return fail(c, HS_ERR_DEVICE_CHECK, buf);
+    }
+  }
+  return HS_OK;
+}
+
+hs_status hs_set_profiling(hs_ctx* c, int32_t enable) {
+  if (!c) return HS_ERR_INVALID_ARG;
+  c->profiling = enable != 0;
+  return HS_OK;
+}
+
+hs_status hs_read_profile(hs_ctx* c, double* ms_out, int64_t* launches_out) {
+  if (!c) return HS_ERR_INVALID_ARG;
+  c->err.clear();
+  double ms[HS_PHASE_COUNT] = {0};
+  cudaError_t first = cudaSuccess;
+  for (auto& r : c->pending) {
+    cudaError_t e = cudaEventSynchronize(r.b);
+    float t = 0.f;
+    if (e == cudaSuccess) e = cudaEventElapsedTime(&t, r.a, r.b);
+    if (e != cudaSuccess && first == cudaSuccess) first = e;
+    ms[r.phase] += t;
+    c->event_pool.push_back(r.a);
+    c->event_pool.push_back(r.b);
+  }
+  c->pending.clear();
+  if (ms_out)
+    for (int i = 0; i < HS_PHASE_COUNT; ++i) ms_out[i] = ms[i];
+  if (launches_out)
+    for (int i = 0; i < HS_PHASE_COUNT; ++i) launches_out[i] = c->launches[i];
+  for (int i = 0; i < HS_PHASE_COUNT; ++i) c->launches[i] = 0;
+  if (first != cudaSuccess) return cuda_fail(c, first, "reading profile events");
+  return HS_OK;
+}
+
+hs_status hs_set_debug(hs_ctx* c, int32_t enable) {
+  if (!c) return HS_ERR_INVALID_ARG;
+  c->debug = enable != 0;
+  return HS_OK;
+}
+
+hs_status hs_debug_grads(hs_ctx* c, float* g_out, float* slabs_out, void* stream) {
+  if (!c) return HS_ERR_INVALID_ARG;
+  c->err.clear();
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (g_out) {
+    if (!c->gdebug_valid || !c->d_gdebug)
+      return fail(c, HS_ERR_INVALID_ARG, "no synchronised gradient kept: call hs_set_debug(ctx, 1) before hs_step");
+    HS_CUDA(c, cudaMemcpyAsync(g_out, c->d_gdebug, sizeof(float) * c->P, cudaMemcpyDeviceToDevice, s));
+  }
+  if (slabs_out) {
+    HS_CUDA(c, cudaMemcpy2DAsync(slabs_out, sizeof(float) * c->P, c->d_slabs, sizeof(float) * c->Ps,
+                                 sizeof(float) * c->P, c->M, cudaMemcpyDeviceToDevice, s));
+  }
+  return HS_OK;
+}
+
+hs_status hs_worker_losses(hs_ctx* c, float* losses_out) {
+  if (!c || !losses_out) return HS_ERR_INVALID_ARG;
+  c->err.clear();
+  HS_CUDA(c, cudaDeviceSynchronize());
+  HS_CUDA(c, cudaMemcpy(losses_out, c->d_lm, sizeof(float) * c->M, cudaMemcpyDeviceToHost));
+  return HS_OK;
+}
+
+void hs_destroy(hs_ctx* c) {
+  if (!c) return;
+  cudaDeviceSynchronize();
+  free_all(c);
+  delete c;
+}
+
+hs_status hs_debug_gemm_bf16(int32_t mode, int32_t M, int32_t N, int32_t K, const void* A, int64_t lda, const void* B,
+                             int64_t ldb, void* D, int64_t ldd, const float* bias, const void* Z, int64_t ldz,
+                             const int32_t* k_offsets_host, int32_t groups, int64_t d_gstride, void* stream) {
+  g_init_error.clear();
+  if (M < 1 || N < 1 || K < 0 || !A || !B || !D) return fail(nullptr, HS_ERR_INVALID_ARG, "bad GEMM arguments");
+  const bool bf16_out = (mode == HS_GEMM_FWD_RELU || mode == HS_GEMM_DGRAD);
+  if (lda % 8 || ldb % 8 || (bf16_out ? ldd % 8 : ldd % 4) || (mode == HS_GEMM_DGRAD && (ldz % 8 || !Z)) ||
+      d_gstride % 4)
+    return fail(nullptr, HS_ERR_INVALID_ARG, "leading dimensions must be multiples of 8 elements");
+  auto a16 = [](const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; };
+  if (!a16(D) || (bias && !a16(bias)) || (Z && !a16(Z)))
+    return fail(nullptr, HS_ERR_INVALID_ARG, "D, bias and Z must be 16-byte aligned");
+  if (mode < HS_GEMM_FWD_RELU || mode > HS_GEMM_WGRAD) return fail(nullptr, HS_ERR_INVALID_ARG, "unknown mode");
+  if ((mode == HS_GEMM_FWD_RELU || mode == HS_GEMM_FWD_LOGITS) && !bias)
+    return fail(nullptr, HS_ERR_INVALID_ARG, "bias required");
+  const char* why = nullptr;
+  if (!hs::tc_init_driver(&why)) return fail(nullptr, HS_ERR_CUDA, why);
+  int dev = 0, sms = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  std::vector<hs::TcGemmParams> plans;
+  const auto* pa = reinterpret_cast<const __nv_bfloat16*>(A);
+  const auto* pb = reinterpret_cast<const __nv_bfloat16*>(B);
+  if (mode == HS_GEMM_WGRAD) {
+    if (!k_offsets_host || groups < 1) return fail(nullptr, HS_ERR_INVALID_ARG, "k_offsets and groups required");
+    for (int g0 = 0; g0 < groups; g0 += hs::kTcMaxGroups) {
+      const int ng = std::min(hs::kTcMaxGroups, groups - g0);
+      plans.emplace_back();
+      hs::TcGemmParams& p = plans.back();
+      std::memset(&p, 0, sizeof(p));
+      for (int g = 0; g < ng; ++g) {
+        const int64_t k0 = k_offsets_host[g0 + g], kn = k_offsets_host[g0 + g + 1] - k0;
+        if (kn < 1) return fail(nullptr, HS_ERR_INVALID_ARG, "every group needs K >= 1");
+        if (!hs::tc_make_mnmajor_map(&p.tmA[g], hs::TcOperand{pa + k0 * lda, kn, M, lda}, &why) ||
+            !hs::tc_make_mnmajor_map(&p.tmB[g], hs::TcOperand{pb + k0 * ldb, kn, N, ldb}, &why))
+          return fail(nullptr, HS_ERR_INVALID_ARG, why);
+        p.num_kb[g] = (int)((kn + hs::kTcBK - 1) / hs::kTcBK);
+      }
+      p.groups = ng;
+      p.epi = hs::kTcEpiStoreF32;
+      p.a_mn = 1;
+      p.b_mn = 1;
+      p.D = reinterpret_cast<float*>(D) + (int64_t)g0 * d_gstride;
+      p.d_gstride = d_gstride;
+    }
+  } else {
+    if (K < 1) return fail(nullptr, HS_ERR_INVALID_ARG, "K must be >= 1");
+    plans.emplace_back();
+    hs::TcGemmParams& p = plans.back();
+    std::memset(&p, 0, sizeof(p));
+    bool ok = hs::tc_make_kmajor_map(&p.tmA[0], hs::TcOperand{pa, M, K, lda}, hs::kTcBM, &why);
+    if (mode == HS_GEMM_DGRAD) ok = ok && hs::tc_make_mnmajor_map(&p.tmB[0], hs::TcOperand{pb, K, N, ldb}, &why);
+    else ok = ok && hs::tc_make_kmajor_map(&p.tmB[0], hs::TcOperand{pb, N, K, ldb}, hs::kTcBN, &why);
+    if (!ok) return fail(nullptr, HS_ERR_INVALID_ARG, why);
+    p.num_kb[0] = (K + hs::kTcBK - 1) / hs::kTcBK;
+    p.groups = 1;
+    p.epi = mode == HS_GEMM_FWD_RELU ? hs::kTcEpiBiasReluBf16
+          : mode == HS_GEMM_FWD_LOGITS ? hs::kTcEpiBiasF32 : hs::kTcEpiMaskBf16;
+    p.b_mn = (mode == HS_GEMM_DGRAD);
+    p.D = D;
+    p.bias = bias;
+    p.Z = reinterpret_cast<const __nv_bfloat16*>(Z);
+    p.ldz = ldz;
+  }
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  for (hs::TcGemmParams& p : plans) {
+    p.Mdim = M;
+    p.Ndim = N;
+    p.n_store = N;
+    p.tiles_m = (M + hs::kTcBM - 1) / hs::kTcBM;
+    p.tiles_n = (N + hs::kTcBN - 1) / hs::kTcBN;
+    p.ldd = ldd;
+    p.st = nullptr;
+    cudaError_t e = hs::launch_tc_gemm(p, sms, s);
+    if (e != cudaSuccess) return cuda_fail(nullptr, e, "GEMM launch");
+  }
+  cudaError_t e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) return cuda_fail(nullptr, e, "GEMM run");
+  return HS_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,265 @@
+// Bandwidth-bound kernels of the step: input cast, partition scatter, fused softmax
+// cross-entropy, per-worker loss and bias-gradient reductions, and the fused gradient
+// reduction + SGD update.  All reductions run in a fixed order (deterministic results).
+#include "common.cuh"
+
+namespace hs {
+
+// ------------------------------------------------------------------------------------ cast
+__global__ void cast_f32_bf16_kernel(const float* __restrict__ x, __nv_bfloat16* __restrict__ y,
+                                     int64_t n) {
+  const int64_t nvec = n / 4;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t v = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; v < nvec; v += stride) {
+    const float4 a = __ldcs(reinterpret_cast<const float4*>(x) + v);
+    __nv_bfloat162 lo = __floats2bfloat162_rn(a.x, a.y);
+    __nv_bfloat162 hi = __floats2bfloat162_rn(a.z, a.w);
+    uint2 packed;
+    packed.x = *reinterpret_cast<uint32_t*>(&lo);
+    packed.y = *reinterpret_cast<uint32_t*>(&hi);
+    reinterpret_cast<uint2*>(y)[v] = packed;
+  }
+  for (int64_t j = nvec * 4 + (int64_t)blockIdx.x * blockDim.x + threadIdx.x; j < n; j += stride)
+    y[j] = __float2bfloat16_rn(x[j]);
+}
+
+void launch_cast_f32_bf16(const float* x, __nv_bfloat16* y, int64_t n, cudaStream_t s) {
+  if (n <= 0) return;
+  int64_t blocks = (n / 4 + 255) / 256;
+  if (blocks < 1) blocks = 1;
+  if (blocks > 4096) blocks = 4096;
+  cast_f32_bf16_kernel<<<(int)blocks, 256, 0, s>>>(x, y, n);
+}
+
+// ------------------------------------------------------------------------ partition scatter
+// Algorithm 1 fixes the partition sizes; samples are laid out as contiguous worker segments:
+// index_map[i] = m for offsets[m] <= i < offsets[m+1], scale[i] = 1 / n_m (Eq. 1's mean).
+__global__ void partition_scatter_kernel(const int32_t* __restrict__ offsets, int M, int N,
+                                         int32_t* __restrict__ index_map, float* __restrict__ scale,
+                                         int32_t* __restrict__ index_map_out) {
+  extern __shared__ int32_t s_off[];
+  for (int k = threadIdx.x; k <= M; k += blockDim.x) s_off[k] = offsets[k];
+  __syncthreads();
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= N) return;
+  int lo = 0, hi = M - 1;          // largest m with s_off[m] <= i
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (s_off[mid] <= i) lo = mid; else hi = mid - 1;
+  }
+  index_map[i] = lo;
+  scale[i] = 1.0f / (float)(s_off[lo + 1] - s_off[lo]);
+  if (index_map_out) index_map_out[i] = lo;
+}
+
+void launch_partition_scatter(const int32_t* d_offsets, int M, int N, int32_t* index_map,
+                              float* scale, int32_t* index_map_out, cudaStream_t s) {
+  const int threads = 256;
+  const int blocks = (N + threads - 1) / threads;
+  partition_scatter_kernel<<<blocks, threads, (M + 1) * sizeof(int32_t), s>>>(
+      d_offsets, M, N, index_map, scale, index_map_out);
+}
+
+// ------------------------------------------------------------------ softmax cross-entropy
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  return v;
+}
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+__device__ __forceinline__ void record_error(DevStatus* st, int32_t code, int32_t info) {
+  if (atomicCAS(&st->err, 0, code) == 0) st->err_info = info;
+}
+
+// One warp per sample row i (Eq. 1 per-sample loss and its gradient):
+//   ce_i = logsumexp(z_i) - z_{i,y_i},  delta_i = (softmax(z_i) - onehot(y_i)) * scale_i,
+// scale_i = 1/n_{m(i)} (the derivative of worker m(i)'s mean loss).
+template <bool kBf16>
+__global__ void softmax_xent_kernel(const float* __restrict__ logits, int ldl,
+                                    const int32_t* __restrict__ y, const float* __restrict__ scale,
+                                    int N, int C, void* __restrict__ delta, int ldd,
+                                    float* __restrict__ ce, DevStatus* st) {
+  const int warps_per_block = blockDim.x >> 5;
+  const int row = blockIdx.x * warps_per_block + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (row >= N) return;
+  const float* z = logits + (int64_t)row * ldl;
+  int label = y[row];
+  if (label < 0 || label >= C) {
+    if (lane == 0) record_error(st, kDevBadLabel, row);
+    label = label < 0 ? 0 : C - 1;
+  }
+  float mx = -INFINITY;
+  for (int j = lane; j < C; j += 32) mx = fmaxf(mx, z[j]);
+  mx = warp_max(mx);
+  float se = 0.f;
+  for (int j = lane; j < C; j += 32) se += expf(z[j] - mx);
+  se = warp_sum(se);
+  const float lse = mx + logf(se);
+  if (lane == 0) ce[row] = lse - z[label];
+  const float inv = 1.0f / se;
+  const float sc = scale[row];
+  for (int j = lane; j < ldd; j += 32) {
+    float d = 0.f;
+    if (j < C) d = (expf(z[j] - mx) * inv - (j == label ? 1.f : 0.f)) * sc;
+    if (kBf16)
+      reinterpret_cast<__nv_bfloat16*>(delta)[(int64_t)row * ldd + j] = __float2bfloat16_rn(d);
+    else
+      reinterpret_cast<float*>(delta)[(int64_t)row * ldd + j] = d;
+  }
+}
+
+void launch_softmax_xent(const float* logits, int ldl, const int32_t* y, const float* scale, int N,
+                         int C, void* delta, int ldd, bool delta_bf16, float* ce, DevStatus* st,
+                         cudaStream_t s) {
+  const int threads = 256;
+  const int rows_per_block = threads / 32;
+  const int blocks = (N + rows_per_block - 1) / rows_per_block;
+  if (delta_bf16)
+    softmax_xent_kernel<true><<<blocks, threads, 0, s>>>(logits, ldl, y, scale, N, C, delta, ldd, ce, st);
+  else
+    softmax_xent_kernel<false><<<blocks, threads, 0, s>>>(logits, ldl, y, scale, N, C, delta, ldd, ce, st);
+}
+
+// ------------------------------------------------------------------ per-worker loss reduction
+// L_m = (1/n_m) sum_{i in seg_m} ce_i (Eq. 1); loss = sum_m w_m L_m.  One block, fixed order.
+__global__ void loss_reduce_kernel(const float* __restrict__ ce, const int32_t* __restrict__ offsets,
+                                   int M, const float* __restrict__ w, float* __restrict__ lm,
+                                   DevStatus* st) {
+  __shared__ float red[1024];
+  for (int m = 0; m < M; ++m) {
+    const int b = offsets[m], e = offsets[m + 1];
+    float acc = 0.f;
+    for (int i = b + threadIdx.x; i < e; i += blockDim.x) acc += ce[i];
+    red[threadIdx.x] = acc;
+    __syncthreads();
+    for (int h = blockDim.x >> 1; h > 0; h >>= 1) {
+      if (threadIdx.x < h) red[threadIdx.x] += red[threadIdx.x + h];
+      __syncthreads();
+    }
+    if (threadIdx.x == 0) lm[m] = red[0] / (float)(e - b);
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) {
+    float loss = 0.f;
+    for (int m = 0; m < M; ++m) loss += w[m] * lm[m];
+    st->loss = loss;
+  }
+}
+
+void launch_loss_reduce(const float* ce, const int32_t* d_offsets, int M, const float* d_w,
+                        float* lm, DevStatus* st, cudaStream_t s) {
+  loss_reduce_kernel<<<1, 1024, 0, s>>>(ce, d_offsets, M, d_w, lm, st);
+}
+
+// ------------------------------------------------------------------ per-worker bias gradient
+// G_m[b_l][j] = sum_{i in seg_m} delta_l[i][j]: one thread per column, rows in order.
+template <bool kBf16>
+__global__ void bias_grad_kernel(const void* __restrict__ delta, int ld, int width,
+                                 const int32_t* __restrict__ offsets, float* __restrict__ slabs,
+                                 int64_t Ps, int64_t b_off) {
+  const int m = blockIdx.y;
+  const int j = blockIdx.x * blockDim.x + threadIdx.x;
+  if (j >= width) return;
+  const int b = offsets[m], e = offsets[m + 1];
+  float acc = 0.f;
+#pragma unroll 8
+  for (int i = b; i < e; ++i) {
+    if (kBf16)
+      acc += __bfloat162float(reinterpret_cast<const __nv_bfloat16*>(delta)[(int64_t)i * ld + j]);
+    else
+      acc += reinterpret_cast<const float*>(delta)[(int64_t)i * ld + j];
+  }
+  slabs[(int64_t)m * Ps + b_off + j] = acc;
+}
+
+void launch_bias_grad(const void* delta, bool delta_bf16, int ld, int width, const int32_t* d_offsets,
+                      int M, float* slabs, int64_t Ps, int64_t b_off, cudaStream_t s) {
+  dim3 grid((width + 127) / 128, M);
+  if (delta_bf16)
+    bias_grad_kernel<true><<<grid, 128, 0, s>>>(delta, ld, width, d_offsets, slabs, Ps, b_off);
+  else
+    bias_grad_kernel<false><<<grid, 128, 0, s>>>(delta, ld, width, d_offsets, slabs, Ps, b_off);
+}
+
+// ------------------------------------------------------------------ fused reduce + SGD update
+// Section 1: g = sum_m w_m g^m (w_m = 1/M; Section 4.2: compute-power weights), then
+// theta <- theta - lr * g.  One HBM pass: M slab reads + theta read, theta + bf16 shadow writes.
+__global__ void __launch_bounds__(512) reduce_update_kernel(
+    float* __restrict__ theta, const float* __restrict__ slabs, int64_t Ps, int M,
+    const float* __restrict__ w, float lr, int64_t P, __nv_bfloat16* __restrict__ shadow,
+    float* __restrict__ gdebug) {
+  __shared__ float sw[kMaxWorkers];
+  for (int m = threadIdx.x; m < M; m += blockDim.x) sw[m] = w[m];
+  __syncthreads();
+  const int64_t nvec = P / 4;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  const float4* s4 = reinterpret_cast<const float4*>(slabs);
+  const int64_t ps4 = Ps / 4;
+  for (int64_t v = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; v < nvec; v += stride) {
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    int m = 0;
+    for (; m + 8 <= M; m += 8) {
+      float4 g[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) g[u] = __ldcs(s4 + (int64_t)(m + u) * ps4 + v);
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const float wm = sw[m + u];
+        acc.x = fmaf(wm, g[u].x, acc.x);
+        acc.y = fmaf(wm, g[u].y, acc.y);
+        acc.z = fmaf(wm, g[u].z, acc.z);
+        acc.w = fmaf(wm, g[u].w, acc.w);
+      }
+    }
+    for (; m < M; ++m) {
+      const float4 g = __ldcs(s4 + (int64_t)m * ps4 + v);
+      const float wm = sw[m];
+      acc.x = fmaf(wm, g.x, acc.x);
+      acc.y = fmaf(wm, g.y, acc.y);
+      acc.z = fmaf(wm, g.z, acc.z);
+      acc.w = fmaf(wm, g.w, acc.w);
+    }
+    float4 t = reinterpret_cast<float4*>(theta)[v];
+    t.x = fmaf(-lr, acc.x, t.x);
+    t.y = fmaf(-lr, acc.y, t.y);
+    t.z = fmaf(-lr, acc.z, t.z);
+    t.w = fmaf(-lr, acc.w, t.w);
+    reinterpret_cast<float4*>(theta)[v] = t;
+    if (shadow) {
+      __nv_bfloat162 lo = __floats2bfloat162_rn(t.x, t.y);
+      __nv_bfloat162 hi = __floats2bfloat162_rn(t.z, t.w);
+      uint2 packed;
+      packed.x = *reinterpret_cast<uint32_t*>(&lo);
+      packed.y = *reinterpret_cast<uint32_t*>(&hi);
+      reinterpret_cast<uint2*>(shadow)[v] = packed;
+    }
+    if (gdebug) reinterpret_cast<float4*>(gdebug)[v] = acc;
+  }
+  for (int64_t j = nvec * 4 + (int64_t)blockIdx.x * blockDim.x + threadIdx.x; j < P; j += stride) {
+    float acc = 0.f;
+    for (int m = 0; m < M; ++m) acc = fmaf(sw[m], slabs[(int64_t)m * Ps + j], acc);
+    const float t = fmaf(-lr, acc, theta[j]);
+    theta[j] = t;
+    if (shadow) shadow[j] = __float2bfloat16_rn(t);
+    if (gdebug) gdebug[j] = acc;
+  }
+}
+
+void launch_reduce_update(float* theta, const float* slabs, int64_t Ps, int M, const float* d_w,
+                          float lr, int64_t P, __nv_bfloat16* shadow, float* gdebug, int num_sms,
+                          cudaStream_t s) {
+  const int threads = 512;
+  int64_t blocks = (P / 4 + threads - 1) / threads;
+  const int64_t cap = (int64_t)num_sms * 4;
+  if (blocks > cap) blocks = cap;
+  if (blocks < 1) blocks = 1;
+  reduce_update_kernel<<<(int)blocks, threads, 0, s>>>(theta, slabs, Ps, M, d_w, lr, P, shadow, gdebug);
+}
+
+}  // namespace hs

@@ -1,0 +1,77 @@
+"""Shared helpers for the GPU parity tests: run the library through its binding and the oracle
+on identical seeded inputs."""
+import numpy as np
+import torch
+
+import synth
+import paper_2110_08941_gb300 as hs
+from oracle import cnn, mlp, sgd
+from oracle import partition as P
+
+SYNC_TO_ORACLE = {hs.HS_SYNC_MEAN: sgd.SYNC_MEAN, hs.HS_SYNC_CP_WEIGHTED: sgd.SYNC_CP_WEIGHTED,
+                  hs.HS_SYNC_CP_LITERAL: sgd.SYNC_CP_LITERAL}
+
+
+def rel(a, b) -> float:
+    a = np.asarray(a, dtype=np.float64)
+    b = np.asarray(b, dtype=np.float64)
+    return float(np.linalg.norm(a - b) / max(np.linalg.norm(b), 1e-300))
+
+
+def grad_fn(arch):
+    return mlp.worker_loss_grad if arch == synth.MLP else cnn.worker_loss_grad
+
+
+def run_library(arch, dims, M, N, weights, x, y, theta0, lr, steps, precision, sync, repartition=None,
+                keep_slabs=False):
+    """Returns dict(theta, losses, g_first, slabs_first, counts, index_map)."""
+    ctx = hs.hs_init(arch, dims, M, N, compute_weights=weights, precision=precision, sync=sync)
+    try:
+        hs.hs_set_debug(ctx, True)
+        params = torch.tensor(theta0, device="cuda")
+        xd = torch.from_numpy(np.ascontiguousarray(x)).cuda()
+        yd = torch.from_numpy(np.ascontiguousarray(y)).cuda()
+        im = torch.empty(N, dtype=torch.int32, device="cuda")
+        part = hs.hs_partition(ctx, index_map_out=im)
+        out = dict(losses=[], counts=[list(part.counts)], index_maps=[im.cpu().numpy().copy()])
+        for t in range(steps):
+            if repartition is not None and t > 0 and t in repartition:
+                part = hs.hs_partition(ctx, repartition[t], index_map_out=im)
+                out["counts"].append(list(part.counts))
+                out["index_maps"].append(im.cpu().numpy().copy())
+            out["losses"].append(hs.hs_step(ctx, params, xd, yd, part, lr))
+            if t == 0:
+                g = torch.empty(ctx.P, device="cuda")
+                slabs = torch.empty(M, ctx.P, device="cuda") if keep_slabs else None
+                hs.hs_debug_grads(ctx, g, slabs)
+                out["g_first"] = g.cpu().numpy().astype(np.float64)
+                out["slabs_first"] = slabs.cpu().numpy().astype(np.float64) if keep_slabs else None
+                out["worker_losses_first"] = hs.hs_worker_losses(ctx)
+        torch.cuda.synchronize()
+        out["theta"] = params.cpu().numpy().astype(np.float64)
+        return out
+    finally:
+        ctx.close()
+
+
+def run_oracle(arch, dims, M, N, weights, x, y, theta0, lr, steps, sync, repartition=None, keep_slabs=False):
+    fn = grad_fn(arch)
+    mode = SYNC_TO_ORACLE[sync]
+    cp = list(weights) if weights is not None else [1.0] * M
+    sizes = P.partition_sizes(cp, N)
+    th = np.asarray(theta0, dtype=np.float64)
+    out = dict(losses=[], counts=[list(sizes)])
+    for t in range(steps):
+        if repartition is not None and t > 0 and t in repartition:
+            cp = list(repartition[t])
+            sizes = P.partition_sizes(cp, N)
+            out["counts"].append(list(sizes))
+        th, loss, g, slabs, wl = sgd.step(fn, th, dims, x, y, sizes, lr, mode, keep_slabs=(keep_slabs and t == 0),
+                                          cp=cp)
+        out["losses"].append(loss)
+        if t == 0:
+            out["g_first"] = g
+            out["slabs_first"] = slabs
+            out["worker_losses_first"] = wl
+    out["theta"] = th
+    return out

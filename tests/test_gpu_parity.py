@@ -1,0 +1,141 @@
+"""GPU step vs the fp64 oracle on identical seeded inputs.
+
+Acceptance: partitions and index maps bit-exact; the first step's synchronised gradient within
+relative L2 1e-2 (bf16 path) or 1e-5 (fp32 check path); parameters after 10 steps within relative
+L2 2e-2 (also checked on the parameter change theta_10 - theta_0, a stricter reading)."""
+import functools
+
+import numpy as np
+import pytest
+
+import synth
+import paper_2110_08941_gb300 as hs
+from oracle import partition as P
+from tests.gpu_helpers import rel, run_library, run_oracle
+
+pytestmark = pytest.mark.gpu
+
+TOL_G = {hs.HS_BF16: 1e-2, hs.HS_FP32_CHECK: 1e-5}
+TOL_THETA = 2e-2
+
+
+def _check(lib, orc, theta0, precision, n_steps):
+    assert lib["counts"] == orc["counts"]
+    for counts, im in zip(lib["counts"], lib["index_maps"]):
+        assert np.array_equal(im, np.asarray(P.index_map(counts), dtype=np.int32))
+    assert rel(lib["g_first"], orc["g_first"]) <= TOL_G[precision]
+    assert rel(lib["theta"], orc["theta"]) <= TOL_THETA
+    d_lib, d_orc = lib["theta"] - theta0, orc["theta"] - theta0
+    assert rel(d_lib, d_orc) <= (TOL_THETA if precision == hs.HS_BF16 else 1e-4)
+    ltol = 1e-2 if precision == hs.HS_BF16 else 1e-5
+    for a, b in zip(lib["losses"], orc["losses"]):
+        assert abs(a - b) <= ltol * abs(b)
+    for a, b in zip(lib["worker_losses_first"], orc["worker_losses_first"]):
+        assert abs(a - b) <= ltol * abs(b)
+
+
+CASES = [
+    # name, precision, sync
+    (synth.CFG1, hs.HS_FP32_CHECK, hs.HS_SYNC_CP_WEIGHTED),
+    (synth.CFG1, hs.HS_FP32_CHECK, hs.HS_SYNC_MEAN),
+    (synth.CFG1, hs.HS_BF16, hs.HS_SYNC_CP_WEIGHTED),
+    (synth.CFG1, hs.HS_BF16, hs.HS_SYNC_MEAN),
+    (synth.CFG1, hs.HS_BF16, hs.HS_SYNC_CP_LITERAL),
+    (synth.CFG2, hs.HS_FP32_CHECK, hs.HS_SYNC_CP_WEIGHTED),
+    (synth.CFG2, hs.HS_BF16, hs.HS_SYNC_CP_WEIGHTED),
+    (synth.CFG2, hs.HS_BF16, hs.HS_SYNC_MEAN),
+]
+
+
+@functools.lru_cache(maxsize=None)
+def _inputs(name):
+    wl = synth.WORKLOADS[name]
+    x, y = synth.make_batch(wl)
+    return wl, x, y, synth.make_params(wl), synth.initial_weights(wl)
+
+
+@functools.lru_cache(maxsize=None)
+def _oracle_run(name, sync, steps):
+    wl, x, y, theta0, w = _inputs(name)
+    return run_oracle(wl.arch, wl.dims, wl.workers, wl.global_batch, w, x, y, theta0, wl.lr, steps, sync)
+
+
+@pytest.mark.parametrize("name,precision,sync", CASES)
+def test_workload_10_steps(name, precision, sync):
+    wl, x, y, theta0, w = _inputs(name)
+    steps = 10
+    lib = run_library(wl.arch, wl.dims, wl.workers, wl.global_batch, w, x, y, theta0, wl.lr, steps, precision, sync)
+    orc = _oracle_run(name, sync, steps)
+    _check(lib, orc, theta0.astype(np.float64), precision, steps)
+
+
+def test_drift_workload_repartition():
+    """3072->2048->2048->10, N=4096, M=8, seeded drifting worker speeds: the partition is recomputed
+    from windowed throughputs (Eq. 2) between steps; two steps keep the oracle inside the test budget."""
+    wl = synth.WORKLOADS[synth.CFG3]
+    x, y = synth.make_batch(wl)
+    theta0 = synth.make_params(wl)
+    speeds = synth.drift_walk(wl.workers, 20, wl.seed)
+    rep = {1: list(synth.window_throughputs(speeds[0:10]))}
+    lib = run_library(wl.arch, wl.dims, wl.workers, wl.global_batch, None, x, y, theta0, wl.lr, 2, hs.HS_BF16,
+                      hs.HS_SYNC_CP_WEIGHTED, repartition=rep)
+    orc = run_oracle(wl.arch, wl.dims, wl.workers, wl.global_batch, None, x, y, theta0, wl.lr, 2,
+                     hs.HS_SYNC_CP_WEIGHTED, repartition=rep)
+    assert lib["counts"][0] == [512] * 8 and lib["counts"][1] != lib["counts"][0]
+    _check(lib, orc, theta0.astype(np.float64), hs.HS_BF16, 2)
+
+
+EDGE = [
+    # dims, N, M, weights: one sample per worker; ragged tails in every GEMM dimension; M = 1
+    ((24, 16, 3), 5, 5, None),
+    ((64, 40, 7), 300, 3, [1.0, 1.0, 5.0]),
+    ((136, 264, 136, 1000), 517, 7, [0.3, 2.0, 1.0, 1.0, 0.7, 4.0, 0.01]),
+    ((32, 8), 130, 1, None),
+    ((40, 48, 56, 9), 257, 40, None),
+]
+
+
+@pytest.mark.parametrize("precision", [hs.HS_BF16, hs.HS_FP32_CHECK])
+@pytest.mark.parametrize("dims,N,M,weights", EDGE)
+def test_edge_shapes(dims, N, M, weights, precision):
+    rng = np.random.default_rng(len(dims) * 100 + N)
+    x = rng.standard_normal((N, dims[0]), dtype=np.float32)
+    y = rng.integers(0, dims[-1], N, dtype=np.int32)
+    theta0 = synth.he_normal_params(synth.MLP, dims, 7)
+    theta0[theta0.size - dims[-1]:] = rng.standard_normal(dims[-1]).astype(np.float32) * 0.1   # nonzero last bias
+    for sync in (hs.HS_SYNC_MEAN, hs.HS_SYNC_CP_WEIGHTED):
+        lib = run_library(synth.MLP, dims, M, N, weights, x, y, theta0, 0.05, 10, precision, sync)
+        orc = run_oracle(synth.MLP, dims, M, N, weights, x, y, theta0, 0.05, 10, sync)
+        _check(lib, orc, theta0.astype(np.float64), precision, 10)
+
+
+def test_slabs_are_per_worker_gradients():
+    wl = synth.WORKLOADS[synth.CFG2]
+    x, y = synth.make_batch(wl)
+    theta0 = synth.make_params(wl)
+    w = synth.initial_weights(wl)
+    for precision in (hs.HS_FP32_CHECK, hs.HS_BF16):
+        lib = run_library(wl.arch, wl.dims, wl.workers, wl.global_batch, w, x, y, theta0, wl.lr, 1, precision,
+                          hs.HS_SYNC_MEAN, keep_slabs=True)
+        orc = run_oracle(wl.arch, wl.dims, wl.workers, wl.global_batch, w, x, y, theta0, wl.lr, 1,
+                         hs.HS_SYNC_MEAN, keep_slabs=True)
+        for m in range(wl.workers):
+            assert rel(lib["slabs_first"][m], orc["slabs_first"][m]) <= TOL_G[precision], m
+
+
+@pytest.mark.parametrize("dims,N,M", [((13, 7, 5), 11, 3), ((3, 2), 4, 2), ((50, 33, 17, 2), 97, 6)])
+def test_fp32_check_path_odd_widths(dims, N, M):
+    rng = np.random.default_rng(N)
+    x = rng.standard_normal((N, dims[0]), dtype=np.float32)
+    y = rng.integers(0, dims[-1], N, dtype=np.int32)
+    theta0 = synth.he_normal_params(synth.MLP, dims, 3)
+    w = list(rng.uniform(0.5, 2.0, M))
+    lib = run_library(synth.MLP, dims, M, N, w, x, y, theta0, 0.1, 10, hs.HS_FP32_CHECK, hs.HS_SYNC_CP_WEIGHTED)
+    orc = run_oracle(synth.MLP, dims, M, N, w, x, y, theta0, 0.1, 10, hs.HS_SYNC_CP_WEIGHTED)
+    _check(lib, orc, theta0.astype(np.float64), hs.HS_FP32_CHECK, 10)
+
+
+def test_bf16_rejects_unaligned_widths():
+    with pytest.raises(hs.HsError) as e:
+        hs.hs_init(synth.MLP, (13, 7, 5), 2, 8, precision=hs.HS_BF16)
+    assert e.value.status == hs.HS_ERR_UNSUPPORTED
