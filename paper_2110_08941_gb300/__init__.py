@@ -12,5 +12,7 @@ import importlib as _importlib
 def __getattr__(name):
     if name.startswith("__"):
         raise AttributeError(name)
+    if name in ("build", "binding"):
+        return _importlib.import_module(f"{__name__}.{name}")
     binding = _importlib.import_module(__name__ + ".binding")
     return getattr(binding, name)
