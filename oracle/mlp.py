@@ -17,6 +17,16 @@ Back-propagation is written out layer by layer (no autodiff): for the last
 layer dL/dA_L = (softmax(z) - onehot(y)) / n_m, and for every layer
 dW_l = dA_l^T H_{l-1}, db_l = sum_rows dA_l, dA_{l-1} = (dA_l W_l) * 1[A_{l-1} > 0].
 Inputs are the fp32 arrays the GPU path sees, promoted to fp64.
+
+ReLU'(A) = 1[A > 0] is a floating-point value deciding a 0/1.  A kernel with bf16
+operands (fp32 accumulation) decides it from its own pre-activation, which sits
+within bf16 rounding of the exact one; where |A| is that small the two decisions
+differ, and each flip moves a whole entry of the backward signal.  So that both
+sides take the decision in the same precision, `decide` (optional) names an
+operand rounding: the masks then come from the forward pass evaluated with
+rounded operands (H_0 = x, W_l and the stored activations rounded, exact
+accumulation), while every value of the loss and gradient stays fp64.  With
+`decide=None` the masks come from the fp64 forward itself.
 """
 from __future__ import annotations
 
@@ -64,6 +74,30 @@ def forward(theta: np.ndarray, dims: Sequence[int], x: np.ndarray):
     return acts, hs
 
 
+def round_bf16(a) -> np.ndarray:
+    """Round to the nearest bfloat16 (8 significant bits, ties to even), from the fp32 value.
+
+    bfloat16 is the top half of an IEEE fp32 word; round-to-nearest-even on the discarded low
+    16 bits is adding 0x7FFF plus the lowest kept bit, then truncating.  Finite inputs only."""
+    f = np.ascontiguousarray(np.asarray(a, dtype=np.float32))
+    u = f.view(np.uint32).astype(np.uint64)
+    kept_lsb = (u >> np.uint64(16)) & np.uint64(1)
+    r = ((u + np.uint64(0x7FFF) + kept_lsb) >> np.uint64(16)) << np.uint64(16)
+    return r.astype(np.uint32).view(np.float32).astype(np.float64)
+
+
+def relu_decisions(theta: np.ndarray, dims: Sequence[int], x: np.ndarray, rnd) -> List[np.ndarray]:
+    """1[A_l > 0] for each hidden layer, with A_l evaluated from operands rounded by `rnd`."""
+    ws, bs = unpack(np.asarray(theta, dtype=np.float64), dims)
+    h = rnd(x)
+    masks = []
+    for l in range(len(ws) - 1):
+        a = h @ rnd(ws[l]).T + bs[l]
+        masks.append(a > 0.0)
+        h = rnd(np.maximum(a, 0.0))
+    return masks
+
+
 def cross_entropy_rows(z: np.ndarray, y: np.ndarray):
     """Per-row CE(z_i, y_i) = logsumexp(z_i) - z_{i, y_i} and softmax(z_i)."""
     zmax = z.max(axis=1, keepdims=True)
@@ -75,13 +109,19 @@ def cross_entropy_rows(z: np.ndarray, y: np.ndarray):
 
 
 def worker_loss_grad(theta: np.ndarray, dims: Sequence[int], x_m: np.ndarray,
-                     y_m: np.ndarray) -> Tuple[float, np.ndarray]:
-    """L_m and g^m = grad L_m (flat fp64 [P]) on one worker's segment (Eq. 1)."""
+                     y_m: np.ndarray, decide=None) -> Tuple[float, np.ndarray]:
+    """L_m and g^m = grad L_m (flat fp64 [P]) on one worker's segment (Eq. 1).
+
+    decide: None, or an operand rounding (e.g. round_bf16) from which the ReLU' masks are taken."""
     theta = np.asarray(theta, dtype=np.float64)
     ws, _ = unpack(theta, dims)
     lay, p = layout(dims)
     n_m = x_m.shape[0]
     acts, hs = forward(theta, dims, x_m)
+    if decide is None:
+        masks = [a > 0.0 for a in acts[:-1]]
+    else:
+        masks = relu_decisions(theta, dims, x_m, decide)
     y_m = np.asarray(y_m, dtype=np.int64)
     ce, prob = cross_entropy_rows(acts[-1], y_m)
     loss = float(ce.sum() / n_m)
@@ -94,7 +134,7 @@ def worker_loss_grad(theta: np.ndarray, dims: Sequence[int], x_m: np.ndarray,
         g[w_off:w_off + shape[0] * shape[1]] = (d_a.T @ hs[l]).reshape(-1)
         g[b_off:b_off + o] = d_a.sum(axis=0)
         if l > 0:
-            d_a = (d_a @ ws[l]) * (acts[l - 1] > 0.0)
+            d_a = (d_a @ ws[l]) * masks[l - 1]
     return loss, g
 
 

@@ -51,10 +51,11 @@ def worker_grads(grad_fn: Callable, theta, dims, x, y, sizes):
 
 
 def step(grad_fn: Callable, theta, dims, x, y, sizes, lr: float, mode: int,
-         keep_slabs: bool = False, cp=None):
+         keep_slabs: bool = False, cp=None, **grad_kwargs):
     """One synchronous step: per-worker (L_m, g^m), g = sum_m w_m g^m, theta - lr * g.
 
-    Returns (theta_new fp64, loss, g, slabs or None, per-worker losses).
+    Returns (theta_new fp64, loss, g, slabs or None, per-worker losses).  grad_kwargs go to
+    grad_fn (e.g. the ReLU-decision precision of the per-worker gradient).
     Accumulates sum_m w_m g^m worker by worker, so memory stays at O(P) unless
     the per-worker gradients are asked for.
     """
@@ -66,7 +67,7 @@ def step(grad_fn: Callable, theta, dims, x, y, sizes, lr: float, mode: int,
     losses = []
     for m in range(len(sizes)):
         sl = slice(off[m], off[m + 1])
-        l_m, g_m = grad_fn(theta, dims, x[sl], y[sl])
+        l_m, g_m = grad_fn(theta, dims, x[sl], y[sl], **grad_kwargs)
         losses.append(l_m)
         g += w[m] * g_m
         if keep_slabs:

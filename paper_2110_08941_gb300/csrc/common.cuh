@@ -40,6 +40,13 @@ void launch_loss_reduce(const float* ce, const int32_t* d_offsets, int M, const 
 // slabs[m*Ps + b_off + j] = sum_{i in seg_m} delta[i*ld + j], j < width
 void launch_bias_grad(const void* delta, bool delta_bf16, int ld, int width, const int32_t* d_offsets,
                       int M, float* slabs, int64_t Ps, int64_t b_off, cudaStream_t s);
+// Same reduction for bf16 delta with 16-byte rows (ld % 8 == 0): row chunks (worker, begin, end) of at
+// most bias_grad_chunk_rows() rows, chunk_begin[m] = first chunk of worker m (M + 1 entries), partial
+// scratch of n_chunks x width floats.  Launches two kernels.
+int bias_grad_chunk_rows();
+void launch_bias_grad_bf16(const __nv_bfloat16* delta, int ld, int width, const int4* d_chunks, int n_chunks,
+                           const int32_t* d_chunk_begin, int M, float* partial, float* slabs, int64_t Ps,
+                           int64_t b_off, cudaStream_t s);
 // theta[j] -= lr * sum_m w[m] * slabs[m*Ps + j]; shadow[j] = bf16(theta[j]); gdebug[j] = g (optional)
 void launch_reduce_update(float* theta, const float* slabs, int64_t Ps, int M, const float* d_w,
                           float lr, int64_t P, __nv_bfloat16* shadow, float* gdebug, int num_sms,

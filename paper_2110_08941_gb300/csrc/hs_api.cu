@@ -45,6 +45,10 @@ struct hs_ctx {
   int32_t* d_index_map = nullptr;
   float* d_scale = nullptr;
   float* d_w = nullptr;
+  int4* d_bg_chunks = nullptr;       // bias-gradient row chunks (worker, begin, end, 0)
+  int32_t* d_bg_chunk_begin = nullptr;
+  int n_bg_chunks = 0;
+  float* d_bg_partial = nullptr;     // [max chunks, maxw] partial column sums
 
   // workspace
   std::vector<void*> d_act;        // H_0 .. H_{L-1}
@@ -296,8 +300,21 @@ hs_status apply_partition(hs_ctx* c, const std::vector<int32_t>& sizes, const st
   compute_weights(c);
   std::vector<float> wf(c->weights.begin(), c->weights.end());
   HS_CUDA(c, cudaMemcpyAsync(c->d_w, wf.data(), sizeof(float) * c->M, cudaMemcpyHostToDevice, s));
+  std::vector<int4> chunks;
+  std::vector<int32_t> chunk_begin;
   if (changed) {
     HS_CUDA(c, cudaMemcpyAsync(c->d_offsets, c->offsets.data(), sizeof(int32_t) * (c->M + 1),
+                               cudaMemcpyHostToDevice, s));
+    const int R = hs::bias_grad_chunk_rows();
+    for (int m = 0; m < c->M; ++m) {
+      chunk_begin.push_back((int32_t)chunks.size());
+      for (int r = c->offsets[m]; r < c->offsets[m + 1]; r += R)
+        chunks.push_back(make_int4(m, r, std::min(r + R, c->offsets[m + 1]), 0));
+    }
+    chunk_begin.push_back((int32_t)chunks.size());
+    c->n_bg_chunks = (int)chunks.size();
+    HS_CUDA(c, cudaMemcpyAsync(c->d_bg_chunks, chunks.data(), sizeof(int4) * chunks.size(), cudaMemcpyHostToDevice, s));
+    HS_CUDA(c, cudaMemcpyAsync(c->d_bg_chunk_begin, chunk_begin.data(), sizeof(int32_t) * chunk_begin.size(),
                                cudaMemcpyHostToDevice, s));
   }
   if (changed || index_map_out) {
@@ -337,6 +354,7 @@ hs_status dalloc(hs_ctx* c, T** p, size_t bytes) {
 void free_all(hs_ctx* c) {
   auto f = [](void* p) { if (p) cudaFree(p); };
   f(c->d_offsets); f(c->d_index_map); f(c->d_scale); f(c->d_w);
+  f(c->d_bg_chunks); f(c->d_bg_chunk_begin); f(c->d_bg_partial);
   for (void* p : c->d_act) f(p);
   f(c->d_logits); f(c->d_delta[0]); f(c->d_delta[1]); f(c->d_ce); f(c->d_lm); f(c->d_status);
   f(c->d_slabs); f(c->d_shadow); f(c->d_gdebug); f(c->d_xstage); f(c->d_ystage);
@@ -463,9 +481,10 @@ hs_status mlp_step_bf16(hs_ctx* c, float* params, const float* x, const int32_t*
     {
       PhaseScope ph(c, HS_PHASE_BIASGRAD, s);
       const int out_cols = (l == L - 1) ? c->C : ly.out;
-      hs::launch_bias_grad(c->delta_buf(l), true, c->delta_ld(l), out_cols, c->d_offsets, c->M, c->d_slabs, c->Ps,
-                           ly.b_off, s);
-      ph.launched();
+      hs::launch_bias_grad_bf16(reinterpret_cast<const __nv_bfloat16*>(c->delta_buf(l)), c->delta_ld(l), out_cols,
+                                c->d_bg_chunks, c->n_bg_chunks, c->d_bg_chunk_begin, c->M, c->d_bg_partial,
+                                c->d_slabs, c->Ps, ly.b_off, s);
+      ph.launched(2);
     }
     if (l > 0) {
       PhaseScope ph(c, HS_PHASE_DGRAD, s);
@@ -578,6 +597,10 @@ hs_status hs_init(const hs_model_desc* model, int32_t M, const double* compute_w
   chk(dalloc(c, &c->d_index_map, sizeof(int32_t) * N));
   chk(dalloc(c, &c->d_scale, sizeof(float) * N));
   chk(dalloc(c, &c->d_w, sizeof(float) * M));
+  const int max_chunks = c->N / hs::bias_grad_chunk_rows() + M + 1;
+  chk(dalloc(c, &c->d_bg_chunks, sizeof(int4) * max_chunks));
+  chk(dalloc(c, &c->d_bg_chunk_begin, sizeof(int32_t) * (M + 1)));
+  chk(dalloc(c, &c->d_bg_partial, sizeof(float) * (size_t)max_chunks * (size_t)c->maxw));
   c->d_act.assign(c->L, nullptr);
   for (int l = 0; l < c->L; ++l) {
     if (l == 0 && c->precision == HS_FP32_CHECK) continue;   // fp32 reads x in place

@@ -178,6 +178,84 @@ __global__ void bias_grad_kernel(const void* __restrict__ delta, int ld, int wid
   slabs[(int64_t)m * Ps + b_off + j] = acc;
 }
 
+// Two-stage form for bf16 delta (16-byte rows).  Stage 1: each block sums a chunk of <= 128 rows of
+// one worker over 256 columns (a lane owns 8 adjacent columns, loaded as one 16-byte vector; the
+// block's 8 warps take interleaved rows and are combined in a fixed order) into partial[chunk].
+// Stage 2: per worker, the chunk partials are added in chunk order.  Deterministic.
+constexpr int kBgRows = 128;
+constexpr int kBgCols = 256;
+
+__global__ void __launch_bounds__(256) bias_grad_partial_kernel(const __nv_bfloat16* __restrict__ delta, int ld,
+                                                                int width, const int4* __restrict__ chunks,
+                                                                float* __restrict__ partial) {
+  __shared__ float red[8][kBgCols + 8];
+  const int4 ck = chunks[blockIdx.y];       // (worker, row begin, row end, unused)
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int c0 = blockIdx.x * kBgCols + lane * 8;
+  float acc[8];
+#pragma unroll
+  for (int j = 0; j < 8; ++j) acc[j] = 0.f;
+  if (c0 < width) {
+    const __nv_bfloat16* base = delta + c0;
+    int r = ck.y + warp;
+    for (; r + 24 < ck.z; r += 32) {
+      uint4 v[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) v[u] = __ldcs(reinterpret_cast<const uint4*>(base + (int64_t)(r + 8 * u) * ld));
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&v[u]);
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          acc[2 * j] += __low2float(h[j]);
+          acc[2 * j + 1] += __high2float(h[j]);
+        }
+      }
+    }
+    for (; r < ck.z; r += 8) {
+      const uint4 v = __ldcs(reinterpret_cast<const uint4*>(base + (int64_t)r * ld));
+      const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&v);
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        acc[2 * j] += __low2float(h[j]);
+        acc[2 * j + 1] += __high2float(h[j]);
+      }
+    }
+  }
+#pragma unroll
+  for (int j = 0; j < 8; ++j) red[warp][lane * 8 + j] = acc[j];
+  __syncthreads();
+  const int col = blockIdx.x * kBgCols + threadIdx.x;
+  if (col < width) {
+    float t = 0.f;
+#pragma unroll
+    for (int w = 0; w < 8; ++w) t += red[w][threadIdx.x];
+    partial[(int64_t)blockIdx.y * width + col] = t;
+  }
+}
+
+__global__ void bias_grad_combine_kernel(const float* __restrict__ partial, int width,
+                                         const int32_t* __restrict__ chunk_begin, float* __restrict__ slabs,
+                                         int64_t Ps, int64_t b_off) {
+  const int m = blockIdx.y;
+  const int col = blockIdx.x * blockDim.x + threadIdx.x;
+  if (col >= width) return;
+  float t = 0.f;
+  for (int c = chunk_begin[m]; c < chunk_begin[m + 1]; ++c) t += partial[(int64_t)c * width + col];
+  slabs[(int64_t)m * Ps + b_off + col] = t;
+}
+
+int bias_grad_chunk_rows() { return kBgRows; }
+
+void launch_bias_grad_bf16(const __nv_bfloat16* delta, int ld, int width, const int4* d_chunks, int n_chunks,
+                           const int32_t* d_chunk_begin, int M, float* partial, float* slabs, int64_t Ps,
+                           int64_t b_off, cudaStream_t s) {
+  dim3 g1((width + kBgCols - 1) / kBgCols, n_chunks);
+  bias_grad_partial_kernel<<<g1, 256, 0, s>>>(delta, ld, width, d_chunks, partial);
+  dim3 g2((width + 255) / 256, M);
+  bias_grad_combine_kernel<<<g2, 256, 0, s>>>(partial, width, d_chunk_begin, slabs, Ps, b_off);
+}
+
 void launch_bias_grad(const void* delta, bool delta_bf16, int ld, int width, const int32_t* d_offsets,
                       int M, float* slabs, int64_t Ps, int64_t b_off, cudaStream_t s) {
   dim3 grid((width + 127) / 128, M);

@@ -54,8 +54,16 @@ def run_library(arch, dims, M, N, weights, x, y, theta0, lr, steps, precision, s
         ctx.close()
 
 
-def run_oracle(arch, dims, M, N, weights, x, y, theta0, lr, steps, sync, repartition=None, keep_slabs=False):
+def decide_for(precision):
+    """The bf16 kernels take the ReLU' decision from bf16-operand pre-activations; the oracle takes it
+    in the same precision (values stay fp64).  The fp32 check path is compared with the exact oracle."""
+    return mlp.round_bf16 if precision == hs.HS_BF16 else None
+
+
+def run_oracle(arch, dims, M, N, weights, x, y, theta0, lr, steps, sync, repartition=None, keep_slabs=False,
+               decide=None):
     fn = grad_fn(arch)
+    kw = {} if decide is None else {"decide": decide}
     mode = SYNC_TO_ORACLE[sync]
     cp = list(weights) if weights is not None else [1.0] * M
     sizes = P.partition_sizes(cp, N)
@@ -67,7 +75,7 @@ def run_oracle(arch, dims, M, N, weights, x, y, theta0, lr, steps, sync, reparti
             sizes = P.partition_sizes(cp, N)
             out["counts"].append(list(sizes))
         th, loss, g, slabs, wl = sgd.step(fn, th, dims, x, y, sizes, lr, mode, keep_slabs=(keep_slabs and t == 0),
-                                          cp=cp)
+                                          cp=cp, **kw)
         out["losses"].append(loss)
         if t == 0:
             out["g_first"] = g

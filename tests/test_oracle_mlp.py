@@ -168,3 +168,49 @@ def test_loss_decreases():
         theta, loss, _, _, _ = sgd.step(mlp.worker_loss_grad, theta, dims, x, y, sizes, 0.05, sgd.SYNC_CP_WEIGHTED)
         losses.append(loss)
     assert all(b < a for a, b in zip(losses, losses[1:]))
+
+
+def test_round_bf16_matches_torch():
+    rng = np.random.default_rng(0)
+    vals = np.concatenate([
+        rng.standard_normal(20000).astype(np.float32) * np.float32(10.0) ** rng.integers(-30, 30, 20000),
+        rng.standard_normal(1000).astype(np.float32) * np.float32(1e-39),      # fp32 subnormals
+    ]).astype(np.float32)
+    # exact ties: low 16 bits = 0x8000, with even and odd kept parts
+    base = rng.integers(0x3F800000, 0x40800000, 2000, dtype=np.uint32) & np.uint32(0xFFFF0000)
+    ties = (base | np.uint32(0x8000)).view(np.float32)
+    vals = np.concatenate([vals, ties, -ties, np.array([0.0, -0.0, 1.0, -1.0], dtype=np.float32)])
+    want = torch.from_numpy(vals).to(torch.bfloat16).to(torch.float64).numpy()
+    got = mlp.round_bf16(vals)
+    assert np.array_equal(got, want)
+
+
+def test_decision_mode_identity_rounding_is_exact_oracle():
+    dims = (12, 9, 7, 4)
+    theta, x, y = _tiny(dims, 11, 3)
+    l0, g0 = mlp.worker_loss_grad(theta, dims, x, y)
+    l1, g1 = mlp.worker_loss_grad(theta, dims, x, y, decide=lambda a: np.asarray(a, dtype=np.float64))
+    assert l0 == l1 and np.array_equal(g0, g1)
+
+
+def test_bf16_decisions_differ_only_near_kinks():
+    # A decision taken from bf16-rounded operands can only disagree with the exact one where the
+    # exact pre-activation lies within the bf16 rounding of the operands (|A| small).
+    dims = (256, 128, 64, 10)
+    rng = np.random.default_rng(4)
+    _, p = mlp.layout(dims)
+    theta = rng.standard_normal(p) * 0.1
+    x = rng.standard_normal((200, 256))
+    acts, _ = mlp.forward(theta, dims, x)
+    masks = mlp.relu_decisions(theta, dims, x, mlp.round_bf16)
+    flips = 0
+    for a, m in zip(acts[:-1], masks):
+        diff = (a > 0) != m
+        flips += int(diff.sum())
+        if diff.any():
+            assert np.abs(a[diff]).max() < 0.05 * np.abs(a).std()
+    assert flips < 0.01 * sum(a.size for a in acts[:-1])
+    # and the gradient with bf16 decisions stays close to the exact one
+    _, g0 = mlp.worker_loss_grad(theta, dims, x[:50], y := rng.integers(0, 10, 50))
+    _, g1 = mlp.worker_loss_grad(theta, dims, x[:50], y, decide=mlp.round_bf16)
+    assert np.linalg.norm(g1 - g0) < 0.2 * np.linalg.norm(g0)
