@@ -188,6 +188,25 @@ hs_status hs_set_profiling(hs_ctx* ctx, int32_t enable);
  * Waits for the recorded events.  Launch counts are kept whether or not profiling is on. */
 hs_status hs_read_profile(hs_ctx* ctx, double* ms_out, int64_t* launches_out);
 
+/* The partition of hs_partition and its sample->worker map without a context and without
+ * allocating any device memory.  The paper has no counterpart: this is a service for callers
+ * that cannot call cudaMalloc - a data-loading process that shares the GPU under a fixed memory
+ * budget, or code running under an allocator that forbids new device allocations after start-up -
+ * and so cannot create a context (hs_init allocates the whole training workspace).
+ *   cp:            host [M] compute powers (as for hs_partition_sizes); M <= 1024, N >= M.
+ *   counts_out:    host [M] n_m, or NULL.
+ *   index_map_out: device int32 [N], caller-owned: index_map[i] = m for samples of worker m's
+ *                  contiguous segment (identical to hs_partition's index_map_out).
+ * Device scratch: a static offsets table of 1025 int32 in the library's device image, held by
+ * every GPU that loads the library until the process exits.  The first call on a device looks up
+ * that table's device address (cudaGetSymbolAddress, with that device current); make that first
+ * call before any stream capture.  All calls share the table and it keeps the last call's
+ * offsets; calls whose kernels overlap on the GPU (different streams) race on it.
+ * Errors: HS_ERR_INVALID_ARG for M > 1024 or any hs_partition_sizes error, HS_ERR_CUDA; the
+ * message is returned by hs_last_init_error().  Asynchronous on `stream`. */
+hs_status hs_partition_noalloc(int32_t M, int32_t N, const double* cp, int32_t* counts_out,
+                               int32_t* index_map_out, void* stream);
+
 /* Free the context and all its device memory (synchronises the device first).
  * NULL is a no-op. */
 void hs_destroy(hs_ctx* ctx);

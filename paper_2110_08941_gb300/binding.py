@@ -24,7 +24,8 @@ HS_GEMM_FWD_RELU, HS_GEMM_FWD_LOGITS, HS_GEMM_DGRAD, HS_GEMM_WGRAD = 0, 1, 2, 3
 
 EXPORTED = ("hs_partition_sizes", "hs_param_count", "hs_init", "hs_partition", "hs_step", "hs_sync_params",
             "hs_set_debug", "hs_debug_grads", "hs_worker_losses", "hs_destroy", "hs_status_string",
-            "hs_last_error", "hs_last_init_error", "hs_debug_gemm_bf16", "hs_set_profiling", "hs_read_profile")
+            "hs_last_error", "hs_last_init_error", "hs_debug_gemm_bf16", "hs_set_profiling", "hs_read_profile",
+            "hs_partition_noalloc")
 PHASES = ("cast", "forward", "loss", "wgrad", "biasgrad", "dgrad", "update")
 
 
@@ -52,6 +53,7 @@ def _load() -> ctypes.CDLL:
     S = c_int32
     sig = {
         "hs_partition_sizes": (S, [c_int32, c_int32, POINTER(c_double), POINTER(c_int32)]),
+        "hs_partition_noalloc": (S, [c_int32, c_int32, POINTER(c_double), POINTER(c_int32), c_void_p, c_void_p]),
         "hs_param_count": (S, [POINTER(hs_model_desc), POINTER(c_int64)]),
         "hs_init": (S, [POINTER(hs_model_desc), c_int32, POINTER(c_double), c_int32, POINTER(c_void_p)]),
         "hs_partition": (S, [c_void_p, POINTER(c_double), POINTER(c_int32), c_void_p, c_void_p,
@@ -115,6 +117,16 @@ def hs_partition_sizes(cp: Sequence[float], n: int) -> List[int]:
     cpa = (c_double * max(m, 1))(*[float(v) for v in cp])
     out = (c_int32 * max(m, 1))()
     _check(_lib.hs_partition_sizes(m, int(n), cpa, out))
+    return list(out[:m])
+
+
+def hs_partition_noalloc(cp: Sequence[float], n: int, index_map_out, stream=None) -> List[int]:
+    """Partition sizes and the device index map without a context or any device allocation."""
+    m = len(cp)
+    cpa = (c_double * max(m, 1))(*[float(v) for v in cp])
+    out = (c_int32 * max(m, 1))()
+    _check(_lib.hs_partition_noalloc(m, int(n), cpa, out, c_void_p(index_map_out.data_ptr()),
+                                     c_void_p(_stream_ptr(stream))))
     return list(out[:m])
 
 

@@ -26,6 +26,8 @@ struct DevStatus {
 
 hs_status partition_sizes_impl(int32_t M, int32_t N, const double* cp, int32_t* sizes,
                                double* cp_norm, const char** why);
+// Sets the calling thread's message returned by hs_last_init_error() (calls without a context).
+void set_init_error(const char* msg);
 
 // ---------------------------------------------------------------- elementwise / reduction kernels
 void launch_cast_f32_bf16(const float* x, __nv_bfloat16* y, int64_t n, cudaStream_t s);

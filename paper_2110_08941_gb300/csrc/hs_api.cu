@@ -498,6 +498,8 @@ hs_status mlp_step_bf16(hs_ctx* c, float* params, const float* x, const int32_t*
 
 }  // namespace
 
+void hs::set_init_error(const char* msg) { g_init_error = msg ? msg : ""; }
+
 // ====================================================================== C ABI
 extern "C" {
 
