@@ -78,6 +78,24 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* tm,
       ::"r"(dst), "l"(reinterpret_cast<uint64_t>(tm)), "r"(c0), "r"(c1), "r"(bar)
       : "memory");
 }
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap* tm, uint32_t src, int c0, int c1) {
+  asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%1, %2}], [%3];"
+               ::"l"(reinterpret_cast<uint64_t>(tm)), "r"(c0), "r"(c1), "r"(src)
+               : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+// At most one bulk group may still be reading shared memory.
+__device__ __forceinline__ void bulk_wait_read_1() {
+  asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
+}
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+__device__ __forceinline__ void st_shared_v4(uint32_t addr, uint4 v) {
+  asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w)
+               : "memory");
+}
 __device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap* tm) {
   asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(tm)) : "memory");
 }
@@ -188,85 +206,85 @@ __device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
   return *reinterpret_cast<uint32_t*>(&v);
 }
 
+// One epilogue unit: a 128-byte column strip of one accumulator row (32 fp32 or 64 bf16 outputs),
+// computed from `r` (columns n_base..n_base+31) and, for bf16 outputs, `r2` (n_base+32..+63), packed
+// into eight 16-byte words.  Columns past n_store are computed but never stored (the TMA store
+// clips them); only the bias and mask reads are guarded.
 template <int EPI>
-__device__ __forceinline__ void epilogue_chunk(const TcGemmParams& p, uint8_t* dbase, int row, int n_base,
-                                               const uint32_t (&r)[32]) {
-  float v[32];
-  const bool full = (n_base + 32 <= p.n_store);
-  if (EPI == kTcEpiBiasReluBf16 || EPI == kTcEpiBiasF32) {
+__device__ __forceinline__ void epilogue_unit(const TcGemmParams& p, int row, int n_base, const uint32_t (&r)[32],
+                                              const uint32_t (&r2)[32], uint4 (&o)[8]) {
+  if (EPI == kTcEpiStoreF32) {
+#pragma unroll
+    for (int j = 0; j < 8; ++j) o[j] = make_uint4(r[4 * j], r[4 * j + 1], r[4 * j + 2], r[4 * j + 3]);
+  } else if (EPI == kTcEpiBiasF32) {
+    float b[32];
     if (n_base + 32 <= p.Ndim) {
       const float4* b4 = reinterpret_cast<const float4*>(p.bias + n_base);
 #pragma unroll
       for (int j = 0; j < 8; ++j) {
-        const float4 b = __ldg(b4 + j);
-        v[4 * j + 0] = u2f(r[4 * j + 0]) + b.x;
-        v[4 * j + 1] = u2f(r[4 * j + 1]) + b.y;
-        v[4 * j + 2] = u2f(r[4 * j + 2]) + b.z;
-        v[4 * j + 3] = u2f(r[4 * j + 3]) + b.w;
+        const float4 t = __ldg(b4 + j);
+        b[4 * j] = t.x; b[4 * j + 1] = t.y; b[4 * j + 2] = t.z; b[4 * j + 3] = t.w;
       }
     } else {
 #pragma unroll
-      for (int j = 0; j < 32; ++j) v[j] = u2f(r[j]) + ((n_base + j < p.Ndim) ? __ldg(p.bias + n_base + j) : 0.f);
+      for (int j = 0; j < 32; ++j) b[j] = (n_base + j < p.Ndim) ? __ldg(p.bias + n_base + j) : 0.f;
+    }
+#pragma unroll
+    for (int j = 0; j < 8; ++j)
+      o[j] = make_uint4(__float_as_uint(u2f(r[4 * j]) + b[4 * j]), __float_as_uint(u2f(r[4 * j + 1]) + b[4 * j + 1]),
+                        __float_as_uint(u2f(r[4 * j + 2]) + b[4 * j + 2]),
+                        __float_as_uint(u2f(r[4 * j + 3]) + b[4 * j + 3]));
+  } else {
+    // bf16 outputs: 64 columns
+    float v[64];
+#pragma unroll
+    for (int j = 0; j < 32; ++j) {
+      v[j] = u2f(r[j]);
+      v[32 + j] = u2f(r2[j]);
     }
     if (EPI == kTcEpiBiasReluBf16) {
+      if (n_base + 64 <= p.Ndim) {
+        const float4* b4 = reinterpret_cast<const float4*>(p.bias + n_base);
 #pragma unroll
-      for (int j = 0; j < 32; ++j) v[j] = fmaxf(v[j], 0.f);
-    }
-  } else if (EPI == kTcEpiMaskBf16) {
-    const __nv_bfloat16* z = p.Z + (int64_t)row * p.ldz + n_base;
-    if (full) {
-      const uint4* z4 = reinterpret_cast<const uint4*>(z);
+        for (int j = 0; j < 16; ++j) {
+          const float4 t = __ldg(b4 + j);
+          v[4 * j] = fmaxf(v[4 * j] + t.x, 0.f);
+          v[4 * j + 1] = fmaxf(v[4 * j + 1] + t.y, 0.f);
+          v[4 * j + 2] = fmaxf(v[4 * j + 2] + t.z, 0.f);
+          v[4 * j + 3] = fmaxf(v[4 * j + 3] + t.w, 0.f);
+        }
+      } else {
 #pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        const uint4 zz = __ldg(z4 + j);
-        const uint32_t w[4] = {zz.x, zz.y, zz.z, zz.w};
+        for (int j = 0; j < 64; ++j)
+          v[j] = fmaxf(v[j] + ((n_base + j < p.Ndim) ? __ldg(p.bias + n_base + j) : 0.f), 0.f);
+      }
+    } else {   // kTcEpiMaskBf16: ReLU' from the stored activation of the same row
+      if (row < p.Mdim) {
+        const __nv_bfloat16* z = p.Z + (int64_t)row * p.ldz + n_base;
+        if (n_base + 64 <= p.n_store) {
+          const uint4* z4 = reinterpret_cast<const uint4*>(z);
 #pragma unroll
-        for (int h = 0; h < 4; ++h) {
-          const __nv_bfloat162 pr = *reinterpret_cast<const __nv_bfloat162*>(&w[h]);
-          const int k = 8 * j + 2 * h;
-          v[k] = (__low2float(pr) > 0.f) ? u2f(r[k]) : 0.f;
-          v[k + 1] = (__high2float(pr) > 0.f) ? u2f(r[k + 1]) : 0.f;
+          for (int j = 0; j < 8; ++j) {
+            const uint4 zz = __ldg(z4 + j);
+            const uint32_t w[4] = {zz.x, zz.y, zz.z, zz.w};
+#pragma unroll
+            for (int h = 0; h < 4; ++h) {
+              const __nv_bfloat162 pr = *reinterpret_cast<const __nv_bfloat162*>(&w[h]);
+              const int k = 8 * j + 2 * h;
+              v[k] = (__low2float(pr) > 0.f) ? v[k] : 0.f;
+              v[k + 1] = (__high2float(pr) > 0.f) ? v[k + 1] : 0.f;
+            }
+          }
+        } else {
+#pragma unroll
+          for (int j = 0; j < 64; ++j) v[j] = (n_base + j < p.n_store && __bfloat162float(z[j]) > 0.f) ? v[j] : 0.f;
         }
       }
-    } else {
-#pragma unroll
-      for (int j = 0; j < 32; ++j)
-        v[j] = (n_base + j < p.n_store && __bfloat162float(z[j]) > 0.f) ? u2f(r[j]) : 0.f;
     }
-  } else {
 #pragma unroll
-    for (int j = 0; j < 32; ++j) v[j] = u2f(r[j]);
-  }
-
-  if (EPI == kTcEpiBiasReluBf16 || EPI == kTcEpiMaskBf16) {
-    __nv_bfloat16* d = reinterpret_cast<__nv_bfloat16*>(dbase) + (int64_t)row * p.ldd + n_base;
-    if (full) {
-      uint4* d4 = reinterpret_cast<uint4*>(d);
-#pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        uint4 o;
-        o.x = pack_bf16(v[8 * j + 0], v[8 * j + 1]);
-        o.y = pack_bf16(v[8 * j + 2], v[8 * j + 3]);
-        o.z = pack_bf16(v[8 * j + 4], v[8 * j + 5]);
-        o.w = pack_bf16(v[8 * j + 6], v[8 * j + 7]);
-        d4[j] = o;
-      }
-    } else {
-#pragma unroll
-      for (int j = 0; j < 32; ++j)
-        if (n_base + j < p.n_store) d[j] = __float2bfloat16_rn(v[j]);
-    }
-  } else {
-    float* d = reinterpret_cast<float*>(dbase) + (int64_t)row * p.ldd + n_base;
-    if (full) {
-      float4* d4 = reinterpret_cast<float4*>(d);
-#pragma unroll
-      for (int j = 0; j < 8; ++j) d4[j] = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
-    } else {
-#pragma unroll
-      for (int j = 0; j < 32; ++j)
-        if (n_base + j < p.n_store) d[j] = v[j];
-    }
+    for (int j = 0; j < 8; ++j)
+      o[j] = make_uint4(pack_bf16(v[8 * j], v[8 * j + 1]), pack_bf16(v[8 * j + 2], v[8 * j + 3]),
+                        pack_bf16(v[8 * j + 4], v[8 * j + 5]), pack_bf16(v[8 * j + 6], v[8 * j + 7]));
   }
 }
 
@@ -276,7 +294,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sA = smem;
   uint8_t* sB = smem + S * A_STAGE;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(sB + S * B_STAGE);
+  uint8_t* sStage = sB + S * B_STAGE;                 // epilogue staging, 1 KB aligned
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sStage + kTcStagingBytes);
   uint64_t* full_bar = bars;
   uint64_t* empty_bar = bars + S;
   uint64_t* tfull_bar = bars + 2 * S;
@@ -401,10 +420,18 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
     }
   } else {
     // -------------------------------------------------------------- epilogue (warps 2..5)
+    // Each warp owns 32 accumulator rows (its TMEM lane quadrant) and two 4 KB staging buffers.
+    // Per unit: tcgen05.ld -> fused math -> 16-byte stores into a 128-byte-swizzled 32 x 128 B
+    // box -> one TMA bulk store of the box (double-buffered: the store of one unit overlaps the
+    // math of the next).
+    constexpr bool kF32Out = (EPI == kTcEpiBiasF32 || EPI == kTcEpiStoreF32);
+    constexpr int kUnitCols = kF32Out ? 32 : 64;
+    constexpr int kUnits = BN / kUnitCols;
     const int q = warp & 3;   // the TMEM lane quadrant this warp may read
+    const uint32_t stage_base = smem_u32(sStage) + (uint32_t)((warp - 2) * 8192);
+    int sb = 0;
     int ab = 0;
     uint32_t aph = 0;
-    const size_t esize = (EPI == kTcEpiBiasF32 || EPI == kTcEpiStoreF32) ? 4 : 2;
     for (int t = blockIdx.x; t < total; t += gridDim.x) {
       const TileCoord c = decode_tile(t, p.tiles_m, p.tiles_n);
       int ok = 1;
@@ -419,24 +446,41 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
       }
       __syncwarp();
       tc_fence_after();
-      const int row = c.tm * BM + q * 32 + lane;
-      const bool row_ok = row < p.Mdim;
-      uint8_t* dbase = reinterpret_cast<uint8_t*>(p.D) + (size_t)c.g * (size_t)p.d_gstride * esize;
+      const int row0 = c.tm * BM + q * 32;
+      const int row = row0 + lane;
+      const CUtensorMap* td = &p.tmD[c.g];
       const uint32_t t_row = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(ab * BN);
 #pragma unroll 1
-      for (int ch = 0; ch < BN / 32; ++ch) {
-        const int n_base = c.tn * BN + ch * 32;
+      for (int u = 0; u < kUnits; ++u) {
+        const int n_base = c.tn * BN + u * kUnitCols;
         if (n_base >= p.n_store) break;
-        uint32_t r[32];
-        tmem_ld32(t_row + (uint32_t)(ch * 32), r);
+        uint32_t r[32], r2[32];
+        tmem_ld32(t_row + (uint32_t)(u * kUnitCols), r);
+        if (!kF32Out) tmem_ld32(t_row + (uint32_t)(u * kUnitCols + 32), r2);
         tmem_ld_wait(r);
-        if (row_ok) epilogue_chunk<EPI>(p, dbase, row, n_base, r);
+        if (!kF32Out) tmem_ld_wait(r2);
+        uint4 o[8];
+        epilogue_unit<EPI>(p, row, n_base, r, r2, o);
+        if (lane == 0) bulk_wait_read_1();   // the store that last used this buffer has read it
+        __syncwarp();
+        const uint32_t buf = stage_base + (uint32_t)(sb * 4096);
+        const uint32_t rbase = buf + (uint32_t)(lane * 128);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) st_shared_v4(rbase + (uint32_t)(((j ^ (lane & 7)) << 4)), o[j]);
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) {
+          tma_store_2d(td, buf, n_base, row0);
+          bulk_commit();
+        }
+        sb ^= 1;
       }
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(smem_u32(&tempty_bar[ab]));
       if (++ab == 2) { ab = 0; aph ^= 1u; }
     }
+    if (lane == 0) bulk_wait_all();
   }
 
   tc_fence_before();
@@ -486,7 +530,8 @@ bool tc_init_driver(const char** why) {
 }
 
 static bool encode_2d(CUtensorMap* tm, const void* base, uint64_t inner, uint64_t outer, uint64_t row_bytes,
-                      uint32_t box_inner, uint32_t box_outer, const char** why) {
+                      uint32_t box_inner, uint32_t box_outer, const char** why,
+                      CUtensorMapDataType dtype = CU_TENSOR_MAP_DATA_TYPE_BFLOAT16) {
   if (!g_encode && !tc_init_driver(why)) return false;
   if ((reinterpret_cast<uintptr_t>(base) & 15u) != 0 || (row_bytes & 15u) != 0) {
     *why = "TMA operand base or row stride is not 16-byte aligned";
@@ -496,7 +541,7 @@ static bool encode_2d(CUtensorMap* tm, const void* base, uint64_t inner, uint64_
   cuuint64_t strides[1] = {row_bytes};
   cuuint32_t box[2] = {box_inner, box_outer};
   cuuint32_t estr[2] = {1, 1};
-  CUresult r = g_encode(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+  CUresult r = g_encode(tm, dtype, 2, const_cast<void*>(base), dims, strides, box, estr,
                         CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                         CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (r != CUDA_SUCCESS) {
@@ -513,6 +558,13 @@ bool tc_make_kmajor_map(CUtensorMap* tm, const TcOperand& op, int box_rows, cons
 
 bool tc_make_mnmajor_map(CUtensorMap* tm, const TcOperand& op, const char** why) {
   return encode_2d(tm, op.base, (uint64_t)op.cols, (uint64_t)op.rows, (uint64_t)op.ld * 2, 64, BK, why);
+}
+
+bool tc_make_store_map(CUtensorMap* tm, void* base, bool fp32, int64_t rows, int64_t cols, int64_t ld,
+                       const char** why) {
+  const uint64_t es = fp32 ? 4 : 2;
+  return encode_2d(tm, base, (uint64_t)cols, (uint64_t)rows, (uint64_t)ld * es, (uint32_t)(128 / es), 32, why,
+                   fp32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16);
 }
 
 cudaError_t launch_tc_gemm(const TcGemmParams& p, int num_sms, cudaStream_t s) {

@@ -26,6 +26,7 @@ enum TcEpi : int32_t {
 struct TcGemmParams {
   CUtensorMap tmA[kTcMaxGroups];
   CUtensorMap tmB[kTcMaxGroups];
+  CUtensorMap tmD[kTcMaxGroups];   // output (store) maps: box of 32 rows x 128 bytes
   int32_t num_kb[kTcMaxGroups];
   int32_t groups;
   int32_t Mdim, Ndim, n_store;
@@ -53,9 +54,15 @@ bool tc_init_driver(const char** why);
 bool tc_make_kmajor_map(CUtensorMap* tm, const TcOperand& op, int box_rows, const char** why);
 // MN-major operand: matrix [K rows][MN] with MN contiguous; box = 64 (MN) x 64 (K).
 bool tc_make_mnmajor_map(CUtensorMap* tm, const TcOperand& op, const char** why);
+// Output matrix [rows][cols] (row stride ld elements, fp32 or bf16) for TMA stores of 32-row x
+// 128-byte boxes; rows >= `rows` and columns >= `cols` of a box are not written.
+bool tc_make_store_map(CUtensorMap* tm, void* base, bool fp32, int64_t rows, int64_t cols, int64_t ld,
+                       const char** why);
 
 constexpr int kTcBM = 128, kTcBN = 256, kTcBK = 64, kTcStages = 4;
-constexpr int kTcSmemBytes = kTcStages * (kTcBM + kTcBN) * kTcBK * 2 + 1024 /*align*/ + 256 /*barriers*/;
+constexpr int kTcStagingBytes = 4 * 2 * 32 * 128;   // 4 epilogue warps x 2 buffers x (32 rows x 128 B)
+constexpr int kTcSmemBytes =
+    kTcStages * (kTcBM + kTcBN) * kTcBK * 2 + kTcStagingBytes + 1024 /*align*/ + 256 /*barriers*/;
 
 // Launch on `num_sms` persistent CTAs (capped by the tile count).
 cudaError_t launch_tc_gemm(const TcGemmParams& p, int num_sms, cudaStream_t s);

@@ -207,6 +207,7 @@ hs_status build_tc_static(hs_ctx* c) {
     f.D = last ? static_cast<void*>(c->d_logits) : c->d_act[l + 1];
     f.ldd = last ? c->Cp : ly.out;
     f.st = c->d_status;
+    if (!hs::tc_make_store_map(&f.tmD[0], f.D, last, c->N, f.n_store, f.ldd, &why)) return fail(c, HS_ERR_CUDA, why);
     if (l == 0) continue;
     // input gradient of layer l: A = delta_l [N, out] (K-major), B = W_l [out, in] (MN-major)
     hs::TcGemmParams& d = c->tc_dgrad[l];
@@ -230,6 +231,7 @@ hs_status build_tc_static(hs_ctx* c) {
     d.Z = reinterpret_cast<const __nv_bfloat16*>(c->d_act[l]);
     d.ldz = ly.in;
     d.st = c->d_status;
+    if (!hs::tc_make_store_map(&d.tmD[0], d.D, false, c->N, d.n_store, d.ldd, &why)) return fail(c, HS_ERR_CUDA, why);
   }
   return HS_OK;
 }
@@ -255,7 +257,9 @@ hs_status build_tc_wgrad(hs_ctx* c) {
                         ldd_delta};
         // B: H_{l-1} rows of worker m as [n rows][in cols] (MN-major: in contiguous)
         hs::TcOperand b{reinterpret_cast<const __nv_bfloat16*>(c->d_act[l]) + off * ly.in, n, ly.in, ly.in};
-        if (!hs::tc_make_mnmajor_map(&w.tmA[g], a, &why) || !hs::tc_make_mnmajor_map(&w.tmB[g], b, &why))
+        float* dg = c->d_slabs + (int64_t)m * c->Ps + ly.w_off;
+        if (!hs::tc_make_mnmajor_map(&w.tmA[g], a, &why) || !hs::tc_make_mnmajor_map(&w.tmB[g], b, &why) ||
+            !hs::tc_make_store_map(&w.tmD[g], dg, true, out_cols, ly.in, ly.in, &why))
           return fail(c, HS_ERR_CUDA, why);
         w.num_kb[g] = (int32_t)((n + hs::kTcBK - 1) / hs::kTcBK);
       }
@@ -847,7 +851,9 @@ hs_status hs_debug_gemm_bf16(int32_t mode, int32_t M, int32_t N, int32_t K, cons
         const int64_t k0 = k_offsets_host[g0 + g], kn = k_offsets_host[g0 + g + 1] - k0;
         if (kn < 1) return fail(nullptr, HS_ERR_INVALID_ARG, "every group needs K >= 1");
         if (!hs::tc_make_mnmajor_map(&p.tmA[g], hs::TcOperand{pa + k0 * lda, kn, M, lda}, &why) ||
-            !hs::tc_make_mnmajor_map(&p.tmB[g], hs::TcOperand{pb + k0 * ldb, kn, N, ldb}, &why))
+            !hs::tc_make_mnmajor_map(&p.tmB[g], hs::TcOperand{pb + k0 * ldb, kn, N, ldb}, &why) ||
+            !hs::tc_make_store_map(&p.tmD[g], reinterpret_cast<float*>(D) + (int64_t)(g0 + g) * d_gstride, true, M,
+                                   N, ldd, &why))
           return fail(nullptr, HS_ERR_INVALID_ARG, why);
         p.num_kb[g] = (int)((kn + hs::kTcBK - 1) / hs::kTcBK);
       }
@@ -876,6 +882,8 @@ hs_status hs_debug_gemm_bf16(int32_t mode, int32_t M, int32_t N, int32_t K, cons
     p.bias = bias;
     p.Z = reinterpret_cast<const __nv_bfloat16*>(Z);
     p.ldz = ldz;
+    if (!hs::tc_make_store_map(&p.tmD[0], D, mode == HS_GEMM_FWD_LOGITS, M, N, ldd, &why))
+      return fail(nullptr, HS_ERR_INVALID_ARG, why);
   }
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   for (hs::TcGemmParams& p : plans) {
