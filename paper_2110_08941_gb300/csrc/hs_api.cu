@@ -10,137 +10,14 @@
 #include "../../include/hs_debug.h"
 #include "common.cuh"
 #include "gemm_tc.cuh"
+#include "ctx.cuh"
 
 using hs::DevStatus;
+using namespace hs;
 
 namespace {
 
 thread_local std::string g_init_error;
-
-struct Layer {
-  int in, out;
-  int64_t w_off, b_off;
-};
-
-int64_t round_up(int64_t v, int64_t m) { return (v + m - 1) / m * m; }
-
-}  // namespace
-
-struct hs_ctx {
-  int device = 0;
-  int num_sms = 0;
-  int arch = HS_MLP, precision = HS_BF16, sync = HS_SYNC_MEAN;
-  std::vector<int32_t> dims;
-  std::vector<Layer> layers;
-  int L = 0;
-  int M = 0, N = 0;
-  int64_t P = 0, Ps = 0;
-  int C = 0, Cp = 0, maxw = 0;
-
-  // partition state (host mirror + device copies)
-  std::vector<int32_t> counts, offsets;
-  std::vector<double> weights, cp_norm;
-  uint64_t version = 0;
-  int32_t* d_offsets = nullptr;
-  int32_t* d_index_map = nullptr;
-  float* d_scale = nullptr;
-  float* d_w = nullptr;
-  int4* d_bg_chunks = nullptr;       // bias-gradient row chunks (worker, begin, end, 0)
-  int32_t* d_bg_chunk_begin = nullptr;
-  int n_bg_chunks = 0;
-  float* d_bg_partial = nullptr;     // [max chunks, maxw] partial column sums
-
-  // workspace
-  std::vector<void*> d_act;        // H_0 .. H_{L-1}
-  float* d_logits = nullptr;       // [N, Cp]
-  void* d_delta[2] = {nullptr, nullptr};
-  float* d_ce = nullptr;
-  float* d_lm = nullptr;
-  DevStatus* d_status = nullptr;
-  DevStatus* h_status = nullptr;   // pinned
-  float* d_slabs = nullptr;        // [M, Ps]
-  __nv_bfloat16* d_shadow = nullptr;
-  float* d_gdebug = nullptr;
-  void* d_xstage = nullptr;
-  int32_t* d_ystage = nullptr;
-  const float* shadow_src = nullptr;
-  bool shadow_valid = false;
-  bool debug = false;
-  bool gdebug_valid = false;
-  std::string err;
-
-  // profiling: per-phase event pairs recorded on the step's stream, summed on read
-  bool profiling = false;
-  struct Rec { int phase; cudaEvent_t a, b; };
-  std::vector<Rec> pending;
-  std::vector<cudaEvent_t> event_pool;
-  int64_t launches[HS_PHASE_COUNT] = {0};
-
-  cudaEvent_t take_event() {
-    if (!event_pool.empty()) {
-      cudaEvent_t e = event_pool.back();
-      event_pool.pop_back();
-      return e;
-    }
-    cudaEvent_t e = nullptr;
-    if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
-    return e;
-  }
-
-  // tensor-core launch parameters (bf16 precision)
-  std::vector<hs::TcGemmParams> tc_fwd;                // per layer
-  std::vector<hs::TcGemmParams> tc_dgrad;              // per layer (index 0 unused)
-  std::vector<std::vector<hs::TcGemmParams>> tc_wgrad; // per layer, per chunk of <= 32 workers
-
-  size_t act_elem() const { return precision == HS_BF16 ? 2 : 4; }
-  int delta_ld(int l) const { return l == L - 1 ? Cp : layers[l].out; }     // l: 0-based layer
-  void* delta_buf(int l) const { return d_delta[(L - 1 - l) & 1]; }
-};
-
-namespace {
-
-// Brackets one phase of the step with CUDA events when profiling is on.
-class PhaseScope {
- public:
-  PhaseScope(hs_ctx* c, int phase, cudaStream_t s) : c_(c), phase_(phase), s_(s) {
-    if (c_->profiling) {
-      a_ = c_->take_event();
-      if (a_) cudaEventRecord(a_, s_);
-    }
-  }
-  ~PhaseScope() {
-    if (c_->profiling && a_) {
-      cudaEvent_t b = c_->take_event();
-      if (b) {
-        cudaEventRecord(b, s_);
-        c_->pending.push_back({phase_, a_, b});
-      }
-    }
-  }
-  void launched(int n = 1) { c_->launches[phase_] += n; }
-
- private:
-  hs_ctx* c_;
-  int phase_;
-  cudaStream_t s_;
-  cudaEvent_t a_ = nullptr;
-};
-
-hs_status fail(hs_ctx* c, hs_status s, const std::string& msg) {
-  if (c) c->err = msg; else g_init_error = msg;
-  return s;
-}
-
-hs_status cuda_fail(hs_ctx* c, cudaError_t e, const char* what) {
-  return fail(c, e == cudaErrorMemoryAllocation ? HS_ERR_OOM : HS_ERR_CUDA,
-              std::string(what) + ": " + cudaGetErrorString(e));
-}
-
-#define HS_CUDA(ctx, call)                                   \
-  do {                                                       \
-    cudaError_t e_ = (call);                                 \
-    if (e_ != cudaSuccess) return cuda_fail(ctx, e_, #call); \
-  } while (0)
 
 hs_status validate_model(const hs_model_desc* m, std::vector<int32_t>* dims, std::string* why) {
   if (!m || !m->dims) { *why = "model or model->dims is NULL"; return HS_ERR_INVALID_ARG; }
@@ -346,14 +223,6 @@ void fill_partition_view(const hs_ctx* c, hs_partition_t* out) {
   out->version = c->version;
 }
 
-template <typename T>
-hs_status dalloc(hs_ctx* c, T** p, size_t bytes) {
-  *p = nullptr;
-  if (bytes == 0) bytes = 16;
-  cudaError_t e = cudaMalloc(reinterpret_cast<void**>(p), bytes);
-  if (e != cudaSuccess) return cuda_fail(c, e, "cudaMalloc");
-  return HS_OK;
-}
 
 void free_all(hs_ctx* c) {
   auto f = [](void* p) { if (p) cudaFree(p); };
