@@ -107,11 +107,23 @@ class ClockSampler:
 
 # ------------------------------------------------------------------------------ workload math
 def gemm_flops(wl):
-    dims = wl.dims
-    sw = sum(dims[l] * dims[l - 1] for l in range(1, len(dims)))
-    sw_dgrad = sum(dims[l] * dims[l - 1] for l in range(2, len(dims)))
+    """Algorithmic flops of the step's products (forward, per-worker weight gradient, input gradient)."""
     n = wl.global_batch
-    return dict(forward=2.0 * n * sw, wgrad=2.0 * n * sw, dgrad=2.0 * n * sw_dgrad)
+    if wl.arch == synth.MLP:
+        dims = wl.dims
+        sw = sum(dims[l] * dims[l - 1] for l in range(1, len(dims)))
+        sw_dgrad = sum(dims[l] * dims[l - 1] for l in range(2, len(dims)))
+        return dict(forward=2.0 * n * sw, wgrad=2.0 * n * sw, dgrad=2.0 * n * sw_dgrad)
+    cin, h, w, c1, c2, c3, classes = wl.dims
+    per = []                       # (rows per sample x Cout x Cin*9) of each conv
+    prev = cin
+    for c, s in zip((c1, c2, c3), (1, 2, 2)):
+        h, w = (h + 2 - 3) // s + 1, (w + 2 - 3) // s + 1
+        per.append(h * w * c * prev * 9)
+        prev = c
+    fc = classes * c3
+    return dict(forward=2.0 * n * (sum(per) + fc), wgrad=2.0 * n * (sum(per) + fc),
+                dgrad=2.0 * n * (per[1] + per[2] + fc))
 
 
 def update_bytes(wl, P):
@@ -124,9 +136,10 @@ def oracle_sample(wl, seconds_target=12.0, max_workers=None):
     """Time the oracle (as it stands) on whole worker segments of the workload: the smallest
     workers first, adding workers until about `seconds_target` of CPU time.  Returns
     (samples/s, description, cores)."""
-    from oracle import mlp, sgd
+    from oracle import cnn, mlp, sgd
     from oracle import partition as P
 
+    fn = mlp.worker_loss_grad if wl.arch == synth.MLP else cnn.worker_loss_grad
     try:
         from threadpoolctl import threadpool_info
         threads = max([i.get("num_threads", 1) for i in threadpool_info()] or [1])
@@ -143,7 +156,7 @@ def oracle_sample(wl, seconds_target=12.0, max_workers=None):
     for m in order:
         xs, ys = x[off[m]:off[m + 1]], y[off[m]:off[m + 1]]
         t0 = time.perf_counter()
-        sgd.step(mlp.worker_loss_grad, theta, wl.dims, xs, ys, [sizes[m]], wl.lr, sgd.SYNC_CP_WEIGHTED)
+        sgd.step(fn, theta, wl.dims, xs, ys, [sizes[m]], wl.lr, sgd.SYNC_CP_WEIGHTED)
         elapsed += time.perf_counter() - t0
         done_samples += sizes[m]
         used.append(m)
@@ -158,8 +171,9 @@ def oracle_sample(wl, seconds_target=12.0, max_workers=None):
 def run_reference(args, wl, rank, world):
     if rank != 0:
         return
-    from oracle import mlp, sgd
+    from oracle import cnn, mlp, sgd
     from oracle import partition as P
+    fn = mlp.worker_loss_grad if wl.arch == synth.MLP else cnn.worker_loss_grad
     try:
         from threadpoolctl import threadpool_info
         cores = max([i.get("num_threads", 1) for i in threadpool_info()] or [1])
@@ -174,8 +188,7 @@ def run_reference(args, wl, rank, world):
 
     def one():
         nonlocal theta
-        theta, _, _, _, _ = sgd.step(mlp.worker_loss_grad, theta, wl.dims, xs, ys, [sizes[m]], wl.lr,
-                                     sgd.SYNC_CP_WEIGHTED)
+        theta, _, _, _, _ = sgd.step(fn, theta, wl.dims, xs, ys, [sizes[m]], wl.lr, sgd.SYNC_CP_WEIGHTED)
 
     for _ in range(args.warmup):
         one()
@@ -301,7 +314,8 @@ def run_ours(args, wl, rank, world, local_rank):
             "vs_baseline": None, "dtype": "bf16" if precision == hs.HS_BF16 else "f32", "data": "synthetic",
             "config": {"workload": wl.name, "global_batch": wl.global_batch, "workers": wl.workers,
                        "dims": list(wl.dims), "sync": "cp_weighted", "parallelism": f"replicas{world}",
-                       "l2": "working set > L2 (7 GB slabs, 0.9 GB activations per step), no flush"},
+                       "l2": ("working set > L2 (7 GB slabs, 0.9 GB activations per step), no flush"
+                              if wl.name == DEFAULT_WORKLOAD else "small workload: working set may sit in L2")},
             "roofline": roofline,
             "roofline_gemm_phase": {"bound": "tensor", "achieved": gemm_total / (gemm_ms * 1e-3) / 1e12,
                                     "peak": peaks["bf16_sust"], "unit": "TFLOP/s",

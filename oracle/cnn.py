@@ -16,6 +16,11 @@ the sum; the backward pass is the same sum read the other way (weight gradient
 = patches^T dOut, input gradient = scatter-add of dOut W back to the padded
 input).  Parameters: flat [conv1.W, conv1.b, conv2.W, conv2.b, conv3.W,
 conv3.b, fc.W, fc.b], conv weights [Cout, Cin, 3, 3], fc.W [classes, C3].
+
+`decide` (optional) is the same device as in oracle.mlp: an operand rounding from which
+the ReLU' masks are taken (the forward evaluated with rounded input, weights and stored
+activations, exact accumulation), so that a bf16 kernel and the oracle take those 0/1
+decisions in the same precision; every value stays fp64.
 """
 from __future__ import annotations
 
@@ -108,6 +113,18 @@ def forward(theta: np.ndarray, dims: Sequence[int], x: np.ndarray):
     return z, dict(pre=pre, ins=ins, cols=cols, last=h, pooled=pooled, parts=parts)
 
 
+def relu_decisions(theta: np.ndarray, dims: Sequence[int], x: np.ndarray, rnd):
+    """1[A_k > 0] for each convolution, with A_k evaluated from operands rounded by `rnd`."""
+    parts = unpack(np.asarray(theta, dtype=np.float64), dims)
+    h = rnd(x)
+    masks = []
+    for k, s in enumerate(STRIDES):
+        a, _ = conv_forward(h, rnd(parts[2 * k]), parts[2 * k + 1], s)
+        masks.append(a > 0.0)
+        h = rnd(np.maximum(a, 0.0))
+    return masks
+
+
 def _ce(z: np.ndarray, y: np.ndarray):
     zmax = z.max(axis=1, keepdims=True)
     e = np.exp(z - zmax)
@@ -117,11 +134,16 @@ def _ce(z: np.ndarray, y: np.ndarray):
 
 
 def worker_loss_grad(theta: np.ndarray, dims: Sequence[int], x_m: np.ndarray,
-                     y_m: np.ndarray) -> Tuple[float, np.ndarray]:
+                     y_m: np.ndarray, decide=None) -> Tuple[float, np.ndarray]:
+    """L_m and g^m (flat fp64 [P]) on one worker's segment (Eq. 1); decide as in the module doc."""
     theta = np.asarray(theta, dtype=np.float64)
     n_m = x_m.shape[0]
     y_m = np.asarray(y_m, dtype=np.int64)
     z, c = forward(theta, dims, x_m)
+    if decide is None:
+        masks = [a > 0.0 for a in c["pre"]]
+    else:
+        masks = relu_decisions(theta, dims, x_m, decide)
     ce, prob = _ce(z, y_m)
     loss = float(ce.sum() / n_m)
     dz = prob.copy()
@@ -137,7 +159,7 @@ def worker_loss_grad(theta: np.ndarray, dims: Sequence[int], x_m: np.ndarray,
     dh = np.broadcast_to(dpool[:, :, None, None] / area, last.shape)
     for k in range(len(STRIDES) - 1, -1, -1):
         s = STRIDES[k]
-        da = dh * (c["pre"][k] > 0.0)
+        da = dh * masks[k]
         w = parts[2 * k]
         cout = w.shape[0]
         n, _, ho, wo = da.shape

@@ -1,0 +1,489 @@
+// The CNN workload (stand-in for the paper's ResNet50 / VGG16 on CIFAR10, Section 5): three 3x3
+// convolutions with padding 1 (strides 1, 2, 2, ReLU), global average pooling, one fully
+// connected layer.  Every convolution runs as a product over explicit patch rows (im2col) on
+// the same GEMM kernels as the MLP: forward (bias + ReLU fused), input gradient (a product into
+// patch space, then a gather back to the input grid with ReLU' fused), and the per-worker
+// weight gradient G_m[W] = dA[seg_m]^T patches[seg_m] (Eq. 1's per-worker gradient), whose K =
+// n_m * Ho * Wo is split into chunks so that the few output tiles still fill the GPU; the chunk
+// partials are added per worker in a fixed order.  Activations are NHWC (channels last).
+#include <algorithm>
+#include <cstring>
+
+#include "ctx.cuh"
+
+namespace hs {
+
+namespace {
+
+template <typename T>
+__device__ __forceinline__ float to_f(T v);
+template <>
+__device__ __forceinline__ float to_f<float>(float v) { return v; }
+template <>
+__device__ __forceinline__ float to_f<__nv_bfloat16>(__nv_bfloat16 v) { return __bfloat162float(v); }
+template <typename T>
+__device__ __forceinline__ T from_f(float v);
+template <>
+__device__ __forceinline__ float from_f<float>(float v) { return v; }
+template <>
+__device__ __forceinline__ __nv_bfloat16 from_f<__nv_bfloat16>(float v) { return __float2bfloat16_rn(v); }
+
+// Patch rows of the first convolution from the NCHW fp32 input: col[r][ci*9 + kh*3 + kw] =
+// x_pad[n][ci][s*ho + kh][s*wo + kw], r = (n*Ho + ho)*Wo + wo; columns K..Kp-1 are zero.
+template <typename T>
+__global__ void im2col_nchw_kernel(const float* __restrict__ x, int N, int C, int H, int W, int Ho, int Wo, int s,
+                                   T* __restrict__ col, int Kp) {
+  const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const int64_t rows = (int64_t)N * Ho * Wo;
+  if (idx >= rows * C) return;
+  const int ci = (int)(idx % C);
+  const int64_t r = idx / C;
+  const int wo = (int)(r % Wo);
+  const int ho = (int)((r / Wo) % Ho);
+  const int n = (int)(r / ((int64_t)Wo * Ho));
+  T* dst = col + r * Kp + ci * 9;
+  const float* src = x + ((int64_t)n * C + ci) * H * W;
+#pragma unroll
+  for (int kh = 0; kh < 3; ++kh) {
+    const int hi = s * ho + kh - 1;
+#pragma unroll
+    for (int kw = 0; kw < 3; ++kw) {
+      const int wi = s * wo + kw - 1;
+      const float v = (hi >= 0 && hi < H && wi >= 0 && wi < W) ? src[(int64_t)hi * W + wi] : 0.f;
+      dst[kh * 3 + kw] = from_f<T>(v);
+    }
+  }
+  if (ci == 0)
+    for (int k = C * 9; k < Kp; ++k) col[r * Kp + k] = from_f<T>(0.f);
+}
+
+// Patch rows from an NHWC activation h[n][hi][wi][ci] (same column order as above).
+template <typename T>
+__global__ void im2col_nhwc_kernel(const T* __restrict__ h, int N, int C, int H, int W, int Ho, int Wo, int s,
+                                   T* __restrict__ col, int Kp) {
+  const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const int64_t rows = (int64_t)N * Ho * Wo;
+  if (idx >= rows * C) return;
+  const int ci = (int)(idx % C);
+  const int64_t r = idx / C;
+  const int wo = (int)(r % Wo);
+  const int ho = (int)((r / Wo) % Ho);
+  const int n = (int)(r / ((int64_t)Wo * Ho));
+  T* dst = col + r * Kp + ci * 9;
+#pragma unroll
+  for (int kh = 0; kh < 3; ++kh) {
+    const int hi = s * ho + kh - 1;
+#pragma unroll
+    for (int kw = 0; kw < 3; ++kw) {
+      const int wi = s * wo + kw - 1;
+      dst[kh * 3 + kw] = (hi >= 0 && hi < H && wi >= 0 && wi < W)
+                             ? h[(((int64_t)n * H + hi) * W + wi) * C + ci]
+                             : from_f<T>(0.f);
+    }
+  }
+}
+
+// pooled[n][c] = mean over the HW rows of sample n (global average pooling).
+template <typename T>
+__global__ void gap_forward_kernel(const T* __restrict__ h, int N, int HW, int C, T* __restrict__ pooled) {
+  const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= (int64_t)N * C) return;
+  const int c = (int)(idx % C);
+  const int64_t n = idx / C;
+  float acc = 0.f;
+  for (int p = 0; p < HW; ++p) acc += to_f<T>(h[(n * HW + p) * C + c]);
+  pooled[idx] = from_f<T>(acc / (float)HW);
+}
+
+// dA[n][p][c] = dpooled[n][c] / HW * 1[h[n][p][c] > 0] (pooling backward with ReLU').
+template <typename T>
+__global__ void gap_backward_kernel(const float* __restrict__ dpooled, const T* __restrict__ h, int N, int HW, int C,
+                                    T* __restrict__ dA) {
+  const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= (int64_t)N * HW * C) return;
+  const int c = (int)(idx % C);
+  const int64_t n = idx / ((int64_t)HW * C);
+  const float g = dpooled[n * C + c] / (float)HW;
+  dA[idx] = from_f<T>(to_f<T>(h[idx]) > 0.f ? g : 0.f);
+}
+
+// Input gradient on the input grid: the adjoint of im2col (each input element sums the patch
+// entries that read it), then ReLU' of that input: dA[n][hi][wi][ci].
+template <typename T>
+__global__ void col2im_nhwc_kernel(const float* __restrict__ dcol, int ldc, const T* __restrict__ h, int N, int C,
+                                   int H, int W, int Ho, int Wo, int s, T* __restrict__ dA) {
+  const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= (int64_t)N * H * W * C) return;
+  const int ci = (int)(idx % C);
+  const int wi = (int)((idx / C) % W);
+  const int hi = (int)((idx / ((int64_t)C * W)) % H);
+  const int n = (int)(idx / ((int64_t)C * W * H));
+  float acc = 0.f;
+#pragma unroll
+  for (int kh = 0; kh < 3; ++kh) {
+    const int th = hi + 1 - kh;
+    if (th < 0 || th % s) continue;
+    const int ho = th / s;
+    if (ho >= Ho) continue;
+#pragma unroll
+    for (int kw = 0; kw < 3; ++kw) {
+      const int tw = wi + 1 - kw;
+      if (tw < 0 || tw % s) continue;
+      const int wo = tw / s;
+      if (wo >= Wo) continue;
+      acc += dcol[(((int64_t)n * Ho + ho) * Wo + wo) * ldc + ci * 9 + kh * 3 + kw];
+    }
+  }
+  dA[idx] = from_f<T>(to_f<T>(h[idx]) > 0.f ? acc : 0.f);
+}
+
+// bf16 copy of the first convolution's weights with rows padded from K to Kp (16-byte rows).
+__global__ void pad_weights_kernel(const float* __restrict__ w, int rows, int K, int Kp, __nv_bfloat16* __restrict__ wp) {
+  const int idx = blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= rows * Kp) return;
+  const int k = idx % Kp, r = idx / Kp;
+  wp[idx] = __float2bfloat16_rn(k < K ? w[(int64_t)r * K + k] : 0.f);
+}
+
+// slabs[m][w_off + co*K + k] = sum over worker m's chunks (in order) of partial[chunk][co][k].
+__global__ void splitk_reduce_kernel(const float* __restrict__ partial, int rows, int K, int ldp,
+                                     const int32_t* __restrict__ chunk_begin, float* __restrict__ slabs, int64_t Ps,
+                                     int64_t w_off) {
+  const int m = blockIdx.y;
+  const int idx = blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= rows * K) return;
+  const int k = idx % K, co = idx / K;
+  float acc = 0.f;
+  for (int c = chunk_begin[m]; c < chunk_begin[m + 1]; ++c) acc += partial[((int64_t)c * rows + co) * ldp + k];
+  slabs[(int64_t)m * Ps + w_off + idx] = acc;
+}
+
+inline int blocks_for(int64_t n, int threads) { return (int)((n + threads - 1) / threads); }
+
+}  // namespace
+
+// ---------------------------------------------------------------------------------- plans
+// Weight-gradient plan for one layer: groups = (worker, K chunk); both operands MN-major
+// [rows][cols]; chunk partial g lands at partial + g * rows_out * ldp.
+hs_status cnn_build_wgrad_plan(hs_ctx* c, int layer, const __nv_bfloat16* a, int a_cols, int64_t lda,
+                               const __nv_bfloat16* b, int b_cols, int64_t ldb, int64_t rows_per_sample) {
+  const char* why = nullptr;
+  CnnWgrad& wg = c->cnn_wgrad[layer];
+  wg.plans.clear();
+  wg.rows_out = a_cols;
+  wg.K = b_cols;
+  wg.ldp = (int)round_up(b_cols, 4);
+  const int tiles = (int)(((a_cols + kTcBM - 1) / kTcBM) * ((b_cols + kTcBN - 1) / kTcBN));
+  const int64_t total_rows = (int64_t)c->N * rows_per_sample;
+  const int64_t target_groups = std::max<int64_t>(1, (2LL * c->num_sms + tiles - 1) / tiles);
+  const int64_t chunk = std::max<int64_t>(512, round_up((total_rows + target_groups - 1) / target_groups, kTcBK));
+  std::vector<std::pair<int64_t, int64_t>> ranges;
+  std::vector<int32_t> begin;
+  for (int m = 0; m < c->M; ++m) {
+    begin.push_back((int32_t)ranges.size());
+    const int64_t r0 = (int64_t)c->offsets[m] * rows_per_sample, r1 = (int64_t)c->offsets[m + 1] * rows_per_sample;
+    for (int64_t r = r0; r < r1; r += chunk) ranges.push_back({r, std::min(chunk, r1 - r)});
+  }
+  begin.push_back((int32_t)ranges.size());
+  const int G = (int)ranges.size();
+  if ((int64_t)G * wg.rows_out * wg.ldp > wg.partial_capacity) return fail(c, HS_ERR_OOM, "split-K partial buffer too small");
+  for (int g0 = 0; g0 < G; g0 += kTcMaxGroups) {
+    const int ng = std::min(kTcMaxGroups, G - g0);
+    wg.plans.emplace_back();
+    TcGemmParams& p = wg.plans.back();
+    std::memset(&p, 0, sizeof(p));
+    for (int g = 0; g < ng; ++g) {
+      const auto& rg = ranges[g0 + g];
+      float* dg = wg.d_partial + (int64_t)(g0 + g) * wg.rows_out * wg.ldp;
+      if (!tc_make_mnmajor_map(&p.tmA[g], TcOperand{a + rg.first * lda, rg.second, a_cols, lda}, &why) ||
+          !tc_make_mnmajor_map(&p.tmB[g], TcOperand{b + rg.first * ldb, rg.second, b_cols, ldb}, &why) ||
+          !tc_make_store_map(&p.tmD[g], dg, true, a_cols, b_cols, wg.ldp, &why))
+        return fail(c, HS_ERR_CUDA, why);
+      p.num_kb[g] = (int32_t)((rg.second + kTcBK - 1) / kTcBK);
+    }
+    p.groups = ng;
+    p.Mdim = a_cols;
+    p.Ndim = b_cols;
+    p.n_store = b_cols;
+    p.tiles_m = (a_cols + kTcBM - 1) / kTcBM;
+    p.tiles_n = (b_cols + kTcBN - 1) / kTcBN;
+    p.epi = kTcEpiStoreF32;
+    p.a_mn = 1;
+    p.b_mn = 1;
+    p.D = wg.d_partial + (int64_t)g0 * wg.rows_out * wg.ldp;
+    p.ldd = wg.ldp;
+    p.d_gstride = (int64_t)wg.rows_out * wg.ldp;
+    p.st = c->d_status;
+  }
+  cudaError_t e = cudaMemcpy(wg.d_chunk_begin, begin.data(), sizeof(int32_t) * begin.size(), cudaMemcpyHostToDevice);
+  if (e != cudaSuccess) return cuda_fail(c, e, "split-K chunk table");
+  return HS_OK;
+}
+
+namespace {
+
+hs_status plan_dense(hs_ctx* c, TcGemmParams* p, int epi, const __nv_bfloat16* a, int64_t a_rows, int a_cols,
+                     int64_t lda, const __nv_bfloat16* b, int64_t b_rows, int b_cols, int64_t ldb, bool b_mn,
+                     void* d, bool d_f32, int Mdim, int Ndim, int n_store, int64_t ldd, const __nv_bfloat16* z,
+                     int64_t ldz) {
+  const char* why = nullptr;
+  std::memset(p, 0, sizeof(*p));
+  bool ok = tc_make_kmajor_map(&p->tmA[0], TcOperand{a, a_rows, a_cols, lda}, kTcBM, &why);
+  ok = ok && (b_mn ? tc_make_mnmajor_map(&p->tmB[0], TcOperand{b, b_rows, b_cols, ldb}, &why)
+                   : tc_make_kmajor_map(&p->tmB[0], TcOperand{b, b_rows, b_cols, ldb}, kTcBN, &why));
+  ok = ok && tc_make_store_map(&p->tmD[0], d, d_f32, Mdim, n_store, ldd, &why);
+  if (!ok) return fail(c, HS_ERR_CUDA, why);
+  const int K = b_mn ? (int)b_rows : b_cols;
+  p->num_kb[0] = (K + kTcBK - 1) / kTcBK;
+  p->groups = 1;
+  p->Mdim = Mdim;
+  p->Ndim = Ndim;
+  p->n_store = n_store;
+  p->tiles_m = (Mdim + kTcBM - 1) / kTcBM;
+  p->tiles_n = (n_store + kTcBN - 1) / kTcBN;
+  p->epi = epi;
+  p->a_mn = 0;
+  p->b_mn = b_mn ? 1 : 0;
+  p->D = d;
+  p->ldd = ldd;
+  p->Z = z;
+  p->ldz = ldz;
+  p->st = c->d_status;
+  return HS_OK;
+}
+
+}  // namespace
+
+hs_status cnn_build_static(hs_ctx* c) {
+  const char* why = nullptr;
+  if (!tc_init_driver(&why)) return fail(c, HS_ERR_CUDA, why);
+  const int N = c->N;
+  auto bf = [](void* p) { return reinterpret_cast<const __nv_bfloat16*>(p); };
+  c->tc_fwd.assign(4, TcGemmParams{});
+  c->tc_dgrad.assign(4, TcGemmParams{});
+  for (int k = 0; k < 3; ++k) {
+    const ConvLayer& L = c->convs[k];
+    const __nv_bfloat16* wb = (k == 0) ? c->d_w1p : c->d_shadow + L.w_off;
+    const int64_t ldw = (k == 0) ? L.Kp : L.K;
+    hs_status st = plan_dense(c, &c->tc_fwd[k], kTcEpiBiasReluBf16, bf(c->d_col[k]), L.rows, L.K, L.Kp, wb, L.cout,
+                              L.K, ldw, false, c->d_cact[k], false, (int)L.rows, L.cout, L.cout, L.cout, nullptr, 0);
+    if (st != HS_OK) return st;
+  }
+  // fully connected layer on the pooled features
+  const int c3 = c->convs[2].cout;
+  hs_status st = plan_dense(c, &c->tc_fwd[3], kTcEpiBiasF32, bf(c->d_pooled), N, c3, c3, c->d_shadow + c->fc_w_off,
+                            c->C, c3, c3, false, c->d_logits, true, N, c->C, c->Cp, c->Cp, nullptr, 0);
+  if (st != HS_OK) return st;
+  // input gradients: fc -> pooled features (fp32), conv3 / conv2 -> patch space (fp32)
+  st = plan_dense(c, &c->tc_dgrad[3], kTcEpiStoreF32, bf(c->d_delta[0]), N, c->C, c->Cp, c->d_shadow + c->fc_w_off,
+                  c->C, c3, c3, true, c->d_dpooled, true, N, c3, c3, c3, nullptr, 0);
+  if (st != HS_OK) return st;
+  for (int k = 2; k >= 1; --k) {
+    const ConvLayer& L = c->convs[k];
+    st = plan_dense(c, &c->tc_dgrad[k], kTcEpiStoreF32, bf(c->d_dA[k]), L.rows, L.cout, L.cout,
+                    c->d_shadow + L.w_off, L.cout, L.K, L.K, true, c->d_dcol, true, (int)L.rows, L.K, L.K, L.K,
+                    nullptr, 0);
+    if (st != HS_OK) return st;
+  }
+  return HS_OK;
+}
+
+hs_status cnn_build_partition_plans(hs_ctx* c) {
+  auto bf = [](void* p) { return reinterpret_cast<const __nv_bfloat16*>(p); };
+  // fc: A^T = delta [N][C] (ld Cp), B = pooled [N][c3]
+  const int c3 = c->convs[2].cout;
+  hs_status st = cnn_build_wgrad_plan(c, 3, bf(c->d_delta[0]), c->C, c->Cp, bf(c->d_pooled), c3, c3, 1);
+  for (int k = 2; k >= 0 && st == HS_OK; --k) {
+    const ConvLayer& L = c->convs[k];
+    st = cnn_build_wgrad_plan(c, k, bf(c->d_dA[k]), L.cout, L.cout, bf(c->d_col[k]), L.K, L.Kp,
+                              (int64_t)L.hout * L.wout);
+  }
+  return st;
+}
+
+// ---------------------------------------------------------------------------------- the step
+hs_status cnn_step(hs_ctx* c, float* params, const float* x, const int32_t* y, cudaStream_t s) {
+  const bool bf16 = (c->precision == HS_BF16);
+  const int N = c->N, T = 256;
+  const ConvLayer* L = c->convs.data();
+  const int c3 = L[2].cout;
+  const int hw3 = L[2].hout * L[2].wout;
+  {
+    PhaseScope ph(c, HS_PHASE_CAST, s);
+    if (bf16) {
+      pad_weights_kernel<<<blocks_for((int64_t)L[0].cout * L[0].Kp, T), T, 0, s>>>(params + L[0].w_off, L[0].cout, L[0].K,
+                                                                                   L[0].Kp, c->d_w1p);
+      ph.launched();
+    }
+  }
+  {
+    PhaseScope ph(c, HS_PHASE_FORWARD, s);
+    for (int k = 0; k < 3; ++k) {
+      const int64_t n_items = L[k].rows * L[k].cin;
+      if (k == 0) {
+        if (bf16)
+          im2col_nchw_kernel<__nv_bfloat16><<<blocks_for(n_items, T), T, 0, s>>>(
+              x, N, L[0].cin, L[0].hin, L[0].win, L[0].hout, L[0].wout, L[0].stride,
+              reinterpret_cast<__nv_bfloat16*>(c->d_col[0]), L[0].Kp);
+        else
+          im2col_nchw_kernel<float><<<blocks_for(n_items, T), T, 0, s>>>(
+              x, N, L[0].cin, L[0].hin, L[0].win, L[0].hout, L[0].wout, L[0].stride,
+              reinterpret_cast<float*>(c->d_col[0]), L[0].Kp);
+      } else {
+        if (bf16)
+          im2col_nhwc_kernel<__nv_bfloat16><<<blocks_for(n_items, T), T, 0, s>>>(
+              reinterpret_cast<const __nv_bfloat16*>(c->d_cact[k - 1]), N, L[k].cin, L[k].hin, L[k].win, L[k].hout,
+              L[k].wout, L[k].stride, reinterpret_cast<__nv_bfloat16*>(c->d_col[k]), L[k].Kp);
+        else
+          im2col_nhwc_kernel<float><<<blocks_for(n_items, T), T, 0, s>>>(
+              reinterpret_cast<const float*>(c->d_cact[k - 1]), N, L[k].cin, L[k].hin, L[k].win, L[k].hout,
+              L[k].wout, L[k].stride, reinterpret_cast<float*>(c->d_col[k]), L[k].Kp);
+      }
+      ph.launched();
+      if (bf16) {
+        TcGemmParams& f = c->tc_fwd[k];
+        f.bias = params + L[k].b_off;
+        cudaError_t e = launch_tc_gemm(f, c->num_sms, s);
+        if (e != cudaSuccess) return cuda_fail(c, e, "conv forward GEMM launch");
+      } else {
+        GemmF32Args g{};
+        g.A = reinterpret_cast<const float*>(c->d_col[k]); g.a_sm = L[k].Kp; g.a_sk = 1;
+        g.B = params + L[k].w_off; g.b_sk = 1; g.b_sn = L[k].K;
+        g.C = reinterpret_cast<float*>(c->d_cact[k]); g.ldc = L[k].cout;
+        g.Mdim = (int)L[k].rows; g.Ndim = L[k].cout; g.Kdim = L[k].K;
+        g.epi = kEpiBiasRelu; g.bias = params + L[k].b_off;
+        launch_gemm_f32(g, s);
+      }
+      ph.launched();
+    }
+    if (bf16)
+      gap_forward_kernel<__nv_bfloat16><<<blocks_for((int64_t)N * c3, T), T, 0, s>>>(
+          reinterpret_cast<const __nv_bfloat16*>(c->d_cact[2]), N, hw3, c3, reinterpret_cast<__nv_bfloat16*>(c->d_pooled));
+    else
+      gap_forward_kernel<float><<<blocks_for((int64_t)N * c3, T), T, 0, s>>>(
+          reinterpret_cast<const float*>(c->d_cact[2]), N, hw3, c3, reinterpret_cast<float*>(c->d_pooled));
+    ph.launched();
+    if (bf16) {
+      TcGemmParams& f = c->tc_fwd[3];
+      f.bias = params + c->fc_b_off;
+      cudaError_t e = launch_tc_gemm(f, c->num_sms, s);
+      if (e != cudaSuccess) return cuda_fail(c, e, "fc forward GEMM launch");
+    } else {
+      GemmF32Args g{};
+      g.A = reinterpret_cast<const float*>(c->d_pooled); g.a_sm = c3; g.a_sk = 1;
+      g.B = params + c->fc_w_off; g.b_sk = 1; g.b_sn = c3;
+      g.C = c->d_logits; g.ldc = c->Cp;
+      g.Mdim = N; g.Ndim = c->C; g.Kdim = c3;
+      g.epi = kEpiBias; g.bias = params + c->fc_b_off;
+      launch_gemm_f32(g, s);
+    }
+    ph.launched();
+  }
+  {
+    PhaseScope ph(c, HS_PHASE_LOSS, s);
+    launch_softmax_xent(c->d_logits, c->Cp, y, c->d_scale, N, c->C, c->d_delta[0], c->Cp, bf16, c->d_ce, c->d_status,
+                        s);
+    launch_loss_reduce(c->d_ce, c->d_offsets, c->M, c->d_w, c->d_lm, c->d_status, s);
+    ph.launched(2);
+  }
+  // ---- backward: layer index 3 = fc, 2..0 = conv3..conv1
+  for (int k = 3; k >= 0; --k) {
+    const bool fc = (k == 3);
+    const int width = fc ? c->C : L[k].cout;
+    void* delta = fc ? c->d_delta[0] : c->d_dA[k];
+    const int ld_delta = fc ? c->Cp : L[k].cout;
+    const int64_t w_off = fc ? c->fc_w_off : L[k].w_off;
+    const int64_t b_off = fc ? c->fc_b_off : L[k].b_off;
+    {
+      PhaseScope ph(c, HS_PHASE_WGRAD, s);
+      if (bf16) {
+        CnnWgrad& wg = c->cnn_wgrad[k];
+        for (const TcGemmParams& p : wg.plans) {
+          cudaError_t e = launch_tc_gemm(p, c->num_sms, s);
+          if (e != cudaSuccess) return cuda_fail(c, e, "conv weight-gradient GEMM launch");
+          ph.launched();
+        }
+        dim3 grid(blocks_for((int64_t)wg.rows_out * wg.K, T), c->M);
+        splitk_reduce_kernel<<<grid, T, 0, s>>>(wg.d_partial, wg.rows_out, wg.K, wg.ldp, wg.d_chunk_begin, c->d_slabs,
+                                                c->Ps, w_off);
+        ph.launched();
+      } else {
+        GemmF32Args w{};
+        w.A = reinterpret_cast<const float*>(delta); w.a_sm = 1; w.a_sk = ld_delta;
+        if (fc) {
+          w.B = reinterpret_cast<const float*>(c->d_pooled); w.b_sk = c3; w.b_sn = 1; w.Ndim = c3;
+        } else {
+          w.B = reinterpret_cast<const float*>(c->d_col[k]); w.b_sk = L[k].Kp; w.b_sn = 1; w.Ndim = L[k].K;
+        }
+        w.C = c->d_slabs + w_off; w.ldc = w.Ndim;
+        w.Mdim = width; w.Kdim = 0;
+        w.epi = kEpiStore;
+        w.k_offsets = c->d_row_off[k]; w.groups = c->M; w.c_gstride = c->Ps;
+        launch_gemm_f32(w, s);
+        ph.launched();
+      }
+    }
+    {
+      PhaseScope ph(c, HS_PHASE_BIASGRAD, s);
+      if (bf16) {
+        const ChunkTable& ct = c->cnn_chunks[k];
+        launch_bias_grad_bf16(reinterpret_cast<const __nv_bfloat16*>(delta), ld_delta, width, ct.d_chunks, ct.n,
+                              ct.d_begin, c->M, c->d_bg_partial, c->d_slabs, c->Ps, b_off, s);
+        ph.launched(2);
+      } else {
+        launch_bias_grad(delta, false, ld_delta, width, c->d_row_off[k], c->M, c->d_slabs, c->Ps, b_off, s);
+        ph.launched();
+      }
+    }
+    if (k == 0) break;
+    PhaseScope ph(c, HS_PHASE_DGRAD, s);
+    if (fc) {
+      // dpooled = delta W_fc, then pooling backward with ReLU' into conv3's output gradient
+      if (bf16) {
+        cudaError_t e = launch_tc_gemm(c->tc_dgrad[3], c->num_sms, s);
+        if (e != cudaSuccess) return cuda_fail(c, e, "fc input-gradient GEMM launch");
+      } else {
+        GemmF32Args d{};
+        d.A = reinterpret_cast<const float*>(c->d_delta[0]); d.a_sm = c->Cp; d.a_sk = 1;
+        d.B = params + c->fc_w_off; d.b_sk = c3; d.b_sn = 1;
+        d.C = c->d_dpooled; d.ldc = c3;
+        d.Mdim = N; d.Ndim = c3; d.Kdim = c->C; d.epi = kEpiStore;
+        launch_gemm_f32(d, s);
+      }
+      if (bf16)
+        gap_backward_kernel<__nv_bfloat16><<<blocks_for((int64_t)N * hw3 * c3, T), T, 0, s>>>(
+            c->d_dpooled, reinterpret_cast<const __nv_bfloat16*>(c->d_cact[2]), N, hw3, c3,
+            reinterpret_cast<__nv_bfloat16*>(c->d_dA[2]));
+      else
+        gap_backward_kernel<float><<<blocks_for((int64_t)N * hw3 * c3, T), T, 0, s>>>(
+            c->d_dpooled, reinterpret_cast<const float*>(c->d_cact[2]), N, hw3, c3, reinterpret_cast<float*>(c->d_dA[2]));
+      ph.launched(2);
+    } else {
+      // dcol = dA_k W_k (patch space, fp32), then gather back to layer k's input grid with ReLU'
+      if (bf16) {
+        cudaError_t e = launch_tc_gemm(c->tc_dgrad[k], c->num_sms, s);
+        if (e != cudaSuccess) return cuda_fail(c, e, "conv input-gradient GEMM launch");
+      } else {
+        GemmF32Args d{};
+        d.A = reinterpret_cast<const float*>(c->d_dA[k]); d.a_sm = L[k].cout; d.a_sk = 1;
+        d.B = params + L[k].w_off; d.b_sk = L[k].K; d.b_sn = 1;
+        d.C = c->d_dcol; d.ldc = L[k].K;
+        d.Mdim = (int)L[k].rows; d.Ndim = L[k].K; d.Kdim = L[k].cout; d.epi = kEpiStore;
+        launch_gemm_f32(d, s);
+      }
+      const int64_t n_in = (int64_t)N * L[k].hin * L[k].win * L[k].cin;
+      if (bf16)
+        col2im_nhwc_kernel<__nv_bfloat16><<<blocks_for(n_in, T), T, 0, s>>>(
+            c->d_dcol, L[k].K, reinterpret_cast<const __nv_bfloat16*>(c->d_cact[k - 1]), N, L[k].cin, L[k].hin,
+            L[k].win, L[k].hout, L[k].wout, L[k].stride, reinterpret_cast<__nv_bfloat16*>(c->d_dA[k - 1]));
+      else
+        col2im_nhwc_kernel<float><<<blocks_for(n_in, T), T, 0, s>>>(
+            c->d_dcol, L[k].K, reinterpret_cast<const float*>(c->d_cact[k - 1]), N, L[k].cin, L[k].hin, L[k].win,
+            L[k].hout, L[k].wout, L[k].stride, reinterpret_cast<float*>(c->d_dA[k - 1]));
+      ph.launched(2);
+    }
+  }
+  return HS_OK;
+}
+
+}  // namespace hs

@@ -33,6 +33,15 @@ struct ChunkTable {
   int rows_per_sample = 1;
 };
 
+// Split-K weight-gradient plan of one CNN layer (groups = (worker, row chunk)).
+struct CnnWgrad {
+  std::vector<TcGemmParams> plans;
+  int rows_out = 0, K = 0, ldp = 0;
+  float* d_partial = nullptr;        // [groups][rows_out][ldp]
+  int64_t partial_capacity = 0;      // floats
+  int32_t* d_chunk_begin = nullptr;  // [M + 1]
+};
+
 }  // namespace hs
 
 struct hs_ctx {
@@ -96,6 +105,21 @@ struct hs_ctx {
     return e;
   }
 
+  // CNN workload: convs[0..2], then the fully connected layer (index 3 in per-layer arrays)
+  int64_t in_features = 0;
+  std::vector<hs::ConvLayer> convs;
+  int64_t fc_w_off = 0, fc_b_off = 0;
+  void* d_col[3] = {nullptr, nullptr, nullptr};
+  void* d_cact[3] = {nullptr, nullptr, nullptr};
+  void* d_pooled = nullptr;
+  float* d_dpooled = nullptr;
+  void* d_dA[3] = {nullptr, nullptr, nullptr};
+  float* d_dcol = nullptr;
+  __nv_bfloat16* d_w1p = nullptr;
+  int32_t* d_row_off[4] = {nullptr, nullptr, nullptr, nullptr};
+  hs::ChunkTable cnn_chunks[4];
+  hs::CnnWgrad cnn_wgrad[4];
+
   // tensor-core launch parameters (bf16 precision)
   std::vector<hs::TcGemmParams> tc_fwd;                // per layer
   std::vector<hs::TcGemmParams> tc_dgrad;              // per layer (index 0 unused)
@@ -158,5 +182,10 @@ inline hs_status dalloc(hs_ctx* c, T** p, size_t bytes) {
   if (e != cudaSuccess) return cuda_fail(c, e, "cudaMalloc");
   return HS_OK;
 }
+
+// CNN workload (csrc/cnn.cu)
+hs_status cnn_build_static(hs_ctx* c);
+hs_status cnn_build_partition_plans(hs_ctx* c);
+hs_status cnn_step(hs_ctx* c, float* params, const float* x, const int32_t* y, cudaStream_t s);
 
 }  // namespace hs

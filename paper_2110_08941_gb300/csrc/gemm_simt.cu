@@ -26,12 +26,16 @@ __global__ void __launch_bounds__(256) gemm_f32_kernel(GemmF32Args a) {
   }
   const bool a_kmajor = (a.a_sk == 1);
   const bool b_kmajor = (a.b_sk == 1);
-  float acc[4][4];
+  // Two-level fp32 sum: `acc` collects 16 k-tiles (256 products), then folds into `tot`, so the
+  // rounding error grows with sqrt(256) + sqrt(K / 256) instead of sqrt(K) for long K (the
+  // per-worker weight gradients of the convolutions sum over n_m * Ho * Wo rows).
+  float acc[4][4], tot[4][4];
 #pragma unroll
   for (int i = 0; i < 4; ++i)
 #pragma unroll
-    for (int j = 0; j < 4; ++j) acc[i][j] = 0.f;
+    for (int j = 0; j < 4; ++j) acc[i][j] = tot[i][j] = 0.f;
 
+  int tiles_done = 0;
   for (int k0 = kbeg; k0 < kend; k0 += BK) {
 #pragma unroll
     for (int r = 0; r < 4; ++r) {
@@ -59,7 +63,21 @@ __global__ void __launch_bounds__(256) gemm_f32_kernel(GemmF32Args a) {
         for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(ar[i], br[j], acc[i][j]);
     }
     __syncthreads();
+    if (++tiles_done == 16) {
+      tiles_done = 0;
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          tot[i][j] += acc[i][j];
+          acc[i][j] = 0.f;
+        }
+    }
   }
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+#pragma unroll
+    for (int j = 0; j < 4; ++j) acc[i][j] += tot[i][j];
 #pragma unroll
   for (int i = 0; i < 4; ++i) {
     const int gm = m0 + ty * 4 + i;

@@ -576,6 +576,7 @@ cudaError_t launch_tc_gemm(const TcGemmParams& p, int num_sms, cudaStream_t s) {
   if (p.epi == kTcEpiMaskBf16 && !p.a_mn && p.b_mn) return launch_variant<kTcEpiMaskBf16, false, true>(p, grid, s);
   if (p.epi == kTcEpiStoreF32 && p.a_mn && p.b_mn) return launch_variant<kTcEpiStoreF32, true, true>(p, grid, s);
   if (p.epi == kTcEpiStoreF32 && !p.a_mn && !p.b_mn) return launch_variant<kTcEpiStoreF32, false, false>(p, grid, s);
+  if (p.epi == kTcEpiStoreF32 && !p.a_mn && p.b_mn) return launch_variant<kTcEpiStoreF32, false, true>(p, grid, s);
   return cudaErrorInvalidValue;
 }
 

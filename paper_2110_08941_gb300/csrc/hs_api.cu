@@ -208,6 +208,32 @@ hs_status apply_partition(hs_ctx* c, const std::vector<int32_t>& sizes, const st
     hs_status st = build_tc_wgrad(c);
     if (st != HS_OK) return st;
   }
+  if (changed && c->arch == HS_CNN) {
+    // per-layer row offsets (a sample is Ho*Wo rows of a conv product, one row of the fc product)
+    const int R = hs::bias_grad_chunk_rows();
+    for (int k = 0; k < 4; ++k) {
+      const int64_t rps = c->cnn_chunks[k].rows_per_sample;
+      std::vector<int32_t> ro(c->M + 1), begin;
+      std::vector<int4> chunks;
+      for (int m = 0; m <= c->M; ++m) ro[m] = (int32_t)(c->offsets[m] * rps);
+      for (int m = 0; m < c->M; ++m) {
+        begin.push_back((int32_t)chunks.size());
+        for (int64_t r = ro[m]; r < ro[m + 1]; r += R)
+          chunks.push_back(make_int4(m, (int)r, (int)std::min<int64_t>(r + R, ro[m + 1]), 0));
+      }
+      begin.push_back((int32_t)chunks.size());
+      c->cnn_chunks[k].n = (int)chunks.size();
+      HS_CUDA(c, cudaMemcpy(c->d_row_off[k], ro.data(), sizeof(int32_t) * ro.size(), cudaMemcpyHostToDevice));
+      HS_CUDA(c, cudaMemcpy(c->cnn_chunks[k].d_chunks, chunks.data(), sizeof(int4) * chunks.size(),
+                            cudaMemcpyHostToDevice));
+      HS_CUDA(c, cudaMemcpy(c->cnn_chunks[k].d_begin, begin.data(), sizeof(int32_t) * begin.size(),
+                            cudaMemcpyHostToDevice));
+    }
+    if (c->precision == HS_BF16) {
+      hs_status st = cnn_build_partition_plans(c);
+      if (st != HS_OK) return st;
+    }
+  }
   return HS_OK;
 }
 
@@ -228,6 +254,12 @@ void free_all(hs_ctx* c) {
   auto f = [](void* p) { if (p) cudaFree(p); };
   f(c->d_offsets); f(c->d_index_map); f(c->d_scale); f(c->d_w);
   f(c->d_bg_chunks); f(c->d_bg_chunk_begin); f(c->d_bg_partial);
+  for (int k = 0; k < 3; ++k) { f(c->d_col[k]); f(c->d_cact[k]); f(c->d_dA[k]); }
+  f(c->d_pooled); f(c->d_dpooled); f(c->d_dcol); f(c->d_w1p);
+  for (int k = 0; k < 4; ++k) {
+    f(c->d_row_off[k]); f(c->cnn_chunks[k].d_chunks); f(c->cnn_chunks[k].d_begin);
+    f(c->cnn_wgrad[k].d_partial); f(c->cnn_wgrad[k].d_chunk_begin);
+  }
   for (void* p : c->d_act) f(p);
   f(c->d_logits); f(c->d_delta[0]); f(c->d_delta[1]); f(c->d_ce); f(c->d_lm); f(c->d_status);
   f(c->d_slabs); f(c->d_shadow); f(c->d_gdebug); f(c->d_xstage); f(c->d_ystage);
@@ -412,7 +444,6 @@ hs_status hs_init(const hs_model_desc* model, int32_t M, const double* compute_w
   if (st != HS_OK) return fail(nullptr, st, why);
   if (M < 1 || M > hs::kMaxWorkers) return fail(nullptr, HS_ERR_INVALID_ARG, "M must be in [1, 1024]");
   if (global_batch < M) return fail(nullptr, HS_ERR_INVALID_ARG, "global_batch must be >= M");
-  if (model->arch == HS_CNN) return fail(nullptr, HS_ERR_UNSUPPORTED, "CNN workloads are not built yet");
 
   std::vector<double> cp(M, 1.0);
   if (compute_weights) cp.assign(compute_weights, compute_weights + M);
@@ -440,29 +471,72 @@ hs_status hs_init(const hs_model_desc* model, int32_t M, const double* compute_w
   c->dims = dims;
   c->M = M;
   c->N = global_batch;
-  c->L = model->n_layers;
-  if (c->precision == HS_BF16) {
-    for (int l = 0; l < c->L; ++l)
-      if (dims[l] % 8 != 0) {
-        delete c;
-        return fail(nullptr, HS_ERR_UNSUPPORTED, "bf16 precision needs input and hidden widths divisible by 8");
-      }
+  c->L = model->arch == HS_MLP ? model->n_layers : 0;
+  const bool bf16 = (c->precision == HS_BF16);
+  if (c->arch == HS_MLP) {
+    if (bf16) {
+      for (int l = 0; l < c->L; ++l)
+        if (dims[l] % 8 != 0) {
+          delete c;
+          return fail(nullptr, HS_ERR_UNSUPPORTED, "bf16 precision needs input and hidden widths divisible by 8");
+        }
+    }
+    int64_t off = 0;
+    for (int l = 0; l < c->L; ++l) {
+      Layer ly{dims[l], dims[l + 1], 0, 0};
+      ly.w_off = off;
+      off += (int64_t)ly.in * ly.out;
+      ly.b_off = off;
+      off += ly.out;
+      c->layers.push_back(ly);
+    }
+    c->P = off;
+    c->C = dims[c->L];
+    c->Cp = (int)round_up(c->C, 8);
+    c->maxw = c->Cp;
+    for (int l = 1; l < c->L; ++l) c->maxw = std::max(c->maxw, dims[l]);
+    c->in_features = dims[0];
+  } else {
+    // Cin, H, W, c1, c2, c3, classes: 3x3 convs (padding 1, strides 1, 2, 2), pooling, fc
+    if (bf16 && (dims[3] % 8 || dims[4] % 8 || dims[5] % 8)) {
+      delete c;
+      return fail(nullptr, HS_ERR_UNSUPPORTED, "bf16 precision needs conv widths divisible by 8");
+    }
+    const int strides[3] = {1, 2, 2};
+    int64_t off = 0;
+    int h = dims[1], w = dims[2], prev = dims[0];
+    for (int k = 0; k < 3; ++k) {
+      ConvLayer L{};
+      L.cin = prev;
+      L.cout = dims[3 + k];
+      L.hin = h;
+      L.win = w;
+      L.stride = strides[k];
+      L.hout = (h + 2 - 3) / L.stride + 1;
+      L.wout = (w + 2 - 3) / L.stride + 1;
+      L.K = prev * 9;
+      L.Kp = bf16 ? (int)round_up(L.K, 8) : L.K;
+      L.w_off = off;
+      off += (int64_t)L.cout * L.K;
+      L.b_off = off;
+      off += L.cout;
+      L.rows = (int64_t)global_batch * L.hout * L.wout;
+      c->convs.push_back(L);
+      h = L.hout;
+      w = L.wout;
+      prev = L.cout;
+    }
+    c->fc_w_off = off;
+    off += (int64_t)dims[6] * prev;
+    c->fc_b_off = off;
+    off += dims[6];
+    c->P = off;
+    c->C = dims[6];
+    c->Cp = (int)round_up(c->C, 8);
+    c->maxw = std::max(c->Cp, std::max(dims[3], std::max(dims[4], dims[5])));
+    c->in_features = (int64_t)dims[0] * dims[1] * dims[2];
   }
-  int64_t off = 0;
-  for (int l = 0; l < c->L; ++l) {
-    Layer ly{dims[l], dims[l + 1], 0, 0};
-    ly.w_off = off;
-    off += (int64_t)ly.in * ly.out;
-    ly.b_off = off;
-    off += ly.out;
-    c->layers.push_back(ly);
-  }
-  c->P = off;
   c->Ps = round_up(c->P, 64);
-  c->C = dims[c->L];
-  c->Cp = (int)round_up(c->C, 8);
-  c->maxw = c->Cp;
-  for (int l = 1; l < c->L; ++l) c->maxw = std::max(c->maxw, dims[l]);
 
   const size_t N = (size_t)c->N;
   const size_t es = c->act_elem();
@@ -472,18 +546,59 @@ hs_status hs_init(const hs_model_desc* model, int32_t M, const double* compute_w
   chk(dalloc(c, &c->d_index_map, sizeof(int32_t) * N));
   chk(dalloc(c, &c->d_scale, sizeof(float) * N));
   chk(dalloc(c, &c->d_w, sizeof(float) * M));
-  const int max_chunks = c->N / hs::bias_grad_chunk_rows() + M + 1;
+  const int R = hs::bias_grad_chunk_rows();
+  const int max_chunks = c->N / R + M + 1;
   chk(dalloc(c, &c->d_bg_chunks, sizeof(int4) * max_chunks));
   chk(dalloc(c, &c->d_bg_chunk_begin, sizeof(int32_t) * (M + 1)));
-  chk(dalloc(c, &c->d_bg_partial, sizeof(float) * (size_t)max_chunks * (size_t)c->maxw));
-  c->d_act.assign(c->L, nullptr);
-  for (int l = 0; l < c->L; ++l) {
-    if (l == 0 && c->precision == HS_FP32_CHECK) continue;   // fp32 reads x in place
-    chk(dalloc(c, &c->d_act[l], es * N * (size_t)dims[l]));
+  size_t delta_elems = N * (size_t)c->maxw;
+  size_t bg_partial = (size_t)max_chunks * (size_t)c->maxw;
+  if (c->arch == HS_MLP) {
+    c->d_act.assign(c->L, nullptr);
+    for (int l = 0; l < c->L; ++l) {
+      if (l == 0 && !bf16) continue;   // fp32 reads x in place
+      chk(dalloc(c, &c->d_act[l], es * N * (size_t)dims[l]));
+    }
+  } else {
+    const int c3 = c->convs[2].cout;
+    int64_t dcol = 0;
+    for (int k = 0; k < 3; ++k) {
+      const ConvLayer& L = c->convs[k];
+      chk(dalloc(c, &c->d_col[k], es * (size_t)L.rows * L.Kp));
+      chk(dalloc(c, &c->d_cact[k], es * (size_t)L.rows * L.cout));
+      chk(dalloc(c, &c->d_dA[k], es * (size_t)L.rows * L.cout));
+      if (k > 0) dcol = std::max<int64_t>(dcol, L.rows * L.K);
+    }
+    chk(dalloc(c, &c->d_pooled, es * N * c3));
+    chk(dalloc(c, &c->d_dpooled, sizeof(float) * N * c3));
+    chk(dalloc(c, &c->d_dcol, sizeof(float) * (size_t)dcol));
+    if (bf16) chk(dalloc(c, &c->d_w1p, sizeof(__nv_bfloat16) * (size_t)c->convs[0].cout * c->convs[0].Kp));
+    delta_elems = N * (size_t)c->Cp;
+    for (int k = 0; k < 4; ++k) {
+      const bool fc = (k == 3);
+      const int64_t rps = fc ? 1 : (int64_t)c->convs[k].hout * c->convs[k].wout;
+      const int width = fc ? c->C : c->convs[k].cout;
+      const int64_t chunks = (int64_t)c->N * rps / R + M + 1;
+      chk(dalloc(c, &c->d_row_off[k], sizeof(int32_t) * (M + 1)));
+      chk(dalloc(c, &c->cnn_chunks[k].d_chunks, sizeof(int4) * (size_t)chunks));
+      chk(dalloc(c, &c->cnn_chunks[k].d_begin, sizeof(int32_t) * (M + 1)));
+      c->cnn_chunks[k].rows_per_sample = (int)rps;
+      bg_partial = std::max(bg_partial, (size_t)chunks * (size_t)width);
+      if (bf16) {
+        CnnWgrad& wg = c->cnn_wgrad[k];
+        const int rows_out = width;
+        const int kcols = fc ? c3 : c->convs[k].K;
+        const int tiles = ((rows_out + kTcBM - 1) / kTcBM) * ((kcols + kTcBN - 1) / kTcBN);
+        const int64_t target = std::max<int64_t>(1, (2LL * c->num_sms + tiles - 1) / tiles);
+        wg.partial_capacity = (target + M + 1) * rows_out * round_up(kcols, 4);
+        chk(dalloc(c, &wg.d_partial, sizeof(float) * (size_t)wg.partial_capacity));
+        chk(dalloc(c, &wg.d_chunk_begin, sizeof(int32_t) * (M + 1)));
+      }
+    }
   }
+  chk(dalloc(c, &c->d_bg_partial, sizeof(float) * bg_partial));
   chk(dalloc(c, &c->d_logits, sizeof(float) * N * c->Cp));
-  chk(dalloc(c, &c->d_delta[0], es * N * c->maxw));
-  chk(dalloc(c, &c->d_delta[1], es * N * c->maxw));
+  chk(dalloc(c, &c->d_delta[0], es * delta_elems));
+  chk(dalloc(c, &c->d_delta[1], es * (c->arch == HS_MLP ? delta_elems : 8)));
   chk(dalloc(c, &c->d_ce, sizeof(float) * N));
   chk(dalloc(c, &c->d_lm, sizeof(float) * M));
   chk(dalloc(c, &c->d_status, sizeof(DevStatus)));
@@ -497,11 +612,11 @@ hs_status hs_init(const hs_model_desc* model, int32_t M, const double* compute_w
     e = cudaMemset(c->d_status, 0, sizeof(DevStatus));
     if (e == cudaSuccess) e = cudaMemset(c->d_slabs, 0, sizeof(float) * (size_t)M * (size_t)c->Ps);
     if (e == cudaSuccess && c->d_shadow) e = cudaMemset(c->d_shadow, 0, sizeof(__nv_bfloat16) * (size_t)c->Ps);
-    if (e == cudaSuccess) e = cudaMemset(c->d_delta[0], 0, es * N * c->maxw);
-    if (e == cudaSuccess) e = cudaMemset(c->d_delta[1], 0, es * N * c->maxw);
+    if (e == cudaSuccess) e = cudaMemset(c->d_delta[0], 0, es * delta_elems);
+    if (e == cudaSuccess && c->arch == HS_MLP) e = cudaMemset(c->d_delta[1], 0, es * delta_elems);
     if (e != cudaSuccess) s2 = cuda_fail(c, e, "cudaMemset");
   }
-  if (s2 == HS_OK && c->precision == HS_BF16) s2 = build_tc_static(c);
+  if (s2 == HS_OK && bf16) s2 = c->arch == HS_MLP ? build_tc_static(c) : cnn_build_static(c);
   if (s2 == HS_OK) s2 = apply_partition(c, sizes, cpn, nullptr, 0);
   if (s2 == HS_OK) {
     e = cudaDeviceSynchronize();
@@ -561,7 +676,7 @@ hs_status hs_step(hs_ctx* c, float* params, const void* x, const int32_t* y, con
     return fail(c, HS_ERR_INVALID_ARG, "partition does not match the context's current partition");
   if (!is_device_ptr(params)) return fail(c, HS_ERR_INVALID_ARG, "params must be a device pointer");
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  const size_t in_feat = (size_t)c->layers[0].in;
+  const size_t in_feat = (size_t)c->in_features;
   const float* xd = reinterpret_cast<const float*>(x);
   const int32_t* yd = y;
   if (!is_device_ptr(x)) {
@@ -589,7 +704,9 @@ hs_status hs_step(hs_ctx* c, float* params, const void* x, const int32_t* y, con
     hs_status r = dalloc(c, &c->d_gdebug, sizeof(float) * c->Ps);
     if (r != HS_OK) return r;
   }
-  hs_status st = c->precision == HS_BF16 ? mlp_step_bf16(c, params, xd, yd, s) : mlp_step_fp32(c, params, xd, yd, s);
+  hs_status st = c->arch == HS_CNN            ? cnn_step(c, params, xd, yd, s)
+                 : c->precision == HS_BF16 ? mlp_step_bf16(c, params, xd, yd, s)
+                                           : mlp_step_fp32(c, params, xd, yd, s);
   if (st != HS_OK) return st;
   {
     PhaseScope ph(c, HS_PHASE_UPDATE, s);

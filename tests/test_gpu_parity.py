@@ -162,3 +162,39 @@ def test_bf16_against_exact_decisions(name):
     orc = run_oracle(wl.arch, wl.dims, wl.workers, wl.global_batch, w, x, y, theta0, wl.lr, 1,
                      hs.HS_SYNC_CP_WEIGHTED)
     assert rel(lib["g_first"], orc["g_first"]) <= 6e-2
+
+
+# ------------------------------------------------------------------------------------------ CNN
+@pytest.mark.parametrize("precision,steps", [(hs.HS_BF16, 10), (hs.HS_FP32_CHECK, 3)])
+def test_cnn_workload(precision, steps):
+    """CNN 3x32x32 -> conv64 -> conv128/2 -> conv256/2 -> pool -> fc10, N = 512, M = 4 (1:2:3:6)."""
+    wl, x, y, theta0, w = _inputs(synth.CFG4)
+    lib = run_library(wl.arch, wl.dims, wl.workers, wl.global_batch, w, x, y, theta0, wl.lr, steps, precision,
+                      hs.HS_SYNC_CP_WEIGHTED, keep_slabs=True)
+    orc = run_oracle(wl.arch, wl.dims, wl.workers, wl.global_batch, w, x, y, theta0, wl.lr, steps,
+                     hs.HS_SYNC_CP_WEIGHTED, keep_slabs=True, decide=decide_for(precision))
+    assert lib["counts"][0] == [43, 85, 128, 256]
+    _check(lib, orc, theta0.astype(np.float64), precision, steps)
+    for m in range(wl.workers):
+        assert rel(lib["slabs_first"][m], orc["slabs_first"][m]) <= TOL_G[precision], m
+
+
+CNN_EDGE = [
+    # Cin, H, W, c1, c2, c3, classes; N; M; weights (odd spatial sizes, one sample per worker)
+    ((3, 9, 7, 8, 16, 24, 5), 7, 3, [1.0, 2.0, 4.0]),
+    ((2, 6, 6, 16, 8, 8, 3), 4, 4, None),
+    ((3, 16, 16, 32, 32, 64, 10), 33, 2, [1.0, 5.0]),
+]
+
+
+@pytest.mark.parametrize("precision", [hs.HS_BF16, hs.HS_FP32_CHECK])
+@pytest.mark.parametrize("dims,N,M,weights", CNN_EDGE)
+def test_cnn_edge_shapes(dims, N, M, weights, precision):
+    rng = np.random.default_rng(N + dims[1])
+    x = rng.standard_normal((N,) + tuple(dims[:3]), dtype=np.float32)
+    y = rng.integers(0, dims[-1], N, dtype=np.int32)
+    theta0 = synth.he_normal_params(synth.CNN, dims, 5)
+    for sync in (hs.HS_SYNC_MEAN, hs.HS_SYNC_CP_WEIGHTED):
+        lib = run_library(synth.CNN, dims, M, N, weights, x, y, theta0, 0.05, 10, precision, sync)
+        orc = run_oracle(synth.CNN, dims, M, N, weights, x, y, theta0, 0.05, 10, sync, decide=decide_for(precision))
+        _check(lib, orc, theta0.astype(np.float64), precision, 10)

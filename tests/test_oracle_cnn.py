@@ -85,3 +85,26 @@ def test_cp_weighted_is_full_batch():
     sizes = P.partition_sizes([1, 2, 3, 6], 12)
     _, _, g, _, _ = sgd.step(cnn.worker_loss_grad, theta, TINY, x, y, sizes, 0.0, sgd.SYNC_CP_WEIGHTED)
     assert np.linalg.norm(g - g_full) <= 1e-12 * np.linalg.norm(g_full)
+
+
+def test_decision_mode_identity_is_exact():
+    theta, x, y = _tiny(TINY, 4, 5)
+    l0, g0 = cnn.worker_loss_grad(theta, TINY, x, y)
+    l1, g1 = cnn.worker_loss_grad(theta, TINY, x, y, decide=lambda a: np.asarray(a, dtype=np.float64))
+    assert l0 == l1 and np.array_equal(g0, g1)
+
+
+def test_bf16_decisions_differ_only_near_kinks():
+    from oracle import mlp
+    dims = (3, 16, 16, 16, 24, 32, 10)
+    theta, x, y = _tiny(dims, 6, 8)
+    theta *= 0.5
+    _, c = cnn.forward(theta, dims, x)
+    masks = cnn.relu_decisions(theta, dims, x, mlp.round_bf16)
+    flips = 0
+    for a, m in zip(c["pre"], masks):
+        diff = (a > 0) != m
+        flips += int(diff.sum())
+        if diff.any():
+            assert np.abs(a[diff]).max() < 0.05 * np.abs(a).std()
+    assert flips < 0.01 * sum(a.size for a in c["pre"])
