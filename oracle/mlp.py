@@ -86,6 +86,11 @@ def round_bf16(a) -> np.ndarray:
     return r.astype(np.uint32).view(np.float32).astype(np.float64)
 
 
+def round_fp32(a) -> np.ndarray:
+    """Round to the nearest fp32 value (the storage precision of the fp32 check path)."""
+    return np.asarray(a, dtype=np.float32).astype(np.float64)
+
+
 def relu_decisions(theta: np.ndarray, dims: Sequence[int], x: np.ndarray, rnd) -> List[np.ndarray]:
     """1[A_l > 0] for each hidden layer, with A_l evaluated from operands rounded by `rnd`."""
     ws, bs = unpack(np.asarray(theta, dtype=np.float64), dims)

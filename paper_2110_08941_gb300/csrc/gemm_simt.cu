@@ -10,6 +10,9 @@ namespace {
 
 constexpr int BM = 64, BN = 64, BK = 16;
 
+// Acc = double for the forward products: the ReLU' decisions taken from their results then match
+// an exact evaluation on the same fp32 operands; float (two-level) for the backward products.
+template <typename Acc>
 __global__ void __launch_bounds__(256) gemm_f32_kernel(GemmF32Args a) {
   __shared__ float As[BK][BM + 4];
   __shared__ float Bs[BK][BN + 4];
@@ -29,7 +32,7 @@ __global__ void __launch_bounds__(256) gemm_f32_kernel(GemmF32Args a) {
   // Two-level fp32 sum: `acc` collects 16 k-tiles (256 products), then folds into `tot`, so the
   // rounding error grows with sqrt(256) + sqrt(K / 256) instead of sqrt(K) for long K (the
   // per-worker weight gradients of the convolutions sum over n_m * Ho * Wo rows).
-  float acc[4][4], tot[4][4];
+  Acc acc[4][4], tot[4][4];
 #pragma unroll
   for (int i = 0; i < 4; ++i)
 #pragma unroll
@@ -60,7 +63,7 @@ __global__ void __launch_bounds__(256) gemm_f32_kernel(GemmF32Args a) {
 #pragma unroll
       for (int i = 0; i < 4; ++i)
 #pragma unroll
-        for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(ar[i], br[j], acc[i][j]);
+        for (int j = 0; j < 4; ++j) acc[i][j] = fma((Acc)ar[i], (Acc)br[j], acc[i][j]);
     }
     __syncthreads();
     if (++tiles_done == 16) {
@@ -86,14 +89,14 @@ __global__ void __launch_bounds__(256) gemm_f32_kernel(GemmF32Args a) {
     for (int j = 0; j < 4; ++j) {
       const int gn = n0 + tx * 4 + j;
       if (gn >= a.Ndim) continue;
-      float v = acc[i][j];
+      Acc v = acc[i][j];
       switch (a.epi) {
-        case kEpiBias: v += a.bias[gn]; break;
-        case kEpiBiasRelu: v = fmaxf(v + a.bias[gn], 0.f); break;
-        case kEpiMask: v = (a.Z[(int64_t)gm * a.ldz + gn] > 0.f) ? v : 0.f; break;
+        case kEpiBias: v += (Acc)a.bias[gn]; break;
+        case kEpiBiasRelu: v = v + (Acc)a.bias[gn] > (Acc)0 ? v + (Acc)a.bias[gn] : (Acc)0; break;
+        case kEpiMask: v = (a.Z[(int64_t)gm * a.ldz + gn] > 0.f) ? v : (Acc)0; break;
         default: break;
       }
-      C[(int64_t)gm * a.ldc + gn] = v;
+      C[(int64_t)gm * a.ldc + gn] = (float)v;
     }
   }
 }
@@ -103,7 +106,10 @@ __global__ void __launch_bounds__(256) gemm_f32_kernel(GemmF32Args a) {
 void launch_gemm_f32(const GemmF32Args& a, cudaStream_t s) {
   if (a.Mdim <= 0 || a.Ndim <= 0) return;
   dim3 grid((a.Ndim + BN - 1) / BN, (a.Mdim + BM - 1) / BM, a.k_offsets ? a.groups : 1);
-  gemm_f32_kernel<<<grid, 256, 0, s>>>(a);
+  if (a.epi == kEpiBias || a.epi == kEpiBiasRelu)
+    gemm_f32_kernel<double><<<grid, 256, 0, s>>>(a);
+  else
+    gemm_f32_kernel<float><<<grid, 256, 0, s>>>(a);
 }
 
 }  // namespace hs

@@ -167,15 +167,21 @@ __global__ void bias_grad_kernel(const void* __restrict__ delta, int ld, int wid
   const int j = blockIdx.x * blockDim.x + threadIdx.x;
   if (j >= width) return;
   const int b = offsets[m], e = offsets[m + 1];
-  float acc = 0.f;
+  // two-level sum (blocks of 256 rows) keeps the fp32 rounding of long segments small
+  float tot = 0.f;
+  for (int i0 = b; i0 < e; i0 += 256) {
+    const int i1 = min(e, i0 + 256);
+    float acc = 0.f;
 #pragma unroll 8
-  for (int i = b; i < e; ++i) {
-    if (kBf16)
-      acc += __bfloat162float(reinterpret_cast<const __nv_bfloat16*>(delta)[(int64_t)i * ld + j]);
-    else
-      acc += reinterpret_cast<const float*>(delta)[(int64_t)i * ld + j];
+    for (int i = i0; i < i1; ++i) {
+      if (kBf16)
+        acc += __bfloat162float(reinterpret_cast<const __nv_bfloat16*>(delta)[(int64_t)i * ld + j]);
+      else
+        acc += reinterpret_cast<const float*>(delta)[(int64_t)i * ld + j];
+    }
+    tot += acc;
   }
-  slabs[(int64_t)m * Ps + b_off + j] = acc;
+  slabs[(int64_t)m * Ps + b_off + j] = tot;
 }
 
 // Two-stage form for bf16 delta (16-byte rows).  Stage 1: each block sums a chunk of <= 128 rows of

@@ -55,9 +55,10 @@ def run_library(arch, dims, M, N, weights, x, y, theta0, lr, steps, precision, s
 
 
 def decide_for(precision):
-    """The bf16 kernels take the ReLU' decision from bf16-operand pre-activations; the oracle takes it
-    in the same precision (values stay fp64).  The fp32 check path is compared with the exact oracle."""
-    return mlp.round_bf16 if precision == hs.HS_BF16 else None
+    """The kernels take the ReLU' decision from pre-activations of rounded operands (bf16 operands;
+    fp32 stored activations with fp64-accumulated forward products on the check path); the oracle
+    takes it in the same precision, and every value it computes stays fp64."""
+    return mlp.round_bf16 if precision == hs.HS_BF16 else mlp.round_fp32
 
 
 def run_oracle(arch, dims, M, N, weights, x, y, theta0, lr, steps, sync, repartition=None, keep_slabs=False,

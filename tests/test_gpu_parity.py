@@ -141,7 +141,8 @@ def test_fp32_check_path_odd_widths(dims, N, M):
     theta0 = synth.he_normal_params(synth.MLP, dims, 3)
     w = list(rng.uniform(0.5, 2.0, M))
     lib = run_library(synth.MLP, dims, M, N, w, x, y, theta0, 0.1, 10, hs.HS_FP32_CHECK, hs.HS_SYNC_CP_WEIGHTED)
-    orc = run_oracle(synth.MLP, dims, M, N, w, x, y, theta0, 0.1, 10, hs.HS_SYNC_CP_WEIGHTED)
+    orc = run_oracle(synth.MLP, dims, M, N, w, x, y, theta0, 0.1, 10, hs.HS_SYNC_CP_WEIGHTED,
+                     decide=decide_for(hs.HS_FP32_CHECK))
     _check(lib, orc, theta0.astype(np.float64), hs.HS_FP32_CHECK, 10)
 
 

@@ -1,0 +1,163 @@
+"""Behaviour of hs_step beyond single-step parity: determinism, checkpoint/resume, host inputs,
+device-side checks, stale partitions, and the full-size workload (sampled against the oracle)."""
+import numpy as np
+import pytest
+import torch
+
+import synth
+import paper_2110_08941_gb300 as hs
+from oracle import mlp
+from oracle import partition as P
+from tests.gpu_helpers import rel
+
+pytestmark = pytest.mark.gpu
+
+
+def _ctx_and_data(name, precision=hs.HS_BF16, sync=hs.HS_SYNC_CP_WEIGHTED):
+    wl = synth.WORKLOADS[name]
+    x, y = synth.make_batch(wl)
+    theta0 = synth.make_params(wl)
+    ctx = hs.hs_init(wl.arch, wl.dims, wl.workers, wl.global_batch, compute_weights=synth.initial_weights(wl),
+                     precision=precision, sync=sync)
+    return wl, ctx, torch.from_numpy(x).cuda(), torch.from_numpy(y).cuda(), theta0
+
+
+@pytest.mark.parametrize("name", [synth.CFG2, synth.CFG4])
+def test_steps_are_bit_deterministic(name):
+    wl, ctx, xd, yd, theta0 = _ctx_and_data(name)
+    try:
+        outs = []
+        for _ in range(2):
+            p = torch.tensor(theta0, device="cuda")
+            hs.hs_sync_params(ctx, p)
+            for _ in range(3):
+                hs.hs_step(ctx, p, xd, yd, None, wl.lr, want_loss=False)
+            torch.cuda.synchronize()
+            outs.append(p.clone())
+        assert torch.equal(outs[0], outs[1])
+    finally:
+        ctx.close()
+
+
+def test_checkpoint_resume_is_bit_exact():
+    """5 steps, save theta and the partition state, restore into a fresh context, 5 more steps ==
+    10 straight steps (with a repartition at step 5 in both runs)."""
+    wl = synth.WORKLOADS[synth.CFG3]
+    x, y = synth.make_batch(wl)
+    theta0 = synth.make_params(wl)
+    speeds = synth.drift_walk(wl.workers, 10, wl.seed)
+    tp = list(synth.window_throughputs(speeds[0:5]))
+    xd, yd = torch.from_numpy(x).cuda(), torch.from_numpy(y).cuda()
+
+    def run(ctx, p, t0, t1):
+        for t in range(t0, t1):
+            if t == 5:
+                hs.hs_partition(ctx, tp)
+            hs.hs_step(ctx, p, xd, yd, None, wl.lr, want_loss=False)
+
+    c1 = hs.hs_init(wl.arch, wl.dims, wl.workers, wl.global_batch)
+    p1 = torch.tensor(theta0, device="cuda")
+    run(c1, p1, 0, 10)
+    torch.cuda.synchronize()
+    c1.close()
+
+    c2 = hs.hs_init(wl.arch, wl.dims, wl.workers, wl.global_batch)
+    p2 = torch.tensor(theta0, device="cuda")
+    run(c2, p2, 0, 5)
+    saved = p2.cpu().clone()
+    part_state = list(c2.partition.cp)
+    c2.close()
+    c3 = hs.hs_init(wl.arch, wl.dims, wl.workers, wl.global_batch, compute_weights=part_state)
+    p3 = saved.cuda()
+    run(c3, p3, 5, 10)
+    torch.cuda.synchronize()
+    c3.close()
+    assert torch.equal(p1, p3)
+
+
+@pytest.mark.parametrize("name", [synth.CFG1, synth.CFG4])
+def test_host_inputs_match_device_inputs(name):
+    wl, ctx, xd, yd, theta0 = _ctx_and_data(name)
+    try:
+        pa = torch.tensor(theta0, device="cuda")
+        la = hs.hs_step(ctx, pa, xd, yd, None, wl.lr)
+        pb = torch.tensor(theta0, device="cuda")
+        hs.hs_sync_params(ctx, pb)
+        lb = hs.hs_step(ctx, pb, xd.cpu().pin_memory(), yd.cpu(), None, wl.lr)   # pinned x, pageable y
+        assert la == lb
+        assert torch.equal(pa, pb)
+    finally:
+        ctx.close()
+
+
+def test_label_out_of_range_is_reported_not_faulted():
+    wl, ctx, xd, yd, theta0 = _ctx_and_data(synth.CFG1)
+    try:
+        p = torch.tensor(theta0, device="cuda")
+        bad = yd.clone()
+        bad[5] = wl.n_classes + 3
+        with pytest.raises(hs.HsError) as e:
+            hs.hs_step(ctx, p, xd, bad, None, wl.lr)
+        assert e.value.status == hs.HS_ERR_DEVICE_CHECK
+        # the context stays usable and the flag was cleared
+        hs.hs_step(ctx, p, xd, yd, None, wl.lr)
+    finally:
+        ctx.close()
+
+
+def test_stale_partition_and_bad_throughputs_rejected():
+    wl, ctx, xd, yd, theta0 = _ctx_and_data(synth.CFG2)
+    try:
+        p = torch.tensor(theta0, device="cuda")
+        old = ctx.partition
+        new = hs.hs_partition(ctx, [1.0, 2.0, 3.0, 4.0])
+        assert new.version == old.version + 1
+        with pytest.raises(hs.HsError) as e:
+            hs.hs_step(ctx, p, xd, yd, old, wl.lr)
+        assert e.value.status == hs.HS_ERR_INVALID_ARG
+        for bad in ([1.0, 0.0, 1.0, 1.0], [1.0, float("nan"), 1.0, 1.0], [1.0, -2.0, 1.0, 1.0]):
+            with pytest.raises(hs.HsError) as e:
+                hs.hs_partition(ctx, bad)
+            assert e.value.status == hs.HS_ERR_INVALID_ARG
+        assert hs.hs_partition(ctx).version == new.version
+        hs.hs_step(ctx, p, xd, yd, hs.hs_partition(ctx), wl.lr)
+    finally:
+        ctx.close()
+
+
+def test_headline_workload_sampled_parity():
+    """MLP 4096-8192-8192-1000, N = 16384, M = 16 at full size, in the launch configuration the
+    benchmark times: the two smallest workers' gradient slabs and losses against the oracle (worker
+    by worker), the index map bit-exact, and the fused update checked as a property of the slabs."""
+    wl, ctx, xd, yd, theta0 = _ctx_and_data(synth.CFG5)
+    try:
+        hs.hs_set_debug(ctx, True)
+        p = torch.tensor(theta0, device="cuda")
+        im = torch.empty(wl.global_batch, dtype=torch.int32, device="cuda")
+        part = hs.hs_partition(ctx, index_map_out=im)
+        sizes = P.partition_sizes(list(synth.initial_weights(wl)), wl.global_batch)
+        assert part.counts == sizes
+        assert np.array_equal(im.cpu().numpy(), np.asarray(P.index_map(sizes), dtype=np.int32))
+        hs.hs_step(ctx, p, xd, yd, part, wl.lr)
+        losses = hs.hs_worker_losses(ctx)
+        off = P.offsets(sizes)
+        x, y = xd.cpu().numpy(), yd.cpu().numpy()
+        g = torch.empty(ctx.P, device="cuda")
+        hs.hs_debug_grads(ctx, g, None)
+        slab = torch.empty(wl.workers, ctx.P, device="cuda")
+        hs.hs_debug_grads(ctx, None, slab)
+        for m in sorted(range(wl.workers), key=lambda k: sizes[k])[:2]:
+            lm, gm = mlp.worker_loss_grad(theta0, wl.dims, x[off[m]:off[m + 1]], y[off[m]:off[m + 1]],
+                                          decide=mlp.round_bf16)
+            assert rel(slab[m].cpu().numpy(), gm) <= 1e-2, m
+            assert abs(losses[m] - lm) <= 1e-2 * abs(lm)
+        del slab
+        # update property: theta_1 = theta_0 - lr * g (fp32) with g the synchronised gradient, to within
+        # the rounding of the fp32 result
+        th1 = p.cpu().numpy()
+        want = theta0.astype(np.float64) - np.float64(np.float32(wl.lr)) * g.cpu().double().numpy()
+        big = np.maximum(np.abs(theta0), np.abs(th1)).astype(np.float32)
+        ulp = np.spacing(big).astype(np.float64)
+        assert np.all(np.abs(th1.astype(np.float64) - want) <= 2 * ulp + 1e-12)
+    finally:
+        ctx.close()
