@@ -167,6 +167,26 @@ def oracle_sample(wl, seconds_target=12.0, max_workers=None):
     return done_samples / elapsed, desc, threads
 
 
+# ------------------------------------------------------------------------------ ranks
+def max_over_ranks(value: float) -> float:
+    """Max of a per-rank number over all ranks of the default process group (identity without one).
+    NCCL groups reduce a CUDA tensor, gloo groups a CPU tensor."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return float(value)
+    dev = torch.device("cuda", torch.cuda.current_device()) if dist.get_backend() == "nccl" else torch.device("cpu")
+    t = torch.tensor([float(value)], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier():
+    import torch.distributed as dist
+    if dist.is_available() and dist.is_initialized() and dist.get_world_size() > 1:
+        dist.barrier()
+
+
 # ------------------------------------------------------------------------------ arms
 def run_reference(args, wl, rank, world):
     if rank != 0:
@@ -214,15 +234,6 @@ def run_ours(args, wl, rank, world, local_rank):
 
     torch.cuda.set_device(local_rank)
     dev = torch.device("cuda", local_rank)
-    dist = None
-    if world > 1:
-        import torch.distributed as dist_mod
-        dist = dist_mod
-
-    def barrier():
-        if dist is not None:
-            dist.barrier()
-
     precision = hs.HS_BF16 if args.precision == "bf16" else hs.HS_FP32_CHECK
     x, y = synth.make_batch(wl)
     theta0 = synth.make_params(wl)
@@ -257,10 +268,7 @@ def run_ours(args, wl, rank, world, local_rank):
     ms = e0.elapsed_time(e1)
     prof = hs.hs_read_profile(ctx)
     hs.hs_set_profiling(ctx, False)
-    if dist is not None:
-        t = torch.tensor([ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = max_over_ranks(ms)
     loss = hs.hs_step(ctx, params, xd, yd, part, 0.0, stream=stream, want_loss=True)   # finite-loss check
 
     # end to end through the public API: host (pinned) inputs, loss read back every step
@@ -273,10 +281,7 @@ def run_ours(args, wl, rank, world, local_rank):
     for _ in range(k_e2e):
         hs.hs_step(ctx, params, xh, yh, part, wl.lr, stream=stream, want_loss=True)
     e2e_s = time.perf_counter() - t0
-    if dist is not None:
-        t = torch.tensor([e2e_s], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_s = float(t.item())
+    e2e_s = max_over_ranks(e2e_s)
 
     P = ctx.P
     peaks = _peaks()
