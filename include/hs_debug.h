@@ -28,6 +28,10 @@ enum {
                           /*   D_g at D + g * d_gstride                                  */
 };
 
+/* Kernel form, OR-ed into mode: 0 = the library's current form, HS_GEMM_FORM_SINGLE = one SM per
+ * 128 x 256 tile, HS_GEMM_FORM_PAIR = a two-SM cluster per 256 x 256 tile (tcgen05 cta_group::2). */
+enum { HS_GEMM_FORM_SINGLE = 0x100, HS_GEMM_FORM_PAIR = 0x200 };
+
 /* A, B, Z: bf16; bias: fp32 [N]; k_offsets_host: host int32 [groups+1] (HS_GEMM_WGRAD only,
  * else NULL with groups = 1).  Returns HS_ERR_INVALID_ARG for shapes the kernel cannot take
  * (leading dimensions must be multiples of 8 elements, pointers 16-byte aligned),

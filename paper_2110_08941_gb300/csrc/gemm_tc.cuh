@@ -64,7 +64,17 @@ constexpr int kTcStagingBytes = 4 * 2 * 32 * 128;   // 4 epilogue warps x 2 buff
 constexpr int kTcSmemBytes =
     kTcStages * (kTcBM + kTcBN) * kTcBK * 2 + kTcStagingBytes + 1024 /*align*/ + 256 /*barriers*/;
 
-// Launch on `num_sms` persistent CTAs (capped by the tile count).
+constexpr int kTcBoxB = 128;   // rows of a K-major B box (the 256-row B tile is two boxes)
+
+// Kernel form: one SM per 128 x 256 tile, or an SM pair (cluster of 2, tcgen05 cta_group::2) per
+// 256 x 256 tile.  Both read the same tensor maps; tiles_m / tiles_n are derived from the form.
+enum TcForm : int32_t { kTcFormSingle = 1, kTcFormPair = 2 };
+void tc_set_form(int form);
+int tc_get_form();
+
+// Launch on `num_sms` persistent CTAs (capped by the tile count) in the current form.
 cudaError_t launch_tc_gemm(const TcGemmParams& p, int num_sms, cudaStream_t s);
+cudaError_t launch_tc_gemm_form(const TcGemmParams& p, int num_sms, cudaStream_t s, int form);
+cudaError_t launch_tc_gemm_pair(const TcGemmParams& p, int num_sms, cudaStream_t s);
 
 }  // namespace hs

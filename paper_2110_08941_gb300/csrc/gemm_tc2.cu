@@ -1,0 +1,362 @@
+// SM-pair form of the tensor-core GEMM: a cluster of two CTAs computes one 256 x 256 output tile
+// with tcgen05.mma.cta_group::2.  Each CTA of the pair stages 128 rows of A and half of B (128 of
+// the 256 N columns) per k-block, so each SM reads 8 KB of operands from shared memory per
+// 128-cycle MMA instead of the 12 KB of the one-SM 128 x 256 form; the freed shared-memory
+// bandwidth is what the fp32 weight-gradient epilogue needs.  Same products and epilogues as
+// gemm_tc.cu (forward, input gradient, per-worker grouped weight gradient of Eq. 1's g^m).
+//
+// Roles (192 threads per CTA, one CTA per SM, clusters of 2):
+//   warp 0      (both CTAs) TMA loads of the CTA's A and B halves; completion is signalled on the
+//               leader CTA's stage barrier (the .cta_group::2 form of the bulk tensor copy)
+//   warp 1      (both CTAs) the collective tensor-memory allocation; in the leader CTA one thread
+//               issues the pair MMAs and commits them to both CTAs' barriers (multicast)
+//   warps 2..5  (both CTAs) epilogue of the CTA's 128 accumulator rows; each warp reports the
+//               accumulator free on the leader's barrier
+// Every mbarrier wait is bounded as in the one-SM kernel.
+#include <cudaTypedefs.h>
+
+#include "tc_device.cuh"
+
+namespace hs {
+
+namespace {
+
+using namespace tcdev;
+
+constexpr int PM = 256, PN = 256;                  // pair tile
+constexpr int HM = PM / 2, HN = PN / 2;            // per-CTA halves
+constexpr int S2 = 6;                              // pipeline stages
+constexpr int A_HALF = HM * BK * 2;                // 16 KB
+constexpr int B_HALF = HN * BK * 2;                // 16 KB
+constexpr int STAGE2 = A_HALF + B_HALF;
+constexpr uint32_t PAIR_TX = 2 * STAGE2;           // bytes landing per stage on the leader's barrier
+constexpr int kThreads2 = 192;
+constexpr uint32_t kTmemCols2 = 2 * PN;            // two accumulators of 128 lanes x 256 columns
+constexpr int kSmem2 = S2 * STAGE2 + kTcStagingBytes + 1024 + 256;
+
+static_assert(kSmem2 <= 232448, "shared memory budget");
+
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+// Address of the same shared-memory variable in CTA `rank` of the cluster.
+__device__ __forceinline__ uint32_t map_to_rank(uint32_t addr, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
+  return r;
+}
+__device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const CUtensorMap* tm, int c0, int c1,
+                                                 uint32_t leader_bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];"
+      ::"r"(dst), "l"(reinterpret_cast<uint64_t>(tm)), "r"(c0), "r"(c1), "r"(leader_bar)
+      : "memory");
+}
+__device__ __forceinline__ void tmem_alloc_pair(uint32_t dst_smem, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst_smem), "r"(ncols)
+               : "memory");
+}
+__device__ __forceinline__ void tmem_relinquish_pair() {
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc_pair(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+__device__ __forceinline__ void umma_bf16_pair(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                               uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}"
+      ::"r"(d_tmem), "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+// Arrive (once the issuing thread's MMAs complete) on the barrier at this offset in both CTAs.
+__device__ __forceinline__ void umma_commit_pair(uint32_t bar) {
+  const uint16_t mask = 3;
+  asm volatile("tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;"
+               ::"r"(bar), "h"(mask)
+               : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
+}
+
+template <int EPI, bool A_MN, bool B_MN>
+__global__ void __launch_bounds__(kThreads2, 1) tc_gemm_pair_kernel(const __grid_constant__ TcGemmParams p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sStage = smem + S2 * STAGE2;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sStage + kTcStagingBytes);
+  uint64_t* full_bar = bars;
+  uint64_t* empty_bar = bars + S2;
+  uint64_t* tfull_bar = bars + 2 * S2;
+  uint64_t* tempty_bar = bars + 2 * S2 + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * S2 + 4);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_rank();
+  const bool leader = (rank == 0);
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < S2; ++s) {
+      mbar_init(smem_u32(&full_bar[s]), 1);
+      mbar_init(smem_u32(&empty_bar[s]), 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(smem_u32(&tfull_bar[b]), 1);
+      mbar_init(smem_u32(&tempty_bar[b]), 8);   // 4 epilogue warps in each CTA of the pair
+    }
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc_pair(smem_u32(tmem_slot), kTmemCols2);
+    tmem_relinquish_pair();
+  }
+  tc_fence_before();
+  cluster_sync();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  const int tiles_m = (p.Mdim + PM - 1) / PM;
+  const int tiles_n = (p.n_store + PN - 1) / PN;
+  const int total = p.groups * tiles_m * tiles_n;
+  const int pair_id = blockIdx.x >> 1;
+  const int n_pairs = gridDim.x >> 1;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ------------------------------------------------------------ TMA producer (both CTAs)
+      int s = 0;
+      uint32_t ph = 0;
+      int last_g = -1;
+      for (int t = pair_id; t < total && !*abort_flag; t += n_pairs) {
+        const TileCoord c = decode_tile(t, tiles_m, tiles_n);
+        const CUtensorMap* ta = &p.tmA[c.g];
+        const CUtensorMap* tb = &p.tmB[c.g];
+        if (c.g != last_g) {
+          tma_prefetch_desc(ta);
+          tma_prefetch_desc(tb);
+          last_g = c.g;
+        }
+        const int nkb = p.num_kb[c.g];
+        const int m0 = c.tm * PM + (int)rank * HM;
+        const int n0 = c.tn * PN + (int)rank * HN;
+        bool ok = true;
+        for (int kb = 0; kb < nkb; ++kb) {
+          if (!mbar_wait(smem_u32(&empty_bar[s]), ph ^ 1u, abort_flag)) { ok = false; break; }
+          const uint32_t fb_local = smem_u32(&full_bar[s]);
+          const uint32_t fb = map_to_rank(fb_local, 0);
+          if (leader) mbar_expect_tx(fb_local, PAIR_TX);
+          const int k0 = kb * BK;
+          const uint32_t a_dst = smem_u32(smem + s * STAGE2);
+          const uint32_t b_dst = a_dst + A_HALF;
+          if (A_MN) {
+#pragma unroll
+            for (int j = 0; j < HM / 64; ++j) tma_load_2d_pair(a_dst + j * MN_CHUNK, ta, m0 + 64 * j, k0, fb);
+          } else {
+            tma_load_2d_pair(a_dst, ta, k0, m0, fb);
+          }
+          if (B_MN) {
+#pragma unroll
+            for (int j = 0; j < HN / 64; ++j) tma_load_2d_pair(b_dst + j * MN_CHUNK, tb, n0 + 64 * j, k0, fb);
+          } else {
+            tma_load_2d_pair(b_dst, tb, k0, n0, fb);
+          }
+          if (++s == S2) { s = 0; ph ^= 1u; }
+        }
+        if (!ok) {
+          record_error(p.st, kDevWaitTimeout, 11);
+          *abort_flag = 1;
+          break;
+        }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0 && leader) {
+      // ------------------------------------------------------------ pair MMA issuer (leader)
+      constexpr uint32_t idesc = make_idesc(A_MN, B_MN, PM, PN);
+      int s = 0;
+      uint32_t ph = 0;
+      int ab = 0;
+      uint32_t aph = 0;
+      for (int t = pair_id; t < total && !*abort_flag; t += n_pairs) {
+        const TileCoord c = decode_tile(t, tiles_m, tiles_n);
+        const int nkb = p.num_kb[c.g];
+        if (!mbar_wait(smem_u32(&tempty_bar[ab]), aph ^ 1u, abort_flag)) {
+          record_error(p.st, kDevWaitTimeout, 12);
+          *abort_flag = 1;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + (uint32_t)(ab * PN);
+        bool ok = true;
+        for (int kb = 0; kb < nkb; ++kb) {
+          if (!mbar_wait(smem_u32(&full_bar[s]), ph, abort_flag)) { ok = false; break; }
+          tc_fence_after();
+          const uint32_t a_base = smem_u32(smem + s * STAGE2);
+          const uint32_t b_base = a_base + A_HALF;
+#pragma unroll
+          for (int kk = 0; kk < BK / 16; ++kk) {
+            const uint64_t ad = A_MN ? make_sdesc(a_base + kk * 2048, MN_CHUNK, 1024)
+                                     : make_sdesc(a_base + kk * 32, 16, 1024);
+            const uint64_t bd = B_MN ? make_sdesc(b_base + kk * 2048, MN_CHUNK, 1024)
+                                     : make_sdesc(b_base + kk * 32, 16, 1024);
+            umma_bf16_pair(d_tmem, ad, bd, idesc, (kb | kk) != 0 ? 1u : 0u);
+          }
+          umma_commit_pair(smem_u32(&empty_bar[s]));
+          if (++s == S2) { s = 0; ph ^= 1u; }
+        }
+        if (!ok) {
+          record_error(p.st, kDevWaitTimeout, 13);
+          *abort_flag = 1;
+          break;
+        }
+        umma_commit_pair(smem_u32(&tfull_bar[ab]));
+        if (++ab == 2) { ab = 0; aph ^= 1u; }
+      }
+    }
+  } else {
+    // -------------------------------------------------------------- epilogue (warps 2..5, both CTAs)
+    constexpr bool kF32Out = (EPI == kTcEpiBiasF32 || EPI == kTcEpiStoreF32);
+    constexpr int kUnitCols = kF32Out ? 32 : 64;
+    constexpr int kUnits = PN / kUnitCols;
+    const int q = warp & 3;
+    const uint32_t stage_base = smem_u32(sStage) + (uint32_t)((warp - 2) * 8192);
+    int sb = 0;
+    int ab = 0;
+    uint32_t aph = 0;
+    for (int t = pair_id; t < total; t += n_pairs) {
+      const TileCoord c = decode_tile(t, tiles_m, tiles_n);
+      int ok = 1;
+      if (lane == 0) ok = mbar_wait(smem_u32(&tfull_bar[ab]), aph, abort_flag) ? 1 : 0;
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+      if (!ok) {
+        if (lane == 0) {
+          record_error(p.st, kDevWaitTimeout, 14);
+          *abort_flag = 1;
+        }
+        break;
+      }
+      __syncwarp();
+      tc_fence_after();
+      const int row0 = c.tm * PM + (int)rank * HM + q * 32;
+      const int row = row0 + lane;
+      const CUtensorMap* td = &p.tmD[c.g];
+      const uint32_t t_row = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(ab * PN);
+#pragma unroll 1
+      for (int u = 0; u < kUnits; ++u) {
+        const int n_base = c.tn * PN + u * kUnitCols;
+        if (n_base >= p.n_store) break;
+        uint32_t r[32], r2[32];
+        tmem_ld32(t_row + (uint32_t)(u * kUnitCols), r);
+        if (!kF32Out) tmem_ld32(t_row + (uint32_t)(u * kUnitCols + 32), r2);
+        tmem_ld_wait(r);
+        if (!kF32Out) tmem_ld_wait(r2);
+        uint4 o[8];
+        epilogue_unit<EPI>(p, row, n_base, r, r2, o);
+        if (lane == 0) bulk_wait_read_1();
+        __syncwarp();
+        const uint32_t buf = stage_base + (uint32_t)(sb * 4096);
+        const uint32_t rbase = buf + (uint32_t)(lane * 128);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) st_shared_v4(rbase + (uint32_t)(((j ^ (lane & 7)) << 4)), o[j]);
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) {
+          tma_store_2d(td, buf, n_base, row0);
+          bulk_commit();
+        }
+        sb ^= 1;
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_cluster(map_to_rank(smem_u32(&tempty_bar[ab]), 0));
+      if (++ab == 2) { ab = 0; aph ^= 1u; }
+    }
+    if (lane == 0) bulk_wait_all();
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (*abort_flag && threadIdx.x == 0) {
+    const uint64_t t0 = globaltimer();
+    while (globaltimer() - t0 < 2000000ull) {
+    }
+  }
+  // Neither CTA may leave while the pair's MMAs, multicast commits or remote arrivals can still
+  // touch its shared memory or tensor memory.
+  cluster_sync();
+  if (warp == 1) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc_pair(tmem_base, kTmemCols2);
+  }
+}
+
+template <int EPI, bool A_MN, bool B_MN>
+cudaError_t launch_pair_variant(const TcGemmParams& p, int pairs_wanted, int num_sms, cudaStream_t s) {
+  static bool configured = false;
+  static int max_clusters = 0;
+  auto kern = tc_gemm_pair_kernel<EPI, A_MN, B_MN>;
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.blockDim = dim3(kThreads2, 1, 1);
+  cfg.dynamicSmemBytes = kSmem2;
+  cfg.stream = s;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  if (!configured) {
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmem2);
+    if (e != cudaSuccess) return e;
+    // Persistent grid: no more clusters than can be resident at once (SMs pair up within a GPC).
+    cfg.gridDim = dim3(num_sms & ~1, 1, 1);
+    int n = 0;
+    e = cudaOccupancyMaxActiveClusters(&n, kern, &cfg);
+    if (e != cudaSuccess || n < 1) {
+      cudaGetLastError();
+      n = num_sms / 2;
+    }
+    max_clusters = n;
+    configured = true;
+  }
+  int pairs = pairs_wanted < max_clusters ? pairs_wanted : max_clusters;
+  if (pairs < 1) pairs = 1;
+  const int grid = 2 * pairs;
+  cfg.gridDim = dim3(grid, 1, 1);
+  cudaError_t e = cudaLaunchKernelEx(&cfg, kern, p);
+  if (e != cudaSuccess) return e;
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_tc_gemm_pair(const TcGemmParams& p, int num_sms, cudaStream_t s) {
+  const int tiles_m = (p.Mdim + PM - 1) / PM;
+  const int tiles_n = (p.n_store + PN - 1) / PN;
+  const int total = p.groups * tiles_m * tiles_n;
+  if (total <= 0) return cudaSuccess;
+  const int pairs = total;
+  const int grid = num_sms;   // forwarded as the SM count for the residency query
+  if (p.epi == kTcEpiBiasReluBf16 && !p.a_mn && !p.b_mn) return launch_pair_variant<kTcEpiBiasReluBf16, false, false>(p, pairs, grid, s);
+  if (p.epi == kTcEpiBiasF32 && !p.a_mn && !p.b_mn) return launch_pair_variant<kTcEpiBiasF32, false, false>(p, pairs, grid, s);
+  if (p.epi == kTcEpiMaskBf16 && !p.a_mn && p.b_mn) return launch_pair_variant<kTcEpiMaskBf16, false, true>(p, pairs, grid, s);
+  if (p.epi == kTcEpiStoreF32 && p.a_mn && p.b_mn) return launch_pair_variant<kTcEpiStoreF32, true, true>(p, pairs, grid, s);
+  if (p.epi == kTcEpiStoreF32 && !p.a_mn && !p.b_mn) return launch_pair_variant<kTcEpiStoreF32, false, false>(p, pairs, grid, s);
+  if (p.epi == kTcEpiStoreF32 && !p.a_mn && p.b_mn) return launch_pair_variant<kTcEpiStoreF32, false, true>(p, pairs, grid, s);
+  return cudaErrorInvalidValue;
+}
+
+}  // namespace hs

@@ -71,7 +71,7 @@ hs_status build_tc_static(hs_ctx* c) {
     hs::TcOperand a{reinterpret_cast<const __nv_bfloat16*>(c->d_act[l]), c->N, ly.in, ly.in};
     hs::TcOperand b{c->d_shadow + ly.w_off, ly.out, ly.in, ly.in};
     if (!hs::tc_make_kmajor_map(&f.tmA[0], a, hs::kTcBM, &why) ||
-        !hs::tc_make_kmajor_map(&f.tmB[0], b, hs::kTcBN, &why))
+        !hs::tc_make_kmajor_map(&f.tmB[0], b, hs::kTcBoxB, &why))
       return fail(c, HS_ERR_CUDA, why);
     f.num_kb[0] = (ly.in + hs::kTcBK - 1) / hs::kTcBK;
     f.groups = 1;
@@ -807,6 +807,9 @@ hs_status hs_debug_gemm_bf16(int32_t mode, int32_t M, int32_t N, int32_t K, cons
                              int64_t ldb, void* D, int64_t ldd, const float* bias, const void* Z, int64_t ldz,
                              const int32_t* k_offsets_host, int32_t groups, int64_t d_gstride, void* stream) {
   g_init_error.clear();
+  const int form = mode >> 8;
+  mode &= 0xFF;
+  if (form < 0 || form > 2) return fail(nullptr, HS_ERR_INVALID_ARG, "unknown kernel form");
   if (M < 1 || N < 1 || K < 0 || !A || !B || !D) return fail(nullptr, HS_ERR_INVALID_ARG, "bad GEMM arguments");
   const bool bf16_out = (mode == HS_GEMM_FWD_RELU || mode == HS_GEMM_DGRAD);
   if (lda % 8 || ldb % 8 || (bf16_out ? ldd % 8 : ldd % 4) || (mode == HS_GEMM_DGRAD && (ldz % 8 || !Z)) ||
@@ -857,7 +860,7 @@ hs_status hs_debug_gemm_bf16(int32_t mode, int32_t M, int32_t N, int32_t K, cons
     std::memset(&p, 0, sizeof(p));
     bool ok = hs::tc_make_kmajor_map(&p.tmA[0], hs::TcOperand{pa, M, K, lda}, hs::kTcBM, &why);
     if (mode == HS_GEMM_DGRAD) ok = ok && hs::tc_make_mnmajor_map(&p.tmB[0], hs::TcOperand{pb, K, N, ldb}, &why);
-    else ok = ok && hs::tc_make_kmajor_map(&p.tmB[0], hs::TcOperand{pb, N, K, ldb}, hs::kTcBN, &why);
+    else ok = ok && hs::tc_make_kmajor_map(&p.tmB[0], hs::TcOperand{pb, N, K, ldb}, hs::kTcBoxB, &why);
     if (!ok) return fail(nullptr, HS_ERR_INVALID_ARG, why);
     p.num_kb[0] = (K + hs::kTcBK - 1) / hs::kTcBK;
     p.groups = 1;
@@ -880,7 +883,7 @@ hs_status hs_debug_gemm_bf16(int32_t mode, int32_t M, int32_t N, int32_t K, cons
     p.tiles_n = (N + hs::kTcBN - 1) / hs::kTcBN;
     p.ldd = ldd;
     p.st = nullptr;
-    cudaError_t e = hs::launch_tc_gemm(p, sms, s);
+    cudaError_t e = hs::launch_tc_gemm_form(p, sms, s, form ? form : hs::tc_get_form());
     if (e != cudaSuccess) return cuda_fail(nullptr, e, "GEMM launch");
   }
   cudaError_t e = cudaStreamSynchronize(s);

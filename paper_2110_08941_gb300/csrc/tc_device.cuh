@@ -1,0 +1,275 @@
+// Device-side building blocks shared by the tensor-core GEMM kernels (one-SM and SM-pair forms):
+// PTX wrappers for mbarriers, TMA, tcgen05, the descriptors, tile decoding and the fused
+// epilogue unit.  Internal to libhs.
+#pragma once
+
+#include "gemm_tc.cuh"
+
+namespace hs {
+namespace tcdev {
+
+constexpr int BK = kTcBK;
+constexpr int MN_CHUNK = 64 * BK * 2;                // one 64-wide MN slab of an MN-major tile (8 KB)
+constexpr uint64_t kWaitLimitNs = 2000000000ull;     // 2 s per wait
+
+// ------------------------------------------------------------------ PTX wrappers
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ uint64_t globaltimer() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+__device__ __forceinline__ void fence_mbar_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+// Wait for the phase with the given parity; false if the abort flag rises or the limit passes.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = globaltimer();
+  while (true) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if (*abort_flag) return false;
+    if (globaltimer() - t0 > kWaitLimitNs) return false;
+  }
+}
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* tm, int c0, int c1,
+                                            uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];"
+      ::"r"(dst), "l"(reinterpret_cast<uint64_t>(tm)), "r"(c0), "r"(c1), "r"(bar)
+      : "memory");
+}
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap* tm, uint32_t src, int c0, int c1) {
+  asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%1, %2}], [%3];"
+               ::"l"(reinterpret_cast<uint64_t>(tm)), "r"(c0), "r"(c1), "r"(src)
+               : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+// At most one bulk group may still be reading shared memory.
+__device__ __forceinline__ void bulk_wait_read_1() {
+  asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
+}
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+__device__ __forceinline__ void st_shared_v4(uint32_t addr, uint4 v) {
+  asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w)
+               : "memory");
+}
+__device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap* tm) {
+  asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(tm)) : "memory");
+}
+__device__ __forceinline__ void tmem_alloc(uint32_t dst_smem, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst_smem),
+               "r"(ncols)
+               : "memory");
+}
+__device__ __forceinline__ void tmem_relinquish() {
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                          uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}"
+      ::"r"(d_tmem), "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+__device__ __forceinline__ void umma_commit(uint32_t bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+               : "memory");
+}
+// 32 lanes x 32 consecutive fp32 columns: thread t receives row (quadrant base + t).
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
+      "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]),
+        "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]),
+        "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]),
+        "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+}
+// The wait names the destination registers so no use of them is scheduled above it.
+__device__ __forceinline__ void tmem_ld_wait(uint32_t (&r)[32]) {
+  asm volatile("tcgen05.wait::ld.sync.aligned;"
+               : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]),
+                 "+r"(r[7]), "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]), "+r"(r[13]),
+                 "+r"(r[14]), "+r"(r[15]), "+r"(r[16]), "+r"(r[17]), "+r"(r[18]), "+r"(r[19]),
+                 "+r"(r[20]), "+r"(r[21]), "+r"(r[22]), "+r"(r[23]), "+r"(r[24]), "+r"(r[25]),
+                 "+r"(r[26]), "+r"(r[27]), "+r"(r[28]), "+r"(r[29]), "+r"(r[30]), "+r"(r[31])
+               :
+               : "memory");
+}
+
+// Instruction descriptor, kind::f16: D fp32, A/B bf16, per-operand major-ness, N = BN, M = BM.
+__host__ __device__ constexpr uint32_t make_idesc(bool a_mn, bool b_mn, int m, int n) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((a_mn ? 1u : 0u) << 15) | ((b_mn ? 1u : 0u) << 16) |
+         ((uint32_t)(n >> 3) << 17) | ((uint32_t)(m >> 4) << 24);
+}
+
+// Shared-memory matrix descriptor, 128-byte swizzle.  lbo/sbo in bytes.
+//   K-major tile (rows x 64 K, 128 B per row, 8-row swizzle atoms of 1 KB): SBO = 1 KB between
+//     8-row groups; LBO unused.  The K step of 16 elements advances the start by 32 B.
+//   MN-major tile (64 K rows x 128 B per 64-wide MN slab): SBO = 1 KB between 8-row K groups,
+//     LBO = 8 KB between 64-wide MN slabs.  The K step of 16 rows advances the start by 2 KB.
+__device__ __forceinline__ uint64_t make_sdesc(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);
+  d |= (uint64_t)((lbo >> 4) & 0x3FFFu) << 16;
+  d |= (uint64_t)((sbo >> 4) & 0x3FFFu) << 32;
+  d |= 1ull << 46;
+  d |= 2ull << 61;
+  return d;
+}
+
+__device__ __forceinline__ void record_error(DevStatus* st, int32_t code, int32_t info) {
+  if (st && atomicCAS(&st->err, 0, code) == 0) st->err_info = info;
+}
+
+struct TileCoord {
+  int g, tm, tn;
+};
+
+// Tiles are numbered group-major; within a group, bands of 16 M-tiles are walked N-tile by
+// N-tile so that the CTAs running at the same time share A and B panels in L2.
+__device__ __forceinline__ TileCoord decode_tile(int t, int tiles_m, int tiles_n) {
+  const int per_group = tiles_m * tiles_n;
+  TileCoord c;
+  c.g = t / per_group;
+  const int r = t - c.g * per_group;
+  constexpr int GM = 16;
+  const int band = r / (GM * tiles_n);
+  const int within = r - band * GM * tiles_n;
+  const int rows = min(GM, tiles_m - band * GM);
+  c.tm = band * GM + within % rows;
+  c.tn = within / rows;
+  return c;
+}
+
+__device__ __forceinline__ float u2f(uint32_t u) { return __uint_as_float(u); }
+
+__device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
+  __nv_bfloat162 v = __floats2bfloat162_rn(a, b);
+  return *reinterpret_cast<uint32_t*>(&v);
+}
+
+// One epilogue unit: a 128-byte column strip of one accumulator row (32 fp32 or 64 bf16 outputs),
+// computed from `r` (columns n_base..n_base+31) and, for bf16 outputs, `r2` (n_base+32..+63), packed
+// into eight 16-byte words.  Columns past n_store are computed but never stored (the TMA store
+// clips them); only the bias and mask reads are guarded.
+template <int EPI>
+__device__ __forceinline__ void epilogue_unit(const TcGemmParams& p, int row, int n_base, const uint32_t (&r)[32],
+                                              const uint32_t (&r2)[32], uint4 (&o)[8]) {
+  if (EPI == kTcEpiStoreF32) {
+#pragma unroll
+    for (int j = 0; j < 8; ++j) o[j] = make_uint4(r[4 * j], r[4 * j + 1], r[4 * j + 2], r[4 * j + 3]);
+  } else if (EPI == kTcEpiBiasF32) {
+    float b[32];
+    if (n_base + 32 <= p.Ndim) {
+      const float4* b4 = reinterpret_cast<const float4*>(p.bias + n_base);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const float4 t = __ldg(b4 + j);
+        b[4 * j] = t.x; b[4 * j + 1] = t.y; b[4 * j + 2] = t.z; b[4 * j + 3] = t.w;
+      }
+    } else {
+#pragma unroll
+      for (int j = 0; j < 32; ++j) b[j] = (n_base + j < p.Ndim) ? __ldg(p.bias + n_base + j) : 0.f;
+    }
+#pragma unroll
+    for (int j = 0; j < 8; ++j)
+      o[j] = make_uint4(__float_as_uint(u2f(r[4 * j]) + b[4 * j]), __float_as_uint(u2f(r[4 * j + 1]) + b[4 * j + 1]),
+                        __float_as_uint(u2f(r[4 * j + 2]) + b[4 * j + 2]),
+                        __float_as_uint(u2f(r[4 * j + 3]) + b[4 * j + 3]));
+  } else {
+    // bf16 outputs: 64 columns
+    float v[64];
+#pragma unroll
+    for (int j = 0; j < 32; ++j) {
+      v[j] = u2f(r[j]);
+      v[32 + j] = u2f(r2[j]);
+    }
+    if (EPI == kTcEpiBiasReluBf16) {
+      if (n_base + 64 <= p.Ndim) {
+        const float4* b4 = reinterpret_cast<const float4*>(p.bias + n_base);
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
+          const float4 t = __ldg(b4 + j);
+          v[4 * j] = fmaxf(v[4 * j] + t.x, 0.f);
+          v[4 * j + 1] = fmaxf(v[4 * j + 1] + t.y, 0.f);
+          v[4 * j + 2] = fmaxf(v[4 * j + 2] + t.z, 0.f);
+          v[4 * j + 3] = fmaxf(v[4 * j + 3] + t.w, 0.f);
+        }
+      } else {
+#pragma unroll
+        for (int j = 0; j < 64; ++j)
+          v[j] = fmaxf(v[j] + ((n_base + j < p.Ndim) ? __ldg(p.bias + n_base + j) : 0.f), 0.f);
+      }
+    } else {   // kTcEpiMaskBf16: ReLU' from the stored activation of the same row
+      if (row < p.Mdim) {
+        const __nv_bfloat16* z = p.Z + (int64_t)row * p.ldz + n_base;
+        if (n_base + 64 <= p.n_store) {
+          const uint4* z4 = reinterpret_cast<const uint4*>(z);
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            const uint4 zz = __ldg(z4 + j);
+            const uint32_t w[4] = {zz.x, zz.y, zz.z, zz.w};
+#pragma unroll
+            for (int h = 0; h < 4; ++h) {
+              const __nv_bfloat162 pr = *reinterpret_cast<const __nv_bfloat162*>(&w[h]);
+              const int k = 8 * j + 2 * h;
+              v[k] = (__low2float(pr) > 0.f) ? v[k] : 0.f;
+              v[k + 1] = (__high2float(pr) > 0.f) ? v[k + 1] : 0.f;
+            }
+          }
+        } else {
+#pragma unroll
+          for (int j = 0; j < 64; ++j) v[j] = (n_base + j < p.n_store && __bfloat162float(z[j]) > 0.f) ? v[j] : 0.f;
+        }
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < 8; ++j)
+      o[j] = make_uint4(pack_bf16(v[8 * j], v[8 * j + 1]), pack_bf16(v[8 * j + 2], v[8 * j + 3]),
+                        pack_bf16(v[8 * j + 4], v[8 * j + 5]), pack_bf16(v[8 * j + 6], v[8 * j + 7]));
+  }
+}
+
+}  // namespace tcdev
+}  // namespace hs
