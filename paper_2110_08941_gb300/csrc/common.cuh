@@ -50,9 +50,11 @@ void launch_bias_grad_bf16(const __nv_bfloat16* delta, int ld, int width, const 
                            const int32_t* d_chunk_begin, int M, float* partial, float* slabs, int64_t Ps,
                            int64_t b_off, cudaStream_t s);
 // theta[j] -= lr * sum_m w[m] * slabs[m*Ps + j]; shadow[j] = bf16(theta[j]); gdebug[j] = g (optional)
+// Works on any contiguous parameter range (pointers offset to its start, 16-byte aligned; slab m
+// of the range at slabs + m*Ps).  blocks_per_sm = 1 leaves room for a resident GEMM CTA.
 void launch_reduce_update(float* theta, const float* slabs, int64_t Ps, int M, const float* d_w,
                           float lr, int64_t P, __nv_bfloat16* shadow, float* gdebug, int num_sms,
-                          cudaStream_t s);
+                          cudaStream_t s, int blocks_per_sm = 4);
 
 // ---------------------------------------------------------------- fp32 CUDA-core GEMM (check path)
 // C(m, n) = sum_k A(m, k) B(k, n) with A(m,k) = A[m*a_sm + k*a_sk], B(k,n) = B[k*b_sk + n*b_sn],

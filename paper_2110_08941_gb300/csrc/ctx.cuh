@@ -105,6 +105,13 @@ struct hs_ctx {
     return e;
   }
 
+  // per-layer updates overlapped with the rest of the backward pass (bf16 MLP): a side stream that
+  // waits for each layer's backward, and the event the caller's stream waits for at the end
+  bool overlap_update = false;
+  cudaStream_t upd_stream = nullptr;
+  std::vector<cudaEvent_t> upd_ready;
+  cudaEvent_t upd_done = nullptr;
+
   // CNN workload: convs[0..2], then the fully connected layer (index 3 in per-layer arrays)
   int64_t in_features = 0;
   std::vector<hs::ConvLayer> convs;

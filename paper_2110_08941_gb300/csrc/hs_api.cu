@@ -1,6 +1,7 @@
 // C-ABI of libhs: context, Dynamic Partitioning (Algorithm 1) and the synchronous SGD step
 // (Section 1, Eq. 1, Section 4.2) over M logical workers on one GPU.
 #include <cmath>
+#include <cstdlib>
 #include <cstdio>
 #include <cstring>
 #include <string>
@@ -269,6 +270,9 @@ void free_all(hs_ctx* c) {
     cudaEventDestroy(r.b);
   }
   for (cudaEvent_t e : c->event_pool) cudaEventDestroy(e);
+  for (cudaEvent_t e : c->upd_ready) if (e) cudaEventDestroy(e);
+  if (c->upd_done) cudaEventDestroy(c->upd_done);
+  if (c->upd_stream) cudaStreamDestroy(c->upd_stream);
 }
 
 bool is_device_ptr(const void* p) {
@@ -349,7 +353,18 @@ hs_status mlp_step_fp32(hs_ctx* c, float* params, const float* x, const int32_t*
   return HS_OK;
 }
 
-hs_status mlp_step_bf16(hs_ctx* c, float* params, const float* x, const int32_t* y, cudaStream_t s) {
+// theta <- theta - lr * sum_m w_m G_m over layer l's parameter range [W_l, b_l] (Section 1).
+void update_layer_range(hs_ctx* c, float* params, int l, float lr, cudaStream_t s, int blocks_per_sm) {
+  const int64_t start = c->layers[l].w_off;
+  const int64_t end = (l + 1 < c->L) ? c->layers[l + 1].w_off : c->P;
+  PhaseScope ph(c, HS_PHASE_UPDATE, s);
+  hs::launch_reduce_update(params + start, c->d_slabs + start, c->Ps, c->M, c->d_w, lr, end - start,
+                           c->d_shadow + start, c->debug ? c->d_gdebug + start : nullptr, c->num_sms, s,
+                           blocks_per_sm);
+  ph.launched();
+}
+
+hs_status mlp_step_bf16(hs_ctx* c, float* params, const float* x, const int32_t* y, float lr, cudaStream_t s) {
   const int L = c->L;
   {
     PhaseScope ph(c, HS_PHASE_CAST, s);
@@ -397,6 +412,19 @@ hs_status mlp_step_bf16(hs_ctx* c, float* params, const float* x, const int32_t*
       if (e != cudaSuccess) return cuda_fail(c, e, "input-gradient GEMM launch");
       ph.launched();
     }
+    if (c->overlap_update) {
+      // Layer l's slabs are complete and its input-gradient product has read W_l's bf16 shadow: its
+      // update can run beside the remaining (tensor-core bound) backward products.
+      HS_CUDA(c, cudaEventRecord(c->upd_ready[l], s));
+      HS_CUDA(c, cudaStreamWaitEvent(c->upd_stream, c->upd_ready[l], 0));
+      update_layer_range(c, params, l, lr, c->upd_stream, l == 0 ? 4 : 1);
+    }
+  }
+  if (c->overlap_update) {
+    HS_CUDA(c, cudaEventRecord(c->upd_done, c->upd_stream));
+    HS_CUDA(c, cudaStreamWaitEvent(s, c->upd_done, 0));
+  } else {
+    for (int l = L - 1; l >= 0; --l) update_layer_range(c, params, l, lr, s, 4);
   }
   return HS_OK;
 }
@@ -617,6 +645,17 @@ hs_status hs_init(const hs_model_desc* model, int32_t M, const double* compute_w
     if (e != cudaSuccess) s2 = cuda_fail(c, e, "cudaMemset");
   }
   if (s2 == HS_OK && bf16) s2 = c->arch == HS_MLP ? build_tc_static(c) : cnn_build_static(c);
+  if (s2 == HS_OK && bf16 && c->arch == HS_MLP) {
+    const char* ov = getenv("HS_OVERLAP_UPDATE");
+    c->overlap_update = !(ov && !strcmp(ov, "0"));
+    if (c->overlap_update) {
+      e = cudaStreamCreateWithFlags(&c->upd_stream, cudaStreamNonBlocking);
+      c->upd_ready.assign(c->L, nullptr);
+      for (int l = 0; l < c->L && e == cudaSuccess; ++l) e = cudaEventCreateWithFlags(&c->upd_ready[l], cudaEventDisableTiming);
+      if (e == cudaSuccess) e = cudaEventCreateWithFlags(&c->upd_done, cudaEventDisableTiming);
+      if (e != cudaSuccess) s2 = cuda_fail(c, e, "update stream");
+    }
+  }
   if (s2 == HS_OK) s2 = apply_partition(c, sizes, cpn, nullptr, 0);
   if (s2 == HS_OK) {
     e = cudaDeviceSynchronize();
@@ -704,11 +743,12 @@ hs_status hs_step(hs_ctx* c, float* params, const void* x, const int32_t* y, con
     hs_status r = dalloc(c, &c->d_gdebug, sizeof(float) * c->Ps);
     if (r != HS_OK) return r;
   }
-  hs_status st = c->arch == HS_CNN            ? cnn_step(c, params, xd, yd, s)
-                 : c->precision == HS_BF16 ? mlp_step_bf16(c, params, xd, yd, s)
-                                           : mlp_step_fp32(c, params, xd, yd, s);
+  const bool mlp_bf16 = (c->arch == HS_MLP && c->precision == HS_BF16);
+  hs_status st = c->arch == HS_CNN ? cnn_step(c, params, xd, yd, s)
+                 : mlp_bf16        ? mlp_step_bf16(c, params, xd, yd, lr, s)
+                                   : mlp_step_fp32(c, params, xd, yd, s);
   if (st != HS_OK) return st;
-  {
+  if (!mlp_bf16) {
     PhaseScope ph(c, HS_PHASE_UPDATE, s);
     hs::launch_reduce_update(params, c->d_slabs, c->Ps, c->M, c->d_w, lr, c->P,
                              c->precision == HS_BF16 ? c->d_shadow : nullptr, c->debug ? c->d_gdebug : nullptr,

@@ -278,9 +278,9 @@ __global__ void __launch_bounds__(512) reduce_update_kernel(
     float* __restrict__ theta, const float* __restrict__ slabs, int64_t Ps, int M,
     const float* __restrict__ w, float lr, int64_t P, __nv_bfloat16* __restrict__ shadow,
     float* __restrict__ gdebug) {
-  __shared__ float sw[kMaxWorkers];
-  for (int m = threadIdx.x; m < M; m += blockDim.x) sw[m] = w[m];
-  __syncthreads();
+  // The weights stay in global memory (read through the read-only cache): no shared memory, so
+  // blocks of this kernel can share an SM with a resident tensor-core GEMM CTA.
+  const float* __restrict__ sw = w;
   const int64_t nvec = P / 4;
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   const float4* s4 = reinterpret_cast<const float4*>(slabs);
@@ -294,7 +294,7 @@ __global__ void __launch_bounds__(512) reduce_update_kernel(
       for (int u = 0; u < 8; ++u) g[u] = __ldcs(s4 + (int64_t)(m + u) * ps4 + v);
 #pragma unroll
       for (int u = 0; u < 8; ++u) {
-        const float wm = sw[m + u];
+        const float wm = __ldg(sw + m + u);
         acc.x = fmaf(wm, g[u].x, acc.x);
         acc.y = fmaf(wm, g[u].y, acc.y);
         acc.z = fmaf(wm, g[u].z, acc.z);
@@ -303,7 +303,7 @@ __global__ void __launch_bounds__(512) reduce_update_kernel(
     }
     for (; m < M; ++m) {
       const float4 g = __ldcs(s4 + (int64_t)m * ps4 + v);
-      const float wm = sw[m];
+      const float wm = __ldg(sw + m);
       acc.x = fmaf(wm, g.x, acc.x);
       acc.y = fmaf(wm, g.y, acc.y);
       acc.z = fmaf(wm, g.z, acc.z);
@@ -327,7 +327,7 @@ __global__ void __launch_bounds__(512) reduce_update_kernel(
   }
   for (int64_t j = nvec * 4 + (int64_t)blockIdx.x * blockDim.x + threadIdx.x; j < P; j += stride) {
     float acc = 0.f;
-    for (int m = 0; m < M; ++m) acc = fmaf(sw[m], slabs[(int64_t)m * Ps + j], acc);
+    for (int m = 0; m < M; ++m) acc = fmaf(__ldg(sw + m), slabs[(int64_t)m * Ps + j], acc);
     const float t = fmaf(-lr, acc, theta[j]);
     theta[j] = t;
     if (shadow) shadow[j] = __float2bfloat16_rn(t);
@@ -337,10 +337,10 @@ __global__ void __launch_bounds__(512) reduce_update_kernel(
 
 void launch_reduce_update(float* theta, const float* slabs, int64_t Ps, int M, const float* d_w,
                           float lr, int64_t P, __nv_bfloat16* shadow, float* gdebug, int num_sms,
-                          cudaStream_t s) {
+                          cudaStream_t s, int blocks_per_sm) {
   const int threads = 512;
   int64_t blocks = (P / 4 + threads - 1) / threads;
-  const int64_t cap = (int64_t)num_sms * 4;
+  const int64_t cap = (int64_t)num_sms * blocks_per_sm;
   if (blocks > cap) blocks = cap;
   if (blocks < 1) blocks = 1;
   reduce_update_kernel<<<(int)blocks, threads, 0, s>>>(theta, slabs, Ps, M, d_w, lr, P, shadow, gdebug);
