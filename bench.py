@@ -126,6 +126,32 @@ def gemm_flops(wl):
                 dgrad=2.0 * n * (per[1] + per[2] + fc))
 
 
+def recorded_traffic(kernel_tag="tc_gemm_pair_wgrad"):
+    """DRAM bytes per launch of the dominant kernel from the committed ncu summary, or None when the
+    kernel sources changed since those counters were taken."""
+    import glob
+    import hashlib
+    files = glob.glob(os.path.join(ROOT, "profiles", kernel_tag + "_*_dram.md"))
+    if not files:
+        return None
+    text = open(files[0]).read()
+    vals = {}
+    for line in text.splitlines():
+        if ":" in line and line.split(":")[0] in ("traffic_bytes_per_launch", "kernel_source_sha256"):
+            k, v = line.split(":", 1)
+            vals[k] = v.strip()
+    csrc = os.path.join(ROOT, "paper_2110_08941_gb300", "csrc")
+    h = hashlib.sha256()
+    for f in ("gemm_tc2.cu", "tc_device.cuh", "gemm_tc.cuh"):
+        h.update(open(os.path.join(csrc, f), "rb").read())
+    if vals.get("kernel_source_sha256") != h.hexdigest():
+        return None
+    try:
+        return float(vals["traffic_bytes_per_launch"])
+    except (KeyError, ValueError):
+        return None
+
+
 def update_bytes(wl, P):
     # M slab reads + theta read, theta write + bf16 shadow write
     return (wl.workers + 2) * P * 4 + 2 * P
@@ -293,16 +319,23 @@ def run_ours(args, wl, rank, world, local_rank):
     candidates = {k: per_step[k] for k in ("forward", "wgrad", "dgrad", "update")}
     dominant = max(candidates, key=candidates.get)
 
+    launches_per_step = {k: max(1, round(v[1] / args.steps)) for k, v in prof.items()}
+
     def gemm_roof(name):
+        # per launch: the phase's algorithmic flops and time divided by its launches per step
         ach = flops[name] / (per_step[name] * 1e-3) / 1e12
+        traffic = recorded_traffic() if (name == "wgrad" and wl.name == DEFAULT_WORKLOAD) else None
         return {"kernel": f"tc_gemm ({name})", "bound": "tensor", "achieved": ach, "peak": peaks["bf16_sust"],
-                "unit": "TFLOP/s", "frac": ach / peaks["bf16_sust"], "traffic": None,
+                "unit": "TFLOP/s", "frac": ach / peaks["bf16_sust"], "traffic": traffic,
+                "flops_per_launch": flops[name] / launches_per_step[name],
+                "launches_per_step": launches_per_step[name],
                 "peak_kind": f"{peaks['src']} bf16 sustained"}
 
     upd_ach = upd_bytes / (per_step["update"] * 1e-3) / 1e9
     roof_update = {"kernel": "reduce_update", "bound": "hbm", "achieved": upd_ach, "peak": peaks["hbm"],
                    "unit": "GB/s", "frac": upd_ach / peaks["hbm"], "traffic": None,
-                   "peak_kind": f"{peaks['src']} copy bandwidth", "algorithmic_bytes": upd_bytes}
+                   "peak_kind": f"{peaks['src']} copy bandwidth", "algorithmic_bytes": upd_bytes,
+                   "overlapped_with_gemms": os.environ.get("HS_OVERLAP_UPDATE", "1") != "0" and wl.arch == synth.MLP}
     roofline = roof_update if dominant == "update" else gemm_roof(dominant)
     gemm_ms = per_step["forward"] + per_step["wgrad"] + per_step["dgrad"]
     gemm_total = sum(flops.values())
