@@ -152,6 +152,32 @@ def recorded_traffic(kernel_tag="tc_gemm_pair_wgrad"):
         return None
 
 
+def straggler_simulation(seed=0, steps=200, every=10):
+    """Simulated iteration time of the drifting 8-worker workload (the straggler model of Section 3:
+    a synchronous step lasts as long as its slowest worker, X_(M) = max_m n_m / c_m(t)), summed
+    over `steps` steps for three schedules: the even split of Sync-SGD, Dynamic Partitioning
+    (Algorithm 1, repartitioned every `every` steps from the window's measured throughputs through
+    the library's host rule), and the ideal real-valued split n_m proportional to c_m(t).  Host
+    only; speeds c_m(t) from the seeded random walk."""
+    import paper_2110_08941_gb300 as hs
+    wl = synth.WORKLOADS[synth.CFG3]
+    m, n = wl.workers, wl.global_batch
+    c = synth.drift_walk(m, steps, seed)
+    even = hs.hs_partition_sizes([1.0] * m, n)
+    sizes = list(even)
+    t_even = t_dp = t_ideal = 0.0
+    for t in range(steps):
+        ct = c[t]
+        t_even += max(even[k] / ct[k] for k in range(m))
+        t_dp += max(sizes[k] / ct[k] for k in range(m))
+        t_ideal += n / float(np.sum(ct))
+        if (t + 1) % every == 0:
+            sizes = hs.hs_partition_sizes(list(synth.window_throughputs(c[t + 1 - every:t + 1])), n)
+    return {"workload": wl.name, "steps": steps, "repartition_every": every,
+            "sum_max_time_even": t_even, "sum_max_time_dynamic_partitioning": t_dp,
+            "sum_time_ideal_split": t_ideal, "unit": "sample-times (n / speed, speed c_m(0) = 1)"}
+
+
 def update_bytes(wl, P):
     # M slab reads + theta read, theta write + bf16 shadow write
     return (wl.workers + 2) * P * 4 + 2 * P
@@ -366,6 +392,7 @@ def run_ours(args, wl, rank, world, local_rank):
             "e2e": {"value": world * wl.global_batch * k_e2e / e2e_s, "unit": UNIT,
                     "h2d_bytes_per_step": int(x.nbytes + y.nbytes), "d2h_bytes_per_step": 12},
             "clocks": clk,
+            "straggler_sim": straggler_simulation(),
             "loss_after": loss,
         }
         print(json.dumps(out), flush=True)
