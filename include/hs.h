@@ -149,6 +149,24 @@ hs_status hs_partition(hs_ctx* ctx, const double* measured_throughputs, int32_t*
 hs_status hs_step(hs_ctx* ctx, float* params, const void* x, const int32_t* y,
                   const hs_partition_t* part, float lr, void* stream, float* loss_out);
 
+/* The training recipe of the paper's experiments (Section 5: SGD with momentum and weight decay)
+ * in the fused update.  With d = g + weight_decay * theta (g the synchronised gradient):
+ *   b = d on the first step after this call, b = momentum * b + d afterwards, theta <- theta - lr * b.
+ * momentum in [0, 1), weight_decay >= 0; both 0 restores plain SGD.  Allocates the momentum buffer
+ * (device fp32 [P], one more read and write per parameter per step) on first use and restarts it.
+ * Errors: HS_ERR_INVALID_ARG, HS_ERR_OOM. */
+hs_status hs_set_optimizer(hs_ctx* ctx, float momentum, float weight_decay);
+
+/* Checkpointing of the momentum buffer: save != 0 copies it to buf_dev (device fp32 [P]); save == 0
+ * restores it from buf_dev and the next step continues it (no restart).  Enqueued on `stream`.
+ * Errors: HS_ERR_INVALID_ARG without hs_set_optimizer, or when saving a buffer no step started. */
+hs_status hs_optimizer_state(hs_ctx* ctx, float* buf_dev, int32_t save, void* stream);
+
+/* Cosine annealing of the learning rate over T steps (Section 5):
+ * eta_min + (eta0 - eta_min) * (1 + cos(pi * t / T)) / 2, t clamped to [0, T]; T <= 0 gives eta0.
+ * Host only. */
+double hs_cosine_lr(double eta0, double eta_min, int64_t t, int64_t T);
+
 /* The bf16 parameter shadow is refreshed by every hs_step for the params
  * pointer it updated.  A caller that writes params in place between steps
  * (checkpoint restore, manual edits) calls this to re-derive the shadow. */

@@ -13,6 +13,13 @@ Test infrastructure only (see oracle/__init__.py).
 * Update (Section 1): theta_{t+1} = theta_t - eta_t g_t (plain SGD).
 
 The reported loss is sum_m w_m L_m with the same weights, at theta_t.
+
+The training recipe of Section 5 adds, on top of the synchronised gradient g:
+* weight decay lambda and momentum mu (heavy ball, no dampening):
+  d = g + lambda * theta;  b = d on the first step, b = mu * b + d afterwards;
+  theta <- theta - eta_t * b;
+* cosine annealing of the learning rate over T steps:
+  eta_t = eta_min + (eta_0 - eta_min) * (1 + cos(pi * t / T)) / 2.
 """
 from __future__ import annotations
 
@@ -74,3 +81,16 @@ def step(grad_fn: Callable, theta, dims, x, y, sizes, lr: float, mode: int,
             slabs.append(g_m)
     loss = float(np.dot(w, np.asarray(losses)))
     return theta - lr * g, loss, g, slabs, losses
+
+
+def momentum_update(theta, g, buf, lr: float, momentum: float, weight_decay: float):
+    """One update of the Section 5 recipe; buf is None on the first step.  Returns (theta, buf)."""
+    theta = np.asarray(theta, dtype=np.float64)
+    d = np.asarray(g, dtype=np.float64) + weight_decay * theta
+    buf = d.copy() if buf is None else momentum * buf + d
+    return theta - lr * buf, buf
+
+
+def cosine_lr(eta0: float, eta_min: float, t: int, T: int) -> float:
+    """Cosine annealing (Section 5): eta_min + (eta0 - eta_min) * (1 + cos(pi t / T)) / 2."""
+    return eta_min + (eta0 - eta_min) * (1.0 + np.cos(np.pi * t / T)) / 2.0

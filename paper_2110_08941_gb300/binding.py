@@ -26,7 +26,7 @@ HS_GEMM_FORM_SINGLE, HS_GEMM_FORM_PAIR = 0x100, 0x200
 EXPORTED = ("hs_partition_sizes", "hs_param_count", "hs_init", "hs_partition", "hs_step", "hs_sync_params",
             "hs_set_debug", "hs_debug_grads", "hs_worker_losses", "hs_destroy", "hs_status_string",
             "hs_last_error", "hs_last_init_error", "hs_debug_gemm_bf16", "hs_set_profiling", "hs_read_profile",
-            "hs_partition_noalloc")
+            "hs_partition_noalloc", "hs_set_optimizer", "hs_optimizer_state", "hs_cosine_lr")
 PHASES = ("cast", "forward", "loss", "wgrad", "biasgrad", "dgrad", "update")
 
 
@@ -64,6 +64,9 @@ def _load() -> ctypes.CDLL:
         "hs_sync_params": (S, [c_void_p, c_void_p, c_void_p]),
         "hs_set_debug": (S, [c_void_p, c_int32]),
         "hs_set_profiling": (S, [c_void_p, c_int32]),
+        "hs_set_optimizer": (S, [c_void_p, c_float, c_float]),
+        "hs_optimizer_state": (S, [c_void_p, c_void_p, c_int32, c_void_p]),
+        "hs_cosine_lr": (c_double, [c_double, c_double, c_int64, c_int64]),
         "hs_read_profile": (S, [c_void_p, POINTER(c_double), POINTER(c_int64)]),
         "hs_debug_grads": (S, [c_void_p, c_void_p, c_void_p, c_void_p]),
         "hs_worker_losses": (S, [c_void_p, POINTER(c_float)]),
@@ -220,6 +223,19 @@ def hs_sync_params(ctx: Context, params, stream=None):
 
 def hs_set_debug(ctx: Context, enable: bool = True):
     _check(_lib.hs_set_debug(ctx.ptr, 1 if enable else 0), ctx.ptr)
+
+
+def hs_set_optimizer(ctx: Context, momentum: float, weight_decay: float):
+    _check(_lib.hs_set_optimizer(ctx.ptr, float(momentum), float(weight_decay)), ctx.ptr)
+
+
+def hs_optimizer_state(ctx: Context, buf, save: bool, stream=None):
+    _check(_lib.hs_optimizer_state(ctx.ptr, c_void_p(buf.data_ptr()), 1 if save else 0,
+                                   c_void_p(_stream_ptr(stream))), ctx.ptr)
+
+
+def hs_cosine_lr(eta0: float, eta_min: float, t: int, T: int) -> float:
+    return _lib.hs_cosine_lr(float(eta0), float(eta_min), int(t), int(T))
 
 
 def hs_set_profiling(ctx: Context, enable: bool = True):

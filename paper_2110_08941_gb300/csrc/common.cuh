@@ -52,9 +52,15 @@ void launch_bias_grad_bf16(const __nv_bfloat16* delta, int ld, int width, const 
 // theta[j] -= lr * sum_m w[m] * slabs[m*Ps + j]; shadow[j] = bf16(theta[j]); gdebug[j] = g (optional)
 // Works on any contiguous parameter range (pointers offset to its start, 16-byte aligned; slab m
 // of the range at slabs + m*Ps).  blocks_per_sm = 1 leaves room for a resident GEMM CTA.
+// The Section 5 recipe (momentum buffer at `buf`, offset like theta); null = plain SGD.
+struct UpdateRecipe {
+  float* buf;
+  float momentum, weight_decay;
+  int first;   // 1: the buffer starts as d (first step after the recipe was set)
+};
 void launch_reduce_update(float* theta, const float* slabs, int64_t Ps, int M, const float* d_w,
                           float lr, int64_t P, __nv_bfloat16* shadow, float* gdebug, int num_sms,
-                          cudaStream_t s, int blocks_per_sm = 4);
+                          cudaStream_t s, int blocks_per_sm = 4, const UpdateRecipe* recipe = nullptr);
 
 // ---------------------------------------------------------------- fp32 CUDA-core GEMM (check path)
 // C(m, n) = sum_k A(m, k) B(k, n) with A(m,k) = A[m*a_sm + k*a_sk], B(k,n) = B[k*b_sk + n*b_sn],

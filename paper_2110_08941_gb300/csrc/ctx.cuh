@@ -105,6 +105,12 @@ struct hs_ctx {
     return e;
   }
 
+  // training recipe of the paper's experiments (Section 5): momentum + weight decay in the update
+  bool opt_recipe = false;
+  float opt_momentum = 0.f, opt_weight_decay = 0.f;
+  float* d_mom = nullptr;      // momentum buffer [Ps]
+  bool mom_valid = false;      // false: the next step starts the buffer (b = d)
+
   // per-layer updates overlapped with the rest of the backward pass (bf16 MLP): a side stream that
   // waits for each layer's backward, and the event the caller's stream waits for at the end
   bool overlap_update = false;

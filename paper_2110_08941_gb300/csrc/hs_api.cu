@@ -263,7 +263,7 @@ void free_all(hs_ctx* c) {
   }
   for (void* p : c->d_act) f(p);
   f(c->d_logits); f(c->d_delta[0]); f(c->d_delta[1]); f(c->d_ce); f(c->d_lm); f(c->d_status);
-  f(c->d_slabs); f(c->d_shadow); f(c->d_gdebug); f(c->d_xstage); f(c->d_ystage);
+  f(c->d_slabs); f(c->d_shadow); f(c->d_gdebug); f(c->d_xstage); f(c->d_ystage); f(c->d_mom);
   if (c->h_status) cudaFreeHost(c->h_status);
   for (auto& r : c->pending) {
     cudaEventDestroy(r.a);
@@ -358,9 +358,11 @@ void update_layer_range(hs_ctx* c, float* params, int l, float lr, cudaStream_t 
   const int64_t start = c->layers[l].w_off;
   const int64_t end = (l + 1 < c->L) ? c->layers[l + 1].w_off : c->P;
   PhaseScope ph(c, HS_PHASE_UPDATE, s);
+  hs::UpdateRecipe r{c->opt_recipe ? c->d_mom + start : nullptr, c->opt_momentum, c->opt_weight_decay,
+                     c->mom_valid ? 0 : 1};
   hs::launch_reduce_update(params + start, c->d_slabs + start, c->Ps, c->M, c->d_w, lr, end - start,
                            c->d_shadow + start, c->debug ? c->d_gdebug + start : nullptr, c->num_sms, s,
-                           blocks_per_sm);
+                           blocks_per_sm, c->opt_recipe ? &r : nullptr);
   ph.launched();
 }
 
@@ -750,15 +752,17 @@ hs_status hs_step(hs_ctx* c, float* params, const void* x, const int32_t* y, con
   if (st != HS_OK) return st;
   if (!mlp_bf16) {
     PhaseScope ph(c, HS_PHASE_UPDATE, s);
+    hs::UpdateRecipe r{c->d_mom, c->opt_momentum, c->opt_weight_decay, c->mom_valid ? 0 : 1};
     hs::launch_reduce_update(params, c->d_slabs, c->Ps, c->M, c->d_w, lr, c->P,
                              c->precision == HS_BF16 ? c->d_shadow : nullptr, c->debug ? c->d_gdebug : nullptr,
-                             c->num_sms, s);
+                             c->num_sms, s, 4, c->opt_recipe ? &r : nullptr);
     ph.launched();
   }
   HS_CUDA(c, cudaGetLastError());
   c->shadow_src = params;
   c->shadow_valid = (c->precision == HS_BF16);
   c->gdebug_valid = c->debug;
+  if (c->opt_recipe) c->mom_valid = true;
   if (loss_out) {
     HS_CUDA(c, cudaMemcpyAsync(c->h_status, c->d_status, sizeof(DevStatus), cudaMemcpyDeviceToHost, s));
     HS_CUDA(c, cudaStreamSynchronize(s));
@@ -804,6 +808,48 @@ hs_status hs_read_profile(hs_ctx* c, double* ms_out, int64_t* launches_out) {
   for (int i = 0; i < HS_PHASE_COUNT; ++i) c->launches[i] = 0;
   if (first != cudaSuccess) return cuda_fail(c, first, "reading profile events");
   return HS_OK;
+}
+
+hs_status hs_set_optimizer(hs_ctx* c, float momentum, float weight_decay) {
+  if (!c) return HS_ERR_INVALID_ARG;
+  c->err.clear();
+  if (!std::isfinite(momentum) || !std::isfinite(weight_decay) || momentum < 0.f || momentum >= 1.f ||
+      weight_decay < 0.f)
+    return fail(c, HS_ERR_INVALID_ARG, "momentum must be in [0, 1) and weight_decay >= 0");
+  if (momentum == 0.f && weight_decay == 0.f) {
+    c->opt_recipe = false;
+    return HS_OK;
+  }
+  if (!c->d_mom) {
+    hs_status r = dalloc(c, &c->d_mom, sizeof(float) * (size_t)c->Ps);
+    if (r != HS_OK) return r;
+  }
+  c->opt_recipe = true;
+  c->opt_momentum = momentum;
+  c->opt_weight_decay = weight_decay;
+  c->mom_valid = false;
+  return HS_OK;
+}
+
+hs_status hs_optimizer_state(hs_ctx* c, float* buf_dev, int32_t save, void* stream) {
+  if (!c || !buf_dev) return c ? fail(c, HS_ERR_INVALID_ARG, "buf_dev is NULL") : HS_ERR_INVALID_ARG;
+  c->err.clear();
+  if (!c->opt_recipe || !c->d_mom) return fail(c, HS_ERR_INVALID_ARG, "no optimizer state: call hs_set_optimizer first");
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (save) {
+    if (!c->mom_valid) return fail(c, HS_ERR_INVALID_ARG, "the momentum buffer has not been started yet");
+    HS_CUDA(c, cudaMemcpyAsync(buf_dev, c->d_mom, sizeof(float) * c->P, cudaMemcpyDeviceToDevice, s));
+  } else {
+    HS_CUDA(c, cudaMemcpyAsync(c->d_mom, buf_dev, sizeof(float) * c->P, cudaMemcpyDeviceToDevice, s));
+    c->mom_valid = true;
+  }
+  return HS_OK;
+}
+
+double hs_cosine_lr(double eta0, double eta_min, int64_t t, int64_t T) {
+  if (T <= 0) return eta0;
+  if (t > T) t = T;
+  return eta_min + (eta0 - eta_min) * (1.0 + std::cos(M_PI * (double)t / (double)T)) / 2.0;
 }
 
 hs_status hs_set_debug(hs_ctx* c, int32_t enable) {

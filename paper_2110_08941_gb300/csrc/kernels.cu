@@ -274,10 +274,22 @@ void launch_bias_grad(const void* delta, bool delta_bf16, int ld, int width, con
 // ------------------------------------------------------------------ fused reduce + SGD update
 // Section 1: g = sum_m w_m g^m (w_m = 1/M; Section 4.2: compute-power weights), then
 // theta <- theta - lr * g.  One HBM pass: M slab reads + theta read, theta + bf16 shadow writes.
+// kRecipe: the Section 5 training recipe on top of g: d = g + wd*theta, b = d (first step) or
+// mu*b + d, theta <- theta - lr*b, with b kept in `mbuf` (one more read and write per parameter).
+template <bool kRecipe>
+__device__ __forceinline__ float apply_update(float t, float g, float lr, float* mb, float mu, float wd, int first) {
+  if (!kRecipe) return fmaf(-lr, g, t);
+  const float d = fmaf(wd, t, g);
+  const float b = first ? d : fmaf(mu, *mb, d);
+  *mb = b;
+  return fmaf(-lr, b, t);
+}
+
+template <bool kRecipe>
 __global__ void __launch_bounds__(512) reduce_update_kernel(
     float* __restrict__ theta, const float* __restrict__ slabs, int64_t Ps, int M,
     const float* __restrict__ w, float lr, int64_t P, __nv_bfloat16* __restrict__ shadow,
-    float* __restrict__ gdebug) {
+    float* __restrict__ gdebug, float* __restrict__ mbuf, float mu, float wd, int first) {
   // The weights stay in global memory (read through the read-only cache): no shared memory, so
   // blocks of this kernel can share an SM with a resident tensor-core GEMM CTA.
   const float* __restrict__ sw = w;
@@ -310,10 +322,19 @@ __global__ void __launch_bounds__(512) reduce_update_kernel(
       acc.w = fmaf(wm, g.w, acc.w);
     }
     float4 t = reinterpret_cast<float4*>(theta)[v];
-    t.x = fmaf(-lr, acc.x, t.x);
-    t.y = fmaf(-lr, acc.y, t.y);
-    t.z = fmaf(-lr, acc.z, t.z);
-    t.w = fmaf(-lr, acc.w, t.w);
+    if (kRecipe) {
+      float4 b = first ? make_float4(0.f, 0.f, 0.f, 0.f) : reinterpret_cast<const float4*>(mbuf)[v];
+      t.x = apply_update<true>(t.x, acc.x, lr, &b.x, mu, wd, first);
+      t.y = apply_update<true>(t.y, acc.y, lr, &b.y, mu, wd, first);
+      t.z = apply_update<true>(t.z, acc.z, lr, &b.z, mu, wd, first);
+      t.w = apply_update<true>(t.w, acc.w, lr, &b.w, mu, wd, first);
+      reinterpret_cast<float4*>(mbuf)[v] = b;
+    } else {
+      t.x = fmaf(-lr, acc.x, t.x);
+      t.y = fmaf(-lr, acc.y, t.y);
+      t.z = fmaf(-lr, acc.z, t.z);
+      t.w = fmaf(-lr, acc.w, t.w);
+    }
     reinterpret_cast<float4*>(theta)[v] = t;
     if (shadow) {
       __nv_bfloat162 lo = __floats2bfloat162_rn(t.x, t.y);
@@ -328,7 +349,7 @@ __global__ void __launch_bounds__(512) reduce_update_kernel(
   for (int64_t j = nvec * 4 + (int64_t)blockIdx.x * blockDim.x + threadIdx.x; j < P; j += stride) {
     float acc = 0.f;
     for (int m = 0; m < M; ++m) acc = fmaf(__ldg(sw + m), slabs[(int64_t)m * Ps + j], acc);
-    const float t = fmaf(-lr, acc, theta[j]);
+    const float t = apply_update<kRecipe>(theta[j], acc, lr, kRecipe ? mbuf + j : nullptr, mu, wd, first);
     theta[j] = t;
     if (shadow) shadow[j] = __float2bfloat16_rn(t);
     if (gdebug) gdebug[j] = acc;
@@ -337,13 +358,19 @@ __global__ void __launch_bounds__(512) reduce_update_kernel(
 
 void launch_reduce_update(float* theta, const float* slabs, int64_t Ps, int M, const float* d_w,
                           float lr, int64_t P, __nv_bfloat16* shadow, float* gdebug, int num_sms,
-                          cudaStream_t s, int blocks_per_sm) {
+                          cudaStream_t s, int blocks_per_sm, const UpdateRecipe* recipe) {
   const int threads = 512;
   int64_t blocks = (P / 4 + threads - 1) / threads;
   const int64_t cap = (int64_t)num_sms * blocks_per_sm;
   if (blocks > cap) blocks = cap;
   if (blocks < 1) blocks = 1;
-  reduce_update_kernel<<<(int)blocks, threads, 0, s>>>(theta, slabs, Ps, M, d_w, lr, P, shadow, gdebug);
+  if (recipe && recipe->buf)
+    reduce_update_kernel<true><<<(int)blocks, threads, 0, s>>>(theta, slabs, Ps, M, d_w, lr, P, shadow, gdebug,
+                                                               recipe->buf, recipe->momentum, recipe->weight_decay,
+                                                               recipe->first);
+  else
+    reduce_update_kernel<false><<<(int)blocks, threads, 0, s>>>(theta, slabs, Ps, M, d_w, lr, P, shadow, gdebug,
+                                                                nullptr, 0.f, 0.f, 0);
 }
 
 }  // namespace hs

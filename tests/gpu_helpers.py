@@ -22,12 +22,18 @@ def grad_fn(arch):
     return mlp.worker_loss_grad if arch == synth.MLP else cnn.worker_loss_grad
 
 
+def _lr_at(lr, t):
+    return lr(t) if callable(lr) else lr
+
+
 def run_library(arch, dims, M, N, weights, x, y, theta0, lr, steps, precision, sync, repartition=None,
-                keep_slabs=False):
+                keep_slabs=False, recipe=None):
     """Returns dict(theta, losses, g_first, slabs_first, counts, index_map)."""
     ctx = hs.hs_init(arch, dims, M, N, compute_weights=weights, precision=precision, sync=sync)
     try:
         hs.hs_set_debug(ctx, True)
+        if recipe is not None:
+            hs.hs_set_optimizer(ctx, *recipe)
         params = torch.tensor(theta0, device="cuda")
         xd = torch.from_numpy(np.ascontiguousarray(x)).cuda()
         yd = torch.from_numpy(np.ascontiguousarray(y)).cuda()
@@ -39,7 +45,7 @@ def run_library(arch, dims, M, N, weights, x, y, theta0, lr, steps, precision, s
                 part = hs.hs_partition(ctx, repartition[t], index_map_out=im)
                 out["counts"].append(list(part.counts))
                 out["index_maps"].append(im.cpu().numpy().copy())
-            out["losses"].append(hs.hs_step(ctx, params, xd, yd, part, lr))
+            out["losses"].append(hs.hs_step(ctx, params, xd, yd, part, _lr_at(lr, t)))
             if t == 0:
                 g = torch.empty(ctx.P, device="cuda")
                 slabs = torch.empty(M, ctx.P, device="cuda") if keep_slabs else None
@@ -62,7 +68,7 @@ def decide_for(precision):
 
 
 def run_oracle(arch, dims, M, N, weights, x, y, theta0, lr, steps, sync, repartition=None, keep_slabs=False,
-               decide=None):
+               decide=None, recipe=None):
     fn = grad_fn(arch)
     kw = {} if decide is None else {"decide": decide}
     mode = SYNC_TO_ORACLE[sync]
@@ -70,13 +76,19 @@ def run_oracle(arch, dims, M, N, weights, x, y, theta0, lr, steps, sync, reparti
     sizes = P.partition_sizes(cp, N)
     th = np.asarray(theta0, dtype=np.float64)
     out = dict(losses=[], counts=[list(sizes)])
+    buf = None
     for t in range(steps):
         if repartition is not None and t > 0 and t in repartition:
             cp = list(repartition[t])
             sizes = P.partition_sizes(cp, N)
             out["counts"].append(list(sizes))
-        th, loss, g, slabs, wl = sgd.step(fn, th, dims, x, y, sizes, lr, mode, keep_slabs=(keep_slabs and t == 0),
-                                          cp=cp, **kw)
+        lr_t = _lr_at(lr, t)
+        th_next, loss, g, slabs, wl = sgd.step(fn, th, dims, x, y, sizes, lr_t, mode,
+                                               keep_slabs=(keep_slabs and t == 0), cp=cp, **kw)
+        if recipe is None:
+            th = th_next
+        else:
+            th, buf = sgd.momentum_update(th, g, buf if t > 0 else None, lr_t, recipe[0], recipe[1])
         out["losses"].append(loss)
         if t == 0:
             out["g_first"] = g

@@ -104,3 +104,11 @@ def test_status_strings():
     lib.hs_status_string.restype = ctypes.c_char_p
     assert lib.hs_status_string(0) == b"HS_OK"
     assert lib.hs_status_string(5) == b"HS_ERR_DEVICE_CHECK"
+
+
+def test_cosine_lr_matches_oracle():
+    from oracle import sgd
+    for t in range(0, 120, 7):
+        assert hs.hs_cosine_lr(0.1, 0.001, t, 100) == pytest.approx(sgd.cosine_lr(0.1, 0.001, min(t, 100), 100),
+                                                                    rel=0, abs=1e-15)
+    assert hs.hs_cosine_lr(0.1, 0.0, 5, 0) == 0.1

@@ -199,3 +199,18 @@ def test_cnn_edge_shapes(dims, N, M, weights, precision):
         lib = run_library(synth.CNN, dims, M, N, weights, x, y, theta0, 0.05, 10, precision, sync)
         orc = run_oracle(synth.CNN, dims, M, N, weights, x, y, theta0, 0.05, 10, sync, decide=decide_for(precision))
         _check(lib, orc, theta0.astype(np.float64), precision, 10)
+
+
+# ------------------------------------------------------------------ the Section 5 training recipe
+@pytest.mark.parametrize("name,precision", [(synth.CFG2, hs.HS_BF16), (synth.CFG2, hs.HS_FP32_CHECK),
+                                            (synth.CFG4, hs.HS_BF16), (synth.CFG1, hs.HS_BF16)])
+def test_momentum_weight_decay_cosine_lr(name, precision):
+    """SGD momentum 0.9, weight decay 5e-4, cosine-annealed learning rate over the 10 steps."""
+    wl, x, y, theta0, w = _inputs(name)
+    recipe = (0.9, 5e-4)
+    sched = lambda t: hs.hs_cosine_lr(wl.lr, 0.0, t, 10)   # noqa: E731
+    lib = run_library(wl.arch, wl.dims, wl.workers, wl.global_batch, w, x, y, theta0, sched, 10, precision,
+                      hs.HS_SYNC_CP_WEIGHTED, recipe=recipe)
+    orc = run_oracle(wl.arch, wl.dims, wl.workers, wl.global_batch, w, x, y, theta0, sched, 10,
+                     hs.HS_SYNC_CP_WEIGHTED, decide=decide_for(precision), recipe=recipe)
+    _check(lib, orc, theta0.astype(np.float64), precision, 10)

@@ -161,3 +161,43 @@ def test_headline_workload_sampled_parity():
         assert np.all(np.abs(th1.astype(np.float64) - want) <= 2 * ulp + 1e-12)
     finally:
         ctx.close()
+
+
+def test_checkpoint_resume_with_momentum_is_bit_exact():
+    """As above with the Section 5 recipe: the momentum buffer is saved and restored with theta."""
+    wl = synth.WORKLOADS[synth.CFG2]
+    x, y = synth.make_batch(wl)
+    theta0 = synth.make_params(wl)
+    w = synth.initial_weights(wl)
+    xd, yd = torch.from_numpy(x).cuda(), torch.from_numpy(y).cuda()
+
+    def fresh():
+        c = hs.hs_init(wl.arch, wl.dims, wl.workers, wl.global_batch, compute_weights=w)
+        hs.hs_set_optimizer(c, 0.9, 5e-4)
+        return c
+
+    c1 = fresh()
+    p1 = torch.tensor(theta0, device="cuda")
+    for t in range(10):
+        hs.hs_step(c1, p1, xd, yd, None, hs.hs_cosine_lr(wl.lr, 0.0, t, 10), want_loss=False)
+    torch.cuda.synchronize()
+    c1.close()
+
+    c2 = fresh()
+    p2 = torch.tensor(theta0, device="cuda")
+    for t in range(5):
+        hs.hs_step(c2, p2, xd, yd, None, hs.hs_cosine_lr(wl.lr, 0.0, t, 10), want_loss=False)
+    mom = torch.empty(c2.P, device="cuda")
+    hs.hs_optimizer_state(c2, mom, True)
+    torch.cuda.synchronize()
+    saved_theta, saved_mom = p2.cpu().clone(), mom.cpu().clone()
+    c2.close()
+
+    c3 = fresh()
+    p3 = saved_theta.cuda()
+    hs.hs_optimizer_state(c3, saved_mom.cuda(), False)
+    for t in range(5, 10):
+        hs.hs_step(c3, p3, xd, yd, None, hs.hs_cosine_lr(wl.lr, 0.0, t, 10), want_loss=False)
+    torch.cuda.synchronize()
+    c3.close()
+    assert torch.equal(p1, p3)

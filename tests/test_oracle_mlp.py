@@ -214,3 +214,33 @@ def test_bf16_decisions_differ_only_near_kinks():
     _, g0 = mlp.worker_loss_grad(theta, dims, x[:50], y := rng.integers(0, 10, 50))
     _, g1 = mlp.worker_loss_grad(theta, dims, x[:50], y, decide=mlp.round_bf16)
     assert np.linalg.norm(g1 - g0) < 0.2 * np.linalg.norm(g0)
+
+
+def test_momentum_weight_decay_matches_torch_sgd():
+    # Section 5: SGD with momentum 0.9 and weight decay 5e-4, against torch.optim.SGD in fp64.
+    dims = (9, 6, 4)
+    theta, x, y = _tiny(dims, 24, 11)
+    sizes = P.partition_sizes([1, 2, 5], 24)
+    lr, mu, wd = 0.2, 0.9, 5e-4
+    t = torch.tensor(theta, dtype=torch.float64, requires_grad=True)
+    opt = torch.optim.SGD([t], lr=lr, momentum=mu, weight_decay=wd)
+    th, buf = theta.copy(), None
+    for _ in range(5):
+        opt.zero_grad()
+        tt, loss = _torch_loss(t.detach().numpy(), dims, x, y)
+        loss.backward()
+        t.grad = tt.grad.clone()
+        opt.step()
+        _, _, g, _, _ = sgd.step(mlp.worker_loss_grad, th, dims, x, y, sizes, 0.0, sgd.SYNC_CP_WEIGHTED)
+        th, buf = sgd.momentum_update(th, g, buf, lr, mu, wd)
+    assert np.allclose(th, t.detach().numpy(), rtol=0, atol=1e-12)
+
+
+def test_cosine_lr_matches_torch_scheduler():
+    p = torch.nn.Parameter(torch.zeros(1))
+    opt = torch.optim.SGD([p], lr=0.1)
+    sched = torch.optim.lr_scheduler.CosineAnnealingLR(opt, T_max=50, eta_min=0.001)
+    for step in range(50):
+        assert abs(opt.param_groups[0]["lr"] - sgd.cosine_lr(0.1, 0.001, step, 50)) < 1e-12
+        opt.step()
+        sched.step()
