@@ -131,6 +131,17 @@ hs_status hs_init(const hs_model_desc* model, int32_t M, const double* compute_w
 hs_status hs_partition(hs_ctx* ctx, const double* measured_throughputs, int32_t* counts_out,
                        int32_t* index_map_out, void* stream, hs_partition_t* out);
 
+/* Where the compute power handed to Algorithm 1 comes from (Section 4.1: "just the previous
+ * epoch or ... a history of epochs").  Each hs_partition call with measured_throughputs c adds c
+ * to the history, and the partition is sized from the estimate e:
+ *   HS_CP_LAST   e = c (default; param ignored)
+ *   HS_CP_EMA    e = param * c + (1 - param) * e_prev, param in (0, 1]; the first c initialises e
+ *   HS_CP_WINDOW e = mean of the last `param` measurements (integer in [1, 1024]), summed oldest first
+ * fp64 per worker in these operation orders.  Changing the mode clears the history.
+ * Errors: HS_ERR_INVALID_ARG for an unknown mode or a parameter out of range. */
+typedef enum { HS_CP_LAST = 0, HS_CP_EMA = 1, HS_CP_WINDOW = 2 } hs_cp_history;
+hs_status hs_set_cp_history(hs_ctx* ctx, int32_t mode, double param);
+
 /* One synchronous SGD step (Section 1; Eq. 1; Section 4.2 for the weights).
  *   params: device fp32 [P], updated in place: theta <- theta - lr * sum_m w_m G_m,
  *           where G_m is the gradient of worker m's mean cross-entropy over its segment.

@@ -106,3 +106,39 @@ def dynamic_partitioning(t: int, mean_times: Sequence[float], sizes: Sequence[in
     if t == 0:
         return even_sizes(m, n)
     return partition_sizes(compute_power(sizes, mean_times), n)
+
+
+class CPHistory:
+    """Compute-power estimate from a history of measurements (Section 4.1: the CPs may come from
+    the last epoch only, or from a history of epochs).  Reading: mode "last" uses the newest
+    measurement; "ema" keeps e = a * c + (1 - a) * e (the first measurement initialises e);
+    "window" averages the last k measurements (summed oldest first, then divided by their count).
+    fp64, per worker, in exactly these operation orders."""
+
+    def __init__(self, mode: str = "last", param: float = 0.0):
+        self.mode, self.param = mode, float(param)
+        self.ema = None
+        self.window: List[List[float]] = []
+
+    def update(self, cp: Sequence[float]) -> List[float]:
+        cp = [float(c) for c in cp]
+        if self.mode == "last":
+            return cp
+        if self.mode == "ema":
+            a = self.param
+            if self.ema is None:
+                self.ema = list(cp)
+            else:
+                self.ema = [a * c + (1.0 - a) * e for c, e in zip(cp, self.ema)]
+            return list(self.ema)
+        k = int(self.param)
+        self.window.append(cp)
+        if len(self.window) > k:
+            self.window.pop(0)
+        out = []
+        for m in range(len(cp)):
+            acc = 0.0
+            for row in self.window:
+                acc = acc + row[m]
+            out.append(acc / float(len(self.window)))
+        return out

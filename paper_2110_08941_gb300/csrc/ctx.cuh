@@ -105,6 +105,12 @@ struct hs_ctx {
     return e;
   }
 
+  // compute-power history (Section 4.1): 0 = last measurement, 1 = EMA, 2 = window mean
+  int cp_hist_mode = 0;
+  double cp_hist_param = 0.0;
+  std::vector<double> cp_ema;
+  std::vector<std::vector<double>> cp_window;
+
   // training recipe of the paper's experiments (Section 5): momentum + weight decay in the update
   bool opt_recipe = false;
   float opt_momentum = 0.f, opt_weight_decay = 0.f;

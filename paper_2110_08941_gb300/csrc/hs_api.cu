@@ -679,10 +679,32 @@ hs_status hs_partition(hs_ctx* c, const double* measured_throughputs, int32_t* c
   c->err.clear();
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   if (measured_throughputs) {
+    for (int m = 0; m < c->M; ++m)
+      if (!std::isfinite(measured_throughputs[m]) || !(measured_throughputs[m] > 0.0))
+        return fail(c, HS_ERR_INVALID_ARG, "measured_throughputs: compute power must be finite and > 0");
+    // the estimate handed to Algorithm 1: the last measurement, or a history of them (Section 4.1)
+    std::vector<double> est(measured_throughputs, measured_throughputs + c->M);
+    if (c->cp_hist_mode == 1) {
+      const double a = c->cp_hist_param;
+      if (c->cp_ema.empty()) {
+        c->cp_ema = est;
+      } else {
+        for (int m = 0; m < c->M; ++m) c->cp_ema[m] = a * est[m] + (1.0 - a) * c->cp_ema[m];
+      }
+      est = c->cp_ema;
+    } else if (c->cp_hist_mode == 2) {
+      c->cp_window.push_back(est);
+      if ((int)c->cp_window.size() > (int)c->cp_hist_param) c->cp_window.erase(c->cp_window.begin());
+      for (int m = 0; m < c->M; ++m) {
+        double acc = 0.0;
+        for (const auto& row : c->cp_window) acc = acc + row[m];
+        est[m] = acc / (double)c->cp_window.size();
+      }
+    }
     std::vector<int32_t> sizes(c->M);
     std::vector<double> cpn(c->M);
     const char* why = nullptr;
-    hs_status st = hs::partition_sizes_impl(c->M, c->N, measured_throughputs, sizes.data(), cpn.data(), &why);
+    hs_status st = hs::partition_sizes_impl(c->M, c->N, est.data(), sizes.data(), cpn.data(), &why);
     if (st != HS_OK) return fail(c, st, std::string("measured_throughputs: ") + why);
     st = apply_partition(c, sizes, cpn, index_map_out, s);
     if (st != HS_OK) return st;
@@ -807,6 +829,22 @@ hs_status hs_read_profile(hs_ctx* c, double* ms_out, int64_t* launches_out) {
     for (int i = 0; i < HS_PHASE_COUNT; ++i) launches_out[i] = c->launches[i];
   for (int i = 0; i < HS_PHASE_COUNT; ++i) c->launches[i] = 0;
   if (first != cudaSuccess) return cuda_fail(c, first, "reading profile events");
+  return HS_OK;
+}
+
+hs_status hs_set_cp_history(hs_ctx* c, int32_t mode, double param) {
+  if (!c) return HS_ERR_INVALID_ARG;
+  c->err.clear();
+  if (mode == HS_CP_EMA && !(param > 0.0 && param <= 1.0))
+    return fail(c, HS_ERR_INVALID_ARG, "EMA weight must be in (0, 1]");
+  if (mode == HS_CP_WINDOW && !(param >= 1.0 && param <= 1024.0 && param == (double)(int)param))
+    return fail(c, HS_ERR_INVALID_ARG, "window length must be an integer in [1, 1024]");
+  if (mode != HS_CP_LAST && mode != HS_CP_EMA && mode != HS_CP_WINDOW)
+    return fail(c, HS_ERR_INVALID_ARG, "unknown compute-power history mode");
+  c->cp_hist_mode = mode;
+  c->cp_hist_param = param;
+  c->cp_ema.clear();
+  c->cp_window.clear();
   return HS_OK;
 }
 

@@ -201,3 +201,27 @@ def test_checkpoint_resume_with_momentum_is_bit_exact():
     torch.cuda.synchronize()
     c3.close()
     assert torch.equal(p1, p3)
+
+
+@pytest.mark.parametrize("mode,param,name", [(hs.HS_CP_LAST, 0.0, "last"), (hs.HS_CP_EMA, 0.3, "ema"),
+                                             (hs.HS_CP_WINDOW, 3, "window")])
+def test_cp_history_partitions_bit_exact(mode, param, name):
+    """Section 4.1's history of compute-power measurements: a sequence of drifting throughputs gives
+    the same partitions and index maps as the oracle's estimator followed by its partition rule."""
+    wl = synth.WORKLOADS[synth.CFG3]
+    ctx = hs.hs_init(wl.arch, wl.dims, wl.workers, wl.global_batch)
+    try:
+        hs.hs_set_cp_history(ctx, mode, param)
+        est = P.CPHistory(name, param)
+        speeds = synth.drift_walk(wl.workers, 60, 4)
+        im = torch.empty(wl.global_batch, dtype=torch.int32, device="cuda")
+        for t in range(10, 61, 10):
+            tp = list(synth.window_throughputs(speeds[t - 10:t]))
+            part = hs.hs_partition(ctx, tp, index_map_out=im)
+            want = P.partition_sizes(est.update(tp), wl.global_batch)
+            assert part.counts == want, t
+            assert np.array_equal(im.cpu().numpy(), np.asarray(P.index_map(want), dtype=np.int32))
+        with pytest.raises(hs.HsError):
+            hs.hs_set_cp_history(ctx, hs.HS_CP_EMA, 1.5)
+    finally:
+        ctx.close()

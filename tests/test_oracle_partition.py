@@ -152,3 +152,20 @@ def test_offsets_and_index_map():
 def test_invalid_inputs_raise(cp, n):
     with pytest.raises(ValueError):
         P.partition_sizes(cp, n)
+
+
+def test_cp_history_closed_forms():
+    seq = [[1.0, 2.0], [3.0, 2.0], [5.0, 8.0], [7.0, 2.0]]
+    last = P.CPHistory("last")
+    assert [last.update(c) for c in seq][-1] == [7.0, 2.0]
+    ema = P.CPHistory("ema", 0.5)
+    outs = [ema.update(c) for c in seq]
+    assert outs[0] == [1.0, 2.0] and outs[1] == [2.0, 2.0] and outs[2] == [3.5, 5.0] and outs[3] == [5.25, 3.5]
+    win = P.CPHistory("window", 2)
+    outs = [win.update(c) for c in seq]
+    assert outs[0] == [1.0, 2.0] and outs[1] == [2.0, 2.0] and outs[2] == [4.0, 5.0] and outs[3] == [6.0, 5.0]
+    # a constant history is its own estimate, so the partition equals the one-shot rule
+    for h in (P.CPHistory("ema", 0.3), P.CPHistory("window", 3)):
+        for _ in range(5):
+            est = h.update([1.0, 3.0])
+        assert P.partition_sizes(est, 128) == [32, 96]
