@@ -323,6 +323,26 @@ def run_ours(args, wl, rank, world, local_rank):
     ms = max_over_ranks(ms)
     loss = hs.hs_step(ctx, params, xd, yd, part, 0.0, stream=stream, want_loss=True)   # finite-loss check
 
+    # the slab-free formulation of the same step (opt-in variant), timed the same way
+    fused = None
+    if wl.arch == synth.MLP and precision == hs.HS_BF16:
+        hs.hs_set_fused_sync(ctx, True)
+        for _ in range(args.warmup):
+            hs.hs_step(ctx, params, xd, yd, part, wl.lr, stream=stream, want_loss=False)
+        barrier()
+        torch.cuda.synchronize()
+        f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        f0.record(stream)
+        for _ in range(args.steps):
+            hs.hs_step(ctx, params, xd, yd, part, wl.lr, stream=stream, want_loss=False)
+        f1.record(stream)
+        torch.cuda.synchronize()
+        fms = max_over_ranks(f0.elapsed_time(f1))
+        hs.hs_set_fused_sync(ctx, False)
+        fused = {"ms_per_step": fms / args.steps, "value": world * wl.global_batch * args.steps / (fms * 1e-3),
+                 "unit": UNIT, "what": "slab-free formulation: worker weights folded into the loss-gradient "
+                                       "scale, one all-rows weight-gradient product, update of one gradient"}
+
     # end to end through the public API: host (pinned) inputs, loss read back every step
     xh = torch.from_numpy(x).pin_memory()
     yh = torch.from_numpy(y).pin_memory()
@@ -393,6 +413,7 @@ def run_ours(args, wl, rank, world, local_rank):
                     "h2d_bytes_per_step": int(x.nbytes + y.nbytes), "d2h_bytes_per_step": 12},
             "clocks": clk,
             "straggler_sim": straggler_simulation(),
+            "fused_sync_variant": fused,
             "loss_after": loss,
         }
         print(json.dumps(out), flush=True)

@@ -131,6 +131,15 @@ hs_status hs_init(const hs_model_desc* model, int32_t M, const double* compute_w
 hs_status hs_partition(hs_ctx* ctx, const double* measured_throughputs, int32_t* counts_out,
                        int32_t* index_map_out, void* stream, hs_partition_t* out);
 
+/* Slab-free formulation of the same step (MLP only; opt-in, off by default).  Every later
+ * backward signal is linear in the loss gradient, so scaling sample i's loss gradient by
+ * w_{m(i)} / n_{m(i)} instead of 1 / n_{m(i)} makes one weight-gradient product over all N rows
+ * equal to sum_m w_m G_m (Eq. 1 with Section 1's / Section 4.2's weights).  No per-worker slabs
+ * are written and the update reads one gradient instead of M: same parameters up to rounding
+ * order, fewer bytes.  hs_debug_grads then offers g but no slabs (HS_ERR_INVALID_ARG).
+ * Errors: HS_ERR_UNSUPPORTED for the CNN. */
+hs_status hs_set_fused_sync(hs_ctx* ctx, int32_t enable);
+
 /* Where the compute power handed to Algorithm 1 comes from (Section 4.1: "just the previous
  * epoch or ... a history of epochs").  Each hs_partition call with measured_throughputs c adds c
  * to the history, and the partition is sized from the estimate e:

@@ -27,7 +27,7 @@ EXPORTED = ("hs_partition_sizes", "hs_param_count", "hs_init", "hs_partition", "
             "hs_set_debug", "hs_debug_grads", "hs_worker_losses", "hs_destroy", "hs_status_string",
             "hs_last_error", "hs_last_init_error", "hs_debug_gemm_bf16", "hs_set_profiling", "hs_read_profile",
             "hs_partition_noalloc", "hs_set_optimizer", "hs_optimizer_state", "hs_cosine_lr",
-            "hs_set_cp_history")
+            "hs_set_cp_history", "hs_set_fused_sync")
 HS_CP_LAST, HS_CP_EMA, HS_CP_WINDOW = 0, 1, 2
 PHASES = ("cast", "forward", "loss", "wgrad", "biasgrad", "dgrad", "update")
 
@@ -68,6 +68,7 @@ def _load() -> ctypes.CDLL:
         "hs_set_profiling": (S, [c_void_p, c_int32]),
         "hs_set_optimizer": (S, [c_void_p, c_float, c_float]),
         "hs_set_cp_history": (S, [c_void_p, c_int32, c_double]),
+        "hs_set_fused_sync": (S, [c_void_p, c_int32]),
         "hs_optimizer_state": (S, [c_void_p, c_void_p, c_int32, c_void_p]),
         "hs_cosine_lr": (c_double, [c_double, c_double, c_int64, c_int64]),
         "hs_read_profile": (S, [c_void_p, POINTER(c_double), POINTER(c_int64)]),
@@ -226,6 +227,10 @@ def hs_sync_params(ctx: Context, params, stream=None):
 
 def hs_set_debug(ctx: Context, enable: bool = True):
     _check(_lib.hs_set_debug(ctx.ptr, 1 if enable else 0), ctx.ptr)
+
+
+def hs_set_fused_sync(ctx: Context, enable: bool = True):
+    _check(_lib.hs_set_fused_sync(ctx.ptr, 1 if enable else 0), ctx.ptr)
 
 
 def hs_set_cp_history(ctx: Context, mode: int, param: float = 0.0):

@@ -33,6 +33,9 @@ void set_init_error(const char* msg);
 void launch_cast_f32_bf16(const float* x, __nv_bfloat16* y, int64_t n, cudaStream_t s);
 void launch_partition_scatter(const int32_t* d_offsets, int M, int N, int32_t* index_map,
                               float* scale, int32_t* index_map_out, cudaStream_t s);
+// out[i] = w[index_map[i]] * scale[i]
+void launch_scale_by_weight(const int32_t* index_map, const float* scale, const float* w, int N, float* out,
+                            cudaStream_t s);
 // logits [N, ldl] fp32 -> ce[N], delta [N, ldd] (bf16 if delta_bf16 else fp32, columns >= C zeroed)
 void launch_softmax_xent(const float* logits, int ldl, const int32_t* y, const float* scale, int N,
                          int C, void* delta, int ldd, bool delta_bf16, float* ce, DevStatus* st,

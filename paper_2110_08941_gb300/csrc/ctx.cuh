@@ -105,6 +105,15 @@ struct hs_ctx {
     return e;
   }
 
+  // slab-free formulation (opt-in): worker weights folded into the per-sample loss-gradient scale,
+  // one weight-gradient product over all rows into slab 0, and the update with a single "worker"
+  bool fused_sync = false;
+  float* d_scale_fused = nullptr;      // [N] w_{m(i)} / n_{m(i)}
+  int32_t* d_all_off = nullptr;        // {0, N}
+  float* d_w_one = nullptr;            // {1.0f}
+  hs::ChunkTable all_rows;             // bias-gradient chunks over all rows, one worker
+  std::vector<hs::TcGemmParams> tc_wgrad_fused;   // per layer, one group spanning all rows
+
   // compute-power history (Section 4.1): 0 = last measurement, 1 = EMA, 2 = window mean
   int cp_hist_mode = 0;
   double cp_hist_param = 0.0;

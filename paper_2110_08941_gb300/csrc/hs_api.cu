@@ -114,6 +114,36 @@ hs_status build_tc_static(hs_ctx* c) {
   return HS_OK;
 }
 
+// The slab-free formulation's weight gradients: one group over all N rows into slab 0.
+hs_status build_tc_wgrad_fused(hs_ctx* c) {
+  const char* why = nullptr;
+  c->tc_wgrad_fused.assign(c->L, hs::TcGemmParams{});
+  for (int l = 0; l < c->L; ++l) {
+    const Layer& ly = c->layers[l];
+    const int ldd_delta = c->delta_ld(l);
+    const int out_cols = (l == c->L - 1) ? c->C : ly.out;
+    hs::TcGemmParams& w = c->tc_wgrad_fused[l];
+    std::memset(&w, 0, sizeof(w));
+    hs::TcOperand a{reinterpret_cast<const __nv_bfloat16*>(c->delta_buf(l)), c->N, out_cols, ldd_delta};
+    hs::TcOperand b{reinterpret_cast<const __nv_bfloat16*>(c->d_act[l]), c->N, ly.in, ly.in};
+    if (!hs::tc_make_mnmajor_map(&w.tmA[0], a, &why) || !hs::tc_make_mnmajor_map(&w.tmB[0], b, &why) ||
+        !hs::tc_make_store_map(&w.tmD[0], c->d_slabs + ly.w_off, true, out_cols, ly.in, ly.in, &why))
+      return fail(c, HS_ERR_CUDA, why);
+    w.num_kb[0] = (c->N + hs::kTcBK - 1) / hs::kTcBK;
+    w.groups = 1;
+    w.Mdim = out_cols;
+    w.Ndim = ly.in;
+    w.n_store = ly.in;
+    w.epi = hs::kTcEpiStoreF32;
+    w.a_mn = 1;
+    w.b_mn = 1;
+    w.D = c->d_slabs + ly.w_off;
+    w.ldd = ly.in;
+    w.st = c->d_status;
+  }
+  return HS_OK;
+}
+
 // Per-worker weight gradients depend on the segments, so they are rebuilt on repartition.
 hs_status build_tc_wgrad(hs_ctx* c) {
   const char* why = nullptr;
@@ -203,6 +233,10 @@ hs_status apply_partition(hs_ctx* c, const std::vector<int32_t>& sizes, const st
     hs::launch_partition_scatter(c->d_offsets, c->M, c->N, c->d_index_map, c->d_scale, index_map_out, s);
     HS_CUDA(c, cudaGetLastError());
   }
+  if (c->d_scale_fused) {
+    hs::launch_scale_by_weight(c->d_index_map, c->d_scale, c->d_w, c->N, c->d_scale_fused, s);
+    HS_CUDA(c, cudaGetLastError());
+  }
   // the host vectors above are pageable: make sure the copies consumed them before they change
   HS_CUDA(c, cudaStreamSynchronize(s));
   if (changed && c->arch == HS_MLP && c->precision == HS_BF16) {
@@ -255,6 +289,7 @@ void free_all(hs_ctx* c) {
   auto f = [](void* p) { if (p) cudaFree(p); };
   f(c->d_offsets); f(c->d_index_map); f(c->d_scale); f(c->d_w);
   f(c->d_bg_chunks); f(c->d_bg_chunk_begin); f(c->d_bg_partial);
+  f(c->d_scale_fused); f(c->d_all_off); f(c->d_w_one); f(c->all_rows.d_chunks); f(c->all_rows.d_begin);
   for (int k = 0; k < 3; ++k) { f(c->d_col[k]); f(c->d_cact[k]); f(c->d_dA[k]); }
   f(c->d_pooled); f(c->d_dpooled); f(c->d_dcol); f(c->d_w1p);
   for (int k = 0; k < 4; ++k) {
@@ -310,7 +345,8 @@ hs_status mlp_step_fp32(hs_ctx* c, float* params, const float* x, const int32_t*
   }
   {
     PhaseScope ph(c, HS_PHASE_LOSS, s);
-    hs::launch_softmax_xent(c->d_logits, c->Cp, y, c->d_scale, c->N, c->C, c->delta_buf(L - 1), c->Cp, false,
+    hs::launch_softmax_xent(c->d_logits, c->Cp, y, c->fused_sync ? c->d_scale_fused : c->d_scale, c->N, c->C,
+                            c->delta_buf(L - 1), c->Cp, false,
                             c->d_ce, c->d_status, s);
     hs::launch_loss_reduce(c->d_ce, c->d_offsets, c->M, c->d_w, c->d_lm, c->d_status, s);
     ph.launched(2);
@@ -329,13 +365,16 @@ hs_status mlp_step_fp32(hs_ctx* c, float* params, const float* x, const int32_t*
       w.C = c->d_slabs + ly.w_off; w.ldc = ly.in;
       w.Mdim = out_cols; w.Ndim = ly.in; w.Kdim = 0;
       w.epi = hs::kEpiStore;
-      w.k_offsets = c->d_offsets; w.groups = c->M; w.c_gstride = c->Ps;
+      w.k_offsets = c->fused_sync ? c->d_all_off : c->d_offsets;
+      w.groups = c->fused_sync ? 1 : c->M;
+      w.c_gstride = c->Ps;
       hs::launch_gemm_f32(w, s);
       ph.launched();
     }
     {
       PhaseScope ph(c, HS_PHASE_BIASGRAD, s);
-      hs::launch_bias_grad(delta, false, ldd, out_cols, c->d_offsets, c->M, c->d_slabs, c->Ps, ly.b_off, s);
+      hs::launch_bias_grad(delta, false, ldd, out_cols, c->fused_sync ? c->d_all_off : c->d_offsets,
+                           c->fused_sync ? 1 : c->M, c->d_slabs, c->Ps, ly.b_off, s);
       ph.launched();
     }
     if (l > 0) {
@@ -360,7 +399,8 @@ void update_layer_range(hs_ctx* c, float* params, int l, float lr, cudaStream_t 
   PhaseScope ph(c, HS_PHASE_UPDATE, s);
   hs::UpdateRecipe r{c->opt_recipe ? c->d_mom + start : nullptr, c->opt_momentum, c->opt_weight_decay,
                      c->mom_valid ? 0 : 1};
-  hs::launch_reduce_update(params + start, c->d_slabs + start, c->Ps, c->M, c->d_w, lr, end - start,
+  hs::launch_reduce_update(params + start, c->d_slabs + start, c->Ps, c->fused_sync ? 1 : c->M,
+                           c->fused_sync ? c->d_w_one : c->d_w, lr, end - start,
                            c->d_shadow + start, c->debug ? c->d_gdebug + start : nullptr, c->num_sms, s,
                            blocks_per_sm, c->opt_recipe ? &r : nullptr);
   ph.launched();
@@ -385,7 +425,8 @@ hs_status mlp_step_bf16(hs_ctx* c, float* params, const float* x, const int32_t*
   }
   {
     PhaseScope ph(c, HS_PHASE_LOSS, s);
-    hs::launch_softmax_xent(c->d_logits, c->Cp, y, c->d_scale, c->N, c->C, c->delta_buf(L - 1), c->Cp, true,
+    hs::launch_softmax_xent(c->d_logits, c->Cp, y, c->fused_sync ? c->d_scale_fused : c->d_scale, c->N, c->C,
+                            c->delta_buf(L - 1), c->Cp, true,
                             c->d_ce, c->d_status, s);
     hs::launch_loss_reduce(c->d_ce, c->d_offsets, c->M, c->d_w, c->d_lm, c->d_status, s);
     ph.launched(2);
@@ -394,17 +435,29 @@ hs_status mlp_step_bf16(hs_ctx* c, float* params, const float* x, const int32_t*
     const Layer& ly = c->layers[l];
     {
       PhaseScope ph(c, HS_PHASE_WGRAD, s);
-      for (const hs::TcGemmParams& w : c->tc_wgrad[l]) {
-        cudaError_t e = hs::launch_tc_gemm(w, c->num_sms, s);
+      if (c->fused_sync) {
+        cudaError_t e = hs::launch_tc_gemm(c->tc_wgrad_fused[l], c->num_sms, s);
         if (e != cudaSuccess) return cuda_fail(c, e, "weight-gradient GEMM launch");
         ph.launched();
+      } else {
+        for (const hs::TcGemmParams& w : c->tc_wgrad[l]) {
+          cudaError_t e = hs::launch_tc_gemm(w, c->num_sms, s);
+          if (e != cudaSuccess) return cuda_fail(c, e, "weight-gradient GEMM launch");
+          ph.launched();
+        }
       }
     }
     {
       PhaseScope ph(c, HS_PHASE_BIASGRAD, s);
       const int out_cols = (l == L - 1) ? c->C : ly.out;
+      const hs::ChunkTable* ct = nullptr;
+      hs::ChunkTable per_worker;
+      per_worker.d_chunks = c->d_bg_chunks;
+      per_worker.d_begin = c->d_bg_chunk_begin;
+      per_worker.n = c->n_bg_chunks;
+      ct = c->fused_sync ? &c->all_rows : &per_worker;
       hs::launch_bias_grad_bf16(reinterpret_cast<const __nv_bfloat16*>(c->delta_buf(l)), c->delta_ld(l), out_cols,
-                                c->d_bg_chunks, c->n_bg_chunks, c->d_bg_chunk_begin, c->M, c->d_bg_partial,
+                                ct->d_chunks, ct->n, ct->d_begin, c->fused_sync ? 1 : c->M, c->d_bg_partial,
                                 c->d_slabs, c->Ps, ly.b_off, s);
       ph.launched(2);
     }
@@ -588,6 +641,11 @@ hs_status hs_init(const hs_model_desc* model, int32_t M, const double* compute_w
       if (l == 0 && !bf16) continue;   // fp32 reads x in place
       chk(dalloc(c, &c->d_act[l], es * N * (size_t)dims[l]));
     }
+    chk(dalloc(c, &c->d_scale_fused, sizeof(float) * N));
+    chk(dalloc(c, &c->d_all_off, sizeof(int32_t) * 2));
+    chk(dalloc(c, &c->d_w_one, sizeof(float)));
+    chk(dalloc(c, &c->all_rows.d_chunks, sizeof(int4) * (size_t)(c->N / R + 2)));
+    chk(dalloc(c, &c->all_rows.d_begin, sizeof(int32_t) * 2));
   } else {
     const int c3 = c->convs[2].cout;
     int64_t dcol = 0;
@@ -646,7 +704,22 @@ hs_status hs_init(const hs_model_desc* model, int32_t M, const double* compute_w
     if (e == cudaSuccess && c->arch == HS_MLP) e = cudaMemset(c->d_delta[1], 0, es * delta_elems);
     if (e != cudaSuccess) s2 = cuda_fail(c, e, "cudaMemset");
   }
+  if (s2 == HS_OK && c->arch == HS_MLP) {
+    // one-worker tables of the slab-free formulation
+    const int32_t all_off[2] = {0, c->N};
+    const float one = 1.0f;
+    std::vector<int4> chunks;
+    for (int r = 0; r < c->N; r += R) chunks.push_back(make_int4(0, r, std::min(r + R, c->N), 0));
+    const int32_t begin[2] = {0, (int32_t)chunks.size()};
+    c->all_rows.n = (int)chunks.size();
+    e = cudaMemcpy(c->d_all_off, all_off, sizeof(all_off), cudaMemcpyHostToDevice);
+    if (e == cudaSuccess) e = cudaMemcpy(c->d_w_one, &one, sizeof(one), cudaMemcpyHostToDevice);
+    if (e == cudaSuccess) e = cudaMemcpy(c->all_rows.d_chunks, chunks.data(), sizeof(int4) * chunks.size(), cudaMemcpyHostToDevice);
+    if (e == cudaSuccess) e = cudaMemcpy(c->all_rows.d_begin, begin, sizeof(begin), cudaMemcpyHostToDevice);
+    if (e != cudaSuccess) s2 = cuda_fail(c, e, "slab-free tables");
+  }
   if (s2 == HS_OK && bf16) s2 = c->arch == HS_MLP ? build_tc_static(c) : cnn_build_static(c);
+  if (s2 == HS_OK && bf16 && c->arch == HS_MLP) s2 = build_tc_wgrad_fused(c);
   if (s2 == HS_OK && bf16 && c->arch == HS_MLP) {
     const char* ov = getenv("HS_OVERLAP_UPDATE");
     c->overlap_update = !(ov && !strcmp(ov, "0"));
@@ -775,7 +848,8 @@ hs_status hs_step(hs_ctx* c, float* params, const void* x, const int32_t* y, con
   if (!mlp_bf16) {
     PhaseScope ph(c, HS_PHASE_UPDATE, s);
     hs::UpdateRecipe r{c->d_mom, c->opt_momentum, c->opt_weight_decay, c->mom_valid ? 0 : 1};
-    hs::launch_reduce_update(params, c->d_slabs, c->Ps, c->M, c->d_w, lr, c->P,
+    hs::launch_reduce_update(params, c->d_slabs, c->Ps, c->fused_sync ? 1 : c->M,
+                             c->fused_sync ? c->d_w_one : c->d_w, lr, c->P,
                              c->precision == HS_BF16 ? c->d_shadow : nullptr, c->debug ? c->d_gdebug : nullptr,
                              c->num_sms, s, 4, c->opt_recipe ? &r : nullptr);
     ph.launched();
@@ -829,6 +903,14 @@ hs_status hs_read_profile(hs_ctx* c, double* ms_out, int64_t* launches_out) {
     for (int i = 0; i < HS_PHASE_COUNT; ++i) launches_out[i] = c->launches[i];
   for (int i = 0; i < HS_PHASE_COUNT; ++i) c->launches[i] = 0;
   if (first != cudaSuccess) return cuda_fail(c, first, "reading profile events");
+  return HS_OK;
+}
+
+hs_status hs_set_fused_sync(hs_ctx* c, int32_t enable) {
+  if (!c) return HS_ERR_INVALID_ARG;
+  c->err.clear();
+  if (c->arch != HS_MLP) return fail(c, HS_ERR_UNSUPPORTED, "the slab-free formulation is built for the MLP only");
+  c->fused_sync = enable != 0;
   return HS_OK;
 }
 
@@ -906,6 +988,7 @@ hs_status hs_debug_grads(hs_ctx* c, float* g_out, float* slabs_out, void* stream
     HS_CUDA(c, cudaMemcpyAsync(g_out, c->d_gdebug, sizeof(float) * c->P, cudaMemcpyDeviceToDevice, s));
   }
   if (slabs_out) {
+    if (c->fused_sync) return fail(c, HS_ERR_INVALID_ARG, "the slab-free formulation keeps no per-worker slabs");
     HS_CUDA(c, cudaMemcpy2DAsync(slabs_out, sizeof(float) * c->P, c->d_slabs, sizeof(float) * c->Ps,
                                  sizeof(float) * c->P, c->M, cudaMemcpyDeviceToDevice, s));
   }

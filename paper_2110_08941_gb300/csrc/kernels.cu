@@ -60,6 +60,19 @@ void launch_partition_scatter(const int32_t* d_offsets, int M, int N, int32_t* i
       d_offsets, M, N, index_map, scale, index_map_out);
 }
 
+// out[i] = w[m(i)] * scale[i]: the loss-gradient scale of the slab-free formulation, where worker
+// m's weight is folded into its samples (sum_m w_m G_m = one product over all rows).
+__global__ void scale_by_weight_kernel(const int32_t* __restrict__ index_map, const float* __restrict__ scale,
+                                       const float* __restrict__ w, int N, float* __restrict__ out) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < N) out[i] = w[index_map[i]] * scale[i];
+}
+
+void launch_scale_by_weight(const int32_t* index_map, const float* scale, const float* w, int N, float* out,
+                            cudaStream_t s) {
+  scale_by_weight_kernel<<<(N + 255) / 256, 256, 0, s>>>(index_map, scale, w, N, out);
+}
+
 // ------------------------------------------------------------------ softmax cross-entropy
 __device__ __forceinline__ float warp_max(float v) {
 #pragma unroll

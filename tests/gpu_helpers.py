@@ -27,13 +27,15 @@ def _lr_at(lr, t):
 
 
 def run_library(arch, dims, M, N, weights, x, y, theta0, lr, steps, precision, sync, repartition=None,
-                keep_slabs=False, recipe=None):
+                keep_slabs=False, recipe=None, fused=False):
     """Returns dict(theta, losses, g_first, slabs_first, counts, index_map)."""
     ctx = hs.hs_init(arch, dims, M, N, compute_weights=weights, precision=precision, sync=sync)
     try:
         hs.hs_set_debug(ctx, True)
         if recipe is not None:
             hs.hs_set_optimizer(ctx, *recipe)
+        if fused:
+            hs.hs_set_fused_sync(ctx, True)
         params = torch.tensor(theta0, device="cuda")
         xd = torch.from_numpy(np.ascontiguousarray(x)).cuda()
         yd = torch.from_numpy(np.ascontiguousarray(y)).cuda()

@@ -214,3 +214,29 @@ def test_momentum_weight_decay_cosine_lr(name, precision):
     orc = run_oracle(wl.arch, wl.dims, wl.workers, wl.global_batch, w, x, y, theta0, sched, 10,
                      hs.HS_SYNC_CP_WEIGHTED, decide=decide_for(precision), recipe=recipe)
     _check(lib, orc, theta0.astype(np.float64), precision, 10)
+
+
+# ------------------------------------------------------------------ slab-free formulation
+@pytest.mark.parametrize("name,precision,sync", [(synth.CFG1, hs.HS_BF16, hs.HS_SYNC_CP_WEIGHTED),
+                                                 (synth.CFG2, hs.HS_BF16, hs.HS_SYNC_MEAN),
+                                                 (synth.CFG2, hs.HS_FP32_CHECK, hs.HS_SYNC_CP_WEIGHTED),
+                                                 (synth.CFG2, hs.HS_FP32_CHECK, hs.HS_SYNC_MEAN)])
+def test_fused_sync_matches_oracle(name, precision, sync):
+    """sum_m w_m G_m as one all-rows product with the weights folded into the loss-gradient scale."""
+    wl, x, y, theta0, w = _inputs(name)
+    lib = run_library(wl.arch, wl.dims, wl.workers, wl.global_batch, w, x, y, theta0, wl.lr, 10, precision, sync,
+                      fused=True)
+    orc = _oracle_run(name, sync, 10, precision)
+    _check(lib, orc, theta0.astype(np.float64), precision, 10)
+
+
+def test_fused_sync_headline_workload_gradient():
+    """4096-8192-8192-1000, N 16384, M 16: the slab-free gradient equals the slab gradient (same kernels,
+    different summation order) and the step keeps working with the per-worker losses."""
+    wl, x, y, theta0, w = _inputs(synth.CFG5)
+    a = run_library(wl.arch, wl.dims, wl.workers, wl.global_batch, w, x, y, theta0, wl.lr, 1, hs.HS_BF16,
+                    hs.HS_SYNC_CP_WEIGHTED)
+    b = run_library(wl.arch, wl.dims, wl.workers, wl.global_batch, w, x, y, theta0, wl.lr, 1, hs.HS_BF16,
+                    hs.HS_SYNC_CP_WEIGHTED, fused=True)
+    assert rel(b["g_first"], a["g_first"]) <= 5e-3
+    assert a["worker_losses_first"] == b["worker_losses_first"]
