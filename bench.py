@@ -178,6 +178,46 @@ def straggler_simulation(seed=0, steps=200, every=10):
             "sum_time_ideal_split": t_ideal, "unit": "sample-times (n / speed, speed c_m(0) = 1)"}
 
 
+def heterogeneity_simulation(per_sample_s: float, seed: int = 0, workers: int = 8, per_worker: int = 128,
+                             epochs: int = 15, steps_per_epoch: int = 20, jitter: float = 0.05):
+    """Replica of the delay experiments (Section 5.2 / 5.3) on simulated workers.  Every worker
+    processes a sample in `per_sample_s` seconds (from the measured GPU step); half of them also
+    sleep for a fixed delay each minibatch, 25% ("low") or 50% ("high") of the mean minibatch
+    time, with a little multiplicative noise.  Sync-SGD keeps the even split of 128 samples per
+    worker (weak scaling); Dynamic Partitioning (Algorithm 1) re-sizes the partitions every epoch
+    from the mean measured minibatch times of the last epoch (Eq. 2, the library's host rule).
+    A step lasts as long as its slowest worker (Section 3).  Host only."""
+    import paper_2110_08941_gb300 as hs
+    rng = np.random.default_rng(seed + 5)
+    n = workers * per_worker
+    base = per_worker * per_sample_s
+    out = {}
+    for level, frac in (("low", 0.25), ("high", 0.50)):
+        delay = np.array([frac * base if k % 2 == 0 else 0.0 for k in range(workers)])
+        res = {}
+        for sched in ("sync_sgd", "dynamic_partitioning"):
+            sizes = [per_worker] * workers
+            times = []
+            for ep in range(epochs):
+                ep_times = np.zeros(workers)
+                for _ in range(steps_per_epoch):
+                    noise = rng.lognormal(0.0, jitter, workers)
+                    x = (np.asarray(sizes) * per_sample_s + delay) * noise
+                    ep_times += x
+                    times.append(float(x.max()))
+                if sched == "dynamic_partitioning":
+                    mean_x = ep_times / steps_per_epoch
+                    sizes = hs.hs_partition_sizes([sizes[k] / mean_x[k] for k in range(workers)], n)
+            t = np.asarray(times)
+            res[sched] = {"total_s": float(t.sum()), "mean_step_ms": 1e3 * float(t.mean()),
+                          "p50_ms": 1e3 * float(np.percentile(t, 50)), "p90_ms": 1e3 * float(np.percentile(t, 90)),
+                          "last_sizes": [int(v) for v in sizes]}
+        res["speedup"] = res["sync_sgd"]["total_s"] / res["dynamic_partitioning"]["total_s"]
+        out[level] = res
+    out["per_sample_ms"] = 1e3 * per_sample_s
+    return out
+
+
 def update_bytes(wl, P):
     # M slab reads + theta read, theta write + bf16 shadow write
     return (wl.workers + 2) * P * 4 + 2 * P
@@ -414,6 +454,7 @@ def run_ours(args, wl, rank, world, local_rank):
             "clocks": clk,
             "straggler_sim": straggler_simulation(),
             "fused_sync_variant": fused,
+            "heterogeneity_sim": heterogeneity_simulation(ms * 1e-3 / args.steps / wl.global_batch),
             "loss_after": loss,
         }
         print(json.dumps(out), flush=True)

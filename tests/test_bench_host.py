@@ -38,3 +38,15 @@ def test_gemm_flops_of_the_headline_workload():
     assert abs(sum(f.values()) - 9.6014e12) / 9.6014e12 < 1e-4
     cnn = bench.gemm_flops(synth.WORKLOADS[synth.CFG4])
     assert abs(sum(cnn.values()) - 1.196e11) / 1.196e11 < 1e-3
+
+
+def test_heterogeneity_replica_dynamic_partitioning_helps():
+    r = bench.heterogeneity_simulation(4e-7, seed=1)
+    for level in ("low", "high"):
+        assert r[level]["speedup"] > 1.0
+        sizes = r[level]["dynamic_partitioning"]["last_sizes"]
+        assert sum(sizes) == 8 * 128
+        # delayed workers (even index) end with fewer samples than the undelayed ones
+        assert max(sizes[0::2]) < min(sizes[1::2])
+    assert r["high"]["speedup"] > r["low"]["speedup"]
+    assert r == bench.heterogeneity_simulation(4e-7, seed=1)      # seeded, deterministic
