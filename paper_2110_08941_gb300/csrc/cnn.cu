@@ -30,7 +30,15 @@ __device__ __forceinline__ __nv_bfloat16 from_f<__nv_bfloat16>(float v) { return
 
 // Patch rows of the first convolution from the NCHW fp32 input: col[r][ci*9 + kh*3 + kw] =
 // x_pad[n][ci][s*ho + kh][s*wo + kw], r = (n*Ho + ho)*Wo + wo; columns K..Kp-1 are zero.
-template <typename T>
+// Column of patch entry (ci, tap): tap-major (tap*C + ci: neighbouring channels adjacent, used by the
+// bf16 path) or channel-major (ci*9 + tap: the order of theta's [Cout, Cin, 3, 3], used by the fp32
+// check path).
+template <bool kTapMajor>
+__device__ __forceinline__ int patch_col(int ci, int tap, int C) {
+  return kTapMajor ? tap * C + ci : ci * 9 + tap;
+}
+
+template <typename T, bool kTapMajor>
 __global__ void im2col_nchw_kernel(const float* __restrict__ x, int N, int C, int H, int W, int Ho, int Wo, int s,
                                    T* __restrict__ col, int Kp) {
   const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
@@ -41,7 +49,7 @@ __global__ void im2col_nchw_kernel(const float* __restrict__ x, int N, int C, in
   const int wo = (int)(r % Wo);
   const int ho = (int)((r / Wo) % Ho);
   const int n = (int)(r / ((int64_t)Wo * Ho));
-  T* dst = col + r * Kp + ci * 9;
+  T* dst = col + r * Kp;
   const float* src = x + ((int64_t)n * C + ci) * H * W;
 #pragma unroll
   for (int kh = 0; kh < 3; ++kh) {
@@ -50,17 +58,86 @@ __global__ void im2col_nchw_kernel(const float* __restrict__ x, int N, int C, in
     for (int kw = 0; kw < 3; ++kw) {
       const int wi = s * wo + kw - 1;
       const float v = (hi >= 0 && hi < H && wi >= 0 && wi < W) ? src[(int64_t)hi * W + wi] : 0.f;
-      dst[kh * 3 + kw] = from_f<T>(v);
+      dst[patch_col<kTapMajor>(ci, kh * 3 + kw, C)] = from_f<T>(v);
     }
   }
-  if (ci == 0)
-    for (int k = C * 9; k < Kp; ++k) col[r * Kp + k] = from_f<T>(0.f);
+  if (ci == 0)   // tail: the bf16 layout carries a ones column at 9*C (see cnn_build_wgrad_plan)
+    for (int k = C * 9; k < Kp; ++k) col[r * Kp + k] = from_f<T>((kTapMajor && k == C * 9) ? 1.f : 0.f);
 }
 
-// Patch rows from an NHWC activation h[n][hi][wi][ci] (same column order as above).
-template <typename T>
-__global__ void im2col_nhwc_kernel(const T* __restrict__ h, int N, int C, int H, int W, int Ho, int Wo, int s,
-                                   T* __restrict__ col, int Kp) {
+// bf16 patch rows, tap-major, eight channels per thread (16-byte copies).  The tail of each row
+// holds a ones column at 9*C (then zeros): the per-worker weight-gradient product then also
+// yields the bias gradient, sum over the worker's rows of dA.
+__global__ void im2col_nhwc_vec8_kernel(const __nv_bfloat16* __restrict__ h, int N, int C, int H, int W, int Ho,
+                                        int Wo, int s, __nv_bfloat16* __restrict__ col, int Kp) {
+  const int C8 = C >> 3;
+  const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const int64_t rows = (int64_t)N * Ho * Wo;
+  if (idx >= rows * 9 * C8) return;
+  const int c8 = (int)(idx % C8);
+  const int tap = (int)((idx / C8) % 9);
+  const int64_t r = idx / ((int64_t)C8 * 9);
+  const int wo = (int)(r % Wo);
+  const int ho = (int)((r / Wo) % Ho);
+  const int n = (int)(r / ((int64_t)Wo * Ho));
+  const int hi = s * ho + tap / 3 - 1, wi = s * wo + tap % 3 - 1;
+  uint4 v = make_uint4(0u, 0u, 0u, 0u);
+  if (hi >= 0 && hi < H && wi >= 0 && wi < W)
+    v = *reinterpret_cast<const uint4*>(h + (((int64_t)n * H + hi) * W + wi) * C + c8 * 8);
+  *reinterpret_cast<uint4*>(col + r * Kp + tap * C + c8 * 8) = v;
+  if (tap == 0 && c8 == 0)
+    for (int k = 9 * C; k < Kp; ++k) col[r * Kp + k] = __float2bfloat16_rn(k == 9 * C ? 1.f : 0.f);
+}
+
+// Input gradient of a convolution on its input grid (bf16 path): four channels per thread, float4
+// reads of the tap-major patch-space gradient, ReLU' of the input activation fused.
+__global__ void col2im_nhwc_vec4_kernel(const float* __restrict__ dcol, int ldc, const __nv_bfloat16* __restrict__ h,
+                                        int N, int C, int H, int W, int Ho, int Wo, int s,
+                                        __nv_bfloat16* __restrict__ dA) {
+  const int C4 = C >> 2;
+  const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= (int64_t)N * H * W * C4) return;
+  const int c4 = (int)(idx % C4);
+  const int64_t pix = idx / C4;
+  const int wi = (int)(pix % W);
+  const int hi = (int)((pix / W) % H);
+  const int n = (int)(pix / ((int64_t)W * H));
+  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+  for (int kh = 0; kh < 3; ++kh) {
+    const int th = hi + 1 - kh;
+    if (th < 0 || th % s) continue;
+    const int ho = th / s;
+    if (ho >= Ho) continue;
+#pragma unroll
+    for (int kw = 0; kw < 3; ++kw) {
+      const int tw = wi + 1 - kw;
+      if (tw < 0 || tw % s) continue;
+      const int wo = tw / s;
+      if (wo >= Wo) continue;
+      const float4 g = *reinterpret_cast<const float4*>(
+          dcol + (((int64_t)n * Ho + ho) * Wo + wo) * ldc + (kh * 3 + kw) * C + c4 * 4);
+      acc.x += g.x;
+      acc.y += g.y;
+      acc.z += g.z;
+      acc.w += g.w;
+    }
+  }
+  const int64_t o = pix * C + c4 * 4;
+  const uint2 hv = *reinterpret_cast<const uint2*>(h + o);
+  const __nv_bfloat162 h01 = *reinterpret_cast<const __nv_bfloat162*>(&hv.x);
+  const __nv_bfloat162 h23 = *reinterpret_cast<const __nv_bfloat162*>(&hv.y);
+  __nv_bfloat162 lo = __floats2bfloat162_rn(__low2float(h01) > 0.f ? acc.x : 0.f, __high2float(h01) > 0.f ? acc.y : 0.f);
+  __nv_bfloat162 hi2 = __floats2bfloat162_rn(__low2float(h23) > 0.f ? acc.z : 0.f, __high2float(h23) > 0.f ? acc.w : 0.f);
+  uint2 out;
+  out.x = *reinterpret_cast<uint32_t*>(&lo);
+  out.y = *reinterpret_cast<uint32_t*>(&hi2);
+  *reinterpret_cast<uint2*>(dA + o) = out;
+}
+
+// fp32 check path: patch rows from an NHWC activation h[n][hi][wi][ci], channel-major columns.
+__global__ void im2col_nhwc_f32_kernel(const float* __restrict__ h, int N, int C, int H, int W, int Ho, int Wo, int s,
+                                       float* __restrict__ col, int Kp) {
   const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   const int64_t rows = (int64_t)N * Ho * Wo;
   if (idx >= rows * C) return;
@@ -69,16 +146,15 @@ __global__ void im2col_nhwc_kernel(const T* __restrict__ h, int N, int C, int H,
   const int wo = (int)(r % Wo);
   const int ho = (int)((r / Wo) % Ho);
   const int n = (int)(r / ((int64_t)Wo * Ho));
-  T* dst = col + r * Kp + ci * 9;
+  float* dst = col + r * Kp;
 #pragma unroll
   for (int kh = 0; kh < 3; ++kh) {
     const int hi = s * ho + kh - 1;
 #pragma unroll
     for (int kw = 0; kw < 3; ++kw) {
       const int wi = s * wo + kw - 1;
-      dst[kh * 3 + kw] = (hi >= 0 && hi < H && wi >= 0 && wi < W)
-                             ? h[(((int64_t)n * H + hi) * W + wi) * C + ci]
-                             : from_f<T>(0.f);
+      dst[patch_col<false>(ci, kh * 3 + kw, C)] =
+          (hi >= 0 && hi < H && wi >= 0 && wi < W) ? h[(((int64_t)n * H + hi) * W + wi) * C + ci] : 0.f;
     }
   }
 }
@@ -107,11 +183,10 @@ __global__ void gap_backward_kernel(const float* __restrict__ dpooled, const T* 
   dA[idx] = from_f<T>(to_f<T>(h[idx]) > 0.f ? g : 0.f);
 }
 
-// Input gradient on the input grid: the adjoint of im2col (each input element sums the patch
-// entries that read it), then ReLU' of that input: dA[n][hi][wi][ci].
-template <typename T>
-__global__ void col2im_nhwc_kernel(const float* __restrict__ dcol, int ldc, const T* __restrict__ h, int N, int C,
-                                   int H, int W, int Ho, int Wo, int s, T* __restrict__ dA) {
+// Input gradient on the input grid (fp32 check path): the adjoint of im2col (each input element
+// sums the patch entries that read it), then ReLU' of that input: dA[n][hi][wi][ci].
+__global__ void col2im_nhwc_f32_kernel(const float* __restrict__ dcol, int ldc, const float* __restrict__ h, int N,
+                                       int C, int H, int W, int Ho, int Wo, int s, float* __restrict__ dA) {
   const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (idx >= (int64_t)N * H * W * C) return;
   const int ci = (int)(idx % C);
@@ -131,31 +206,47 @@ __global__ void col2im_nhwc_kernel(const float* __restrict__ dcol, int ldc, cons
       if (tw < 0 || tw % s) continue;
       const int wo = tw / s;
       if (wo >= Wo) continue;
-      acc += dcol[(((int64_t)n * Ho + ho) * Wo + wo) * ldc + ci * 9 + kh * 3 + kw];
+      acc += dcol[(((int64_t)n * Ho + ho) * Wo + wo) * ldc + patch_col<false>(ci, kh * 3 + kw, C)];
     }
   }
-  dA[idx] = from_f<T>(to_f<T>(h[idx]) > 0.f ? acc : 0.f);
+  dA[idx] = h[idx] > 0.f ? acc : 0.f;
 }
 
-// bf16 copy of the first convolution's weights with rows padded from K to Kp (16-byte rows).
-__global__ void pad_weights_kernel(const float* __restrict__ w, int rows, int K, int Kp, __nv_bfloat16* __restrict__ wp) {
+// bf16 copy of a convolution's weights in the tap-major column order of the bf16 patch rows:
+// wp[co][tap*Cin + ci] = bf16(w[co][ci][tap]), rows padded from 9*Cin to Kp with zeros.
+__global__ void permute_weights_kernel(const float* __restrict__ w, int cout, int cin, int Kp,
+                                       __nv_bfloat16* __restrict__ wp) {
   const int idx = blockIdx.x * blockDim.x + threadIdx.x;
-  if (idx >= rows * Kp) return;
-  const int k = idx % Kp, r = idx / Kp;
-  wp[idx] = __float2bfloat16_rn(k < K ? w[(int64_t)r * K + k] : 0.f);
+  if (idx >= cout * Kp) return;
+  const int k = idx % Kp, co = idx / Kp;
+  float v = 0.f;
+  if (k < 9 * cin) {
+    const int tap = k / cin, ci = k % cin;
+    v = w[((int64_t)co * cin + ci) * 9 + tap];
+  }
+  wp[idx] = __float2bfloat16_rn(v);
 }
 
-// slabs[m][w_off + co*K + k] = sum over worker m's chunks (in order) of partial[chunk][co][k].
+// slabs[m][w_off + co*K + k] = sum over worker m's chunks (in order) of partial[chunk][co][k'], where
+// k' = k for the fully connected layer (cin = 0) and, for a convolution, the tap-major column of
+// theta's (ci, tap) entry k = ci*9 + tap (k' = tap*cin + ci).
+// With cin != 0 the partial's column 9*cin is the ones column of the patch rows: its sums are the
+// convolution's bias gradient, written at slabs[m][b_off + co].
 __global__ void splitk_reduce_kernel(const float* __restrict__ partial, int rows, int K, int ldp,
                                      const int32_t* __restrict__ chunk_begin, float* __restrict__ slabs, int64_t Ps,
-                                     int64_t w_off) {
+                                     int64_t w_off, int cin, int64_t b_off) {
   const int m = blockIdx.y;
+  const int cols = cin ? K + 1 : K;
   const int idx = blockIdx.x * blockDim.x + threadIdx.x;
-  if (idx >= rows * K) return;
-  const int k = idx % K, co = idx / K;
+  if (idx >= rows * cols) return;
+  const int k = idx % cols, co = idx / cols;
+  const int kp = (cin && k < K) ? (k % 9) * cin + k / 9 : k;
   float acc = 0.f;
-  for (int c = chunk_begin[m]; c < chunk_begin[m + 1]; ++c) acc += partial[((int64_t)c * rows + co) * ldp + k];
-  slabs[(int64_t)m * Ps + w_off + idx] = acc;
+  for (int c = chunk_begin[m]; c < chunk_begin[m + 1]; ++c) acc += partial[((int64_t)c * rows + co) * ldp + kp];
+  if (k < K)
+    slabs[(int64_t)m * Ps + w_off + (int64_t)co * K + k] = acc;
+  else
+    slabs[(int64_t)m * Ps + b_off + co] = acc;
 }
 
 inline int blocks_for(int64_t n, int threads) { return (int)((n + threads - 1) / threads); }
@@ -263,8 +354,8 @@ hs_status cnn_build_static(hs_ctx* c) {
   c->tc_dgrad.assign(4, TcGemmParams{});
   for (int k = 0; k < 3; ++k) {
     const ConvLayer& L = c->convs[k];
-    const __nv_bfloat16* wb = (k == 0) ? c->d_w1p : c->d_shadow + L.w_off;
-    const int64_t ldw = (k == 0) ? L.Kp : L.K;
+    const __nv_bfloat16* wb = c->d_wperm[k];
+    const int64_t ldw = L.Kp;
     hs_status st = plan_dense(c, &c->tc_fwd[k], kTcEpiBiasReluBf16, bf(c->d_col[k]), L.rows, L.K, L.Kp, wb, L.cout,
                               L.K, ldw, false, c->d_cact[k], false, (int)L.rows, L.cout, L.cout, L.cout, nullptr, 0);
     if (st != HS_OK) return st;
@@ -281,7 +372,7 @@ hs_status cnn_build_static(hs_ctx* c) {
   for (int k = 2; k >= 1; --k) {
     const ConvLayer& L = c->convs[k];
     st = plan_dense(c, &c->tc_dgrad[k], kTcEpiStoreF32, bf(c->d_dA[k]), L.rows, L.cout, L.cout,
-                    c->d_shadow + L.w_off, L.cout, L.K, L.K, true, c->d_dcol, true, (int)L.rows, L.K, L.K, L.K,
+                    c->d_wperm[k], L.cout, L.K, L.Kp, true, c->d_dcol, true, (int)L.rows, L.K, L.K, L.K,
                     nullptr, 0);
     if (st != HS_OK) return st;
   }
@@ -295,7 +386,7 @@ hs_status cnn_build_partition_plans(hs_ctx* c) {
   hs_status st = cnn_build_wgrad_plan(c, 3, bf(c->d_delta[0]), c->C, c->Cp, bf(c->d_pooled), c3, c3, 1);
   for (int k = 2; k >= 0 && st == HS_OK; --k) {
     const ConvLayer& L = c->convs[k];
-    st = cnn_build_wgrad_plan(c, k, bf(c->d_dA[k]), L.cout, L.cout, bf(c->d_col[k]), L.K, L.Kp,
+    st = cnn_build_wgrad_plan(c, k, bf(c->d_dA[k]), L.cout, L.cout, bf(c->d_col[k]), L.K + 1, L.Kp,
                               (int64_t)L.hout * L.wout);
   }
   return st;
@@ -311,9 +402,10 @@ hs_status cnn_step(hs_ctx* c, float* params, const float* x, const int32_t* y, c
   {
     PhaseScope ph(c, HS_PHASE_CAST, s);
     if (bf16) {
-      pad_weights_kernel<<<blocks_for((int64_t)L[0].cout * L[0].Kp, T), T, 0, s>>>(params + L[0].w_off, L[0].cout, L[0].K,
-                                                                                   L[0].Kp, c->d_w1p);
-      ph.launched();
+      for (int k = 0; k < 3; ++k)
+        permute_weights_kernel<<<blocks_for((int64_t)L[k].cout * L[k].Kp, T), T, 0, s>>>(
+            params + L[k].w_off, L[k].cout, L[k].cin, L[k].Kp, c->d_wperm[k]);
+      ph.launched(3);
     }
   }
   {
@@ -322,20 +414,20 @@ hs_status cnn_step(hs_ctx* c, float* params, const float* x, const int32_t* y, c
       const int64_t n_items = L[k].rows * L[k].cin;
       if (k == 0) {
         if (bf16)
-          im2col_nchw_kernel<__nv_bfloat16><<<blocks_for(n_items, T), T, 0, s>>>(
+          im2col_nchw_kernel<__nv_bfloat16, true><<<blocks_for(n_items, T), T, 0, s>>>(
               x, N, L[0].cin, L[0].hin, L[0].win, L[0].hout, L[0].wout, L[0].stride,
               reinterpret_cast<__nv_bfloat16*>(c->d_col[0]), L[0].Kp);
         else
-          im2col_nchw_kernel<float><<<blocks_for(n_items, T), T, 0, s>>>(
+          im2col_nchw_kernel<float, false><<<blocks_for(n_items, T), T, 0, s>>>(
               x, N, L[0].cin, L[0].hin, L[0].win, L[0].hout, L[0].wout, L[0].stride,
               reinterpret_cast<float*>(c->d_col[0]), L[0].Kp);
       } else {
         if (bf16)
-          im2col_nhwc_kernel<__nv_bfloat16><<<blocks_for(n_items, T), T, 0, s>>>(
+          im2col_nhwc_vec8_kernel<<<blocks_for(L[k].rows * 9 * (L[k].cin / 8), T), T, 0, s>>>(
               reinterpret_cast<const __nv_bfloat16*>(c->d_cact[k - 1]), N, L[k].cin, L[k].hin, L[k].win, L[k].hout,
               L[k].wout, L[k].stride, reinterpret_cast<__nv_bfloat16*>(c->d_col[k]), L[k].Kp);
         else
-          im2col_nhwc_kernel<float><<<blocks_for(n_items, T), T, 0, s>>>(
+          im2col_nhwc_f32_kernel<<<blocks_for(n_items, T), T, 0, s>>>(
               reinterpret_cast<const float*>(c->d_cact[k - 1]), N, L[k].cin, L[k].hin, L[k].win, L[k].hout,
               L[k].wout, L[k].stride, reinterpret_cast<float*>(c->d_col[k]), L[k].Kp);
       }
@@ -403,9 +495,10 @@ hs_status cnn_step(hs_ctx* c, float* params, const float* x, const int32_t* y, c
           if (e != cudaSuccess) return cuda_fail(c, e, "conv weight-gradient GEMM launch");
           ph.launched();
         }
-        dim3 grid(blocks_for((int64_t)wg.rows_out * wg.K, T), c->M);
-        splitk_reduce_kernel<<<grid, T, 0, s>>>(wg.d_partial, wg.rows_out, wg.K, wg.ldp, wg.d_chunk_begin, c->d_slabs,
-                                                c->Ps, w_off);
+        const int kw = fc ? wg.K : wg.K - 1;   // weight columns (the conv partials carry the bias column)
+        dim3 grid2(blocks_for((int64_t)wg.rows_out * wg.K, T), c->M);
+        splitk_reduce_kernel<<<grid2, T, 0, s>>>(wg.d_partial, wg.rows_out, kw, wg.ldp, wg.d_chunk_begin, c->d_slabs,
+                                                 c->Ps, w_off, fc ? 0 : L[k].cin, b_off);
         ph.launched();
       } else {
         GemmF32Args w{};
@@ -425,7 +518,9 @@ hs_status cnn_step(hs_ctx* c, float* params, const float* x, const int32_t* y, c
     }
     {
       PhaseScope ph(c, HS_PHASE_BIASGRAD, s);
-      if (bf16) {
+      if (bf16 && !fc) {
+        // the convolutions' bias gradients came out of the weight-gradient product (ones column)
+      } else if (bf16) {
         const ChunkTable& ct = c->cnn_chunks[k];
         launch_bias_grad_bf16(reinterpret_cast<const __nv_bfloat16*>(delta), ld_delta, width, ct.d_chunks, ct.n,
                               ct.d_begin, c->M, c->d_bg_partial, c->d_slabs, c->Ps, b_off, s);
@@ -473,11 +568,11 @@ hs_status cnn_step(hs_ctx* c, float* params, const float* x, const int32_t* y, c
       }
       const int64_t n_in = (int64_t)N * L[k].hin * L[k].win * L[k].cin;
       if (bf16)
-        col2im_nhwc_kernel<__nv_bfloat16><<<blocks_for(n_in, T), T, 0, s>>>(
+        col2im_nhwc_vec4_kernel<<<blocks_for(n_in / 4, T), T, 0, s>>>(
             c->d_dcol, L[k].K, reinterpret_cast<const __nv_bfloat16*>(c->d_cact[k - 1]), N, L[k].cin, L[k].hin,
             L[k].win, L[k].hout, L[k].wout, L[k].stride, reinterpret_cast<__nv_bfloat16*>(c->d_dA[k - 1]));
       else
-        col2im_nhwc_kernel<float><<<blocks_for(n_in, T), T, 0, s>>>(
+        col2im_nhwc_f32_kernel<<<blocks_for(n_in, T), T, 0, s>>>(
             c->d_dcol, L[k].K, reinterpret_cast<const float*>(c->d_cact[k - 1]), N, L[k].cin, L[k].hin, L[k].win,
             L[k].hout, L[k].wout, L[k].stride, reinterpret_cast<float*>(c->d_dA[k - 1]));
       ph.launched(2);

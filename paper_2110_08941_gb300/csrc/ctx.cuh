@@ -143,7 +143,7 @@ struct hs_ctx {
   float* d_dpooled = nullptr;
   void* d_dA[3] = {nullptr, nullptr, nullptr};
   float* d_dcol = nullptr;
-  __nv_bfloat16* d_w1p = nullptr;
+  __nv_bfloat16* d_wperm[3] = {nullptr, nullptr, nullptr};   // bf16 [Cout][Kp], tap-major columns
   int32_t* d_row_off[4] = {nullptr, nullptr, nullptr, nullptr};
   hs::ChunkTable cnn_chunks[4];
   hs::CnnWgrad cnn_wgrad[4];

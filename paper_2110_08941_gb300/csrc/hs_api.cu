@@ -245,9 +245,10 @@ hs_status apply_partition(hs_ctx* c, const std::vector<int32_t>& sizes, const st
   }
   if (changed && c->arch == HS_CNN) {
     // per-layer row offsets (a sample is Ho*Wo rows of a conv product, one row of the fc product)
-    const int R = hs::bias_grad_chunk_rows();
     for (int k = 0; k < 4; ++k) {
       const int64_t rps = c->cnn_chunks[k].rows_per_sample;
+      // conv layers have many narrow rows: longer chunks keep the per-worker combine short
+      const int R = rps > 1 ? 16 * hs::bias_grad_chunk_rows() : hs::bias_grad_chunk_rows();
       std::vector<int32_t> ro(c->M + 1), begin;
       std::vector<int4> chunks;
       for (int m = 0; m <= c->M; ++m) ro[m] = (int32_t)(c->offsets[m] * rps);
@@ -291,7 +292,8 @@ void free_all(hs_ctx* c) {
   f(c->d_bg_chunks); f(c->d_bg_chunk_begin); f(c->d_bg_partial);
   f(c->d_scale_fused); f(c->d_all_off); f(c->d_w_one); f(c->all_rows.d_chunks); f(c->all_rows.d_begin);
   for (int k = 0; k < 3; ++k) { f(c->d_col[k]); f(c->d_cact[k]); f(c->d_dA[k]); }
-  f(c->d_pooled); f(c->d_dpooled); f(c->d_dcol); f(c->d_w1p);
+  f(c->d_pooled); f(c->d_dpooled); f(c->d_dcol);
+  for (int k = 0; k < 3; ++k) f(c->d_wperm[k]);
   for (int k = 0; k < 4; ++k) {
     f(c->d_row_off[k]); f(c->cnn_chunks[k].d_chunks); f(c->cnn_chunks[k].d_begin);
     f(c->cnn_wgrad[k].d_partial); f(c->cnn_wgrad[k].d_chunk_begin);
@@ -598,7 +600,7 @@ hs_status hs_init(const hs_model_desc* model, int32_t M, const double* compute_w
       L.hout = (h + 2 - 3) / L.stride + 1;
       L.wout = (w + 2 - 3) / L.stride + 1;
       L.K = prev * 9;
-      L.Kp = bf16 ? (int)round_up(L.K, 8) : L.K;
+      L.Kp = bf16 ? (int)round_up(L.K + 1, 8) : L.K;   // bf16 rows carry a ones column at K
       L.w_off = off;
       off += (int64_t)L.cout * L.K;
       L.b_off = off;
@@ -659,7 +661,9 @@ hs_status hs_init(const hs_model_desc* model, int32_t M, const double* compute_w
     chk(dalloc(c, &c->d_pooled, es * N * c3));
     chk(dalloc(c, &c->d_dpooled, sizeof(float) * N * c3));
     chk(dalloc(c, &c->d_dcol, sizeof(float) * (size_t)dcol));
-    if (bf16) chk(dalloc(c, &c->d_w1p, sizeof(__nv_bfloat16) * (size_t)c->convs[0].cout * c->convs[0].Kp));
+    if (bf16)
+      for (int k = 0; k < 3; ++k)
+        chk(dalloc(c, &c->d_wperm[k], sizeof(__nv_bfloat16) * (size_t)c->convs[k].cout * c->convs[k].Kp));
     delta_elems = N * (size_t)c->Cp;
     for (int k = 0; k < 4; ++k) {
       const bool fc = (k == 3);
@@ -674,7 +678,7 @@ hs_status hs_init(const hs_model_desc* model, int32_t M, const double* compute_w
       if (bf16) {
         CnnWgrad& wg = c->cnn_wgrad[k];
         const int rows_out = width;
-        const int kcols = fc ? c3 : c->convs[k].K;
+        const int kcols = fc ? c3 : c->convs[k].K + 1;
         const int tiles = ((rows_out + kTcBM - 1) / kTcBM) * ((kcols + kTcBN - 1) / kTcBN);
         const int64_t target = std::max<int64_t>(1, (2LL * c->num_sms + tiles - 1) / tiles);
         wg.partial_capacity = (target + M + 1) * rows_out * round_up(kcols, 4);
