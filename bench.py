@@ -259,6 +259,55 @@ def oracle_sample(wl, seconds_target=12.0, max_workers=None):
     return done_samples / elapsed, desc, threads
 
 
+def blas_name():
+    try:
+        from threadpoolctl import threadpool_info
+        info = [i for i in threadpool_info() if i.get("user_api") == "blas"]
+        if info:
+            return ", ".join(f"{i.get('internal_api')} {i.get('version')}" for i in info)
+    except Exception:
+        pass
+    try:
+        b = np.show_config(mode="dicts")["Build Dependencies"]["blas"]
+        return f"{b.get('name')} {b.get('version')}"
+    except Exception:
+        return None
+
+
+def _oracle_one_thread_inproc(name, n_samples):
+    from oracle import cnn, mlp, sgd
+    from oracle import partition as P
+    wl = synth.WORKLOADS[name]
+    fn = mlp.worker_loss_grad if wl.arch == synth.MLP else cnn.worker_loss_grad
+    x, y = synth.make_batch(wl)
+    theta = synth.make_params(wl).astype(np.float64)
+    sizes = P.partition_sizes(list(synth.initial_weights(wl)), wl.global_batch)
+    off = P.offsets(sizes)
+    m = min(range(wl.workers), key=lambda k: sizes[k])
+    n = min(n_samples, sizes[m])
+    xs, ys = x[off[m]:off[m] + n], y[off[m]:off[m] + n]
+    t0 = time.perf_counter()
+    sgd.step(fn, theta, wl.dims, xs, ys, [n], wl.lr, sgd.SYNC_CP_WEIGHTED)
+    dt = time.perf_counter() - t0
+    return [n / dt, f"one thread: oracle fp64 step over the first {n} samples of worker {m}'s segment"]
+
+
+def oracle_one_thread(wl, n_samples=64):
+    """The same oracle step on the first `n_samples` rows of the smallest worker's segment, in a child
+    process whose BLAS pools are held to one thread.  Returns (samples/s, description) or None."""
+    env = dict(os.environ, OPENBLAS_NUM_THREADS="1", OMP_NUM_THREADS="1", MKL_NUM_THREADS="1",
+               BLIS_NUM_THREADS="1", CUDA_VISIBLE_DEVICES="")
+    code = ("import json, bench; "
+            f"print(json.dumps(bench._oracle_one_thread_inproc({wl.name!r}, {int(n_samples)})))")
+    try:
+        r = subprocess.run([sys.executable, "-c", code], cwd=ROOT, env=env, capture_output=True, text=True,
+                           timeout=300)
+        v, desc = json.loads(r.stdout.strip().splitlines()[-1])
+        return float(v), desc
+    except Exception:
+        return None
+
+
 # ------------------------------------------------------------------------------ ranks
 def max_over_ranks(value: float) -> float:
     """Max of a per-rank number over all ranks of the default process group (identity without one).
@@ -349,15 +398,17 @@ def run_ours(args, wl, rank, world, local_rank):
     time.sleep(0.3)
     barrier()
     torch.cuda.synchronize()
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
-    for _ in range(args.steps):
+    # one event after each step: the bracket is the first and last, the step-time spread the rest
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps + 1)]
+    ev[0].record(stream)
+    for i in range(args.steps):
         hs.hs_step(ctx, params, xd, yd, part, wl.lr, stream=stream, want_loss=False)
-    e1.record(stream)
+        ev[i + 1].record(stream)
     torch.cuda.synchronize()
     barrier()
     clk = clocks.stop()
-    ms = e0.elapsed_time(e1)
+    ms = ev[0].elapsed_time(ev[-1])
+    step_ms = np.asarray([ev[i].elapsed_time(ev[i + 1]) for i in range(args.steps)])
     prof = hs.hs_read_profile(ctx)
     hs.hs_set_profiling(ctx, False)
     ms = max_over_ranks(ms)
@@ -382,6 +433,38 @@ def run_ours(args, wl, rank, world, local_rank):
         fused = {"ms_per_step": fms / args.steps, "value": world * wl.global_batch * args.steps / (fms * 1e-3),
                  "unit": UNIT, "what": "slab-free formulation: worker weights folded into the loss-gradient "
                                        "scale, one all-rows weight-gradient product, update of one gradient"}
+
+    # the reduce+update timed on its own: a second context whose per-layer updates run after all
+    # products (HS_OVERLAP_UPDATE=0) instead of beside them, same workload and parameters
+    alone = None
+    if wl.arch == synth.MLP and precision == hs.HS_BF16:
+        prev = os.environ.get("HS_OVERLAP_UPDATE")
+        os.environ["HS_OVERLAP_UPDATE"] = "0"
+        try:
+            ctx2 = hs.hs_init(wl.arch, wl.dims, wl.workers, wl.global_batch, compute_weights=w, precision=precision,
+                              sync=hs.HS_SYNC_CP_WEIGHTED)
+        finally:
+            if prev is None:
+                os.environ.pop("HS_OVERLAP_UPDATE")
+            else:
+                os.environ["HS_OVERLAP_UPDATE"] = prev
+        p2 = params.clone()
+        for _ in range(args.warmup):
+            hs.hs_step(ctx2, p2, xd, yd, ctx2.partition, wl.lr, stream=stream, want_loss=False)
+        torch.cuda.synchronize()
+        hs.hs_read_profile(ctx2)
+        hs.hs_set_profiling(ctx2, True)
+        k2 = max(3, min(args.steps, 10))
+        a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a0.record(stream)
+        for _ in range(k2):
+            hs.hs_step(ctx2, p2, xd, yd, ctx2.partition, wl.lr, stream=stream, want_loss=False)
+        a1.record(stream)
+        torch.cuda.synchronize()
+        prof2 = hs.hs_read_profile(ctx2)
+        alone = {"update_ms": prof2["update"][0] / k2, "step_ms": a0.elapsed_time(a1) / k2}
+        ctx2.close()
+        del p2
 
     # end to end through the public API: host (pinned) inputs, loss read back every step
     xh = torch.from_numpy(x).pin_memory()
@@ -417,11 +500,22 @@ def run_ours(args, wl, rank, world, local_rank):
                 "launches_per_step": launches_per_step[name],
                 "peak_kind": f"{peaks['src']} bf16 sustained"}
 
-    upd_ach = upd_bytes / (per_step["update"] * 1e-3) / 1e9
+    overlapped = os.environ.get("HS_OVERLAP_UPDATE", "1") != "0" and wl.arch == synth.MLP
+    upd_ms = alone["update_ms"] if (alone and overlapped) else per_step["update"]
+    upd_ach = upd_bytes / (upd_ms * 1e-3) / 1e9
     roof_update = {"kernel": "reduce_update", "bound": "hbm", "achieved": upd_ach, "peak": peaks["hbm"],
                    "unit": "GB/s", "frac": upd_ach / peaks["hbm"], "traffic": None,
                    "peak_kind": f"{peaks['src']} copy bandwidth", "algorithmic_bytes": upd_bytes,
-                   "overlapped_with_gemms": os.environ.get("HS_OVERLAP_UPDATE", "1") != "0" and wl.arch == synth.MLP}
+                   "timed": ("alone: per-layer updates after all products (second context, "
+                             "HS_OVERLAP_UPDATE=0)" if (alone and overlapped) else "inside the step"),
+                   "ms_per_step": upd_ms}
+    if alone and overlapped:
+        ov_ach = upd_bytes / (per_step["update"] * 1e-3) / 1e9
+        roof_update["beside_products"] = {"ms_per_step": per_step["update"], "achieved": ov_ach,
+                                          "frac": ov_ach / peaks["hbm"],
+                                          "note": "the default step: updates share HBM and SMs with the "
+                                                  "backward products they overlap"}
+        roof_update["step_ms_updates_after_products"] = alone["step_ms"]
     roofline = roof_update if dominant == "update" else gemm_roof(dominant)
     gemm_ms = per_step["forward"] + per_step["wgrad"] + per_step["dgrad"]
     gemm_total = sum(flops.values())
@@ -430,7 +524,10 @@ def run_ours(args, wl, rank, world, local_rank):
         cpu = None
         if world == 1 and not args.no_cpu_baseline:
             v, desc, cores = oracle_sample(wl)
-            cpu = {"value": v, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": desc}
+            cpu = {"value": v, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": desc, "blas": blas_name()}
+            one = oracle_one_thread(wl)
+            if one is not None:
+                cpu["one_thread"] = {"value": one[0], "unit": UNIT, "cores": 1, "sample": one[1]}
         value = world * wl.global_batch * args.steps / (ms * 1e-3)
         out = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
@@ -446,6 +543,8 @@ def run_ours(args, wl, rank, world, local_rank):
                                     "frac": gemm_total / (gemm_ms * 1e-3) / 1e12 / peaks["bf16_sust"],
                                     "flops_per_step": gemm_total},
             "roofline_reduce_update": roof_update,
+            "step_ms": {"median": float(np.median(step_ms)), "p10": float(np.percentile(step_ms, 10)),
+                        "p90": float(np.percentile(step_ms, 90))},
             "phases_ms_per_step": per_step,
             "gpu_launches": int(launches),
             "cpu_baseline": cpu,

@@ -319,7 +319,7 @@ hs_status plan_dense(hs_ctx* c, TcGemmParams* p, int epi, const __nv_bfloat16* a
                      int64_t ldz) {
   const char* why = nullptr;
   std::memset(p, 0, sizeof(*p));
-  bool ok = tc_make_kmajor_map(&p->tmA[0], TcOperand{a, a_rows, a_cols, lda}, kTcBM, &why);
+  bool ok = tc_make_kmajor_map(&p->tmA[0], TcOperand{a, a_rows, a_cols, lda}, kTcBoxA, &why);
   ok = ok && (b_mn ? tc_make_mnmajor_map(&p->tmB[0], TcOperand{b, b_rows, b_cols, ldb}, &why)
                    : tc_make_kmajor_map(&p->tmB[0], TcOperand{b, b_rows, b_cols, ldb}, kTcBoxB, &why));
   ok = ok && tc_make_store_map(&p->tmD[0], d, d_f32, Mdim, n_store, ldd, &why);

@@ -100,7 +100,9 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
 #pragma unroll
             for (int j = 0; j < BM / 64; ++j) tma_load_2d(a_dst + j * MN_CHUNK, ta, c.tm * BM + 64 * j, k0, fb);
           } else {
-            tma_load_2d(a_dst, ta, k0, c.tm * BM, fb);
+#pragma unroll
+            for (int j = 0; j < BM / kTcBoxA; ++j)
+              tma_load_2d(a_dst + j * (kTcBoxA * BK * 2), ta, k0, c.tm * BM + kTcBoxA * j, fb);
           }
           if (B_MN) {
 #pragma unroll

@@ -64,6 +64,7 @@ constexpr int kTcStagingBytes = 4 * 2 * 32 * 128;   // 4 epilogue warps x 2 buff
 constexpr int kTcSmemBytes =
     kTcStages * (kTcBM + kTcBN) * kTcBK * 2 + kTcStagingBytes + 1024 /*align*/ + 256 /*barriers*/;
 
+constexpr int kTcBoxA = 64;    // rows of a K-major A box (a 128-row A tile is two boxes)
 constexpr int kTcBoxB = 128;   // rows of a K-major B box (the 256-row B tile is two boxes)
 
 // Kernel form: one SM per 128 x 256 tile, or an SM pair (cluster of 2, tcgen05 cta_group::2) per

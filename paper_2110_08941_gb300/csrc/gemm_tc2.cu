@@ -159,11 +159,11 @@ __global__ void __launch_bounds__(kThreads2, 1) tc_gemm_pair_kernel(const __grid
           const int k0 = kb * BK;
           const uint32_t a_dst = smem_u32(smem + s * STAGE2);
           const uint32_t b_dst = a_dst + A_HALF;
-          if (A_MN) {
+          // the A half is two 64-row (K-major) or 64-column (MN-major) boxes of 8 KB
 #pragma unroll
-            for (int j = 0; j < HM / 64; ++j) tma_load_2d_pair(a_dst + j * MN_CHUNK, ta, m0 + 64 * j, k0, fb);
-          } else {
-            tma_load_2d_pair(a_dst, ta, k0, m0, fb);
+          for (int j = 0; j < HM / 64; ++j) {
+            if (A_MN) tma_load_2d_pair(a_dst + j * MN_CHUNK, ta, m0 + 64 * j, k0, fb);
+            else tma_load_2d_pair(a_dst + j * MN_CHUNK, ta, k0, m0 + 64 * j, fb);
           }
           if (B_MN) {
 #pragma unroll

@@ -71,7 +71,7 @@ hs_status build_tc_static(hs_ctx* c) {
     std::memset(&f, 0, sizeof(f));
     hs::TcOperand a{reinterpret_cast<const __nv_bfloat16*>(c->d_act[l]), c->N, ly.in, ly.in};
     hs::TcOperand b{c->d_shadow + ly.w_off, ly.out, ly.in, ly.in};
-    if (!hs::tc_make_kmajor_map(&f.tmA[0], a, hs::kTcBM, &why) ||
+    if (!hs::tc_make_kmajor_map(&f.tmA[0], a, hs::kTcBoxA, &why) ||
         !hs::tc_make_kmajor_map(&f.tmB[0], b, hs::kTcBoxB, &why))
       return fail(c, HS_ERR_CUDA, why);
     f.num_kb[0] = (ly.in + hs::kTcBK - 1) / hs::kTcBK;
@@ -92,7 +92,7 @@ hs_status build_tc_static(hs_ctx* c) {
     std::memset(&d, 0, sizeof(d));
     hs::TcOperand da{reinterpret_cast<const __nv_bfloat16*>(c->delta_buf(l)), c->N, ly.out, c->delta_ld(l)};
     hs::TcOperand db{c->d_shadow + ly.w_off, ly.out, ly.in, ly.in};
-    if (!hs::tc_make_kmajor_map(&d.tmA[0], da, hs::kTcBM, &why) || !hs::tc_make_mnmajor_map(&d.tmB[0], db, &why))
+    if (!hs::tc_make_kmajor_map(&d.tmA[0], da, hs::kTcBoxA, &why) || !hs::tc_make_mnmajor_map(&d.tmB[0], db, &why))
       return fail(c, HS_ERR_CUDA, why);
     d.num_kb[0] = (ly.out + hs::kTcBK - 1) / hs::kTcBK;
     d.groups = 1;
@@ -1069,7 +1069,7 @@ hs_status hs_debug_gemm_bf16(int32_t mode, int32_t M, int32_t N, int32_t K, cons
     plans.emplace_back();
     hs::TcGemmParams& p = plans.back();
     std::memset(&p, 0, sizeof(p));
-    bool ok = hs::tc_make_kmajor_map(&p.tmA[0], hs::TcOperand{pa, M, K, lda}, hs::kTcBM, &why);
+    bool ok = hs::tc_make_kmajor_map(&p.tmA[0], hs::TcOperand{pa, M, K, lda}, hs::kTcBoxA, &why);
     if (mode == HS_GEMM_DGRAD) ok = ok && hs::tc_make_mnmajor_map(&p.tmB[0], hs::TcOperand{pb, K, N, ldb}, &why);
     else ok = ok && hs::tc_make_kmajor_map(&p.tmB[0], hs::TcOperand{pb, N, K, ldb}, hs::kTcBoxB, &why);
     if (!ok) return fail(nullptr, HS_ERR_INVALID_ARG, why);
