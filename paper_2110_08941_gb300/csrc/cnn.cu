@@ -260,6 +260,7 @@ hs_status cnn_build_wgrad_plan(hs_ctx* c, int layer, const __nv_bfloat16* a, int
                                const __nv_bfloat16* b, int b_cols, int64_t ldb, int64_t rows_per_sample) {
   const char* why = nullptr;
   CnnWgrad& wg = c->cnn_wgrad[layer];
+  const ConvLayer* conv = layer < 3 ? &c->convs[layer] : nullptr;
   wg.plans.clear();
   wg.rows_out = a_cols;
   wg.K = b_cols;
@@ -267,7 +268,12 @@ hs_status cnn_build_wgrad_plan(hs_ctx* c, int layer, const __nv_bfloat16* a, int
   const int tiles = (int)(((a_cols + kTcBM - 1) / kTcBM) * ((b_cols + kTcBN - 1) / kTcBN));
   const int64_t total_rows = (int64_t)c->N * rows_per_sample;
   const int64_t target_groups = std::max<int64_t>(1, (2LL * c->num_sms + tiles - 1) / tiles);
-  const int64_t chunk = std::max<int64_t>(512, round_up((total_rows + target_groups - 1) / target_groups, kTcBK));
+  // chunks hold whole samples (so an implicit-patch map can start at a chunk's first image) and
+  // whole 64-row k-blocks
+  const int64_t align = rows_per_sample % kTcBK == 0 ? rows_per_sample
+                      : kTcBK % rows_per_sample == 0 ? kTcBK : rows_per_sample * kTcBK;
+  const int64_t chunk = std::max<int64_t>(round_up(512, align),
+                                          round_up((total_rows + target_groups - 1) / target_groups, align));
   std::vector<std::pair<int64_t, int64_t>> ranges;
   std::vector<int32_t> begin;
   for (int m = 0; m < c->M; ++m) {
@@ -286,10 +292,20 @@ hs_status cnn_build_wgrad_plan(hs_ctx* c, int layer, const __nv_bfloat16* a, int
     for (int g = 0; g < ng; ++g) {
       const auto& rg = ranges[g0 + g];
       float* dg = wg.d_partial + (int64_t)(g0 + g) * wg.rows_out * wg.ldp;
-      if (!tc_make_mnmajor_map(&p.tmA[g], TcOperand{a + rg.first * lda, rg.second, a_cols, lda}, &why) ||
-          !tc_make_mnmajor_map(&p.tmB[g], TcOperand{b + rg.first * ldb, rg.second, b_cols, ldb}, &why) ||
-          !tc_make_store_map(&p.tmD[g], dg, true, a_cols, b_cols, wg.ldp, &why))
-        return fail(c, HS_ERR_CUDA, why);
+      bool ok = tc_make_mnmajor_map(&p.tmA[g], TcOperand{a + rg.first * lda, rg.second, a_cols, lda}, &why) &&
+                tc_make_store_map(&p.tmD[g], dg, true, a_cols, b_cols, wg.ldp, &why);
+      if (conv && conv->implicit) {
+        // B = the implicit patch rows of the chunk's samples, read from the layer's input
+        const int64_t img0 = rg.first / rows_per_sample;
+        const int64_t imgs = (rg.second + rows_per_sample - 1) / rows_per_sample;
+        const __nv_bfloat16* in = reinterpret_cast<const __nv_bfloat16*>(c->d_cact[layer - 1]) +
+                                  img0 * conv->hin * conv->win * conv->cin;
+        ok = ok && tc_make_conv_map(&p.tmB[g], in, imgs, conv->hin, conv->win, conv->cin, conv->hout, conv->wout,
+                                    conv->stride, &why);
+      } else {
+        ok = ok && tc_make_mnmajor_map(&p.tmB[g], TcOperand{b + rg.first * ldb, rg.second, b_cols, ldb}, &why);
+      }
+      if (!ok) return fail(c, HS_ERR_CUDA, why);
       p.num_kb[g] = (int32_t)((rg.second + kTcBK - 1) / kTcBK);
     }
     p.groups = ng;
@@ -301,6 +317,11 @@ hs_status cnn_build_wgrad_plan(hs_ctx* c, int layer, const __nv_bfloat16* a, int
     p.epi = kTcEpiStoreF32;
     p.a_mn = 1;
     p.b_mn = 1;
+    if (conv && conv->implicit) {
+      p.conv_b = 1;
+      p.conv = tc_conv_geom(conv->cin, conv->hout, conv->wout, conv->stride);
+      if (!tc_make_mnmajor_map(&p.tmOnes, TcOperand{c->d_ones, 64, 64, 64}, &why)) return fail(c, HS_ERR_CUDA, why);
+    }
     p.D = wg.d_partial + (int64_t)g0 * wg.rows_out * wg.ldp;
     p.ldd = wg.ldp;
     p.d_gstride = (int64_t)wg.rows_out * wg.ldp;
@@ -313,13 +334,22 @@ hs_status cnn_build_wgrad_plan(hs_ctx* c, int layer, const __nv_bfloat16* a, int
 
 namespace {
 
+// A is K-major [a_rows][a_cols], or (conv != nullptr) the implicit patch rows of that convolution.
 hs_status plan_dense(hs_ctx* c, TcGemmParams* p, int epi, const __nv_bfloat16* a, int64_t a_rows, int a_cols,
                      int64_t lda, const __nv_bfloat16* b, int64_t b_rows, int b_cols, int64_t ldb, bool b_mn,
                      void* d, bool d_f32, int Mdim, int Ndim, int n_store, int64_t ldd, const __nv_bfloat16* z,
-                     int64_t ldz) {
+                     int64_t ldz, const ConvLayer* conv = nullptr) {
   const char* why = nullptr;
   std::memset(p, 0, sizeof(*p));
-  bool ok = tc_make_kmajor_map(&p->tmA[0], TcOperand{a, a_rows, a_cols, lda}, kTcBoxA, &why);
+  bool ok;
+  if (conv) {
+    ok = tc_make_conv_map(&p->tmA[0], a, c->N, conv->hin, conv->win, conv->cin, conv->hout, conv->wout,
+                          conv->stride, &why);
+    p->conv_a = 1;
+    p->conv = tc_conv_geom(conv->cin, conv->hout, conv->wout, conv->stride);
+  } else {
+    ok = tc_make_kmajor_map(&p->tmA[0], TcOperand{a, a_rows, a_cols, lda}, kTcBoxA, &why);
+  }
   ok = ok && (b_mn ? tc_make_mnmajor_map(&p->tmB[0], TcOperand{b, b_rows, b_cols, ldb}, &why)
                    : tc_make_kmajor_map(&p->tmB[0], TcOperand{b, b_rows, b_cols, ldb}, kTcBoxB, &why));
   ok = ok && tc_make_store_map(&p->tmD[0], d, d_f32, Mdim, n_store, ldd, &why);
@@ -348,6 +378,13 @@ hs_status plan_dense(hs_ctx* c, TcGemmParams* p, int epi, const __nv_bfloat16* a
 hs_status cnn_build_static(hs_ctx* c) {
   const char* why = nullptr;
   if (!tc_init_driver(&why)) return fail(c, HS_ERR_CUDA, why);
+  {
+    // the ones column of the implicit patch rows: [64][64] bf16 with column 0 = 1
+    std::vector<__nv_bfloat16> ones(64 * 64, __float2bfloat16(0.f));
+    for (int r = 0; r < 64; ++r) ones[r * 64] = __float2bfloat16(1.f);
+    cudaError_t e = cudaMemcpy(c->d_ones, ones.data(), sizeof(__nv_bfloat16) * ones.size(), cudaMemcpyHostToDevice);
+    if (e != cudaSuccess) return cuda_fail(c, e, "ones tile");
+  }
   const int N = c->N;
   auto bf = [](void* p) { return reinterpret_cast<const __nv_bfloat16*>(p); };
   c->tc_fwd.assign(4, TcGemmParams{});
@@ -356,8 +393,10 @@ hs_status cnn_build_static(hs_ctx* c) {
     const ConvLayer& L = c->convs[k];
     const __nv_bfloat16* wb = c->d_wperm[k];
     const int64_t ldw = L.Kp;
-    hs_status st = plan_dense(c, &c->tc_fwd[k], kTcEpiBiasReluBf16, bf(c->d_col[k]), L.rows, L.K, L.Kp, wb, L.cout,
-                              L.K, ldw, false, c->d_cact[k], false, (int)L.rows, L.cout, L.cout, L.cout, nullptr, 0);
+    const __nv_bfloat16* a = L.implicit ? bf(c->d_cact[k - 1]) : bf(c->d_col[k]);
+    hs_status st = plan_dense(c, &c->tc_fwd[k], kTcEpiBiasReluBf16, a, L.rows, L.K, L.Kp, wb, L.cout, L.K, ldw,
+                              false, c->d_cact[k], false, (int)L.rows, L.cout, L.cout, L.cout, nullptr, 0,
+                              L.implicit ? &L : nullptr);
     if (st != HS_OK) return st;
   }
   // fully connected layer on the pooled features
@@ -421,6 +460,8 @@ hs_status cnn_step(hs_ctx* c, float* params, const float* x, const int32_t* y, c
           im2col_nchw_kernel<float, false><<<blocks_for(n_items, T), T, 0, s>>>(
               x, N, L[0].cin, L[0].hin, L[0].win, L[0].hout, L[0].wout, L[0].stride,
               reinterpret_cast<float*>(c->d_col[0]), L[0].Kp);
+      } else if (L[k].implicit) {
+        // the forward product reads the patch rows straight from d_cact[k - 1]
       } else {
         if (bf16)
           im2col_nhwc_vec8_kernel<<<blocks_for(L[k].rows * 9 * (L[k].cin / 8), T), T, 0, s>>>(
@@ -431,7 +472,7 @@ hs_status cnn_step(hs_ctx* c, float* params, const float* x, const int32_t* y, c
               reinterpret_cast<const float*>(c->d_cact[k - 1]), N, L[k].cin, L[k].hin, L[k].win, L[k].hout,
               L[k].wout, L[k].stride, reinterpret_cast<float*>(c->d_col[k]), L[k].Kp);
       }
-      ph.launched();
+      if (!L[k].implicit) ph.launched();
       if (bf16) {
         TcGemmParams& f = c->tc_fwd[k];
         f.bias = params + L[k].b_off;

@@ -21,6 +21,7 @@ struct ConvLayer {
   int K, Kp;          // Cin*9 and its row stride in the bf16 patch buffer (multiple of 8)
   int64_t w_off, b_off;
   int64_t rows;       // N * hout * wout
+  bool implicit;      // bf16: the products read the patch rows straight from the input (no col buffer)
 };
 
 inline int64_t round_up(int64_t v, int64_t m) { return (v + m - 1) / m * m; }
@@ -144,6 +145,7 @@ struct hs_ctx {
   void* d_dA[3] = {nullptr, nullptr, nullptr};
   float* d_dcol = nullptr;
   __nv_bfloat16* d_wperm[3] = {nullptr, nullptr, nullptr};   // bf16 [Cout][Kp], tap-major columns
+  __nv_bfloat16* d_ones = nullptr;                           // bf16 [64][64], column 0 ones (implicit convs)
   int32_t* d_row_off[4] = {nullptr, nullptr, nullptr, nullptr};
   hs::ChunkTable cnn_chunks[4];
   hs::CnnWgrad cnn_wgrad[4];

@@ -101,12 +101,30 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
             for (int j = 0; j < BM / 64; ++j) tma_load_2d(a_dst + j * MN_CHUNK, ta, c.tm * BM + 64 * j, k0, fb);
           } else {
 #pragma unroll
-            for (int j = 0; j < BM / kTcBoxA; ++j)
-              tma_load_2d(a_dst + j * (kTcBoxA * BK * 2), ta, k0, c.tm * BM + kTcBoxA * j, fb);
+            for (int j = 0; j < BM / kTcBoxA; ++j) {
+              if (p.conv_a) {
+                int cc[4];
+                conv_box_coords(p.conv, c.tm * BM + kTcBoxA * j, k0, cc);
+                tma_load_4d(a_dst + j * (kTcBoxA * BK * 2), ta, cc, fb);
+              } else {
+                tma_load_2d(a_dst + j * (kTcBoxA * BK * 2), ta, k0, c.tm * BM + kTcBoxA * j, fb);
+              }
+            }
           }
           if (B_MN) {
 #pragma unroll
-            for (int j = 0; j < BN / 64; ++j) tma_load_2d(b_dst + j * MN_CHUNK, tb, c.tn * BN + 64 * j, k0, fb);
+            for (int j = 0; j < BN / 64; ++j) {
+              const int col = c.tn * BN + 64 * j;
+              if (!p.conv_b) {
+                tma_load_2d(b_dst + j * MN_CHUNK, tb, col, k0, fb);
+              } else if (col < p.conv.ones_col) {
+                int cc[4];
+                conv_box_coords(p.conv, k0, col, cc);
+                tma_load_4d(b_dst + j * MN_CHUNK, tb, cc, fb);
+              } else {
+                tma_load_2d(b_dst + j * MN_CHUNK, &p.tmOnes, col - p.conv.ones_col, 0, fb);
+              }
+            }
           } else {
 #pragma unroll
             for (int j = 0; j < BN / kTcBoxB; ++j)
@@ -301,6 +319,54 @@ static bool encode_2d(CUtensorMap* tm, const void* base, uint64_t inner, uint64_
 bool tc_make_kmajor_map(CUtensorMap* tm, const TcOperand& op, int box_rows, const char** why) {
   return encode_2d(tm, op.base, (uint64_t)op.cols, (uint64_t)op.rows, (uint64_t)op.ld * 2, kTcBK, (uint32_t)box_rows,
                    why);
+}
+
+bool tc_conv_implicit_ok(int C, int Ho, int Wo, int stride) {
+  if (C < 64 || C % 64 || Wo < 1 || Ho < 1 || 64 % Wo || stride < 1 || stride > 2) return false;
+  const int hw = Ho * Wo;
+  if (hw % 64 && 64 % hw) return false;
+  const int hb = hw >= 64 ? 64 / Wo : Ho;   // output rows a 64-pixel box covers
+  return stride * Wo <= 256 && stride * hb <= 256;
+}
+
+TcConvGeom tc_conv_geom(int C, int Ho, int Wo, int stride) {
+  TcConvGeom g{};
+  g.cblocks = C / 64;
+  g.Wo = Wo;
+  g.hw = Ho * Wo;
+  g.stride = stride;
+  g.ones_col = 9 * C;
+  return g;
+}
+
+bool tc_make_conv_map(CUtensorMap* tm, const __nv_bfloat16* base, int64_t images, int H, int W, int C, int Ho,
+                      int Wo, int stride, const char** why) {
+  if (!g_encode && !tc_init_driver(why)) return false;
+  if (!tc_conv_implicit_ok(C, Ho, Wo, stride) || images < 1) {
+    *why = "convolution geometry not supported by the implicit patch rows";
+    return false;
+  }
+  if ((reinterpret_cast<uintptr_t>(base) & 15u) != 0) {
+    *why = "TMA operand base is not 16-byte aligned";
+    return false;
+  }
+  const int hw = Ho * Wo;
+  const uint32_t hb = hw >= 64 ? (uint32_t)(64 / Wo) : (uint32_t)Ho;
+  const uint32_t nb = hw >= 64 ? 1u : (uint32_t)(64 / hw);
+  // dims innermost first: channels, input columns, input rows, images; a box traverses `stride`
+  // input columns / rows per output pixel and loads ceil(extent / stride) of them
+  cuuint64_t dims[4] = {(cuuint64_t)C, (cuuint64_t)W, (cuuint64_t)H, (cuuint64_t)images};
+  cuuint64_t strides[3] = {(cuuint64_t)C * 2, (cuuint64_t)W * C * 2, (cuuint64_t)H * W * C * 2};
+  cuuint32_t box[4] = {64, (cuuint32_t)(stride * Wo), (cuuint32_t)stride * hb, nb};
+  cuuint32_t estr[4] = {1, (cuuint32_t)stride, (cuuint32_t)stride, 1};
+  CUresult r = g_encode(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<__nv_bfloat16*>(base), dims, strides,
+                        box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) {
+    *why = "cuTensorMapEncodeTiled rejected the convolution operand";
+    return false;
+  }
+  return true;
 }
 
 bool tc_make_mnmajor_map(CUtensorMap* tm, const TcOperand& op, const char** why) {

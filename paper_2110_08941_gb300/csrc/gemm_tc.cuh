@@ -17,16 +17,36 @@ enum TcEpi : int32_t {
   kTcEpiStoreF32 = 3,       // D fp32 = acc                                  (per-worker weight gradient)
 };
 
+// Implicit patch rows of a 3x3, padding-1 convolution over an NHWC bf16 input with C % 64 == 0:
+// row r = (n, ho, wo) of the output grid, column tap * C + ci (tap = kh * 3 + kw), read straight
+// from the input by 4-D TMA boxes of 64 output pixels x 64 channels (padding = the zero fill of
+// out-of-range coordinates, the stride = the box's traversal stride).  Rows are grouped in blocks
+// of 64, which must cover whole output rows (Wo divides 64) and whole images or parts of one
+// (Ho * Wo a multiple or a divisor of 64).
+struct TcConvGeom {
+  int32_t cblocks;    // C / 64
+  int32_t Wo, hw;     // output width, output pixels per image
+  int32_t stride;
+  int32_t ones_col;   // as the B operand: first column past the 9 * C patch columns, which holds
+                      // ones (the bias gradient's column); columns past it read zeros
+};
+
 // D[Mdim x n_store] (row-major, leading dimension ldd) = A[Mdim x K] * B[K x Ndim] + epilogue.
 // Operands are bf16 in global memory and are described by TMA tensor maps:
 //   K-major   ("row-major with K contiguous"): A as [M rows][K], B as [N rows][K]
 //   MN-major  ("K rows, M or N contiguous"):   A as [K rows][M], B as [K rows][N]
 // Grouped launches run `groups` independent products that share Mdim/Ndim but each has its own
 // A/B maps (a worker's row segment) and K extent; group g writes D + g * d_gstride.
+// conv_a: A (K-major) is a convolution's implicit patch rows, tmA[g] a map from tc_make_conv_map.
+// conv_b: B (MN-major) is the implicit patch rows of the group's samples (tmB[g] a conv map over
+// them), and tmOnes supplies the ones column at conv.ones_col.
 struct TcGemmParams {
   CUtensorMap tmA[kTcMaxGroups];
   CUtensorMap tmB[kTcMaxGroups];
   CUtensorMap tmD[kTcMaxGroups];   // output (store) maps: box of 32 rows x 128 bytes
+  CUtensorMap tmOnes;              // MN-major [64][64] bf16, column 0 ones, the rest zero (conv_b)
+  TcConvGeom conv;
+  int32_t conv_a, conv_b;
   int32_t num_kb[kTcMaxGroups];
   int32_t groups;
   int32_t Mdim, Ndim, n_store;
@@ -54,6 +74,12 @@ bool tc_init_driver(const char** why);
 bool tc_make_kmajor_map(CUtensorMap* tm, const TcOperand& op, int box_rows, const char** why);
 // MN-major operand: matrix [K rows][MN] with MN contiguous; box = 64 (MN) x 64 (K).
 bool tc_make_mnmajor_map(CUtensorMap* tm, const TcOperand& op, const char** why);
+// Implicit patch rows of a convolution (see TcConvGeom): input NHWC bf16 [images][H][W][C] at
+// `base`, output grid Ho x Wo.  Box: 64 channels x 64 output pixels.
+bool tc_conv_implicit_ok(int C, int Ho, int Wo, int stride);
+bool tc_make_conv_map(CUtensorMap* tm, const __nv_bfloat16* base, int64_t images, int H, int W, int C, int Ho,
+                      int Wo, int stride, const char** why);
+TcConvGeom tc_conv_geom(int C, int Ho, int Wo, int stride);
 // Output matrix [rows][cols] (row stride ld elements, fp32 or bf16) for TMA stores of 32-row x
 // 128-byte boxes; rows >= `rows` and columns >= `cols` of a box are not written.
 bool tc_make_store_map(CUtensorMap* tm, void* base, bool fp32, int64_t rows, int64_t cols, int64_t ld,

@@ -57,6 +57,14 @@ __device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const CUtensorMap
       ::"r"(dst), "l"(reinterpret_cast<uint64_t>(tm)), "r"(c0), "r"(c1), "r"(leader_bar)
       : "memory");
 }
+__device__ __forceinline__ void tma_load_4d_pair(uint32_t dst, const CUtensorMap* tm, const int (&c)[4],
+                                                 uint32_t leader_bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.4d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes "
+      "[%0], [%1, {%2, %3, %4, %5}], [%6];"
+      ::"r"(dst), "l"(reinterpret_cast<uint64_t>(tm)), "r"(c[0]), "r"(c[1]), "r"(c[2]), "r"(c[3]), "r"(leader_bar)
+      : "memory");
+}
 __device__ __forceinline__ void tmem_alloc_pair(uint32_t dst_smem, uint32_t ncols) {
   asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst_smem), "r"(ncols)
                : "memory");
@@ -162,12 +170,30 @@ __global__ void __launch_bounds__(kThreads2, 1) tc_gemm_pair_kernel(const __grid
           // the A half is two 64-row (K-major) or 64-column (MN-major) boxes of 8 KB
 #pragma unroll
           for (int j = 0; j < HM / 64; ++j) {
-            if (A_MN) tma_load_2d_pair(a_dst + j * MN_CHUNK, ta, m0 + 64 * j, k0, fb);
-            else tma_load_2d_pair(a_dst + j * MN_CHUNK, ta, k0, m0 + 64 * j, fb);
+            if (A_MN) {
+              tma_load_2d_pair(a_dst + j * MN_CHUNK, ta, m0 + 64 * j, k0, fb);
+            } else if (p.conv_a) {
+              int cc[4];
+              conv_box_coords(p.conv, m0 + 64 * j, k0, cc);
+              tma_load_4d_pair(a_dst + j * MN_CHUNK, ta, cc, fb);
+            } else {
+              tma_load_2d_pair(a_dst + j * MN_CHUNK, ta, k0, m0 + 64 * j, fb);
+            }
           }
           if (B_MN) {
 #pragma unroll
-            for (int j = 0; j < HN / 64; ++j) tma_load_2d_pair(b_dst + j * MN_CHUNK, tb, n0 + 64 * j, k0, fb);
+            for (int j = 0; j < HN / 64; ++j) {
+              const int col = n0 + 64 * j;
+              if (!p.conv_b) {
+                tma_load_2d_pair(b_dst + j * MN_CHUNK, tb, col, k0, fb);
+              } else if (col < p.conv.ones_col) {
+                int cc[4];
+                conv_box_coords(p.conv, k0, col, cc);
+                tma_load_4d_pair(b_dst + j * MN_CHUNK, tb, cc, fb);
+              } else {
+                tma_load_2d_pair(b_dst + j * MN_CHUNK, &p.tmOnes, col - p.conv.ones_col, 0, fb);
+              }
+            }
           } else {
             tma_load_2d_pair(b_dst, tb, k0, n0, fb);
           }

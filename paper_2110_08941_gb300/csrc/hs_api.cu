@@ -294,6 +294,7 @@ void free_all(hs_ctx* c) {
   for (int k = 0; k < 3; ++k) { f(c->d_col[k]); f(c->d_cact[k]); f(c->d_dA[k]); }
   f(c->d_pooled); f(c->d_dpooled); f(c->d_dcol);
   for (int k = 0; k < 3; ++k) f(c->d_wperm[k]);
+  f(c->d_ones);
   for (int k = 0; k < 4; ++k) {
     f(c->d_row_off[k]); f(c->cnn_chunks[k].d_chunks); f(c->cnn_chunks[k].d_begin);
     f(c->cnn_wgrad[k].d_partial); f(c->cnn_wgrad[k].d_chunk_begin);
@@ -606,6 +607,10 @@ hs_status hs_init(const hs_model_desc* model, int32_t M, const double* compute_w
       L.b_off = off;
       off += L.cout;
       L.rows = (int64_t)global_batch * L.hout * L.wout;
+      // Implicit patch rows where the geometry allows (HS_CONV_IMPLICIT=0 materialises them all)
+      const char* imp = getenv("HS_CONV_IMPLICIT");
+      L.implicit = bf16 && k > 0 && !(imp && !strcmp(imp, "0")) &&
+                   hs::tc_conv_implicit_ok(L.cin, L.hout, L.wout, L.stride);
       c->convs.push_back(L);
       h = L.hout;
       w = L.wout;
@@ -653,7 +658,7 @@ hs_status hs_init(const hs_model_desc* model, int32_t M, const double* compute_w
     int64_t dcol = 0;
     for (int k = 0; k < 3; ++k) {
       const ConvLayer& L = c->convs[k];
-      chk(dalloc(c, &c->d_col[k], es * (size_t)L.rows * L.Kp));
+      if (!L.implicit) chk(dalloc(c, &c->d_col[k], es * (size_t)L.rows * L.Kp));
       chk(dalloc(c, &c->d_cact[k], es * (size_t)L.rows * L.cout));
       chk(dalloc(c, &c->d_dA[k], es * (size_t)L.rows * L.cout));
       if (k > 0) dcol = std::max<int64_t>(dcol, L.rows * L.K);
@@ -661,9 +666,11 @@ hs_status hs_init(const hs_model_desc* model, int32_t M, const double* compute_w
     chk(dalloc(c, &c->d_pooled, es * N * c3));
     chk(dalloc(c, &c->d_dpooled, sizeof(float) * N * c3));
     chk(dalloc(c, &c->d_dcol, sizeof(float) * (size_t)dcol));
-    if (bf16)
+    if (bf16) {
       for (int k = 0; k < 3; ++k)
         chk(dalloc(c, &c->d_wperm[k], sizeof(__nv_bfloat16) * (size_t)c->convs[k].cout * c->convs[k].Kp));
+      chk(dalloc(c, &c->d_ones, sizeof(__nv_bfloat16) * 64 * 64));
+    }
     delta_elems = N * (size_t)c->Cp;
     for (int k = 0; k < 4; ++k) {
       const bool fc = (k == 3);

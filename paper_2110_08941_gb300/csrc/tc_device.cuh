@@ -61,6 +61,28 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* tm,
       ::"r"(dst), "l"(reinterpret_cast<uint64_t>(tm)), "r"(c0), "r"(c1), "r"(bar)
       : "memory");
 }
+__device__ __forceinline__ void tma_load_4d(uint32_t dst, const CUtensorMap* tm, const int (&c)[4], uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.4d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4, %5}], "
+      "[%6];"
+      ::"r"(dst), "l"(reinterpret_cast<uint64_t>(tm)), "r"(c[0]), "r"(c[1]), "r"(c[2]), "r"(c[3]), "r"(bar)
+      : "memory");
+}
+// Coordinates (channel, input column, input row, image) of the 4-D box holding implicit patch rows
+// row..row+63 (row a multiple of 64) and patch columns kcol..kcol+63 (kcol a multiple of 64 below
+// 9 * C): tap = kcol / C, channels kcol % C onwards, input pixel (stride * ho + kh - 1, kw - 1) for
+// the block's first output pixel (ho, 0).
+__device__ __forceinline__ void conv_box_coords(const TcConvGeom& g, int row, int kcol, int (&c)[4]) {
+  const int blk = kcol >> 6;
+  const int tap = blk / g.cblocks;
+  const int cb = blk - tap * g.cblocks;
+  const int img = row / g.hw;
+  const int ho = (row - img * g.hw) / g.Wo;
+  c[0] = cb * 64;
+  c[1] = tap % 3 - 1;
+  c[2] = g.stride * ho + tap / 3 - 1;
+  c[3] = img;
+}
 __device__ __forceinline__ void tma_store_2d(const CUtensorMap* tm, uint32_t src, int c0, int c1) {
   asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%1, %2}], [%3];"
                ::"l"(reinterpret_cast<uint64_t>(tm)), "r"(c0), "r"(c1), "r"(src)

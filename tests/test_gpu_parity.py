@@ -11,6 +11,7 @@ import functools
 
 import numpy as np
 import pytest
+import torch
 
 import synth
 import paper_2110_08941_gb300 as hs
@@ -185,6 +186,10 @@ CNN_EDGE = [
     ((3, 9, 7, 8, 16, 24, 5), 7, 3, [1.0, 2.0, 4.0]),
     ((2, 6, 6, 16, 8, 8, 3), 4, 4, None),
     ((3, 16, 16, 32, 32, 64, 10), 33, 2, [1.0, 5.0]),
+    # implicit patch rows (bf16): 8x8 and 4x4 output grids (several images per 64-row block), 13 images
+    ((3, 16, 16, 64, 128, 64, 7), 13, 3, [1.0, 2.0, 3.5]),
+    # 8x16 and 4x8 output grids, two workers
+    ((3, 16, 32, 64, 64, 64, 5), 9, 2, [2.0, 1.0]),
 ]
 
 
@@ -240,3 +245,38 @@ def test_fused_sync_headline_workload_gradient():
                     hs.HS_SYNC_CP_WEIGHTED, fused=True)
     assert rel(b["g_first"], a["g_first"]) <= 5e-3
     assert a["worker_losses_first"] == b["worker_losses_first"]
+
+
+# ------------------------------------------------------------------ implicit-GEMM convolutions
+@pytest.mark.parametrize("name", [synth.CFG4])
+def test_implicit_conv_is_bit_identical_to_materialised_patches(name, monkeypatch):
+    """The convolutions' products read their patch rows straight from the NHWC input (4-D TMA boxes)
+    or from materialised patch rows (HS_CONV_IMPLICIT=0): same operand values in the same k-block
+    order, so theta, losses and per-worker gradients agree bit for bit.  The implicit context holds no
+    patch buffers for the second and third convolutions."""
+    wl, x, y, theta0, w = _inputs(name)
+    out = {}
+    for mode in ("1", "0"):
+        monkeypatch.setenv("HS_CONV_IMPLICIT", mode)
+        torch.cuda.synchronize()
+        free0 = torch.cuda.mem_get_info()[0]
+        ctx = hs.hs_init(wl.arch, wl.dims, wl.workers, wl.global_batch, compute_weights=w, precision=hs.HS_BF16)
+        used = free0 - torch.cuda.mem_get_info()[0]
+        try:
+            hs.hs_set_debug(ctx, True)
+            p = torch.tensor(theta0, device="cuda")
+            xd, yd = torch.from_numpy(x).cuda(), torch.from_numpy(y).cuda()
+            losses = [hs.hs_step(ctx, p, xd, yd, None, wl.lr) for _ in range(3)]
+            slabs = torch.empty(wl.workers, ctx.P, device="cuda")
+            hs.hs_debug_grads(ctx, None, slabs)
+            torch.cuda.synchronize()
+            out[mode] = (p.cpu(), losses, slabs.cpu(), used)
+        finally:
+            ctx.close()
+    assert torch.equal(out["1"][0], out["0"][0])
+    assert out["1"][1] == out["0"][1]
+    assert torch.equal(out["1"][2], out["0"][2])
+    # patch rows of conv2 (N*16*16 x 584) and conv3 (N*8*8 x 1160), bf16, not allocated
+    n = wl.global_batch
+    saved = 2 * (n * 256 * 584 + n * 64 * 1160)
+    assert out["0"][3] - out["1"][3] >= 0.9 * saved
