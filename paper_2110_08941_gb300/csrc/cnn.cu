@@ -227,6 +227,26 @@ __global__ void permute_weights_kernel(const float* __restrict__ w, int cout, in
   wp[idx] = __float2bfloat16_rn(v);
 }
 
+// bf16 weights of the four sub-pixel classes of a stride-2 convolution's input gradient (see
+// TcConvGeom): class (ph, pw) = 2 * ph + pw holds [taps x Cout][Cin], row t * Cout + co, where the
+// class's row taps are kh = 1 (ph = 0) or kh = 0, 2 (ph = 1) in that order, columns likewise, and
+// t = th * (number of column taps) + tw.  Classes hold 1, 2, 2, 4 taps and sit back to back.
+__global__ void permute_weights_subpixel_kernel(const float* __restrict__ w, int cout, int cin,
+                                                __nv_bfloat16* __restrict__ wc) {
+  const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= (int64_t)cout * cin * 9) return;
+  const int tap = (int)(idx % 9);
+  const int ci = (int)((idx / 9) % cin);
+  const int co = (int)(idx / (9 * (int64_t)cin));
+  const int kh = tap / 3, kw = tap % 3;
+  const int ph = kh != 1, pw = kw != 1;
+  const int th = (ph && kh == 2) ? 1 : 0, tw = (pw && kw == 2) ? 1 : 0;
+  const int t = th * (pw ? 2 : 1) + tw;
+  const int cls = 2 * ph + pw;
+  const int64_t class_off = (cls == 0 ? 0 : cls == 1 ? 1 : cls == 2 ? 3 : 5) * (int64_t)cout * cin;
+  wc[class_off + ((int64_t)t * cout + co) * cin + ci] = __float2bfloat16_rn(w[idx]);
+}
+
 // slabs[m][w_off + co*K + k] = sum over worker m's chunks (in order) of partial[chunk][co][k'], where
 // k' = k for the fully connected layer (cin = 0) and, for a convolution, the tap-major column of
 // theta's (ci, tap) entry k = ci*9 + tap (k' = tap*cin + ci).
@@ -373,6 +393,52 @@ hs_status plan_dense(hs_ctx* c, TcGemmParams* p, int epi, const __nv_bfloat16* a
   return HS_OK;
 }
 
+// Input gradient of stride-2 convolution k as four grouped class products (see TcConvGeom):
+// A = dA_k [N][Ho][Wo][Cout] (64-pixel boxes), B = the class weights (MN-major), D = the class
+// pixels of dA_{k-1} [N][H][W][Cin] (32-pixel store boxes), ReLU' of h_{k-1} fused.
+hs_status plan_subpixel_dgrad(hs_ctx* c, int k) {
+  const ConvLayer& L = c->convs[k];
+  const char* why = nullptr;
+  TcGemmParams& p = c->tc_dgrad[k];
+  std::memset(&p, 0, sizeof(p));
+  const int64_t hw = (int64_t)L.hout * L.wout;
+  const int taps[4] = {1, 2, 2, 4};
+  int64_t off = 0;
+  auto* dprev = reinterpret_cast<__nv_bfloat16*>(c->d_dA[k - 1]);
+  for (int g = 0; g < 4; ++g) {
+    const int ph = g >> 1, pw = g & 1;
+    const int64_t kg = (int64_t)taps[g] * L.cout;
+    bool ok = tc_make_grid_map(&p.tmA[g], c->d_dA[k], L.cout, L.wout, L.hout, c->N, L.cout, (int64_t)L.wout * L.cout,
+                               hw * L.cout, 64, &why) &&
+              tc_make_mnmajor_map(&p.tmB[g], TcOperand{c->d_wsub[k] + off, kg, L.cin, L.cin}, &why) &&
+              tc_make_grid_map(&p.tmD[g], dprev + ((int64_t)ph * L.win + pw) * L.cin, L.cin, L.wout, L.hout, c->N,
+                               2LL * L.cin, 2LL * L.win * L.cin, (int64_t)L.hin * L.win * L.cin, 32, &why);
+    if (!ok) return fail(c, HS_ERR_CUDA, why);
+    p.num_kb[g] = (int32_t)(kg / kTcBK);
+    off += kg * L.cin;
+  }
+  p.groups = 4;
+  p.Mdim = (int32_t)L.rows;
+  p.Ndim = L.cin;
+  p.n_store = L.cin;
+  p.tiles_m = (p.Mdim + kTcBM - 1) / kTcBM;
+  p.tiles_n = (p.n_store + kTcBN - 1) / kTcBN;
+  p.epi = kTcEpiMaskBf16;
+  p.a_mn = 0;
+  p.b_mn = 1;
+  p.conv_a = 2;
+  p.conv_d = 1;
+  p.conv = tc_conv_geom(L.cout, L.hout, L.wout, L.stride);
+  p.conv.H = L.hin;
+  p.conv.W = L.win;
+  p.D = dprev;
+  p.ldd = L.cin;
+  p.Z = reinterpret_cast<const __nv_bfloat16*>(c->d_cact[k - 1]);
+  p.ldz = L.cin;
+  p.st = c->d_status;
+  return HS_OK;
+}
+
 }  // namespace
 
 hs_status cnn_build_static(hs_ctx* c) {
@@ -410,9 +476,13 @@ hs_status cnn_build_static(hs_ctx* c) {
   if (st != HS_OK) return st;
   for (int k = 2; k >= 1; --k) {
     const ConvLayer& L = c->convs[k];
-    st = plan_dense(c, &c->tc_dgrad[k], kTcEpiStoreF32, bf(c->d_dA[k]), L.rows, L.cout, L.cout,
-                    c->d_wperm[k], L.cout, L.K, L.Kp, true, c->d_dcol, true, (int)L.rows, L.K, L.K, L.K,
-                    nullptr, 0);
+    if (L.subpixel) {
+      st = plan_subpixel_dgrad(c, k);
+    } else {
+      st = plan_dense(c, &c->tc_dgrad[k], kTcEpiStoreF32, bf(c->d_dA[k]), L.rows, L.cout, L.cout,
+                      c->d_wperm[k], L.cout, L.K, L.Kp, true, c->d_dcol, true, (int)L.rows, L.K, L.K, L.K,
+                      nullptr, 0);
+    }
     if (st != HS_OK) return st;
   }
   return HS_OK;
@@ -441,10 +511,16 @@ hs_status cnn_step(hs_ctx* c, float* params, const float* x, const int32_t* y, c
   {
     PhaseScope ph(c, HS_PHASE_CAST, s);
     if (bf16) {
-      for (int k = 0; k < 3; ++k)
+      for (int k = 0; k < 3; ++k) {
         permute_weights_kernel<<<blocks_for((int64_t)L[k].cout * L[k].Kp, T), T, 0, s>>>(
             params + L[k].w_off, L[k].cout, L[k].cin, L[k].Kp, c->d_wperm[k]);
-      ph.launched(3);
+        ph.launched();
+        if (L[k].subpixel) {
+          permute_weights_subpixel_kernel<<<blocks_for(9LL * L[k].cout * L[k].cin, T), T, 0, s>>>(
+              params + L[k].w_off, L[k].cout, L[k].cin, c->d_wsub[k]);
+          ph.launched();
+        }
+      }
     }
   }
   {
@@ -595,6 +671,13 @@ hs_status cnn_step(hs_ctx* c, float* params, const float* x, const int32_t* y, c
             c->d_dpooled, reinterpret_cast<const float*>(c->d_cact[2]), N, hw3, c3, reinterpret_cast<float*>(c->d_dA[2]));
       ph.launched(2);
     } else {
+      if (L[k].subpixel) {
+        // the four class products write dA_{k-1} directly (ReLU' of h_{k-1} fused)
+        cudaError_t e = launch_tc_gemm(c->tc_dgrad[k], c->num_sms, s);
+        if (e != cudaSuccess) return cuda_fail(c, e, "conv sub-pixel input-gradient GEMM launch");
+        ph.launched();
+        continue;
+      }
       // dcol = dA_k W_k (patch space, fp32), then gather back to layer k's input grid with ReLU'
       if (bf16) {
         cudaError_t e = launch_tc_gemm(c->tc_dgrad[k], c->num_sms, s);

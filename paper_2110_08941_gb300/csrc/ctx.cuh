@@ -22,6 +22,7 @@ struct ConvLayer {
   int64_t w_off, b_off;
   int64_t rows;       // N * hout * wout
   bool implicit;      // bf16: the products read the patch rows straight from the input (no col buffer)
+  bool subpixel;      // bf16: the input gradient is the grouped sub-pixel product (no patch-space buffer)
 };
 
 inline int64_t round_up(int64_t v, int64_t m) { return (v + m - 1) / m * m; }
@@ -146,6 +147,7 @@ struct hs_ctx {
   float* d_dcol = nullptr;
   __nv_bfloat16* d_wperm[3] = {nullptr, nullptr, nullptr};   // bf16 [Cout][Kp], tap-major columns
   __nv_bfloat16* d_ones = nullptr;                           // bf16 [64][64], column 0 ones (implicit convs)
+  __nv_bfloat16* d_wsub[3] = {nullptr, nullptr, nullptr};    // bf16 sub-pixel class weights, 9 x Cout x Cin
   int32_t* d_row_off[4] = {nullptr, nullptr, nullptr, nullptr};
   hs::ChunkTable cnn_chunks[4];
   hs::CnnWgrad cnn_wgrad[4];

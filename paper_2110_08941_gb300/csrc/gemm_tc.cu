@@ -31,7 +31,7 @@ constexpr uint32_t STAGE_TX = A_STAGE + B_STAGE;     // bytes landed per stage
 constexpr int kThreads = 192;
 constexpr uint32_t kTmemCols = 2 * BN;               // two accumulator buffers
 
-template <int EPI, bool A_MN, bool B_MN>
+template <int EPI, bool A_MN, bool B_MN, bool CONV>
 __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_constant__ TcGemmParams p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -100,22 +100,23 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
 #pragma unroll
             for (int j = 0; j < BM / 64; ++j) tma_load_2d(a_dst + j * MN_CHUNK, ta, c.tm * BM + 64 * j, k0, fb);
           } else {
+            if (CONV && p.conv_a) {
 #pragma unroll
-            for (int j = 0; j < BM / kTcBoxA; ++j) {
-              if (p.conv_a) {
+              for (int j = 0; j < BM / 64; ++j) {
                 int cc[4];
-                conv_box_coords(p.conv, c.tm * BM + kTcBoxA * j, k0, cc);
-                tma_load_4d(a_dst + j * (kTcBoxA * BK * 2), ta, cc, fb);
-              } else {
-                tma_load_2d(a_dst + j * (kTcBoxA * BK * 2), ta, k0, c.tm * BM + kTcBoxA * j, fb);
+                if (p.conv_a == 2) subpixel_box_coords(p.conv, c.g, c.tm * BM + 64 * j, k0, cc);
+                else conv_box_coords(p.conv, c.tm * BM + 64 * j, k0, cc);
+                tma_load_4d(a_dst + j * MN_CHUNK, ta, cc, fb);
               }
+            } else {
+              tma_load_2d(a_dst, ta, k0, c.tm * BM, fb);
             }
           }
           if (B_MN) {
 #pragma unroll
             for (int j = 0; j < BN / 64; ++j) {
               const int col = c.tn * BN + 64 * j;
-              if (!p.conv_b) {
+              if (!CONV || !p.conv_b) {
                 tma_load_2d(b_dst + j * MN_CHUNK, tb, col, k0, fb);
               } else if (col < p.conv.ones_col) {
                 int cc[4];
@@ -225,7 +226,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
         tmem_ld_wait(r);
         if (!kF32Out) tmem_ld_wait(r2);
         uint4 o[8];
-        epilogue_unit<EPI>(p, row, n_base, r, r2, o);
+        epilogue_unit<EPI, CONV>(p, c.g, row, n_base, r, r2, o);
         if (lane == 0) bulk_wait_read_1();   // the store that last used this buffer has read it
         __syncwarp();
         const uint32_t buf = stage_base + (uint32_t)(sb * 4096);
@@ -235,7 +236,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
         fence_proxy_async_smem();
         __syncwarp();
         if (lane == 0) {
-          tma_store_2d(td, buf, n_base, row0);
+          store_strip<CONV>(p, td, buf, n_base, row0);
           bulk_commit();
         }
         sb ^= 1;
@@ -266,10 +267,10 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
 
 PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 
-template <int EPI, bool A_MN, bool B_MN>
+template <int EPI, bool A_MN, bool B_MN, bool CONV>
 cudaError_t launch_variant(const TcGemmParams& p, int grid, cudaStream_t s) {
   static bool configured = false;
-  auto kern = tc_gemm_kernel<EPI, A_MN, B_MN>;
+  auto kern = tc_gemm_kernel<EPI, A_MN, B_MN, CONV>;
   if (!configured) {
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kTcSmemBytes);
     if (e != cudaSuccess) return e;
@@ -369,6 +370,41 @@ bool tc_make_conv_map(CUtensorMap* tm, const __nv_bfloat16* base, int64_t images
   return true;
 }
 
+bool tc_grid_ok(int rows, int cols, int box_pixels) {
+  if (rows < 1 || cols < 1 || box_pixels % cols) return false;
+  const int hw = rows * cols;
+  return hw % box_pixels == 0 || box_pixels % hw == 0;
+}
+
+bool tc_make_grid_map(CUtensorMap* tm, const void* base, int C, int cols, int rows, int64_t images,
+                      int64_t col_stride, int64_t row_stride, int64_t img_stride, int box_pixels, const char** why) {
+  if (!g_encode && !tc_init_driver(why)) return false;
+  if (C < 64 || C % 64 || images < 1 || !tc_grid_ok(rows, cols, box_pixels)) {
+    *why = "pixel grid not supported by the 4-D boxes";
+    return false;
+  }
+  if ((reinterpret_cast<uintptr_t>(base) & 15u) != 0 || (col_stride * 2) % 16 || (row_stride * 2) % 16 ||
+      (img_stride * 2) % 16) {
+    *why = "TMA grid base or stride is not 16-byte aligned";
+    return false;
+  }
+  const int hw = rows * cols;
+  const uint32_t hb = hw >= box_pixels ? (uint32_t)(box_pixels / cols) : (uint32_t)rows;
+  const uint32_t nb = hw >= box_pixels ? 1u : (uint32_t)(box_pixels / hw);
+  cuuint64_t dims[4] = {(cuuint64_t)C, (cuuint64_t)cols, (cuuint64_t)rows, (cuuint64_t)images};
+  cuuint64_t strides[3] = {(cuuint64_t)col_stride * 2, (cuuint64_t)row_stride * 2, (cuuint64_t)img_stride * 2};
+  cuuint32_t box[4] = {64, (cuuint32_t)cols, hb, nb};
+  cuuint32_t estr[4] = {1, 1, 1, 1};
+  CUresult r = g_encode(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides, box, estr,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) {
+    *why = "cuTensorMapEncodeTiled rejected the pixel grid";
+    return false;
+  }
+  return true;
+}
+
 bool tc_make_mnmajor_map(CUtensorMap* tm, const TcOperand& op, const char** why) {
   return encode_2d(tm, op.base, (uint64_t)op.cols, (uint64_t)op.rows, (uint64_t)op.ld * 2, 64, kTcBK, why);
 }
@@ -406,12 +442,19 @@ cudaError_t launch_tc_gemm_form(const TcGemmParams& p_in, int num_sms, cudaStrea
   const int total = p.groups * p.tiles_m * p.tiles_n;
   if (total <= 0) return cudaSuccess;
   const int grid = total < num_sms ? total : num_sms;
-  if (p.epi == kTcEpiBiasReluBf16 && !p.a_mn && !p.b_mn) return launch_variant<kTcEpiBiasReluBf16, false, false>(p, grid, s);
-  if (p.epi == kTcEpiBiasF32 && !p.a_mn && !p.b_mn) return launch_variant<kTcEpiBiasF32, false, false>(p, grid, s);
-  if (p.epi == kTcEpiMaskBf16 && !p.a_mn && p.b_mn) return launch_variant<kTcEpiMaskBf16, false, true>(p, grid, s);
-  if (p.epi == kTcEpiStoreF32 && p.a_mn && p.b_mn) return launch_variant<kTcEpiStoreF32, true, true>(p, grid, s);
-  if (p.epi == kTcEpiStoreF32 && !p.a_mn && !p.b_mn) return launch_variant<kTcEpiStoreF32, false, false>(p, grid, s);
-  if (p.epi == kTcEpiStoreF32 && !p.a_mn && p.b_mn) return launch_variant<kTcEpiStoreF32, false, true>(p, grid, s);
+  // implicit convolution operands (forward, weight gradient, sub-pixel input gradient)
+  if (p.conv_a || p.conv_b || p.conv_d) {
+    if (p.epi == kTcEpiBiasReluBf16 && !p.a_mn && !p.b_mn) return launch_variant<kTcEpiBiasReluBf16, false, false, true>(p, grid, s);
+    if (p.epi == kTcEpiStoreF32 && p.a_mn && p.b_mn) return launch_variant<kTcEpiStoreF32, true, true, true>(p, grid, s);
+    if (p.epi == kTcEpiMaskBf16 && !p.a_mn && p.b_mn) return launch_variant<kTcEpiMaskBf16, false, true, true>(p, grid, s);
+    return cudaErrorInvalidValue;
+  }
+  if (p.epi == kTcEpiBiasReluBf16 && !p.a_mn && !p.b_mn) return launch_variant<kTcEpiBiasReluBf16, false, false, false>(p, grid, s);
+  if (p.epi == kTcEpiBiasF32 && !p.a_mn && !p.b_mn) return launch_variant<kTcEpiBiasF32, false, false, false>(p, grid, s);
+  if (p.epi == kTcEpiMaskBf16 && !p.a_mn && p.b_mn) return launch_variant<kTcEpiMaskBf16, false, true, false>(p, grid, s);
+  if (p.epi == kTcEpiStoreF32 && p.a_mn && p.b_mn) return launch_variant<kTcEpiStoreF32, true, true, false>(p, grid, s);
+  if (p.epi == kTcEpiStoreF32 && !p.a_mn && !p.b_mn) return launch_variant<kTcEpiStoreF32, false, false, false>(p, grid, s);
+  if (p.epi == kTcEpiStoreF32 && !p.a_mn && p.b_mn) return launch_variant<kTcEpiStoreF32, false, true, false>(p, grid, s);
   return cudaErrorInvalidValue;
 }
 

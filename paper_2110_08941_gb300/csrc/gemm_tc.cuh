@@ -23,12 +23,21 @@ enum TcEpi : int32_t {
 // out-of-range coordinates, the stride = the box's traversal stride).  Rows are grouped in blocks
 // of 64, which must cover whole output rows (Wo divides 64) and whole images or parts of one
 // (Ho * Wo a multiple or a divisor of 64).
+//
+// The input gradient of a stride-2 convolution (even H, W) splits the input pixels into four
+// classes by the parity (ph, pw) of (hi, wi); class pixel (a, b) = input pixel (2a + ph, 2b + pw)
+// receives kernel rows kh = 1 (ph = 0) or kh = 0, 2 (ph = 1), from output rows a, or a + 1 and a
+// (likewise for columns).  Each class is then a product over an Ho x Wo grid: A = the output
+// gradient at (a + dh, b + dw) per tap (4-D boxes, zero fill past the grid), K = taps x Cout,
+// B = the class's weights, D = the class pixels of the input gradient (4-D store boxes), with the
+// ReLU' of the input activation fused.  One grouped launch, group = class = 2 * ph + pw.
 struct TcConvGeom {
-  int32_t cblocks;    // C / 64
-  int32_t Wo, hw;     // output width, output pixels per image
+  int32_t cblocks;    // (channels of the A grid) / 64
+  int32_t Wo, hw;     // width of the A grid (output grid), its pixels per image
   int32_t stride;
   int32_t ones_col;   // as the B operand: first column past the 9 * C patch columns, which holds
                       // ones (the bias gradient's column); columns past it read zeros
+  int32_t H, W;       // input grid (sub-pixel input gradient: where the ReLU' mask is read)
 };
 
 // D[Mdim x n_store] (row-major, leading dimension ldd) = A[Mdim x K] * B[K x Ndim] + epilogue.
@@ -37,7 +46,10 @@ struct TcConvGeom {
 //   MN-major  ("K rows, M or N contiguous"):   A as [K rows][M], B as [K rows][N]
 // Grouped launches run `groups` independent products that share Mdim/Ndim but each has its own
 // A/B maps (a worker's row segment) and K extent; group g writes D + g * d_gstride.
-// conv_a: A (K-major) is a convolution's implicit patch rows, tmA[g] a map from tc_make_conv_map.
+// conv_a = 1: A (K-major) is a convolution's implicit patch rows, tmA[g] from tc_make_conv_map.
+// conv_a = 2: A is the shifted output gradient of the sub-pixel input gradient (tc_make_grid_map,
+//             64-pixel boxes), class = group; conv_d = 1: D rows are that class's input pixels
+//             (tmD[g] from tc_make_grid_map with 32-pixel boxes) and the mask Z is read there.
 // conv_b: B (MN-major) is the implicit patch rows of the group's samples (tmB[g] a conv map over
 // them), and tmOnes supplies the ones column at conv.ones_col.
 struct TcGemmParams {
@@ -46,7 +58,7 @@ struct TcGemmParams {
   CUtensorMap tmD[kTcMaxGroups];   // output (store) maps: box of 32 rows x 128 bytes
   CUtensorMap tmOnes;              // MN-major [64][64] bf16, column 0 ones, the rest zero (conv_b)
   TcConvGeom conv;
-  int32_t conv_a, conv_b;
+  int32_t conv_a, conv_b, conv_d;
   int32_t num_kb[kTcMaxGroups];
   int32_t groups;
   int32_t Mdim, Ndim, n_store;
@@ -80,6 +92,11 @@ bool tc_conv_implicit_ok(int C, int Ho, int Wo, int stride);
 bool tc_make_conv_map(CUtensorMap* tm, const __nv_bfloat16* base, int64_t images, int H, int W, int C, int Ho,
                       int Wo, int stride, const char** why);
 TcConvGeom tc_conv_geom(int C, int Ho, int Wo, int stride);
+// bf16 pixel grid [images][rows][cols][C] with arbitrary (16-byte multiple) strides, given in
+// elements; box = 64 channels x `box_pixels` pixels (whole grid rows, or whole images).
+bool tc_grid_ok(int rows, int cols, int box_pixels);
+bool tc_make_grid_map(CUtensorMap* tm, const void* base, int C, int cols, int rows, int64_t images,
+                      int64_t col_stride, int64_t row_stride, int64_t img_stride, int box_pixels, const char** why);
 // Output matrix [rows][cols] (row stride ld elements, fp32 or bf16) for TMA stores of 32-row x
 // 128-byte boxes; rows >= `rows` and columns >= `cols` of a box are not written.
 bool tc_make_store_map(CUtensorMap* tm, void* base, bool fp32, int64_t rows, int64_t cols, int64_t ld,
@@ -90,7 +107,7 @@ constexpr int kTcStagingBytes = 4 * 2 * 32 * 128;   // 4 epilogue warps x 2 buff
 constexpr int kTcSmemBytes =
     kTcStages * (kTcBM + kTcBN) * kTcBK * 2 + kTcStagingBytes + 1024 /*align*/ + 256 /*barriers*/;
 
-constexpr int kTcBoxA = 64;    // rows of a K-major A box (a 128-row A tile is two boxes)
+constexpr int kTcBoxA = 128;   // rows of a K-major A box (one per 128-row A tile; implicit patch rows: two 64-pixel boxes)
 constexpr int kTcBoxB = 128;   // rows of a K-major B box (the 256-row B tile is two boxes)
 
 // Kernel form: one SM per 128 x 256 tile, or an SM pair (cluster of 2, tcgen05 cta_group::2) per

@@ -95,7 +95,7 @@ __device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr) {
   asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
 }
 
-template <int EPI, bool A_MN, bool B_MN>
+template <int EPI, bool A_MN, bool B_MN, bool CONV>
 __global__ void __launch_bounds__(kThreads2, 1) tc_gemm_pair_kernel(const __grid_constant__ TcGemmParams p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -167,24 +167,27 @@ __global__ void __launch_bounds__(kThreads2, 1) tc_gemm_pair_kernel(const __grid
           const int k0 = kb * BK;
           const uint32_t a_dst = smem_u32(smem + s * STAGE2);
           const uint32_t b_dst = a_dst + A_HALF;
-          // the A half is two 64-row (K-major) or 64-column (MN-major) boxes of 8 KB
+          // the A half: two 64-column boxes (MN-major), two 64-pixel boxes (implicit patch rows) or
+          // one 128-row box (K-major)
+          if (A_MN) {
 #pragma unroll
-          for (int j = 0; j < HM / 64; ++j) {
-            if (A_MN) {
-              tma_load_2d_pair(a_dst + j * MN_CHUNK, ta, m0 + 64 * j, k0, fb);
-            } else if (p.conv_a) {
+            for (int j = 0; j < HM / 64; ++j) tma_load_2d_pair(a_dst + j * MN_CHUNK, ta, m0 + 64 * j, k0, fb);
+          } else if (CONV && p.conv_a) {
+#pragma unroll
+            for (int j = 0; j < HM / 64; ++j) {
               int cc[4];
-              conv_box_coords(p.conv, m0 + 64 * j, k0, cc);
+              if (p.conv_a == 2) subpixel_box_coords(p.conv, c.g, m0 + 64 * j, k0, cc);
+              else conv_box_coords(p.conv, m0 + 64 * j, k0, cc);
               tma_load_4d_pair(a_dst + j * MN_CHUNK, ta, cc, fb);
-            } else {
-              tma_load_2d_pair(a_dst + j * MN_CHUNK, ta, k0, m0 + 64 * j, fb);
             }
+          } else {
+            tma_load_2d_pair(a_dst, ta, k0, m0, fb);
           }
           if (B_MN) {
 #pragma unroll
             for (int j = 0; j < HN / 64; ++j) {
               const int col = n0 + 64 * j;
-              if (!p.conv_b) {
+              if (!CONV || !p.conv_b) {
                 tma_load_2d_pair(b_dst + j * MN_CHUNK, tb, col, k0, fb);
               } else if (col < p.conv.ones_col) {
                 int cc[4];
@@ -288,7 +291,7 @@ __global__ void __launch_bounds__(kThreads2, 1) tc_gemm_pair_kernel(const __grid
         tmem_ld_wait(r);
         if (!kF32Out) tmem_ld_wait(r2);
         uint4 o[8];
-        epilogue_unit<EPI>(p, row, n_base, r, r2, o);
+        epilogue_unit<EPI, CONV>(p, c.g, row, n_base, r, r2, o);
         if (lane == 0) bulk_wait_read_1();
         __syncwarp();
         const uint32_t buf = stage_base + (uint32_t)(sb * 4096);
@@ -298,7 +301,7 @@ __global__ void __launch_bounds__(kThreads2, 1) tc_gemm_pair_kernel(const __grid
         fence_proxy_async_smem();
         __syncwarp();
         if (lane == 0) {
-          tma_store_2d(td, buf, n_base, row0);
+          store_strip<CONV>(p, td, buf, n_base, row0);
           bulk_commit();
         }
         sb ^= 1;
@@ -328,11 +331,11 @@ __global__ void __launch_bounds__(kThreads2, 1) tc_gemm_pair_kernel(const __grid
   }
 }
 
-template <int EPI, bool A_MN, bool B_MN>
+template <int EPI, bool A_MN, bool B_MN, bool CONV>
 cudaError_t launch_pair_variant(const TcGemmParams& p, int pairs_wanted, int num_sms, cudaStream_t s) {
   static bool configured = false;
   static int max_clusters = 0;
-  auto kern = tc_gemm_pair_kernel<EPI, A_MN, B_MN>;
+  auto kern = tc_gemm_pair_kernel<EPI, A_MN, B_MN, CONV>;
   cudaLaunchConfig_t cfg = {};
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -376,12 +379,19 @@ cudaError_t launch_tc_gemm_pair(const TcGemmParams& p, int num_sms, cudaStream_t
   if (total <= 0) return cudaSuccess;
   const int pairs = total;
   const int grid = num_sms;   // forwarded as the SM count for the residency query
-  if (p.epi == kTcEpiBiasReluBf16 && !p.a_mn && !p.b_mn) return launch_pair_variant<kTcEpiBiasReluBf16, false, false>(p, pairs, grid, s);
-  if (p.epi == kTcEpiBiasF32 && !p.a_mn && !p.b_mn) return launch_pair_variant<kTcEpiBiasF32, false, false>(p, pairs, grid, s);
-  if (p.epi == kTcEpiMaskBf16 && !p.a_mn && p.b_mn) return launch_pair_variant<kTcEpiMaskBf16, false, true>(p, pairs, grid, s);
-  if (p.epi == kTcEpiStoreF32 && p.a_mn && p.b_mn) return launch_pair_variant<kTcEpiStoreF32, true, true>(p, pairs, grid, s);
-  if (p.epi == kTcEpiStoreF32 && !p.a_mn && !p.b_mn) return launch_pair_variant<kTcEpiStoreF32, false, false>(p, pairs, grid, s);
-  if (p.epi == kTcEpiStoreF32 && !p.a_mn && p.b_mn) return launch_pair_variant<kTcEpiStoreF32, false, true>(p, pairs, grid, s);
+  // implicit convolution operands (forward, weight gradient, sub-pixel input gradient)
+  if (p.conv_a || p.conv_b || p.conv_d) {
+    if (p.epi == kTcEpiBiasReluBf16 && !p.a_mn && !p.b_mn) return launch_pair_variant<kTcEpiBiasReluBf16, false, false, true>(p, pairs, grid, s);
+    if (p.epi == kTcEpiStoreF32 && p.a_mn && p.b_mn) return launch_pair_variant<kTcEpiStoreF32, true, true, true>(p, pairs, grid, s);
+    if (p.epi == kTcEpiMaskBf16 && !p.a_mn && p.b_mn) return launch_pair_variant<kTcEpiMaskBf16, false, true, true>(p, pairs, grid, s);
+    return cudaErrorInvalidValue;
+  }
+  if (p.epi == kTcEpiBiasReluBf16 && !p.a_mn && !p.b_mn) return launch_pair_variant<kTcEpiBiasReluBf16, false, false, false>(p, pairs, grid, s);
+  if (p.epi == kTcEpiBiasF32 && !p.a_mn && !p.b_mn) return launch_pair_variant<kTcEpiBiasF32, false, false, false>(p, pairs, grid, s);
+  if (p.epi == kTcEpiMaskBf16 && !p.a_mn && p.b_mn) return launch_pair_variant<kTcEpiMaskBf16, false, true, false>(p, pairs, grid, s);
+  if (p.epi == kTcEpiStoreF32 && p.a_mn && p.b_mn) return launch_pair_variant<kTcEpiStoreF32, true, true, false>(p, pairs, grid, s);
+  if (p.epi == kTcEpiStoreF32 && !p.a_mn && !p.b_mn) return launch_pair_variant<kTcEpiStoreF32, false, false, false>(p, pairs, grid, s);
+  if (p.epi == kTcEpiStoreF32 && !p.a_mn && p.b_mn) return launch_pair_variant<kTcEpiStoreF32, false, true, false>(p, pairs, grid, s);
   return cudaErrorInvalidValue;
 }
 

@@ -295,6 +295,7 @@ void free_all(hs_ctx* c) {
   f(c->d_pooled); f(c->d_dpooled); f(c->d_dcol);
   for (int k = 0; k < 3; ++k) f(c->d_wperm[k]);
   f(c->d_ones);
+  for (int k = 0; k < 3; ++k) f(c->d_wsub[k]);
   for (int k = 0; k < 4; ++k) {
     f(c->d_row_off[k]); f(c->cnn_chunks[k].d_chunks); f(c->cnn_chunks[k].d_begin);
     f(c->cnn_wgrad[k].d_partial); f(c->cnn_wgrad[k].d_chunk_begin);
@@ -611,6 +612,11 @@ hs_status hs_init(const hs_model_desc* model, int32_t M, const double* compute_w
       const char* imp = getenv("HS_CONV_IMPLICIT");
       L.implicit = bf16 && k > 0 && !(imp && !strcmp(imp, "0")) &&
                    hs::tc_conv_implicit_ok(L.cin, L.hout, L.wout, L.stride);
+      // ... and the input gradient as the sub-pixel product (HS_CONV_IMPLICIT=fwd keeps the
+      // patch-space product and its gather)
+      L.subpixel = L.implicit && !(imp && !strcmp(imp, "fwd")) && L.stride == 2 && L.hin == 2 * L.hout &&
+                   L.win == 2 * L.wout && L.cout % 64 == 0 && hs::tc_grid_ok(L.hout, L.wout, 64) &&
+                   hs::tc_grid_ok(L.hout, L.wout, 32);
       c->convs.push_back(L);
       h = L.hout;
       w = L.wout;
@@ -661,15 +667,18 @@ hs_status hs_init(const hs_model_desc* model, int32_t M, const double* compute_w
       if (!L.implicit) chk(dalloc(c, &c->d_col[k], es * (size_t)L.rows * L.Kp));
       chk(dalloc(c, &c->d_cact[k], es * (size_t)L.rows * L.cout));
       chk(dalloc(c, &c->d_dA[k], es * (size_t)L.rows * L.cout));
-      if (k > 0) dcol = std::max<int64_t>(dcol, L.rows * L.K);
+      if (k > 0 && !L.subpixel) dcol = std::max<int64_t>(dcol, L.rows * L.K);
     }
     chk(dalloc(c, &c->d_pooled, es * N * c3));
     chk(dalloc(c, &c->d_dpooled, sizeof(float) * N * c3));
-    chk(dalloc(c, &c->d_dcol, sizeof(float) * (size_t)dcol));
+    if (dcol > 0) chk(dalloc(c, &c->d_dcol, sizeof(float) * (size_t)dcol));
     if (bf16) {
       for (int k = 0; k < 3; ++k)
         chk(dalloc(c, &c->d_wperm[k], sizeof(__nv_bfloat16) * (size_t)c->convs[k].cout * c->convs[k].Kp));
       chk(dalloc(c, &c->d_ones, sizeof(__nv_bfloat16) * 64 * 64));
+      for (int k = 1; k < 3; ++k)
+        if (c->convs[k].subpixel)
+          chk(dalloc(c, &c->d_wsub[k], sizeof(__nv_bfloat16) * 9 * (size_t)c->convs[k].cout * c->convs[k].cin));
     }
     delta_elems = N * (size_t)c->Cp;
     for (int k = 0; k < 4; ++k) {

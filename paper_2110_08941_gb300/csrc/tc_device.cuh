@@ -83,10 +83,46 @@ __device__ __forceinline__ void conv_box_coords(const TcConvGeom& g, int row, in
   c[2] = g.stride * ho + tap / 3 - 1;
   c[3] = img;
 }
+// The same for the sub-pixel input gradient of class `cls` = 2 * ph + pw: patch column block
+// kcol / 64 = (tap t of the class, Cout block); the class's row taps are kh = 1 (ph = 0) or kh = 0
+// then 2 (ph = 1), which read output row a + 1 and a (dh = 1, 0); columns likewise.
+__device__ __forceinline__ void subpixel_box_coords(const TcConvGeom& g, int cls, int row, int kcol,
+                                                    int (&c)[4]) {
+  const int blk = kcol >> 6;
+  const int t = blk / g.cblocks;
+  const int cb = blk - t * g.cblocks;
+  const int ph = cls >> 1, pw = cls & 1;
+  const int nw = pw ? 2 : 1;
+  const int th = t / nw, tw = t - th * nw;
+  const int img = row / g.hw;
+  const int a = (row - img * g.hw) / g.Wo;
+  c[0] = cb * 64;
+  c[1] = (pw && tw == 0) ? 1 : 0;
+  c[2] = a + ((ph && th == 0) ? 1 : 0);
+  c[3] = img;
+}
+__device__ __forceinline__ void tma_store_4d(const CUtensorMap* tm, uint32_t src, const int (&c)[4]) {
+  asm volatile("cp.async.bulk.tensor.4d.global.shared::cta.bulk_group [%0, {%1, %2, %3, %4}], [%5];"
+               ::"l"(reinterpret_cast<uint64_t>(tm)), "r"(c[0]), "r"(c[1]), "r"(c[2]), "r"(c[3]), "r"(src)
+               : "memory");
+}
 __device__ __forceinline__ void tma_store_2d(const CUtensorMap* tm, uint32_t src, int c0, int c1) {
   asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%1, %2}], [%3];"
                ::"l"(reinterpret_cast<uint64_t>(tm)), "r"(c0), "r"(c1), "r"(src)
                : "memory");
+}
+// Store the 32-row strip at rows row0.. (row0 a multiple of 32), columns n_base.. through the
+// output map of the group: a 2-D [rows][cols] map, or (conv_d) a class grid of the input gradient.
+template <bool CONV>
+__device__ __forceinline__ void store_strip(const TcGemmParams& p, const CUtensorMap* td, uint32_t buf, int n_base,
+                                            int row0) {
+  if (CONV && p.conv_d) {
+    const int img = row0 / p.conv.hw;
+    const int c[4] = {n_base, 0, (row0 - img * p.conv.hw) / p.conv.Wo, img};
+    tma_store_4d(td, buf, c);
+  } else {
+    tma_store_2d(td, buf, n_base, row0);
+  }
 }
 __device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
 // At most one bulk group may still be reading shared memory.
@@ -215,9 +251,9 @@ __device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
 // computed from `r` (columns n_base..n_base+31) and, for bf16 outputs, `r2` (n_base+32..+63), packed
 // into eight 16-byte words.  Columns past n_store are computed but never stored (the TMA store
 // clips them); only the bias and mask reads are guarded.
-template <int EPI>
-__device__ __forceinline__ void epilogue_unit(const TcGemmParams& p, int row, int n_base, const uint32_t (&r)[32],
-                                              const uint32_t (&r2)[32], uint4 (&o)[8]) {
+template <int EPI, bool CONV>
+__device__ __forceinline__ void epilogue_unit(const TcGemmParams& p, int grp, int row, int n_base,
+                                              const uint32_t (&r)[32], const uint32_t (&r2)[32], uint4 (&o)[8]) {
   if (EPI == kTcEpiStoreF32) {
 #pragma unroll
     for (int j = 0; j < 8; ++j) o[j] = make_uint4(r[4 * j], r[4 * j + 1], r[4 * j + 2], r[4 * j + 3]);
@@ -265,7 +301,14 @@ __device__ __forceinline__ void epilogue_unit(const TcGemmParams& p, int row, in
       }
     } else {   // kTcEpiMaskBf16: ReLU' from the stored activation of the same row
       if (row < p.Mdim) {
-        const __nv_bfloat16* z = p.Z + (int64_t)row * p.ldz + n_base;
+        int64_t zrow = row;
+        if (CONV && p.conv_d) {   // class pixel (a, b) of image img = input pixel (2a + ph, 2b + pw)
+          const int img = row / p.conv.hw;
+          const int rem = row - img * p.conv.hw;
+          const int a = rem / p.conv.Wo, b = rem - a * p.conv.Wo;
+          zrow = ((int64_t)img * p.conv.H + 2 * a + (grp >> 1)) * p.conv.W + 2 * b + (grp & 1);
+        }
+        const __nv_bfloat16* z = p.Z + zrow * p.ldz + n_base;
         if (n_base + 64 <= p.n_store) {
           const uint4* z4 = reinterpret_cast<const uint4*>(z);
 #pragma unroll

@@ -248,35 +248,54 @@ def test_fused_sync_headline_workload_gradient():
 
 
 # ------------------------------------------------------------------ implicit-GEMM convolutions
-@pytest.mark.parametrize("name", [synth.CFG4])
-def test_implicit_conv_is_bit_identical_to_materialised_patches(name, monkeypatch):
-    """The convolutions' products read their patch rows straight from the NHWC input (4-D TMA boxes)
-    or from materialised patch rows (HS_CONV_IMPLICIT=0): same operand values in the same k-block
-    order, so theta, losses and per-worker gradients agree bit for bit.  The implicit context holds no
-    patch buffers for the second and third convolutions."""
-    wl, x, y, theta0, w = _inputs(name)
-    out = {}
-    for mode in ("1", "0"):
-        monkeypatch.setenv("HS_CONV_IMPLICIT", mode)
+def _cnn_run(monkeypatch, mode, wl, x, y, theta0, w, steps):
+    monkeypatch.setenv("HS_CONV_IMPLICIT", mode)
+    torch.cuda.synchronize()
+    free0 = torch.cuda.mem_get_info()[0]
+    ctx = hs.hs_init(wl.arch, wl.dims, wl.workers, wl.global_batch, compute_weights=w, precision=hs.HS_BF16)
+    used = free0 - torch.cuda.mem_get_info()[0]
+    try:
+        hs.hs_set_debug(ctx, True)
+        p = torch.tensor(theta0, device="cuda")
+        xd, yd = torch.from_numpy(x).cuda(), torch.from_numpy(y).cuda()
+        losses, first = [], None
+        for t in range(steps):
+            losses.append(hs.hs_step(ctx, p, xd, yd, None, wl.lr))
+            if t == 0:
+                first = torch.empty(wl.workers, ctx.P, device="cuda")
+                hs.hs_debug_grads(ctx, None, first)
         torch.cuda.synchronize()
-        free0 = torch.cuda.mem_get_info()[0]
-        ctx = hs.hs_init(wl.arch, wl.dims, wl.workers, wl.global_batch, compute_weights=w, precision=hs.HS_BF16)
-        used = free0 - torch.cuda.mem_get_info()[0]
-        try:
-            hs.hs_set_debug(ctx, True)
-            p = torch.tensor(theta0, device="cuda")
-            xd, yd = torch.from_numpy(x).cuda(), torch.from_numpy(y).cuda()
-            losses = [hs.hs_step(ctx, p, xd, yd, None, wl.lr) for _ in range(3)]
-            slabs = torch.empty(wl.workers, ctx.P, device="cuda")
-            hs.hs_debug_grads(ctx, None, slabs)
-            torch.cuda.synchronize()
-            out[mode] = (p.cpu(), losses, slabs.cpu(), used)
-        finally:
-            ctx.close()
-    assert torch.equal(out["1"][0], out["0"][0])
-    assert out["1"][1] == out["0"][1]
-    assert torch.equal(out["1"][2], out["0"][2])
-    # patch rows of conv2 (N*16*16 x 584) and conv3 (N*8*8 x 1160), bf16, not allocated
+        return p.cpu(), losses, first.cpu(), used
+    finally:
+        ctx.close()
+
+
+def test_implicit_conv_is_bit_identical_to_materialised_patches(monkeypatch):
+    """The convolutions' forward and weight-gradient products read their patch rows straight from the
+    NHWC input (4-D TMA boxes; HS_CONV_IMPLICIT=fwd) or from materialised patch rows
+    (HS_CONV_IMPLICIT=0): same operand values in the same k-block order, so theta, losses and
+    per-worker gradients agree bit for bit, and the implicit context holds no patch buffers for the
+    second and third convolutions."""
+    wl, x, y, theta0, w = _inputs(synth.CFG4)
+    imp = _cnn_run(monkeypatch, "fwd", wl, x, y, theta0, w, 3)
+    mat = _cnn_run(monkeypatch, "0", wl, x, y, theta0, w, 3)
+    assert torch.equal(imp[0], mat[0])
+    assert imp[1] == mat[1]
+    assert torch.equal(imp[2], mat[2])
     n = wl.global_batch
-    saved = 2 * (n * 256 * 584 + n * 64 * 1160)
-    assert out["0"][3] - out["1"][3] >= 0.9 * saved
+    saved = 2 * (n * 256 * 584 + n * 64 * 1160)      # bf16 patch rows of conv2 and conv3
+    assert mat[3] - imp[3] >= 0.9 * saved
+
+
+def test_subpixel_input_gradient_matches_patch_space_gather(monkeypatch):
+    """The stride-2 convolutions' input gradients as four grouped sub-pixel products (default) against
+    the patch-space product followed by the gather (HS_CONV_IMPLICIT=fwd): the same sums in another
+    fp32 order, rounded to bf16 once, so first-step gradients agree to bf16 rounding and the
+    patch-space buffer (fp32 N*16*16 x 576) is gone."""
+    wl, x, y, theta0, w = _inputs(synth.CFG4)
+    sub = _cnn_run(monkeypatch, "1", wl, x, y, theta0, w, 3)
+    pat = _cnn_run(monkeypatch, "fwd", wl, x, y, theta0, w, 3)
+    assert rel(sub[2].numpy(), pat[2].numpy()) <= 2e-3
+    assert np.allclose(sub[1], pat[1], rtol=1e-3, atol=0)
+    assert rel(sub[0].numpy(), pat[0].numpy()) <= 1e-5
+    assert pat[3] - sub[3] >= 0.9 * 4 * wl.global_batch * 256 * 576
