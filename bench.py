@@ -414,6 +414,34 @@ def run_ours(args, wl, rank, world, local_rank):
     ms = max_over_ranks(ms)
     loss = hs.hs_step(ctx, params, xd, yd, part, 0.0, stream=stream, want_loss=True)   # finite-loss check
 
+    # the same step replayed from a CUDA graph (captured once, loss not requested): the launch
+    # overhead of the step's kernels removed
+    graph = None
+    try:
+        side = torch.cuda.Stream(dev)
+        side.wait_stream(stream)
+        with torch.cuda.stream(side):
+            hs.hs_step(ctx, params, xd, yd, part, wl.lr, stream=side, want_loss=False)
+        stream.wait_stream(side)
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            hs.hs_step(ctx, params, xd, yd, part, wl.lr, want_loss=False)
+        g.replay()
+        torch.cuda.synchronize()
+        barrier()
+        q0, q1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        q0.record(stream)
+        for _ in range(args.steps):
+            g.replay()
+        q1.record(stream)
+        torch.cuda.synchronize()
+        gms = max_over_ranks(q0.elapsed_time(q1))
+        graph = {"ms_per_step": gms / args.steps, "value": world * wl.global_batch * args.steps / (gms * 1e-3),
+                 "unit": UNIT, "what": "one hs_step captured in a CUDA graph, replayed"}
+        del g
+    except Exception as e:   # capture is an optimisation of the launch path; report why it failed
+        graph = {"unavailable": f"{type(e).__name__}: {e}"[:200]}
+
     # the slab-free formulation of the same step (opt-in variant), timed the same way
     fused = None
     if wl.arch == synth.MLP and precision == hs.HS_BF16:
@@ -553,6 +581,7 @@ def run_ours(args, wl, rank, world, local_rank):
             "clocks": clk,
             "straggler_sim": straggler_simulation(),
             "fused_sync_variant": fused,
+            "graph_replay": graph,
             "heterogeneity_sim": heterogeneity_simulation(ms * 1e-3 / args.steps / wl.global_batch),
             "loss_after": loss,
         }

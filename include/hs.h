@@ -165,7 +165,11 @@ hs_status hs_set_cp_history(hs_ctx* ctx, int32_t mode, double param);
  *           also reports HS_ERR_DEVICE_CHECK if a kernel's bounded wait expired.
  *           When NULL the call is fully asynchronous.
  * Labels outside [0, classes) are clamped by the loss kernel and counted as an
- * error reported through HS_ERR_DEVICE_CHECK at the next synchronising call. */
+ * error reported through HS_ERR_DEVICE_CHECK at the next synchronising call.
+ * CUDA graphs: with device x and y, loss_out NULL and the bf16 shadow current (a previous step
+ * or hs_sync_params on the same params), the call only enqueues work on `stream` and may be
+ * captured into a graph.  The graph holds this call's pointers, lr and partition plans by value:
+ * it stays valid until the next hs_partition, hs_set_* or hs_init/hs_destroy on the context. */
 hs_status hs_step(hs_ctx* ctx, float* params, const void* x, const int32_t* y,
                   const hs_partition_t* part, float lr, void* stream, float* loss_out);
 
