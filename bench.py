@@ -494,17 +494,32 @@ def run_ours(args, wl, rank, world, local_rank):
         ctx2.close()
         del p2
 
-    # end to end through the public API: host (pinned) inputs, loss read back every step
+    # end to end through the public API: every step copies its inputs from pinned host memory and
+    # reads its loss back.  Pipelined: hs_stage_inputs copies step t + 1's inputs on a copy stream
+    # while step t runs (two staging slots); the unpipelined form lets hs_step copy host inputs on
+    # its own stream first.
     xh = torch.from_numpy(x).pin_memory()
     yh = torch.from_numpy(y).pin_memory()
     k_e2e = max(3, min(args.steps, 10))
+    copy_stream = torch.cuda.Stream(dev)
+    hs.hs_step(ctx, params, hs.hs_stage_inputs(ctx, xh, yh, stream=copy_stream), None, part, wl.lr, stream=stream,
+               want_loss=True)
+    barrier()
+    t0 = time.perf_counter()
+    nxt = hs.hs_stage_inputs(ctx, xh, yh, stream=copy_stream)
+    for i in range(k_e2e):
+        cur = nxt
+        if i + 1 < k_e2e:
+            nxt = hs.hs_stage_inputs(ctx, xh, yh, stream=copy_stream)
+        hs.hs_step(ctx, params, cur, None, part, wl.lr, stream=stream, want_loss=True)
+    e2e_s = time.perf_counter() - t0
+    e2e_s = max_over_ranks(e2e_s)
     hs.hs_step(ctx, params, xh, yh, part, wl.lr, stream=stream, want_loss=True)
     barrier()
     t0 = time.perf_counter()
     for _ in range(k_e2e):
         hs.hs_step(ctx, params, xh, yh, part, wl.lr, stream=stream, want_loss=True)
-    e2e_s = time.perf_counter() - t0
-    e2e_s = max_over_ranks(e2e_s)
+    e2e_plain_s = max_over_ranks(time.perf_counter() - t0)
 
     P = ctx.P
     peaks = _peaks()
@@ -577,7 +592,9 @@ def run_ours(args, wl, rank, world, local_rank):
             "gpu_launches": int(launches),
             "cpu_baseline": cpu,
             "e2e": {"value": world * wl.global_batch * k_e2e / e2e_s, "unit": UNIT,
-                    "h2d_bytes_per_step": int(x.nbytes + y.nbytes), "d2h_bytes_per_step": 12},
+                    "h2d_bytes_per_step": int(x.nbytes + y.nbytes), "d2h_bytes_per_step": 12,
+                    "pipelined": "hs_stage_inputs on a copy stream, two slots",
+                    "unpipelined_value": world * wl.global_batch * k_e2e / e2e_plain_s},
             "clocks": clk,
             "straggler_sim": straggler_simulation(),
             "fused_sync_variant": fused,

@@ -173,6 +173,19 @@ hs_status hs_set_cp_history(hs_ctx* ctx, int32_t mode, double param);
 hs_status hs_step(hs_ctx* ctx, float* params, const void* x, const int32_t* y,
                   const hs_partition_t* part, float lr, void* stream, float* loss_out);
 
+/* Double-buffered input staging for a pipelined training loop (an input pipeline; the paper's
+ * workers each read their own data shard, Section 1).  Copies one step's x and y (layouts as in
+ * hs_step) from host memory into the next of two context-owned device slots, enqueued on
+ * `stream` (typically a copy stream other than the step's), after the step that last read that
+ * slot has finished with it; returns the slot's device pointers in *x_dev, *y_dev.  hs_step given
+ * exactly these pointers makes its own stream wait for the copy, so the copy of step t + 1's
+ * inputs overlaps step t.  Pinned host memory makes the copy asynchronous; the host buffers
+ * must stay unchanged until the copy has run.
+ * Errors: HS_ERR_INVALID_ARG for NULL arguments, or when both slots hold inputs that no hs_step
+ * has read yet (at most two staged steps in flight); HS_ERR_OOM on the first use of a slot. */
+hs_status hs_stage_inputs(hs_ctx* ctx, const float* x_host, const int32_t* y_host, void* stream,
+                          const float** x_dev, const int32_t** y_dev);
+
 /* The training recipe of the paper's experiments (Section 5: SGD with momentum and weight decay)
  * in the fused update.  With d = g + weight_decay * theta (g the synchronised gradient):
  *   b = d on the first step after this call, b = momentum * b + d afterwards, theta <- theta - lr * b.

@@ -27,7 +27,7 @@ EXPORTED = ("hs_partition_sizes", "hs_param_count", "hs_init", "hs_partition", "
             "hs_set_debug", "hs_debug_grads", "hs_worker_losses", "hs_destroy", "hs_status_string",
             "hs_last_error", "hs_last_init_error", "hs_debug_gemm_bf16", "hs_set_profiling", "hs_read_profile",
             "hs_partition_noalloc", "hs_set_optimizer", "hs_optimizer_state", "hs_cosine_lr",
-            "hs_set_cp_history", "hs_set_fused_sync")
+            "hs_set_cp_history", "hs_set_fused_sync", "hs_stage_inputs")
 HS_CP_LAST, HS_CP_EMA, HS_CP_WINDOW = 0, 1, 2
 PHASES = ("cast", "forward", "loss", "wgrad", "biasgrad", "dgrad", "update")
 
@@ -64,6 +64,7 @@ def _load() -> ctypes.CDLL:
         "hs_step": (S, [c_void_p, c_void_p, c_void_p, c_void_p, POINTER(hs_partition_t), c_float, c_void_p,
                         POINTER(c_float)]),
         "hs_sync_params": (S, [c_void_p, c_void_p, c_void_p]),
+        "hs_stage_inputs": (S, [c_void_p, c_void_p, c_void_p, c_void_p, POINTER(c_void_p), POINTER(c_void_p)]),
         "hs_set_debug": (S, [c_void_p, c_int32]),
         "hs_set_profiling": (S, [c_void_p, c_int32]),
         "hs_set_optimizer": (S, [c_void_p, c_float, c_float]),
@@ -207,17 +208,39 @@ def hs_partition(ctx: Context, measured_throughputs=None, index_map_out=None, st
     return ctx.partition
 
 
-def hs_step(ctx: Context, params, x, y, part: Optional[Partition] = None, lr: float = 0.01, stream=None,
+class StagedInputs:
+    """One step's x and y in a context staging slot (device pointers from hs_stage_inputs); pass it
+    to hs_step as x (y omitted).  Holds the host tensors until then."""
+
+    def __init__(self, x_ptr: int, y_ptr: int, host):
+        self.x_ptr, self.y_ptr, self._host = x_ptr, y_ptr, host
+
+
+def hs_stage_inputs(ctx: Context, x_host, y_host, stream=None) -> StagedInputs:
+    import torch
+    assert x_host.dtype == torch.float32 and x_host.is_contiguous() and not x_host.is_cuda
+    assert y_host.dtype == torch.int32 and y_host.is_contiguous() and not y_host.is_cuda
+    xp, yp = c_void_p(), c_void_p()
+    _check(_lib.hs_stage_inputs(ctx.ptr, c_void_p(x_host.data_ptr()), c_void_p(y_host.data_ptr()),
+                                c_void_p(_stream_ptr(stream)), ctypes.byref(xp), ctypes.byref(yp)), ctx.ptr)
+    return StagedInputs(xp.value, yp.value, (x_host, y_host))
+
+
+def hs_step(ctx: Context, params, x, y=None, part: Optional[Partition] = None, lr: float = 0.01, stream=None,
             want_loss: bool = True) -> Optional[float]:
     import torch
     assert params.dtype == torch.float32 and params.is_contiguous() and params.is_cuda
-    assert x.dtype == torch.float32 and x.is_contiguous()
-    assert y.dtype == torch.int32 and y.is_contiguous()
+    if isinstance(x, StagedInputs):
+        assert y is None
+        xp, yp = x.x_ptr, x.y_ptr
+    else:
+        assert x.dtype == torch.float32 and x.is_contiguous()
+        assert y.dtype == torch.int32 and y.is_contiguous()
+        xp, yp = x.data_ptr(), y.data_ptr()
     loss = c_float()
     raw = ctypes.byref(part.raw) if part is not None else None
-    _check(_lib.hs_step(ctx.ptr, c_void_p(params.data_ptr()), c_void_p(x.data_ptr()), c_void_p(y.data_ptr()),
-                        raw, float(lr), c_void_p(_stream_ptr(stream)), ctypes.byref(loss) if want_loss else None),
-           ctx.ptr)
+    _check(_lib.hs_step(ctx.ptr, c_void_p(params.data_ptr()), c_void_p(xp), c_void_p(yp), raw, float(lr),
+                        c_void_p(_stream_ptr(stream)), ctypes.byref(loss) if want_loss else None), ctx.ptr)
     return loss.value if want_loss else None
 
 

@@ -83,6 +83,14 @@ struct hs_ctx {
   float* d_gdebug = nullptr;
   void* d_xstage = nullptr;
   int32_t* d_ystage = nullptr;
+  // double-buffered input staging (hs_stage_inputs): slot k holds one step's x and y
+  float* d_xslot[2] = {nullptr, nullptr};
+  int32_t* d_yslot[2] = {nullptr, nullptr};
+  cudaEvent_t slot_staged[2] = {nullptr, nullptr};     // copy into slot k done (on the staging stream)
+  cudaEvent_t slot_consumed[2] = {nullptr, nullptr};   // the step that read slot k done (on its stream)
+  bool slot_pending[2] = {false, false};               // staged, not yet read by a step
+  bool slot_used[2] = {false, false};                  // slot_consumed[k] has been recorded
+  int next_slot = 0;
   const float* shadow_src = nullptr;
   bool shadow_valid = false;
   bool debug = false;

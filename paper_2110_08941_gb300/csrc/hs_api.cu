@@ -309,6 +309,11 @@ void free_all(hs_ctx* c) {
     cudaEventDestroy(r.b);
   }
   for (cudaEvent_t e : c->event_pool) cudaEventDestroy(e);
+  for (int k = 0; k < 2; ++k) {
+    f(c->d_xslot[k]); f(c->d_yslot[k]);
+    if (c->slot_staged[k]) cudaEventDestroy(c->slot_staged[k]);
+    if (c->slot_consumed[k]) cudaEventDestroy(c->slot_consumed[k]);
+  }
   for (cudaEvent_t e : c->upd_ready) if (e) cudaEventDestroy(e);
   if (c->upd_done) cudaEventDestroy(c->upd_done);
   if (c->upd_stream) cudaStreamDestroy(c->upd_stream);
@@ -835,7 +840,14 @@ hs_status hs_step(hs_ctx* c, float* params, const void* x, const int32_t* y, con
   const size_t in_feat = (size_t)c->in_features;
   const float* xd = reinterpret_cast<const float*>(x);
   const int32_t* yd = y;
-  if (!is_device_ptr(x)) {
+  int slot = -1;   // inputs from hs_stage_inputs: wait for their copy, mark the slot read afterwards
+  for (int k = 0; k < 2; ++k)
+    if (c->d_xslot[k] && x == c->d_xslot[k]) slot = k;
+  if (slot >= 0) {
+    if (y != c->d_yslot[slot] || !c->slot_pending[slot])
+      return fail(c, HS_ERR_INVALID_ARG, "staged x and y must come from the same, not yet used hs_stage_inputs call");
+    HS_CUDA(c, cudaStreamWaitEvent(s, c->slot_staged[slot], 0));
+  } else if (!is_device_ptr(x)) {
     if (!c->d_xstage) {
       hs_status r = dalloc(c, &c->d_xstage, sizeof(float) * c->N * in_feat);
       if (r != HS_OK) return r;
@@ -874,6 +886,11 @@ hs_status hs_step(hs_ctx* c, float* params, const void* x, const int32_t* y, con
                              c->num_sms, s, 4, c->opt_recipe ? &r : nullptr);
     ph.launched();
   }
+  if (slot >= 0) {
+    HS_CUDA(c, cudaEventRecord(c->slot_consumed[slot], s));
+    c->slot_pending[slot] = false;
+    c->slot_used[slot] = true;
+  }
   HS_CUDA(c, cudaGetLastError());
   c->shadow_src = params;
   c->shadow_valid = (c->precision == HS_BF16);
@@ -893,6 +910,34 @@ hs_status hs_step(hs_ctx* c, float* params, const void* x, const int32_t* y, con
       return fail(c, HS_ERR_DEVICE_CHECK, buf);
     }
   }
+  return HS_OK;
+}
+
+hs_status hs_stage_inputs(hs_ctx* c, const float* x_host, const int32_t* y_host, void* stream, const float** x_dev,
+                          const int32_t** y_dev) {
+  if (!c) return HS_ERR_INVALID_ARG;
+  c->err.clear();
+  if (!x_host || !y_host || !x_dev || !y_dev) return fail(c, HS_ERR_INVALID_ARG, "x, y and the outputs must be non-NULL");
+  const int k = c->next_slot;
+  if (c->slot_pending[k])
+    return fail(c, HS_ERR_INVALID_ARG, "both staging slots hold inputs no hs_step has read yet");
+  const size_t xbytes = sizeof(float) * (size_t)c->N * (size_t)c->in_features;
+  if (!c->d_xslot[k]) {
+    hs_status r = dalloc(c, &c->d_xslot[k], xbytes);
+    if (r == HS_OK) r = dalloc(c, &c->d_yslot[k], sizeof(int32_t) * (size_t)c->N);
+    if (r != HS_OK) return r;
+    HS_CUDA(c, cudaEventCreateWithFlags(&c->slot_staged[k], cudaEventDisableTiming));
+    HS_CUDA(c, cudaEventCreateWithFlags(&c->slot_consumed[k], cudaEventDisableTiming));
+  }
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (c->slot_used[k]) HS_CUDA(c, cudaStreamWaitEvent(s, c->slot_consumed[k], 0));   // the last reader is done
+  HS_CUDA(c, cudaMemcpyAsync(c->d_xslot[k], x_host, xbytes, cudaMemcpyHostToDevice, s));
+  HS_CUDA(c, cudaMemcpyAsync(c->d_yslot[k], y_host, sizeof(int32_t) * (size_t)c->N, cudaMemcpyHostToDevice, s));
+  HS_CUDA(c, cudaEventRecord(c->slot_staged[k], s));
+  c->slot_pending[k] = true;
+  c->next_slot = k ^ 1;
+  *x_dev = c->d_xslot[k];
+  *y_dev = c->d_yslot[k];
   return HS_OK;
 }
 

@@ -225,3 +225,52 @@ def test_cp_history_partitions_bit_exact(mode, param, name):
             hs.hs_set_cp_history(ctx, hs.HS_CP_EMA, 1.5)
     finally:
         ctx.close()
+
+
+@pytest.mark.parametrize("name", [synth.CFG1, synth.CFG4])
+def test_staged_inputs_pipeline_matches_device_inputs(name):
+    """hs_stage_inputs copies step t + 1's inputs on a copy stream while step t runs (two slots);
+    the steps see the same inputs as device tensors handed to hs_step, bit for bit."""
+    wl, ctx, xd, yd, theta0 = _ctx_and_data(name)
+    try:
+        pa = torch.tensor(theta0, device="cuda")
+        la = [hs.hs_step(ctx, pa, xd, yd, None, wl.lr) for _ in range(4)]
+        pb = torch.tensor(theta0, device="cuda")
+        hs.hs_sync_params(ctx, pb)
+        xh, yh = xd.cpu().pin_memory(), yd.cpu().pin_memory()
+        copy = torch.cuda.Stream()
+        nxt = hs.hs_stage_inputs(ctx, xh, yh, stream=copy)
+        lb = []
+        for t in range(4):
+            cur = nxt
+            if t < 3:
+                nxt = hs.hs_stage_inputs(ctx, xh, yh, stream=copy)
+            lb.append(hs.hs_step(ctx, pb, cur, None, None, wl.lr))
+        assert la == lb
+        assert torch.equal(pa, pb)
+    finally:
+        ctx.close()
+
+
+def test_staging_slots_are_checked():
+    wl, ctx, xd, yd, theta0 = _ctx_and_data(synth.CFG1)
+    try:
+        p = torch.tensor(theta0, device="cuda")
+        xh, yh = xd.cpu().pin_memory(), yd.cpu().pin_memory()
+        a = hs.hs_stage_inputs(ctx, xh, yh)
+        b = hs.hs_stage_inputs(ctx, xh, yh)
+        with pytest.raises(hs.HsError) as e:              # both slots staged, none read yet
+            hs.hs_stage_inputs(ctx, xh, yh)
+        assert e.value.status == hs.HS_ERR_INVALID_ARG
+        mixed = hs.StagedInputs(a.x_ptr, b.y_ptr, None)   # x of one slot with y of the other
+        with pytest.raises(hs.HsError) as e:
+            hs.hs_step(ctx, p, mixed, None, None, wl.lr)
+        assert e.value.status == hs.HS_ERR_INVALID_ARG
+        hs.hs_step(ctx, p, a, None, None, wl.lr)
+        with pytest.raises(hs.HsError):                   # a slot is read once per staging
+            hs.hs_step(ctx, p, a, None, None, wl.lr)
+        hs.hs_step(ctx, p, b, None, None, wl.lr)
+        c = hs.hs_stage_inputs(ctx, xh, yh)               # slots free again
+        hs.hs_step(ctx, p, c, None, None, wl.lr)
+    finally:
+        ctx.close()
