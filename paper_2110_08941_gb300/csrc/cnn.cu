@@ -7,6 +7,7 @@
 // n_m * Ho * Wo is split into chunks so that the few output tiles still fill the GPU; the chunk
 // partials are added per worker in a fixed order.  Activations are NHWC (channels last).
 #include <algorithm>
+#include <climits>
 #include <cstring>
 
 #include "ctx.cuh"
@@ -274,8 +275,10 @@ inline int blocks_for(int64_t n, int threads) { return (int)((n + threads - 1) /
 }  // namespace
 
 // ---------------------------------------------------------------------------------- plans
-// Weight-gradient plan for one layer: groups = (worker, K chunk); both operands MN-major
-// [rows][cols]; chunk partial g lands at partial + g * rows_out * ldp.
+// Weight-gradient plan for one layer: one group per worker (up to 32 per launch), both operands
+// MN-major [rows][cols] over the worker's rows, each worker's reduction split in the kernel into
+// `ksplit` contiguous k-block ranges (parts) so that about 2 x 152 tiles run although the output
+// is only Cout x (9 Cin + 1): part j of worker m lands at partial[m * ksplit + j].
 hs_status cnn_build_wgrad_plan(hs_ctx* c, int layer, const __nv_bfloat16* a, int a_cols, int64_t lda,
                                const __nv_bfloat16* b, int b_cols, int64_t ldb, int64_t rows_per_sample) {
   const char* why = nullptr;
@@ -286,49 +289,45 @@ hs_status cnn_build_wgrad_plan(hs_ctx* c, int layer, const __nv_bfloat16* a, int
   wg.K = b_cols;
   wg.ldp = (int)round_up(b_cols, 4);
   const int tiles = (int)(((a_cols + kTcBM - 1) / kTcBM) * ((b_cols + kTcBN - 1) / kTcBN));
-  const int64_t total_rows = (int64_t)c->N * rows_per_sample;
-  const int64_t target_groups = std::max<int64_t>(1, (2LL * c->num_sms + tiles - 1) / tiles);
-  // chunks hold whole samples (so an implicit-patch map can start at a chunk's first image) and
-  // whole 64-row k-blocks
-  const int64_t align = rows_per_sample % kTcBK == 0 ? rows_per_sample
-                      : kTcBK % rows_per_sample == 0 ? kTcBK : rows_per_sample * kTcBK;
-  const int64_t chunk = std::max<int64_t>(round_up(512, align),
-                                          round_up((total_rows + target_groups - 1) / target_groups, align));
-  std::vector<std::pair<int64_t, int64_t>> ranges;
+  const int64_t part_elems = (int64_t)wg.rows_out * wg.ldp;
+  int64_t min_kb = INT64_MAX;
+  for (int m = 0; m < c->M; ++m)
+    min_kb = std::min<int64_t>(min_kb, ((int64_t)c->counts[m] * rows_per_sample + kTcBK - 1) / kTcBK);
+  const int per_launch = std::min(c->M, kTcMaxGroups);
+  const int64_t want = (2LL * c->num_sms + (int64_t)per_launch * tiles - 1) / ((int64_t)per_launch * tiles);
+  const int64_t fit = wg.partial_capacity / part_elems / c->M;   // parts the partial buffer holds per worker
+  const int ksplit = (int)std::max<int64_t>(1, std::min<int64_t>(std::min<int64_t>(want, min_kb), fit));
+  if ((int64_t)c->M * ksplit * part_elems > wg.partial_capacity)
+    return fail(c, HS_ERR_OOM, "split-K partial buffer too small");
   std::vector<int32_t> begin;
-  for (int m = 0; m < c->M; ++m) {
-    begin.push_back((int32_t)ranges.size());
-    const int64_t r0 = (int64_t)c->offsets[m] * rows_per_sample, r1 = (int64_t)c->offsets[m + 1] * rows_per_sample;
-    for (int64_t r = r0; r < r1; r += chunk) ranges.push_back({r, std::min(chunk, r1 - r)});
-  }
-  begin.push_back((int32_t)ranges.size());
-  const int G = (int)ranges.size();
-  if ((int64_t)G * wg.rows_out * wg.ldp > wg.partial_capacity) return fail(c, HS_ERR_OOM, "split-K partial buffer too small");
-  for (int g0 = 0; g0 < G; g0 += kTcMaxGroups) {
-    const int ng = std::min(kTcMaxGroups, G - g0);
+  for (int m = 0; m <= c->M; ++m) begin.push_back(m * ksplit);
+  for (int g0 = 0; g0 < c->M; g0 += kTcMaxGroups) {
+    const int ng = std::min(kTcMaxGroups, c->M - g0);
     wg.plans.emplace_back();
     TcGemmParams& p = wg.plans.back();
     std::memset(&p, 0, sizeof(p));
     for (int g = 0; g < ng; ++g) {
-      const auto& rg = ranges[g0 + g];
-      float* dg = wg.d_partial + (int64_t)(g0 + g) * wg.rows_out * wg.ldp;
-      bool ok = tc_make_mnmajor_map(&p.tmA[g], TcOperand{a + rg.first * lda, rg.second, a_cols, lda}, &why) &&
-                tc_make_store_map(&p.tmD[g], dg, true, a_cols, b_cols, wg.ldp, &why);
+      const int m = g0 + g;
+      const int64_t r0 = (int64_t)c->offsets[m] * rows_per_sample;
+      const int64_t rows = (int64_t)c->counts[m] * rows_per_sample;
+      float* dg = wg.d_partial + (int64_t)m * ksplit * part_elems;
+      bool ok = tc_make_mnmajor_map(&p.tmA[g], TcOperand{a + r0 * lda, rows, a_cols, lda}, &why) &&
+                (ksplit > 1 ? tc_make_store_map_parts(&p.tmD[g], dg, a_cols, b_cols, wg.ldp, ksplit, part_elems, &why)
+                            : tc_make_store_map(&p.tmD[g], dg, true, a_cols, b_cols, wg.ldp, &why));
       if (conv && conv->implicit) {
-        // B = the implicit patch rows of the chunk's samples, read from the layer's input
-        const int64_t img0 = rg.first / rows_per_sample;
-        const int64_t imgs = (rg.second + rows_per_sample - 1) / rows_per_sample;
+        // B = the implicit patch rows of the worker's samples, read from the layer's input
         const __nv_bfloat16* in = reinterpret_cast<const __nv_bfloat16*>(c->d_cact[layer - 1]) +
-                                  img0 * conv->hin * conv->win * conv->cin;
-        ok = ok && tc_make_conv_map(&p.tmB[g], in, imgs, conv->hin, conv->win, conv->cin, conv->hout, conv->wout,
-                                    conv->stride, &why);
+                                  (int64_t)c->offsets[m] * conv->hin * conv->win * conv->cin;
+        ok = ok && tc_make_conv_map(&p.tmB[g], in, c->counts[m], conv->hin, conv->win, conv->cin, conv->hout,
+                                    conv->wout, conv->stride, &why);
       } else {
-        ok = ok && tc_make_mnmajor_map(&p.tmB[g], TcOperand{b + rg.first * ldb, rg.second, b_cols, ldb}, &why);
+        ok = ok && tc_make_mnmajor_map(&p.tmB[g], TcOperand{b + r0 * ldb, rows, b_cols, ldb}, &why);
       }
       if (!ok) return fail(c, HS_ERR_CUDA, why);
-      p.num_kb[g] = (int32_t)((rg.second + kTcBK - 1) / kTcBK);
+      p.num_kb[g] = (int32_t)((rows + kTcBK - 1) / kTcBK);
     }
     p.groups = ng;
+    p.ksplit = ksplit;
     p.Mdim = a_cols;
     p.Ndim = b_cols;
     p.n_store = b_cols;
@@ -342,9 +341,12 @@ hs_status cnn_build_wgrad_plan(hs_ctx* c, int layer, const __nv_bfloat16* a, int
       p.conv = tc_conv_geom(conv->cin, conv->hout, conv->wout, conv->stride);
       if (!tc_make_mnmajor_map(&p.tmOnes, TcOperand{c->d_ones, 64, 64, 64}, &why)) return fail(c, HS_ERR_CUDA, why);
     }
-    p.D = wg.d_partial + (int64_t)g0 * wg.rows_out * wg.ldp;
+    // outputs of at most 128 rows (Cout <= 128) fill the one-SM form's 128-row tile but only half
+    // of an SM pair's 256 rows
+    if (a_cols <= kTcBM) p.form = kTcFormSingle;
+    p.D = wg.d_partial + (int64_t)g0 * ksplit * part_elems;
     p.ldd = wg.ldp;
-    p.d_gstride = (int64_t)wg.rows_out * wg.ldp;
+    p.d_gstride = (int64_t)ksplit * part_elems;
     p.st = c->d_status;
   }
   cudaError_t e = cudaMemcpy(wg.d_chunk_begin, begin.data(), sizeof(int32_t) * begin.size(), cudaMemcpyHostToDevice);

@@ -70,7 +70,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
 
-  const int total = p.groups * p.tiles_m * p.tiles_n;
+  const int total = p.groups * ksplit_of(p) * p.tiles_m * p.tiles_n;
 
   if (warp == 0) {
     if (lane == 0) {
@@ -79,17 +79,17 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
       uint32_t ph = 0;
       int last_g = -1;
       for (int t = blockIdx.x; t < total && !*abort_flag; t += gridDim.x) {
-        const TileCoord c = decode_tile(t, p.tiles_m, p.tiles_n);
-        const CUtensorMap* ta = &p.tmA[c.g];
-        const CUtensorMap* tb = &p.tmB[c.g];
-        if (c.g != last_g) {
+        const TileWork w = tile_work(p, t, p.tiles_m, p.tiles_n);
+        const TileCoord c = w.c;
+        const CUtensorMap* ta = &p.tmA[w.g];
+        const CUtensorMap* tb = &p.tmB[w.g];
+        if (w.g != last_g) {
           tma_prefetch_desc(ta);
           tma_prefetch_desc(tb);
-          last_g = c.g;
+          last_g = w.g;
         }
-        const int nkb = p.num_kb[c.g];
         bool ok = true;
-        for (int kb = 0; kb < nkb; ++kb) {
+        for (int kb = w.kb_lo; kb < w.kb_hi; ++kb) {
           if (!mbar_wait(smem_u32(&empty_bar[s]), ph ^ 1u, abort_flag)) { ok = false; break; }
           const uint32_t fb = smem_u32(&full_bar[s]);
           mbar_expect_tx(fb, STAGE_TX);
@@ -104,7 +104,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
 #pragma unroll
               for (int j = 0; j < BM / 64; ++j) {
                 int cc[4];
-                if (p.conv_a == 2) subpixel_box_coords(p.conv, c.g, c.tm * BM + 64 * j, k0, cc);
+                if (p.conv_a == 2) subpixel_box_coords(p.conv, w.g, c.tm * BM + 64 * j, k0, cc);
                 else conv_box_coords(p.conv, c.tm * BM + 64 * j, k0, cc);
                 tma_load_4d(a_dst + j * MN_CHUNK, ta, cc, fb);
               }
@@ -149,8 +149,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
       int ab = 0;
       uint32_t aph = 0;
       for (int t = blockIdx.x; t < total && !*abort_flag; t += gridDim.x) {
-        const TileCoord c = decode_tile(t, p.tiles_m, p.tiles_n);
-        const int nkb = p.num_kb[c.g];
+        const TileWork w = tile_work(p, t, p.tiles_m, p.tiles_n);
         if (!mbar_wait(smem_u32(&tempty_bar[ab]), aph ^ 1u, abort_flag)) {
           record_error(p.st, kDevWaitTimeout, 2);
           *abort_flag = 1;
@@ -159,7 +158,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + (uint32_t)(ab * BN);
         bool ok = true;
-        for (int kb = 0; kb < nkb; ++kb) {
+        for (int kb = w.kb_lo; kb < w.kb_hi; ++kb) {
           if (!mbar_wait(smem_u32(&full_bar[s]), ph, abort_flag)) { ok = false; break; }
           tc_fence_after();
           const uint32_t a_base = smem_u32(sA + s * A_STAGE);
@@ -170,7 +169,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
                                      : make_sdesc(a_base + kk * 32, 16, 1024);
             const uint64_t bd = B_MN ? make_sdesc(b_base + kk * 2048, MN_CHUNK, 1024)
                                      : make_sdesc(b_base + kk * 32, 16, 1024);
-            umma_bf16(d_tmem, ad, bd, idesc, (kb | kk) != 0 ? 1u : 0u);
+            umma_bf16(d_tmem, ad, bd, idesc, (kb != w.kb_lo || kk != 0) ? 1u : 0u);
           }
           umma_commit(smem_u32(&empty_bar[s]));
           if (++s == S) { s = 0; ph ^= 1u; }
@@ -199,7 +198,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
     int ab = 0;
     uint32_t aph = 0;
     for (int t = blockIdx.x; t < total; t += gridDim.x) {
-      const TileCoord c = decode_tile(t, p.tiles_m, p.tiles_n);
+      const TileWork w = tile_work(p, t, p.tiles_m, p.tiles_n);
+      const TileCoord c = w.c;
       int ok = 1;
       if (lane == 0) ok = mbar_wait(smem_u32(&tfull_bar[ab]), aph, abort_flag) ? 1 : 0;
       ok = __shfl_sync(0xffffffffu, ok, 0);
@@ -214,7 +214,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
       tc_fence_after();
       const int row0 = c.tm * BM + q * 32;
       const int row = row0 + lane;
-      const CUtensorMap* td = &p.tmD[c.g];
+      const CUtensorMap* td = &p.tmD[w.g];
       const uint32_t t_row = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(ab * BN);
 #pragma unroll 1
       for (int u = 0; u < kUnits; ++u) {
@@ -226,7 +226,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
         tmem_ld_wait(r);
         if (!kF32Out) tmem_ld_wait(r2);
         uint4 o[8];
-        epilogue_unit<EPI, CONV>(p, c.g, row, n_base, r, r2, o);
+        epilogue_unit<EPI, CONV>(p, w.g, row, n_base, r, r2, o);
         if (lane == 0) bulk_wait_read_1();   // the store that last used this buffer has read it
         __syncwarp();
         const uint32_t buf = stage_base + (uint32_t)(sb * 4096);
@@ -236,7 +236,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
         fence_proxy_async_smem();
         __syncwarp();
         if (lane == 0) {
-          store_strip<CONV>(p, td, buf, n_base, row0);
+          store_strip<CONV>(p, td, buf, n_base, row0, w.part);
           bulk_commit();
         }
         sb ^= 1;
@@ -405,6 +405,27 @@ bool tc_make_grid_map(CUtensorMap* tm, const void* base, int C, int cols, int ro
   return true;
 }
 
+bool tc_make_store_map_parts(CUtensorMap* tm, float* base, int64_t rows, int64_t cols, int64_t ld, int64_t parts,
+                             int64_t part_stride, const char** why) {
+  if (!g_encode && !tc_init_driver(why)) return false;
+  if ((reinterpret_cast<uintptr_t>(base) & 15u) != 0 || (ld * 4) % 16 || (part_stride * 4) % 16) {
+    *why = "TMA store base or stride is not 16-byte aligned";
+    return false;
+  }
+  cuuint64_t dims[3] = {(cuuint64_t)cols, (cuuint64_t)rows, (cuuint64_t)parts};
+  cuuint64_t strides[2] = {(cuuint64_t)ld * 4, (cuuint64_t)part_stride * 4};
+  cuuint32_t box[3] = {32, 32, 1};
+  cuuint32_t estr[3] = {1, 1, 1};
+  CUresult r = g_encode(tm, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, base, dims, strides, box, estr,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) {
+    *why = "cuTensorMapEncodeTiled rejected the split-K output";
+    return false;
+  }
+  return true;
+}
+
 bool tc_make_mnmajor_map(CUtensorMap* tm, const TcOperand& op, const char** why) {
   return encode_2d(tm, op.base, (uint64_t)op.cols, (uint64_t)op.rows, (uint64_t)op.ld * 2, 64, kTcBK, why);
 }
@@ -431,7 +452,7 @@ void tc_set_form(int form) { g_form = (form == kTcFormPair) ? kTcFormPair : kTcF
 int tc_get_form() { return g_form; }
 
 cudaError_t launch_tc_gemm(const TcGemmParams& p, int num_sms, cudaStream_t s) {
-  return launch_tc_gemm_form(p, num_sms, s, g_form);
+  return launch_tc_gemm_form(p, num_sms, s, p.form ? p.form : g_form);
 }
 
 cudaError_t launch_tc_gemm_form(const TcGemmParams& p_in, int num_sms, cudaStream_t s, int form) {
@@ -439,7 +460,7 @@ cudaError_t launch_tc_gemm_form(const TcGemmParams& p_in, int num_sms, cudaStrea
   TcGemmParams p = p_in;
   p.tiles_m = (p.Mdim + BM - 1) / BM;
   p.tiles_n = (p.n_store + BN - 1) / BN;
-  const int total = p.groups * p.tiles_m * p.tiles_n;
+  const int total = p.groups * (p.ksplit > 1 ? p.ksplit : 1) * p.tiles_m * p.tiles_n;
   if (total <= 0) return cudaSuccess;
   const int grid = total < num_sms ? total : num_sms;
   // implicit convolution operands (forward, weight gradient, sub-pixel input gradient)

@@ -59,6 +59,10 @@ struct TcGemmParams {
   CUtensorMap tmOnes;              // MN-major [64][64] bf16, column 0 ones, the rest zero (conv_b)
   TcConvGeom conv;
   int32_t conv_a, conv_b, conv_d;
+  int32_t form;                    // kernel form for this product (TcForm), 0 = the process default
+  int32_t ksplit;                  // >= 2: each group's k-blocks split into ksplit contiguous parts, part j
+                                   // a tile of its own writing part j of tmD[g], a 3-D map [parts][rows][cols]
+                                   // (needs num_kb[g] >= ksplit); 0 or 1: no split
   int32_t num_kb[kTcMaxGroups];
   int32_t groups;
   int32_t Mdim, Ndim, n_store;
@@ -101,6 +105,9 @@ bool tc_make_grid_map(CUtensorMap* tm, const void* base, int C, int cols, int ro
 // 128-byte boxes; rows >= `rows` and columns >= `cols` of a box are not written.
 bool tc_make_store_map(CUtensorMap* tm, void* base, bool fp32, int64_t rows, int64_t cols, int64_t ld,
                        const char** why);
+// The same over `parts` such matrices `part_stride` elements apart (split-K partials, fp32).
+bool tc_make_store_map_parts(CUtensorMap* tm, float* base, int64_t rows, int64_t cols, int64_t ld, int64_t parts,
+                             int64_t part_stride, const char** why);
 
 constexpr int kTcBM = 128, kTcBN = 256, kTcBK = 64, kTcStages = 4;
 constexpr int kTcStagingBytes = 4 * 2 * 32 * 128;   // 4 epilogue warps x 2 buffers x (32 rows x 128 B)

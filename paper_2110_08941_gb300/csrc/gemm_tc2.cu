@@ -136,7 +136,7 @@ __global__ void __launch_bounds__(kThreads2, 1) tc_gemm_pair_kernel(const __grid
 
   const int tiles_m = (p.Mdim + PM - 1) / PM;
   const int tiles_n = (p.n_store + PN - 1) / PN;
-  const int total = p.groups * tiles_m * tiles_n;
+  const int total = p.groups * ksplit_of(p) * tiles_m * tiles_n;
   const int pair_id = blockIdx.x >> 1;
   const int n_pairs = gridDim.x >> 1;
 
@@ -147,19 +147,19 @@ __global__ void __launch_bounds__(kThreads2, 1) tc_gemm_pair_kernel(const __grid
       uint32_t ph = 0;
       int last_g = -1;
       for (int t = pair_id; t < total && !*abort_flag; t += n_pairs) {
-        const TileCoord c = decode_tile(t, tiles_m, tiles_n);
-        const CUtensorMap* ta = &p.tmA[c.g];
-        const CUtensorMap* tb = &p.tmB[c.g];
-        if (c.g != last_g) {
+        const TileWork w = tile_work(p, t, tiles_m, tiles_n);
+        const TileCoord c = w.c;
+        const CUtensorMap* ta = &p.tmA[w.g];
+        const CUtensorMap* tb = &p.tmB[w.g];
+        if (w.g != last_g) {
           tma_prefetch_desc(ta);
           tma_prefetch_desc(tb);
-          last_g = c.g;
+          last_g = w.g;
         }
-        const int nkb = p.num_kb[c.g];
         const int m0 = c.tm * PM + (int)rank * HM;
         const int n0 = c.tn * PN + (int)rank * HN;
         bool ok = true;
-        for (int kb = 0; kb < nkb; ++kb) {
+        for (int kb = w.kb_lo; kb < w.kb_hi; ++kb) {
           if (!mbar_wait(smem_u32(&empty_bar[s]), ph ^ 1u, abort_flag)) { ok = false; break; }
           const uint32_t fb_local = smem_u32(&full_bar[s]);
           const uint32_t fb = map_to_rank(fb_local, 0);
@@ -176,7 +176,7 @@ __global__ void __launch_bounds__(kThreads2, 1) tc_gemm_pair_kernel(const __grid
 #pragma unroll
             for (int j = 0; j < HM / 64; ++j) {
               int cc[4];
-              if (p.conv_a == 2) subpixel_box_coords(p.conv, c.g, m0 + 64 * j, k0, cc);
+              if (p.conv_a == 2) subpixel_box_coords(p.conv, w.g, m0 + 64 * j, k0, cc);
               else conv_box_coords(p.conv, m0 + 64 * j, k0, cc);
               tma_load_4d_pair(a_dst + j * MN_CHUNK, ta, cc, fb);
             }
@@ -218,8 +218,7 @@ __global__ void __launch_bounds__(kThreads2, 1) tc_gemm_pair_kernel(const __grid
       int ab = 0;
       uint32_t aph = 0;
       for (int t = pair_id; t < total && !*abort_flag; t += n_pairs) {
-        const TileCoord c = decode_tile(t, tiles_m, tiles_n);
-        const int nkb = p.num_kb[c.g];
+        const TileWork w = tile_work(p, t, tiles_m, tiles_n);
         if (!mbar_wait(smem_u32(&tempty_bar[ab]), aph ^ 1u, abort_flag)) {
           record_error(p.st, kDevWaitTimeout, 12);
           *abort_flag = 1;
@@ -228,7 +227,7 @@ __global__ void __launch_bounds__(kThreads2, 1) tc_gemm_pair_kernel(const __grid
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + (uint32_t)(ab * PN);
         bool ok = true;
-        for (int kb = 0; kb < nkb; ++kb) {
+        for (int kb = w.kb_lo; kb < w.kb_hi; ++kb) {
           if (!mbar_wait(smem_u32(&full_bar[s]), ph, abort_flag)) { ok = false; break; }
           tc_fence_after();
           const uint32_t a_base = smem_u32(smem + s * STAGE2);
@@ -239,7 +238,7 @@ __global__ void __launch_bounds__(kThreads2, 1) tc_gemm_pair_kernel(const __grid
                                      : make_sdesc(a_base + kk * 32, 16, 1024);
             const uint64_t bd = B_MN ? make_sdesc(b_base + kk * 2048, MN_CHUNK, 1024)
                                      : make_sdesc(b_base + kk * 32, 16, 1024);
-            umma_bf16_pair(d_tmem, ad, bd, idesc, (kb | kk) != 0 ? 1u : 0u);
+            umma_bf16_pair(d_tmem, ad, bd, idesc, (kb != w.kb_lo || kk != 0) ? 1u : 0u);
           }
           umma_commit_pair(smem_u32(&empty_bar[s]));
           if (++s == S2) { s = 0; ph ^= 1u; }
@@ -264,7 +263,8 @@ __global__ void __launch_bounds__(kThreads2, 1) tc_gemm_pair_kernel(const __grid
     int ab = 0;
     uint32_t aph = 0;
     for (int t = pair_id; t < total; t += n_pairs) {
-      const TileCoord c = decode_tile(t, tiles_m, tiles_n);
+      const TileWork w = tile_work(p, t, tiles_m, tiles_n);
+      const TileCoord c = w.c;
       int ok = 1;
       if (lane == 0) ok = mbar_wait(smem_u32(&tfull_bar[ab]), aph, abort_flag) ? 1 : 0;
       ok = __shfl_sync(0xffffffffu, ok, 0);
@@ -279,7 +279,7 @@ __global__ void __launch_bounds__(kThreads2, 1) tc_gemm_pair_kernel(const __grid
       tc_fence_after();
       const int row0 = c.tm * PM + (int)rank * HM + q * 32;
       const int row = row0 + lane;
-      const CUtensorMap* td = &p.tmD[c.g];
+      const CUtensorMap* td = &p.tmD[w.g];
       const uint32_t t_row = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(ab * PN);
 #pragma unroll 1
       for (int u = 0; u < kUnits; ++u) {
@@ -291,7 +291,7 @@ __global__ void __launch_bounds__(kThreads2, 1) tc_gemm_pair_kernel(const __grid
         tmem_ld_wait(r);
         if (!kF32Out) tmem_ld_wait(r2);
         uint4 o[8];
-        epilogue_unit<EPI, CONV>(p, c.g, row, n_base, r, r2, o);
+        epilogue_unit<EPI, CONV>(p, w.g, row, n_base, r, r2, o);
         if (lane == 0) bulk_wait_read_1();
         __syncwarp();
         const uint32_t buf = stage_base + (uint32_t)(sb * 4096);
@@ -301,7 +301,7 @@ __global__ void __launch_bounds__(kThreads2, 1) tc_gemm_pair_kernel(const __grid
         fence_proxy_async_smem();
         __syncwarp();
         if (lane == 0) {
-          store_strip<CONV>(p, td, buf, n_base, row0);
+          store_strip<CONV>(p, td, buf, n_base, row0, w.part);
           bulk_commit();
         }
         sb ^= 1;
@@ -375,7 +375,7 @@ cudaError_t launch_pair_variant(const TcGemmParams& p, int pairs_wanted, int num
 cudaError_t launch_tc_gemm_pair(const TcGemmParams& p, int num_sms, cudaStream_t s) {
   const int tiles_m = (p.Mdim + PM - 1) / PM;
   const int tiles_n = (p.n_store + PN - 1) / PN;
-  const int total = p.groups * tiles_m * tiles_n;
+  const int total = p.groups * (p.ksplit > 1 ? p.ksplit : 1) * tiles_m * tiles_n;
   if (total <= 0) return cudaSuccess;
   const int pairs = total;
   const int grid = num_sms;   // forwarded as the SM count for the residency query

@@ -113,10 +113,17 @@ __device__ __forceinline__ void tma_store_2d(const CUtensorMap* tm, uint32_t src
 }
 // Store the 32-row strip at rows row0.. (row0 a multiple of 32), columns n_base.. through the
 // output map of the group: a 2-D [rows][cols] map, or (conv_d) a class grid of the input gradient.
+__device__ __forceinline__ void tma_store_3d(const CUtensorMap* tm, uint32_t src, int c0, int c1, int c2) {
+  asm volatile("cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%1, %2, %3}], [%4];"
+               ::"l"(reinterpret_cast<uint64_t>(tm)), "r"(c0), "r"(c1), "r"(c2), "r"(src)
+               : "memory");
+}
 template <bool CONV>
 __device__ __forceinline__ void store_strip(const TcGemmParams& p, const CUtensorMap* td, uint32_t buf, int n_base,
-                                            int row0) {
-  if (CONV && p.conv_d) {
+                                            int row0, int part) {
+  if (p.ksplit > 1) {
+    tma_store_3d(td, buf, n_base, row0, part);
+  } else if (CONV && p.conv_d) {
     const int img = row0 / p.conv.hw;
     const int c[4] = {n_base, 0, (row0 - img * p.conv.hw) / p.conv.Wo, img};
     tma_store_4d(td, buf, c);
@@ -238,6 +245,32 @@ __device__ __forceinline__ TileCoord decode_tile(int t, int tiles_m, int tiles_n
   c.tm = band * GM + within % rows;
   c.tn = within / rows;
   return c;
+}
+
+// A tile's work: its coordinates, its group and split-K part, and its k-block range.  decode_tile's
+// group index runs over groups x ksplit "virtual groups".
+struct TileWork {
+  TileCoord c;
+  int g, part, kb_lo, kb_hi;
+};
+__device__ __forceinline__ int ksplit_of(const TcGemmParams& p) { return p.ksplit > 1 ? p.ksplit : 1; }
+__device__ __forceinline__ TileWork tile_work(const TcGemmParams& p, int t, int tiles_m, int tiles_n) {
+  TileWork w;
+  w.c = decode_tile(t, tiles_m, tiles_n);
+  if (p.ksplit > 1) {
+    const int ks = p.ksplit;
+    w.g = w.c.g / ks;
+    w.part = w.c.g - w.g * ks;
+    const int nkb = p.num_kb[w.g];
+    w.kb_lo = nkb * w.part / ks;   // nkb * ks stays far below 2^31 (k-blocks of 64 rows, ks <= 304)
+    w.kb_hi = nkb * (w.part + 1) / ks;
+  } else {
+    w.g = w.c.g;
+    w.part = 0;
+    w.kb_lo = 0;
+    w.kb_hi = p.num_kb[w.g];
+  }
+  return w;
 }
 
 __device__ __forceinline__ float u2f(uint32_t u) { return __uint_as_float(u); }
