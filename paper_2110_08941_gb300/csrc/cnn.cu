@@ -66,6 +66,44 @@ __global__ void im2col_nchw_kernel(const float* __restrict__ x, int N, int C, in
     for (int k = C * 9; k < Kp; ++k) col[r * Kp + k] = from_f<T>((kTapMajor && k == C * 9) ? 1.f : 0.f);
 }
 
+// bf16 patch rows of the first convolution from the NCHW fp32 input, one thread per row: the row's
+// 9 * C tap-major values, the ones column and the zero tail are packed in registers and written
+// as 16-byte stores (Kp a multiple of 8, at most 64 here).
+template <int KP>
+__global__ void im2col_nchw_row_kernel(const float* __restrict__ x, int N, int C, int H, int W, int Ho, int Wo,
+                                       int s, __nv_bfloat16* __restrict__ col) {
+  const int64_t r = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (r >= (int64_t)N * Ho * Wo) return;
+  const int wo = (int)(r % Wo);
+  const int ho = (int)((r / Wo) % Ho);
+  const int n = (int)(r / ((int64_t)Wo * Ho));
+  float v[KP];
+#pragma unroll
+  for (int k = 0; k < KP; ++k) {
+    float val = 0.f;
+    if (k < 9 * C) {
+      const int tap = k / C, ci = k - tap * C;
+      const int hi = s * ho + tap / 3 - 1, wi = s * wo + tap % 3 - 1;
+      if (hi >= 0 && hi < H && wi >= 0 && wi < W) val = __ldg(x + (((int64_t)n * C + ci) * H + hi) * W + wi);
+    } else if (k == 9 * C) {
+      val = 1.f;
+    }
+    v[k] = val;
+  }
+  uint4* dst = reinterpret_cast<uint4*>(col + r * KP);
+#pragma unroll
+  for (int j = 0; j < KP / 8; ++j) {
+    __nv_bfloat162 a = __floats2bfloat162_rn(v[8 * j], v[8 * j + 1]), b = __floats2bfloat162_rn(v[8 * j + 2], v[8 * j + 3]);
+    __nv_bfloat162 c = __floats2bfloat162_rn(v[8 * j + 4], v[8 * j + 5]), d = __floats2bfloat162_rn(v[8 * j + 6], v[8 * j + 7]);
+    uint4 o;
+    o.x = *reinterpret_cast<uint32_t*>(&a);
+    o.y = *reinterpret_cast<uint32_t*>(&b);
+    o.z = *reinterpret_cast<uint32_t*>(&c);
+    o.w = *reinterpret_cast<uint32_t*>(&d);
+    dst[j] = o;
+  }
+}
+
 // bf16 patch rows, tap-major, eight channels per thread (16-byte copies).  The tail of each row
 // holds a ones column at 9*C (then zeros): the per-worker weight-gradient product then also
 // yields the bias gradient, sum over the worker's rows of dA.
@@ -173,6 +211,30 @@ __global__ void gap_forward_kernel(const T* __restrict__ h, int N, int HW, int C
 }
 
 // dA[n][p][c] = dpooled[n][c] / HW * 1[h[n][p][c] > 0] (pooling backward with ReLU').
+// The same for bf16 activations, eight channels per thread (16-byte loads and stores; C % 8 == 0).
+__global__ void gap_backward_vec8_kernel(const float* __restrict__ dpooled, const __nv_bfloat16* __restrict__ h,
+                                         int N, int HW, int C, __nv_bfloat16* __restrict__ dA) {
+  const int C8 = C >> 3;
+  const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= (int64_t)N * HW * C8) return;
+  const int c8 = (int)(idx % C8);
+  const int64_t n = idx / ((int64_t)HW * C8);
+  const float4 g0 = __ldg(reinterpret_cast<const float4*>(dpooled + n * C + c8 * 8));
+  const float4 g1 = __ldg(reinterpret_cast<const float4*>(dpooled + n * C + c8 * 8 + 4));
+  const float g[8] = {g0.x, g0.y, g0.z, g0.w, g1.x, g1.y, g1.z, g1.w};
+  const uint4 hv = __ldg(reinterpret_cast<const uint4*>(h) + idx);
+  const uint32_t hw4[4] = {hv.x, hv.y, hv.z, hv.w};
+  uint32_t o[4];
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    const __nv_bfloat162 pr = *reinterpret_cast<const __nv_bfloat162*>(&hw4[j]);
+    __nv_bfloat162 q = __floats2bfloat162_rn(__low2float(pr) > 0.f ? g[2 * j] / (float)HW : 0.f,
+                                             __high2float(pr) > 0.f ? g[2 * j + 1] / (float)HW : 0.f);
+    o[j] = *reinterpret_cast<uint32_t*>(&q);
+  }
+  reinterpret_cast<uint4*>(dA)[idx] = make_uint4(o[0], o[1], o[2], o[3]);
+}
+
 template <typename T>
 __global__ void gap_backward_kernel(const float* __restrict__ dpooled, const T* __restrict__ h, int N, int HW, int C,
                                     T* __restrict__ dA) {
@@ -271,6 +333,25 @@ __global__ void splitk_reduce_kernel(const float* __restrict__ partial, int rows
 }
 
 inline int blocks_for(int64_t n, int threads) { return (int)((n + threads - 1) / threads); }
+
+// bf16 patch rows of the first convolution: one thread per row where the row is short, else the
+// per-channel kernel.
+void launch_im2col_first(const float* x, int N, const ConvLayer& L, __nv_bfloat16* col, cudaStream_t s) {
+  const int T = 256;
+  const int64_t rows = L.rows;
+#define HS_ROW_CASE(KP)                                                                                      \
+  case KP:                                                                                                   \
+    im2col_nchw_row_kernel<KP><<<blocks_for(rows, T), T, 0, s>>>(x, N, L.cin, L.hin, L.win, L.hout, L.wout, \
+                                                                 L.stride, col);                           \
+    return;
+  switch (L.Kp) {
+    HS_ROW_CASE(16) HS_ROW_CASE(24) HS_ROW_CASE(32) HS_ROW_CASE(40) HS_ROW_CASE(48) HS_ROW_CASE(56) HS_ROW_CASE(64)
+    default:
+      im2col_nchw_kernel<__nv_bfloat16, true><<<blocks_for(rows * L.cin, T), T, 0, s>>>(
+          x, N, L.cin, L.hin, L.win, L.hout, L.wout, L.stride, col, L.Kp);
+  }
+#undef HS_ROW_CASE
+}
 
 }  // namespace
 
@@ -531,9 +612,7 @@ hs_status cnn_step(hs_ctx* c, float* params, const float* x, const int32_t* y, c
       const int64_t n_items = L[k].rows * L[k].cin;
       if (k == 0) {
         if (bf16)
-          im2col_nchw_kernel<__nv_bfloat16, true><<<blocks_for(n_items, T), T, 0, s>>>(
-              x, N, L[0].cin, L[0].hin, L[0].win, L[0].hout, L[0].wout, L[0].stride,
-              reinterpret_cast<__nv_bfloat16*>(c->d_col[0]), L[0].Kp);
+          launch_im2col_first(x, N, L[0], reinterpret_cast<__nv_bfloat16*>(c->d_col[0]), s);
         else
           im2col_nchw_kernel<float, false><<<blocks_for(n_items, T), T, 0, s>>>(
               x, N, L[0].cin, L[0].hin, L[0].win, L[0].hout, L[0].wout, L[0].stride,
@@ -665,7 +744,7 @@ hs_status cnn_step(hs_ctx* c, float* params, const float* x, const int32_t* y, c
         launch_gemm_f32(d, s);
       }
       if (bf16)
-        gap_backward_kernel<__nv_bfloat16><<<blocks_for((int64_t)N * hw3 * c3, T), T, 0, s>>>(
+        gap_backward_vec8_kernel<<<blocks_for((int64_t)N * hw3 * (c3 / 8), T), T, 0, s>>>(
             c->d_dpooled, reinterpret_cast<const __nv_bfloat16*>(c->d_cact[2]), N, hw3, c3,
             reinterpret_cast<__nv_bfloat16*>(c->d_dA[2]));
       else
