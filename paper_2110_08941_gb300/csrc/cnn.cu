@@ -673,7 +673,7 @@ hs_status cnn_step(hs_ctx* c, float* params, const float* x, const int32_t* y, c
     PhaseScope ph(c, HS_PHASE_LOSS, s);
     launch_softmax_xent(c->d_logits, c->Cp, y, c->d_scale, N, c->C, c->d_delta[0], c->Cp, bf16, c->d_ce, c->d_status,
                         s);
-    launch_loss_reduce(c->d_ce, c->d_offsets, c->M, c->d_w, c->d_lm, c->d_status, s);
+    launch_loss_reduce(c->d_ce, c->d_offsets, c->M, c->d_w, c->d_lm, c->d_status, c->d_ticket, s);
     ph.launched(2);
   }
   // ---- backward: layer index 3 = fc, 2..0 = conv3..conv1

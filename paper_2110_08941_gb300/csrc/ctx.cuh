@@ -76,6 +76,7 @@ struct hs_ctx {
   void* d_delta[2] = {nullptr, nullptr};
   float* d_ce = nullptr;
   float* d_lm = nullptr;
+  unsigned int* d_ticket = nullptr;   // completion counter of the per-worker loss reduction (zero between steps)
   hs::DevStatus* d_status = nullptr;
   hs::DevStatus* h_status = nullptr;   // pinned
   float* d_slabs = nullptr;        // [M, Ps]

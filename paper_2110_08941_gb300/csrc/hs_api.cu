@@ -301,7 +301,7 @@ void free_all(hs_ctx* c) {
     f(c->cnn_wgrad[k].d_partial); f(c->cnn_wgrad[k].d_chunk_begin);
   }
   for (void* p : c->d_act) f(p);
-  f(c->d_logits); f(c->d_delta[0]); f(c->d_delta[1]); f(c->d_ce); f(c->d_lm); f(c->d_status);
+  f(c->d_logits); f(c->d_delta[0]); f(c->d_delta[1]); f(c->d_ce); f(c->d_lm); f(c->d_status); f(c->d_ticket);
   f(c->d_slabs); f(c->d_shadow); f(c->d_gdebug); f(c->d_xstage); f(c->d_ystage); f(c->d_mom);
   if (c->h_status) cudaFreeHost(c->h_status);
   for (auto& r : c->pending) {
@@ -357,7 +357,7 @@ hs_status mlp_step_fp32(hs_ctx* c, float* params, const float* x, const int32_t*
     hs::launch_softmax_xent(c->d_logits, c->Cp, y, c->fused_sync ? c->d_scale_fused : c->d_scale, c->N, c->C,
                             c->delta_buf(L - 1), c->Cp, false,
                             c->d_ce, c->d_status, s);
-    hs::launch_loss_reduce(c->d_ce, c->d_offsets, c->M, c->d_w, c->d_lm, c->d_status, s);
+    hs::launch_loss_reduce(c->d_ce, c->d_offsets, c->M, c->d_w, c->d_lm, c->d_status, c->d_ticket, s);
     ph.launched(2);
   }
   for (int l = L - 1; l >= 0; --l) {
@@ -437,7 +437,7 @@ hs_status mlp_step_bf16(hs_ctx* c, float* params, const float* x, const int32_t*
     hs::launch_softmax_xent(c->d_logits, c->Cp, y, c->fused_sync ? c->d_scale_fused : c->d_scale, c->N, c->C,
                             c->delta_buf(L - 1), c->Cp, true,
                             c->d_ce, c->d_status, s);
-    hs::launch_loss_reduce(c->d_ce, c->d_offsets, c->M, c->d_w, c->d_lm, c->d_status, s);
+    hs::launch_loss_reduce(c->d_ce, c->d_offsets, c->M, c->d_w, c->d_lm, c->d_status, c->d_ticket, s);
     ph.launched(2);
   }
   for (int l = L - 1; l >= 0; --l) {
@@ -715,6 +715,7 @@ hs_status hs_init(const hs_model_desc* model, int32_t M, const double* compute_w
   chk(dalloc(c, &c->d_ce, sizeof(float) * N));
   chk(dalloc(c, &c->d_lm, sizeof(float) * M));
   chk(dalloc(c, &c->d_status, sizeof(DevStatus)));
+  chk(dalloc(c, &c->d_ticket, sizeof(unsigned int)));
   chk(dalloc(c, &c->d_slabs, sizeof(float) * (size_t)M * (size_t)c->Ps));
   if (c->precision == HS_BF16) chk(dalloc(c, &c->d_shadow, sizeof(__nv_bfloat16) * (size_t)c->Ps));
   if (s2 == HS_OK) {
@@ -723,6 +724,7 @@ hs_status hs_init(const hs_model_desc* model, int32_t M, const double* compute_w
   }
   if (s2 == HS_OK) {
     e = cudaMemset(c->d_status, 0, sizeof(DevStatus));
+    if (e == cudaSuccess) e = cudaMemset(c->d_ticket, 0, sizeof(unsigned int));
     if (e == cudaSuccess) e = cudaMemset(c->d_slabs, 0, sizeof(float) * (size_t)M * (size_t)c->Ps);
     if (e == cudaSuccess && c->d_shadow) e = cudaMemset(c->d_shadow, 0, sizeof(__nv_bfloat16) * (size_t)c->Ps);
     if (e == cudaSuccess) e = cudaMemset(c->d_delta[0], 0, es * delta_elems);

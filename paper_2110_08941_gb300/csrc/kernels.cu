@@ -127,12 +127,85 @@ __global__ void softmax_xent_kernel(const float* __restrict__ logits, int ldl,
   }
 }
 
+// The same with the row held in registers (C <= 32 * 4 * KV, ldl and ldd multiples of 4): one
+// float4 read of the logits per chunk, exp evaluated once per entry, 8- or 16-byte stores of delta.
+template <bool kBf16, int KV>
+__global__ void softmax_xent_reg_kernel(const float* __restrict__ logits, int ldl,
+                                        const int32_t* __restrict__ y, const float* __restrict__ scale,
+                                        int N, int C, void* __restrict__ delta, int ldd,
+                                        float* __restrict__ ce, DevStatus* st) {
+  const int warps_per_block = blockDim.x >> 5;
+  const int row = blockIdx.x * warps_per_block + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (row >= N) return;
+  const float* z = logits + (int64_t)row * ldl;
+  int label = y[row];
+  if (label < 0 || label >= C) {
+    if (lane == 0) record_error(st, kDevBadLabel, row);
+    label = label < 0 ? 0 : C - 1;
+  }
+  float v[KV][4];
+  float mx = -INFINITY;
+#pragma unroll
+  for (int k = 0; k < KV; ++k) {
+    const int j = 4 * (lane + 32 * k);
+    float4 q = make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY);
+    if (j < C) q = __ldg(reinterpret_cast<const float4*>(z + j));
+    v[k][0] = q.x; v[k][1] = (j + 1 < C) ? q.y : -INFINITY;
+    v[k][2] = (j + 2 < C) ? q.z : -INFINITY; v[k][3] = (j + 3 < C) ? q.w : -INFINITY;
+#pragma unroll
+    for (int e = 0; e < 4; ++e) mx = fmaxf(mx, v[k][e]);
+  }
+  mx = warp_max(mx);
+  float se = 0.f;
+#pragma unroll
+  for (int k = 0; k < KV; ++k)
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      v[k][e] = (4 * (lane + 32 * k) + e < C) ? expf(v[k][e] - mx) : 0.f;
+      se += v[k][e];
+    }
+  se = warp_sum(se);
+  const float lse = mx + logf(se);
+  if (lane == 0) ce[row] = lse - z[label];
+  const float inv = 1.0f / se;
+  const float sc = scale[row];
+#pragma unroll
+  for (int k = 0; k < KV; ++k) {
+    const int j = 4 * (lane + 32 * k);
+    if (j >= ldd) break;
+    float d[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) d[e] = (j + e < C) ? (v[k][e] * inv - (j + e == label ? 1.f : 0.f)) * sc : 0.f;
+    if (kBf16) {
+      __nv_bfloat162 a = __floats2bfloat162_rn(d[0], d[1]), b = __floats2bfloat162_rn(d[2], d[3]);
+      uint2 o;
+      o.x = *reinterpret_cast<uint32_t*>(&a);
+      o.y = *reinterpret_cast<uint32_t*>(&b);
+      *reinterpret_cast<uint2*>(reinterpret_cast<__nv_bfloat16*>(delta) + (int64_t)row * ldd + j) = o;
+    } else {
+      *reinterpret_cast<float4*>(reinterpret_cast<float*>(delta) + (int64_t)row * ldd + j) =
+          make_float4(d[0], d[1], d[2], d[3]);
+    }
+  }
+}
+
 void launch_softmax_xent(const float* logits, int ldl, const int32_t* y, const float* scale, int N,
                          int C, void* delta, int ldd, bool delta_bf16, float* ce, DevStatus* st,
                          cudaStream_t s) {
   const int threads = 256;
   const int rows_per_block = threads / 32;
   const int blocks = (N + rows_per_block - 1) / rows_per_block;
+  if (ldl % 4 == 0 && ldd % 4 == 0 && ldd <= 1024 && C <= ldd) {
+    if (ldd <= 128) {
+      if (delta_bf16) softmax_xent_reg_kernel<true, 1><<<blocks, threads, 0, s>>>(logits, ldl, y, scale, N, C, delta, ldd, ce, st);
+      else softmax_xent_reg_kernel<false, 1><<<blocks, threads, 0, s>>>(logits, ldl, y, scale, N, C, delta, ldd, ce, st);
+    } else {
+      if (delta_bf16) softmax_xent_reg_kernel<true, 8><<<blocks, threads, 0, s>>>(logits, ldl, y, scale, N, C, delta, ldd, ce, st);
+      else softmax_xent_reg_kernel<false, 8><<<blocks, threads, 0, s>>>(logits, ldl, y, scale, N, C, delta, ldd, ce, st);
+    }
+    return;
+  }
   if (delta_bf16)
     softmax_xent_kernel<true><<<blocks, threads, 0, s>>>(logits, ldl, y, scale, N, C, delta, ldd, ce, st);
   else
@@ -141,33 +214,43 @@ void launch_softmax_xent(const float* logits, int ldl, const int32_t* y, const f
 
 // ------------------------------------------------------------------ per-worker loss reduction
 // L_m = (1/n_m) sum_{i in seg_m} ce_i (Eq. 1); loss = sum_m w_m L_m.  One block, fixed order.
+// One block per worker: L_m = mean of its per-sample losses (strided partial sums, then a tree, in
+// a fixed order); the last block to finish forms sum_m w_m L_m in worker order and resets the
+// ticket for the next step.
 __global__ void loss_reduce_kernel(const float* __restrict__ ce, const int32_t* __restrict__ offsets,
                                    int M, const float* __restrict__ w, float* __restrict__ lm,
-                                   DevStatus* st) {
+                                   DevStatus* st, unsigned int* ticket) {
   __shared__ float red[1024];
-  for (int m = 0; m < M; ++m) {
-    const int b = offsets[m], e = offsets[m + 1];
-    float acc = 0.f;
-    for (int i = b + threadIdx.x; i < e; i += blockDim.x) acc += ce[i];
-    red[threadIdx.x] = acc;
-    __syncthreads();
-    for (int h = blockDim.x >> 1; h > 0; h >>= 1) {
-      if (threadIdx.x < h) red[threadIdx.x] += red[threadIdx.x + h];
-      __syncthreads();
-    }
-    if (threadIdx.x == 0) lm[m] = red[0] / (float)(e - b);
+  __shared__ bool last;
+  const int m = blockIdx.x;
+  const int b = offsets[m], e = offsets[m + 1];
+  float acc = 0.f;
+  for (int i = b + threadIdx.x; i < e; i += blockDim.x) acc += ce[i];
+  red[threadIdx.x] = acc;
+  __syncthreads();
+  for (int h = blockDim.x >> 1; h > 0; h >>= 1) {
+    if (threadIdx.x < h) red[threadIdx.x] += red[threadIdx.x + h];
     __syncthreads();
   }
   if (threadIdx.x == 0) {
+    lm[m] = red[0] / (float)(e - b);
+    __threadfence();
+    last = (atomicAdd(ticket, 1u) == (unsigned int)(M - 1));
+  }
+  __syncthreads();
+  if (last && threadIdx.x == 0) {
+    __threadfence();
+    const volatile float* lmv = lm;
     float loss = 0.f;
-    for (int m = 0; m < M; ++m) loss += w[m] * lm[m];
+    for (int k = 0; k < M; ++k) loss += w[k] * lmv[k];
     st->loss = loss;
+    *ticket = 0u;
   }
 }
 
 void launch_loss_reduce(const float* ce, const int32_t* d_offsets, int M, const float* d_w,
-                        float* lm, DevStatus* st, cudaStream_t s) {
-  loss_reduce_kernel<<<1, 1024, 0, s>>>(ce, d_offsets, M, d_w, lm, st);
+                        float* lm, DevStatus* st, unsigned int* ticket, cudaStream_t s) {
+  loss_reduce_kernel<<<M, 1024, 0, s>>>(ce, d_offsets, M, d_w, lm, st, ticket);
 }
 
 // ------------------------------------------------------------------ per-worker bias gradient

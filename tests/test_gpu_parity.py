@@ -190,6 +190,11 @@ CNN_EDGE = [
     ((3, 16, 16, 64, 128, 64, 7), 13, 3, [1.0, 2.0, 3.5]),
     # 8x16 and 4x8 output grids, two workers
     ((3, 16, 32, 64, 64, 64, 5), 9, 2, [2.0, 1.0]),
+    # 15x15 input: conv 2 implicit but with an odd input grid (patch-space input gradient), conv 3
+    # implicit and sub-pixel
+    ((3, 15, 15, 64, 128, 64, 6), 11, 3, [1.0, 1.0, 3.0]),
+    # 36 workers: weight-gradient plans over two launches, split-K parts bounded by the smallest worker
+    ((3, 16, 16, 64, 128, 64, 7), 40, 36, None),
 ]
 
 
