@@ -32,10 +32,17 @@ enum {
  * 128 x 256 tile, HS_GEMM_FORM_PAIR = a two-SM cluster per 256 x 256 tile (tcgen05 cta_group::2). */
 enum { HS_GEMM_FORM_SINGLE = 0x100, HS_GEMM_FORM_PAIR = 0x200 };
 
+/* OR-ed into mode: the kernel's TMA producer issues no loads, so the MMA issuer's bounded wait on
+ * the first stage expires (2 s of %globaltimer) and the kernel leaves through its error path:
+ * status word set, abort flag raised for the other roles, tensor memory freed, no fault.  The
+ * call then returns HS_ERR_DEVICE_CHECK.  Exercises the device-side failure detection. */
+enum { HS_GEMM_TEST_STALL = 0x1000 };
+
 /* A, B, Z: bf16; bias: fp32 [N]; k_offsets_host: host int32 [groups+1] (HS_GEMM_WGRAD only,
  * else NULL with groups = 1).  Returns HS_ERR_INVALID_ARG for shapes the kernel cannot take
  * (leading dimensions must be multiples of 8 elements, pointers 16-byte aligned),
- * HS_ERR_CUDA on a launch or runtime error. */
+ * HS_ERR_CUDA on a launch or runtime error, HS_ERR_DEVICE_CHECK when a bounded wait in the
+ * kernel expired. */
 hs_status hs_debug_gemm_bf16(int32_t mode, int32_t M, int32_t N, int32_t K, const void* A, int64_t lda,
                              const void* B, int64_t ldb, void* D, int64_t ldd, const float* bias,
                              const void* Z, int64_t ldz, const int32_t* k_offsets_host, int32_t groups,

@@ -22,6 +22,7 @@ HS_BF16, HS_FP32_CHECK = 0, 1
 HS_SYNC_MEAN, HS_SYNC_CP_WEIGHTED, HS_SYNC_CP_LITERAL = 0, 1, 2
 HS_GEMM_FWD_RELU, HS_GEMM_FWD_LOGITS, HS_GEMM_DGRAD, HS_GEMM_WGRAD = 0, 1, 2, 3
 HS_GEMM_FORM_SINGLE, HS_GEMM_FORM_PAIR = 0x100, 0x200
+HS_GEMM_TEST_STALL = 0x1000
 
 EXPORTED = ("hs_partition_sizes", "hs_param_count", "hs_init", "hs_partition", "hs_step", "hs_sync_params",
             "hs_set_debug", "hs_debug_grads", "hs_worker_losses", "hs_destroy", "hs_status_string",

@@ -78,7 +78,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
       int s = 0;
       uint32_t ph = 0;
       int last_g = -1;
-      for (int t = blockIdx.x; t < total && !*abort_flag; t += gridDim.x) {
+      for (int t = blockIdx.x; t < total && !*abort_flag && !p.test_stall; t += gridDim.x) {
         const TileWork w = tile_work(p, t, p.tiles_m, p.tiles_n);
         const TileCoord c = w.c;
         const CUtensorMap* ta = &p.tmA[w.g];

@@ -146,7 +146,7 @@ __global__ void __launch_bounds__(kThreads2, 1) tc_gemm_pair_kernel(const __grid
       int s = 0;
       uint32_t ph = 0;
       int last_g = -1;
-      for (int t = pair_id; t < total && !*abort_flag; t += n_pairs) {
+      for (int t = pair_id; t < total && !*abort_flag && !p.test_stall; t += n_pairs) {
         const TileWork w = tile_work(p, t, tiles_m, tiles_n);
         const TileCoord c = w.c;
         const CUtensorMap* ta = &p.tmA[w.g];

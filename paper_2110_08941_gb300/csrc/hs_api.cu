@@ -1081,6 +1081,8 @@ hs_status hs_debug_gemm_bf16(int32_t mode, int32_t M, int32_t N, int32_t K, cons
                              int64_t ldb, void* D, int64_t ldd, const float* bias, const void* Z, int64_t ldz,
                              const int32_t* k_offsets_host, int32_t groups, int64_t d_gstride, void* stream) {
   g_init_error.clear();
+  const bool stall = (mode & HS_GEMM_TEST_STALL) != 0;
+  mode &= ~HS_GEMM_TEST_STALL;
   const int form = mode >> 8;
   mode &= 0xFF;
   if (form < 0 || form > 2) return fail(nullptr, HS_ERR_INVALID_ARG, "unknown kernel form");
@@ -1149,6 +1151,14 @@ hs_status hs_debug_gemm_bf16(int32_t mode, int32_t M, int32_t N, int32_t K, cons
       return fail(nullptr, HS_ERR_INVALID_ARG, why);
   }
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  DevStatus* dst = nullptr;   // the kernel's status word for this call
+  cudaError_t ea = cudaMalloc(reinterpret_cast<void**>(&dst), sizeof(DevStatus));
+  if (ea != cudaSuccess) return cuda_fail(nullptr, ea, "status word");
+  ea = cudaMemsetAsync(dst, 0, sizeof(DevStatus), s);
+  if (ea != cudaSuccess) {
+    cudaFree(dst);
+    return cuda_fail(nullptr, ea, "status word");
+  }
   for (hs::TcGemmParams& p : plans) {
     p.Mdim = M;
     p.Ndim = N;
@@ -1156,12 +1166,24 @@ hs_status hs_debug_gemm_bf16(int32_t mode, int32_t M, int32_t N, int32_t K, cons
     p.tiles_m = (M + hs::kTcBM - 1) / hs::kTcBM;
     p.tiles_n = (N + hs::kTcBN - 1) / hs::kTcBN;
     p.ldd = ldd;
-    p.st = nullptr;
+    p.st = dst;
+    p.test_stall = stall ? 1 : 0;
     cudaError_t e = hs::launch_tc_gemm_form(p, sms, s, form ? form : hs::tc_get_form());
-    if (e != cudaSuccess) return cuda_fail(nullptr, e, "GEMM launch");
+    if (e != cudaSuccess) {
+      cudaFree(dst);
+      return cuda_fail(nullptr, e, "GEMM launch");
+    }
   }
   cudaError_t e = cudaStreamSynchronize(s);
+  DevStatus hst{};
+  if (e == cudaSuccess) e = cudaMemcpy(&hst, dst, sizeof(DevStatus), cudaMemcpyDeviceToHost);
+  cudaFree(dst);
   if (e != cudaSuccess) return cuda_fail(nullptr, e, "GEMM run");
+  if (hst.err != hs::kDevOk) {
+    char buf[128];
+    std::snprintf(buf, sizeof(buf), "device check failed in the GEMM: code %d, detail %d", hst.err, hst.err_info);
+    return fail(nullptr, HS_ERR_DEVICE_CHECK, buf);
+  }
   return HS_OK;
 }
 

@@ -224,6 +224,7 @@ __device__ __forceinline__ uint64_t make_sdesc(uint32_t saddr, uint32_t lbo, uin
 }
 
 __device__ __forceinline__ void record_error(DevStatus* st, int32_t code, int32_t info) {
+  if (!st) return;
   if (st && atomicCAS(&st->err, 0, code) == 0) st->err_info = info;
 }
 
