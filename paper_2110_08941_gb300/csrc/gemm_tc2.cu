@@ -265,6 +265,8 @@ __global__ void __launch_bounds__(kThreads2, 1) tc_gemm_pair_kernel(const __grid
     for (int t = pair_id; t < total; t += n_pairs) {
       const TileWork w = tile_work(p, t, tiles_m, tiles_n);
       const TileCoord c = w.c;
+      uint4 zq[8];   // mask operand of the tile's first unit, loaded before the accumulator is ready
+      if (EPI == kTcEpiMaskBf16) load_mask_unit<CONV>(p, w.g, c.tm * PM + (int)rank * HM + q * 32 + lane, c.tn * PN, zq);
       int ok = 1;
       if (lane == 0) ok = mbar_wait(smem_u32(&tfull_bar[ab]), aph, abort_flag) ? 1 : 0;
       ok = __shfl_sync(0xffffffffu, ok, 0);
@@ -291,7 +293,9 @@ __global__ void __launch_bounds__(kThreads2, 1) tc_gemm_pair_kernel(const __grid
         tmem_ld_wait(r);
         if (!kF32Out) tmem_ld_wait(r2);
         uint4 o[8];
-        epilogue_unit<EPI, CONV>(p, w.g, row, n_base, r, r2, o);
+        epilogue_unit<EPI, CONV>(p, w.g, row, n_base, r, r2, zq, o);
+        if (EPI == kTcEpiMaskBf16 && u + 1 < kUnits)   // the next unit's mask, behind this unit's stores
+          load_mask_unit<CONV>(p, w.g, row, n_base + kUnitCols, zq);
         if (lane == 0) bulk_wait_read_1();
         __syncwarp();
         const uint32_t buf = stage_base + (uint32_t)(sb * 4096);

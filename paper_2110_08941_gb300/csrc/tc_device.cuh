@@ -285,9 +285,37 @@ __device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
 // computed from `r` (columns n_base..n_base+31) and, for bf16 outputs, `r2` (n_base+32..+63), packed
 // into eight 16-byte words.  Columns past n_store are computed but never stored (the TMA store
 // clips them); only the bias and mask reads are guarded.
+// The mask operand of one kTcEpiMaskBf16 unit: Z's 64 bf16 values at (row, n_base..n_base+63) (for
+// the sub-pixel input gradient, row is class pixel (a, b) of group grp = input pixel
+// (2a + ph, 2b + pw)); zero past Mdim rows or n_store columns.  Loaded ahead of the accumulator
+// so that the global-load latency overlaps the main loop.
+template <bool CONV>
+__device__ __forceinline__ void load_mask_unit(const TcGemmParams& p, int grp, int row, int n_base, uint4 (&zq)[8]) {
+#pragma unroll
+  for (int j = 0; j < 8; ++j) zq[j] = make_uint4(0u, 0u, 0u, 0u);
+  if (row >= p.Mdim || n_base >= p.n_store) return;
+  int64_t zrow = row;
+  if (CONV && p.conv_d) {
+    const int img = row / p.conv.hw;
+    const int rem = row - img * p.conv.hw;
+    const int a = rem / p.conv.Wo, b = rem - a * p.conv.Wo;
+    zrow = ((int64_t)img * p.conv.H + 2 * a + (grp >> 1)) * p.conv.W + 2 * b + (grp & 1);
+  }
+  const __nv_bfloat16* z = p.Z + zrow * p.ldz + n_base;
+  if (n_base + 64 <= p.n_store) {
+    const uint4* z4 = reinterpret_cast<const uint4*>(z);
+#pragma unroll
+    for (int j = 0; j < 8; ++j) zq[j] = __ldg(z4 + j);
+  } else {
+    uint16_t* zs = reinterpret_cast<uint16_t*>(zq);
+    for (int j = 0; j < 64 && n_base + j < p.n_store; ++j) zs[j] = reinterpret_cast<const uint16_t*>(z)[j];
+  }
+}
+
 template <int EPI, bool CONV>
 __device__ __forceinline__ void epilogue_unit(const TcGemmParams& p, int grp, int row, int n_base,
-                                              const uint32_t (&r)[32], const uint32_t (&r2)[32], uint4 (&o)[8]) {
+                                              const uint32_t (&r)[32], const uint32_t (&r2)[32], const uint4 (&zq)[8],
+                                              uint4 (&o)[8]) {
   if (EPI == kTcEpiStoreF32) {
 #pragma unroll
     for (int j = 0; j < 8; ++j) o[j] = make_uint4(r[4 * j], r[4 * j + 1], r[4 * j + 2], r[4 * j + 3]);
@@ -333,33 +361,16 @@ __device__ __forceinline__ void epilogue_unit(const TcGemmParams& p, int grp, in
         for (int j = 0; j < 64; ++j)
           v[j] = fmaxf(v[j] + ((n_base + j < p.Ndim) ? __ldg(p.bias + n_base + j) : 0.f), 0.f);
       }
-    } else {   // kTcEpiMaskBf16: ReLU' from the stored activation of the same row
-      if (row < p.Mdim) {
-        int64_t zrow = row;
-        if (CONV && p.conv_d) {   // class pixel (a, b) of image img = input pixel (2a + ph, 2b + pw)
-          const int img = row / p.conv.hw;
-          const int rem = row - img * p.conv.hw;
-          const int a = rem / p.conv.Wo, b = rem - a * p.conv.Wo;
-          zrow = ((int64_t)img * p.conv.H + 2 * a + (grp >> 1)) * p.conv.W + 2 * b + (grp & 1);
-        }
-        const __nv_bfloat16* z = p.Z + zrow * p.ldz + n_base;
-        if (n_base + 64 <= p.n_store) {
-          const uint4* z4 = reinterpret_cast<const uint4*>(z);
+    } else {   // kTcEpiMaskBf16: ReLU' from the stored activation of the same row (prefetched in zq)
 #pragma unroll
-          for (int j = 0; j < 8; ++j) {
-            const uint4 zz = __ldg(z4 + j);
-            const uint32_t w[4] = {zz.x, zz.y, zz.z, zz.w};
+      for (int j = 0; j < 8; ++j) {
+        const uint32_t w[4] = {zq[j].x, zq[j].y, zq[j].z, zq[j].w};
 #pragma unroll
-            for (int h = 0; h < 4; ++h) {
-              const __nv_bfloat162 pr = *reinterpret_cast<const __nv_bfloat162*>(&w[h]);
-              const int k = 8 * j + 2 * h;
-              v[k] = (__low2float(pr) > 0.f) ? v[k] : 0.f;
-              v[k + 1] = (__high2float(pr) > 0.f) ? v[k + 1] : 0.f;
-            }
-          }
-        } else {
-#pragma unroll
-          for (int j = 0; j < 64; ++j) v[j] = (n_base + j < p.n_store && __bfloat162float(z[j]) > 0.f) ? v[j] : 0.f;
+        for (int h = 0; h < 4; ++h) {
+          const __nv_bfloat162 pr = *reinterpret_cast<const __nv_bfloat162*>(&w[h]);
+          const int k = 8 * j + 2 * h;
+          v[k] = (__low2float(pr) > 0.f) ? v[k] : 0.f;
+          v[k + 1] = (__high2float(pr) > 0.f) ? v[k + 1] : 0.f;
         }
       }
     }
