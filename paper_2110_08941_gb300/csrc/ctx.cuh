@@ -81,6 +81,9 @@ struct hs_ctx {
   hs::DevStatus* h_status = nullptr;   // pinned
   float* d_slabs = nullptr;        // [M, Ps]
   __nv_bfloat16* d_shadow = nullptr;
+  // overlapped updates: layers 2..L write their new bf16 weights here while the same step's
+  // input-gradient products still read d_shadow; copied over d_shadow before the step ends
+  __nv_bfloat16* d_shadow_next = nullptr;
   float* d_gdebug = nullptr;
   void* d_xstage = nullptr;
   int32_t* d_ystage = nullptr;
@@ -143,6 +146,7 @@ struct hs_ctx {
   cudaStream_t upd_stream = nullptr;
   std::vector<cudaEvent_t> upd_ready;
   cudaEvent_t upd_done = nullptr;
+  cudaEvent_t dgrad_done = nullptr;   // the step's last input-gradient product has read d_shadow
 
   // CNN workload: convs[0..2], then the fully connected layer (index 3 in per-layer arrays)
   int64_t in_features = 0;

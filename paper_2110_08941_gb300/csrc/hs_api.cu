@@ -302,7 +302,7 @@ void free_all(hs_ctx* c) {
   }
   for (void* p : c->d_act) f(p);
   f(c->d_logits); f(c->d_delta[0]); f(c->d_delta[1]); f(c->d_ce); f(c->d_lm); f(c->d_status); f(c->d_ticket);
-  f(c->d_slabs); f(c->d_shadow); f(c->d_gdebug); f(c->d_xstage); f(c->d_ystage); f(c->d_mom);
+  f(c->d_slabs); f(c->d_shadow); f(c->d_shadow_next); f(c->d_gdebug); f(c->d_xstage); f(c->d_ystage); f(c->d_mom);
   if (c->h_status) cudaFreeHost(c->h_status);
   for (auto& r : c->pending) {
     cudaEventDestroy(r.a);
@@ -316,6 +316,7 @@ void free_all(hs_ctx* c) {
   }
   for (cudaEvent_t e : c->upd_ready) if (e) cudaEventDestroy(e);
   if (c->upd_done) cudaEventDestroy(c->upd_done);
+  if (c->dgrad_done) cudaEventDestroy(c->dgrad_done);
   if (c->upd_stream) cudaStreamDestroy(c->upd_stream);
 }
 
@@ -402,15 +403,19 @@ hs_status mlp_step_fp32(hs_ctx* c, float* params, const float* x, const int32_t*
 }
 
 // theta <- theta - lr * sum_m w_m G_m over layer l's parameter range [W_l, b_l] (Section 1).
-void update_layer_range(hs_ctx* c, float* params, int l, float lr, cudaStream_t s, int blocks_per_sm) {
+// The update of layer l's parameter range [W_l, b_l]; the new bf16 weights go to `shadow` (the
+// step's shadow, or the second shadow while input-gradient products still read the first).
+void update_layer_range(hs_ctx* c, float* params, int l, float lr, cudaStream_t s, int blocks_per_sm,
+                        __nv_bfloat16* shadow = nullptr) {
   const int64_t start = c->layers[l].w_off;
   const int64_t end = (l + 1 < c->L) ? c->layers[l + 1].w_off : c->P;
+  if (!shadow) shadow = c->d_shadow;
   PhaseScope ph(c, HS_PHASE_UPDATE, s);
   hs::UpdateRecipe r{c->opt_recipe ? c->d_mom + start : nullptr, c->opt_momentum, c->opt_weight_decay,
                      c->mom_valid ? 0 : 1};
   hs::launch_reduce_update(params + start, c->d_slabs + start, c->Ps, c->fused_sync ? 1 : c->M,
                            c->fused_sync ? c->d_w_one : c->d_w, lr, end - start,
-                           c->d_shadow + start, c->debug ? c->d_gdebug + start : nullptr, c->num_sms, s,
+                           shadow + start, c->debug ? c->d_gdebug + start : nullptr, c->num_sms, s,
                            blocks_per_sm, c->opt_recipe ? &r : nullptr);
   ph.launched();
 }
@@ -470,18 +475,28 @@ hs_status mlp_step_bf16(hs_ctx* c, float* params, const float* x, const int32_t*
                                 c->d_slabs, c->Ps, ly.b_off, s);
       ph.launched(2);
     }
+    if (c->overlap_update) {
+      // Layer l's slabs are complete: its update runs beside the remaining (tensor-core bound)
+      // backward products.  Its input-gradient product (next, on the step's stream) still reads
+      // W_l's bf16 weights, so layers 2..L write theirs to the second shadow, copied over the
+      // first once the last input-gradient product is done; layer 1 has none and writes in place.
+      HS_CUDA(c, cudaEventRecord(c->upd_ready[l], s));
+      HS_CUDA(c, cudaStreamWaitEvent(c->upd_stream, c->upd_ready[l], 0));
+      if (l == 0 && L > 1) {
+        // the second shadow's ranges (layers 2..L) over the first, after the last input gradient
+        HS_CUDA(c, cudaStreamWaitEvent(c->upd_stream, c->dgrad_done, 0));
+        const int64_t w1 = c->layers[1].w_off;
+        HS_CUDA(c, cudaMemcpyAsync(c->d_shadow + w1, c->d_shadow_next + w1, sizeof(__nv_bfloat16) * (c->P - w1),
+                                   cudaMemcpyDeviceToDevice, c->upd_stream));
+      }
+      update_layer_range(c, params, l, lr, c->upd_stream, l == 0 ? 4 : 1, l > 0 ? c->d_shadow_next : c->d_shadow);
+    }
     if (l > 0) {
       PhaseScope ph(c, HS_PHASE_DGRAD, s);
       cudaError_t e = hs::launch_tc_gemm(c->tc_dgrad[l], c->num_sms, s);
       if (e != cudaSuccess) return cuda_fail(c, e, "input-gradient GEMM launch");
       ph.launched();
-    }
-    if (c->overlap_update) {
-      // Layer l's slabs are complete and its input-gradient product has read W_l's bf16 shadow: its
-      // update can run beside the remaining (tensor-core bound) backward products.
-      HS_CUDA(c, cudaEventRecord(c->upd_ready[l], s));
-      HS_CUDA(c, cudaStreamWaitEvent(c->upd_stream, c->upd_ready[l], 0));
-      update_layer_range(c, params, l, lr, c->upd_stream, l == 0 ? 4 : 1);
+      if (c->overlap_update && l == 1) HS_CUDA(c, cudaEventRecord(c->dgrad_done, s));
     }
   }
   if (c->overlap_update) {
@@ -755,7 +770,9 @@ hs_status hs_init(const hs_model_desc* model, int32_t M, const double* compute_w
       c->upd_ready.assign(c->L, nullptr);
       for (int l = 0; l < c->L && e == cudaSuccess; ++l) e = cudaEventCreateWithFlags(&c->upd_ready[l], cudaEventDisableTiming);
       if (e == cudaSuccess) e = cudaEventCreateWithFlags(&c->upd_done, cudaEventDisableTiming);
+      if (e == cudaSuccess) e = cudaEventCreateWithFlags(&c->dgrad_done, cudaEventDisableTiming);
       if (e != cudaSuccess) s2 = cuda_fail(c, e, "update stream");
+      if (s2 == HS_OK) s2 = dalloc(c, &c->d_shadow_next, sizeof(__nv_bfloat16) * (size_t)c->Ps);
     }
   }
   if (s2 == HS_OK) s2 = apply_partition(c, sizes, cpn, nullptr, 0);
