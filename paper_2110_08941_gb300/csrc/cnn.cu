@@ -1,11 +1,16 @@
 // The CNN workload (stand-in for the paper's ResNet50 / VGG16 on CIFAR10, Section 5): three 3x3
 // convolutions with padding 1 (strides 1, 2, 2, ReLU), global average pooling, one fully
-// connected layer.  Every convolution runs as a product over explicit patch rows (im2col) on
-// the same GEMM kernels as the MLP: forward (bias + ReLU fused), input gradient (a product into
-// patch space, then a gather back to the input grid with ReLU' fused), and the per-worker
-// weight gradient G_m[W] = dA[seg_m]^T patches[seg_m] (Eq. 1's per-worker gradient), whose K =
-// n_m * Ho * Wo is split into chunks so that the few output tiles still fill the GPU; the chunk
-// partials are added per worker in a fixed order.  Activations are NHWC (channels last).
+// connected layer.  Activations are NHWC (channels last).  Every convolution is a product over
+// its patch rows (tap-major columns) on the same GEMM kernels as the MLP:
+//   forward: bias + ReLU fused; the patch rows are read straight from the input by 4-D TMA boxes
+//     (implicit GEMM) where the input has a multiple of 64 channels, else materialised (im2col);
+//   per-worker weight gradient G_m[W] = dA[seg_m]^T patches[seg_m] (Eq. 1's per-worker
+//     gradient), its reduction over n_m * Ho * Wo rows split into k-block parts inside the kernel
+//     so that the few output tiles still fill the GPU; the parts are added per worker in a fixed
+//     order, and a ones column of the patch rows yields the bias gradient;
+//   input gradient: for stride-2 convolutions four grouped sub-pixel products straight into the
+//     input grid, else a product into patch space and a gather back, with ReLU' fused.
+// The fp32 check path materialises everything and uses the SIMT products.
 #include <algorithm>
 #include <climits>
 #include <cstring>
@@ -310,7 +315,7 @@ __global__ void permute_weights_subpixel_kernel(const float* __restrict__ w, int
   wc[class_off + ((int64_t)t * cout + co) * cin + ci] = __float2bfloat16_rn(w[idx]);
 }
 
-// slabs[m][w_off + co*K + k] = sum over worker m's chunks (in order) of partial[chunk][co][k'], where
+// slabs[m][w_off + co*K + k] = sum over worker m's split-K parts (in order) of partial[part][co][k'], where
 // k' = k for the fully connected layer (cin = 0) and, for a convolution, the tap-major column of
 // theta's (ci, tap) entry k = ci*9 + tap (k' = tap*cin + ci).
 // With cin != 0 the partial's column 9*cin is the ones column of the patch rows: its sums are the
@@ -431,7 +436,7 @@ hs_status cnn_build_wgrad_plan(hs_ctx* c, int layer, const __nv_bfloat16* a, int
     p.st = c->d_status;
   }
   cudaError_t e = cudaMemcpy(wg.d_chunk_begin, begin.data(), sizeof(int32_t) * begin.size(), cudaMemcpyHostToDevice);
-  if (e != cudaSuccess) return cuda_fail(c, e, "split-K chunk table");
+  if (e != cudaSuccess) return cuda_fail(c, e, "split-K part table");
   return HS_OK;
 }
 

@@ -35,13 +35,13 @@ struct ChunkTable {
   int rows_per_sample = 1;
 };
 
-// Split-K weight-gradient plan of one CNN layer (groups = (worker, row chunk)).
+// Split-K weight-gradient plan of one CNN layer (groups = workers, each split into k-block parts).
 struct CnnWgrad {
   std::vector<TcGemmParams> plans;
   int rows_out = 0, K = 0, ldp = 0;
-  float* d_partial = nullptr;        // [groups][rows_out][ldp]
+  float* d_partial = nullptr;        // [workers x parts][rows_out][ldp]
   int64_t partial_capacity = 0;      // floats
-  int32_t* d_chunk_begin = nullptr;  // [M + 1]
+  int32_t* d_chunk_begin = nullptr;  // [M + 1]: worker m's parts are [begin[m], begin[m + 1])
 };
 
 }  // namespace hs
