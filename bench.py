@@ -520,6 +520,16 @@ def run_ours(args, wl, rank, world, local_rank):
     for _ in range(k_e2e):
         hs.hs_step(ctx, params, xh, yh, part, wl.lr, stream=stream, want_loss=True)
     e2e_plain_s = max_over_ranks(time.perf_counter() - t0)
+    # the host-to-device copy alone (context for the end-to-end figure): one step's inputs, timed
+    # on the copy stream after the step that read the slot
+    c0, c1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    c0.record(copy_stream)
+    staged = hs.hs_stage_inputs(ctx, xh, yh, stream=copy_stream)
+    c1.record(copy_stream)
+    torch.cuda.synchronize()
+    h2d_ms = c0.elapsed_time(c1)
+    hs.hs_step(ctx, params, staged, None, part, wl.lr, stream=stream, want_loss=True)   # consume the slot
 
     P = ctx.P
     peaks = _peaks()
@@ -594,7 +604,9 @@ def run_ours(args, wl, rank, world, local_rank):
             "e2e": {"value": world * wl.global_batch * k_e2e / e2e_s, "unit": UNIT,
                     "h2d_bytes_per_step": int(x.nbytes + y.nbytes), "d2h_bytes_per_step": 12,
                     "pipelined": "hs_stage_inputs on a copy stream, two slots",
-                    "unpipelined_value": world * wl.global_batch * k_e2e / e2e_plain_s},
+                    "unpipelined_value": world * wl.global_batch * k_e2e / e2e_plain_s,
+                    "h2d_ms_per_step_alone": h2d_ms,
+                    "h2d_gbs_alone": (x.nbytes + y.nbytes) / (h2d_ms * 1e-3) / 1e9},
             "clocks": clk,
             "straggler_sim": straggler_simulation(),
             "fused_sync_variant": fused,
