@@ -443,10 +443,11 @@ hs_status cnn_build_wgrad_plan(hs_ctx* c, int layer, const __nv_bfloat16* a, int
 namespace {
 
 // A is K-major [a_rows][a_cols], or (conv != nullptr) the implicit patch rows of that convolution.
+// narrow = true: 256 x 128 SM-pair tiles for a product at most 128 wide (K-major B in 64-row boxes).
 hs_status plan_dense(hs_ctx* c, TcGemmParams* p, int epi, const __nv_bfloat16* a, int64_t a_rows, int a_cols,
                      int64_t lda, const __nv_bfloat16* b, int64_t b_rows, int b_cols, int64_t ldb, bool b_mn,
                      void* d, bool d_f32, int Mdim, int Ndim, int n_store, int64_t ldd, const __nv_bfloat16* z,
-                     int64_t ldz, const ConvLayer* conv = nullptr) {
+                     int64_t ldz, const ConvLayer* conv = nullptr, bool narrow = false) {
   const char* why = nullptr;
   std::memset(p, 0, sizeof(*p));
   bool ok;
@@ -459,7 +460,12 @@ hs_status plan_dense(hs_ctx* c, TcGemmParams* p, int epi, const __nv_bfloat16* a
     ok = tc_make_kmajor_map(&p->tmA[0], TcOperand{a, a_rows, a_cols, lda}, kTcBoxA, &why);
   }
   ok = ok && (b_mn ? tc_make_mnmajor_map(&p->tmB[0], TcOperand{b, b_rows, b_cols, ldb}, &why)
-                   : tc_make_kmajor_map(&p->tmB[0], TcOperand{b, b_rows, b_cols, ldb}, kTcBoxB, &why));
+                   : tc_make_kmajor_map(&p->tmB[0], TcOperand{b, b_rows, b_cols, ldb}, narrow ? kTcBoxB / 2 : kTcBoxB,
+                                        &why));
+  if (narrow) {
+    p->pn = 128;
+    p->form = kTcFormPair;
+  }
   ok = ok && tc_make_store_map(&p->tmD[0], d, d_f32, Mdim, n_store, ldd, &why);
   if (!ok) return fail(c, HS_ERR_CUDA, why);
   const int K = b_mn ? (int)b_rows : b_cols;
@@ -516,6 +522,10 @@ hs_status plan_subpixel_dgrad(hs_ctx* c, int k) {
   p.b_mn = 1;
   p.conv_a = 2;
   p.conv_d = 1;
+  if (L.cin <= 128) {   // 256 x 128 SM-pair tiles (the class weights are MN-major: 64-column boxes)
+    p.pn = 128;
+    p.form = kTcFormPair;
+  }
   p.conv = tc_conv_geom(L.cout, L.hout, L.wout, L.stride);
   p.conv.H = L.hin;
   p.conv.W = L.win;
@@ -550,7 +560,7 @@ hs_status cnn_build_static(hs_ctx* c) {
     const __nv_bfloat16* a = L.implicit ? bf(c->d_cact[k - 1]) : bf(c->d_col[k]);
     hs_status st = plan_dense(c, &c->tc_fwd[k], kTcEpiBiasReluBf16, a, L.rows, L.K, L.Kp, wb, L.cout, L.K, ldw,
                               false, c->d_cact[k], false, (int)L.rows, L.cout, L.cout, L.cout, nullptr, 0,
-                              L.implicit ? &L : nullptr);
+                              L.implicit ? &L : nullptr, L.cout <= 128);
     if (st != HS_OK) return st;
   }
   // fully connected layer on the pooled features

@@ -60,6 +60,8 @@ struct TcGemmParams {
   TcConvGeom conv;
   int32_t conv_a, conv_b, conv_d;
   int32_t form;                    // kernel form for this product (TcForm), 0 = the process default
+  int32_t pn;                      // SM-pair tile width: 0 or 256, or 128 (then K-major B maps have
+                                   // 64-row boxes and form must be kTcFormPair)
   int32_t test_stall;              // test hook only: the producer issues no loads (bounded waits expire)
   int32_t ksplit;                  // >= 2: each group's k-blocks split into ksplit contiguous parts, part j
                                    // a tile of its own writing part j of tmD[g], a 3-D map [parts][rows][cols]

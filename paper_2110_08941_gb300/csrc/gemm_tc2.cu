@@ -23,18 +23,25 @@ namespace {
 
 using namespace tcdev;
 
-constexpr int PM = 256, PN = 256;                  // pair tile
-constexpr int HM = PM / 2, HN = PN / 2;            // per-CTA halves
-constexpr int S2 = 6;                              // pipeline stages
+constexpr int PM = 256;                            // pair tile rows
+constexpr int HM = PM / 2;                         // per-CTA half
 constexpr int A_HALF = HM * BK * 2;                // 16 KB
-constexpr int B_HALF = HN * BK * 2;                // 16 KB
-constexpr int STAGE2 = A_HALF + B_HALF;
-constexpr uint32_t PAIR_TX = 2 * STAGE2;           // bytes landing per stage on the leader's barrier
 constexpr int kThreads2 = 192;
-constexpr uint32_t kTmemCols2 = 2 * PN;            // two accumulators of 128 lanes x 256 columns
-constexpr int kSmem2 = S2 * STAGE2 + kTcStagingBytes + 1024 + 256;
 
-static_assert(kSmem2 <= 232448, "shared memory budget");
+// Pair tile of 256 x TN (TN = 256, or 128 for products at most 128 wide): per-CTA B half, stages
+// (more of them when the B half is smaller), two TN-column accumulators in tensor memory.
+template <int TN>
+struct PairCfg {
+  static constexpr int PN = TN;
+  static constexpr int HN = TN / 2;
+  static constexpr int B_HALF = HN * BK * 2;
+  static constexpr int STAGE2 = A_HALF + B_HALF;
+  static constexpr int S2 = TN == 256 ? 6 : 8;
+  static constexpr uint32_t PAIR_TX = 2 * STAGE2;   // bytes landing per stage on the leader's barrier
+  static constexpr uint32_t kTmemCols2 = 2 * TN;
+  static constexpr int kSmem2 = S2 * STAGE2 + kTcStagingBytes + 1024 + 256;
+  static_assert(kSmem2 <= 232448, "shared memory budget");
+};
 
 __device__ __forceinline__ uint32_t cluster_rank() {
   uint32_t r;
@@ -95,8 +102,11 @@ __device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr) {
   asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
 }
 
-template <int EPI, bool A_MN, bool B_MN, bool CONV>
+template <int EPI, bool A_MN, bool B_MN, bool CONV, int TN>
 __global__ void __launch_bounds__(kThreads2, 1) tc_gemm_pair_kernel(const __grid_constant__ TcGemmParams p) {
+  using Cfg = PairCfg<TN>;
+  constexpr int PN = Cfg::PN, HN = Cfg::HN, S2 = Cfg::S2, STAGE2 = Cfg::STAGE2;
+  constexpr uint32_t PAIR_TX = Cfg::PAIR_TX, kTmemCols2 = Cfg::kTmemCols2;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sStage = smem + S2 * STAGE2;
@@ -335,11 +345,12 @@ __global__ void __launch_bounds__(kThreads2, 1) tc_gemm_pair_kernel(const __grid
   }
 }
 
-template <int EPI, bool A_MN, bool B_MN, bool CONV>
+template <int EPI, bool A_MN, bool B_MN, bool CONV, int TN = 256>
 cudaError_t launch_pair_variant(const TcGemmParams& p, int pairs_wanted, int num_sms, cudaStream_t s) {
   static bool configured = false;
   static int max_clusters = 0;
-  auto kern = tc_gemm_pair_kernel<EPI, A_MN, B_MN, CONV>;
+  constexpr int kSmem2 = PairCfg<TN>::kSmem2;
+  auto kern = tc_gemm_pair_kernel<EPI, A_MN, B_MN, CONV, TN>;
   cudaLaunchConfig_t cfg = {};
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -377,12 +388,22 @@ cudaError_t launch_pair_variant(const TcGemmParams& p, int pairs_wanted, int num
 }  // namespace
 
 cudaError_t launch_tc_gemm_pair(const TcGemmParams& p, int num_sms, cudaStream_t s) {
+  const int tn = p.pn == 128 ? 128 : 256;
   const int tiles_m = (p.Mdim + PM - 1) / PM;
-  const int tiles_n = (p.n_store + PN - 1) / PN;
+  const int tiles_n = (p.n_store + tn - 1) / tn;
   const int total = p.groups * (p.ksplit > 1 ? p.ksplit : 1) * tiles_m * tiles_n;
   if (total <= 0) return cudaSuccess;
   const int pairs = total;
   const int grid = num_sms;   // forwarded as the SM count for the residency query
+  if (tn == 128) {
+    // 256 x 128 tiles (K-major B maps with 64-row boxes): the narrow products of the convolutions
+    if (p.epi == kTcEpiBiasReluBf16 && !p.a_mn && !p.b_mn)
+      return (p.conv_a ? launch_pair_variant<kTcEpiBiasReluBf16, false, false, true, 128>
+                       : launch_pair_variant<kTcEpiBiasReluBf16, false, false, false, 128>)(p, pairs, grid, s);
+    if (p.epi == kTcEpiMaskBf16 && !p.a_mn && p.b_mn && (p.conv_a || p.conv_d))
+      return launch_pair_variant<kTcEpiMaskBf16, false, true, true, 128>(p, pairs, grid, s);
+    return cudaErrorInvalidValue;
+  }
   // implicit convolution operands (forward, weight gradient, sub-pixel input gradient)
   if (p.conv_a || p.conv_b || p.conv_d) {
     if (p.epi == kTcEpiBiasReluBf16 && !p.a_mn && !p.b_mn) return launch_pair_variant<kTcEpiBiasReluBf16, false, false, true>(p, pairs, grid, s);
