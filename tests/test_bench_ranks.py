@@ -59,3 +59,24 @@ def test_reference_arm_runs_on_rank_zero_only(capsys):
         steps, warmup = 1, 0
     bench.run_reference(A, synth.WORKLOADS[synth.CFG1], rank=1, world=2)
     assert capsys.readouterr().out == ""
+
+
+def test_reference_arm_prints_the_contract_line(capsys):
+    """Rank 0 of the reference arm times the oracle and prints one JSON line with the contract's
+    keys (impl, metric, value, unit, e2e with zero copies, cpu_baseline describing the run)."""
+    sys.path.insert(0, ROOT)
+    import json
+    import bench
+    import synth
+
+    class A:
+        steps, warmup = 2, 1
+    bench.run_reference(A, synth.WORKLOADS[synth.CFG1], rank=0, world=1)
+    lines = [l for l in capsys.readouterr().out.splitlines() if l.startswith("{")]
+    assert len(lines) == 1
+    d = json.loads(lines[0])
+    assert d["impl"] == "reference" and d["metric"] == bench.METRIC and d["unit"] == bench.UNIT
+    assert d["value"] > 0 and d["steps"] == 2 and d["warmup"] == 1 and d["higher_is_better"] is True
+    assert d["e2e"] == {"value": d["value"], "unit": d["unit"], "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}
+    assert d["cpu_baseline"]["kind"] == "oracle" and d["cpu_baseline"]["value"] == d["value"]
+    assert d["config"]["workload"] == synth.CFG1
