@@ -96,6 +96,24 @@ def test_drift_workload_repartition():
     _check(lib, orc, theta0.astype(np.float64), hs.HS_BF16, 2)
 
 
+@pytest.mark.parametrize("precision", [hs.HS_BF16, hs.HS_FP32_CHECK])
+def test_cnn_repartition(precision):
+    """The CNN with a repartition between steps (Algorithm 1 on new throughputs): the split-K
+    weight-gradient plans, chunk tables and index map are rebuilt for the new segments."""
+    dims, N, M = (3, 16, 16, 64, 128, 64, 7), 24, 3
+    rng = np.random.default_rng(11)
+    x = rng.standard_normal((N,) + tuple(dims[:3]), dtype=np.float32)
+    y = rng.integers(0, dims[-1], N, dtype=np.int32)
+    theta0 = synth.he_normal_params(synth.CNN, dims, 3)
+    rep = {2: [1.0, 4.0, 2.0]}
+    lib = run_library(synth.CNN, dims, M, N, [3.0, 1.0, 1.0], x, y, theta0, 0.05, 4, precision,
+                      hs.HS_SYNC_CP_WEIGHTED, repartition=rep)
+    orc = run_oracle(synth.CNN, dims, M, N, [3.0, 1.0, 1.0], x, y, theta0, 0.05, 4, hs.HS_SYNC_CP_WEIGHTED,
+                     repartition=rep, decide=decide_for(precision))
+    assert lib["counts"] == [[14, 5, 5], [3, 14, 7]]
+    _check(lib, orc, theta0.astype(np.float64), precision, 4)
+
+
 EDGE = [
     # dims, N, M, weights: one sample per worker; ragged tails in every GEMM dimension; M = 1
     ((24, 16, 3), 5, 5, None),
