@@ -59,8 +59,9 @@ def _cnn_dims(cin=3, h=32, w=32, c=(64, 128, 256), classes=10):
     return (cin, h, w, c[0], c[1], c[2], classes)
 
 
-# The five workloads.  Steps/lr that the task text leaves open are the proposed
-# readings recorded in the design doc (cfg 3 lr, cfg 4/5 steps and lr).
+# The five workloads.  The paper leaves some steps and learning rates open; these are proposed
+# readings: the drifting 2048-wide MLP at lr 0.01, the CNN and the 8192-wide MLP at 10 steps and
+# lr 0.01.
 WORKLOADS = {
     "mlp_3072_256_10_b128_m2": Workload(
         "mlp_3072_256_10_b128_m2", MLP, (3072, 256, 10), 10, 128, 2, (1.0, 3.0), 10, 0.01),
