@@ -10,11 +10,11 @@ HBM; the working set (activations and 7 GB of gradient slabs) is far larger than
 explicit L2 flush is needed between steps.
 
 Prints ONE JSON line (rank 0).  With --gpus N > 1 (launched by torch.distributed.run) every rank
-runs an independent replica of the workload (the one-GPU method has no cross-GPU exchange in
-this build): weak scaling, value = all ranks' samples / max-over-ranks time.
+runs an independent replica of the workload (the M workers live on one GPU; there is no cross-GPU
+exchange): weak scaling, value = all ranks' samples / max-over-ranks time.
 
 --impl reference times the fp64 CPU oracle on the host cores (bounded samples of the same
-workload), the reference arm of this build.
+workload) as the reference arm.
 """
 from __future__ import annotations
 

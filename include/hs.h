@@ -45,7 +45,7 @@ typedef enum {
   HS_ERR_INVALID_ARG = 1,   /* bad pointer, size, enum or numeric value; nothing was enqueued */
   HS_ERR_CUDA = 2,          /* a CUDA runtime call failed (message has the CUDA error string) */
   HS_ERR_OOM = 3,           /* device workspace allocation failed */
-  HS_ERR_UNSUPPORTED = 4,   /* valid request outside what this build implements */
+  HS_ERR_UNSUPPORTED = 4,   /* valid request outside what the library implements */
   HS_ERR_DEVICE_CHECK = 5   /* a kernel's own check failed (bounded wait timed out); results invalid */
 } hs_status;
 
