@@ -166,6 +166,12 @@ struct hs_ctx {
   hs::CnnWgrad cnn_wgrad[4];
 
   // tensor-core launch parameters (bf16 precision)
+  // per-worker weight gradients averaged in tensor memory and applied in the same kernel
+  // (launch_tc_wgrad_avg): per layer, valid where avg_ok[l]; tmT points at avg_theta's weights
+  bool tile_avg = false;
+  std::vector<hs::TcGemmParams> tc_wgrad_avg;
+  std::vector<char> avg_ok;
+  const float* avg_theta = nullptr;
   std::vector<hs::TcGemmParams> tc_fwd;                // per layer
   std::vector<hs::TcGemmParams> tc_dgrad;              // per layer (index 0 unused)
   std::vector<std::vector<hs::TcGemmParams>> tc_wgrad; // per layer, per chunk of <= 32 workers

@@ -301,7 +301,8 @@ bool tc_init_driver(const char** why) {
 
 static bool encode_2d(CUtensorMap* tm, const void* base, uint64_t inner, uint64_t outer, uint64_t row_bytes,
                       uint32_t box_inner, uint32_t box_outer, const char** why,
-                      CUtensorMapDataType dtype = CU_TENSOR_MAP_DATA_TYPE_BFLOAT16) {
+                      CUtensorMapDataType dtype = CU_TENSOR_MAP_DATA_TYPE_BFLOAT16,
+                      CUtensorMapSwizzle swizzle = CU_TENSOR_MAP_SWIZZLE_128B) {
   if (!g_encode && !tc_init_driver(why)) return false;
   if ((reinterpret_cast<uintptr_t>(base) & 15u) != 0 || (row_bytes & 15u) != 0) {
     *why = "TMA operand base or row stride is not 16-byte aligned";
@@ -312,7 +313,7 @@ static bool encode_2d(CUtensorMap* tm, const void* base, uint64_t inner, uint64_
   cuuint32_t box[2] = {box_inner, box_outer};
   cuuint32_t estr[2] = {1, 1};
   CUresult r = g_encode(tm, dtype, 2, const_cast<void*>(base), dims, strides, box, estr,
-                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle,
                         CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (r != CUDA_SUCCESS) {
     *why = "cuTensorMapEncodeTiled rejected the operand";
@@ -439,6 +440,12 @@ bool tc_make_store_map(CUtensorMap* tm, void* base, bool fp32, int64_t rows, int
   const uint64_t es = fp32 ? 4 : 2;
   return encode_2d(tm, base, (uint64_t)cols, (uint64_t)rows, (uint64_t)ld * es, (uint32_t)(128 / es), 32, why,
                    fp32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16);
+}
+
+bool tc_make_store_map_bf16_32(CUtensorMap* tm, void* base, int64_t rows, int64_t cols, int64_t ld,
+                               const char** why) {
+  return encode_2d(tm, base, (uint64_t)cols, (uint64_t)rows, (uint64_t)ld * 2, 32, 32, why,
+                   CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, CU_TENSOR_MAP_SWIZZLE_NONE);
 }
 
 namespace {

@@ -15,6 +15,8 @@ enum TcEpi : int32_t {
   kTcEpiBiasF32 = 1,        // D fp32 = acc + bias[n] (n < Ndim), 0 beyond   (logits)
   kTcEpiMaskBf16 = 2,       // D bf16 = bf16(acc * (Z(m, n) > 0))            (input gradient + ReLU')
   kTcEpiStoreF32 = 3,       // D fp32 = acc                                  (per-worker weight gradient)
+  kTcEpiAvgUpdate = 4,      // theta -= lr * sum_g wavg[g] * acc_g, bf16 copy of the new theta
+                            //   (per-worker weight gradients averaged in tensor memory; launch_tc_wgrad_avg)
 };
 
 // Implicit patch rows of a 3x3, padding-1 convolution over an NHWC bf16 input with C % 64 == 0:
@@ -63,6 +65,11 @@ struct TcGemmParams {
   int32_t pn;                      // SM-pair tile width: 0 or 256, or 128 (then K-major B maps have
                                    // 64-row boxes and form must be kTcFormPair)
   int32_t test_stall;              // test hook only: the producer issues no loads (bounded waits expire)
+  // kTcEpiAvgUpdate: the update's operands
+  CUtensorMap tmT;                 // fp32 theta of the layer's weights [Mdim][n_store] (tc_make_store_map)
+  CUtensorMap tmS;                 // bf16 copy of those weights, written beside theta (tc_make_store_map_bf16_32)
+  const float* wavg;               // [groups] averaging weight of group (worker) g, on the device
+  float lr;
   int32_t ksplit;                  // >= 2: each group's k-blocks split into ksplit contiguous parts, part j
                                    // a tile of its own writing part j of tmD[g], a 3-D map [parts][rows][cols]
                                    // (needs num_kb[g] >= ksplit); 0 or 1: no split
@@ -108,6 +115,10 @@ bool tc_make_grid_map(CUtensorMap* tm, const void* base, int C, int cols, int ro
 // 128-byte boxes; rows >= `rows` and columns >= `cols` of a box are not written.
 bool tc_make_store_map(CUtensorMap* tm, void* base, bool fp32, int64_t rows, int64_t cols, int64_t ld,
                        const char** why);
+// bf16 output matrix for TMA stores of 32-row x 32-column (64-byte) boxes, unswizzled (row r of a
+// box at byte 64 * r of the staging buffer).
+bool tc_make_store_map_bf16_32(CUtensorMap* tm, void* base, int64_t rows, int64_t cols, int64_t ld,
+                               const char** why);
 // The same over `parts` such matrices `part_stride` elements apart (split-K partials, fp32).
 bool tc_make_store_map_parts(CUtensorMap* tm, float* base, int64_t rows, int64_t cols, int64_t ld, int64_t parts,
                              int64_t part_stride, const char** why);
@@ -130,5 +141,17 @@ int tc_get_form();
 cudaError_t launch_tc_gemm(const TcGemmParams& p, int num_sms, cudaStream_t s);
 cudaError_t launch_tc_gemm_form(const TcGemmParams& p, int num_sms, cudaStream_t s, int form);
 cudaError_t launch_tc_gemm_pair(const TcGemmParams& p, int num_sms, cudaStream_t s);
+
+// The per-worker weight gradients of one layer, averaged and applied (Eq. 1's g^m, the weighted
+// average of Section 1 and Section 4.2, theta <- theta - lr * g).  Operands as for a kTcEpiStoreF32
+// grouped launch with MN-major A and B (A_g = delta rows of worker g, B_g = input rows of worker g,
+// groups <= kTcMaxGroups); no product is written out.  Each SM pair owns 256 x 256 tiles of the
+// layer's weights and, per tile, runs the groups in order: group g's product accumulates in one of
+// two tensor-memory buffers (fresh at its first k-block, exactly the per-worker gradient of the
+// grouped launch) while the epilogue folds the previous group into a running sum in registers,
+// sum = fma(wavg[g], acc_g, sum) from sum = 0 (the fixed worker order of reduce_update_kernel).
+// After the last group: theta = fma(-lr, sum, theta) through tmT, the bf16 copy through tmS.
+// The result equals the grouped launch followed by reduce_update_kernel bit for bit.
+cudaError_t launch_tc_wgrad_avg(const TcGemmParams& p, int num_sms, cudaStream_t s);
 
 }  // namespace hs

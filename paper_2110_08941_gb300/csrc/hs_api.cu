@@ -189,6 +189,61 @@ hs_status build_tc_wgrad(hs_ctx* c) {
   return HS_OK;
 }
 
+// The tile-averaged weight gradients: per layer one launch over all workers (groups), the update
+// fused in (launch_tc_wgrad_avg).  Layers 2..L write their bf16 weights to the second shadow (their
+// input-gradient products still read the first); layer 1 writes the first.  theta's maps are bound
+// per step (bind_avg_theta).  A layer whose operands the kernel cannot take keeps the slab path.
+hs_status build_tc_wgrad_avg(hs_ctx* c) {
+  const char* why = nullptr;
+  c->tc_wgrad_avg.assign(c->L, hs::TcGemmParams{});
+  c->avg_ok.assign(c->L, 0);
+  c->avg_theta = nullptr;
+  if (!c->tile_avg || c->M > hs::kTcMaxGroups) return HS_OK;
+  for (int l = 0; l < c->L; ++l) {
+    const Layer& ly = c->layers[l];
+    const int ldd_delta = c->delta_ld(l);
+    const int out_cols = (l == c->L - 1) ? c->C : ly.out;
+    hs::TcGemmParams& w = c->tc_wgrad_avg[l];
+    std::memset(&w, 0, sizeof(w));
+    bool ok = true;
+    for (int m = 0; m < c->M && ok; ++m) {
+      const int64_t off = c->offsets[m], n = c->counts[m];
+      hs::TcOperand a{reinterpret_cast<const __nv_bfloat16*>(c->delta_buf(l)) + off * ldd_delta, n, out_cols,
+                      ldd_delta};
+      hs::TcOperand b{reinterpret_cast<const __nv_bfloat16*>(c->d_act[l]) + off * ly.in, n, ly.in, ly.in};
+      ok = n >= 1 && hs::tc_make_mnmajor_map(&w.tmA[m], a, &why) && hs::tc_make_mnmajor_map(&w.tmB[m], b, &why);
+      w.num_kb[m] = (int32_t)((n + hs::kTcBK - 1) / hs::kTcBK);
+    }
+    __nv_bfloat16* shadow = (l > 0 ? c->d_shadow_next : c->d_shadow) + ly.w_off;
+    ok = ok && shadow && hs::tc_make_store_map_bf16_32(&w.tmS, shadow, out_cols, ly.in, ly.in, &why);
+    w.groups = c->M;
+    w.Mdim = out_cols;
+    w.Ndim = ly.in;
+    w.n_store = ly.in;
+    w.epi = hs::kTcEpiAvgUpdate;
+    w.a_mn = 1;
+    w.b_mn = 1;
+    w.wavg = c->d_w;
+    w.st = c->d_status;
+    c->avg_ok[l] = ok ? 1 : 0;
+  }
+  return HS_OK;
+}
+
+// Point the tile-averaged launches' theta maps at `params` (a layer whose weights TMA cannot
+// address, e.g. not 16-byte aligned, falls back to the slab path).
+void bind_avg_theta(hs_ctx* c, float* params) {
+  if (c->avg_theta == params) return;
+  const char* why = nullptr;
+  for (int l = 0; l < c->L; ++l) {
+    if (!c->avg_ok[l]) continue;
+    const Layer& ly = c->layers[l];
+    hs::TcGemmParams& w = c->tc_wgrad_avg[l];
+    if (!hs::tc_make_store_map(&w.tmT, params + ly.w_off, true, w.Mdim, ly.in, ly.in, &why)) c->avg_ok[l] = 0;
+  }
+  c->avg_theta = params;
+}
+
 void compute_weights(hs_ctx* c) {
   c->weights.assign(c->M, 0.0);
   for (int m = 0; m < c->M; ++m) {
@@ -241,6 +296,7 @@ hs_status apply_partition(hs_ctx* c, const std::vector<int32_t>& sizes, const st
   HS_CUDA(c, cudaStreamSynchronize(s));
   if (changed && c->arch == HS_MLP && c->precision == HS_BF16) {
     hs_status st = build_tc_wgrad(c);
+    if (st == HS_OK) st = build_tc_wgrad_avg(c);
     if (st != HS_OK) return st;
   }
   if (changed && c->arch == HS_CNN) {
@@ -420,6 +476,16 @@ void update_layer_range(hs_ctx* c, float* params, int l, float lr, cudaStream_t 
   ph.launched();
 }
 
+// theta <- theta - lr * sum_m w_m G_m over [start, end) of the slabs (the bias range of a layer whose
+// weights the tile-averaged launch updated), bf16 copy into `shadow`.
+void update_range(hs_ctx* c, float* params, int64_t start, int64_t end, float lr, cudaStream_t s,
+                  __nv_bfloat16* shadow) {
+  PhaseScope ph(c, HS_PHASE_UPDATE, s);
+  hs::launch_reduce_update(params + start, c->d_slabs + start, c->Ps, c->M, c->d_w, lr, end - start, shadow + start,
+                           nullptr, c->num_sms, s, 1, nullptr);
+  ph.launched();
+}
+
 hs_status mlp_step_bf16(hs_ctx* c, float* params, const float* x, const int32_t* y, float lr, cudaStream_t s) {
   const int L = c->L;
   {
@@ -445,11 +511,25 @@ hs_status mlp_step_bf16(hs_ctx* c, float* params, const float* x, const int32_t*
     hs::launch_loss_reduce(c->d_ce, c->d_offsets, c->M, c->d_w, c->d_lm, c->d_status, c->d_ticket, s);
     ph.launched(2);
   }
+  // Per-worker weight gradients averaged tile by tile in tensor memory, the update fused in: the
+  // default where the layer's operands allow it; debug read-back, the slab-free formulation and
+  // the momentum recipe take the slab path.
+  const bool avg = c->tile_avg && !c->fused_sync && !c->debug && !c->opt_recipe;
+  if (avg) bind_avg_theta(c, params);
+  bool side = false;   // work queued on the update stream this step
   for (int l = L - 1; l >= 0; --l) {
     const Layer& ly = c->layers[l];
+    const bool tile = avg && c->avg_ok[l];
+    __nv_bfloat16* shadow_l = (l > 0 && c->d_shadow_next) ? c->d_shadow_next : c->d_shadow;
     {
       PhaseScope ph(c, HS_PHASE_WGRAD, s);
-      if (c->fused_sync) {
+      if (tile) {
+        hs::TcGemmParams& w = c->tc_wgrad_avg[l];
+        w.lr = lr;
+        cudaError_t e = hs::launch_tc_wgrad_avg(w, c->num_sms, s);
+        if (e != cudaSuccess) return cuda_fail(c, e, "weight-gradient GEMM launch");
+        ph.launched();
+      } else if (c->fused_sync) {
         cudaError_t e = hs::launch_tc_gemm(c->tc_wgrad_fused[l], c->num_sms, s);
         if (e != cudaSuccess) return cuda_fail(c, e, "weight-gradient GEMM launch");
         ph.launched();
@@ -475,35 +555,42 @@ hs_status mlp_step_bf16(hs_ctx* c, float* params, const float* x, const int32_t*
                                 c->d_slabs, c->Ps, ly.b_off, s);
       ph.launched(2);
     }
-    if (c->overlap_update) {
+    if (tile) {
+      // the bias range's update (its weights were updated inside the weight-gradient launch)
+      const int64_t end = (l + 1 < L) ? c->layers[l + 1].w_off : c->P;
+      update_range(c, params, ly.b_off, end, lr, s, shadow_l);
+    } else if (c->overlap_update) {
       // Layer l's slabs are complete: its update runs beside the remaining (tensor-core bound)
       // backward products.  Its input-gradient product (next, on the step's stream) still reads
       // W_l's bf16 weights, so layers 2..L write theirs to the second shadow, copied over the
       // first once the last input-gradient product is done; layer 1 has none and writes in place.
       HS_CUDA(c, cudaEventRecord(c->upd_ready[l], s));
       HS_CUDA(c, cudaStreamWaitEvent(c->upd_stream, c->upd_ready[l], 0));
-      if (l == 0 && L > 1) {
-        // the second shadow's ranges (layers 2..L) over the first, after the last input gradient
-        HS_CUDA(c, cudaStreamWaitEvent(c->upd_stream, c->dgrad_done, 0));
-        const int64_t w1 = c->layers[1].w_off;
-        HS_CUDA(c, cudaMemcpyAsync(c->d_shadow + w1, c->d_shadow_next + w1, sizeof(__nv_bfloat16) * (c->P - w1),
-                                   cudaMemcpyDeviceToDevice, c->upd_stream));
-      }
-      update_layer_range(c, params, l, lr, c->upd_stream, l == 0 ? 4 : 1, l > 0 ? c->d_shadow_next : c->d_shadow);
+      update_layer_range(c, params, l, lr, c->upd_stream, l == 0 ? 4 : 1, shadow_l);
+      side = true;
+    } else {
+      update_layer_range(c, params, l, lr, s, 4, shadow_l);
     }
     if (l > 0) {
       PhaseScope ph(c, HS_PHASE_DGRAD, s);
       cudaError_t e = hs::launch_tc_gemm(c->tc_dgrad[l], c->num_sms, s);
       if (e != cudaSuccess) return cuda_fail(c, e, "input-gradient GEMM launch");
       ph.launched();
-      if (c->overlap_update && l == 1) HS_CUDA(c, cudaEventRecord(c->dgrad_done, s));
+    }
+    if (l == 1 && c->d_shadow_next) {
+      // The last input-gradient product has read the first shadow: the second shadow's ranges
+      // (layers 2..L) go over it, on the copy engine beside layer 1's weight gradient.
+      const int64_t w1 = c->layers[1].w_off;
+      HS_CUDA(c, cudaEventRecord(c->dgrad_done, s));
+      HS_CUDA(c, cudaStreamWaitEvent(c->upd_stream, c->dgrad_done, 0));
+      HS_CUDA(c, cudaMemcpyAsync(c->d_shadow + w1, c->d_shadow_next + w1, sizeof(__nv_bfloat16) * (c->P - w1),
+                                 cudaMemcpyDeviceToDevice, c->upd_stream));
+      side = true;
     }
   }
-  if (c->overlap_update) {
+  if (side) {
     HS_CUDA(c, cudaEventRecord(c->upd_done, c->upd_stream));
     HS_CUDA(c, cudaStreamWaitEvent(s, c->upd_done, 0));
-  } else {
-    for (int l = L - 1; l >= 0; --l) update_layer_range(c, params, l, lr, s, 4);
   }
   return HS_OK;
 }
@@ -763,17 +850,19 @@ hs_status hs_init(const hs_model_desc* model, int32_t M, const double* compute_w
   if (s2 == HS_OK && bf16) s2 = c->arch == HS_MLP ? build_tc_static(c) : cnn_build_static(c);
   if (s2 == HS_OK && bf16 && c->arch == HS_MLP) s2 = build_tc_wgrad_fused(c);
   if (s2 == HS_OK && bf16 && c->arch == HS_MLP) {
+    // HS_OVERLAP_UPDATE=0: slab-path updates on the step's stream instead of the update stream;
+    // HS_TILE_AVERAGE=0: every layer on the slab path (per-worker gradients stored, then reduced)
     const char* ov = getenv("HS_OVERLAP_UPDATE");
     c->overlap_update = !(ov && !strcmp(ov, "0"));
-    if (c->overlap_update) {
-      e = cudaStreamCreateWithFlags(&c->upd_stream, cudaStreamNonBlocking);
-      c->upd_ready.assign(c->L, nullptr);
-      for (int l = 0; l < c->L && e == cudaSuccess; ++l) e = cudaEventCreateWithFlags(&c->upd_ready[l], cudaEventDisableTiming);
-      if (e == cudaSuccess) e = cudaEventCreateWithFlags(&c->upd_done, cudaEventDisableTiming);
-      if (e == cudaSuccess) e = cudaEventCreateWithFlags(&c->dgrad_done, cudaEventDisableTiming);
-      if (e != cudaSuccess) s2 = cuda_fail(c, e, "update stream");
-      if (s2 == HS_OK) s2 = dalloc(c, &c->d_shadow_next, sizeof(__nv_bfloat16) * (size_t)c->Ps);
-    }
+    const char* ta = getenv("HS_TILE_AVERAGE");
+    c->tile_avg = !(ta && !strcmp(ta, "0")) && c->M <= hs::kTcMaxGroups;
+    e = cudaStreamCreateWithFlags(&c->upd_stream, cudaStreamNonBlocking);
+    c->upd_ready.assign(c->L, nullptr);
+    for (int l = 0; l < c->L && e == cudaSuccess; ++l) e = cudaEventCreateWithFlags(&c->upd_ready[l], cudaEventDisableTiming);
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&c->upd_done, cudaEventDisableTiming);
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&c->dgrad_done, cudaEventDisableTiming);
+    if (e != cudaSuccess) s2 = cuda_fail(c, e, "update stream");
+    if (s2 == HS_OK) s2 = dalloc(c, &c->d_shadow_next, sizeof(__nv_bfloat16) * (size_t)c->Ps);
   }
   if (s2 == HS_OK) s2 = apply_partition(c, sizes, cpn, nullptr, 0);
   if (s2 == HS_OK) {

@@ -27,11 +27,14 @@ def _lr_at(lr, t):
 
 
 def run_library(arch, dims, M, N, weights, x, y, theta0, lr, steps, precision, sync, repartition=None,
-                keep_slabs=False, recipe=None, fused=False):
-    """Returns dict(theta, losses, g_first, slabs_first, counts, index_map)."""
+                keep_slabs=False, recipe=None, fused=False, debug=True):
+    """Returns dict(theta, losses, g_first, slabs_first, counts, index_map).  debug=False runs the
+    step as users do (no gradient read-back: the MLP weight gradients take the tile-averaged launch)
+    and returns no g_first / slabs_first."""
     ctx = hs.hs_init(arch, dims, M, N, compute_weights=weights, precision=precision, sync=sync)
     try:
-        hs.hs_set_debug(ctx, True)
+        if debug:
+            hs.hs_set_debug(ctx, True)
         if recipe is not None:
             hs.hs_set_optimizer(ctx, *recipe)
         if fused:
@@ -48,7 +51,7 @@ def run_library(arch, dims, M, N, weights, x, y, theta0, lr, steps, precision, s
                 out["counts"].append(list(part.counts))
                 out["index_maps"].append(im.cpu().numpy().copy())
             out["losses"].append(hs.hs_step(ctx, params, xd, yd, part, _lr_at(lr, t)))
-            if t == 0:
+            if t == 0 and debug:
                 g = torch.empty(ctx.P, device="cuda")
                 slabs = torch.empty(M, ctx.P, device="cuda") if keep_slabs else None
                 hs.hs_debug_grads(ctx, g, slabs)

@@ -1,0 +1,115 @@
+"""The tile-averaged weight-gradient launch: each worker's weight gradient g^m (Eq. 1) formed tile
+by tile in tensor memory, averaged in worker order (Section 1; Section 4.2's weights) and applied to
+theta in the same kernel.  It must leave theta and the bf16 weight copy exactly where the slab path
+(per-worker gradients stored, then reduce_update_kernel) leaves them, and within the oracle's
+tolerance, over several steps, repartitions, worker counts, sync rules and ragged shapes."""
+import os
+
+import numpy as np
+import pytest
+import torch
+
+import synth
+import paper_2110_08941_gb300 as hs
+from tests.gpu_helpers import decide_for, rel, run_library, run_oracle
+
+pytestmark = pytest.mark.gpu
+
+
+def _init(dims, M, N, weights, sync, tile):
+    old = os.environ.get("HS_TILE_AVERAGE")
+    os.environ["HS_TILE_AVERAGE"] = "1" if tile else "0"
+    try:
+        return hs.hs_init(hs.HS_MLP, dims, M, N, compute_weights=weights, sync=sync)
+    finally:
+        if old is None:
+            os.environ.pop("HS_TILE_AVERAGE")
+        else:
+            os.environ["HS_TILE_AVERAGE"] = old
+
+
+def _run(dims, M, N, weights, sync, tile, steps, lr, x, y, theta0, repartition=None):
+    ctx = _init(dims, M, N, weights, sync, tile)
+    try:
+        p = torch.tensor(theta0, device="cuda")
+        xd, yd = torch.from_numpy(x).cuda(), torch.from_numpy(y).cuda()
+        losses = []
+        for t in range(steps):
+            if repartition is not None and t in repartition:
+                hs.hs_partition(ctx, repartition[t])
+            losses.append(hs.hs_step(ctx, p, xd, yd, None, lr))
+        # one more forward pass reads the bf16 weight copy the last update wrote
+        losses.append(hs.hs_step(ctx, p, xd, yd, None, 0.0))
+        torch.cuda.synchronize()
+        return p.cpu(), losses
+    finally:
+        ctx.close()
+
+
+def _data(dims, N, seed):
+    wl = synth.Workload("t", synth.MLP, tuple(dims), dims[-1], N, 1, (1.0,), 1, 0.0, seed=seed)
+    x, y = synth.make_batch(wl)
+    return np.ascontiguousarray(x), np.ascontiguousarray(y), synth.he_normal_params(synth.MLP, dims, seed)
+
+
+CASES = [
+    # dims, N, M, compute weights, sync
+    ((3072, 1024, 1024, 10), 1024, 4, (1.0, 1.0, 2.0, 4.0), hs.HS_SYNC_CP_WEIGHTED),
+    ((3072, 1024, 1024, 10), 1024, 4, (1.0, 1.0, 2.0, 4.0), hs.HS_SYNC_MEAN),
+    ((3072, 1024, 1024, 10), 1024, 4, (1.0, 1.0, 2.0, 4.0), hs.HS_SYNC_CP_LITERAL),
+    # ragged: widths not multiples of the 256-wide tile, worker rows not multiples of 64
+    ((264, 200, 136, 10), 300, 5, (1.0, 2.0, 3.0, 1.5, 0.7), hs.HS_SYNC_CP_WEIGHTED),
+    # 1000 classes (partial last row tile), 16 lognormal workers
+    ((512, 768, 1000), 2048, 16, tuple(synth.lognormal_weights(16, 3)), hs.HS_SYNC_CP_WEIGHTED),
+    # the most groups one launch takes
+    ((256, 512, 10), 2048, 32, tuple(np.linspace(0.5, 2.0, 32)), hs.HS_SYNC_MEAN),
+    # one worker; a worker left with a single sample
+    ((256, 512, 10), 512, 1, (1.0,), hs.HS_SYNC_MEAN),
+    ((256, 512, 10), 96, 4, (1e-6, 1.0, 1.0, 1.0), hs.HS_SYNC_CP_WEIGHTED),
+    # more workers than one launch takes: the slab path on both sides
+    ((256, 512, 10), 2048, 33, tuple(np.linspace(0.5, 2.0, 33)), hs.HS_SYNC_CP_WEIGHTED),
+]
+
+
+@pytest.mark.parametrize("dims,N,M,weights,sync", CASES)
+def test_tile_average_equals_slab_path(dims, N, M, weights, sync):
+    x, y, theta0 = _data(dims, N, seed=11)
+    rep = {2: tuple(reversed(weights))} if M > 1 else None
+    a, la = _run(dims, M, N, weights, sync, True, 4, 0.05, x, y, theta0, rep)
+    b, lb = _run(dims, M, N, weights, sync, False, 4, 0.05, x, y, theta0, rep)
+    assert torch.equal(a, b)
+    assert la == lb
+    assert not torch.equal(a, torch.from_numpy(theta0))
+
+
+@pytest.mark.parametrize("name", [synth.CFG2, synth.CFG3])
+def test_tile_average_matches_oracle(name):
+    wl = synth.WORKLOADS[name]
+    x, y = synth.make_batch(wl)
+    theta0 = synth.make_params(wl)
+    weights = synth.initial_weights(wl)
+    steps = 3
+    lib = run_library(wl.arch, wl.dims, wl.workers, wl.global_batch, weights, x, y, theta0, wl.lr, steps,
+                      hs.HS_BF16, hs.HS_SYNC_CP_WEIGHTED, debug=False)
+    orc = run_oracle(wl.arch, wl.dims, wl.workers, wl.global_batch, weights, x, y, theta0, wl.lr, steps,
+                     hs.HS_SYNC_CP_WEIGHTED, decide=decide_for(hs.HS_BF16))
+    d_lib = lib["theta"] - theta0
+    d_orc = orc["theta"] - theta0
+    assert rel(lib["theta"], orc["theta"]) <= 2e-2
+    assert rel(d_lib, d_orc) <= 5e-2
+    assert np.allclose(lib["losses"], orc["losses"], rtol=2e-2)
+
+
+def test_tile_average_full_size_equals_slab_path():
+    """The 4096-8192-8192-1000 workload (N 16384, 16 workers): two steps on each path, theta equal
+    bit for bit."""
+    wl = synth.WORKLOADS[synth.CFG5]
+    x, y = synth.make_batch(wl)
+    theta0 = synth.make_params(wl)
+    weights = tuple(synth.initial_weights(wl))
+    a, la = _run(wl.dims, wl.workers, wl.global_batch, weights, hs.HS_SYNC_CP_WEIGHTED, True, 2, wl.lr,
+                 x, y, theta0)
+    b, lb = _run(wl.dims, wl.workers, wl.global_batch, weights, hs.HS_SYNC_CP_WEIGHTED, False, 2, wl.lr,
+                 x, y, theta0)
+    assert torch.equal(a, b)
+    assert la == lb
