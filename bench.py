@@ -4,10 +4,12 @@
 
 A step is one synchronous SGD step of the whole hot path through libhs: per-worker forward and
 backward over M = 16 compute-proportional segments of a 16384-sample batch (MLP
-4096 -> 8192 -> 8192 -> 1000, bf16 tensor cores), softmax cross-entropy, per-worker gradient
-slabs, and the fused reduce + update.  Inputs are seeded synthetic data already resident in
-HBM; the working set (activations and 7 GB of gradient slabs) is far larger than L2, so no
-explicit L2 flush is needed between steps.
+4096 -> 8192 -> 8192 -> 1000, bf16 tensor cores), softmax cross-entropy, each worker's weight
+gradient formed tile by tile in tensor memory and averaged there with the update applied in the
+same kernel (biases through per-worker slabs and the reduce + update).  Inputs are seeded
+synthetic data already resident in HBM; the working set (over 1 GB of bf16 activations and input
+gradients, 0.44 GB of fp32 parameters per step) is far larger than L2, so no explicit L2 flush
+is needed between steps.
 
 Prints ONE JSON line (rank 0).  With --gpus N > 1 (launched by torch.distributed.run) every rank
 runs an independent replica of the workload (the M workers live on one GPU; there is no cross-GPU
@@ -126,7 +128,7 @@ def gemm_flops(wl):
                 dgrad=2.0 * n * (per[1] + per[2] + fc))
 
 
-def recorded_traffic(kernel_tag="tc_gemm_pair_wgrad"):
+def recorded_traffic(kernel_tag="tc_wgrad_avg_pair"):
     """DRAM bytes per launch of the dominant kernel from the committed ncu summary, or None when the
     kernel sources changed since those counters were taken."""
     import glob
@@ -142,7 +144,7 @@ def recorded_traffic(kernel_tag="tc_gemm_pair_wgrad"):
             vals[k] = v.strip()
     csrc = os.path.join(ROOT, "paper_2110_08941_gb300", "csrc")
     h = hashlib.sha256()
-    for f in ("gemm_tc2.cu", "tc_device.cuh", "gemm_tc.cuh"):
+    for f in ("gemm_avg.cu", "tc_pair.cuh", "tc_device.cuh", "gemm_tc.cuh"):
         h.update(open(os.path.join(csrc, f), "rb").read())
     if vals.get("kernel_source_sha256") != h.hexdigest():
         return None
@@ -462,37 +464,52 @@ def run_ours(args, wl, rank, world, local_rank):
                  "unit": UNIT, "what": "slab-free formulation: worker weights folded into the loss-gradient "
                                        "scale, one all-rows weight-gradient product, update of one gradient"}
 
-    # the reduce+update timed on its own: a second context whose per-layer updates run after all
-    # products (HS_OVERLAP_UPDATE=0) instead of beside them, same workload and parameters
-    alone = None
-    if wl.arch == synth.MLP and precision == hs.HS_BF16:
-        prev = os.environ.get("HS_OVERLAP_UPDATE")
-        os.environ["HS_OVERLAP_UPDATE"] = "0"
+    # The slab path (HS_TILE_AVERAGE=0: per-worker weight gradients stored as fp32 slabs, then one
+    # reduce+update pass) in two further contexts on the same workload and parameters: with the
+    # per-layer updates on the step's stream, which times reduce_update_kernel alone, and in its
+    # default form, updates on a side stream beside the remaining products.
+    def slab_context(overlap):
+        env = {"HS_TILE_AVERAGE": "0", "HS_OVERLAP_UPDATE": "1" if overlap else "0"}
+        prev = {k: os.environ.get(k) for k in env}
+        os.environ.update(env)
         try:
-            ctx2 = hs.hs_init(wl.arch, wl.dims, wl.workers, wl.global_batch, compute_weights=w, precision=precision,
+            return hs.hs_init(wl.arch, wl.dims, wl.workers, wl.global_batch, compute_weights=w, precision=precision,
                               sync=hs.HS_SYNC_CP_WEIGHTED)
         finally:
-            if prev is None:
-                os.environ.pop("HS_OVERLAP_UPDATE")
-            else:
-                os.environ["HS_OVERLAP_UPDATE"] = prev
-        p2 = params.clone()
-        for _ in range(args.warmup):
-            hs.hs_step(ctx2, p2, xd, yd, ctx2.partition, wl.lr, stream=stream, want_loss=False)
-        torch.cuda.synchronize()
-        hs.hs_read_profile(ctx2)
-        hs.hs_set_profiling(ctx2, True)
+            for k, v in prev.items():
+                if v is None:
+                    os.environ.pop(k)
+                else:
+                    os.environ[k] = v
+
+    alone = None
+    slab = None
+    if wl.arch == synth.MLP and precision == hs.HS_BF16:
         k2 = max(3, min(args.steps, 10))
-        a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        a0.record(stream)
-        for _ in range(k2):
-            hs.hs_step(ctx2, p2, xd, yd, ctx2.partition, wl.lr, stream=stream, want_loss=False)
-        a1.record(stream)
-        torch.cuda.synchronize()
-        prof2 = hs.hs_read_profile(ctx2)
-        alone = {"update_ms": prof2["update"][0] / k2, "step_ms": a0.elapsed_time(a1) / k2}
-        ctx2.close()
-        del p2
+        for overlap in (False, True):
+            ctx2 = slab_context(overlap)
+            p2 = params.clone()
+            for _ in range(args.warmup):
+                hs.hs_step(ctx2, p2, xd, yd, ctx2.partition, wl.lr, stream=stream, want_loss=False)
+            torch.cuda.synchronize()
+            hs.hs_read_profile(ctx2)
+            hs.hs_set_profiling(ctx2, not overlap)
+            a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a0.record(stream)
+            for _ in range(k2):
+                hs.hs_step(ctx2, p2, xd, yd, ctx2.partition, wl.lr, stream=stream, want_loss=False)
+            a1.record(stream)
+            torch.cuda.synchronize()
+            sms = max_over_ranks(a0.elapsed_time(a1)) / k2
+            if overlap:
+                slab = {"ms_per_step": sms, "value": world * wl.global_batch / (sms * 1e-3), "unit": UNIT,
+                        "what": "slab path (HS_TILE_AVERAGE=0): per-worker weight gradients stored as fp32 "
+                                "slabs, reduce+update per layer on a side stream beside the remaining products"}
+            else:
+                prof2 = hs.hs_read_profile(ctx2)
+                alone = {"update_ms": prof2["update"][0] / k2, "step_ms": sms}
+            ctx2.close()
+            del p2
 
     # end to end through the public API: every step copies its inputs from pinned host memory and
     # reads its loss back.  Pipelined: hs_stage_inputs copies step t + 1's inputs on a copy stream
@@ -546,29 +563,26 @@ def run_ours(args, wl, rank, world, local_rank):
     def gemm_roof(name):
         # per launch: the phase's algorithmic flops and time divided by its launches per step
         ach = flops[name] / (per_step[name] * 1e-3) / 1e12
-        traffic = recorded_traffic() if (name == "wgrad" and wl.name == DEFAULT_WORKLOAD) else None
-        return {"kernel": f"tc_gemm ({name})", "bound": "tensor", "achieved": ach, "peak": peaks["bf16_sust"],
+        tile = name == "wgrad" and wl.arch == synth.MLP and precision == hs.HS_BF16
+        traffic = recorded_traffic() if (tile and wl.name == DEFAULT_WORKLOAD) else None
+        kernel = ("tc_wgrad_avg_pair_kernel (per-worker weight gradients averaged in tensor memory, "
+                  "update fused)" if tile else f"tc_gemm_pair_kernel ({name})")
+        return {"kernel": kernel, "bound": "tensor", "achieved": ach, "peak": peaks["bf16_sust"],
                 "unit": "TFLOP/s", "frac": ach / peaks["bf16_sust"], "traffic": traffic,
                 "flops_per_launch": flops[name] / launches_per_step[name],
                 "launches_per_step": launches_per_step[name],
                 "peak_kind": f"{peaks['src']} bf16 sustained"}
 
-    overlapped = os.environ.get("HS_OVERLAP_UPDATE", "1") != "0" and wl.arch == synth.MLP
-    upd_ms = alone["update_ms"] if (alone and overlapped) else per_step["update"]
+    upd_ms = alone["update_ms"] if alone else per_step["update"]
     upd_ach = upd_bytes / (upd_ms * 1e-3) / 1e9
     roof_update = {"kernel": "reduce_update", "bound": "hbm", "achieved": upd_ach, "peak": peaks["hbm"],
                    "unit": "GB/s", "frac": upd_ach / peaks["hbm"], "traffic": None,
                    "peak_kind": f"{peaks['src']} copy bandwidth", "algorithmic_bytes": upd_bytes,
-                   "timed": ("alone: per-layer updates after all products (second context, "
-                             "HS_OVERLAP_UPDATE=0)" if (alone and overlapped) else "inside the step"),
+                   "timed": ("slab path (HS_TILE_AVERAGE=0), per-layer updates on the step's stream "
+                             "(HS_OVERLAP_UPDATE=0), all P parameters" if alone else "inside the step"),
                    "ms_per_step": upd_ms}
-    if alone and overlapped:
-        ov_ach = upd_bytes / (per_step["update"] * 1e-3) / 1e9
-        roof_update["beside_products"] = {"ms_per_step": per_step["update"], "achieved": ov_ach,
-                                          "frac": ov_ach / peaks["hbm"],
-                                          "note": "the default step: updates share HBM and SMs with the "
-                                                  "backward products they overlap"}
-        roof_update["step_ms_updates_after_products"] = alone["step_ms"]
+    if alone:
+        roof_update["step_ms_slab_path_inline_updates"] = alone["step_ms"]
     roofline = roof_update if dominant == "update" else gemm_roof(dominant)
     gemm_ms = per_step["forward"] + per_step["wgrad"] + per_step["dgrad"]
     gemm_total = sum(flops.values())
@@ -588,7 +602,8 @@ def run_ours(args, wl, rank, world, local_rank):
             "vs_baseline": None, "dtype": "bf16" if precision == hs.HS_BF16 else "f32", "data": "synthetic",
             "config": {"workload": wl.name, "global_batch": wl.global_batch, "workers": wl.workers,
                        "dims": list(wl.dims), "sync": "cp_weighted", "parallelism": f"replicas{world}",
-                       "l2": ("working set > L2 (7 GB slabs, 0.9 GB activations per step), no flush"
+                       "l2": ("working set > L2 (over 1 GB of activations and input gradients, 0.44 GB theta per "
+                                     "step), no flush"
                               if wl.name == DEFAULT_WORKLOAD else "small workload: working set may sit in L2")},
             "roofline": roofline,
             "roofline_gemm_phase": {"bound": "tensor", "achieved": gemm_total / (gemm_ms * 1e-3) / 1e12,
@@ -610,6 +625,7 @@ def run_ours(args, wl, rank, world, local_rank):
             "clocks": clk,
             "straggler_sim": straggler_simulation(),
             "fused_sync_variant": fused,
+            "slab_path": slab,
             "graph_replay": graph,
             "heterogeneity_sim": heterogeneity_simulation(ms * 1e-3 / args.steps / wl.global_batch),
             "loss_after": loss,
