@@ -15,8 +15,13 @@
  *
  * On one GPU the M workers are contiguous segments of one global minibatch:
  * worker m owns samples [off_m, off_m + n_m).  Each segment gets its own
- * forward and backward pass (the per-worker gradient slab G_m), then one fused
- * pass reduces sum_m w_m G_m and applies the update.
+ * forward and backward pass and its own gradient G_m, and the update applies
+ * sum_m w_m G_m.  On the bf16 MLP step each tile of a layer's weight gradient
+ * G_m is formed in tensor memory and folded into the weighted sum there, in
+ * worker order, by the kernel that also applies the update; bias gradients (and
+ * every range on the slab path: debug read-back, the momentum recipe, more than
+ * 32 workers, the fp32 check path, the CNN) go through per-worker fp32 slabs in
+ * device memory and one reduce-and-update pass.  Both forms give the same bits.
  *
  * Conventions for every entry point:
  *   - Pointers marked "device" are CUDA device pointers on the device that was
@@ -215,8 +220,11 @@ hs_status hs_set_debug(hs_ctx* ctx, int32_t enable);
 
 /* Copy the last step's synchronised gradient g (device fp32 [P]; needs
  * hs_set_debug(ctx, 1) before that step, else HS_ERR_INVALID_ARG) and/or the
- * per-worker gradient slabs G_m (device fp32 [M, P], row m = worker m).  Either
- * pointer may be NULL.  Copies are enqueued on `stream`. */
+ * per-worker gradient slabs G_m (device fp32 [M, P], row m = worker m; a bf16
+ * MLP step without debug keeps the weight ranges in tensor memory only, so
+ * slabs_out then also needs hs_set_debug(ctx, 1) before the step, else
+ * HS_ERR_INVALID_ARG).  Either pointer may be NULL.  Copies are enqueued on
+ * `stream`. */
 hs_status hs_debug_grads(hs_ctx* ctx, float* g_out, float* slabs_out, void* stream);
 
 /* Per-worker losses L_m of the last step (host float [M]); synchronises. */

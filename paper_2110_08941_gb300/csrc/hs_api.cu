@@ -516,6 +516,8 @@ hs_status mlp_step_bf16(hs_ctx* c, float* params, const float* x, const int32_t*
   // the momentum recipe take the slab path.
   const bool avg = c->tile_avg && !c->fused_sync && !c->debug && !c->opt_recipe;
   if (avg) bind_avg_theta(c, params);
+  c->tile_step = false;
+  for (int l = 0; l < L && avg; ++l) c->tile_step = c->tile_step || c->avg_ok[l];
   bool side = false;   // work queued on the update stream this step
   for (int l = L - 1; l >= 0; --l) {
     const Layer& ly = c->layers[l];
@@ -1162,6 +1164,10 @@ hs_status hs_debug_grads(hs_ctx* c, float* g_out, float* slabs_out, void* stream
   }
   if (slabs_out) {
     if (c->fused_sync) return fail(c, HS_ERR_INVALID_ARG, "the slab-free formulation keeps no per-worker slabs");
+    if (c->tile_step)
+      return fail(c, HS_ERR_INVALID_ARG,
+                  "the last step kept the per-worker weight gradients in tensor memory: call hs_set_debug(ctx, 1) "
+                  "before hs_step for slabs");
     HS_CUDA(c, cudaMemcpy2DAsync(slabs_out, sizeof(float) * c->P, c->d_slabs, sizeof(float) * c->Ps,
                                  sizeof(float) * c->P, c->M, cudaMemcpyDeviceToDevice, s));
   }

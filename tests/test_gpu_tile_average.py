@@ -113,3 +113,25 @@ def test_tile_average_full_size_equals_slab_path():
                  x, y, theta0)
     assert torch.equal(a, b)
     assert la == lb
+
+
+def test_slab_read_back_needs_debug_after_a_tile_step():
+    """A step without debug keeps the weight ranges of the per-worker gradients in tensor memory:
+    asking for the slabs afterwards is an argument error, and a debug step provides them."""
+    dims, N, M = (256, 512, 10), 512, 4
+    x, y, theta0 = _data(dims, N, seed=5)
+    ctx = _init(dims, M, N, (1.0, 2.0, 3.0, 4.0), hs.HS_SYNC_CP_WEIGHTED, True)
+    try:
+        p = torch.tensor(theta0, device="cuda")
+        xd, yd = torch.from_numpy(x).cuda(), torch.from_numpy(y).cuda()
+        hs.hs_step(ctx, p, xd, yd, None, 0.05)
+        slabs = torch.empty(M, ctx.P, device="cuda")
+        with pytest.raises(hs.HsError):
+            hs.hs_debug_grads(ctx, None, slabs)
+        hs.hs_set_debug(ctx, True)
+        hs.hs_step(ctx, p, xd, yd, None, 0.05)
+        hs.hs_debug_grads(ctx, None, slabs)
+        torch.cuda.synchronize()
+        assert torch.isfinite(slabs).all() and slabs.abs().sum() > 0
+    finally:
+        ctx.close()
