@@ -188,6 +188,9 @@ __global__ void __launch_bounds__(kAvThreads, 1) tc_wgrad_avg_pair_kernel(const 
     if (lane == 0 && leader) {
       // ------------------------------------------------------------ pair MMA issuer (leader)
       constexpr uint32_t idesc = make_idesc(true, true, AV_PM, AV_PN);
+      constexpr uint64_t kStageDesc = AV_STAGE >> 4;   // one stage, in the descriptor's address field
+      const uint64_t a_desc0 = make_sdesc(smem_u32(smem), MN_CHUNK, 1024);
+      const uint64_t b_desc0 = make_sdesc(smem_u32(smem) + AV_A_HALF, MN_CHUNK, 1024);
       int s = 0;
       uint32_t ph = 0;
       int ab = 0;
@@ -198,20 +201,29 @@ __global__ void __launch_bounds__(kAvThreads, 1) tc_wgrad_avg_pair_kernel(const 
           if (!mbar_wait(smem_u32(&tempty_bar[ab]), aph ^ 1u, abort_flag)) { ok = false; break; }
           tc_fence_after();
           const uint32_t d_tmem = tmem_base + (uint32_t)(ab * AV_PN);
+          // full k-blocks, then the worker's partial last k-block
+          const LastKb lk = last_kb_of(p, g);
           const int nkb = p.num_kb[g];
-          for (int kb = 0; kb < nkb; ++kb) {
+          const int kb_full = lk.kb_last >= 0 ? lk.kb_last : nkb;
+          int kb = 0;
+          for (; kb < kb_full; ++kb) {
             if (!mbar_wait(smem_u32(&full_bar[s]), ph, abort_flag)) { ok = false; break; }
             tc_fence_after();
-            const uint32_t a_base = smem_u32(smem + s * AV_STAGE);
-            const uint32_t b_base = a_base + AV_A_HALF;
-#pragma unroll
-            for (int kk = 0; kk < BK / 16; ++kk) {
-              const uint64_t ad = make_sdesc(a_base + kk * 2048, MN_CHUNK, 1024);
-              const uint64_t bd = make_sdesc(b_base + kk * 2048, MN_CHUNK, 1024);
-              umma_bf16_pair(d_tmem, ad, bd, idesc, (kb != 0 || kk != 0) ? 1u : 0u);
-            }
+            const uint64_t off = kStageDesc * (uint64_t)s;
+            mma_kblock_pair<true, true>(d_tmem, a_desc0 + off, b_desc0 + off, idesc, kb != 0 ? 1u : 0u);
             umma_commit_pair(smem_u32(&empty_bar[s]));
             if (++s == AV_S) { s = 0; ph ^= 1u; }
+          }
+          if (ok && kb < nkb) {
+            if (!mbar_wait(smem_u32(&full_bar[s]), ph, abort_flag)) {
+              ok = false;
+            } else {
+              tc_fence_after();
+              const uint64_t off = kStageDesc * (uint64_t)s;
+              mma_ksteps_pair<true, true>(d_tmem, a_desc0 + off, b_desc0 + off, idesc, kb != 0 ? 1u : 0u, lk.steps);
+              umma_commit_pair(smem_u32(&empty_bar[s]));
+              if (++s == AV_S) { s = 0; ph ^= 1u; }
+            }
           }
           if (!ok) break;
           umma_commit_pair(smem_u32(&tfull_bar[ab]));

@@ -144,6 +144,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
     if (lane == 0) {
       // ------------------------------------------------------------ MMA issuer
       constexpr uint32_t idesc = make_idesc(A_MN, B_MN, BM, BN);
+      const uint64_t a_desc0 = make_sdesc(smem_u32(sA), A_MN ? MN_CHUNK : 16, 1024);
+      const uint64_t b_desc0 = make_sdesc(smem_u32(sB), B_MN ? MN_CHUNK : 16, 1024);
       int s = 0;
       uint32_t ph = 0;
       int ab = 0;
@@ -158,19 +160,13 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + (uint32_t)(ab * BN);
         bool ok = true;
+        const LastKb lk = last_kb_of(p, w.g);
         for (int kb = w.kb_lo; kb < w.kb_hi; ++kb) {
           if (!mbar_wait(smem_u32(&full_bar[s]), ph, abort_flag)) { ok = false; break; }
           tc_fence_after();
-          const uint32_t a_base = smem_u32(sA + s * A_STAGE);
-          const uint32_t b_base = smem_u32(sB + s * B_STAGE);
-#pragma unroll
-          for (int kk = 0; kk < BK / 16; ++kk) {
-            const uint64_t ad = A_MN ? make_sdesc(a_base + kk * 2048, MN_CHUNK, 1024)
-                                     : make_sdesc(a_base + kk * 32, 16, 1024);
-            const uint64_t bd = B_MN ? make_sdesc(b_base + kk * 2048, MN_CHUNK, 1024)
-                                     : make_sdesc(b_base + kk * 32, 16, 1024);
-            umma_bf16(d_tmem, ad, bd, idesc, (kb != w.kb_lo || kk != 0) ? 1u : 0u);
-          }
+          const int nks = kb == lk.kb_last ? lk.steps : BK / 16;
+          mma_ksteps<A_MN, B_MN>(d_tmem, a_desc0 + (uint64_t)((s * A_STAGE) >> 4),
+                                 b_desc0 + (uint64_t)((s * B_STAGE) >> 4), idesc, kb != w.kb_lo ? 1u : 0u, nks);
           umma_commit(smem_u32(&empty_bar[s]));
           if (++s == S) { s = 0; ph ^= 1u; }
         }

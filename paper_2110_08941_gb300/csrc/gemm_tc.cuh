@@ -74,6 +74,8 @@ struct TcGemmParams {
                                    // a tile of its own writing part j of tmD[g], a 3-D map [parts][rows][cols]
                                    // (needs num_kb[g] >= ksplit); 0 or 1: no split
   int32_t num_kb[kTcMaxGroups];
+  int32_t last_ksteps[kTcMaxGroups];   // 16-row MMA steps holding rows in group g's last k-block (1..4;
+                                       // 0 = all 4): the zero-filled steps past the group's rows are skipped
   int32_t groups;
   int32_t Mdim, Ndim, n_store;
   int32_t tiles_m, tiles_n;

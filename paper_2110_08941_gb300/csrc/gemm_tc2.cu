@@ -165,6 +165,9 @@ __global__ void __launch_bounds__(kThreads2, 1) tc_gemm_pair_kernel(const __grid
     if (lane == 0 && leader) {
       // ------------------------------------------------------------ pair MMA issuer (leader)
       constexpr uint32_t idesc = make_idesc(A_MN, B_MN, PM, PN);
+      constexpr uint64_t kStageDesc = STAGE2 >> 4;   // one stage, in the descriptor's address field
+      const uint64_t a_desc0 = make_sdesc(smem_u32(smem), A_MN ? MN_CHUNK : 16, 1024);
+      const uint64_t b_desc0 = make_sdesc(smem_u32(smem) + A_HALF, B_MN ? MN_CHUNK : 16, 1024);
       int s = 0;
       uint32_t ph = 0;
       int ab = 0;
@@ -179,21 +182,30 @@ __global__ void __launch_bounds__(kThreads2, 1) tc_gemm_pair_kernel(const __grid
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + (uint32_t)(ab * PN);
         bool ok = true;
-        for (int kb = w.kb_lo; kb < w.kb_hi; ++kb) {
+        // full k-blocks, then (when this tile holds it) the group's partial last k-block
+        const LastKb lk = last_kb_of(p, w.g);
+        const bool tail = lk.kb_last >= w.kb_lo && lk.kb_last < w.kb_hi;
+        const int kb_full = tail ? lk.kb_last : w.kb_hi;
+        int kb = w.kb_lo;
+        for (; kb < kb_full; ++kb) {
           if (!mbar_wait(smem_u32(&full_bar[s]), ph, abort_flag)) { ok = false; break; }
           tc_fence_after();
-          const uint32_t a_base = smem_u32(smem + s * STAGE2);
-          const uint32_t b_base = a_base + A_HALF;
-#pragma unroll
-          for (int kk = 0; kk < BK / 16; ++kk) {
-            const uint64_t ad = A_MN ? make_sdesc(a_base + kk * 2048, MN_CHUNK, 1024)
-                                     : make_sdesc(a_base + kk * 32, 16, 1024);
-            const uint64_t bd = B_MN ? make_sdesc(b_base + kk * 2048, MN_CHUNK, 1024)
-                                     : make_sdesc(b_base + kk * 32, 16, 1024);
-            umma_bf16_pair(d_tmem, ad, bd, idesc, (kb != w.kb_lo || kk != 0) ? 1u : 0u);
-          }
+          const uint64_t off = kStageDesc * (uint64_t)s;
+          mma_kblock_pair<A_MN, B_MN>(d_tmem, a_desc0 + off, b_desc0 + off, idesc, kb != w.kb_lo ? 1u : 0u);
           umma_commit_pair(smem_u32(&empty_bar[s]));
           if (++s == S2) { s = 0; ph ^= 1u; }
+        }
+        if (ok && tail) {
+          if (!mbar_wait(smem_u32(&full_bar[s]), ph, abort_flag)) {
+            ok = false;
+          } else {
+            tc_fence_after();
+            const uint64_t off = kStageDesc * (uint64_t)s;
+            mma_ksteps_pair<A_MN, B_MN>(d_tmem, a_desc0 + off, b_desc0 + off, idesc, kb != w.kb_lo ? 1u : 0u,
+                                        lk.steps);
+            umma_commit_pair(smem_u32(&empty_bar[s]));
+            if (++s == S2) { s = 0; ph ^= 1u; }
+          }
         }
         if (!ok) {
           record_error(p.st, kDevWaitTimeout, 13);

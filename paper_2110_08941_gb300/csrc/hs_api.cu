@@ -114,6 +114,13 @@ hs_status build_tc_static(hs_ctx* c) {
   return HS_OK;
 }
 
+// MMA steps of 16 rows holding data in the last k-block of a K extent of n rows (1..3), or 0 when
+// that k-block is full (all four steps, the kernels' straight-line path).
+int32_t last_ksteps(int64_t n) {
+  const int64_t r = n < 1 ? 0 : ((n - 1) % hs::kTcBK) / 16 + 1;
+  return r == hs::kTcBK / 16 ? 0 : (int32_t)r;
+}
+
 // The slab-free formulation's weight gradients: one group over all N rows into slab 0.
 hs_status build_tc_wgrad_fused(hs_ctx* c) {
   const char* why = nullptr;
@@ -170,6 +177,7 @@ hs_status build_tc_wgrad(hs_ctx* c) {
             !hs::tc_make_store_map(&w.tmD[g], dg, true, out_cols, ly.in, ly.in, &why))
           return fail(c, HS_ERR_CUDA, why);
         w.num_kb[g] = (int32_t)((n + hs::kTcBK - 1) / hs::kTcBK);
+        w.last_ksteps[g] = last_ksteps(n);
       }
       w.groups = ng;
       w.Mdim = out_cols;
@@ -213,6 +221,7 @@ hs_status build_tc_wgrad_avg(hs_ctx* c) {
       hs::TcOperand b{reinterpret_cast<const __nv_bfloat16*>(c->d_act[l]) + off * ly.in, n, ly.in, ly.in};
       ok = n >= 1 && hs::tc_make_mnmajor_map(&w.tmA[m], a, &why) && hs::tc_make_mnmajor_map(&w.tmB[m], b, &why);
       w.num_kb[m] = (int32_t)((n + hs::kTcBK - 1) / hs::kTcBK);
+      w.last_ksteps[m] = last_ksteps(n);
     }
     __nv_bfloat16* shadow = (l > 0 ? c->d_shadow_next : c->d_shadow) + ly.w_off;
     ok = ok && shadow && hs::tc_make_store_map_bf16_32(&w.tmS, shadow, out_cols, ly.in, ly.in, &why);
@@ -1233,6 +1242,7 @@ hs_status hs_debug_gemm_bf16(int32_t mode, int32_t M, int32_t N, int32_t K, cons
                                    N, ldd, &why))
           return fail(nullptr, HS_ERR_INVALID_ARG, why);
         p.num_kb[g] = (int)((kn + hs::kTcBK - 1) / hs::kTcBK);
+        p.last_ksteps[g] = last_ksteps(kn);
       }
       p.groups = ng;
       p.epi = hs::kTcEpiStoreF32;

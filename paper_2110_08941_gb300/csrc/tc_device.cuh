@@ -274,6 +274,39 @@ __device__ __forceinline__ TileWork tile_work(const TcGemmParams& p, int t, int 
   return w;
 }
 
+// MMA steps of 16 rows in group g's last k-block, whose rows past the group's extent are zero
+// fill (their products add nothing): kb_last = that k-block (-1: issue all 4 everywhere).  Read
+// once per group, outside the k-block loop: the issuing thread is on the tensor core's critical
+// path, and a parameter load per k-block shows up in the main loop.
+struct LastKb {
+  int kb_last, steps;
+};
+__device__ __forceinline__ LastKb last_kb_of(const TcGemmParams& p, int g) {
+  const int l = p.last_ksteps[g];
+  LastKb r;
+  r.kb_last = l > 0 ? p.num_kb[g] - 1 : -1;
+  r.steps = l;
+  return r;
+}
+
+// The one-SM MMAs of one k-block (four 16-row steps; see mma_kblock_pair), or of its first
+// `steps` steps.
+template <bool A_MN, bool B_MN>
+__device__ __forceinline__ void mma_ksteps(uint32_t d_tmem, uint64_t ad, uint64_t bd, uint32_t idesc, uint32_t acc0,
+                                           int steps) {
+  constexpr uint64_t kA = A_MN ? (2048 >> 4) : (32 >> 4);
+  constexpr uint64_t kB = B_MN ? (2048 >> 4) : (32 >> 4);
+  if (steps == BK / 16) {
+    umma_bf16(d_tmem, ad, bd, idesc, acc0);
+    umma_bf16(d_tmem, ad + kA, bd + kB, idesc, 1u);
+    umma_bf16(d_tmem, ad + 2 * kA, bd + 2 * kB, idesc, 1u);
+    umma_bf16(d_tmem, ad + 3 * kA, bd + 3 * kB, idesc, 1u);
+  } else {
+#pragma unroll 1
+    for (int kk = 0; kk < steps; ++kk) umma_bf16(d_tmem, ad + kk * kA, bd + kk * kB, idesc, kk ? 1u : acc0);
+  }
+}
+
 __device__ __forceinline__ float u2f(uint32_t u) { return __uint_as_float(u); }
 
 __device__ __forceinline__ uint32_t pack_bf16(float a, float b) {

@@ -67,5 +67,31 @@ __device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr) {
   asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
 }
 
+
+// The pair MMAs of one k-block (64 rows of K, four 16-row steps) from the stage whose A and B
+// descriptors are `ad` and `bd`: within a stage a K step advances the start address by 2 KB
+// (MN-major tile) or 32 B (K-major tile), i.e. the descriptor's address field by 128 or 2.  The
+// issuing thread is on the tensor core's critical path, so descriptors are formed by one add.
+template <bool A_MN, bool B_MN>
+__device__ __forceinline__ void mma_kblock_pair(uint32_t d_tmem, uint64_t ad, uint64_t bd, uint32_t idesc,
+                                                uint32_t acc0) {
+  constexpr uint64_t kA = A_MN ? (2048 >> 4) : (32 >> 4);
+  constexpr uint64_t kB = B_MN ? (2048 >> 4) : (32 >> 4);
+  umma_bf16_pair(d_tmem, ad, bd, idesc, acc0);
+  umma_bf16_pair(d_tmem, ad + kA, bd + kB, idesc, 1u);
+  umma_bf16_pair(d_tmem, ad + 2 * kA, bd + 2 * kB, idesc, 1u);
+  umma_bf16_pair(d_tmem, ad + 3 * kA, bd + 3 * kB, idesc, 1u);
+}
+// The first `steps` (1..4) of them: a group's last k-block, whose later steps are zero fill.
+template <bool A_MN, bool B_MN>
+__device__ __forceinline__ void mma_ksteps_pair(uint32_t d_tmem, uint64_t ad, uint64_t bd, uint32_t idesc,
+                                                uint32_t acc0, int steps) {
+  constexpr uint64_t kA = A_MN ? (2048 >> 4) : (32 >> 4);
+  constexpr uint64_t kB = B_MN ? (2048 >> 4) : (32 >> 4);
+#pragma unroll 1
+  for (int kk = 0; kk < steps; ++kk)
+    umma_bf16_pair(d_tmem, ad + kk * kA, bd + kk * kB, idesc, kk ? 1u : acc0);
+}
+
 }  // namespace tcpair
 }  // namespace hs
