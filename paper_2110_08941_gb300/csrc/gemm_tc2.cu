@@ -27,32 +27,37 @@ using namespace tcpair;
 constexpr int PM = 256;                            // pair tile rows
 constexpr int HM = PM / 2;                         // per-CTA half
 constexpr int A_HALF = HM * BK * 2;                // 16 KB
-constexpr int kThreads2 = 192;
-
 // Pair tile of 256 x TN (TN = 256, or 128 for products at most 128 wide): per-CTA B half, stages
-// (more of them when the B half is smaller), two TN-column accumulators in tensor memory.
-template <int TN>
+// (more of them when the B half is smaller), two TN-column accumulators in tensor memory.  EW
+// epilogue warps (4, or 8 for short-K products whose epilogue outlasts the main loop: two per
+// tensor-memory lane quadrant, each on half of the tile's columns, with one stage fewer to fit
+// their staging buffers).
+template <int TN, int EW>
 struct PairCfg {
   static constexpr int PN = TN;
   static constexpr int HN = TN / 2;
   static constexpr int B_HALF = HN * BK * 2;
   static constexpr int STAGE2 = A_HALF + B_HALF;
-  static constexpr int S2 = TN == 256 ? 6 : 8;
+  static constexpr int S2 = TN == 256 ? (EW == 8 ? 5 : 6) : 8;
+  static constexpr int kThreads = 64 + 32 * EW;
   static constexpr uint32_t PAIR_TX = 2 * STAGE2;   // bytes landing per stage on the leader's barrier
   static constexpr uint32_t kTmemCols2 = 2 * TN;
-  static constexpr int kSmem2 = S2 * STAGE2 + kTcStagingBytes + 1024 + 256;
+  static constexpr int kStaging = EW * 8192;         // two 32-row x 128-byte buffers per epilogue warp
+  static constexpr int kSmem2 = S2 * STAGE2 + kStaging + 1024 + 256;
   static_assert(kSmem2 <= 232448, "shared memory budget");
+  static_assert(EW == 4 || (EW == 8 && TN == 256), "epilogue warps");
 };
 
-template <int EPI, bool A_MN, bool B_MN, bool CONV, int TN>
-__global__ void __launch_bounds__(kThreads2, 1) tc_gemm_pair_kernel(const __grid_constant__ TcGemmParams p) {
-  using Cfg = PairCfg<TN>;
+template <int EPI, bool A_MN, bool B_MN, bool CONV, int TN, int EW>
+__global__ void __launch_bounds__(PairCfg<TN, EW>::kThreads, 1)
+    tc_gemm_pair_kernel(const __grid_constant__ TcGemmParams p) {
+  using Cfg = PairCfg<TN, EW>;
   constexpr int PN = Cfg::PN, HN = Cfg::HN, S2 = Cfg::S2, STAGE2 = Cfg::STAGE2;
   constexpr uint32_t PAIR_TX = Cfg::PAIR_TX, kTmemCols2 = Cfg::kTmemCols2;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sStage = smem + S2 * STAGE2;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(sStage + kTcStagingBytes);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sStage + Cfg::kStaging);
   uint64_t* full_bar = bars;
   uint64_t* empty_bar = bars + S2;
   uint64_t* tfull_bar = bars + 2 * S2;
@@ -72,7 +77,7 @@ __global__ void __launch_bounds__(kThreads2, 1) tc_gemm_pair_kernel(const __grid
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(smem_u32(&tfull_bar[b]), 1);
-      mbar_init(smem_u32(&tempty_bar[b]), 8);   // 4 epilogue warps in each CTA of the pair
+      mbar_init(smem_u32(&tempty_bar[b]), 2 * EW);   // the epilogue warps of both CTAs of the pair
     }
     *abort_flag = 0;
     fence_mbar_init();
@@ -220,8 +225,9 @@ __global__ void __launch_bounds__(kThreads2, 1) tc_gemm_pair_kernel(const __grid
     // -------------------------------------------------------------- epilogue (warps 2..5, both CTAs)
     constexpr bool kF32Out = (EPI == kTcEpiBiasF32 || EPI == kTcEpiStoreF32);
     constexpr int kUnitCols = kF32Out ? 32 : 64;
-    constexpr int kUnits = PN / kUnitCols;
+    constexpr int kUnits = PN / kUnitCols / (EW / 4);   // units of this warp's column share
     const int q = warp & 3;
+    const int col_share = (warp - 2) >> 2;             // 0, or 1 for the second warp of a quadrant
     const uint32_t stage_base = smem_u32(sStage) + (uint32_t)((warp - 2) * 8192);
     int sb = 0;
     int ab = 0;
@@ -230,7 +236,8 @@ __global__ void __launch_bounds__(kThreads2, 1) tc_gemm_pair_kernel(const __grid
       const TileWork w = tile_work(p, t, tiles_m, tiles_n);
       const TileCoord c = w.c;
       uint4 zq[8];   // mask operand of the tile's first unit, loaded before the accumulator is ready
-      if (EPI == kTcEpiMaskBf16) load_mask_unit<CONV>(p, w.g, c.tm * PM + (int)rank * HM + q * 32 + lane, c.tn * PN, zq);
+      const int n_warp = c.tn * PN + col_share * kUnits * kUnitCols;   // this warp's first column
+      if (EPI == kTcEpiMaskBf16) load_mask_unit<CONV>(p, w.g, c.tm * PM + (int)rank * HM + q * 32 + lane, n_warp, zq);
       int ok = 1;
       if (lane == 0) ok = mbar_wait(smem_u32(&tfull_bar[ab]), aph, abort_flag) ? 1 : 0;
       ok = __shfl_sync(0xffffffffu, ok, 0);
@@ -246,10 +253,11 @@ __global__ void __launch_bounds__(kThreads2, 1) tc_gemm_pair_kernel(const __grid
       const int row0 = c.tm * PM + (int)rank * HM + q * 32;
       const int row = row0 + lane;
       const CUtensorMap* td = &p.tmD[w.g];
-      const uint32_t t_row = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(ab * PN);
+      const uint32_t t_row = tmem_base + ((uint32_t)(q * 32) << 16) +
+                             (uint32_t)(ab * PN + col_share * kUnits * kUnitCols);
 #pragma unroll 1
       for (int u = 0; u < kUnits; ++u) {
-        const int n_base = c.tn * PN + u * kUnitCols;
+        const int n_base = n_warp + u * kUnitCols;
         if (n_base >= p.n_store) break;
         uint32_t r[32], r2[32];
         tmem_ld32(t_row + (uint32_t)(u * kUnitCols), r);
@@ -299,19 +307,19 @@ __global__ void __launch_bounds__(kThreads2, 1) tc_gemm_pair_kernel(const __grid
   }
 }
 
-template <int EPI, bool A_MN, bool B_MN, bool CONV, int TN = 256>
+template <int EPI, bool A_MN, bool B_MN, bool CONV, int TN = 256, int EW = 4>
 cudaError_t launch_pair_variant(const TcGemmParams& p, int pairs_wanted, int num_sms, cudaStream_t s) {
   static bool configured = false;
   static int max_clusters = 0;
-  constexpr int kSmem2 = PairCfg<TN>::kSmem2;
-  auto kern = tc_gemm_pair_kernel<EPI, A_MN, B_MN, CONV, TN>;
+  constexpr int kSmem2 = PairCfg<TN, EW>::kSmem2;
+  auto kern = tc_gemm_pair_kernel<EPI, A_MN, B_MN, CONV, TN, EW>;
   cudaLaunchConfig_t cfg = {};
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = 2;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
-  cfg.blockDim = dim3(kThreads2, 1, 1);
+  cfg.blockDim = dim3(PairCfg<TN, EW>::kThreads, 1, 1);
   cfg.dynamicSmemBytes = kSmem2;
   cfg.stream = s;
   cfg.attrs = attr;
@@ -363,6 +371,13 @@ cudaError_t launch_tc_gemm_pair(const TcGemmParams& p, int num_sms, cudaStream_t
     if (p.epi == kTcEpiBiasReluBf16 && !p.a_mn && !p.b_mn) return launch_pair_variant<kTcEpiBiasReluBf16, false, false, true>(p, pairs, grid, s);
     if (p.epi == kTcEpiStoreF32 && p.a_mn && p.b_mn) return launch_pair_variant<kTcEpiStoreF32, true, true, true>(p, pairs, grid, s);
     if (p.epi == kTcEpiMaskBf16 && !p.a_mn && p.b_mn) return launch_pair_variant<kTcEpiMaskBf16, false, true, true>(p, pairs, grid, s);
+    return cudaErrorInvalidValue;
+  }
+  if (p.ew == 8) {
+    // short-K input gradients, whose epilogue (mask read, bf16 store) keeps up with the main loop
+    // only with eight epilogue warps
+    if (p.epi == kTcEpiMaskBf16 && !p.a_mn && p.b_mn)
+      return launch_pair_variant<kTcEpiMaskBf16, false, true, false, 256, 8>(p, pairs, grid, s);
     return cudaErrorInvalidValue;
   }
   if (p.epi == kTcEpiBiasReluBf16 && !p.a_mn && !p.b_mn) return launch_pair_variant<kTcEpiBiasReluBf16, false, false, false>(p, pairs, grid, s);

@@ -82,6 +82,7 @@ hs_status build_tc_static(hs_ctx* c) {
     f.tiles_m = (c->N + hs::kTcBM - 1) / hs::kTcBM;
     f.tiles_n = (f.n_store + hs::kTcBN - 1) / hs::kTcBN;
     f.epi = last ? hs::kTcEpiBiasF32 : hs::kTcEpiBiasReluBf16;
+    f.ew = 4;
     f.D = last ? static_cast<void*>(c->d_logits) : c->d_act[l + 1];
     f.ldd = last ? c->Cp : ly.out;
     f.st = c->d_status;
@@ -104,6 +105,7 @@ hs_status build_tc_static(hs_ctx* c) {
     d.epi = hs::kTcEpiMaskBf16;
     d.a_mn = 0;
     d.b_mn = 1;
+    d.ew = ly.out <= 2048 ? 8 : 4;   // short K: the epilogue outlasts the main loop
     d.D = c->delta_buf(l - 1);
     d.ldd = c->delta_ld(l - 1);
     d.Z = reinterpret_cast<const __nv_bfloat16*>(c->d_act[l]);
