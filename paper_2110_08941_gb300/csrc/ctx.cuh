@@ -169,6 +169,7 @@ struct hs_ctx {
   // per-worker weight gradients averaged in tensor memory and applied in the same kernel
   // (launch_tc_wgrad_avg): per layer, valid where avg_ok[l]; tmT points at avg_theta's weights
   bool tile_avg = false;
+  bool tile_avg_all = false;   // also layers with fewer weight tiles than SM pairs
   std::vector<hs::TcGemmParams> tc_wgrad_avg;
   std::vector<char> avg_ok;
   const float* avg_theta = nullptr;

@@ -200,7 +200,8 @@ hs_status build_tc_wgrad(hs_ctx* c) {
 }
 
 // The tile-averaged weight gradients: per layer one launch over all workers (groups), the update
-// fused in (launch_tc_wgrad_avg).  Layers 2..L write their bf16 weights to the second shadow (their
+// fused in (launch_tc_wgrad_avg), for layers with at least one 256 x 256 weight tile per SM pair
+// (all layers with HS_TILE_AVERAGE=all).  Layers 2..L write their bf16 weights to the second shadow (their
 // input-gradient products still read the first); layer 1 writes the first.  theta's maps are bound
 // per step (bind_avg_theta).  A layer whose operands the kernel cannot take keeps the slab path.
 hs_status build_tc_wgrad_avg(hs_ctx* c) {
@@ -227,6 +228,10 @@ hs_status build_tc_wgrad_avg(hs_ctx* c) {
     }
     __nv_bfloat16* shadow = (l > 0 ? c->d_shadow_next : c->d_shadow) + ly.w_off;
     ok = ok && shadow && hs::tc_make_store_map_bf16_32(&w.tmS, shadow, out_cols, ly.in, ly.in, &why);
+    // One SM pair per 256 x 256 tile of the layer's weights: with fewer tiles than pairs the
+    // grouped slab launch (a tile per worker) keeps more of the GPU busy.
+    const int64_t tiles = ((out_cols + 255) / 256) * (int64_t)((ly.in + 255) / 256);
+    if (!c->tile_avg_all && tiles < c->num_sms / 2) ok = false;
     w.groups = c->M;
     w.Mdim = out_cols;
     w.Ndim = ly.in;
@@ -864,11 +869,13 @@ hs_status hs_init(const hs_model_desc* model, int32_t M, const double* compute_w
   if (s2 == HS_OK && bf16 && c->arch == HS_MLP) s2 = build_tc_wgrad_fused(c);
   if (s2 == HS_OK && bf16 && c->arch == HS_MLP) {
     // HS_OVERLAP_UPDATE=0: slab-path updates on the step's stream instead of the update stream;
-    // HS_TILE_AVERAGE=0: every layer on the slab path (per-worker gradients stored, then reduced)
+    // HS_TILE_AVERAGE=0: every layer on the slab path (per-worker gradients stored, then reduced);
+    // =all: the tile-averaged launch also for layers with fewer weight tiles than SM pairs
     const char* ov = getenv("HS_OVERLAP_UPDATE");
     c->overlap_update = !(ov && !strcmp(ov, "0"));
     const char* ta = getenv("HS_TILE_AVERAGE");
     c->tile_avg = !(ta && !strcmp(ta, "0")) && c->M <= hs::kTcMaxGroups;
+    c->tile_avg_all = ta && !strcmp(ta, "all");
     e = cudaStreamCreateWithFlags(&c->upd_stream, cudaStreamNonBlocking);
     c->upd_ready.assign(c->L, nullptr);
     for (int l = 0; l < c->L && e == cudaSuccess; ++l) e = cudaEventCreateWithFlags(&c->upd_ready[l], cudaEventDisableTiming);

@@ -18,7 +18,7 @@ pytestmark = pytest.mark.gpu
 
 def _init(dims, M, N, weights, sync, tile):
     old = os.environ.get("HS_TILE_AVERAGE")
-    os.environ["HS_TILE_AVERAGE"] = "1" if tile else "0"
+    os.environ["HS_TILE_AVERAGE"] = "all" if tile else "0"
     try:
         return hs.hs_init(hs.HS_MLP, dims, M, N, compute_weights=weights, sync=sync)
     finally:
@@ -83,7 +83,8 @@ def test_tile_average_equals_slab_path(dims, N, M, weights, sync):
 
 
 @pytest.mark.parametrize("name", [synth.CFG2, synth.CFG3])
-def test_tile_average_matches_oracle(name):
+def test_tile_average_matches_oracle(name, monkeypatch):
+    monkeypatch.setenv("HS_TILE_AVERAGE", "all")   # every layer, however few its weight tiles
     wl = synth.WORKLOADS[name]
     x, y = synth.make_batch(wl)
     theta0 = synth.make_params(wl)
@@ -135,3 +136,24 @@ def test_slab_read_back_needs_debug_after_a_tile_step():
         assert torch.isfinite(slabs).all() and slabs.abs().sum() > 0
     finally:
         ctx.close()
+
+
+def test_default_takes_the_tile_launch_where_a_layer_fills_the_pairs():
+    """Default selection: the tile-averaged launch for layers with at least one 256 x 256 weight
+    tile per SM pair, the slab path for the rest, in one step (bit for bit the slab path)."""
+    dims, N, M = (256, 4096, 8192, 10), 1024, 4   # layer 2: 32 x 16 tiles (tile launch); 1, 3: slab
+    x, y, theta0 = _data(dims, N, seed=9)
+    os.environ.pop("HS_TILE_AVERAGE", None)
+    ctx = hs.hs_init(hs.HS_MLP, dims, M, N, compute_weights=(1.0, 2.0, 3.0, 4.0))
+    try:
+        p = torch.tensor(theta0, device="cuda")
+        xd, yd = torch.from_numpy(x).cuda(), torch.from_numpy(y).cuda()
+        for _ in range(2):
+            hs.hs_step(ctx, p, xd, yd, None, 0.05)
+        torch.cuda.synchronize()
+        with pytest.raises(hs.HsError):   # a tile step: its weight ranges are not in the slabs
+            hs.hs_debug_grads(ctx, None, torch.empty(M, ctx.P, device="cuda"))
+    finally:
+        ctx.close()
+    b, _ = _run(dims, M, N, (1.0, 2.0, 3.0, 4.0), hs.HS_SYNC_CP_WEIGHTED, False, 2, 0.05, x, y, theta0)
+    assert torch.equal(p.cpu(), b)
