@@ -649,10 +649,23 @@ def main():
     ap.add_argument("--impl", default="ours", choices=("ours", "reference"))
     ap.add_argument("--precision", default="bf16", choices=("bf16", "fp32"))
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--mlp-dims", default=None,
+                    help="profiling aid: an MLP of these comma-separated widths in place of the named "
+                         "workload's (with --batch and --workers; lognormal compute weights)")
+    ap.add_argument("--batch", type=int, default=None)
+    ap.add_argument("--workers", type=int, default=None)
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "ours":
         args.warmup = 3
     wl = synth.WORKLOADS[args.workload]
+    if args.mlp_dims:
+        import dataclasses
+        dims = tuple(int(v) for v in args.mlp_dims.split(","))
+        n = args.batch or wl.global_batch
+        m = args.workers or wl.workers
+        wl = dataclasses.replace(wl, name=f"mlp_{'_'.join(map(str, dims))}_b{n}_m{m}", arch=synth.MLP, dims=dims,
+                                 n_classes=dims[-1], global_batch=n, workers=m, weights=None,
+                                 weight_kind="lognormal", repartition_every=0)
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))

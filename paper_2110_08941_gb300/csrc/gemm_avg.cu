@@ -43,7 +43,7 @@ constexpr int AV_S = 6;
 constexpr uint32_t AV_TX = 2 * AV_STAGE;             // bytes landing per stage on the leader's barrier
 constexpr uint32_t AV_TMEM_COLS = 2 * AV_PN;
 constexpr int AV_BUF = 32 * 128;                     // per epilogue warp: one 32-row x 128-byte box
-constexpr int kAvSmem = AV_S * AV_STAGE + kAvEpiWarps * AV_BUF + 1024 + 256;
+constexpr int kAvSmem = AV_S * AV_STAGE + kAvEpiWarps * AV_BUF + 1024 + 512;
 static_assert(kAvSmem <= 232448, "shared memory budget");
 constexpr int AV_GM = 8;                             // M-tiles per band of the tile order
 
@@ -109,6 +109,9 @@ __global__ void __launch_bounds__(kAvThreads, 1) tc_wgrad_avg_pair_kernel(const 
   uint64_t* tload_bar = bars + 2 * AV_S + 4;        // [8] theta box landed in epilogue warp e's buffer
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * AV_S + 4 + kAvEpiWarps);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  // per group: k-blocks, MMA steps in the last one (a shared-memory copy: the producer and the
+  // MMA issuer read it at every worker switch, where a parameter-space load would stall them)
+  int2* kbinfo = reinterpret_cast<int2*>(bars + 32);
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -125,6 +128,7 @@ __global__ void __launch_bounds__(kAvThreads, 1) tc_wgrad_avg_pair_kernel(const 
       mbar_init(smem_u32(&tempty_bar[b]), 2 * kAvEpiWarps);
     }
     for (int e = 0; e < kAvEpiWarps; ++e) mbar_init(smem_u32(&tload_bar[e]), 1);
+    for (int g = 0; g < p.groups; ++g) kbinfo[g] = make_int2(p.num_kb[g], p.last_ksteps[g]);
     *abort_flag = 0;
     fence_mbar_init();
   }
@@ -162,7 +166,11 @@ __global__ void __launch_bounds__(kAvThreads, 1) tc_wgrad_avg_pair_kernel(const 
         for (int g = 0; g < G && ok; ++g) {
           const CUtensorMap* ta = &p.tmA[g];
           const CUtensorMap* tb = &p.tmB[g];
-          const int nkb = p.num_kb[g];
+          const int nkb = kbinfo[g].x;
+          // the next worker's descriptors, ahead of its first load
+          const int gn = g + 1 < G ? g + 1 : 0;
+          tma_prefetch_desc(&p.tmA[gn]);
+          tma_prefetch_desc(&p.tmB[gn]);
           for (int kb = 0; kb < nkb; ++kb) {
             if (!mbar_wait(smem_u32(&empty_bar[s]), ph ^ 1u, abort_flag)) { ok = false; break; }
             const uint32_t fb_local = smem_u32(&full_bar[s]);
@@ -202,8 +210,11 @@ __global__ void __launch_bounds__(kAvThreads, 1) tc_wgrad_avg_pair_kernel(const 
           tc_fence_after();
           const uint32_t d_tmem = tmem_base + (uint32_t)(ab * AV_PN);
           // full k-blocks, then the worker's partial last k-block
-          const LastKb lk = last_kb_of(p, g);
-          const int nkb = p.num_kb[g];
+          const int2 ki = kbinfo[g];
+          const int nkb = ki.x;
+          LastKb lk;
+          lk.kb_last = ki.y > 0 ? nkb - 1 : -1;
+          lk.steps = ki.y;
           const int kb_full = lk.kb_last >= 0 ? lk.kb_last : nkb;
           int kb = 0;
           for (; kb < kb_full; ++kb) {
