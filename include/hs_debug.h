@@ -48,6 +48,23 @@ hs_status hs_debug_gemm_bf16(int32_t mode, int32_t M, int32_t N, int32_t K, cons
                              const void* Z, int64_t ldz, const int32_t* k_offsets_host, int32_t groups,
                              int64_t d_gstride, void* stream);
 
+/* The per-worker weight gradients of one layer averaged in tensor memory with the update fused
+ * (the kernel hs_step uses for large bf16 MLP layers; Eq. 1's g^m, the weighted average of
+ * Section 1 / Section 4.2, theta <- theta - lr * g), run alone:
+ *   theta[M, N] <- theta - lr * sum_g wavg[g] * A[k_g, M]^T B[k_g, N]   (g = 0 .. groups-1 in order)
+ *   shadow[M, N] = bf16(new theta)
+ * with rows k_g = [k_offsets_host[g], k_offsets_host[g+1]) of A (bf16 [K][M], MN-major, leading
+ * dimension lda) and B (bf16 [K][N], ldb).  theta: device fp32, leading dimension ld_theta,
+ * updated in place; shadow: device bf16, ld_shadow; wavg: device fp32 [groups].  groups in
+ * 1..32, every group at least one row; leading dimensions multiples of 8 elements, pointers
+ * 16-byte aligned.  test_stall = 1: the kernel's loads are never issued, its bounded waits expire
+ * (2 s) and the call returns HS_ERR_DEVICE_CHECK with theta unchanged (the failure-detection
+ * test).  Synchronous; HS_ERR_INVALID_ARG / HS_ERR_CUDA / HS_ERR_DEVICE_CHECK as above. */
+hs_status hs_debug_wgrad_avg(int32_t M, int32_t N, const void* A, int64_t lda, const void* B, int64_t ldb,
+                             const int32_t* k_offsets_host, int32_t groups, const float* wavg, float lr,
+                             float* theta, int64_t ld_theta, void* shadow, int64_t ld_shadow, int32_t test_stall,
+                             void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -28,7 +28,7 @@ EXPORTED = ("hs_partition_sizes", "hs_param_count", "hs_init", "hs_partition", "
             "hs_set_debug", "hs_debug_grads", "hs_worker_losses", "hs_destroy", "hs_status_string",
             "hs_last_error", "hs_last_init_error", "hs_debug_gemm_bf16", "hs_set_profiling", "hs_read_profile",
             "hs_partition_noalloc", "hs_set_optimizer", "hs_optimizer_state", "hs_cosine_lr",
-            "hs_set_cp_history", "hs_set_fused_sync", "hs_stage_inputs")
+            "hs_set_cp_history", "hs_set_fused_sync", "hs_stage_inputs", "hs_debug_wgrad_avg")
 HS_CP_LAST, HS_CP_EMA, HS_CP_WINDOW = 0, 1, 2
 PHASES = ("cast", "forward", "loss", "wgrad", "biasgrad", "dgrad", "update")
 
@@ -83,6 +83,8 @@ def _load() -> ctypes.CDLL:
         "hs_debug_gemm_bf16": (S, [c_int32, c_int32, c_int32, c_int32, c_void_p, c_int64, c_void_p, c_int64,
                                    c_void_p, c_int64, c_void_p, c_void_p, c_int64, POINTER(c_int32), c_int32,
                                    c_int64, c_void_p]),
+        "hs_debug_wgrad_avg": (S, [c_int32, c_int32, c_void_p, c_int64, c_void_p, c_int64, POINTER(c_int32), c_int32,
+                                   c_void_p, ctypes.c_float, c_void_p, c_int64, c_void_p, c_int64, c_int32, c_void_p]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -300,6 +302,18 @@ def hs_worker_losses(ctx: Context) -> List[float]:
 
 def hs_destroy(ctx: Context):
     ctx.close()
+
+
+def hs_debug_wgrad_avg(A, B, k_offsets, wavg, lr: float, theta, shadow, test_stall: bool = False, stream=None):
+    """theta -= lr * sum_g wavg[g] A[k_g]^T B[k_g]; shadow = bf16(theta) (test hook, include/hs_debug.h).
+    A: bf16 [K, M], B: bf16 [K, N], wavg: fp32 [groups], theta: fp32 [M, N], shadow: bf16 [M, N]
+    (device tensors); k_offsets: groups + 1 row offsets."""
+    ko = (c_int32 * len(k_offsets))(*[int(v) for v in k_offsets])
+    M, N = int(theta.shape[0]), int(theta.shape[1])
+    _check(_lib.hs_debug_wgrad_avg(M, N, c_void_p(A.data_ptr()), int(A.stride(0)), c_void_p(B.data_ptr()),
+                                   int(B.stride(0)), ko, len(k_offsets) - 1, c_void_p(wavg.data_ptr()), float(lr),
+                                   c_void_p(theta.data_ptr()), int(theta.stride(0)), c_void_p(shadow.data_ptr()),
+                                   int(shadow.stride(0)), 1 if test_stall else 0, c_void_p(_stream_ptr(stream))))
 
 
 def hs_debug_gemm_bf16(mode: int, M: int, N: int, K: int, A, B, D, bias=None, Z=None, k_offsets=None,

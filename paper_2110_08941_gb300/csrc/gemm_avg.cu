@@ -158,7 +158,7 @@ __global__ void __launch_bounds__(kAvThreads, 1) tc_wgrad_avg_pair_kernel(const 
       int s = 0;
       uint32_t ph = 0;
       bool ok = true;
-      for (int t = pair_id; t < total && ok && !*abort_flag; t += n_pairs) {
+      for (int t = pair_id; t < total && ok && !*abort_flag && !p.test_stall; t += n_pairs) {
         int tm, tn;
         av_decode(t, tiles_m, tiles_n, tm, tn);
         const int m0 = tm * AV_PM + (int)rank * AV_HM;

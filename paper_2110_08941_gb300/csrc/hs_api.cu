@@ -1318,4 +1318,69 @@ hs_status hs_debug_gemm_bf16(int32_t mode, int32_t M, int32_t N, int32_t K, cons
   return HS_OK;
 }
 
+hs_status hs_debug_wgrad_avg(int32_t M, int32_t N, const void* A, int64_t lda, const void* B, int64_t ldb,
+                             const int32_t* k_offsets_host, int32_t groups, const float* wavg, float lr,
+                             float* theta, int64_t ld_theta, void* shadow, int64_t ld_shadow, int32_t test_stall,
+                             void* stream) {
+  g_init_error.clear();
+  if (M < 1 || N < 1 || !A || !B || !k_offsets_host || !wavg || !theta || !shadow || groups < 1 ||
+      groups > hs::kTcMaxGroups)
+    return fail(nullptr, HS_ERR_INVALID_ARG, "bad arguments (groups must be 1..32)");
+  if (lda % 8 || ldb % 8 || ld_theta % 8 || ld_shadow % 8 || lda < M || ldb < N || ld_theta < N || ld_shadow < N)
+    return fail(nullptr, HS_ERR_INVALID_ARG, "leading dimensions must be multiples of 8 elements");
+  auto a16 = [](const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; };
+  if (!a16(A) || !a16(B) || !a16(theta) || !a16(shadow))
+    return fail(nullptr, HS_ERR_INVALID_ARG, "pointers must be 16-byte aligned");
+  const char* why = nullptr;
+  if (!hs::tc_init_driver(&why)) return fail(nullptr, HS_ERR_CUDA, why);
+  int dev = 0, sms = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  hs::TcGemmParams p;
+  std::memset(&p, 0, sizeof(p));
+  const auto* pa = reinterpret_cast<const __nv_bfloat16*>(A);
+  const auto* pb = reinterpret_cast<const __nv_bfloat16*>(B);
+  for (int g = 0; g < groups; ++g) {
+    const int64_t k0 = k_offsets_host[g], kn = k_offsets_host[g + 1] - k0;
+    if (kn < 1) return fail(nullptr, HS_ERR_INVALID_ARG, "every group needs at least one row");
+    if (!hs::tc_make_mnmajor_map(&p.tmA[g], hs::TcOperand{pa + k0 * lda, kn, M, lda}, &why) ||
+        !hs::tc_make_mnmajor_map(&p.tmB[g], hs::TcOperand{pb + k0 * ldb, kn, N, ldb}, &why))
+      return fail(nullptr, HS_ERR_INVALID_ARG, why);
+    p.num_kb[g] = (int32_t)((kn + hs::kTcBK - 1) / hs::kTcBK);
+    p.last_ksteps[g] = last_ksteps(kn);
+  }
+  if (!hs::tc_make_store_map(&p.tmT, theta, true, M, N, ld_theta, &why) ||
+      !hs::tc_make_store_map_bf16_32(&p.tmS, shadow, M, N, ld_shadow, &why))
+    return fail(nullptr, HS_ERR_INVALID_ARG, why);
+  p.groups = groups;
+  p.Mdim = M;
+  p.Ndim = N;
+  p.n_store = N;
+  p.epi = hs::kTcEpiAvgUpdate;
+  p.a_mn = 1;
+  p.b_mn = 1;
+  p.wavg = wavg;
+  p.lr = lr;
+  p.test_stall = test_stall ? 1 : 0;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  DevStatus* dst = nullptr;
+  cudaError_t e = cudaMalloc(reinterpret_cast<void**>(&dst), sizeof(DevStatus));
+  if (e != cudaSuccess) return cuda_fail(nullptr, e, "status word");
+  e = cudaMemsetAsync(dst, 0, sizeof(DevStatus), s);
+  p.st = dst;
+  if (e == cudaSuccess) e = hs::launch_tc_wgrad_avg(p, sms, s);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  DevStatus hst{};
+  if (e == cudaSuccess) e = cudaMemcpy(&hst, dst, sizeof(DevStatus), cudaMemcpyDeviceToHost);
+  cudaFree(dst);
+  if (e != cudaSuccess) return cuda_fail(nullptr, e, "weight-gradient average launch");
+  if (hst.err != hs::kDevOk) {
+    char buf[128];
+    std::snprintf(buf, sizeof(buf), "device check failed in the weight-gradient average: code %d, detail %d", hst.err,
+                  hst.err_info);
+    return fail(nullptr, HS_ERR_DEVICE_CHECK, buf);
+  }
+  return HS_OK;
+}
+
 }  // extern "C"

@@ -157,3 +157,58 @@ def test_default_takes_the_tile_launch_where_a_layer_fills_the_pairs():
         ctx.close()
     b, _ = _run(dims, M, N, (1.0, 2.0, 3.0, 4.0), hs.HS_SYNC_CP_WEIGHTED, False, 2, 0.05, x, y, theta0)
     assert torch.equal(p.cpu(), b)
+
+
+def _bf(r, c, g):
+    """bf16 [r, c] view of a [r, c rounded up to 8] buffer (16-byte rows), and its fp64 copy."""
+    t = (torch.randn(r, (c + 7) // 8 * 8, generator=g, device="cuda") * 0.5).to(torch.bfloat16)[:, :c]
+    return t, t.double()
+
+
+@pytest.mark.parametrize("M,N,groups", [(256, 256, [64]), (300, 520, [1, 63, 64, 65, 200]),
+                                        (1000, 512, [242, 2410, 316]), (264, 136, [7] * 32),
+                                        (512, 768, [1024, 16, 17, 900])])
+def test_kernel_alone_matches_plain_reference(M, N, groups):
+    """The kernel through its test hook: theta - lr * sum_g w_g A_g^T B_g against fp64 products of
+    the same bf16 operands, over ragged groups (1 row, 63/64/65 rows, 32 groups) and partial
+    tiles; the bf16 copy is the rounding of the new theta."""
+    g = torch.Generator(device="cuda").manual_seed(M * 7 + N + len(groups))
+    K = sum(groups)
+    ko = [0]
+    for n in groups:
+        ko.append(ko[-1] + n)
+    A, a = _bf(K, M, g)
+    B, b = _bf(K, N, g)
+    w = torch.rand(len(groups), generator=g, device="cuda") + 0.5
+    theta = torch.randn(M, N, generator=g, device="cuda")
+    t0 = theta.double().clone()
+    shadow = torch.empty(M, N, device="cuda", dtype=torch.bfloat16)
+    lr = 0.03
+    hs.hs_debug_wgrad_avg(A, B, ko, w, lr, theta, shadow)
+    torch.cuda.synchronize()
+    gsum = torch.zeros(M, N, device="cuda", dtype=torch.float64)
+    for gi in range(len(groups)):
+        gsum += float(w[gi]) * (a[ko[gi]:ko[gi + 1]].t() @ b[ko[gi]:ko[gi + 1]])
+    ref = t0 - lr * gsum
+    d = theta.double() - t0
+    assert float((d - (ref - t0)).norm() / (ref - t0).norm()) < 1e-5
+    assert torch.equal(shadow, theta.to(torch.bfloat16))
+
+
+def test_kernel_alone_bounded_wait_reports_and_leaves_theta():
+    """Failure detection without a GPU fault: the kernel's loads are withheld, its bounded waits
+    expire, the call reports HS_ERR_DEVICE_CHECK, theta is unchanged and the next call works."""
+    g = torch.Generator(device="cuda").manual_seed(3)
+    A, _ = _bf(128, 256, g)
+    B, _ = _bf(128, 256, g)
+    w = torch.ones(2, device="cuda")
+    theta = torch.randn(256, 256, generator=g, device="cuda")
+    before = theta.clone()
+    shadow = torch.empty(256, 256, device="cuda", dtype=torch.bfloat16)
+    with pytest.raises(hs.HsError) as e:
+        hs.hs_debug_wgrad_avg(A, B, [0, 64, 128], w, 0.1, theta, shadow, test_stall=True)
+    assert e.value.status == hs.HS_ERR_DEVICE_CHECK
+    assert torch.equal(theta, before)
+    hs.hs_debug_wgrad_avg(A, B, [0, 64, 128], w, 0.1, theta, shadow)
+    torch.cuda.synchronize()
+    assert not torch.equal(theta, before)
