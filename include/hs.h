@@ -19,8 +19,9 @@
  * sum_m w_m G_m.  On the bf16 MLP step each tile of a layer's weight gradient
  * G_m is formed in tensor memory and folded into the weighted sum there, in
  * worker order, by the kernel that also applies the update; bias gradients (and
- * every range on the slab path: debug read-back, the momentum recipe, more than
- * 32 workers, the fp32 check path, the CNN) go through per-worker fp32 slabs in
+ * every range on the slab path: debug read-back, more than 32 workers, layers
+ * with fewer 256 x 256 weight tiles than SM pairs, the slab-free variant, the
+ * fp32 check path, the CNN) go through per-worker fp32 slabs in
  * device memory and one reduce-and-update pass.  Both forms give the same bits.
  *
  * Conventions for every entry point:

@@ -173,6 +173,7 @@ struct hs_ctx {
   std::vector<hs::TcGemmParams> tc_wgrad_avg;
   std::vector<char> avg_ok;
   const float* avg_theta = nullptr;
+  bool avg_recipe = false;     // the maps are bound for the momentum recipe's update
   bool tile_step = false;   // the last step used it for some layer (its slabs lack those weight ranges)
   std::vector<hs::TcGemmParams> tc_fwd;                // per layer
   std::vector<hs::TcGemmParams> tc_dgrad;              // per layer (index 0 unused)

@@ -97,6 +97,10 @@ __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatil
   return ok != 0;
 }
 
+// RECIPE: the update of the paper's experiments (Section 5): d = g + wd * theta, b = d (first step)
+// or mu * b + d, theta <- theta - lr * b, with b read and written through tmM; theta, b and the
+// bf16 copy then move in 16-column boxes (two fp32 boxes share the warp's 4 KB buffer).
+template <bool RECIPE>
 __global__ void __launch_bounds__(kAvThreads, 1) tc_wgrad_avg_pair_kernel(const __grid_constant__ TcGemmParams p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -271,10 +275,14 @@ __global__ void __launch_bounds__(kAvThreads, 1) tc_wgrad_avg_pair_kernel(const 
 #pragma unroll 1
       for (int g = 0; g < G; ++g) {
         if (g == G - 1 && lane == 0 && rows_live) {
-          // theta's block into L2 while the last group runs
+          // theta's block (and the momentum's) into L2 while the last group runs
+          constexpr int kBox = RECIPE ? 16 : 32;
 #pragma unroll
-          for (int u = 0; u < AV_HN / 32; ++u)
-            if (col0 + 32 * u < p.n_store) tma_prefetch_l2_2d(&p.tmT, col0 + 32 * u, row0);
+          for (int u = 0; u < AV_HN / kBox; ++u) {
+            if (col0 + kBox * u >= p.n_store) break;
+            tma_prefetch_l2_2d(&p.tmT, col0 + kBox * u, row0);
+            if (RECIPE && !p.first) tma_prefetch_l2_2d(&p.tmM, col0 + kBox * u, row0);
+          }
         }
         if (!warp_wait(smem_u32(&tfull_bar[ab]), aph, abort_flag, lane)) {
           if (lane == 0) {
@@ -301,6 +309,77 @@ __global__ void __launch_bounds__(kAvThreads, 1) tc_wgrad_avg_pair_kernel(const 
         if (++ab == 2) { ab = 0; aph ^= 1u; }
       }
       if (!ok || !rows_live) continue;
+      if (RECIPE) {
+        // d = sum + wd * theta, b = d or mu * b + d, theta <- theta - lr * b: 16 columns at a time,
+        // theta's 32 x 16 box at buf, the momentum's at buf + 2 KB (64-byte rows, no swizzle), then
+        // the bf16 copy (32-byte rows) through the same buffer
+        const float mu = p.mu, wd = p.wd;
+        const bool first = p.first != 0;
+#pragma unroll
+        for (int u = 0; u < AV_HN / 16; ++u) {
+          const int n_base = col0 + 16 * u;
+          if (n_base >= p.n_store) break;
+          if (lane == 0) {
+            bulk_wait_read_0();
+            mbar_expect_tx(tbar, first ? AV_BUF / 2 : AV_BUF);
+            tma_load_2d(buf, &p.tmT, n_base, row0, tbar);
+            if (!first) tma_load_2d(buf + AV_BUF / 2, &p.tmM, n_base, row0, tbar);
+          }
+          if (!warp_wait(tbar, tph, abort_flag, lane)) {
+            if (lane == 0) {
+              record_error(p.st, kDevWaitTimeout, 25);
+              *abort_flag = 1;
+            }
+            ok = false;
+            break;
+          }
+          tph ^= 1u;
+          const uint32_t ta = buf + (uint32_t)(lane * 64);
+          const uint32_t ma = ta + AV_BUF / 2;
+          uint32_t sh[8];
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            const uint4 tv = ld_shared_v4(ta + 16u * j);
+            const uint4 bv = first ? make_uint4(0u, 0u, 0u, 0u) : ld_shared_v4(ma + 16u * j);
+            const float tin[4] = {__uint_as_float(tv.x), __uint_as_float(tv.y), __uint_as_float(tv.z),
+                                  __uint_as_float(tv.w)};
+            const float bin[4] = {__uint_as_float(bv.x), __uint_as_float(bv.y), __uint_as_float(bv.z),
+                                  __uint_as_float(bv.w)};
+            float tout[4], bout[4];
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+              const float d = fmaf(wd, tin[k], sum[u * 16 + 4 * j + k]);
+              bout[k] = first ? d : fmaf(mu, bin[k], d);
+              tout[k] = fmaf(neg_lr, bout[k], tin[k]);
+            }
+            st_shared_v4(ta + 16u * j, make_uint4(__float_as_uint(tout[0]), __float_as_uint(tout[1]),
+                                                  __float_as_uint(tout[2]), __float_as_uint(tout[3])));
+            st_shared_v4(ma + 16u * j, make_uint4(__float_as_uint(bout[0]), __float_as_uint(bout[1]),
+                                                  __float_as_uint(bout[2]), __float_as_uint(bout[3])));
+            sh[2 * j] = pack_bf16(tout[0], tout[1]);
+            sh[2 * j + 1] = pack_bf16(tout[2], tout[3]);
+          }
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) {
+            tma_store_2d(&p.tmT, buf, n_base, row0);
+            tma_store_2d(&p.tmM, buf + AV_BUF / 2, n_base, row0);
+            bulk_commit();
+            bulk_wait_read_0();
+          }
+          __syncwarp();
+          const uint32_t sbase = buf + (uint32_t)(lane * 32);
+          st_shared_v4(sbase, make_uint4(sh[0], sh[1], sh[2], sh[3]));
+          st_shared_v4(sbase + 16u, make_uint4(sh[4], sh[5], sh[6], sh[7]));
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) {
+            tma_store_2d(&p.tmS, buf, n_base, row0);
+            bulk_commit();
+          }
+        }
+        continue;
+      }
       // theta <- fma(-lr, sum, theta), 32 columns at a time through the warp's buffer (128-byte
       // swizzle: 16-byte chunk j of row r sits at chunk j ^ (r % 8)), then the same 32 columns of
       // the bf16 copy (64-byte rows, no swizzle).
@@ -376,15 +455,12 @@ __global__ void __launch_bounds__(kAvThreads, 1) tc_wgrad_avg_pair_kernel(const 
 
 }  // namespace
 
-cudaError_t launch_tc_wgrad_avg(const TcGemmParams& p, int num_sms, cudaStream_t s) {
-  if (p.groups < 1 || p.groups > kTcMaxGroups || !p.a_mn || !p.b_mn || !p.wavg) return cudaErrorInvalidValue;
-  for (int g = 0; g < p.groups; ++g)
-    if (p.num_kb[g] < 1) return cudaErrorInvalidValue;
-  const int total = ((p.Mdim + AV_PM - 1) / AV_PM) * ((p.n_store + AV_PN - 1) / AV_PN);
-  if (total <= 0) return cudaSuccess;
+namespace {
+template <bool RECIPE>
+cudaError_t launch_avg_variant(const TcGemmParams& p, int total, int num_sms, cudaStream_t s) {
   static bool configured = false;
   static int max_clusters = 0;
-  auto kern = tc_wgrad_avg_pair_kernel;
+  auto kern = tc_wgrad_avg_pair_kernel<RECIPE>;
   cudaLaunchConfig_t cfg = {};
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -414,6 +490,16 @@ cudaError_t launch_tc_wgrad_avg(const TcGemmParams& p, int num_sms, cudaStream_t
   cudaError_t e = cudaLaunchKernelEx(&cfg, kern, p);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
+}
+}  // namespace
+
+cudaError_t launch_tc_wgrad_avg(const TcGemmParams& p, int num_sms, cudaStream_t s) {
+  if (p.groups < 1 || p.groups > kTcMaxGroups || !p.a_mn || !p.b_mn || !p.wavg) return cudaErrorInvalidValue;
+  for (int g = 0; g < p.groups; ++g)
+    if (p.num_kb[g] < 1) return cudaErrorInvalidValue;
+  const int total = ((p.Mdim + AV_PM - 1) / AV_PM) * ((p.n_store + AV_PN - 1) / AV_PN);
+  if (total <= 0) return cudaSuccess;
+  return p.recipe ? launch_avg_variant<true>(p, total, num_sms, s) : launch_avg_variant<false>(p, total, num_sms, s);
 }
 
 }  // namespace hs

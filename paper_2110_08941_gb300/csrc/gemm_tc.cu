@@ -444,6 +444,12 @@ bool tc_make_store_map_bf16_32(CUtensorMap* tm, void* base, int64_t rows, int64_
                    CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, CU_TENSOR_MAP_SWIZZLE_NONE);
 }
 
+bool tc_make_store_map_16(CUtensorMap* tm, void* base, bool fp32, int64_t rows, int64_t cols, int64_t ld,
+                          const char** why) {
+  return encode_2d(tm, base, (uint64_t)cols, (uint64_t)rows, (uint64_t)ld * (fp32 ? 4 : 2), 16, 32, why,
+                   fp32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, CU_TENSOR_MAP_SWIZZLE_NONE);
+}
+
 namespace {
 // Default form (SM pairs); HS_TC_FORM=single|pair in the environment overrides it at load time.
 int initial_form() {

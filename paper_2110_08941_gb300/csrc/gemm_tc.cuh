@@ -72,6 +72,12 @@ struct TcGemmParams {
   CUtensorMap tmS;                 // bf16 copy of those weights, written beside theta (tc_make_store_map_bf16_32)
   const float* wavg;               // [groups] averaging weight of group (worker) g, on the device
   float lr;
+  // recipe = 1: momentum mu and weight decay wd in the update, the momentum buffer through tmM
+  // (first = 1: it starts as d); tmT, tmM and tmS then have 32-row x 16-column boxes
+  // (tc_make_store_map_16)
+  CUtensorMap tmM;
+  int32_t recipe, first;
+  float mu, wd;
   int32_t ksplit;                  // >= 2: each group's k-blocks split into ksplit contiguous parts, part j
                                    // a tile of its own writing part j of tmD[g], a 3-D map [parts][rows][cols]
                                    // (needs num_kb[g] >= ksplit); 0 or 1: no split
@@ -123,6 +129,10 @@ bool tc_make_store_map(CUtensorMap* tm, void* base, bool fp32, int64_t rows, int
 // box at byte 64 * r of the staging buffer).
 bool tc_make_store_map_bf16_32(CUtensorMap* tm, void* base, int64_t rows, int64_t cols, int64_t ld,
                                const char** why);
+// fp32 or bf16 matrix for TMA loads and stores of 32-row x 16-column boxes, unswizzled (row r of a
+// box at byte 64 * r, fp32, or 32 * r, bf16, of the staging buffer).
+bool tc_make_store_map_16(CUtensorMap* tm, void* base, bool fp32, int64_t rows, int64_t cols, int64_t ld,
+                          const char** why);
 // The same over `parts` such matrices `part_stride` elements apart (split-K partials, fp32).
 bool tc_make_store_map_parts(CUtensorMap* tm, float* base, int64_t rows, int64_t cols, int64_t ld, int64_t parts,
                              int64_t part_stride, const char** why);

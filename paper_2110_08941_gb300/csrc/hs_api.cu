@@ -226,8 +226,7 @@ hs_status build_tc_wgrad_avg(hs_ctx* c) {
       w.num_kb[m] = (int32_t)((n + hs::kTcBK - 1) / hs::kTcBK);
       w.last_ksteps[m] = last_ksteps(n);
     }
-    __nv_bfloat16* shadow = (l > 0 ? c->d_shadow_next : c->d_shadow) + ly.w_off;
-    ok = ok && shadow && hs::tc_make_store_map_bf16_32(&w.tmS, shadow, out_cols, ly.in, ly.in, &why);
+    ok = ok && c->d_shadow_next && c->d_shadow;
     // One SM pair per 256 x 256 tile of the layer's weights: with fewer tiles than pairs the
     // grouped slab launch (a tile per worker) keeps more of the GPU busy.
     const int64_t tiles = ((out_cols + 255) / 256) * (int64_t)((ly.in + 255) / 256);
@@ -246,18 +245,31 @@ hs_status build_tc_wgrad_avg(hs_ctx* c) {
   return HS_OK;
 }
 
-// Point the tile-averaged launches' theta maps at `params` (a layer whose weights TMA cannot
-// address, e.g. not 16-byte aligned, falls back to the slab path).
+// Point the tile-averaged launches' update maps at `params`, the bf16 copies and (with the
+// momentum recipe) the momentum buffer, in the box shapes of the update in use (a layer whose
+// weights TMA cannot address, e.g. not 16-byte aligned, falls back to the slab path).
 void bind_avg_theta(hs_ctx* c, float* params) {
-  if (c->avg_theta == params) return;
+  const bool recipe = c->opt_recipe && c->d_mom;
+  if (c->avg_theta == params && c->avg_recipe == recipe) return;
   const char* why = nullptr;
   for (int l = 0; l < c->L; ++l) {
     if (!c->avg_ok[l]) continue;
     const Layer& ly = c->layers[l];
     hs::TcGemmParams& w = c->tc_wgrad_avg[l];
-    if (!hs::tc_make_store_map(&w.tmT, params + ly.w_off, true, w.Mdim, ly.in, ly.in, &why)) c->avg_ok[l] = 0;
+    __nv_bfloat16* shadow = (l > 0 ? c->d_shadow_next : c->d_shadow) + ly.w_off;
+    bool ok;
+    if (recipe)
+      ok = hs::tc_make_store_map_16(&w.tmT, params + ly.w_off, true, w.Mdim, ly.in, ly.in, &why) &&
+           hs::tc_make_store_map_16(&w.tmM, c->d_mom + ly.w_off, true, w.Mdim, ly.in, ly.in, &why) &&
+           hs::tc_make_store_map_16(&w.tmS, shadow, false, w.Mdim, ly.in, ly.in, &why);
+    else
+      ok = hs::tc_make_store_map(&w.tmT, params + ly.w_off, true, w.Mdim, ly.in, ly.in, &why) &&
+           hs::tc_make_store_map_bf16_32(&w.tmS, shadow, w.Mdim, ly.in, ly.in, &why);
+    if (!ok) c->avg_ok[l] = 0;
+    w.recipe = recipe ? 1 : 0;
   }
   c->avg_theta = params;
+  c->avg_recipe = recipe;
 }
 
 void compute_weights(hs_ctx* c) {
@@ -493,12 +505,15 @@ void update_layer_range(hs_ctx* c, float* params, int l, float lr, cudaStream_t 
 }
 
 // theta <- theta - lr * sum_m w_m G_m over [start, end) of the slabs (the bias range of a layer whose
-// weights the tile-averaged launch updated), bf16 copy into `shadow`.
+// weights the tile-averaged launch updated; the momentum recipe as in the rest of the update),
+// bf16 copy into `shadow`.
 void update_range(hs_ctx* c, float* params, int64_t start, int64_t end, float lr, cudaStream_t s,
                   __nv_bfloat16* shadow) {
   PhaseScope ph(c, HS_PHASE_UPDATE, s);
+  hs::UpdateRecipe r{c->opt_recipe ? c->d_mom + start : nullptr, c->opt_momentum, c->opt_weight_decay,
+                     c->mom_valid ? 0 : 1};
   hs::launch_reduce_update(params + start, c->d_slabs + start, c->Ps, c->M, c->d_w, lr, end - start, shadow + start,
-                           nullptr, c->num_sms, s, 1, nullptr);
+                           nullptr, c->num_sms, s, 1, c->opt_recipe ? &r : nullptr);
   ph.launched();
 }
 
@@ -530,7 +545,7 @@ hs_status mlp_step_bf16(hs_ctx* c, float* params, const float* x, const int32_t*
   // Per-worker weight gradients averaged tile by tile in tensor memory, the update fused in: the
   // default where the layer's operands allow it; debug read-back, the slab-free formulation and
   // the momentum recipe take the slab path.
-  const bool avg = c->tile_avg && !c->fused_sync && !c->debug && !c->opt_recipe;
+  const bool avg = c->tile_avg && !c->fused_sync && !c->debug;
   if (avg) bind_avg_theta(c, params);
   c->tile_step = false;
   for (int l = 0; l < L && avg; ++l) c->tile_step = c->tile_step || c->avg_ok[l];
@@ -544,6 +559,9 @@ hs_status mlp_step_bf16(hs_ctx* c, float* params, const float* x, const int32_t*
       if (tile) {
         hs::TcGemmParams& w = c->tc_wgrad_avg[l];
         w.lr = lr;
+        w.mu = c->opt_momentum;
+        w.wd = c->opt_weight_decay;
+        w.first = c->mom_valid ? 0 : 1;
         cudaError_t e = hs::launch_tc_wgrad_avg(w, c->num_sms, s);
         if (e != cudaSuccess) return cuda_fail(c, e, "weight-gradient GEMM launch");
         ph.launched();

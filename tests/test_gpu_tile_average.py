@@ -28,9 +28,11 @@ def _init(dims, M, N, weights, sync, tile):
             os.environ["HS_TILE_AVERAGE"] = old
 
 
-def _run(dims, M, N, weights, sync, tile, steps, lr, x, y, theta0, repartition=None):
+def _run(dims, M, N, weights, sync, tile, steps, lr, x, y, theta0, repartition=None, recipe=None):
     ctx = _init(dims, M, N, weights, sync, tile)
     try:
+        if recipe is not None:
+            hs.hs_set_optimizer(ctx, *recipe)
         p = torch.tensor(theta0, device="cuda")
         xd, yd = torch.from_numpy(x).cuda(), torch.from_numpy(y).cuda()
         losses = []
@@ -80,6 +82,37 @@ def test_tile_average_equals_slab_path(dims, N, M, weights, sync):
     assert torch.equal(a, b)
     assert la == lb
     assert not torch.equal(a, torch.from_numpy(theta0))
+
+
+@pytest.mark.parametrize("dims,N,M,weights", [((3072, 1024, 1024, 10), 1024, 4, (1.0, 1.0, 2.0, 4.0)),
+                                               ((264, 200, 136, 10), 300, 5, (1.0, 2.0, 3.0, 1.5, 0.7))])
+def test_tile_average_with_momentum_equals_slab_path(dims, N, M, weights):
+    """The experiments' optimiser (Section 5: momentum 0.9, weight decay 5e-4) in the tile kernel's
+    epilogue: the momentum buffer starts as d on the first step and both forms agree bit for bit."""
+    x, y, theta0 = _data(dims, N, seed=13)
+    rep = {3: tuple(reversed(weights))}
+    a, la = _run(dims, M, N, weights, hs.HS_SYNC_CP_WEIGHTED, True, 5, 0.05, x, y, theta0, rep, (0.9, 5e-4))
+    b, lb = _run(dims, M, N, weights, hs.HS_SYNC_CP_WEIGHTED, False, 5, 0.05, x, y, theta0, rep, (0.9, 5e-4))
+    assert torch.equal(a, b)
+    assert la == lb
+
+
+def test_tile_average_momentum_matches_oracle(monkeypatch):
+    """Momentum 0.9, weight decay 5e-4 and a cosine learning rate over 10 steps through the tile
+    kernel (no debug read-back), against the oracle's recipe."""
+    monkeypatch.setenv("HS_TILE_AVERAGE", "all")
+    wl = synth.WORKLOADS[synth.CFG2]
+    x, y = synth.make_batch(wl)
+    theta0 = synth.make_params(wl)
+    weights = synth.initial_weights(wl)
+    recipe = (0.9, 5e-4)
+    sched = lambda t: hs.hs_cosine_lr(wl.lr, 0.0, t, 10)   # noqa: E731
+    lib = run_library(wl.arch, wl.dims, wl.workers, wl.global_batch, weights, x, y, theta0, sched, 10,
+                      hs.HS_BF16, hs.HS_SYNC_CP_WEIGHTED, recipe=recipe, debug=False)
+    orc = run_oracle(wl.arch, wl.dims, wl.workers, wl.global_batch, weights, x, y, theta0, sched, 10,
+                     hs.HS_SYNC_CP_WEIGHTED, decide=decide_for(hs.HS_BF16), recipe=recipe)
+    assert rel(lib["theta"], orc["theta"]) <= 2e-2
+    assert rel(lib["theta"] - theta0, orc["theta"] - theta0) <= 5e-2
 
 
 @pytest.mark.parametrize("name", [synth.CFG2, synth.CFG3])
