@@ -1,12 +1,14 @@
 /*
- * hs_debug.h - test hook into libhs's tensor-core GEMM.
+ * hs_debug.h - test hooks into libhs's tensor-core kernels.
  *
- * Not part of the training API.  It runs one product through the same
- * tcgen05/TMA kernel that hs_step uses for the per-worker forward and backward
- * passes (Eq. 1's per-worker gradients g^m, Section 1), so tests can check that
- * kernel in isolation against a plain reference.  All matrix pointers are
- * device pointers, row-major, with leading dimensions in elements; the call is
- * synchronous (it waits for the kernel and reports launch/runtime errors).
+ * Not part of the training API.  hs_debug_gemm_bf16 runs one product through
+ * the same tcgen05/TMA kernel that hs_step uses for the per-worker forward and
+ * backward passes (Eq. 1's per-worker gradients g^m, Section 1);
+ * hs_debug_wgrad_avg runs the kernel that forms the per-worker weight gradients
+ * of a layer, averages them and applies the update.  Tests check each kernel in
+ * isolation against a plain reference.  All matrix pointers are device
+ * pointers, row-major, with leading dimensions in elements; the calls are
+ * synchronous (they wait for the kernel and report launch/runtime errors).
  */
 #ifndef HS_DEBUG_H_
 #define HS_DEBUG_H_
