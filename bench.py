@@ -392,6 +392,10 @@ def run_ours(args, wl, rank, world, local_rank):
     for _ in range(args.warmup):
         hs.hs_step(ctx, params, xd, yd, part, wl.lr, stream=stream, want_loss=False)
     torch.cuda.synchronize()
+    hs.hs_read_profile(ctx)                 # discard warm-up counts
+    # CUDA events around every phase of the timed steps, on the step's stream: the live kernel
+    # times behind the roofline (a few microseconds of event records per step)
+    hs.hs_set_profiling(ctx, True)
 
     clocks = ClockSampler(local_rank)
     clocks.start()
@@ -410,13 +414,6 @@ def run_ours(args, wl, rank, world, local_rank):
     ms = ev[0].elapsed_time(ev[-1])
     step_ms = np.asarray([ev[i].elapsed_time(ev[i + 1]) for i in range(args.steps)])
     ms = max_over_ranks(ms)
-    # the phase split (and the launch count) from the same number of steps run again with CUDA
-    # events around every phase; the timed steps above run without them
-    hs.hs_read_profile(ctx)                 # discard warm-up counts
-    hs.hs_set_profiling(ctx, True)
-    for _ in range(args.steps):
-        hs.hs_step(ctx, params, xd, yd, part, wl.lr, stream=stream, want_loss=False)
-    torch.cuda.synchronize()
     prof = hs.hs_read_profile(ctx)
     hs.hs_set_profiling(ctx, False)
     loss = hs.hs_step(ctx, params, xd, yd, part, 0.0, stream=stream, want_loss=True)   # finite-loss check
