@@ -122,7 +122,18 @@ hs_status hs_param_count(const hs_model_desc* model, int64_t* P);
  * rows, the bf16 parameter shadow) and computes the initial partition
  * synchronously.  Errors: HS_ERR_INVALID_ARG (bad model/M/N/weights),
  * HS_ERR_UNSUPPORTED (shape constraint of the precision), HS_ERR_OOM,
- * HS_ERR_CUDA.  On error *out is NULL. */
+ * HS_ERR_CUDA.  On error *out is NULL.
+ * Read here from the environment (all give the same results; they select how):
+ *   HS_TILE_AVERAGE=0    bf16 MLP: every layer's weight gradients through the
+ *                        per-worker slabs (default: averaged in tensor memory
+ *                        where a layer has a 256 x 256 weight tile per SM
+ *                        pair); =all: averaged in tensor memory on every layer
+ *   HS_OVERLAP_UPDATE=0  slab-path updates on the step's stream, not beside the
+ *                        remaining products
+ *   HS_CONV_IMPLICIT=0|fwd  bf16 CNN: materialised patch rows everywhere, or
+ *                        for the input gradients only
+ *   HS_TC_FORM=single    one-SM tensor-core tiles instead of SM pairs (read
+ *                        when the library loads) */
 hs_status hs_init(const hs_model_desc* model, int32_t M, const double* compute_weights,
                   int32_t global_batch, hs_ctx** out);
 
