@@ -144,6 +144,8 @@ __global__ void __launch_bounds__(kAvThreads, 1) tc_wgrad_avg_pair_kernel(const 
   cluster_sync();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  grid_dependency_wait();
+  grid_dependents_launch();
 
   const int tiles_m = (p.Mdim + AV_PM - 1) / AV_PM;
   const int tiles_n = (p.n_store + AV_PN - 1) / AV_PN;
@@ -462,16 +464,18 @@ cudaError_t launch_avg_variant(const TcGemmParams& p, int total, int num_sms, cu
   static int max_clusters = 0;
   auto kern = tc_wgrad_avg_pair_kernel<RECIPE>;
   cudaLaunchConfig_t cfg = {};
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = 2;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;   // see grid_dependency_wait
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.blockDim = dim3(kAvThreads, 1, 1);
   cfg.dynamicSmemBytes = kAvSmem;
   cfg.stream = s;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 1;   // the occupancy query takes the cluster shape only
   if (!configured) {
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kAvSmem);
     if (e != cudaSuccess) return e;
@@ -487,6 +491,7 @@ cudaError_t launch_avg_variant(const TcGemmParams& p, int total, int num_sms, cu
   }
   const int pairs = total < max_clusters ? total : max_clusters;
   cfg.gridDim = dim3(2 * (pairs < 1 ? 1 : pairs), 1, 1);
+  cfg.numAttrs = 2;
   cudaError_t e = cudaLaunchKernelEx(&cfg, kern, p);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();

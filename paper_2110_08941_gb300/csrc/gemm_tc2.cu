@@ -90,6 +90,8 @@ __global__ void __launch_bounds__(PairCfg<TN, EW>::kThreads, 1)
   cluster_sync();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  grid_dependency_wait();
+  grid_dependents_launch();
 
   const int tiles_m = (p.Mdim + PM - 1) / PM;
   const int tiles_n = (p.n_store + PN - 1) / PN;
@@ -314,16 +316,18 @@ cudaError_t launch_pair_variant(const TcGemmParams& p, int pairs_wanted, int num
   constexpr int kSmem2 = PairCfg<TN, EW>::kSmem2;
   auto kern = tc_gemm_pair_kernel<EPI, A_MN, B_MN, CONV, TN, EW>;
   cudaLaunchConfig_t cfg = {};
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = 2;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;   // see grid_dependency_wait
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.blockDim = dim3(PairCfg<TN, EW>::kThreads, 1, 1);
   cfg.dynamicSmemBytes = kSmem2;
   cfg.stream = s;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 1;   // the occupancy query takes the cluster shape only
   if (!configured) {
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmem2);
     if (e != cudaSuccess) return e;
@@ -342,6 +346,7 @@ cudaError_t launch_pair_variant(const TcGemmParams& p, int pairs_wanted, int num
   if (pairs < 1) pairs = 1;
   const int grid = 2 * pairs;
   cfg.gridDim = dim3(grid, 1, 1);
+  cfg.numAttrs = 2;
   cudaError_t e = cudaLaunchKernelEx(&cfg, kern, p);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();

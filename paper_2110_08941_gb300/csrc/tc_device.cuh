@@ -144,6 +144,15 @@ __device__ __forceinline__ void st_shared_v4(uint32_t addr, uint4 v) {
   asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w)
                : "memory");
 }
+// Programmatic dependent launch.  The GEMM kernels are launched with programmatic stream
+// serialisation, so they may start while the previous kernel of the stream is finishing: each
+// waits here, after its prologue (barriers, tensor memory, cluster sync) and before its first
+// global-memory access, until that kernel has completed and its writes are visible; then it lets
+// the next kernel of the stream start its own prologue on SMs as they free up.
+__device__ __forceinline__ void grid_dependency_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void grid_dependents_launch() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
 __device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap* tm) {
   asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(tm)) : "memory");
 }
