@@ -47,6 +47,8 @@ __device__ __forceinline__ int patch_col(int ci, int tap, int C) {
 template <typename T, bool kTapMajor>
 __global__ void im2col_nchw_kernel(const float* __restrict__ x, int N, int C, int H, int W, int Ho, int Wo, int s,
                                    T* __restrict__ col, int Kp) {
+  pdl_wait();
+  pdl_trigger();
   const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   const int64_t rows = (int64_t)N * Ho * Wo;
   if (idx >= rows * C) return;
@@ -77,6 +79,8 @@ __global__ void im2col_nchw_kernel(const float* __restrict__ x, int N, int C, in
 template <int KP>
 __global__ void im2col_nchw_row_kernel(const float* __restrict__ x, int N, int C, int H, int W, int Ho, int Wo,
                                        int s, __nv_bfloat16* __restrict__ col) {
+  pdl_wait();
+  pdl_trigger();
   const int64_t r = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (r >= (int64_t)N * Ho * Wo) return;
   const int wo = (int)(r % Wo);
@@ -114,6 +118,8 @@ __global__ void im2col_nchw_row_kernel(const float* __restrict__ x, int N, int C
 // yields the bias gradient, sum over the worker's rows of dA.
 __global__ void im2col_nhwc_vec8_kernel(const __nv_bfloat16* __restrict__ h, int N, int C, int H, int W, int Ho,
                                         int Wo, int s, __nv_bfloat16* __restrict__ col, int Kp) {
+  pdl_wait();
+  pdl_trigger();
   const int C8 = C >> 3;
   const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   const int64_t rows = (int64_t)N * Ho * Wo;
@@ -138,6 +144,8 @@ __global__ void im2col_nhwc_vec8_kernel(const __nv_bfloat16* __restrict__ h, int
 __global__ void col2im_nhwc_vec4_kernel(const float* __restrict__ dcol, int ldc, const __nv_bfloat16* __restrict__ h,
                                         int N, int C, int H, int W, int Ho, int Wo, int s,
                                         __nv_bfloat16* __restrict__ dA) {
+  pdl_wait();
+  pdl_trigger();
   const int C4 = C >> 2;
   const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (idx >= (int64_t)N * H * W * C4) return;
@@ -182,6 +190,8 @@ __global__ void col2im_nhwc_vec4_kernel(const float* __restrict__ dcol, int ldc,
 // fp32 check path: patch rows from an NHWC activation h[n][hi][wi][ci], channel-major columns.
 __global__ void im2col_nhwc_f32_kernel(const float* __restrict__ h, int N, int C, int H, int W, int Ho, int Wo, int s,
                                        float* __restrict__ col, int Kp) {
+  pdl_wait();
+  pdl_trigger();
   const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   const int64_t rows = (int64_t)N * Ho * Wo;
   if (idx >= rows * C) return;
@@ -206,6 +216,8 @@ __global__ void im2col_nhwc_f32_kernel(const float* __restrict__ h, int N, int C
 // pooled[n][c] = mean over the HW rows of sample n (global average pooling).
 template <typename T>
 __global__ void gap_forward_kernel(const T* __restrict__ h, int N, int HW, int C, T* __restrict__ pooled) {
+  pdl_wait();
+  pdl_trigger();
   const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (idx >= (int64_t)N * C) return;
   const int c = (int)(idx % C);
@@ -219,6 +231,8 @@ __global__ void gap_forward_kernel(const T* __restrict__ h, int N, int HW, int C
 // The same for bf16 activations, eight channels per thread (16-byte loads and stores; C % 8 == 0).
 __global__ void gap_backward_vec8_kernel(const float* __restrict__ dpooled, const __nv_bfloat16* __restrict__ h,
                                          int N, int HW, int C, __nv_bfloat16* __restrict__ dA) {
+  pdl_wait();
+  pdl_trigger();
   const int C8 = C >> 3;
   const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (idx >= (int64_t)N * HW * C8) return;
@@ -243,6 +257,8 @@ __global__ void gap_backward_vec8_kernel(const float* __restrict__ dpooled, cons
 template <typename T>
 __global__ void gap_backward_kernel(const float* __restrict__ dpooled, const T* __restrict__ h, int N, int HW, int C,
                                     T* __restrict__ dA) {
+  pdl_wait();
+  pdl_trigger();
   const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (idx >= (int64_t)N * HW * C) return;
   const int c = (int)(idx % C);
@@ -255,6 +271,8 @@ __global__ void gap_backward_kernel(const float* __restrict__ dpooled, const T* 
 // sums the patch entries that read it), then ReLU' of that input: dA[n][hi][wi][ci].
 __global__ void col2im_nhwc_f32_kernel(const float* __restrict__ dcol, int ldc, const float* __restrict__ h, int N,
                                        int C, int H, int W, int Ho, int Wo, int s, float* __restrict__ dA) {
+  pdl_wait();
+  pdl_trigger();
   const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (idx >= (int64_t)N * H * W * C) return;
   const int ci = (int)(idx % C);
@@ -284,6 +302,8 @@ __global__ void col2im_nhwc_f32_kernel(const float* __restrict__ dcol, int ldc, 
 // wp[co][tap*Cin + ci] = bf16(w[co][ci][tap]), rows padded from 9*Cin to Kp with zeros.
 __global__ void permute_weights_kernel(const float* __restrict__ w, int cout, int cin, int Kp,
                                        __nv_bfloat16* __restrict__ wp) {
+  pdl_wait();
+  pdl_trigger();
   const int idx = blockIdx.x * blockDim.x + threadIdx.x;
   if (idx >= cout * Kp) return;
   const int k = idx % Kp, co = idx / Kp;
@@ -301,6 +321,8 @@ __global__ void permute_weights_kernel(const float* __restrict__ w, int cout, in
 // t = th * (number of column taps) + tw.  Classes hold 1, 2, 2, 4 taps and sit back to back.
 __global__ void permute_weights_subpixel_kernel(const float* __restrict__ w, int cout, int cin,
                                                 __nv_bfloat16* __restrict__ wc) {
+  pdl_wait();
+  pdl_trigger();
   const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (idx >= (int64_t)cout * cin * 9) return;
   const int tap = (int)(idx % 9);
@@ -323,6 +345,8 @@ __global__ void permute_weights_subpixel_kernel(const float* __restrict__ w, int
 __global__ void splitk_reduce_kernel(const float* __restrict__ partial, int rows, int K, int ldp,
                                      const int32_t* __restrict__ chunk_begin, float* __restrict__ slabs, int64_t Ps,
                                      int64_t w_off, int cin, int64_t b_off) {
+  pdl_wait();
+  pdl_trigger();
   const int m = blockIdx.y;
   const int cols = cin ? K + 1 : K;
   const int idx = blockIdx.x * blockDim.x + threadIdx.x;
@@ -346,13 +370,13 @@ void launch_im2col_first(const float* x, int N, const ConvLayer& L, __nv_bfloat1
   const int64_t rows = L.rows;
 #define HS_ROW_CASE(KP)                                                                                      \
   case KP:                                                                                                   \
-    im2col_nchw_row_kernel<KP><<<blocks_for(rows, T), T, 0, s>>>(x, N, L.cin, L.hin, L.win, L.hout, L.wout, \
+    launch_pdl(im2col_nchw_row_kernel<KP>, blocks_for(rows, T), T, 0, s, x, N, L.cin, L.hin, L.win, L.hout, L.wout, \
                                                                  L.stride, col);                           \
     return;
   switch (L.Kp) {
     HS_ROW_CASE(16) HS_ROW_CASE(24) HS_ROW_CASE(32) HS_ROW_CASE(40) HS_ROW_CASE(48) HS_ROW_CASE(56) HS_ROW_CASE(64)
     default:
-      im2col_nchw_kernel<__nv_bfloat16, true><<<blocks_for(rows * L.cin, T), T, 0, s>>>(
+      launch_pdl(im2col_nchw_kernel<__nv_bfloat16, true>, blocks_for(rows * L.cin, T), T, 0, s,
           x, N, L.cin, L.hin, L.win, L.hout, L.wout, L.stride, col, L.Kp);
   }
 #undef HS_ROW_CASE
@@ -610,11 +634,11 @@ hs_status cnn_step(hs_ctx* c, float* params, const float* x, const int32_t* y, c
     PhaseScope ph(c, HS_PHASE_CAST, s);
     if (bf16) {
       for (int k = 0; k < 3; ++k) {
-        permute_weights_kernel<<<blocks_for((int64_t)L[k].cout * L[k].Kp, T), T, 0, s>>>(
+        launch_pdl(permute_weights_kernel, blocks_for((int64_t)L[k].cout * L[k].Kp, T), T, 0, s,
             params + L[k].w_off, L[k].cout, L[k].cin, L[k].Kp, c->d_wperm[k]);
         ph.launched();
         if (L[k].subpixel) {
-          permute_weights_subpixel_kernel<<<blocks_for(9LL * L[k].cout * L[k].cin, T), T, 0, s>>>(
+          launch_pdl(permute_weights_subpixel_kernel, blocks_for(9LL * L[k].cout * L[k].cin, T), T, 0, s,
               params + L[k].w_off, L[k].cout, L[k].cin, c->d_wsub[k]);
           ph.launched();
         }
@@ -629,18 +653,18 @@ hs_status cnn_step(hs_ctx* c, float* params, const float* x, const int32_t* y, c
         if (bf16)
           launch_im2col_first(x, N, L[0], reinterpret_cast<__nv_bfloat16*>(c->d_col[0]), s);
         else
-          im2col_nchw_kernel<float, false><<<blocks_for(n_items, T), T, 0, s>>>(
+          launch_pdl(im2col_nchw_kernel<float, false>, blocks_for(n_items, T), T, 0, s,
               x, N, L[0].cin, L[0].hin, L[0].win, L[0].hout, L[0].wout, L[0].stride,
               reinterpret_cast<float*>(c->d_col[0]), L[0].Kp);
       } else if (L[k].implicit) {
         // the forward product reads the patch rows straight from d_cact[k - 1]
       } else {
         if (bf16)
-          im2col_nhwc_vec8_kernel<<<blocks_for(L[k].rows * 9 * (L[k].cin / 8), T), T, 0, s>>>(
+          launch_pdl(im2col_nhwc_vec8_kernel, blocks_for(L[k].rows * 9 * (L[k].cin / 8), T), T, 0, s,
               reinterpret_cast<const __nv_bfloat16*>(c->d_cact[k - 1]), N, L[k].cin, L[k].hin, L[k].win, L[k].hout,
               L[k].wout, L[k].stride, reinterpret_cast<__nv_bfloat16*>(c->d_col[k]), L[k].Kp);
         else
-          im2col_nhwc_f32_kernel<<<blocks_for(n_items, T), T, 0, s>>>(
+          launch_pdl(im2col_nhwc_f32_kernel, blocks_for(n_items, T), T, 0, s,
               reinterpret_cast<const float*>(c->d_cact[k - 1]), N, L[k].cin, L[k].hin, L[k].win, L[k].hout,
               L[k].wout, L[k].stride, reinterpret_cast<float*>(c->d_col[k]), L[k].Kp);
       }
@@ -662,10 +686,10 @@ hs_status cnn_step(hs_ctx* c, float* params, const float* x, const int32_t* y, c
       ph.launched();
     }
     if (bf16)
-      gap_forward_kernel<__nv_bfloat16><<<blocks_for((int64_t)N * c3, T), T, 0, s>>>(
+      launch_pdl(gap_forward_kernel<__nv_bfloat16>, blocks_for((int64_t)N * c3, T), T, 0, s,
           reinterpret_cast<const __nv_bfloat16*>(c->d_cact[2]), N, hw3, c3, reinterpret_cast<__nv_bfloat16*>(c->d_pooled));
     else
-      gap_forward_kernel<float><<<blocks_for((int64_t)N * c3, T), T, 0, s>>>(
+      launch_pdl(gap_forward_kernel<float>, blocks_for((int64_t)N * c3, T), T, 0, s,
           reinterpret_cast<const float*>(c->d_cact[2]), N, hw3, c3, reinterpret_cast<float*>(c->d_pooled));
     ph.launched();
     if (bf16) {
@@ -710,7 +734,7 @@ hs_status cnn_step(hs_ctx* c, float* params, const float* x, const int32_t* y, c
         }
         const int kw = fc ? wg.K : wg.K - 1;   // weight columns (the conv partials carry the bias column)
         dim3 grid2(blocks_for((int64_t)wg.rows_out * wg.K, T), c->M);
-        splitk_reduce_kernel<<<grid2, T, 0, s>>>(wg.d_partial, wg.rows_out, kw, wg.ldp, wg.d_chunk_begin, c->d_slabs,
+        launch_pdl(splitk_reduce_kernel, grid2, T, 0, s, wg.d_partial, wg.rows_out, kw, wg.ldp, wg.d_chunk_begin, c->d_slabs,
                                                  c->Ps, w_off, fc ? 0 : L[k].cin, b_off);
         ph.launched();
       } else {
@@ -759,11 +783,11 @@ hs_status cnn_step(hs_ctx* c, float* params, const float* x, const int32_t* y, c
         launch_gemm_f32(d, s);
       }
       if (bf16)
-        gap_backward_vec8_kernel<<<blocks_for((int64_t)N * hw3 * (c3 / 8), T), T, 0, s>>>(
+        launch_pdl(gap_backward_vec8_kernel, blocks_for((int64_t)N * hw3 * (c3 / 8), T), T, 0, s,
             c->d_dpooled, reinterpret_cast<const __nv_bfloat16*>(c->d_cact[2]), N, hw3, c3,
             reinterpret_cast<__nv_bfloat16*>(c->d_dA[2]));
       else
-        gap_backward_kernel<float><<<blocks_for((int64_t)N * hw3 * c3, T), T, 0, s>>>(
+        launch_pdl(gap_backward_kernel<float>, blocks_for((int64_t)N * hw3 * c3, T), T, 0, s,
             c->d_dpooled, reinterpret_cast<const float*>(c->d_cact[2]), N, hw3, c3, reinterpret_cast<float*>(c->d_dA[2]));
       ph.launched(2);
     } else {
@@ -788,11 +812,11 @@ hs_status cnn_step(hs_ctx* c, float* params, const float* x, const int32_t* y, c
       }
       const int64_t n_in = (int64_t)N * L[k].hin * L[k].win * L[k].cin;
       if (bf16)
-        col2im_nhwc_vec4_kernel<<<blocks_for(n_in / 4, T), T, 0, s>>>(
+        launch_pdl(col2im_nhwc_vec4_kernel, blocks_for(n_in / 4, T), T, 0, s,
             c->d_dcol, L[k].K, reinterpret_cast<const __nv_bfloat16*>(c->d_cact[k - 1]), N, L[k].cin, L[k].hin,
             L[k].win, L[k].hout, L[k].wout, L[k].stride, reinterpret_cast<__nv_bfloat16*>(c->d_dA[k - 1]));
       else
-        col2im_nhwc_f32_kernel<<<blocks_for(n_in, T), T, 0, s>>>(
+        launch_pdl(col2im_nhwc_f32_kernel, blocks_for(n_in, T), T, 0, s,
             c->d_dcol, L[k].K, reinterpret_cast<const float*>(c->d_cact[k - 1]), N, L[k].cin, L[k].hin, L[k].win,
             L[k].hout, L[k].wout, L[k].stride, reinterpret_cast<float*>(c->d_dA[k - 1]));
       ph.launched(2);

@@ -18,6 +18,28 @@ enum DevErr : int32_t {
   kDevBadLabel = 2,      // a label outside [0, classes) reached the loss kernel
 };
 
+// Programmatic dependent launch for the elementwise and reduction kernels (the tensor-core kernels
+// do the same after their prologue): a kernel launched by launch_pdl may start while the previous
+// kernel of its stream is finishing, so it first waits for that kernel's completion (pdl_wait, its
+// first statement, before any global-memory access), then releases the next one (pdl_trigger).
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                              Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, static_cast<KArgs>(args)...);
+}
+
 struct DevStatus {
   float loss;         // sum_m w_m L_m of the last step
   int32_t err;        // DevErr

@@ -8,6 +8,8 @@ namespace hs {
 // ------------------------------------------------------------------------------------ cast
 __global__ void cast_f32_bf16_kernel(const float* __restrict__ x, __nv_bfloat16* __restrict__ y,
                                      int64_t n) {
+  pdl_wait();
+  pdl_trigger();
   const int64_t nvec = n / 4;
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   for (int64_t v = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; v < nvec; v += stride) {
@@ -28,7 +30,7 @@ void launch_cast_f32_bf16(const float* x, __nv_bfloat16* y, int64_t n, cudaStrea
   int64_t blocks = (n / 4 + 255) / 256;
   if (blocks < 1) blocks = 1;
   if (blocks > 4096) blocks = 4096;
-  cast_f32_bf16_kernel<<<(int)blocks, 256, 0, s>>>(x, y, n);
+  launch_pdl(cast_f32_bf16_kernel, (int)blocks, 256, 0, s, x, y, n);
 }
 
 // ------------------------------------------------------------------------ partition scatter
@@ -37,6 +39,8 @@ void launch_cast_f32_bf16(const float* x, __nv_bfloat16* y, int64_t n, cudaStrea
 __global__ void partition_scatter_kernel(const int32_t* __restrict__ offsets, int M, int N,
                                          int32_t* __restrict__ index_map, float* __restrict__ scale,
                                          int32_t* __restrict__ index_map_out) {
+  pdl_wait();
+  pdl_trigger();
   extern __shared__ int32_t s_off[];
   for (int k = threadIdx.x; k <= M; k += blockDim.x) s_off[k] = offsets[k];
   __syncthreads();
@@ -56,7 +60,7 @@ void launch_partition_scatter(const int32_t* d_offsets, int M, int N, int32_t* i
                               float* scale, int32_t* index_map_out, cudaStream_t s) {
   const int threads = 256;
   const int blocks = (N + threads - 1) / threads;
-  partition_scatter_kernel<<<blocks, threads, (M + 1) * sizeof(int32_t), s>>>(
+  launch_pdl(partition_scatter_kernel, blocks, threads, (M + 1) * sizeof(int32_t), s,
       d_offsets, M, N, index_map, scale, index_map_out);
 }
 
@@ -64,13 +68,15 @@ void launch_partition_scatter(const int32_t* d_offsets, int M, int N, int32_t* i
 // m's weight is folded into its samples (sum_m w_m G_m = one product over all rows).
 __global__ void scale_by_weight_kernel(const int32_t* __restrict__ index_map, const float* __restrict__ scale,
                                        const float* __restrict__ w, int N, float* __restrict__ out) {
+  pdl_wait();
+  pdl_trigger();
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i < N) out[i] = w[index_map[i]] * scale[i];
 }
 
 void launch_scale_by_weight(const int32_t* index_map, const float* scale, const float* w, int N, float* out,
                             cudaStream_t s) {
-  scale_by_weight_kernel<<<(N + 255) / 256, 256, 0, s>>>(index_map, scale, w, N, out);
+  launch_pdl(scale_by_weight_kernel, (N + 255) / 256, 256, 0, s, index_map, scale, w, N, out);
 }
 
 // ------------------------------------------------------------------ softmax cross-entropy
@@ -97,6 +103,8 @@ __global__ void softmax_xent_kernel(const float* __restrict__ logits, int ldl,
                                     const int32_t* __restrict__ y, const float* __restrict__ scale,
                                     int N, int C, void* __restrict__ delta, int ldd,
                                     float* __restrict__ ce, DevStatus* st) {
+  pdl_wait();
+  pdl_trigger();
   const int warps_per_block = blockDim.x >> 5;
   const int row = blockIdx.x * warps_per_block + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
@@ -134,6 +142,8 @@ __global__ void softmax_xent_reg_kernel(const float* __restrict__ logits, int ld
                                         const int32_t* __restrict__ y, const float* __restrict__ scale,
                                         int N, int C, void* __restrict__ delta, int ldd,
                                         float* __restrict__ ce, DevStatus* st) {
+  pdl_wait();
+  pdl_trigger();
   const int warps_per_block = blockDim.x >> 5;
   const int row = blockIdx.x * warps_per_block + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
@@ -198,18 +208,18 @@ void launch_softmax_xent(const float* logits, int ldl, const int32_t* y, const f
   const int blocks = (N + rows_per_block - 1) / rows_per_block;
   if (ldl % 4 == 0 && ldd % 4 == 0 && ldd <= 1024 && C <= ldd) {
     if (ldd <= 128) {
-      if (delta_bf16) softmax_xent_reg_kernel<true, 1><<<blocks, threads, 0, s>>>(logits, ldl, y, scale, N, C, delta, ldd, ce, st);
-      else softmax_xent_reg_kernel<false, 1><<<blocks, threads, 0, s>>>(logits, ldl, y, scale, N, C, delta, ldd, ce, st);
+      if (delta_bf16) launch_pdl(softmax_xent_reg_kernel<true, 1>, blocks, threads, 0, s, logits, ldl, y, scale, N, C, delta, ldd, ce, st);
+      else launch_pdl(softmax_xent_reg_kernel<false, 1>, blocks, threads, 0, s, logits, ldl, y, scale, N, C, delta, ldd, ce, st);
     } else {
-      if (delta_bf16) softmax_xent_reg_kernel<true, 8><<<blocks, threads, 0, s>>>(logits, ldl, y, scale, N, C, delta, ldd, ce, st);
-      else softmax_xent_reg_kernel<false, 8><<<blocks, threads, 0, s>>>(logits, ldl, y, scale, N, C, delta, ldd, ce, st);
+      if (delta_bf16) launch_pdl(softmax_xent_reg_kernel<true, 8>, blocks, threads, 0, s, logits, ldl, y, scale, N, C, delta, ldd, ce, st);
+      else launch_pdl(softmax_xent_reg_kernel<false, 8>, blocks, threads, 0, s, logits, ldl, y, scale, N, C, delta, ldd, ce, st);
     }
     return;
   }
   if (delta_bf16)
-    softmax_xent_kernel<true><<<blocks, threads, 0, s>>>(logits, ldl, y, scale, N, C, delta, ldd, ce, st);
+    launch_pdl(softmax_xent_kernel<true>, blocks, threads, 0, s, logits, ldl, y, scale, N, C, delta, ldd, ce, st);
   else
-    softmax_xent_kernel<false><<<blocks, threads, 0, s>>>(logits, ldl, y, scale, N, C, delta, ldd, ce, st);
+    launch_pdl(softmax_xent_kernel<false>, blocks, threads, 0, s, logits, ldl, y, scale, N, C, delta, ldd, ce, st);
 }
 
 // ------------------------------------------------------------------ per-worker loss reduction
@@ -220,6 +230,8 @@ void launch_softmax_xent(const float* logits, int ldl, const int32_t* y, const f
 __global__ void loss_reduce_kernel(const float* __restrict__ ce, const int32_t* __restrict__ offsets,
                                    int M, const float* __restrict__ w, float* __restrict__ lm,
                                    DevStatus* st, unsigned int* ticket) {
+  pdl_wait();
+  pdl_trigger();
   __shared__ float red[1024];
   __shared__ bool last;
   const int m = blockIdx.x;
@@ -250,7 +262,7 @@ __global__ void loss_reduce_kernel(const float* __restrict__ ce, const int32_t* 
 
 void launch_loss_reduce(const float* ce, const int32_t* d_offsets, int M, const float* d_w,
                         float* lm, DevStatus* st, unsigned int* ticket, cudaStream_t s) {
-  loss_reduce_kernel<<<M, 1024, 0, s>>>(ce, d_offsets, M, d_w, lm, st, ticket);
+  launch_pdl(loss_reduce_kernel, M, 1024, 0, s, ce, d_offsets, M, d_w, lm, st, ticket);
 }
 
 // ------------------------------------------------------------------ per-worker bias gradient
@@ -259,6 +271,8 @@ template <bool kBf16>
 __global__ void bias_grad_kernel(const void* __restrict__ delta, int ld, int width,
                                  const int32_t* __restrict__ offsets, float* __restrict__ slabs,
                                  int64_t Ps, int64_t b_off) {
+  pdl_wait();
+  pdl_trigger();
   const int m = blockIdx.y;
   const int j = blockIdx.x * blockDim.x + threadIdx.x;
   if (j >= width) return;
@@ -290,6 +304,8 @@ constexpr int kBgCols = 256;
 __global__ void __launch_bounds__(256) bias_grad_partial_kernel(const __nv_bfloat16* __restrict__ delta, int ld,
                                                                 int width, const int4* __restrict__ chunks,
                                                                 float* __restrict__ partial) {
+  pdl_wait();
+  pdl_trigger();
   __shared__ float red[8][kBgCols + 8];
   const int4 ck = chunks[blockIdx.y];       // (worker, row begin, row end, unused)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -339,6 +355,8 @@ __global__ void __launch_bounds__(256) bias_grad_partial_kernel(const __nv_bfloa
 __global__ void bias_grad_combine_kernel(const float* __restrict__ partial, int width,
                                          const int32_t* __restrict__ chunk_begin, float* __restrict__ slabs,
                                          int64_t Ps, int64_t b_off) {
+  pdl_wait();
+  pdl_trigger();
   const int m = blockIdx.y;
   const int col = blockIdx.x * blockDim.x + threadIdx.x;
   if (col >= width) return;
@@ -353,18 +371,18 @@ void launch_bias_grad_bf16(const __nv_bfloat16* delta, int ld, int width, const 
                            const int32_t* d_chunk_begin, int M, float* partial, float* slabs, int64_t Ps,
                            int64_t b_off, cudaStream_t s) {
   dim3 g1((width + kBgCols - 1) / kBgCols, n_chunks);
-  bias_grad_partial_kernel<<<g1, 256, 0, s>>>(delta, ld, width, d_chunks, partial);
+  launch_pdl(bias_grad_partial_kernel, g1, 256, 0, s, delta, ld, width, d_chunks, partial);
   dim3 g2((width + 255) / 256, M);
-  bias_grad_combine_kernel<<<g2, 256, 0, s>>>(partial, width, d_chunk_begin, slabs, Ps, b_off);
+  launch_pdl(bias_grad_combine_kernel, g2, 256, 0, s, partial, width, d_chunk_begin, slabs, Ps, b_off);
 }
 
 void launch_bias_grad(const void* delta, bool delta_bf16, int ld, int width, const int32_t* d_offsets,
                       int M, float* slabs, int64_t Ps, int64_t b_off, cudaStream_t s) {
   dim3 grid((width + 127) / 128, M);
   if (delta_bf16)
-    bias_grad_kernel<true><<<grid, 128, 0, s>>>(delta, ld, width, d_offsets, slabs, Ps, b_off);
+    launch_pdl(bias_grad_kernel<true>, grid, 128, 0, s, delta, ld, width, d_offsets, slabs, Ps, b_off);
   else
-    bias_grad_kernel<false><<<grid, 128, 0, s>>>(delta, ld, width, d_offsets, slabs, Ps, b_off);
+    launch_pdl(bias_grad_kernel<false>, grid, 128, 0, s, delta, ld, width, d_offsets, slabs, Ps, b_off);
 }
 
 // ------------------------------------------------------------------ fused reduce + SGD update
@@ -386,6 +404,8 @@ __global__ void __launch_bounds__(512) reduce_update_kernel(
     float* __restrict__ theta, const float* __restrict__ slabs, int64_t Ps, int M,
     const float* __restrict__ w, float lr, int64_t P, __nv_bfloat16* __restrict__ shadow,
     float* __restrict__ gdebug, float* __restrict__ mbuf, float mu, float wd, int first) {
+  pdl_wait();
+  pdl_trigger();
   // The weights stay in global memory (read through the read-only cache): no shared memory, so
   // blocks of this kernel can share an SM with a resident tensor-core GEMM CTA.
   const float* __restrict__ sw = w;
@@ -461,11 +481,11 @@ void launch_reduce_update(float* theta, const float* slabs, int64_t Ps, int M, c
   if (blocks > cap) blocks = cap;
   if (blocks < 1) blocks = 1;
   if (recipe && recipe->buf)
-    reduce_update_kernel<true><<<(int)blocks, threads, 0, s>>>(theta, slabs, Ps, M, d_w, lr, P, shadow, gdebug,
+    launch_pdl(reduce_update_kernel<true>, (int)blocks, threads, 0, s, theta, slabs, Ps, M, d_w, lr, P, shadow, gdebug,
                                                                recipe->buf, recipe->momentum, recipe->weight_decay,
                                                                recipe->first);
   else
-    reduce_update_kernel<false><<<(int)blocks, threads, 0, s>>>(theta, slabs, Ps, M, d_w, lr, P, shadow, gdebug,
+    launch_pdl(reduce_update_kernel<false>, (int)blocks, threads, 0, s, theta, slabs, Ps, M, d_w, lr, P, shadow, gdebug,
                                                                 nullptr, 0.f, 0.f, 0);
 }
 
