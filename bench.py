@@ -565,10 +565,21 @@ def run_ours(args, wl, rank, world, local_rank):
     def gemm_roof(name):
         # per launch: the phase's algorithmic flops and time divided by its launches per step
         ach = flops[name] / (per_step[name] * 1e-3) / 1e12
-        tile = name == "wgrad" and wl.arch == synth.MLP and precision == hs.HS_BF16
+        # the library's rule: the tile-averaged launch for layers with a 256 x 256 weight tile per
+        # SM pair (HS_TILE_AVERAGE=0 disables it, =all applies it to every layer)
+        pairs = torch.cuda.get_device_properties(dev).multi_processor_count // 2
+        env = os.environ.get("HS_TILE_AVERAGE", "1")
+        tiles = [-(-wl.dims[i + 1] // 256) * -(-wl.dims[i] // 256) for i in range(len(wl.dims) - 1)]
+        tile_layers = [t >= pairs or env == "all" for t in tiles] if env != "0" else [False] * len(tiles)
+        tile = (name == "wgrad" and wl.arch == synth.MLP and precision == hs.HS_BF16 and wl.workers <= 32
+                and any(tile_layers))
         traffic = recorded_traffic() if (tile and wl.name == DEFAULT_WORKLOAD) else None
-        kernel = ("tc_wgrad_avg_pair_kernel (per-worker weight gradients averaged in tensor memory, "
-                  "update fused)" if tile else f"tc_gemm_pair_kernel ({name})")
+        if tile:
+            kernel = ("tc_wgrad_avg_pair_kernel (per-worker weight gradients averaged in tensor memory, "
+                      "update fused)" + ("" if all(tile_layers) else "; slab-path tc_gemm_pair_kernel on "
+                                         f"{tile_layers.count(False)} of {len(tile_layers)} layers"))
+        else:
+            kernel = f"tc_gemm_pair_kernel ({name})"
         return {"kernel": kernel, "bound": "tensor", "achieved": ach, "peak": peaks["bf16_sust"],
                 "unit": "TFLOP/s", "frac": ach / peaks["bf16_sust"], "traffic": traffic,
                 "flops_per_launch": flops[name] / launches_per_step[name],
