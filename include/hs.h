@@ -130,6 +130,8 @@ hs_status hs_param_count(const hs_model_desc* model, int64_t* P);
  *                        pair); =all: averaged in tensor memory on every layer
  *   HS_OVERLAP_UPDATE=0  slab-path updates on the step's stream, not beside the
  *                        remaining products
+ *   HS_RELU_BITS=0       bf16 MLP: the input-gradient products read ReLU' from
+ *                        the stored activations instead of packed bits
  *   HS_CONV_IMPLICIT=0|fwd  bf16 CNN: materialised patch rows everywhere, or
  *                        for the input gradients only
  *   HS_TC_FORM=single    one-SM tensor-core tiles instead of SM pairs (read

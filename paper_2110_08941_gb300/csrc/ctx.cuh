@@ -72,6 +72,7 @@ struct hs_ctx {
 
   // workspace
   std::vector<void*> d_act;        // H_0 .. H_{L-1}
+  std::vector<uint64_t*> d_relu_bits;   // bf16: ReLU' of H_1 .. H_{L-1} as bits, [width / 64][N] words
   float* d_logits = nullptr;       // [N, Cp]
   void* d_delta[2] = {nullptr, nullptr};
   float* d_ce = nullptr;

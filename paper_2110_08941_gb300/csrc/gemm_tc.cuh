@@ -95,6 +95,12 @@ struct TcGemmParams {
   const float* bias;
   const __nv_bfloat16* Z;
   int64_t ldz;
+  // ReLU' as bits, word [n / 64][row] (bits_ld rows per column unit): written by a
+  // kTcEpiBiasReluBf16 launch (relu_bits_out), read by a kTcEpiMaskBf16 one in place of Z
+  // (relu_bits_in); both null: Z as above
+  uint64_t* relu_bits_out;
+  const uint64_t* relu_bits_in;
+  int64_t bits_ld;
   DevStatus* st;
 };
 

@@ -82,6 +82,10 @@ hs_status build_tc_static(hs_ctx* c) {
     f.tiles_m = (c->N + hs::kTcBM - 1) / hs::kTcBM;
     f.tiles_n = (f.n_store + hs::kTcBN - 1) / hs::kTcBN;
     f.epi = last ? hs::kTcEpiBiasF32 : hs::kTcEpiBiasReluBf16;
+    if (!last && c->d_relu_bits.size() > (size_t)(l + 1) && c->d_relu_bits[l + 1]) {
+      f.relu_bits_out = c->d_relu_bits[l + 1];
+      f.bits_ld = c->N;
+    }
     f.ew = 4;
     f.D = last ? static_cast<void*>(c->d_logits) : c->d_act[l + 1];
     f.ldd = last ? c->Cp : ly.out;
@@ -110,6 +114,10 @@ hs_status build_tc_static(hs_ctx* c) {
     d.ldd = c->delta_ld(l - 1);
     d.Z = reinterpret_cast<const __nv_bfloat16*>(c->d_act[l]);
     d.ldz = ly.in;
+    if (c->d_relu_bits.size() > (size_t)l && c->d_relu_bits[l]) {
+      d.relu_bits_in = c->d_relu_bits[l];
+      d.bits_ld = c->N;
+    }
     d.st = c->d_status;
     if (!hs::tc_make_store_map(&d.tmD[0], d.D, false, c->N, d.n_store, d.ldd, &why)) return fail(c, HS_ERR_CUDA, why);
   }
@@ -386,6 +394,7 @@ void free_all(hs_ctx* c) {
   }
   for (void* p : c->d_act) f(p);
   f(c->d_logits); f(c->d_delta[0]); f(c->d_delta[1]); f(c->d_ce); f(c->d_lm); f(c->d_status); f(c->d_ticket);
+  for (uint64_t* b : c->d_relu_bits) f(b);
   f(c->d_slabs); f(c->d_shadow); f(c->d_shadow_next); f(c->d_gdebug); f(c->d_xstage); f(c->d_ystage); f(c->d_mom);
   if (c->h_status) cudaFreeHost(c->h_status);
   for (auto& r : c->pending) {
@@ -796,6 +805,14 @@ hs_status hs_init(const hs_model_desc* model, int32_t M, const double* compute_w
     for (int l = 0; l < c->L; ++l) {
       if (l == 0 && !bf16) continue;   // fp32 reads x in place
       chk(dalloc(c, &c->d_act[l], es * N * (size_t)dims[l]));
+    }
+    // ReLU' of the hidden activations as bits for the input-gradient products (HS_RELU_BITS=0: read
+    // the bf16 activations instead)
+    const char* rb = getenv("HS_RELU_BITS");
+    if (bf16 && !(rb && !strcmp(rb, "0"))) {
+      c->d_relu_bits.assign(c->L, nullptr);
+      for (int l = 1; l < c->L; ++l)
+        chk(dalloc(c, &c->d_relu_bits[l], sizeof(uint64_t) * N * (size_t)((dims[l] + 63) / 64)));
     }
     chk(dalloc(c, &c->d_scale_fused, sizeof(float) * N));
     chk(dalloc(c, &c->d_all_off, sizeof(int32_t) * 2));

@@ -336,6 +336,14 @@ __device__ __forceinline__ void load_mask_unit(const TcGemmParams& p, int grp, i
 #pragma unroll
   for (int j = 0; j < 8; ++j) zq[j] = make_uint4(0u, 0u, 0u, 0u);
   if (row >= p.Mdim || n_base >= p.n_store) return;
+  if (!CONV && p.relu_bits_in) {
+    // the packed form of the same decisions, one 64-bit word per row and 64-column unit
+    const unsigned long long b =
+        __ldg(reinterpret_cast<const unsigned long long*>(p.relu_bits_in) + (int64_t)(n_base >> 6) * p.bits_ld + row);
+    zq[0].x = (uint32_t)b;
+    zq[0].y = (uint32_t)(b >> 32);
+    return;
+  }
   int64_t zrow = row;
   if (CONV && p.conv_d) {
     const int img = row / p.conv.hw;
@@ -403,6 +411,10 @@ __device__ __forceinline__ void epilogue_unit(const TcGemmParams& p, int grp, in
         for (int j = 0; j < 64; ++j)
           v[j] = fmaxf(v[j] + ((n_base + j < p.Ndim) ? __ldg(p.bias + n_base + j) : 0.f), 0.f);
       }
+    } else if (!CONV && p.relu_bits_in) {   // kTcEpiMaskBf16, ReLU' from the packed bits (in zq[0])
+      const uint64_t bits = (uint64_t)zq[0].x | ((uint64_t)zq[0].y << 32);
+#pragma unroll
+      for (int k = 0; k < 64; ++k) v[k] = ((bits >> k) & 1ull) ? v[k] : 0.f;
     } else {   // kTcEpiMaskBf16: ReLU' from the stored activation of the same row (prefetched in zq)
 #pragma unroll
       for (int j = 0; j < 8; ++j) {
@@ -420,6 +432,22 @@ __device__ __forceinline__ void epilogue_unit(const TcGemmParams& p, int grp, in
     for (int j = 0; j < 8; ++j)
       o[j] = make_uint4(pack_bf16(v[8 * j], v[8 * j + 1]), pack_bf16(v[8 * j + 2], v[8 * j + 3]),
                         pack_bf16(v[8 * j + 4], v[8 * j + 5]), pack_bf16(v[8 * j + 6], v[8 * j + 7]));
+    if (EPI == kTcEpiBiasReluBf16 && p.relu_bits_out && row < p.Mdim && n_base < p.n_store) {
+      // ReLU' of the stored (bf16) activations for the input-gradient product: bit k = value > 0
+      uint64_t bits = 0;
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const uint32_t w[4] = {o[j].x, o[j].y, o[j].z, o[j].w};
+#pragma unroll
+        for (int h = 0; h < 4; ++h) {
+          const __nv_bfloat162 pr = *reinterpret_cast<const __nv_bfloat162*>(&w[h]);
+          const int k = 8 * j + 2 * h;
+          bits |= (uint64_t)(__low2float(pr) > 0.f) << k;
+          bits |= (uint64_t)(__high2float(pr) > 0.f) << (k + 1);
+        }
+      }
+      reinterpret_cast<unsigned long long*>(p.relu_bits_out)[(int64_t)(n_base >> 6) * p.bits_ld + row] = bits;
+    }
   }
 }
 

@@ -245,3 +245,19 @@ def test_kernel_alone_bounded_wait_reports_and_leaves_theta():
     hs.hs_debug_wgrad_avg(A, B, [0, 64, 128], w, 0.1, theta, shadow)
     torch.cuda.synchronize()
     assert not torch.equal(theta, before)
+
+
+@pytest.mark.parametrize("dims,N,M", [((3072, 1024, 1024, 10), 1024, 4), ((264, 200, 136, 10), 300, 5),
+                                      ((512, 768, 1000), 2048, 16)])
+def test_relu_bits_equal_the_activation_mask(dims, N, M, monkeypatch):
+    """The input-gradient products take ReLU' from bits the forward epilogue packs (one per stored
+    activation, value > 0); with HS_RELU_BITS=0 they read the bf16 activations: the same decisions,
+    so the same parameters bit for bit."""
+    x, y, theta0 = _data(dims, N, seed=21)
+    weights = tuple(float(v) for v in np.linspace(1.0, 2.0, M))
+    out = []
+    for bits in ("1", "0"):
+        monkeypatch.setenv("HS_RELU_BITS", bits)
+        out.append(_run(dims, M, N, weights, hs.HS_SYNC_CP_WEIGHTED, True, 3, 0.05, x, y, theta0))
+    assert torch.equal(out[0][0], out[1][0])
+    assert out[0][1] == out[1][1]
