@@ -108,3 +108,96 @@ def test_bf16_decisions_differ_only_near_kinks():
         if diff.any():
             assert np.abs(a[diff]).max() < 0.05 * np.abs(a).std()
     assert flips < 0.01 * sum(a.size for a in c["pre"])
+
+
+# ---------------------------------------------------------------------------------------------
+# Hand-worked pins of the ReLU'-decision mode on a 1x1 image with one channel per layer.  With
+# padding 1 a 3x3 convolution of a 1x1 image reads the real pixel through its centre tap only; the
+# eight other taps multiply the zero padding (set to 5 here, so any padding mistake shows), and
+# every stride gives a 1x1 output.  The net is then a chain of scalars: A_k = c_k h_{k-1} + b_k,
+# h_k = ReLU(A_k), pooled = h_3, z = [h_3, -h_3] (fc W = [[1], [-1]], b = 0), y = 0, so
+# dL/dh_3 = -2 sigmoid(-2 h_3), dL/dA_k = dL/dh_k * mask_k, dL/dh_{k-1} = c_k dL/dA_k.
+# bf16 keeps 8 significant bits: 1 + 2^-8 is a tie that rounds to 1, 1 - 2^-10 rounds to 1.
+E8, E9, E10 = 2.0 ** -8, 2.0 ** -9, 2.0 ** -10
+ONE = (1, 1, 1, 1, 1, 1, 2)
+
+
+def _chain(x, centres, biases):
+    parts = []
+    for c, b in zip(centres, biases):
+        w = np.full((3, 3), 5.0)
+        w[1, 1] = c
+        parts += list(w.ravel()) + [b]
+    parts += [1.0, -1.0, 0.0, 0.0]
+    return np.asarray(parts, dtype=np.float64), np.array([[[[x]]]])
+
+
+def _hand_grad(x, centres, biases, masks):
+    """The gradient of the scalar chain written out: values exact, decisions as given."""
+    h = [x]
+    for c, b in zip(centres, biases):
+        h.append(max(c * h[-1] + b, 0.0))
+    s = 1.0 / (1.0 + np.exp(2.0 * h[3]))                 # sigmoid(-2 h3)
+    p0 = 1.0 - s
+    dh = -2.0 * s
+    g = [None] * 3
+    for k in (2, 1, 0):
+        da = dh * masks[k]
+        gw = np.zeros(9)
+        gw[4] = da * h[k]
+        g[k] = list(gw) + [da]
+        dh = da * centres[k]
+    return np.asarray(g[0] + g[1] + g[2] + [(p0 - 1.0) * h[3], (1.0 - p0) * h[3], p0 - 1.0, 1.0 - p0])
+
+
+def _cnn_masks(theta, x, rnd):
+    return [bool(m.ravel()[0]) for m in cnn.relu_decisions(theta, ONE, x, rnd)]
+
+
+def _exact(a):
+    return np.asarray(a, dtype=np.float64)
+
+
+def _check_case(x, centres, biases, want):
+    """want: {rounding: masks}; the gradient with each rounding's decisions equals the chain's."""
+    from oracle import mlp
+    theta, xa = _chain(x, centres, biases)
+    for name, masks in want.items():
+        rnd = {"bf16": mlp.round_bf16, "fp32": mlp.round_fp32, "exact": _exact}[name]
+        assert _cnn_masks(theta, xa, rnd) == masks, name
+        kw = {} if name == "exact" else {"decide": rnd}
+        _, g = cnn.worker_loss_grad(theta, ONE, xa, np.array([0]), **kw)
+        assert np.allclose(g, _hand_grad(x, centres, biases, masks), rtol=1e-14, atol=1e-300), name
+        assert np.all(g[[k for k in range(30) if k % 10 not in (4, 9)]] == 0.0)   # padding taps
+
+
+def test_hand_pin_input_rounding_flips_first_conv():
+    # x = 1 + 2^-8, c1 = 1, b1 = -(1 + 2^-9): exact A1 = 2^-9 > 0, bf16 A1 = 1 - (1 + 2^-9) < 0.
+    # b2 = 1 keeps conv 2 (and conv 3) on whatever h1 is.
+    _check_case(1.0 + E8, [1.0, 1.0, 1.0], [-(1.0 + E9), 1.0, 0.0],
+                {"bf16": [False, True, True], "fp32": [True, True, True], "exact": [True, True, True]})
+
+
+def test_hand_pin_weight_rounding_flips_first_conv():
+    _check_case(1.0, [1.0 + E8, 1.0, 1.0], [-(1.0 + E9), 1.0, 0.0],
+                {"bf16": [False, True, True], "fp32": [True, True, True]})
+
+
+def test_hand_pin_conv_bias_is_not_rounded():
+    # b1 = -(1 - 2^-10) as stored gives A1 = 2^-10 > 0; a bf16-rounded bias (-1) would give 0 (off).
+    _check_case(1.0, [1.0, 1.0, 1.0], [-(1.0 - E10), 1.0, 0.0], {"bf16": [True, True, True]})
+
+
+def test_hand_pin_stored_activation_rounding_flips_second_conv():
+    # A1 = 1 + 2^-8 in every precision; the stored h1 rounds to 1 in bf16, so with c2 = 1,
+    # b2 = -(1 + 2^-9) the exact A2 = 2^-9 is on and the bf16 A2 = -2^-9 is off.  b3 = 1 keeps conv 3
+    # on, so the flip shows in the gradient: nothing reaches conv 2 or conv 1 under bf16 decisions.
+    _check_case(1.0, [1.0, 1.0, 1.0], [E8, -(1.0 + E9), 1.0],
+                {"bf16": [True, False, True], "fp32": [True, True, True], "exact": [True, True, True]})
+
+
+def test_hand_pin_fp32_rounding_of_stored_conv_activations():
+    # x = 1, c1 = 1, b1 = 2^-30: A1 = 1 + 2^-30, stored in fp32 as 1; c2 = 1, b2 = -1: exact A2 = 2^-30
+    # (on), fp32 A2 = 0 (off, ReLU'(0) = 0).
+    _check_case(1.0, [1.0, 1.0, 1.0], [2.0 ** -30, -1.0, 1.0],
+                {"fp32": [True, False, True], "exact": [True, True, True]})

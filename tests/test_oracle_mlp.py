@@ -244,3 +244,133 @@ def test_cosine_lr_matches_torch_scheduler():
         assert abs(opt.param_groups[0]["lr"] - sgd.cosine_lr(0.1, 0.001, step, 50)) < 1e-12
         opt.step()
         sched.step()
+
+
+# ---------------------------------------------------------------------------------------------
+# Hand-worked pins of the ReLU'-decision mode.  Each net has one hidden unit per layer, one
+# sample and two classes with W_out = [[1], [-1]], b_out = 0, y = 0, so the arithmetic fits in a
+# comment.  The operands sit next to bf16 ties: bf16 keeps 8 significant bits, so between 1 and 2
+# the representable values are 2^-7 apart, 1 + 2^-8 is a tie (rounds to the even 1), and
+# 1 - 2^-10 rounds to 1.  With last hidden activation h the logits are z = [h, -h], softmax
+# p0 = sigmoid(2h), and dL/dh = (p0 - 1) - (1 - p0) = -2 sigmoid(-2h).
+E8, E9, E10 = 2.0 ** -8, 2.0 ** -9, 2.0 ** -10
+
+
+def _sigmoid(v):
+    return 1.0 / (1.0 + np.exp(-v))
+
+
+def _one_unit_net(ws, bs):
+    """Flat theta of an MLP with one unit per hidden layer and the fixed two-class output layer."""
+    parts = []
+    for w, b in zip(ws, bs):
+        parts += list(np.ravel(w)) + [b]
+    parts += [1.0, -1.0, 0.0, 0.0]
+    return np.asarray(parts, dtype=np.float64)
+
+
+def _masks(theta, dims, x, rnd):
+    return [bool(m[0, 0]) for m in mlp.relu_decisions(theta, dims, x, rnd)]
+
+
+def test_hand_pin_input_rounding_flips_first_layer():
+    # x = 1 + 2^-8, W1 = 1, b1 = -(1 + 2^-9): exact A1 = 2^-9 > 0.  bf16(x) = 1 (tie to even), so
+    # the bf16 decision sees 1 - (1 + 2^-9) = -2^-9 < 0.  x is an fp32 value: fp32 keeps the unit.
+    dims = (1, 1, 2)
+    x = np.array([[1.0 + E8]])
+    theta = _one_unit_net([[1.0]], [-(1.0 + E9)])
+    assert _masks(theta, dims, x, mlp.round_bf16) == [False]
+    assert _masks(theta, dims, x, mlp.round_fp32) == [True]
+    h = E9
+    d = -2.0 * _sigmoid(-2.0 * h)                       # dL/dA1 when the unit is on
+    loss, g_exact = mlp.worker_loss_grad(theta, dims, x, [0])
+    _, g_bf16 = mlp.worker_loss_grad(theta, dims, x, [0], decide=mlp.round_bf16)
+    assert abs(loss - np.log1p(np.exp(-2.0 * h))) <= 1e-15
+    # layout [W1, b1, W2 (2x1), b2 (2)]
+    p0 = _sigmoid(2.0 * h)
+    want_exact = [d * (1.0 + E8), d, (p0 - 1.0) * h, (1.0 - p0) * h, p0 - 1.0, 1.0 - p0]
+    want_bf16 = [0.0, 0.0] + want_exact[2:]              # unit off: no signal reaches W1, b1
+    assert np.allclose(g_exact, want_exact, rtol=1e-14, atol=0)
+    assert np.allclose(g_bf16, want_bf16, rtol=1e-14, atol=0)
+    assert g_bf16[0] == 0.0 and g_bf16[1] == 0.0
+
+
+def test_hand_pin_weight_rounding_flips_first_layer():
+    # The same with the off-grid value in the weight: x = 1, W1 = 1 + 2^-8.
+    dims = (1, 1, 2)
+    x = np.array([[1.0]])
+    theta = _one_unit_net([[1.0 + E8]], [-(1.0 + E9)])
+    assert _masks(theta, dims, x, mlp.round_bf16) == [False]
+    assert _masks(theta, dims, x, mlp.round_fp32) == [True]
+    _, g = mlp.worker_loss_grad(theta, dims, x, [0], decide=mlp.round_bf16)
+    assert g[0] == 0.0 and g[1] == 0.0
+    _, g = mlp.worker_loss_grad(theta, dims, x, [0])
+    assert np.isclose(g[0], -2.0 * _sigmoid(-2.0 * E9), rtol=1e-14, atol=0)
+
+
+def test_hand_pin_bias_is_not_rounded():
+    # The kernels add the fp32 bias to the fp32 accumulator: only products see bf16 operands.
+    # x = 1, W1 = 1, b1 = -(1 - 2^-10): A1 = 2^-10 > 0 with the bias as stored; a bf16-rounded
+    # bias (-1) would give A1 = 0 and switch the unit off (ReLU'(0) = 0).
+    dims = (1, 1, 2)
+    x = np.array([[1.0]])
+    theta = _one_unit_net([[1.0]], [-(1.0 - E10)])
+    assert mlp.round_bf16(np.array([-(1.0 - E10)]))[0] == -1.0     # the premise
+    assert _masks(theta, dims, x, mlp.round_bf16) == [True]
+    _, g = mlp.worker_loss_grad(theta, dims, x, [0], decide=mlp.round_bf16)
+    d = -2.0 * _sigmoid(-2.0 * E10)
+    assert np.allclose(g[:2], [d, d], rtol=1e-14, atol=0)
+
+
+def test_hand_pin_rounding_can_switch_a_unit_on():
+    # x = 1 + 2^-7 - 2^-9 rounds up to 1 + 2^-7 (0.75 of a bf16 step); b1 = -(1 + 2^-7 - 2^-10):
+    # exact A1 = -2^-10 (off), bf16 A1 = +2^-10 (on).  The values stay fp64: h = ReLU(exact A1) = 0,
+    # z = [0, 0], p0 = 1/2, so dL/dA1 = 2 (1/2 - 1) = -1 reaches W1 and b1 through the bf16 mask.
+    dims = (1, 1, 2)
+    xv = 1.0 + 2.0 ** -7 - E9
+    x = np.array([[xv]])
+    theta = _one_unit_net([[1.0]], [-(1.0 + 2.0 ** -7 - E10)])
+    assert _masks(theta, dims, x, mlp.round_bf16) == [True]
+    assert _masks(theta, dims, x, mlp.round_fp32) == [False]
+    _, g = mlp.worker_loss_grad(theta, dims, x, [0], decide=mlp.round_bf16)
+    assert np.allclose(g, [-xv, -1.0, 0.0, 0.0, -0.5, 0.5], rtol=1e-15, atol=0)
+    _, g = mlp.worker_loss_grad(theta, dims, x, [0])
+    assert np.allclose(g, [0.0, 0.0, 0.0, 0.0, -0.5, 0.5], rtol=1e-15, atol=0)
+
+
+def test_hand_pin_stored_activation_rounding_flips_second_layer():
+    # x = 1, W1 = 1, b1 = 2^-8: A1 = 1 + 2^-8 in every precision (x and W1 are bf16 values, the bias
+    # is not rounded), so layer 1 is on everywhere.  The stored activation H1 = 1 + 2^-8 rounds to 1
+    # in bf16; with W2 = 1, b2 = -(1 + 2^-9) the exact A2 = 2^-9 > 0 but the bf16 A2 = -2^-9.  Only the
+    # rounding of H1 flips layer 2.
+    dims = (1, 1, 1, 2)
+    x = np.array([[1.0]])
+    theta = _one_unit_net([[1.0], [1.0]], [E8, -(1.0 + E9)])
+    assert _masks(theta, dims, x, mlp.round_bf16) == [True, False]
+    assert _masks(theta, dims, x, mlp.round_fp32) == [True, True]
+    h2 = E9
+    d = -2.0 * _sigmoid(-2.0 * h2)
+    p0 = _sigmoid(2.0 * h2)
+    out = [(p0 - 1.0) * h2, (1.0 - p0) * h2, p0 - 1.0, 1.0 - p0]
+    # layout [W1, b1, W2, b2, W3 (2x1), b3 (2)]; dL/dA2 = d, dL/dA1 = d * W2 = d, H1 = 1 + 2^-8
+    _, g = mlp.worker_loss_grad(theta, dims, x, [0])
+    assert np.allclose(g, [d * 1.0, d, d * (1.0 + E8), d] + out, rtol=1e-14, atol=0)
+    _, g = mlp.worker_loss_grad(theta, dims, x, [0], decide=mlp.round_bf16)
+    assert np.allclose(g, [0.0, 0.0, 0.0, 0.0] + out, rtol=1e-14, atol=0)
+
+
+def test_hand_pin_fp32_rounding_of_stored_activations():
+    # The fp32 check path stores fp32 activations.  x = [1, 2^-30], W1 = [1, 1], b1 = 0: A1 = 1 + 2^-30
+    # in fp64, which fp32 (24 significant bits) rounds to 1.  W2 = 1, b2 = -1: exact A2 = 2^-30 > 0, fp32
+    # A2 = 0, off (ReLU'(0) = 0).  bf16 agrees with fp32 here; the exact oracle keeps the unit.
+    dims = (2, 1, 1, 2)
+    x = np.array([[1.0, 2.0 ** -30]])
+    theta = _one_unit_net([[1.0, 1.0], [1.0]], [0.0, -1.0])
+    assert _masks(theta, dims, x, mlp.round_fp32) == [True, False]
+    assert _masks(theta, dims, x, mlp.round_bf16) == [True, False]
+    assert _masks(theta, dims, x, lambda a: np.asarray(a, dtype=np.float64)) == [True, True]
+    _, g = mlp.worker_loss_grad(theta, dims, x, [0], decide=mlp.round_fp32)
+    assert np.all(g[:4] == 0.0)
+    _, g = mlp.worker_loss_grad(theta, dims, x, [0])
+    d = -2.0 * _sigmoid(-2.0 * 2.0 ** -30)
+    assert np.allclose(g[:5], [d, d * 2.0 ** -30, d, d * (1.0 + 2.0 ** -30), d], rtol=1e-14, atol=0)
