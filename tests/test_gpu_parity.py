@@ -3,10 +3,12 @@
 Acceptance: partitions and index maps bit-exact; the first step's synchronised gradient within
 relative L2 1e-2 (bf16 path) or 1e-5 (fp32 check path); parameters after 10 steps within relative
 L2 2e-2, also checked on the parameter change theta_10 - theta_0 (a stricter reading: 5e-2 for
-bf16, whose rounding biases the small last-layer bias updates - a CPU emulation of the exact bf16
-arithmetic gives 3.0e-2 on 3072-1024-1024-10 at lr 0.05 - and 2e-3 for fp32, where one ReLU kink
-decided differently by fp32 accumulation moves the trajectory by ~1e-3).  For the bf16 path the oracle takes the ReLU' decisions in the kernel's
-precision (bf16 operands); every value it computes stays fp64."""
+bf16, whose rounding biases the small last-layer bias updates - the CPU emulation of the bf16
+arithmetic in tests/bf16_emulation.py gives 2.9e-2 on 3072-1024-1024-10 at lr 0.05 - and 2e-3 for
+fp32, where one ReLU kink decided differently by fp32 accumulation moves the trajectory by ~1e-3).
+For the bf16 path the oracle takes the ReLU' decisions in the kernel's precision (bf16 operands);
+every value it computes stays fp64 (a departure from taking them exactly, bounded separately in
+test_bf16_against_exact_decisions)."""
 import functools
 
 import numpy as np
@@ -17,6 +19,7 @@ import synth
 import paper_2110_08941_gb300 as hs
 from oracle import partition as P
 from oracle import mlp
+from tests.bf16_emulation import BOUND_DTHETA, BOUND_LOSS_AFTER_FIRST, BOUND_VS_EXACT_DECISIONS
 from tests.gpu_helpers import decide_for, rel, run_library, run_oracle
 
 pytestmark = pytest.mark.gpu
@@ -32,13 +35,13 @@ def _check(lib, orc, theta0, precision, n_steps):
     assert rel(lib["g_first"], orc["g_first"]) <= TOL_G[precision]
     assert rel(lib["theta"], orc["theta"]) <= TOL_THETA
     d_lib, d_orc = lib["theta"] - theta0, orc["theta"] - theta0
-    assert rel(d_lib, d_orc) <= (5e-2 if precision == hs.HS_BF16 else 2e-3)
+    assert rel(d_lib, d_orc) <= (BOUND_DTHETA if precision == hs.HS_BF16 else 2e-3)
     ltol = 1e-2 if precision == hs.HS_BF16 else 1e-5
     # the first loss is at identical parameters; later ones follow the bf16 trajectory, whose loss
-    # drifts by up to 1.2e-2 from the oracle's on 3072-1024-1024-10 at lr 0.05 in a CPU emulation
-    # of the exact bf16 arithmetic
+    # drifts by up to 1.2e-2 from the oracle's on 3072-1024-1024-10 at lr 0.05 in the CPU emulation
+    # of the bf16 arithmetic
     for t, (a, b) in enumerate(zip(lib["losses"], orc["losses"])):
-        tol = ltol if (t == 0 or precision != hs.HS_BF16) else 3e-2
+        tol = ltol if (t == 0 or precision != hs.HS_BF16) else BOUND_LOSS_AFTER_FIRST
         assert abs(a - b) <= tol * abs(b), t
     for a, b in zip(lib["worker_losses_first"], orc["worker_losses_first"]):
         assert abs(a - b) <= ltol * abs(b)
@@ -171,17 +174,25 @@ def test_bf16_rejects_unaligned_widths():
     assert e.value.status == hs.HS_ERR_UNSUPPORTED
 
 
-@pytest.mark.parametrize("name", [synth.CFG1, synth.CFG2])
+# The first-step gradient against the oracle with exact (fp64) ReLU' decisions differs by the kink
+# flips that bf16 operand rounding causes.  The bounds come from the CPU emulation of the bf16
+# arithmetic (tests/bf16_emulation.py: RECORDED holds how far it lands from the exact-decision
+# oracle on the same step, BOUND_VS_EXACT_DECISIONS sits at least 1.4x above).  The
+# 4096-8192-8192-1000 workload's two smallest workers are checked in
+# test_gpu_step_behaviour.test_headline_workload_sampled_parity.
+EXACT_DECISION_GAP = [synth.CFG1, synth.CFG2, synth.CFG3, synth.CFG4]
+
+
+@pytest.mark.parametrize("name", EXACT_DECISION_GAP)
 def test_bf16_against_exact_decisions(name):
-    """Against the oracle with exact (fp64) ReLU' decisions the bf16 gradient differs by the kink
-    flips that bf16 operand rounding causes: 4.1e-2 (3072-256-10, 128 samples) and 1.4e-2
-    (3072-1024-1024-10, 1024 samples) in the CPU emulation of the same arithmetic."""
     wl, x, y, theta0, w = _inputs(name)
+    if wl.weight_kind == "drift":
+        w = None                       # the drifting workload starts from the even split
     lib = run_library(wl.arch, wl.dims, wl.workers, wl.global_batch, w, x, y, theta0, wl.lr, 1, hs.HS_BF16,
                       hs.HS_SYNC_CP_WEIGHTED)
     orc = run_oracle(wl.arch, wl.dims, wl.workers, wl.global_batch, w, x, y, theta0, wl.lr, 1,
                      hs.HS_SYNC_CP_WEIGHTED)
-    assert rel(lib["g_first"], orc["g_first"]) <= 6e-2
+    assert rel(lib["g_first"], orc["g_first"]) <= BOUND_VS_EXACT_DECISIONS[name]
 
 
 # ------------------------------------------------------------------------------------------ CNN
