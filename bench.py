@@ -331,6 +331,14 @@ def barrier():
 
 
 # ------------------------------------------------------------------------------ arms
+def bench_config(wl, world):
+    """The workload description both arms print (same dict, so the two lines compare directly)."""
+    return {"workload": wl.name, "global_batch": wl.global_batch, "workers": wl.workers,
+            "dims": list(wl.dims), "sync": "cp_weighted", "parallelism": f"replicas{world}",
+            "l2": ("working set > L2 (over 1 GB of activations and input gradients, 0.44 GB theta per "
+                   "step), no flush" if wl.name == DEFAULT_WORKLOAD else "small workload: working set may sit in L2")}
+
+
 def run_reference(args, wl, rank, world):
     if rank != 0:
         return
@@ -364,8 +372,7 @@ def run_reference(args, wl, rank, world):
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * dt / args.steps,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-            "data": "synthetic", "config": {"workload": wl.name, "global_batch": wl.global_batch,
-                                            "workers": wl.workers},
+            "data": "synthetic", "config": bench_config(wl, world),
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": sample},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
@@ -562,6 +569,21 @@ def run_ours(args, wl, rank, world, local_rank):
 
     launches_per_step = {k: max(1, round(v[1] / args.steps)) for k, v in prof.items()}
 
+    # Which bf16 denominator: the burst figure (cuBLAS timed alone, clocks at their maximum) for a
+    # short timed region whose SM clock stayed at its maximum; the sustained one (cuBLAS back to
+    # back for seconds, at the power cap) once the timed region is long or the clock dropped.
+    timed_s = ms * 1e-3
+    at_max = bool(clk) and clk["sm_mhz"] >= 0.97 * clk["sm_max_mhz"]
+    burst = timed_s < 2.0 and (at_max or not clk)
+    bf16_peak = peaks["bf16"] if burst else peaks["bf16_sust"]
+    bf16_kind = f"{peaks['src']} bf16 {'burst' if burst else 'sustained'}"
+
+    def tensor_frac(ach):
+        frac = ach / bf16_peak
+        # a plain cuBLAS GEMM sets the denominator: far above it means the timing is not the work
+        assert frac <= 1.2, f"tensor roofline fraction {frac:.3f} > 1.2 against {bf16_kind} {bf16_peak}"
+        return frac
+
     def gemm_roof(name):
         # per launch: the phase's algorithmic flops and time divided by its launches per step
         ach = flops[name] / (per_step[name] * 1e-3) / 1e12
@@ -580,11 +602,12 @@ def run_ours(args, wl, rank, world, local_rank):
                                          f"{tile_layers.count(False)} of {len(tile_layers)} layers"))
         else:
             kernel = f"tc_gemm_pair_kernel ({name})"
-        return {"kernel": kernel, "bound": "tensor", "achieved": ach, "peak": peaks["bf16_sust"],
-                "unit": "TFLOP/s", "frac": ach / peaks["bf16_sust"], "traffic": traffic,
+        return {"kernel": kernel, "bound": "tensor", "achieved": ach, "peak": bf16_peak,
+                "unit": "TFLOP/s", "frac": tensor_frac(ach), "traffic": traffic,
                 "flops_per_launch": flops[name] / launches_per_step[name],
                 "launches_per_step": launches_per_step[name],
-                "peak_kind": f"{peaks['src']} bf16 sustained"}
+                "peak_kind": bf16_kind,
+                "frac_vs_burst": ach / peaks["bf16"], "frac_vs_sustained": ach / peaks["bf16_sust"]}
 
     upd_ms = alone["update_ms"] if alone else per_step["update"]
     upd_ach = upd_bytes / (upd_ms * 1e-3) / 1e9
@@ -613,15 +636,13 @@ def run_ours(args, wl, rank, world, local_rank):
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "bf16" if precision == hs.HS_BF16 else "f32", "data": "synthetic",
-            "config": {"workload": wl.name, "global_batch": wl.global_batch, "workers": wl.workers,
-                       "dims": list(wl.dims), "sync": "cp_weighted", "parallelism": f"replicas{world}",
-                       "l2": ("working set > L2 (over 1 GB of activations and input gradients, 0.44 GB theta per "
-                                     "step), no flush"
-                              if wl.name == DEFAULT_WORKLOAD else "small workload: working set may sit in L2")},
+            "config": bench_config(wl, world),
             "roofline": roofline,
             "roofline_gemm_phase": {"bound": "tensor", "achieved": gemm_total / (gemm_ms * 1e-3) / 1e12,
-                                    "peak": peaks["bf16_sust"], "unit": "TFLOP/s",
-                                    "frac": gemm_total / (gemm_ms * 1e-3) / 1e12 / peaks["bf16_sust"],
+                                    "peak": bf16_peak, "unit": "TFLOP/s", "peak_kind": bf16_kind,
+                                    "frac": tensor_frac(gemm_total / (gemm_ms * 1e-3) / 1e12),
+                                    "frac_vs_burst": gemm_total / (gemm_ms * 1e-3) / 1e12 / peaks["bf16"],
+                                    "frac_vs_sustained": gemm_total / (gemm_ms * 1e-3) / 1e12 / peaks["bf16_sust"],
                                     "flops_per_step": gemm_total},
             "roofline_reduce_update": roof_update,
             "step_ms": {"median": float(np.median(step_ms)), "p10": float(np.percentile(step_ms, 10)),

@@ -80,3 +80,5 @@ def test_reference_arm_prints_the_contract_line(capsys):
     assert d["e2e"] == {"value": d["value"], "unit": d["unit"], "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}
     assert d["cpu_baseline"]["kind"] == "oracle" and d["cpu_baseline"]["value"] == d["value"]
     assert d["config"]["workload"] == synth.CFG1
+    # the same config dict as the GPU arm prints for this workload, so the two lines compare
+    assert d["config"] == bench.bench_config(synth.WORKLOADS[synth.CFG1], 1)
