@@ -279,8 +279,11 @@ hs_status hs_read_profile(hs_ctx* ctx, double* ms_out, int64_t* launches_out);
  * that table's device address (cudaGetSymbolAddress, with that device current); make that first
  * call before any stream capture.  All calls share the table and it keeps the last call's
  * offsets; calls whose kernels overlap on the GPU (different streams) race on it.
- * Errors: HS_ERR_INVALID_ARG for M > 1024 or any hs_partition_sizes error, HS_ERR_CUDA; the
- * message is returned by hs_last_init_error().  Asynchronous on `stream`. */
+ * `stream` must belong to the current device (the table's address is looked up per device).
+ * Each call copies the M + 1 offsets from a host stack array (pageable memory) with
+ * cudaMemcpyAsync on `stream`; the runtime stages that copy before the call returns.
+ * Errors: HS_ERR_INVALID_ARG for M > 1024, any hs_partition_sizes error, or a stream of another
+ * device; HS_ERR_CUDA; the message is returned by hs_last_init_error().  Asynchronous on `stream`. */
 hs_status hs_partition_noalloc(int32_t M, int32_t N, const double* cp, int32_t* counts_out,
                                int32_t* index_map_out, void* stream);
 

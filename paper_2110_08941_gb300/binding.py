@@ -132,8 +132,18 @@ def hs_partition_sizes(cp: Sequence[float], n: int) -> List[int]:
     return list(out[:m])
 
 
+def _check_index_map(index_map_out, n: int):
+    """The library writes n int32 through index_map_out's pointer: reject anything else first."""
+    import torch
+    if not (isinstance(index_map_out, torch.Tensor) and index_map_out.is_cuda
+            and index_map_out.dtype == torch.int32 and index_map_out.is_contiguous()
+            and index_map_out.numel() == n and index_map_out.device.index == torch.cuda.current_device()):
+        raise ValueError(f"index_map_out must be a contiguous int32 CUDA tensor of {n} elements on the current device")
+
+
 def hs_partition_noalloc(cp: Sequence[float], n: int, index_map_out, stream=None) -> List[int]:
     """Partition sizes and the device index map without a context or any device allocation."""
+    _check_index_map(index_map_out, int(n))
     m = len(cp)
     cpa = (c_double * max(m, 1))(*[float(v) for v in cp])
     out = (c_int32 * max(m, 1))()
@@ -202,8 +212,7 @@ def hs_partition(ctx: Context, measured_throughputs=None, index_map_out=None, st
     raw = hs_partition_t()
     im = None
     if index_map_out is not None:
-        import torch
-        assert index_map_out.is_cuda and index_map_out.dtype == torch.int32 and index_map_out.numel() == ctx.N
+        _check_index_map(index_map_out, ctx.N)
         im = c_void_p(index_map_out.data_ptr())
     s = c_void_p(_stream_ptr(stream)) if (tp is not None or im is not None) else c_void_p(0)
     _check(_lib.hs_partition(ctx.ptr, tp, None, im, s, ctypes.byref(raw)), ctx.ptr)

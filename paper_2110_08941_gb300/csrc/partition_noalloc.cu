@@ -72,6 +72,17 @@ extern "C" hs_status hs_partition_noalloc(int32_t M, int32_t N, const double* cp
     cudaGetLastError();
     return fail(HS_ERR_CUDA, "hs_partition_noalloc: no usable current CUDA device");
   }
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (s) {
+    // The table's address is per device: a stream of another device would get the wrong one.
+    int sdev = -1;
+    if (cudaStreamGetDevice(s, &sdev) != cudaSuccess) {
+      cudaGetLastError();
+      return fail(HS_ERR_INVALID_ARG, "hs_partition_noalloc: stream is not a valid CUDA stream");
+    }
+    if (sdev != dev)
+      return fail(HS_ERR_INVALID_ARG, "hs_partition_noalloc: stream belongs to another device than the current one");
+  }
   int32_t* d_off = nullptr;
   {
     // Set-up, once per device with that device current: the host-side name of the static array is
@@ -88,7 +99,6 @@ extern "C" hs_status hs_partition_noalloc(int32_t M, int32_t N, const double* cp
     }
     d_off = g_offsets_addr[dev];
   }
-  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   // Pageable source: the copy is staged before the call returns, so the stack table may go away.
   cudaError_t e = cudaMemcpyAsync(d_off, offsets, sizeof(int32_t) * (M + 1), cudaMemcpyHostToDevice, s);
   if (e != cudaSuccess) return fail(HS_ERR_CUDA, cudaGetErrorString(e));

@@ -112,3 +112,30 @@ def test_cosine_lr_matches_oracle():
         assert hs.hs_cosine_lr(0.1, 0.001, t, 100) == pytest.approx(sgd.cosine_lr(0.1, 0.001, min(t, 100), 100),
                                                                     rel=0, abs=1e-15)
     assert hs.hs_cosine_lr(0.1, 0.0, 5, 0) == 0.1
+
+
+def test_index_map_outputs_are_checked_before_the_library_is_called(monkeypatch):
+    """hs_partition_noalloc writes N int32 through the tensor's pointer: a short, int64, strided
+    or host tensor is refused by the binding before any library call (so before any launch)."""
+    import torch
+    from paper_2110_08941_gb300 import binding
+
+    calls = []
+
+    class Recorder:
+        def __getattr__(self, name):
+            def f(*a):
+                calls.append(name)
+                return 0
+            return f
+
+    monkeypatch.setattr(binding, "_lib", Recorder())
+    bad = [torch.zeros(7, dtype=torch.int32),                       # host memory, right length
+           torch.zeros(6, dtype=torch.int32),                       # short
+           torch.zeros(7, dtype=torch.int64),                       # wrong element type
+           torch.zeros(14, dtype=torch.int32)[::2],                 # not contiguous
+           np.zeros(7, dtype=np.int32)]                             # not a tensor
+    for t in bad:
+        with pytest.raises(ValueError):
+            hs.hs_partition_noalloc([1.0, 2.0], 7, t)
+    assert calls == []
