@@ -466,6 +466,13 @@ hs_status cnn_build_wgrad_plan(hs_ctx* c, int layer, const __nv_bfloat16* a, int
 
 namespace {
 
+// Epilogue warps of the 256 x 128 SM-pair tiles: two groups of four on alternate tiles (the
+// default), or four (HS_NARROW_EW=4).
+int narrow_epilogue_warps() {
+  const char* v = getenv("HS_NARROW_EW");
+  return (v && !strcmp(v, "4")) ? 4 : 8;
+}
+
 // A is K-major [a_rows][a_cols], or (conv != nullptr) the implicit patch rows of that convolution.
 // narrow = true: 256 x 128 SM-pair tiles for a product at most 128 wide (K-major B in 64-row boxes).
 hs_status plan_dense(hs_ctx* c, TcGemmParams* p, int epi, const __nv_bfloat16* a, int64_t a_rows, int a_cols,
@@ -489,6 +496,7 @@ hs_status plan_dense(hs_ctx* c, TcGemmParams* p, int epi, const __nv_bfloat16* a
   if (narrow) {
     p->pn = 128;
     p->form = kTcFormPair;
+    p->ew = narrow_epilogue_warps();
   }
   ok = ok && tc_make_store_map(&p->tmD[0], d, d_f32, Mdim, n_store, ldd, &why);
   if (!ok) return fail(c, HS_ERR_CUDA, why);
@@ -549,6 +557,7 @@ hs_status plan_subpixel_dgrad(hs_ctx* c, int k) {
   if (L.cin <= 128) {   // 256 x 128 SM-pair tiles (the class weights are MN-major: 64-column boxes)
     p.pn = 128;
     p.form = kTcFormPair;
+    p.ew = narrow_epilogue_warps();
   }
   p.conv = tc_conv_geom(L.cout, L.hout, L.wout, L.stride);
   p.conv.H = L.hin;

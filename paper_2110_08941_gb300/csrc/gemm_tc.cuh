@@ -65,8 +65,9 @@ struct TcGemmParams {
   int32_t pn;                      // SM-pair tile width: 0 or 256, or 128 (then K-major B maps have
                                    // 64-row boxes and form must be kTcFormPair)
   int32_t test_stall;              // test hook only: the producer issues no loads (bounded waits expire)
-  int32_t ew;                      // SM-pair form: 8 = eight epilogue warps (input-gradient products,
-                                   // 256-wide tiles, no convolution operands); 0 or 4: four
+  int32_t ew;                      // SM-pair form: 8 = eight epilogue warps (256-wide tiles: the MLP's
+                                   // short-K input gradients, two warps per lane quadrant; 128-wide
+                                   // tiles: two groups of four on alternate tiles); 0 or 4: four
   // kTcEpiAvgUpdate: the update's operands
   CUtensorMap tmT;                 // fp32 theta of the layer's weights [Mdim][n_store] (tc_make_store_map)
   CUtensorMap tmS;                 // bf16 copy of those weights, written beside theta (tc_make_store_map_bf16_32)

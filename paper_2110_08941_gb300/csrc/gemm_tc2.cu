@@ -29,23 +29,28 @@ constexpr int HM = PM / 2;                         // per-CTA half
 constexpr int A_HALF = HM * BK * 2;                // 16 KB
 // Pair tile of 256 x TN (TN = 256, or 128 for products at most 128 wide): per-CTA B half, stages
 // (more of them when the B half is smaller), two TN-column accumulators in tensor memory.  EW
-// epilogue warps (4, or 8 for short-K products whose epilogue outlasts the main loop: two per
-// tensor-memory lane quadrant, each on half of the tile's columns, with one stage fewer to fit
-// their staging buffers).
+// epilogue warps: 4, or 8 for short-K products whose epilogue outlasts the main loop.  With
+// 256-wide tiles the eight are two per tensor-memory lane quadrant, each on half of the tile's
+// columns; with 128-wide tiles (kAlt) they are two groups of four, each draining every other tile
+// (one accumulator buffer each), so two tiles' epilogues run at once even where the product is
+// only 64 wide.  Eight epilogue warps cost stages to fit their staging buffers.
 template <int TN, int EW>
 struct PairCfg {
   static constexpr int PN = TN;
   static constexpr int HN = TN / 2;
   static constexpr int B_HALF = HN * BK * 2;
   static constexpr int STAGE2 = A_HALF + B_HALF;
-  static constexpr int S2 = TN == 256 ? (EW == 8 ? 5 : 6) : 8;
+  static constexpr bool kAlt = (TN == 128 && EW == 8);
+  static constexpr int S2 = TN == 256 ? (EW == 8 ? 5 : 6) : (EW == 8 ? 6 : 8);
   static constexpr int kThreads = 64 + 32 * EW;
   static constexpr uint32_t PAIR_TX = 2 * STAGE2;   // bytes landing per stage on the leader's barrier
   static constexpr uint32_t kTmemCols2 = 2 * TN;
   static constexpr int kStaging = EW * 8192;         // two 32-row x 128-byte buffers per epilogue warp
   static constexpr int kSmem2 = S2 * STAGE2 + kStaging + 1024 + 256;
+  // arrivals that free one accumulator buffer: the epilogue warps of both CTAs that drain it
+  static constexpr uint32_t kFreeArrivals = 2 * (kAlt ? 4 : EW);
   static_assert(kSmem2 <= 232448, "shared memory budget");
-  static_assert(EW == 4 || (EW == 8 && TN == 256), "epilogue warps");
+  static_assert(EW == 4 || EW == 8, "epilogue warps");
 };
 
 template <int EPI, bool A_MN, bool B_MN, bool CONV, int TN, int EW>
@@ -77,7 +82,7 @@ __global__ void __launch_bounds__(PairCfg<TN, EW>::kThreads, 1)
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(smem_u32(&tfull_bar[b]), 1);
-      mbar_init(smem_u32(&tempty_bar[b]), 2 * EW);   // the epilogue warps of both CTAs of the pair
+      mbar_init(smem_u32(&tempty_bar[b]), Cfg::kFreeArrivals);
     }
     *abort_flag = 0;
     fence_mbar_init();
@@ -226,15 +231,21 @@ __global__ void __launch_bounds__(PairCfg<TN, EW>::kThreads, 1)
   } else {
     // -------------------------------------------------------------- epilogue (warps 2..5, both CTAs)
     constexpr bool kF32Out = (EPI == kTcEpiBiasF32 || EPI == kTcEpiStoreF32);
+    constexpr bool kAlt = Cfg::kAlt;
     constexpr int kUnitCols = kF32Out ? 32 : 64;
-    constexpr int kUnits = PN / kUnitCols / (EW / 4);   // units of this warp's column share
+    constexpr int kUnits = kAlt ? PN / kUnitCols : PN / kUnitCols / (EW / 4);   // units of this warp's share
     const int q = warp & 3;
-    const int col_share = (warp - 2) >> 2;             // 0, or 1 for the second warp of a quadrant
+    const int second = (warp - 2) >> 2;                // 0, or 1 for the second warp of a quadrant
+    const int col_share = kAlt ? 0 : second;           // 256-wide tiles: the second warp takes half the columns
     const uint32_t stage_base = smem_u32(sStage) + (uint32_t)((warp - 2) * 8192);
     int sb = 0;
-    int ab = 0;
+    // kAlt: the MMA issuer fills buffer i % 2 for its i-th tile; group `second` drains buffer
+    // `second`, i.e. every other tile starting at the group's first
+    int ab = kAlt ? second : 0;
     uint32_t aph = 0;
-    for (int t = pair_id; t < total; t += n_pairs) {
+    const int t_first = pair_id + (kAlt ? second * n_pairs : 0);
+    const int t_step = kAlt ? 2 * n_pairs : n_pairs;
+    for (int t = t_first; t < total; t += t_step) {
       const TileWork w = tile_work(p, t, tiles_m, tiles_n);
       const TileCoord c = w.c;
       uint4 zq[8];   // mask operand of the tile's first unit, loaded before the accumulator is ready
@@ -287,7 +298,12 @@ __global__ void __launch_bounds__(PairCfg<TN, EW>::kThreads, 1)
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive_cluster(map_to_rank(smem_u32(&tempty_bar[ab]), 0));
-      if (++ab == 2) { ab = 0; aph ^= 1u; }
+      if (kAlt) {
+        aph ^= 1u;
+      } else if (++ab == 2) {
+        ab = 0;
+        aph ^= 1u;
+      }
     }
     if (lane == 0) bulk_wait_all();
   }
@@ -363,12 +379,18 @@ cudaError_t launch_tc_gemm_pair(const TcGemmParams& p, int num_sms, cudaStream_t
   const int pairs = total;
   const int grid = num_sms;   // forwarded as the SM count for the residency query
   if (tn == 128) {
-    // 256 x 128 tiles (K-major B maps with 64-row boxes): the narrow products of the convolutions
-    if (p.epi == kTcEpiBiasReluBf16 && !p.a_mn && !p.b_mn)
+    // 256 x 128 tiles (K-major B maps with 64-row boxes): the narrow products of the convolutions,
+    // with four epilogue warps or two groups of four on alternate tiles
+    if (p.epi == kTcEpiBiasReluBf16 && !p.a_mn && !p.b_mn) {
+      if (p.ew == 8)
+        return (p.conv_a ? launch_pair_variant<kTcEpiBiasReluBf16, false, false, true, 128, 8>
+                         : launch_pair_variant<kTcEpiBiasReluBf16, false, false, false, 128, 8>)(p, pairs, grid, s);
       return (p.conv_a ? launch_pair_variant<kTcEpiBiasReluBf16, false, false, true, 128>
                        : launch_pair_variant<kTcEpiBiasReluBf16, false, false, false, 128>)(p, pairs, grid, s);
+    }
     if (p.epi == kTcEpiMaskBf16 && !p.a_mn && p.b_mn && (p.conv_a || p.conv_d))
-      return launch_pair_variant<kTcEpiMaskBf16, false, true, true, 128>(p, pairs, grid, s);
+      return p.ew == 8 ? launch_pair_variant<kTcEpiMaskBf16, false, true, true, 128, 8>(p, pairs, grid, s)
+                       : launch_pair_variant<kTcEpiMaskBf16, false, true, true, 128>(p, pairs, grid, s);
     return cudaErrorInvalidValue;
   }
   // implicit convolution operands (forward, weight gradient, sub-pixel input gradient)
