@@ -399,10 +399,6 @@ def run_ours(args, wl, rank, world, local_rank):
     for _ in range(args.warmup):
         hs.hs_step(ctx, params, xd, yd, part, wl.lr, stream=stream, want_loss=False)
     torch.cuda.synchronize()
-    hs.hs_read_profile(ctx)                 # discard warm-up counts
-    # CUDA events around every phase of the timed steps, on the step's stream: the live kernel
-    # times behind the roofline (a few microseconds of event records per step)
-    hs.hs_set_profiling(ctx, True)
 
     clocks = ClockSampler(local_rank)
     clocks.start()
@@ -417,11 +413,27 @@ def run_ours(args, wl, rank, world, local_rank):
         ev[i + 1].record(stream)
     torch.cuda.synchronize()
     barrier()
-    clk = clocks.stop()
     ms = ev[0].elapsed_time(ev[-1])
     step_ms = np.asarray([ev[i].elapsed_time(ev[i + 1]) for i in range(args.steps)])
     ms = max_over_ranks(ms)
+    # The same K steps again with CUDA events around every phase, on the step's stream: the live
+    # kernel times behind the roofline.  A second pass because recording (or, on a replayed step,
+    # re-pointing) two events per phase costs host time that would show in the small workloads'
+    # step time; the library captures the profiled step in the first two of its warm-up steps.
+    hs.hs_set_profiling(ctx, True)
+    for _ in range(3):
+        hs.hs_step(ctx, params, xd, yd, part, wl.lr, stream=stream, want_loss=False)
+    torch.cuda.synchronize()
+    hs.hs_read_profile(ctx)                 # discard warm-up counts
+    pv0, pv1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    pv0.record(stream)
+    for _ in range(args.steps):
+        hs.hs_step(ctx, params, xd, yd, part, wl.lr, stream=stream, want_loss=False)
+    pv1.record(stream)
+    torch.cuda.synchronize()
+    clk = clocks.stop()
     prof = hs.hs_read_profile(ctx)
+    profiled_ms = pv0.elapsed_time(pv1) / args.steps
     hs.hs_set_profiling(ctx, False)
     loss = hs.hs_step(ctx, params, xd, yd, part, 0.0, stream=stream, want_loss=True)   # finite-loss check
 
@@ -498,11 +510,11 @@ def run_ours(args, wl, rank, world, local_rank):
         for overlap in (False, True):
             ctx2 = slab_context(overlap)
             p2 = params.clone()
+            hs.hs_set_profiling(ctx2, not overlap)
             for _ in range(args.warmup):
                 hs.hs_step(ctx2, p2, xd, yd, ctx2.partition, wl.lr, stream=stream, want_loss=False)
             torch.cuda.synchronize()
             hs.hs_read_profile(ctx2)
-            hs.hs_set_profiling(ctx2, not overlap)
             a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             a0.record(stream)
             for _ in range(k2):
@@ -528,8 +540,9 @@ def run_ours(args, wl, rank, world, local_rank):
     yh = torch.from_numpy(y).pin_memory()
     k_e2e = max(3, min(args.steps, 10))
     copy_stream = torch.cuda.Stream(dev)
-    hs.hs_step(ctx, params, hs.hs_stage_inputs(ctx, xh, yh, stream=copy_stream), None, part, wl.lr, stream=stream,
-               want_loss=True)
+    for _ in range(3):   # both staging slots' steps captured before the timed loop
+        hs.hs_step(ctx, params, hs.hs_stage_inputs(ctx, xh, yh, stream=copy_stream), None, part, wl.lr,
+                   stream=stream, want_loss=True)
     barrier()
     t0 = time.perf_counter()
     nxt = hs.hs_stage_inputs(ctx, xh, yh, stream=copy_stream)
@@ -540,7 +553,8 @@ def run_ours(args, wl, rank, world, local_rank):
         hs.hs_step(ctx, params, cur, None, part, wl.lr, stream=stream, want_loss=True)
     e2e_s = time.perf_counter() - t0
     e2e_s = max_over_ranks(e2e_s)
-    hs.hs_step(ctx, params, xh, yh, part, wl.lr, stream=stream, want_loss=True)
+    for _ in range(2):
+        hs.hs_step(ctx, params, xh, yh, part, wl.lr, stream=stream, want_loss=True)
     barrier()
     t0 = time.perf_counter()
     for _ in range(k_e2e):
@@ -648,6 +662,9 @@ def run_ours(args, wl, rank, world, local_rank):
             "step_ms": {"median": float(np.median(step_ms)), "p10": float(np.percentile(step_ms, 10)),
                         "p90": float(np.percentile(step_ms, 90))},
             "phases_ms_per_step": per_step,
+            "phases_pass": {"ms_per_step": profiled_ms,
+                            "what": "the same steps with CUDA events around every phase, right after the "
+                                    "timed region; phase times and the roofline's kernel time come from it"},
             "gpu_launches": int(launches),
             "cpu_baseline": cpu,
             "e2e": {"value": world * wl.global_batch * k_e2e / e2e_s, "unit": UNIT,

@@ -135,7 +135,12 @@ hs_status hs_param_count(const hs_model_desc* model, int64_t* P);
  *   HS_CONV_IMPLICIT=0|fwd  bf16 CNN: materialised patch rows everywhere, or
  *                        for the input gradients only
  *   HS_TC_FORM=single    one-SM tensor-core tiles instead of SM pairs (read
- *                        when the library loads) */
+ *                        when the library loads)
+ *   HS_NARROW_EW=4       256 x 128 SM-pair tiles with four epilogue warps instead
+ *                        of two groups of four on alternate tiles
+ *   HS_STEP_GRAPH=0      every hs_step enqueues its kernels one by one (no
+ *                        replay of a captured step, see hs_step); =1 replays
+ *                        captured steps also above 1e11 parameter-samples */
 hs_status hs_init(const hs_model_desc* model, int32_t M, const double* compute_weights,
                   int32_t global_batch, hs_ctx** out);
 
@@ -188,7 +193,16 @@ hs_status hs_set_cp_history(hs_ctx* ctx, int32_t mode, double param);
  * CUDA graphs: with device x and y, loss_out NULL and the bf16 shadow current (a previous step
  * or hs_sync_params on the same params), the call only enqueues work on `stream` and may be
  * captured into a graph.  The graph holds this call's pointers, lr and partition plans by value:
- * it stays valid until the next hs_partition, hs_set_* or hs_init/hs_destroy on the context. */
+ * it stays valid until the next hs_partition, hs_set_* or hs_init/hs_destroy on the context.
+ * The library's own graph of the step (contexts of at most 1e11 parameter-samples, P * N, whose
+ * step is short enough for its launches to show): once a context has run a step, hs_step captures the step's
+ * kernels into a CUDA graph per combination of params, the device x and y it reads (caller's,
+ * staging slot or its own copy), momentum state and profiling, keeps the four last used, and
+ * replays them, writing lr to device memory with one small kernel first; the kernels and their
+ * order are the eager step's, so results are identical.  A call on a stream the caller is
+ * capturing is enqueued kernel by kernel.  hs_partition with new sizes, hs_set_debug,
+ * hs_set_fused_sync and hs_set_optimizer drop the captured steps; HS_STEP_GRAPH=0 (read by
+ * hs_init) keeps every step eager. */
 hs_status hs_step(hs_ctx* ctx, float* params, const void* x, const int32_t* y,
                   const hs_partition_t* part, float lr, void* stream, float* loss_out);
 

@@ -83,9 +83,13 @@ struct UpdateRecipe {
   float momentum, weight_decay;
   int first;   // 1: the buffer starts as d (first step after the recipe was set)
 };
+// lr_dev: when non-null the kernel reads the learning rate there (a step replayed from a CUDA
+// graph) instead of taking `lr`.
 void launch_reduce_update(float* theta, const float* slabs, int64_t Ps, int M, const float* d_w,
                           float lr, int64_t P, __nv_bfloat16* shadow, float* gdebug, int num_sms,
-                          cudaStream_t s, int blocks_per_sm = 4, const UpdateRecipe* recipe = nullptr);
+                          cudaStream_t s, int blocks_per_sm = 4, const UpdateRecipe* recipe = nullptr,
+                          const float* lr_dev = nullptr);
+void launch_set_scalar(float* dst, float v, cudaStream_t s);
 
 // ---------------------------------------------------------------- fp32 CUDA-core GEMM (check path)
 // C(m, n) = sum_k A(m, k) B(k, n) with A(m,k) = A[m*a_sm + k*a_sk], B(k,n) = B[k*b_sk + n*b_sn],

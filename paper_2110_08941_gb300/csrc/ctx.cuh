@@ -109,6 +109,32 @@ struct hs_ctx {
   std::vector<cudaEvent_t> event_pool;
   int64_t launches[HS_PHASE_COUNT] = {0};
 
+  // The step's kernels as a CUDA graph: captured once per key (parameters, inputs, momentum state,
+  // profiling), replayed by later steps with the learning rate written to d_lr first.  The launch
+  // overhead of a step's 20-40 kernels is then paid once; the kernels and their order are the
+  // eager path's.  Invalidated by every call that changes what a step enqueues; HS_STEP_GRAPH=0
+  // keeps every step eager.
+  struct StepGraph {
+    const float* params = nullptr;
+    const float* x = nullptr;
+    const int32_t* y = nullptr;
+    bool mom_valid = false, profiling = false;
+    cudaGraph_t graph = nullptr;
+    cudaGraphExec_t exec = nullptr;
+    struct PhaseNodes { int phase; cudaGraphNode_t a, b; };   // the profile's event-record nodes
+    std::vector<PhaseNodes> phase_nodes;
+    int64_t launches[HS_PHASE_COUNT] = {0};                   // kernel launches of one step, by phase
+    uint64_t last_use = 0;
+  };
+  bool graph_on = true;
+  bool graph_force = false;       // HS_STEP_GRAPH=1: also for the largest steps
+  bool graph_warm = false;        // a step ran eagerly since the last invalidation (kernels loaded)
+  bool capturing = false;         // the step's work is being captured (phase events become nodes)
+  uint64_t graph_clock = 0;
+  std::vector<StepGraph> graphs;  // at most kMaxStepGraphs, least recently used replaced
+  float* d_lr = nullptr;
+  cudaStream_t cap_stream = nullptr;
+
   cudaEvent_t take_event() {
     if (!event_pool.empty()) {
       cudaEvent_t e = event_pool.back();
@@ -192,14 +218,14 @@ class PhaseScope {
   PhaseScope(hs_ctx* c, int phase, cudaStream_t s) : c_(c), phase_(phase), s_(s) {
     if (c_->profiling) {
       a_ = c_->take_event();
-      if (a_) cudaEventRecord(a_, s_);
+      if (a_) record(a_);
     }
   }
   ~PhaseScope() {
     if (c_->profiling && a_) {
       cudaEvent_t b = c_->take_event();
       if (b) {
-        cudaEventRecord(b, s_);
+        record(b);
         c_->pending.push_back({phase_, a_, b});
       }
     }
@@ -207,6 +233,11 @@ class PhaseScope {
   void launched(int n = 1) { c_->launches[phase_] += n; }
 
  private:
+  // under capture the record becomes an event-record node of the step's graph
+  void record(cudaEvent_t e) {
+    if (c_->capturing) cudaEventRecordWithFlags(e, s_, cudaEventRecordExternal);
+    else cudaEventRecord(e, s_);
+  }
   hs_ctx* c_;
   int phase_;
   cudaStream_t s_;

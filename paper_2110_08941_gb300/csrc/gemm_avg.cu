@@ -260,7 +260,7 @@ __global__ void __launch_bounds__(kAvThreads, 1) tc_wgrad_avg_pair_kernel(const 
     const uint32_t buf = smem_u32(sBuf) + (uint32_t)(e * AV_BUF);
     const uint32_t rbase = buf + (uint32_t)(lane * 128);
     const uint32_t tbar = smem_u32(&tload_bar[e]);
-    const float neg_lr = -p.lr;
+    const float neg_lr = -(p.lr_dev ? *p.lr_dev : p.lr);
     int ab = 0;
     uint32_t aph = 0, tph = 0;
     bool ok = true;

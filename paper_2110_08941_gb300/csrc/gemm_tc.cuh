@@ -73,6 +73,7 @@ struct TcGemmParams {
   CUtensorMap tmS;                 // bf16 copy of those weights, written beside theta (tc_make_store_map_bf16_32)
   const float* wavg;               // [groups] averaging weight of group (worker) g, on the device
   float lr;
+  const float* lr_dev;             // non-null: the learning rate is read here (a step replayed from a graph)
   // recipe = 1: momentum mu and weight decay wd in the update, the momentum buffer through tmM
   // (first = 1: it starts as d); tmT, tmM and tmS then have 32-row x 16-column boxes
   // (tc_make_store_map_16)

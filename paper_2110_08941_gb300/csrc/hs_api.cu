@@ -290,11 +290,14 @@ void compute_weights(hs_ctx* c) {
 }
 
 // Apply a new partition (sizes already validated) and push it to the device on `s`.
+void invalidate_step_graphs(hs_ctx* c);
+
 hs_status apply_partition(hs_ctx* c, const std::vector<int32_t>& sizes, const std::vector<double>& cpn,
                           int32_t* index_map_out, cudaStream_t s) {
   const bool changed = (sizes != c->counts);
   c->cp_norm = cpn;
   if (changed) {
+    invalidate_step_graphs(c);   // the plans below change what a step enqueues
     c->counts = sizes;
     c->offsets.assign(c->M + 1, 0);
     for (int m = 0; m < c->M; ++m) c->offsets[m + 1] = c->offsets[m] + sizes[m];
@@ -411,6 +414,8 @@ void free_all(hs_ctx* c) {
   if (c->upd_done) cudaEventDestroy(c->upd_done);
   if (c->dgrad_done) cudaEventDestroy(c->dgrad_done);
   if (c->upd_stream) cudaStreamDestroy(c->upd_stream);
+  f(c->d_lr);
+  if (c->cap_stream) cudaStreamDestroy(c->cap_stream);
 }
 
 bool is_device_ptr(const void* p) {
@@ -498,8 +503,8 @@ hs_status mlp_step_fp32(hs_ctx* c, float* params, const float* x, const int32_t*
 // theta <- theta - lr * sum_m w_m G_m over layer l's parameter range [W_l, b_l] (Section 1).
 // The update of layer l's parameter range [W_l, b_l]; the new bf16 weights go to `shadow` (the
 // step's shadow, or the second shadow while input-gradient products still read the first).
-void update_layer_range(hs_ctx* c, float* params, int l, float lr, cudaStream_t s, int blocks_per_sm,
-                        __nv_bfloat16* shadow = nullptr) {
+void update_layer_range(hs_ctx* c, float* params, int l, float lr, const float* lr_dev, cudaStream_t s,
+                        int blocks_per_sm, __nv_bfloat16* shadow = nullptr) {
   const int64_t start = c->layers[l].w_off;
   const int64_t end = (l + 1 < c->L) ? c->layers[l + 1].w_off : c->P;
   if (!shadow) shadow = c->d_shadow;
@@ -509,24 +514,25 @@ void update_layer_range(hs_ctx* c, float* params, int l, float lr, cudaStream_t 
   hs::launch_reduce_update(params + start, c->d_slabs + start, c->Ps, c->fused_sync ? 1 : c->M,
                            c->fused_sync ? c->d_w_one : c->d_w, lr, end - start,
                            shadow + start, c->debug ? c->d_gdebug + start : nullptr, c->num_sms, s,
-                           blocks_per_sm, c->opt_recipe ? &r : nullptr);
+                           blocks_per_sm, c->opt_recipe ? &r : nullptr, lr_dev);
   ph.launched();
 }
 
 // theta <- theta - lr * sum_m w_m G_m over [start, end) of the slabs (the bias range of a layer whose
 // weights the tile-averaged launch updated; the momentum recipe as in the rest of the update),
 // bf16 copy into `shadow`.
-void update_range(hs_ctx* c, float* params, int64_t start, int64_t end, float lr, cudaStream_t s,
-                  __nv_bfloat16* shadow) {
+void update_range(hs_ctx* c, float* params, int64_t start, int64_t end, float lr, const float* lr_dev,
+                  cudaStream_t s, __nv_bfloat16* shadow) {
   PhaseScope ph(c, HS_PHASE_UPDATE, s);
   hs::UpdateRecipe r{c->opt_recipe ? c->d_mom + start : nullptr, c->opt_momentum, c->opt_weight_decay,
                      c->mom_valid ? 0 : 1};
   hs::launch_reduce_update(params + start, c->d_slabs + start, c->Ps, c->M, c->d_w, lr, end - start, shadow + start,
-                           nullptr, c->num_sms, s, 1, c->opt_recipe ? &r : nullptr);
+                           nullptr, c->num_sms, s, 1, c->opt_recipe ? &r : nullptr, lr_dev);
   ph.launched();
 }
 
-hs_status mlp_step_bf16(hs_ctx* c, float* params, const float* x, const int32_t* y, float lr, cudaStream_t s) {
+hs_status mlp_step_bf16(hs_ctx* c, float* params, const float* x, const int32_t* y, float lr, const float* lr_dev,
+                        cudaStream_t s) {
   const int L = c->L;
   {
     PhaseScope ph(c, HS_PHASE_CAST, s);
@@ -568,6 +574,7 @@ hs_status mlp_step_bf16(hs_ctx* c, float* params, const float* x, const int32_t*
       if (tile) {
         hs::TcGemmParams& w = c->tc_wgrad_avg[l];
         w.lr = lr;
+        w.lr_dev = lr_dev;
         w.mu = c->opt_momentum;
         w.wd = c->opt_weight_decay;
         w.first = c->mom_valid ? 0 : 1;
@@ -603,7 +610,7 @@ hs_status mlp_step_bf16(hs_ctx* c, float* params, const float* x, const int32_t*
     if (tile) {
       // the bias range's update (its weights were updated inside the weight-gradient launch)
       const int64_t end = (l + 1 < L) ? c->layers[l + 1].w_off : c->P;
-      update_range(c, params, ly.b_off, end, lr, s, shadow_l);
+      update_range(c, params, ly.b_off, end, lr, lr_dev, s, shadow_l);
     } else if (c->overlap_update) {
       // Layer l's slabs are complete: its update runs beside the remaining (tensor-core bound)
       // backward products.  Its input-gradient product (next, on the step's stream) still reads
@@ -611,10 +618,10 @@ hs_status mlp_step_bf16(hs_ctx* c, float* params, const float* x, const int32_t*
       // first once the last input-gradient product is done; layer 1 has none and writes in place.
       HS_CUDA(c, cudaEventRecord(c->upd_ready[l], s));
       HS_CUDA(c, cudaStreamWaitEvent(c->upd_stream, c->upd_ready[l], 0));
-      update_layer_range(c, params, l, lr, c->upd_stream, l == 0 ? 4 : 1, shadow_l);
+      update_layer_range(c, params, l, lr, lr_dev, c->upd_stream, l == 0 ? 4 : 1, shadow_l);
       side = true;
     } else {
-      update_layer_range(c, params, l, lr, s, 4, shadow_l);
+      update_layer_range(c, params, l, lr, lr_dev, s, 4, shadow_l);
     }
     if (l > 0) {
       PhaseScope ph(c, HS_PHASE_DGRAD, s);
@@ -637,6 +644,170 @@ hs_status mlp_step_bf16(hs_ctx* c, float* params, const float* x, const int32_t*
     HS_CUDA(c, cudaEventRecord(c->upd_done, c->upd_stream));
     HS_CUDA(c, cudaStreamWaitEvent(s, c->upd_done, 0));
   }
+  return HS_OK;
+}
+
+// The step's kernels after the input handling: per-worker forward and backward passes, the
+// synchronisation and the update.  lr_dev: non-null when the learning rate is read from device
+// memory (a step captured into a graph).
+hs_status step_body(hs_ctx* c, float* params, const float* xd, const int32_t* yd, float lr, const float* lr_dev,
+                    cudaStream_t s) {
+  const bool mlp_bf16 = (c->arch == HS_MLP && c->precision == HS_BF16);
+  hs_status st = c->arch == HS_CNN ? cnn_step(c, params, xd, yd, s)
+                 : mlp_bf16        ? mlp_step_bf16(c, params, xd, yd, lr, lr_dev, s)
+                                   : mlp_step_fp32(c, params, xd, yd, s);
+  if (st != HS_OK) return st;
+  if (!mlp_bf16) {
+    PhaseScope ph(c, HS_PHASE_UPDATE, s);
+    hs::UpdateRecipe r{c->d_mom, c->opt_momentum, c->opt_weight_decay, c->mom_valid ? 0 : 1};
+    hs::launch_reduce_update(params, c->d_slabs, c->Ps, c->fused_sync ? 1 : c->M,
+                             c->fused_sync ? c->d_w_one : c->d_w, lr, c->P,
+                             c->precision == HS_BF16 ? c->d_shadow : nullptr, c->debug ? c->d_gdebug : nullptr,
+                             c->num_sms, s, 4, c->opt_recipe ? &r : nullptr, lr_dev);
+    ph.launched();
+  }
+  return HS_OK;
+}
+
+constexpr size_t kMaxStepGraphs = 4;
+
+void destroy_step_graph(hs_ctx::StepGraph& g) {
+  if (g.exec) cudaGraphExecDestroy(g.exec);   // an in-flight replay is freed on completion
+  if (g.graph) cudaGraphDestroy(g.graph);
+  g.exec = nullptr;
+  g.graph = nullptr;
+}
+
+// Every captured step is stale once plans, flags or the optimizer change.
+void invalidate_step_graphs(hs_ctx* c) {
+  for (auto& g : c->graphs) destroy_step_graph(g);
+  c->graphs.clear();
+  c->graph_warm = false;
+}
+
+void disable_step_graphs(hs_ctx* c) {
+  invalidate_step_graphs(c);
+  c->graph_on = false;
+  cudaGetLastError();
+}
+
+// Capture the step for key `k` on the context's capture stream (nothing runs), instantiate it and
+// note its launches per phase and its profile event nodes.  On any failure the context falls back
+// to eager steps for good (returns false, *st = HS_OK) unless the step itself failed (*st).
+bool capture_step(hs_ctx* c, hs_ctx::StepGraph& k, float* params, const float* xd, const int32_t* yd, float lr,
+                  hs_status* st) {
+  *st = HS_OK;
+  if (!c->d_lr && dalloc(c, &c->d_lr, sizeof(float)) != HS_OK) return false;
+  if (!c->cap_stream && cudaStreamCreateWithFlags(&c->cap_stream, cudaStreamNonBlocking) != cudaSuccess) return false;
+  int64_t before[HS_PHASE_COUNT];
+  for (int i = 0; i < HS_PHASE_COUNT; ++i) before[i] = c->launches[i];
+  const size_t pend0 = c->pending.size();
+  if (cudaStreamBeginCapture(c->cap_stream, cudaStreamCaptureModeRelaxed) != cudaSuccess) return false;
+  c->capturing = true;
+  hs_status body = step_body(c, params, xd, yd, lr, c->d_lr, c->cap_stream);
+  c->capturing = false;
+  cudaGraph_t graph = nullptr;
+  const cudaError_t end = cudaStreamEndCapture(c->cap_stream, &graph);
+  for (int i = 0; i < HS_PHASE_COUNT; ++i) {
+    k.launches[i] = c->launches[i] - before[i];
+    c->launches[i] = before[i];
+  }
+  std::vector<hs_ctx::Rec> recs(c->pending.begin() + (std::ptrdiff_t)pend0, c->pending.end());
+  c->pending.resize(pend0);
+  for (auto& r : recs) {   // nodes of the graph refer to them; replays swap in fresh events
+    c->event_pool.push_back(r.a);
+    c->event_pool.push_back(r.b);
+  }
+  if (body != HS_OK || end != cudaSuccess || !graph) {
+    if (graph) cudaGraphDestroy(graph);
+    *st = body;
+    return false;
+  }
+  cudaGraphExec_t exec = nullptr;
+  if (cudaGraphInstantiate(&exec, graph, 0) != cudaSuccess) {
+    cudaGraphDestroy(graph);
+    return false;
+  }
+  if (!recs.empty()) {
+    size_t n = 0;
+    cudaGraphGetNodes(graph, nullptr, &n);
+    std::vector<cudaGraphNode_t> nodes(n);
+    if (n) cudaGraphGetNodes(graph, nodes.data(), &n);
+    std::vector<std::pair<cudaEvent_t, cudaGraphNode_t>> by_event;
+    for (cudaGraphNode_t nd : nodes) {
+      cudaGraphNodeType t;
+      cudaEvent_t ev = nullptr;
+      if (cudaGraphNodeGetType(nd, &t) == cudaSuccess && t == cudaGraphNodeTypeEventRecord &&
+          cudaGraphEventRecordNodeGetEvent(nd, &ev) == cudaSuccess)
+        by_event.push_back({ev, nd});
+    }
+    auto node_of = [&](cudaEvent_t e) -> cudaGraphNode_t {
+      for (auto& pr : by_event)
+        if (pr.first == e) return pr.second;
+      return nullptr;
+    };
+    for (auto& r : recs) {
+      cudaGraphNode_t a = node_of(r.a), b = node_of(r.b);
+      if (!a || !b) {   // the profile would miss phases: replay without profile is not what was asked
+        cudaGraphExecDestroy(exec);
+        cudaGraphDestroy(graph);
+        return false;
+      }
+      k.phase_nodes.push_back({r.phase, a, b});
+    }
+  }
+  k.graph = graph;
+  k.exec = exec;
+  return true;
+}
+
+// One step through the graph cache: eager until a step has run since the last invalidation, then
+// the key's graph (captured on first use), launched after the learning rate is written to d_lr.
+hs_status step_via_graph(hs_ctx* c, float* params, const float* xd, const int32_t* yd, float lr, cudaStream_t s) {
+  if (!c->graph_warm) {
+    hs_status st = step_body(c, params, xd, yd, lr, nullptr, s);
+    if (st == HS_OK) c->graph_warm = true;
+    return st;
+  }
+  hs_ctx::StepGraph* g = nullptr;
+  for (auto& e : c->graphs)
+    if (e.params == params && e.x == xd && e.y == yd && e.mom_valid == c->mom_valid && e.profiling == c->profiling)
+      g = &e;
+  if (!g) {
+    hs_ctx::StepGraph k;
+    k.params = params;
+    k.x = xd;
+    k.y = yd;
+    k.mom_valid = c->mom_valid;
+    k.profiling = c->profiling;
+    hs_status st = HS_OK;
+    if (!capture_step(c, k, params, xd, yd, lr, &st)) {
+      if (st != HS_OK) return st;
+      disable_step_graphs(c);
+      return step_body(c, params, xd, yd, lr, nullptr, s);
+    }
+    if (c->graphs.size() >= kMaxStepGraphs) {
+      size_t lru = 0;
+      for (size_t i = 1; i < c->graphs.size(); ++i)
+        if (c->graphs[i].last_use < c->graphs[lru].last_use) lru = i;
+      destroy_step_graph(c->graphs[lru]);
+      c->graphs.erase(c->graphs.begin() + (std::ptrdiff_t)lru);
+    }
+    c->graphs.push_back(std::move(k));
+    g = &c->graphs.back();
+  }
+  g->last_use = ++c->graph_clock;
+  hs::launch_set_scalar(c->d_lr, lr, s);
+  c->launches[HS_PHASE_UPDATE] += 1;
+  for (auto& pn : g->phase_nodes) {
+    cudaEvent_t a = c->take_event(), b = c->take_event();
+    if (!a || !b) return fail(c, HS_ERR_CUDA, "profile events");
+    HS_CUDA(c, cudaGraphExecEventRecordNodeSetEvent(g->exec, pn.a, a));
+    HS_CUDA(c, cudaGraphExecEventRecordNodeSetEvent(g->exec, pn.b, b));
+    c->pending.push_back({pn.phase, a, b});
+  }
+  HS_CUDA(c, cudaGraphLaunch(g->exec, s));
+  for (int i = 0; i < HS_PHASE_COUNT; ++i) c->launches[i] += g->launches[i];
   return HS_OK;
 }
 
@@ -711,6 +882,12 @@ hs_status hs_init(const hs_model_desc* model, int32_t M, const double* compute_w
   c->M = M;
   c->N = global_batch;
   c->L = model->arch == HS_MLP ? model->n_layers : 0;
+  // The step's own graph pays where launches outlast the GPU work; a step of more than 1e11
+  // parameter-samples (P * N: the 4096-8192-8192-1000 workload's 1.8e12 is 5.6 ms of GPU work for
+  // about 0.1 ms of host launches) keeps eager launches.  HS_STEP_GRAPH=0 / =1 force either.
+  const char* sg = getenv("HS_STEP_GRAPH");
+  c->graph_on = !(sg && !strcmp(sg, "0"));
+  c->graph_force = sg && !strcmp(sg, "1");
   const bool bf16 = (c->precision == HS_BF16);
   if (c->arch == HS_MLP) {
     if (bf16) {
@@ -785,6 +962,7 @@ hs_status hs_init(const hs_model_desc* model, int32_t M, const double* compute_w
     c->in_features = (int64_t)dims[0] * dims[1] * dims[2];
   }
   c->Ps = round_up(c->P, 64);
+  if (!c->graph_force && (double)c->P * (double)c->N > 1e11) c->graph_on = false;
 
   const size_t N = (size_t)c->N;
   const size_t es = c->act_elem();
@@ -1035,20 +1213,13 @@ hs_status hs_step(hs_ctx* c, float* params, const void* x, const int32_t* y, con
     hs_status r = dalloc(c, &c->d_gdebug, sizeof(float) * c->Ps);
     if (r != HS_OK) return r;
   }
-  const bool mlp_bf16 = (c->arch == HS_MLP && c->precision == HS_BF16);
-  hs_status st = c->arch == HS_CNN ? cnn_step(c, params, xd, yd, s)
-                 : mlp_bf16        ? mlp_step_bf16(c, params, xd, yd, lr, s)
-                                   : mlp_step_fp32(c, params, xd, yd, s);
+  // A caller capturing its own graph gets the step's kernels enqueued as they are.
+  cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+  const bool caller_capture = cudaStreamIsCapturing(s, &cap) != cudaSuccess || cap != cudaStreamCaptureStatusNone;
+  if (caller_capture) cudaGetLastError();
+  hs_status st = (c->graph_on && !caller_capture) ? step_via_graph(c, params, xd, yd, lr, s)
+                                                  : step_body(c, params, xd, yd, lr, nullptr, s);
   if (st != HS_OK) return st;
-  if (!mlp_bf16) {
-    PhaseScope ph(c, HS_PHASE_UPDATE, s);
-    hs::UpdateRecipe r{c->d_mom, c->opt_momentum, c->opt_weight_decay, c->mom_valid ? 0 : 1};
-    hs::launch_reduce_update(params, c->d_slabs, c->Ps, c->fused_sync ? 1 : c->M,
-                             c->fused_sync ? c->d_w_one : c->d_w, lr, c->P,
-                             c->precision == HS_BF16 ? c->d_shadow : nullptr, c->debug ? c->d_gdebug : nullptr,
-                             c->num_sms, s, 4, c->opt_recipe ? &r : nullptr);
-    ph.launched();
-  }
   if (slot >= 0) {
     HS_CUDA(c, cudaEventRecord(c->slot_consumed[slot], s));
     c->slot_pending[slot] = false;
@@ -1138,6 +1309,7 @@ hs_status hs_set_fused_sync(hs_ctx* c, int32_t enable) {
   if (!c) return HS_ERR_INVALID_ARG;
   c->err.clear();
   if (c->arch != HS_MLP) return fail(c, HS_ERR_UNSUPPORTED, "the slab-free formulation is built for the MLP only");
+  if (c->fused_sync != (enable != 0)) invalidate_step_graphs(c);
   c->fused_sync = enable != 0;
   return HS_OK;
 }
@@ -1164,6 +1336,7 @@ hs_status hs_set_optimizer(hs_ctx* c, float momentum, float weight_decay) {
   if (!std::isfinite(momentum) || !std::isfinite(weight_decay) || momentum < 0.f || momentum >= 1.f ||
       weight_decay < 0.f)
     return fail(c, HS_ERR_INVALID_ARG, "momentum must be in [0, 1) and weight_decay >= 0");
+  invalidate_step_graphs(c);
   if (momentum == 0.f && weight_decay == 0.f) {
     c->opt_recipe = false;
     return HS_OK;
@@ -1202,6 +1375,7 @@ double hs_cosine_lr(double eta0, double eta_min, int64_t t, int64_t T) {
 
 hs_status hs_set_debug(hs_ctx* c, int32_t enable) {
   if (!c) return HS_ERR_INVALID_ARG;
+  if (c->debug != (enable != 0)) invalidate_step_graphs(c);
   c->debug = enable != 0;
   return HS_OK;
 }
@@ -1238,6 +1412,7 @@ hs_status hs_worker_losses(hs_ctx* c, float* losses_out) {
 void hs_destroy(hs_ctx* c) {
   if (!c) return;
   cudaDeviceSynchronize();
+  invalidate_step_graphs(c);
   free_all(c);
   delete c;
 }

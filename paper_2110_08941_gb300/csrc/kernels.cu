@@ -402,10 +402,13 @@ __device__ __forceinline__ float apply_update(float t, float g, float lr, float*
 template <bool kRecipe>
 __global__ void __launch_bounds__(512) reduce_update_kernel(
     float* __restrict__ theta, const float* __restrict__ slabs, int64_t Ps, int M,
-    const float* __restrict__ w, float lr, int64_t P, __nv_bfloat16* __restrict__ shadow,
-    float* __restrict__ gdebug, float* __restrict__ mbuf, float mu, float wd, int first) {
+    const float* __restrict__ w, float lr_arg, const float* __restrict__ lr_dev, int64_t P,
+    __nv_bfloat16* __restrict__ shadow, float* __restrict__ gdebug, float* __restrict__ mbuf, float mu, float wd,
+    int first) {
   pdl_wait();
   pdl_trigger();
+  // the step's learning rate: the argument, or (a step replayed from a CUDA graph) device memory
+  const float lr = lr_dev ? __ldg(lr_dev) : lr_arg;
   // The weights stay in global memory (read through the read-only cache): no shared memory, so
   // blocks of this kernel can share an SM with a resident tensor-core GEMM CTA.
   const float* __restrict__ sw = w;
@@ -474,19 +477,23 @@ __global__ void __launch_bounds__(512) reduce_update_kernel(
 
 void launch_reduce_update(float* theta, const float* slabs, int64_t Ps, int M, const float* d_w,
                           float lr, int64_t P, __nv_bfloat16* shadow, float* gdebug, int num_sms,
-                          cudaStream_t s, int blocks_per_sm, const UpdateRecipe* recipe) {
+                          cudaStream_t s, int blocks_per_sm, const UpdateRecipe* recipe, const float* lr_dev) {
   const int threads = 512;
   int64_t blocks = (P / 4 + threads - 1) / threads;
   const int64_t cap = (int64_t)num_sms * blocks_per_sm;
   if (blocks > cap) blocks = cap;
   if (blocks < 1) blocks = 1;
   if (recipe && recipe->buf)
-    launch_pdl(reduce_update_kernel<true>, (int)blocks, threads, 0, s, theta, slabs, Ps, M, d_w, lr, P, shadow, gdebug,
-                                                               recipe->buf, recipe->momentum, recipe->weight_decay,
-                                                               recipe->first);
+    launch_pdl(reduce_update_kernel<true>, (int)blocks, threads, 0, s, theta, slabs, Ps, M, d_w, lr, lr_dev, P, shadow,
+               gdebug, recipe->buf, recipe->momentum, recipe->weight_decay, recipe->first);
   else
-    launch_pdl(reduce_update_kernel<false>, (int)blocks, threads, 0, s, theta, slabs, Ps, M, d_w, lr, P, shadow, gdebug,
-                                                                nullptr, 0.f, 0.f, 0);
+    launch_pdl(reduce_update_kernel<false>, (int)blocks, threads, 0, s, theta, slabs, Ps, M, d_w, lr, lr_dev, P, shadow,
+               gdebug, nullptr, 0.f, 0.f, 0);
 }
+
+// *dst = v: the learning rate of a step replayed from a CUDA graph, written ahead of the replay.
+__global__ void set_scalar_kernel(float* dst, float v) { *dst = v; }
+
+void launch_set_scalar(float* dst, float v, cudaStream_t s) { set_scalar_kernel<<<1, 1, 0, s>>>(dst, v); }
 
 }  // namespace hs
