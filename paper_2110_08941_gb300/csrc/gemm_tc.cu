@@ -5,8 +5,9 @@
 //   input grad    dH    = (delta_l W_l) * 1[H_{l-1} > 0]   A: K-major, B: MN-major
 //   weight grad   G_m   = delta_l[seg_m]^T H_{l-1}[seg_m]  A: MN-major, B: MN-major, one group per worker
 //
-// CTA layout (192 threads, one CTA per SM):
-//   warp 0      one elected thread issues TMA tile loads into a 4-stage shared-memory ring
+// CTA layout (192 threads, one CTA per SM; 224 for convolution products):
+//   warp 0      one elected thread issues TMA tile loads into a 4-stage shared-memory ring (with
+//               warp 6 for convolution products, each issuing every other box of a k-block)
 //   warp 1      owns the tensor-memory allocation; one elected thread issues tcgen05.mma
 //   warps 2..5  epilogue: tcgen05.ld from tensor memory, fused bias/ReLU/mask, global stores
 // Two 128x256 fp32 accumulators (512 TMEM columns) let the epilogue of one tile overlap the
@@ -30,9 +31,15 @@ constexpr int B_STAGE = BN * BK * 2;                 // 32 KB
 constexpr uint32_t STAGE_TX = A_STAGE + B_STAGE;     // bytes landed per stage
 constexpr int kThreads = 192;
 constexpr uint32_t kTmemCols = 2 * BN;               // two accumulator buffers
+// Convolution products: a second TMA producer warp (warp 6) shares each k-block's boxes with warp 0
+// (their implicit operands come in 8 KB 4-D boxes, slower to issue than the MMAs consume them).
+constexpr int kConvProducers1 = 2;
+template <bool CONV>
+constexpr int threads_of() { return kThreads + (CONV ? 32 * (kConvProducers1 - 1) : 0); }
 
 template <int EPI, bool A_MN, bool B_MN, bool CONV>
-__global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_constant__ TcGemmParams p) {
+__global__ void __launch_bounds__(threads_of<CONV>(), 1) tc_gemm_kernel(const __grid_constant__ TcGemmParams p) {
+  constexpr int NP = CONV ? kConvProducers1 : 1;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sA = smem;
@@ -74,9 +81,12 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
 
   const int total = p.groups * ksplit_of(p) * p.tiles_m * p.tiles_n;
 
-  if (warp == 0) {
+  const int prod = (warp == 0) ? 0 : (NP > 1 && warp >= 6) ? warp - 6 + 1 : -1;
+  if (prod >= 0) {
     if (lane == 0) {
-      // ------------------------------------------------------------ TMA producer
+      // ------------------------------------------------------------ TMA producers
+      // A k-block's boxes, A then B, numbered in order; producer `prod` issues those whose number is
+      // prod mod NP (producer 0 also sets the stage's expected bytes).
       int s = 0;
       uint32_t ph = 0;
       int last_g = -1;
@@ -90,39 +100,60 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
           tma_prefetch_desc(tb);
           last_g = w.g;
         }
+        // implicit patch rows: the output-pixel part of the A boxes and the patch-column part of
+        // the B boxes once per tile
+        ConvRowPart arow[BM / 64];
+        ConvColPart bcol[BN / 64];
+        if (CONV && p.conv_a) {
+#pragma unroll
+          for (int j = 0; j < BM / 64; ++j)
+            arow[j] = p.conv_a == 2 ? subpixel_row_part(p.conv, c.tm * BM + 64 * j)
+                                    : conv_row_part(p.conv, c.tm * BM + 64 * j);
+        }
+        if (CONV && B_MN && p.conv_b) {
+#pragma unroll
+          for (int j = 0; j < BN / 64; ++j)
+            if (c.tn * BN + 64 * j < p.conv.ones_col) bcol[j] = conv_col_part(p.conv, c.tn * BN + 64 * j);
+        }
         bool ok = true;
         for (int kb = w.kb_lo; kb < w.kb_hi; ++kb) {
           if (!mbar_wait(smem_u32(&empty_bar[s]), ph ^ 1u, abort_flag)) { ok = false; break; }
           const uint32_t fb = smem_u32(&full_bar[s]);
-          mbar_expect_tx(fb, STAGE_TX);
+          if (prod == 0) mbar_expect_tx(fb, STAGE_TX);
           const int k0 = kb * BK;
           const uint32_t a_dst = smem_u32(sA + s * A_STAGE);
           const uint32_t b_dst = smem_u32(sB + s * B_STAGE);
+          int box = 0;
           if (A_MN) {
 #pragma unroll
-            for (int j = 0; j < BM / 64; ++j) tma_load_2d(a_dst + j * MN_CHUNK, ta, c.tm * BM + 64 * j, k0, fb);
-          } else {
-            if (CONV && p.conv_a) {
+            for (int j = 0; j < BM / 64; ++j)
+              if (box++ % NP == prod) tma_load_2d(a_dst + j * MN_CHUNK, ta, c.tm * BM + 64 * j, k0, fb);
+          } else if (CONV && p.conv_a) {
+            ConvColPart kc;
+            if (NP == 1 || prod < BM / 64)
+              kc = p.conv_a == 2 ? subpixel_col_part(p.conv, w.g, k0) : conv_col_part(p.conv, k0);
 #pragma unroll
-              for (int j = 0; j < BM / 64; ++j) {
+            for (int j = 0; j < BM / 64; ++j)
+              if (box++ % NP == prod) {
                 int cc[4];
-                if (p.conv_a == 2) subpixel_box_coords(p.conv, w.g, c.tm * BM + 64 * j, k0, cc);
-                else conv_box_coords(p.conv, c.tm * BM + 64 * j, k0, cc);
+                conv_coords(arow[j], kc, cc);
                 tma_load_4d(a_dst + j * MN_CHUNK, ta, cc, fb);
               }
-            } else {
-              tma_load_2d(a_dst, ta, k0, c.tm * BM, fb);
-            }
+          } else {
+            if (box++ % NP == prod) tma_load_2d(a_dst, ta, k0, c.tm * BM, fb);
           }
           if (B_MN) {
+            ConvRowPart krow;
+            if (CONV && p.conv_b) krow = conv_row_part(p.conv, k0);
 #pragma unroll
             for (int j = 0; j < BN / 64; ++j) {
+              if (box++ % NP != prod) continue;
               const int col = c.tn * BN + 64 * j;
               if (!CONV || !p.conv_b) {
                 tma_load_2d(b_dst + j * MN_CHUNK, tb, col, k0, fb);
               } else if (col < p.conv.ones_col) {
                 int cc[4];
-                conv_box_coords(p.conv, k0, col, cc);
+                conv_coords(krow, bcol[j], cc);
                 tma_load_4d(b_dst + j * MN_CHUNK, tb, cc, fb);
               } else {
                 tma_load_2d(b_dst + j * MN_CHUNK, &p.tmOnes, col - p.conv.ones_col, 0, fb);
@@ -131,7 +162,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
           } else {
 #pragma unroll
             for (int j = 0; j < BN / kTcBoxB; ++j)
-              tma_load_2d(b_dst + j * (kTcBoxB * BK * 2), tb, k0, c.tn * BN + kTcBoxB * j, fb);
+              if (box++ % NP == prod) tma_load_2d(b_dst + j * (kTcBoxB * BK * 2), tb, k0, c.tn * BN + kTcBoxB * j, fb);
           }
           if (++s == S) { s = 0; ph ^= 1u; }
         }
@@ -283,7 +314,7 @@ cudaError_t launch_variant(const TcGemmParams& p, int grid, cudaStream_t s) {
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;   // see grid_dependency_wait
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.gridDim = dim3(grid, 1, 1);
-  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.blockDim = dim3(threads_of<CONV>(), 1, 1);
   cfg.dynamicSmemBytes = kTcSmemBytes;
   cfg.stream = s;
   cfg.attrs = attr;

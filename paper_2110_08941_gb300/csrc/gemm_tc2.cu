@@ -5,9 +5,11 @@
 // bandwidth is what the fp32 weight-gradient epilogue needs.  Same products and epilogues as
 // gemm_tc.cu (forward, input gradient, per-worker grouped weight gradient of Eq. 1's g^m).
 //
-// Roles (192 threads per CTA, one CTA per SM, clusters of 2):
+// Roles (64 + 32 x epilogue warps threads per CTA, one more warp for convolution products; one
+// CTA per SM, clusters of 2):
 //   warp 0      (both CTAs) TMA loads of the CTA's A and B halves; completion is signalled on the
-//               leader CTA's stage barrier (the .cta_group::2 form of the bulk tensor copy)
+//               leader CTA's stage barrier (the .cta_group::2 form of the bulk tensor copy); for
+//               convolution products the warp after the epilogue warps issues every other box
 //   warp 1      (both CTAs) the collective tensor-memory allocation; in the leader CTA one thread
 //               issues the pair MMAs and commits them to both CTAs' barriers (multicast)
 //   warps 2..5  (both CTAs) epilogue of the CTA's 128 accumulator rows; each warp reports the
@@ -34,7 +36,7 @@ constexpr int A_HALF = HM * BK * 2;                // 16 KB
 // columns; with 128-wide tiles (kAlt) they are two groups of four, each draining every other tile
 // (one accumulator buffer each), so two tiles' epilogues run at once even where the product is
 // only 64 wide.  Eight epilogue warps cost stages to fit their staging buffers.
-template <int TN, int EW>
+template <int TN, int EW, int NP = 1>
 struct PairCfg {
   static constexpr int PN = TN;
   static constexpr int HN = TN / 2;
@@ -42,7 +44,7 @@ struct PairCfg {
   static constexpr int STAGE2 = A_HALF + B_HALF;
   static constexpr bool kAlt = (TN == 128 && EW == 8);
   static constexpr int S2 = TN == 256 ? (EW == 8 ? 5 : 6) : (EW == 8 ? 6 : 8);
-  static constexpr int kThreads = 64 + 32 * EW;
+  static constexpr int kThreads = 64 + 32 * EW + 32 * (NP - 1);   // NP TMA producer warps
   static constexpr uint32_t PAIR_TX = 2 * STAGE2;   // bytes landing per stage on the leader's barrier
   static constexpr uint32_t kTmemCols2 = 2 * TN;
   static constexpr int kStaging = EW * 8192;         // two 32-row x 128-byte buffers per epilogue warp
@@ -53,10 +55,16 @@ struct PairCfg {
   static_assert(EW == 4 || EW == 8, "epilogue warps");
 };
 
+// Convolution products keep two TMA producer warps busy: their operands come in 8 KB 4-D boxes
+// (one output-pixel block of one tap each) whose issue, one thread at a time, took longer than the
+// k-block's MMAs.  The producers split each k-block's boxes round-robin.
+constexpr int kConvProducers = 2;
+
 template <int EPI, bool A_MN, bool B_MN, bool CONV, int TN, int EW>
-__global__ void __launch_bounds__(PairCfg<TN, EW>::kThreads, 1)
+__global__ void __launch_bounds__(PairCfg<TN, EW, CONV ? kConvProducers : 1>::kThreads, 1)
     tc_gemm_pair_kernel(const __grid_constant__ TcGemmParams p) {
-  using Cfg = PairCfg<TN, EW>;
+  constexpr int NP = CONV ? kConvProducers : 1;
+  using Cfg = PairCfg<TN, EW, NP>;
   constexpr int PN = Cfg::PN, HN = Cfg::HN, S2 = Cfg::S2, STAGE2 = Cfg::STAGE2;
   constexpr uint32_t PAIR_TX = Cfg::PAIR_TX, kTmemCols2 = Cfg::kTmemCols2;
   extern __shared__ uint8_t smem_raw[];
@@ -104,9 +112,13 @@ __global__ void __launch_bounds__(PairCfg<TN, EW>::kThreads, 1)
   const int pair_id = blockIdx.x >> 1;
   const int n_pairs = gridDim.x >> 1;
 
-  if (warp == 0) {
+  // TMA producer warps: warp 0 and, for convolution products, the warps after the epilogue's
+  const int prod = (warp == 0) ? 0 : (NP > 1 && warp >= 2 + EW) ? warp - (2 + EW) + 1 : -1;
+  if (prod >= 0) {
     if (lane == 0) {
-      // ------------------------------------------------------------ TMA producer (both CTAs)
+      // ------------------------------------------------------------ TMA producers (both CTAs)
+      // A k-block's boxes, A half then B half, numbered in order; producer `prod` issues those whose
+      // number is prod mod NP (producer 0 also sets the leader's expected bytes).
       int s = 0;
       uint32_t ph = 0;
       int last_g = -1;
@@ -122,47 +134,69 @@ __global__ void __launch_bounds__(PairCfg<TN, EW>::kThreads, 1)
         }
         const int m0 = c.tm * PM + (int)rank * HM;
         const int n0 = c.tn * PN + (int)rank * HN;
+        // implicit patch rows: the output-pixel part of the A boxes once per tile, the patch-column
+        // part of the B boxes once per tile
+        ConvRowPart arow[HM / 64];
+        ConvColPart bcol[HN / 64];
+        if (CONV && p.conv_a) {
+#pragma unroll
+          for (int j = 0; j < HM / 64; ++j)
+            arow[j] = p.conv_a == 2 ? subpixel_row_part(p.conv, m0 + 64 * j) : conv_row_part(p.conv, m0 + 64 * j);
+        }
+        if (CONV && B_MN && p.conv_b) {
+#pragma unroll
+          for (int j = 0; j < HN / 64; ++j)
+            if (n0 + 64 * j < p.conv.ones_col) bcol[j] = conv_col_part(p.conv, n0 + 64 * j);
+        }
         bool ok = true;
         for (int kb = w.kb_lo; kb < w.kb_hi; ++kb) {
           if (!mbar_wait(smem_u32(&empty_bar[s]), ph ^ 1u, abort_flag)) { ok = false; break; }
           const uint32_t fb_local = smem_u32(&full_bar[s]);
           const uint32_t fb = map_to_rank(fb_local, 0);
-          if (leader) mbar_expect_tx(fb_local, PAIR_TX);
+          if (prod == 0 && leader) mbar_expect_tx(fb_local, PAIR_TX);
           const int k0 = kb * BK;
           const uint32_t a_dst = smem_u32(smem + s * STAGE2);
           const uint32_t b_dst = a_dst + A_HALF;
+          int box = 0;
           // the A half: two 64-column boxes (MN-major), two 64-pixel boxes (implicit patch rows) or
           // one 128-row box (K-major)
           if (A_MN) {
 #pragma unroll
-            for (int j = 0; j < HM / 64; ++j) tma_load_2d_pair(a_dst + j * MN_CHUNK, ta, m0 + 64 * j, k0, fb);
+            for (int j = 0; j < HM / 64; ++j)
+              if (box++ % NP == prod) tma_load_2d_pair(a_dst + j * MN_CHUNK, ta, m0 + 64 * j, k0, fb);
           } else if (CONV && p.conv_a) {
+            ConvColPart kc;
+            if (NP == 1 || prod < HM / 64)
+              kc = p.conv_a == 2 ? subpixel_col_part(p.conv, w.g, k0) : conv_col_part(p.conv, k0);
 #pragma unroll
-            for (int j = 0; j < HM / 64; ++j) {
-              int cc[4];
-              if (p.conv_a == 2) subpixel_box_coords(p.conv, w.g, m0 + 64 * j, k0, cc);
-              else conv_box_coords(p.conv, m0 + 64 * j, k0, cc);
-              tma_load_4d_pair(a_dst + j * MN_CHUNK, ta, cc, fb);
-            }
+            for (int j = 0; j < HM / 64; ++j)
+              if (box++ % NP == prod) {
+                int cc[4];
+                conv_coords(arow[j], kc, cc);
+                tma_load_4d_pair(a_dst + j * MN_CHUNK, ta, cc, fb);
+              }
           } else {
-            tma_load_2d_pair(a_dst, ta, k0, m0, fb);
+            if (box++ % NP == prod) tma_load_2d_pair(a_dst, ta, k0, m0, fb);
           }
           if (B_MN) {
+            ConvRowPart krow;
+            if (CONV && p.conv_b) krow = conv_row_part(p.conv, k0);
 #pragma unroll
             for (int j = 0; j < HN / 64; ++j) {
+              if (box++ % NP != prod) continue;
               const int col = n0 + 64 * j;
               if (!CONV || !p.conv_b) {
                 tma_load_2d_pair(b_dst + j * MN_CHUNK, tb, col, k0, fb);
               } else if (col < p.conv.ones_col) {
                 int cc[4];
-                conv_box_coords(p.conv, k0, col, cc);
+                conv_coords(krow, bcol[j], cc);
                 tma_load_4d_pair(b_dst + j * MN_CHUNK, tb, cc, fb);
               } else {
                 tma_load_2d_pair(b_dst + j * MN_CHUNK, &p.tmOnes, col - p.conv.ones_col, 0, fb);
               }
             }
           } else {
-            tma_load_2d_pair(b_dst, tb, k0, n0, fb);
+            if (box++ % NP == prod) tma_load_2d_pair(b_dst, tb, k0, n0, fb);
           }
           if (++s == S2) { s = 0; ph ^= 1u; }
         }
@@ -329,7 +363,8 @@ template <int EPI, bool A_MN, bool B_MN, bool CONV, int TN = 256, int EW = 4>
 cudaError_t launch_pair_variant(const TcGemmParams& p, int pairs_wanted, int num_sms, cudaStream_t s) {
   static bool configured = false;
   static int max_clusters = 0;
-  constexpr int kSmem2 = PairCfg<TN, EW>::kSmem2;
+  using Cfg = PairCfg<TN, EW, CONV ? kConvProducers : 1>;
+  constexpr int kSmem2 = Cfg::kSmem2;
   auto kern = tc_gemm_pair_kernel<EPI, A_MN, B_MN, CONV, TN, EW>;
   cudaLaunchConfig_t cfg = {};
   cudaLaunchAttribute attr[2];
@@ -339,7 +374,7 @@ cudaError_t launch_pair_variant(const TcGemmParams& p, int pairs_wanted, int num
   attr[0].val.clusterDim.z = 1;
   attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;   // see grid_dependency_wait
   attr[1].val.programmaticStreamSerializationAllowed = 1;
-  cfg.blockDim = dim3(PairCfg<TN, EW>::kThreads, 1, 1);
+  cfg.blockDim = dim3(Cfg::kThreads, 1, 1);
   cfg.dynamicSmemBytes = kSmem2;
   cfg.stream = s;
   cfg.attrs = attr;

@@ -101,6 +101,43 @@ __device__ __forceinline__ void subpixel_box_coords(const TcConvGeom& g, int cls
   c[2] = a + ((ph && th == 0) ? 1 : 0);
   c[3] = img;
 }
+// The same coordinates in two parts, so a producer forms each part once per tile or per k-block
+// instead of per box: the output-pixel part (image, first input row = stride * output row; for the
+// sub-pixel product the class-grid row) and the patch-column part (channel block, column and row
+// offsets of the tap).  Box coordinates: {c0, dw, h + dh, img}.
+struct ConvRowPart { int img, h; };
+struct ConvColPart { int c0, dw, dh; };
+__device__ __forceinline__ ConvRowPart conv_row_part(const TcConvGeom& g, int row) {
+  const int img = row / g.hw;
+  const int ho = (row - img * g.hw) / g.Wo;
+  return {img, g.stride * ho};
+}
+__device__ __forceinline__ ConvColPart conv_col_part(const TcConvGeom& g, int kcol) {
+  const int blk = kcol >> 6;
+  const int tap = blk / g.cblocks;
+  const int cb = blk - tap * g.cblocks;
+  return {cb * 64, tap % 3 - 1, tap / 3 - 1};
+}
+__device__ __forceinline__ ConvRowPart subpixel_row_part(const TcConvGeom& g, int row) {
+  const int img = row / g.hw;
+  return {img, (row - img * g.hw) / g.Wo};
+}
+__device__ __forceinline__ ConvColPart subpixel_col_part(const TcConvGeom& g, int cls, int kcol) {
+  const int blk = kcol >> 6;
+  const int t = blk / g.cblocks;
+  const int cb = blk - t * g.cblocks;
+  const int ph = cls >> 1, pw = cls & 1;
+  const int nw = pw ? 2 : 1;
+  const int th = t / nw, tw = t - th * nw;
+  return {cb * 64, (pw && tw == 0) ? 1 : 0, (ph && th == 0) ? 1 : 0};
+}
+__device__ __forceinline__ void conv_coords(const ConvRowPart& r, const ConvColPart& k, int (&c)[4]) {
+  c[0] = k.c0;
+  c[1] = k.dw;
+  c[2] = r.h + k.dh;
+  c[3] = r.img;
+}
+
 __device__ __forceinline__ void tma_store_4d(const CUtensorMap* tm, uint32_t src, const int (&c)[4]) {
   asm volatile("cp.async.bulk.tensor.4d.global.shared::cta.bulk_group [%0, {%1, %2, %3, %4}], [%5];"
                ::"l"(reinterpret_cast<uint64_t>(tm)), "r"(c[0]), "r"(c[1]), "r"(c[2]), "r"(c[3]), "r"(src)
