@@ -361,6 +361,137 @@ __global__ void splitk_reduce_kernel(const float* __restrict__ partial, int rows
     slabs[(int64_t)m * Ps + b_off + co] = acc;
 }
 
+// The update of reduce_update_kernel (Section 1; Section 5's recipe with kRecipe), for the fused CNN update.
+template <bool kRecipe>
+__device__ __forceinline__ float apply_update_cnn(float t, float g, float lr, float* mb, float mu, float wd, int first) {
+  if (!kRecipe) return fmaf(-lr, g, t);
+  const float d = fmaf(wd, t, g);
+  const float b = first ? d : fmaf(mu, *mb, d);
+  *mb = b;
+  return fmaf(-lr, b, t);
+}
+
+// The CNN step's synchronisation and update in one pass (Section 1; Section 4.2 for the weights;
+// Section 5's momentum and weight decay with kRecipe): for every parameter, worker m's gradient is
+// the sum of its split-K parts in part order (as splitk_reduce_kernel forms it), g = sum_m w_m g^m
+// in worker order and theta's update as in reduce_update_kernel - the same fp32 operations in the
+// same order, so the same bits - and the new value goes to theta, its bf16 shadow and the bf16
+// copies the next step's products read: the tap-major rows of the forward (wperm) and the
+// sub-pixel class matrices of the input gradient (wsub).  One work item per (output channel,
+// column of the partials): columns are tap-major (tap * Cin + ci) as the products leave them, the
+// ones column 9 * Cin holds the bias gradient; the fc layer's columns are its inputs, its bias
+// gradients sit in the per-worker slabs.
+struct CnnUpdLayer {
+  const float* partial;       // [parts][rows][ldp]
+  const int32_t* begin;       // [M + 1] worker m's parts are [begin[m], begin[m + 1])
+  int rows, ldp, cols, cin;   // cols: weight columns (+ the ones column for a convolution); cin 0: fc
+  int64_t w_off, b_off, first;   // theta offsets; first work item of the layer
+  __nv_bfloat16* wperm;       // tap-major bf16 copy [rows][Kp] (convolutions)
+  int Kp;
+  __nv_bfloat16* wsub;        // sub-pixel class copy (stride-2 convolutions whose input gradient is sub-pixel)
+};
+struct CnnUpdArgs {
+  CnnUpdLayer layer[4];
+  int block_first[5];         // first block of each layer's items, then of the fc bias
+  int64_t items;              // work items of the four layers
+  int64_t fc_b_off;           // the fc bias: C items after them, gradients from the slabs
+  int C;
+  const float* slabs;
+  int64_t Ps;
+};
+
+// One layer's items for one block: the layer is the block's (blocks are assigned to layers in
+// order), read into registers through a switch so the kernel never indexes its parameter array
+// at run time.
+template <bool kRecipe>
+__device__ __forceinline__ void cnn_update_item(const CnnUpdLayer& L, int64_t it, float* __restrict__ theta, int M,
+                                                const float* __restrict__ w, float lr,
+                                                __nv_bfloat16* __restrict__ shadow, float* __restrict__ mbuf,
+                                                float mu, float wd, int first) {
+  const int co = (int)(it / L.cols);
+  const int pc = (int)(it - (int64_t)co * L.cols);   // column of the partials
+  int tap = 0, ci = 0;
+  int64_t j;
+  if (L.cin) {
+    if (pc < 9 * L.cin) {
+      tap = pc / L.cin;
+      ci = pc - tap * L.cin;
+      j = L.w_off + ((int64_t)co * L.cin + ci) * 9 + tap;
+    } else {
+      j = L.b_off + co;
+    }
+  } else {
+    j = L.w_off + (int64_t)co * L.cols + pc;
+  }
+  const int64_t part_stride = (int64_t)L.rows * L.ldp;
+  const float* col = L.partial + (int64_t)co * L.ldp + pc;
+  float acc = 0.f;
+  for (int m = 0; m < M; ++m) {
+    // worker m's parts summed in part order; eight loads in flight, added in the same order
+    float gm = 0.f;
+    int c = __ldg(L.begin + m);
+    const int ce = __ldg(L.begin + m + 1);
+    for (; c + 8 <= ce; c += 8) {
+      float v[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) v[u] = __ldcs(col + (int64_t)(c + u) * part_stride);
+#pragma unroll
+      for (int u = 0; u < 8; ++u) gm += v[u];
+    }
+    for (; c < ce; ++c) gm += __ldcs(col + (int64_t)c * part_stride);
+    acc = fmaf(__ldg(w + m), gm, acc);
+  }
+  const float t = apply_update_cnn<kRecipe>(theta[j], acc, lr, kRecipe ? mbuf + j : nullptr, mu, wd, first);
+  theta[j] = t;
+  const __nv_bfloat16 tb = __float2bfloat16_rn(t);
+  shadow[j] = tb;
+  if (L.cin && pc < 9 * L.cin) {
+    L.wperm[(int64_t)co * L.Kp + pc] = tb;
+    if (L.wsub) {
+      const int kh = tap / 3, kw = tap % 3;
+      const int ph = kh != 1, pw = kw != 1;
+      const int th = (ph && kh == 2) ? 1 : 0, tw = (pw && kw == 2) ? 1 : 0;
+      const int t2 = th * (pw ? 2 : 1) + tw;
+      const int cls = 2 * ph + pw;
+      const int64_t class_off = (cls == 0 ? 0 : cls == 1 ? 1 : cls == 2 ? 3 : 5) * (int64_t)L.rows * L.cin;
+      L.wsub[class_off + ((int64_t)t2 * L.rows + co) * L.cin + ci] = tb;
+    }
+  }
+}
+
+template <bool kRecipe>
+__global__ void __launch_bounds__(256) cnn_update_kernel(const CnnUpdArgs a, float* __restrict__ theta, int M,
+                                                         const float* __restrict__ w, float lr_arg,
+                                                         const float* __restrict__ lr_dev,
+                                                         __nv_bfloat16* __restrict__ shadow, float* __restrict__ mbuf,
+                                                         float mu, float wd, int first) {
+  pdl_wait();
+  pdl_trigger();
+  const float lr = lr_dev ? __ldg(lr_dev) : lr_arg;
+  const int b = blockIdx.x;
+  if (b >= a.block_first[4]) {
+    // the fc bias: gradients from the per-worker slabs
+    const int co = (b - a.block_first[4]) * blockDim.x + threadIdx.x;
+    if (co >= a.C) return;
+    const int64_t j = a.fc_b_off + co;
+    float acc = 0.f;
+    for (int m = 0; m < M; ++m) acc = fmaf(__ldg(w + m), a.slabs[(int64_t)m * a.Ps + j], acc);
+    const float t = apply_update_cnn<kRecipe>(theta[j], acc, lr, kRecipe ? mbuf + j : nullptr, mu, wd, first);
+    theta[j] = t;
+    shadow[j] = __float2bfloat16_rn(t);
+    return;
+  }
+  CnnUpdLayer L;
+  int base;
+  if (b >= a.block_first[3]) { L = a.layer[3]; base = a.block_first[3]; }
+  else if (b >= a.block_first[2]) { L = a.layer[2]; base = a.block_first[2]; }
+  else if (b >= a.block_first[1]) { L = a.layer[1]; base = a.block_first[1]; }
+  else { L = a.layer[0]; base = 0; }
+  const int64_t it = (int64_t)(b - base) * blockDim.x + threadIdx.x;
+  if (it >= (int64_t)L.rows * L.cols) return;
+  cnn_update_item<kRecipe>(L, it, theta, M, w, lr, shadow, mbuf, mu, wd, first);
+}
+
 inline int blocks_for(int64_t n, int threads) { return (int)((n + threads - 1) / threads); }
 
 // bf16 patch rows of the first convolution: one thread per row where the row is short, else the
@@ -639,21 +770,7 @@ hs_status cnn_step(hs_ctx* c, float* params, const float* x, const int32_t* y, c
   const ConvLayer* L = c->convs.data();
   const int c3 = L[2].cout;
   const int hw3 = L[2].hout * L[2].wout;
-  {
-    PhaseScope ph(c, HS_PHASE_CAST, s);
-    if (bf16) {
-      for (int k = 0; k < 3; ++k) {
-        launch_pdl(permute_weights_kernel, blocks_for((int64_t)L[k].cout * L[k].Kp, T), T, 0, s,
-            params + L[k].w_off, L[k].cout, L[k].cin, L[k].Kp, c->d_wperm[k]);
-        ph.launched();
-        if (L[k].subpixel) {
-          launch_pdl(permute_weights_subpixel_kernel, blocks_for(9LL * L[k].cout * L[k].cin, T), T, 0, s,
-              params + L[k].w_off, L[k].cout, L[k].cin, c->d_wsub[k]);
-          ph.launched();
-        }
-      }
-    }
-  }
+  // (the bf16 weight copies the products read are current: cnn_refresh_weights or the fused update)
   {
     PhaseScope ph(c, HS_PHASE_FORWARD, s);
     for (int k = 0; k < 3; ++k) {
@@ -741,11 +858,13 @@ hs_status cnn_step(hs_ctx* c, float* params, const float* x, const int32_t* y, c
           if (e != cudaSuccess) return cuda_fail(c, e, "conv weight-gradient GEMM launch");
           ph.launched();
         }
-        const int kw = fc ? wg.K : wg.K - 1;   // weight columns (the conv partials carry the bias column)
-        dim3 grid2(blocks_for((int64_t)wg.rows_out * wg.K, T), c->M);
-        launch_pdl(splitk_reduce_kernel, grid2, T, 0, s, wg.d_partial, wg.rows_out, kw, wg.ldp, wg.d_chunk_begin, c->d_slabs,
-                                                 c->Ps, w_off, fc ? 0 : L[k].cin, b_off);
-        ph.launched();
+        if (!cnn_fused_update(c)) {   // else the fused update reads the split-K parts itself
+          const int kw = fc ? wg.K : wg.K - 1;   // weight columns (the conv partials carry the bias column)
+          dim3 grid2(blocks_for((int64_t)wg.rows_out * wg.K, T), c->M);
+          launch_pdl(splitk_reduce_kernel, grid2, T, 0, s, wg.d_partial, wg.rows_out, kw, wg.ldp, wg.d_chunk_begin,
+                     c->d_slabs, c->Ps, w_off, fc ? 0 : L[k].cin, b_off);
+          ph.launched();
+        }
       } else {
         GemmF32Args w{};
         w.A = reinterpret_cast<const float*>(delta); w.a_sm = 1; w.a_sk = ld_delta;
@@ -831,6 +950,78 @@ hs_status cnn_step(hs_ctx* c, float* params, const float* x, const int32_t* y, c
       ph.launched(2);
     }
   }
+  return HS_OK;
+}
+
+bool cnn_fused_update(const hs_ctx* c) {
+  return c->arch == HS_CNN && c->precision == HS_BF16 && c->cnn_fuse_update && !c->debug;
+}
+
+// The bf16 copies of theta the CNN's products read: tap-major rows (forward, patch-space input
+// gradient) and, for the sub-pixel input gradients, the class matrices.  The fused update writes
+// them beside theta; this runs when they are stale (first step, external change of params, a
+// step on the slab path).
+hs_status cnn_refresh_weights(hs_ctx* c, const float* params, cudaStream_t s) {
+  const int T = 256;
+  PhaseScope ph(c, HS_PHASE_CAST, s);
+  for (int k = 0; k < 3; ++k) {
+    const ConvLayer& L = c->convs[k];
+    launch_pdl(permute_weights_kernel, blocks_for((int64_t)L.cout * L.Kp, T), T, 0, s,
+        params + L.w_off, L.cout, L.cin, L.Kp, c->d_wperm[k]);
+    ph.launched();
+    if (L.subpixel) {
+      launch_pdl(permute_weights_subpixel_kernel, blocks_for(9LL * L.cout * L.cin, T), T, 0, s,
+          params + L.w_off, L.cout, L.cin, c->d_wsub[k]);
+      ph.launched();
+    }
+  }
+  HS_CUDA(c, cudaGetLastError());
+  return HS_OK;
+}
+
+hs_status launch_cnn_update(hs_ctx* c, float* params, float lr, const float* lr_dev, cudaStream_t s) {
+  CnnUpdArgs a{};
+  int64_t items = 0;
+  const int T = 256;
+  int blocks = 0;
+  for (int k = 0; k < 4; ++k) {
+    const bool fc = (k == 3);
+    const CnnWgrad& wg = c->cnn_wgrad[k];
+    CnnUpdLayer& u = a.layer[k];
+    u.partial = wg.d_partial;
+    u.begin = wg.d_chunk_begin;
+    u.rows = wg.rows_out;
+    u.ldp = wg.ldp;
+    u.cols = wg.K;   // convolutions: 9 * Cin weight columns and the ones column; fc: its inputs
+    u.cin = fc ? 0 : c->convs[k].cin;
+    u.w_off = fc ? c->fc_w_off : c->convs[k].w_off;
+    u.b_off = fc ? c->fc_b_off : c->convs[k].b_off;
+    u.first = items;
+    u.wperm = fc ? nullptr : c->d_wperm[k];
+    u.Kp = fc ? 0 : c->convs[k].Kp;
+    u.wsub = (!fc && c->convs[k].subpixel) ? c->d_wsub[k] : nullptr;
+    a.block_first[k] = blocks;
+    blocks += blocks_for((int64_t)u.rows * u.cols, T);
+    items += (int64_t)u.rows * u.cols;
+  }
+  a.block_first[4] = blocks;
+  blocks += blocks_for(c->C, T);
+  a.items = items;
+  a.fc_b_off = c->fc_b_off;
+  a.C = c->C;
+  a.slabs = c->d_slabs;
+  a.Ps = c->Ps;
+  if (items + c->C != c->P) return fail(c, HS_ERR_CUDA, "fused CNN update does not cover the parameters");
+  PhaseScope ph(c, HS_PHASE_UPDATE, s);
+  if (c->opt_recipe)
+    launch_pdl(cnn_update_kernel<true>, blocks, T, 0, s, a, params, c->M,
+               static_cast<const float*>(c->d_w), lr, lr_dev, c->d_shadow, c->d_mom, c->opt_momentum,
+               c->opt_weight_decay, c->mom_valid ? 0 : 1);
+  else
+    launch_pdl(cnn_update_kernel<false>, blocks, T, 0, s, a, params, c->M,
+               static_cast<const float*>(c->d_w), lr, lr_dev, c->d_shadow, static_cast<float*>(nullptr), 0.f, 0.f, 0);
+  ph.launched();
+  HS_CUDA(c, cudaGetLastError());
   return HS_OK;
 }
 

@@ -191,6 +191,8 @@ struct hs_ctx {
   int32_t* d_row_off[4] = {nullptr, nullptr, nullptr, nullptr};
   hs::ChunkTable cnn_chunks[4];
   hs::CnnWgrad cnn_wgrad[4];
+  bool cnn_fuse_update = true;        // HS_CNN_FUSED_UPDATE=0: split-K reductions, slab update and permutations apart
+  const float* cnn_wcopy_src = nullptr;   // the params the bf16 weight copies (wperm, wsub) were last written from
 
   // tensor-core launch parameters (bf16 precision)
   // per-worker weight gradients averaged in tensor memory and applied in the same kernel
@@ -273,5 +275,10 @@ inline hs_status dalloc(hs_ctx* c, T** p, size_t bytes) {
 hs_status cnn_build_static(hs_ctx* c);
 hs_status cnn_build_partition_plans(hs_ctx* c);
 hs_status cnn_step(hs_ctx* c, float* params, const float* x, const int32_t* y, cudaStream_t s);
+// bf16 CNN without debug read-back: one kernel sums the split-K parts per worker, synchronises,
+// updates theta and writes the bf16 copies the next step reads (cnn_update_kernel)
+bool cnn_fused_update(const hs_ctx* c);
+hs_status cnn_refresh_weights(hs_ctx* c, const float* params, cudaStream_t s);
+hs_status launch_cnn_update(hs_ctx* c, float* params, float lr, const float* lr_dev, cudaStream_t s);
 
 }  // namespace hs

@@ -657,6 +657,7 @@ hs_status step_body(hs_ctx* c, float* params, const float* xd, const int32_t* yd
                  : mlp_bf16        ? mlp_step_bf16(c, params, xd, yd, lr, lr_dev, s)
                                    : mlp_step_fp32(c, params, xd, yd, s);
   if (st != HS_OK) return st;
+  if (hs::cnn_fused_update(c)) return hs::launch_cnn_update(c, params, lr, lr_dev, s);
   if (!mlp_bf16) {
     PhaseScope ph(c, HS_PHASE_UPDATE, s);
     hs::UpdateRecipe r{c->d_mom, c->opt_momentum, c->opt_weight_decay, c->mom_valid ? 0 : 1};
@@ -885,6 +886,8 @@ hs_status hs_init(const hs_model_desc* model, int32_t M, const double* compute_w
   // The step's own graph pays where launches outlast the GPU work; a step of more than 1e11
   // parameter-samples (P * N: the 4096-8192-8192-1000 workload's 1.8e12 is 5.6 ms of GPU work for
   // about 0.1 ms of host launches) keeps eager launches.  HS_STEP_GRAPH=0 / =1 force either.
+  const char* cf = getenv("HS_CNN_FUSED_UPDATE");
+  c->cnn_fuse_update = !(cf && !strcmp(cf, "0"));
   const char* sg = getenv("HS_STEP_GRAPH");
   c->graph_on = !(sg && !strcmp(sg, "0"));
   c->graph_force = sg && !strcmp(sg, "1");
@@ -1164,6 +1167,7 @@ hs_status hs_sync_params(hs_ctx* c, const float* params, void* stream) {
   HS_CUDA(c, cudaGetLastError());
   c->shadow_src = params;
   c->shadow_valid = true;
+  c->cnn_wcopy_src = nullptr;   // the CNN's permuted copies are re-derived by the next step
   return HS_OK;
 }
 
@@ -1213,6 +1217,10 @@ hs_status hs_step(hs_ctx* c, float* params, const void* x, const int32_t* y, con
     hs_status r = dalloc(c, &c->d_gdebug, sizeof(float) * c->Ps);
     if (r != HS_OK) return r;
   }
+  if (c->arch == HS_CNN && c->precision == HS_BF16 && c->cnn_wcopy_src != params) {
+    hs_status r = hs::cnn_refresh_weights(c, params, s);
+    if (r != HS_OK) return r;
+  }
   // A caller capturing its own graph gets the step's kernels enqueued as they are.
   cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
   const bool caller_capture = cudaStreamIsCapturing(s, &cap) != cudaSuccess || cap != cudaStreamCaptureStatusNone;
@@ -1228,6 +1236,7 @@ hs_status hs_step(hs_ctx* c, float* params, const void* x, const int32_t* y, con
   HS_CUDA(c, cudaGetLastError());
   c->shadow_src = params;
   c->shadow_valid = (c->precision == HS_BF16);
+  c->cnn_wcopy_src = hs::cnn_fused_update(c) ? params : nullptr;   // the fused update wrote the copies
   c->gdebug_valid = c->debug;
   if (c->opt_recipe) c->mom_valid = true;
   if (loss_out) {

@@ -1,4 +1,5 @@
-"""The two largest MLP workloads against the fp64 oracle, through the step as users run it.
+"""The two largest MLP workloads and the CNN against the fp64 oracle, through the step as users
+run it.
 
 * 3072-2048-2048-10, N 4096, M 8, drifting worker speeds: 20 steps with the partition recomputed
   at step 10 from the window's throughputs (Algorithm 1 on Eq. 2's compute power), on the default
@@ -9,6 +10,9 @@
   read back on the slab path, which equals the default path bit for bit
   (test_gpu_tile_average.test_tile_average_full_size_equals_slab_path); and 10 steps on the
   default path, theta_10 against the oracle's.
+* The CNN (N 512, M 4): its fused update (split-K parts, synchronisation, update and the bf16
+  weight copies in one kernel) equal bit for bit to the separate passes, and 10 steps on the
+  default path against the oracle.
 
 Tolerances: gradient rel. L2 1e-2, parameters after the run 2e-2 (the required ones); the
 parameter change theta_T - theta_0 and the losses after the first step have bounds set above the
@@ -19,6 +23,7 @@ import functools
 
 import numpy as np
 import pytest
+import torch
 
 import synth
 import paper_2110_08941_gb300 as hs
@@ -94,6 +99,59 @@ def test_headline_workload_10_steps_default_path():
                       SYNC, debug=False)
     orc = _headline_oracle(steps)
     th0 = theta0.astype(np.float64)
+    assert rel(lib["theta"], orc["theta"]) <= 2e-2
+    assert rel(lib["theta"] - th0, orc["theta"] - th0) <= BOUND_DTHETA
+    for t in range(steps):
+        tol = 1e-2 if t == 0 else BOUND_LOSS_AFTER_FIRST
+        assert abs(lib["losses"][t] - orc["losses"][t]) <= tol * abs(orc["losses"][t]), t
+
+
+# ------------------------------------------------------------------------------------------ CNN
+def _cnn_run(monkeypatch, fused, dims, M, N, weights, x, y, theta0, lr, steps, recipe=None, repartition=None):
+    monkeypatch.setenv("HS_CNN_FUSED_UPDATE", "1" if fused else "0")
+    ctx = hs.hs_init(synth.CNN, dims, M, N, compute_weights=weights, precision=hs.HS_BF16, sync=SYNC)
+    try:
+        if recipe:
+            hs.hs_set_optimizer(ctx, *recipe)
+        p = torch.tensor(theta0, device="cuda")
+        xd, yd = torch.from_numpy(x).cuda(), torch.from_numpy(y).cuda()
+        losses = []
+        for t in range(steps):
+            if repartition and t in repartition:
+                hs.hs_partition(ctx, repartition[t])
+            losses.append(hs.hs_step(ctx, p, xd, yd, None, lr if not callable(lr) else lr(t)))
+        torch.cuda.synchronize()
+        return p.cpu(), losses
+    finally:
+        ctx.close()
+
+
+@pytest.mark.parametrize("recipe", [None, (0.9, 5e-4)])
+def test_cnn_fused_update_equals_separate_passes(monkeypatch, recipe):
+    """The CNN's fused update (split-K parts summed per worker, synchronisation, update and the bf16
+    weight copies in one kernel) against the split-K reductions, the slab update and the weight
+    permutations as separate launches: the same fp32 operations in the same order, so theta and the
+    losses agree bit for bit, through a repartition and a learning rate that changes every step."""
+    wl, x, y, theta0, w = _inputs(synth.CFG4)
+    lr = lambda t: hs.hs_cosine_lr(wl.lr, 0.0, t, 6)   # noqa: E731
+    rep = {3: [2.0, 1.0, 3.0, 1.0]}
+    a = _cnn_run(monkeypatch, True, wl.dims, wl.workers, wl.global_batch, w, x, y, theta0, lr, 6, recipe, rep)
+    b = _cnn_run(monkeypatch, False, wl.dims, wl.workers, wl.global_batch, w, x, y, theta0, lr, 6, recipe, rep)
+    assert torch.equal(a[0], b[0])
+    assert a[1] == b[1]
+
+
+def test_cnn_workload_10_steps_default_path():
+    """The CNN workload (N 512, M 4, 1:2:3:6) as users run it (fused update, the step's own graph)
+    against the oracle: theta after 10 steps, the parameter change and the losses."""
+    wl, x, y, theta0, w = _inputs(synth.CFG4)
+    steps = 10
+    lib = run_library(wl.arch, wl.dims, wl.workers, wl.global_batch, w, x, y, theta0, wl.lr, steps, hs.HS_BF16,
+                      SYNC, debug=False)
+    orc = run_oracle(wl.arch, wl.dims, wl.workers, wl.global_batch, w, x, y, theta0, wl.lr, steps, SYNC,
+                     decide=decide_for(hs.HS_BF16))
+    th0 = theta0.astype(np.float64)
+    assert lib["counts"][0] == [43, 85, 128, 256]
     assert rel(lib["theta"], orc["theta"]) <= 2e-2
     assert rel(lib["theta"] - th0, orc["theta"] - th0) <= BOUND_DTHETA
     for t in range(steps):
