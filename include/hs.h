@@ -138,6 +138,10 @@ hs_status hs_param_count(const hs_model_desc* model, int64_t* P);
  *                        when the library loads)
  *   HS_NARROW_EW=4       256 x 128 SM-pair tiles with four epilogue warps instead
  *                        of two groups of four on alternate tiles
+ *   HS_CNN_FUSED_UPDATE=0  bf16 CNN: per-worker split-K reductions into the slabs,
+ *                        the slab update and the weight permutations as separate
+ *                        launches instead of one update kernel (debug read-back
+ *                        always takes the separate launches)
  *   HS_STEP_GRAPH=0      every hs_step enqueues its kernels one by one (no
  *                        replay of a captured step, see hs_step); =1 replays
  *                        captured steps also above 1e11 parameter-samples */
