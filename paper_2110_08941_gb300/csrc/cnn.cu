@@ -604,6 +604,20 @@ int narrow_epilogue_warps() {
   return (v && !strcmp(v, "4")) ? 4 : 8;
 }
 
+// Output pixels per A box of a convolution product: 128 where the output grid allows it (whole
+// output rows of one image, or whole images), which halves the boxes a k-block issues; else 64.
+// HS_CONV_ABOX=64 keeps 64.
+int conv_a_box(int C, int Ho, int Wo, int stride) {
+  const char* v = getenv("HS_CONV_ABOX");
+  if (v && !strcmp(v, "64")) return 64;
+  return tc_conv_implicit_ok(C, Ho, Wo, stride, 128) ? 128 : 64;
+}
+int grid_a_box(int rows, int cols) {
+  const char* v = getenv("HS_CONV_ABOX");
+  if (v && !strcmp(v, "64")) return 64;
+  return tc_grid_ok(rows, cols, 128) ? 128 : 64;
+}
+
 // A is K-major [a_rows][a_cols], or (conv != nullptr) the implicit patch rows of that convolution.
 // narrow = true: 256 x 128 SM-pair tiles for a product at most 128 wide (K-major B in 64-row boxes).
 hs_status plan_dense(hs_ctx* c, TcGemmParams* p, int epi, const __nv_bfloat16* a, int64_t a_rows, int a_cols,
@@ -614,10 +628,12 @@ hs_status plan_dense(hs_ctx* c, TcGemmParams* p, int epi, const __nv_bfloat16* a
   std::memset(p, 0, sizeof(*p));
   bool ok;
   if (conv) {
+    const int abox = conv_a_box(conv->cin, conv->hout, conv->wout, conv->stride);
     ok = tc_make_conv_map(&p->tmA[0], a, c->N, conv->hin, conv->win, conv->cin, conv->hout, conv->wout,
-                          conv->stride, &why);
+                          conv->stride, &why, abox);
     p->conv_a = 1;
     p->conv = tc_conv_geom(conv->cin, conv->hout, conv->wout, conv->stride);
+    p->conv.a_box = abox;
   } else {
     ok = tc_make_kmajor_map(&p->tmA[0], TcOperand{a, a_rows, a_cols, lda}, kTcBoxA, &why);
   }
@@ -662,11 +678,12 @@ hs_status plan_subpixel_dgrad(hs_ctx* c, int k) {
   const int taps[4] = {1, 2, 2, 4};
   int64_t off = 0;
   auto* dprev = reinterpret_cast<__nv_bfloat16*>(c->d_dA[k - 1]);
+  const int abox = grid_a_box(L.hout, L.wout);
   for (int g = 0; g < 4; ++g) {
     const int ph = g >> 1, pw = g & 1;
     const int64_t kg = (int64_t)taps[g] * L.cout;
     bool ok = tc_make_grid_map(&p.tmA[g], c->d_dA[k], L.cout, L.wout, L.hout, c->N, L.cout, (int64_t)L.wout * L.cout,
-                               hw * L.cout, 64, &why) &&
+                               hw * L.cout, abox, &why) &&
               tc_make_mnmajor_map(&p.tmB[g], TcOperand{c->d_wsub[k] + off, kg, L.cin, L.cin}, &why) &&
               tc_make_grid_map(&p.tmD[g], dprev + ((int64_t)ph * L.win + pw) * L.cin, L.cin, L.wout, L.hout, c->N,
                                2LL * L.cin, 2LL * L.win * L.cin, (int64_t)L.hin * L.win * L.cin, 32, &why);
@@ -691,6 +708,7 @@ hs_status plan_subpixel_dgrad(hs_ctx* c, int k) {
     p.ew = narrow_epilogue_warps();
   }
   p.conv = tc_conv_geom(L.cout, L.hout, L.wout, L.stride);
+  p.conv.a_box = abox;
   p.conv.H = L.hin;
   p.conv.W = L.win;
   p.D = dprev;

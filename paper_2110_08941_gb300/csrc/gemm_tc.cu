@@ -115,6 +115,11 @@ __global__ void __launch_bounds__(threads_of<CONV>(), 1) tc_gemm_kernel(const __
           for (int j = 0; j < BN / 64; ++j)
             if (c.tn * BN + 64 * j < p.conv.ones_col) bcol[j] = conv_col_part(p.conv, c.tn * BN + 64 * j);
         }
+        // patch-column blocks of A and pixel blocks of B, stepped once per k-block
+        ConvColIter a_it;
+        ConvRowIter b_it;
+        if (CONV && p.conv_a) a_it.init(p.conv, p.conv_a == 2 ? w.g : -1, w.kb_lo * BK);
+        if (CONV && B_MN && p.conv_b) b_it.init(p.conv, w.kb_lo * BK);
         bool ok = true;
         for (int kb = w.kb_lo; kb < w.kb_hi; ++kb) {
           if (!mbar_wait(smem_u32(&empty_bar[s]), ph ^ 1u, abort_flag)) { ok = false; break; }
@@ -129,22 +134,29 @@ __global__ void __launch_bounds__(threads_of<CONV>(), 1) tc_gemm_kernel(const __
             for (int j = 0; j < BM / 64; ++j)
               if (box++ % NP == prod) tma_load_2d(a_dst + j * MN_CHUNK, ta, c.tm * BM + 64 * j, k0, fb);
           } else if (CONV && p.conv_a) {
-            ConvColPart kc;
-            if (NP == 1 || prod < BM / 64)
-              kc = p.conv_a == 2 ? subpixel_col_part(p.conv, w.g, k0) : conv_col_part(p.conv, k0);
-#pragma unroll
-            for (int j = 0; j < BM / 64; ++j)
+            const ConvColPart kc = a_it.part();
+            if (p.conv.a_box == BM) {
+              // one box of the tile's 128 output pixels (lands as the two 64-row boxes would)
               if (box++ % NP == prod) {
                 int cc[4];
-                conv_coords(arow[j], kc, cc);
-                tma_load_4d(a_dst + j * MN_CHUNK, ta, cc, fb);
+                conv_coords(arow[0], kc, cc);
+                tma_load_4d(a_dst, ta, cc, fb);
               }
+            } else {
+#pragma unroll
+              for (int j = 0; j < BM / 64; ++j)
+                if (box++ % NP == prod) {
+                  int cc[4];
+                  conv_coords(arow[j], kc, cc);
+                  tma_load_4d(a_dst + j * MN_CHUNK, ta, cc, fb);
+                }
+            }
           } else {
             if (box++ % NP == prod) tma_load_2d(a_dst, ta, k0, c.tm * BM, fb);
           }
           if (B_MN) {
             ConvRowPart krow;
-            if (CONV && p.conv_b) krow = conv_row_part(p.conv, k0);
+            if (CONV && p.conv_b) krow = b_it.part();
 #pragma unroll
             for (int j = 0; j < BN / 64; ++j) {
               if (box++ % NP != prod) continue;
@@ -164,6 +176,8 @@ __global__ void __launch_bounds__(threads_of<CONV>(), 1) tc_gemm_kernel(const __
             for (int j = 0; j < BN / kTcBoxB; ++j)
               if (box++ % NP == prod) tma_load_2d(b_dst + j * (kTcBoxB * BK * 2), tb, k0, c.tn * BN + kTcBoxB * j, fb);
           }
+          if (CONV && p.conv_a) a_it.next();
+          if (CONV && B_MN && p.conv_b) b_it.next();
           if (++s == S) { s = 0; ph ^= 1u; }
         }
         if (!ok) {
@@ -367,11 +381,12 @@ bool tc_make_kmajor_map(CUtensorMap* tm, const TcOperand& op, int box_rows, cons
                    why);
 }
 
-bool tc_conv_implicit_ok(int C, int Ho, int Wo, int stride) {
-  if (C < 64 || C % 64 || Wo < 1 || Ho < 1 || 64 % Wo || stride < 1 || stride > 2) return false;
+bool tc_conv_implicit_ok(int C, int Ho, int Wo, int stride, int box_px) {
+  if (box_px != 64 && box_px != 128) return false;
+  if (C < 64 || C % 64 || Wo < 1 || Ho < 1 || box_px % Wo || stride < 1 || stride > 2) return false;
   const int hw = Ho * Wo;
-  if (hw % 64 && 64 % hw) return false;
-  const int hb = hw >= 64 ? 64 / Wo : Ho;   // output rows a 64-pixel box covers
+  if (hw % box_px && box_px % hw) return false;
+  const int hb = hw >= box_px ? box_px / Wo : Ho;   // output rows a box covers
   return stride * Wo <= 256 && stride * hb <= 256;
 }
 
@@ -382,13 +397,14 @@ TcConvGeom tc_conv_geom(int C, int Ho, int Wo, int stride) {
   g.hw = Ho * Wo;
   g.stride = stride;
   g.ones_col = 9 * C;
+  g.a_box = 64;
   return g;
 }
 
 bool tc_make_conv_map(CUtensorMap* tm, const __nv_bfloat16* base, int64_t images, int H, int W, int C, int Ho,
-                      int Wo, int stride, const char** why) {
+                      int Wo, int stride, const char** why, int box_px) {
   if (!g_encode && !tc_init_driver(why)) return false;
-  if (!tc_conv_implicit_ok(C, Ho, Wo, stride) || images < 1) {
+  if (!tc_conv_implicit_ok(C, Ho, Wo, stride, box_px) || images < 1) {
     *why = "convolution geometry not supported by the implicit patch rows";
     return false;
   }
@@ -397,8 +413,8 @@ bool tc_make_conv_map(CUtensorMap* tm, const __nv_bfloat16* base, int64_t images
     return false;
   }
   const int hw = Ho * Wo;
-  const uint32_t hb = hw >= 64 ? (uint32_t)(64 / Wo) : (uint32_t)Ho;
-  const uint32_t nb = hw >= 64 ? 1u : (uint32_t)(64 / hw);
+  const uint32_t hb = hw >= box_px ? (uint32_t)(box_px / Wo) : (uint32_t)Ho;
+  const uint32_t nb = hw >= box_px ? 1u : (uint32_t)(box_px / hw);
   // dims innermost first: channels, input columns, input rows, images; a box traverses `stride`
   // input columns / rows per output pixel and loads ceil(extent / stride) of them
   cuuint64_t dims[4] = {(cuuint64_t)C, (cuuint64_t)W, (cuuint64_t)H, (cuuint64_t)images};

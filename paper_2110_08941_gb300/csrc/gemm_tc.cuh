@@ -40,6 +40,8 @@ struct TcConvGeom {
   int32_t ones_col;   // as the B operand: first column past the 9 * C patch columns, which holds
                       // ones (the bias gradient's column); columns past it read zeros
   int32_t H, W;       // input grid (sub-pixel input gradient: where the ReLU' mask is read)
+  int32_t a_box;      // output pixels per A box (conv_a): 64, or 128 (one box per 128 rows, whole
+                      // output rows of one image or whole images; half the box issues per k-block)
 };
 
 // D[Mdim x n_store] (row-major, leading dimension ldd) = A[Mdim x K] * B[K x Ndim] + epilogue.
@@ -119,10 +121,10 @@ bool tc_make_kmajor_map(CUtensorMap* tm, const TcOperand& op, int box_rows, cons
 // MN-major operand: matrix [K rows][MN] with MN contiguous; box = 64 (MN) x 64 (K).
 bool tc_make_mnmajor_map(CUtensorMap* tm, const TcOperand& op, const char** why);
 // Implicit patch rows of a convolution (see TcConvGeom): input NHWC bf16 [images][H][W][C] at
-// `base`, output grid Ho x Wo.  Box: 64 channels x 64 output pixels.
-bool tc_conv_implicit_ok(int C, int Ho, int Wo, int stride);
+// `base`, output grid Ho x Wo.  Box: 64 channels x `box_px` output pixels (64 or 128).
+bool tc_conv_implicit_ok(int C, int Ho, int Wo, int stride, int box_px = 64);
 bool tc_make_conv_map(CUtensorMap* tm, const __nv_bfloat16* base, int64_t images, int H, int W, int C, int Ho,
-                      int Wo, int stride, const char** why);
+                      int Wo, int stride, const char** why, int box_px = 64);
 TcConvGeom tc_conv_geom(int C, int Ho, int Wo, int stride);
 // bf16 pixel grid [images][rows][cols][C] with arbitrary (16-byte multiple) strides, given in
 // elements; box = 64 channels x `box_pixels` pixels (whole grid rows, or whole images).

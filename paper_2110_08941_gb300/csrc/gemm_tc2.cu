@@ -17,6 +17,8 @@
 // Every mbarrier wait is bounded as in the one-SM kernel.
 #include <cudaTypedefs.h>
 
+#include <cstdlib>
+
 #include "tc_pair.cuh"
 
 namespace hs {
@@ -36,14 +38,18 @@ constexpr int A_HALF = HM * BK * 2;                // 16 KB
 // columns; with 128-wide tiles (kAlt) they are two groups of four, each draining every other tile
 // (one accumulator buffer each), so two tiles' epilogues run at once even where the product is
 // only 64 wide.  Eight epilogue warps cost stages to fit their staging buffers.
-template <int TN, int EW, int NP = 1>
+// KS k-blocks per pipeline stage: one barrier round trip (the producer's wait, expected-bytes
+// arrive and box issues; the MMA issuer's wait and commit, each a few hundred cycles on one
+// thread) then feeds KS k-blocks of MMAs.  A 256 x 128 tile's k-block is about 0.17 us of MMA,
+// less than one round trip, so those products take KS = 2 (the same slots, paired).
+template <int TN, int EW, int NP = 1, int KS = 1>
 struct PairCfg {
   static constexpr int PN = TN;
   static constexpr int HN = TN / 2;
   static constexpr int B_HALF = HN * BK * 2;
   static constexpr int STAGE2 = A_HALF + B_HALF;
   static constexpr bool kAlt = (TN == 128 && EW == 8);
-  static constexpr int S2 = TN == 256 ? (EW == 8 ? 5 : 6) : (EW == 8 ? 6 : 8);
+  static constexpr int S2 = TN == 256 ? (EW == 8 ? (KS == 2 ? 4 : 5) : 6) : (EW == 8 ? 6 : 8);   // slots
   static constexpr int kThreads = 64 + 32 * EW + 32 * (NP - 1);   // NP TMA producer warps
   static constexpr uint32_t PAIR_TX = 2 * STAGE2;   // bytes landing per stage on the leader's barrier
   static constexpr uint32_t kTmemCols2 = 2 * TN;
@@ -51,8 +57,10 @@ struct PairCfg {
   static constexpr int kSmem2 = S2 * STAGE2 + kStaging + 1024 + 256;
   // arrivals that free one accumulator buffer: the epilogue warps of both CTAs that drain it
   static constexpr uint32_t kFreeArrivals = 2 * (kAlt ? 4 : EW);
+  static constexpr int NB = S2 / KS;                 // pipeline stages (barrier pairs) of KS slots each
   static_assert(kSmem2 <= 232448, "shared memory budget");
   static_assert(EW == 4 || EW == 8, "epilogue warps");
+  static_assert((KS == 1 || KS == 2) && S2 % KS == 0, "k-blocks per stage");
 };
 
 // Convolution products keep two TMA producer warps busy: their operands come in 8 KB 4-D boxes
@@ -60,12 +68,12 @@ struct PairCfg {
 // k-block's MMAs.  The producers split each k-block's boxes round-robin.
 constexpr int kConvProducers = 2;
 
-template <int EPI, bool A_MN, bool B_MN, bool CONV, int TN, int EW>
-__global__ void __launch_bounds__(PairCfg<TN, EW, CONV ? kConvProducers : 1>::kThreads, 1)
+template <int EPI, bool A_MN, bool B_MN, bool CONV, int TN, int EW, int KS>
+__global__ void __launch_bounds__(PairCfg<TN, EW, CONV ? kConvProducers : 1, KS>::kThreads, 1)
     tc_gemm_pair_kernel(const __grid_constant__ TcGemmParams p) {
   constexpr int NP = CONV ? kConvProducers : 1;
-  using Cfg = PairCfg<TN, EW, NP>;
-  constexpr int PN = Cfg::PN, HN = Cfg::HN, S2 = Cfg::S2, STAGE2 = Cfg::STAGE2;
+  using Cfg = PairCfg<TN, EW, NP, KS>;
+  constexpr int PN = Cfg::PN, HN = Cfg::HN, S2 = Cfg::S2, STAGE2 = Cfg::STAGE2, NB = Cfg::NB;
   constexpr uint32_t PAIR_TX = Cfg::PAIR_TX, kTmemCols2 = Cfg::kTmemCols2;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -84,7 +92,7 @@ __global__ void __launch_bounds__(PairCfg<TN, EW, CONV ? kConvProducers : 1>::kT
   const bool leader = (rank == 0);
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < S2; ++s) {
+    for (int s = 0; s < NB; ++s) {
       mbar_init(smem_u32(&full_bar[s]), 1);
       mbar_init(smem_u32(&empty_bar[s]), 1);
     }
@@ -148,16 +156,26 @@ __global__ void __launch_bounds__(PairCfg<TN, EW, CONV ? kConvProducers : 1>::kT
           for (int j = 0; j < HN / 64; ++j)
             if (n0 + 64 * j < p.conv.ones_col) bcol[j] = conv_col_part(p.conv, n0 + 64 * j);
         }
+        // patch-column blocks of A and pixel blocks of B, stepped once per k-block
+        ConvColIter a_it;
+        ConvRowIter b_it;
+        if (CONV && p.conv_a) a_it.init(p.conv, p.conv_a == 2 ? w.g : -1, w.kb_lo * BK);
+        if (CONV && B_MN && p.conv_b) b_it.init(p.conv, w.kb_lo * BK);
         bool ok = true;
-        for (int kb = w.kb_lo; kb < w.kb_hi; ++kb) {
+        for (int kb = w.kb_lo; kb < w.kb_hi; kb += KS) {
+          // the stage's k-blocks: KS, or one where the tile's k-block count is odd
+          const int nk = (KS == 1 || kb + 1 >= w.kb_hi) ? 1 : KS;
           if (!mbar_wait(smem_u32(&empty_bar[s]), ph ^ 1u, abort_flag)) { ok = false; break; }
           const uint32_t fb_local = smem_u32(&full_bar[s]);
           const uint32_t fb = map_to_rank(fb_local, 0);
-          if (prod == 0 && leader) mbar_expect_tx(fb_local, PAIR_TX);
-          const int k0 = kb * BK;
-          const uint32_t a_dst = smem_u32(smem + s * STAGE2);
-          const uint32_t b_dst = a_dst + A_HALF;
+          if (prod == 0 && leader) mbar_expect_tx(fb_local, PAIR_TX * (uint32_t)nk);
           int box = 0;
+#pragma unroll
+          for (int js = 0; js < KS; ++js) {
+          if (js >= nk) break;
+          const int k0 = (kb + js) * BK;
+          const uint32_t a_dst = smem_u32(smem + (s * KS + js) * STAGE2);
+          const uint32_t b_dst = a_dst + A_HALF;
           // the A half: two 64-column boxes (MN-major), two 64-pixel boxes (implicit patch rows) or
           // one 128-row box (K-major)
           if (A_MN) {
@@ -165,22 +183,29 @@ __global__ void __launch_bounds__(PairCfg<TN, EW, CONV ? kConvProducers : 1>::kT
             for (int j = 0; j < HM / 64; ++j)
               if (box++ % NP == prod) tma_load_2d_pair(a_dst + j * MN_CHUNK, ta, m0 + 64 * j, k0, fb);
           } else if (CONV && p.conv_a) {
-            ConvColPart kc;
-            if (NP == 1 || prod < HM / 64)
-              kc = p.conv_a == 2 ? subpixel_col_part(p.conv, w.g, k0) : conv_col_part(p.conv, k0);
-#pragma unroll
-            for (int j = 0; j < HM / 64; ++j)
+            const ConvColPart kc = a_it.part();
+            if (p.conv.a_box == HM) {
+              // one box of the half's 128 output pixels (lands as the two 64-row boxes would)
               if (box++ % NP == prod) {
                 int cc[4];
-                conv_coords(arow[j], kc, cc);
-                tma_load_4d_pair(a_dst + j * MN_CHUNK, ta, cc, fb);
+                conv_coords(arow[0], kc, cc);
+                tma_load_4d_pair(a_dst, ta, cc, fb);
               }
+            } else {
+#pragma unroll
+              for (int j = 0; j < HM / 64; ++j)
+                if (box++ % NP == prod) {
+                  int cc[4];
+                  conv_coords(arow[j], kc, cc);
+                  tma_load_4d_pair(a_dst + j * MN_CHUNK, ta, cc, fb);
+                }
+            }
           } else {
             if (box++ % NP == prod) tma_load_2d_pair(a_dst, ta, k0, m0, fb);
           }
           if (B_MN) {
             ConvRowPart krow;
-            if (CONV && p.conv_b) krow = conv_row_part(p.conv, k0);
+            if (CONV && p.conv_b) krow = b_it.part();
 #pragma unroll
             for (int j = 0; j < HN / 64; ++j) {
               if (box++ % NP != prod) continue;
@@ -198,7 +223,10 @@ __global__ void __launch_bounds__(PairCfg<TN, EW, CONV ? kConvProducers : 1>::kT
           } else {
             if (box++ % NP == prod) tma_load_2d_pair(b_dst, tb, k0, n0, fb);
           }
-          if (++s == S2) { s = 0; ph ^= 1u; }
+          if (CONV && p.conv_a) a_it.next();
+          if (CONV && B_MN && p.conv_b) b_it.next();
+          }
+          if (++s == NB) { s = 0; ph ^= 1u; }
         }
         if (!ok) {
           record_error(p.st, kDevWaitTimeout, 11);
@@ -211,7 +239,7 @@ __global__ void __launch_bounds__(PairCfg<TN, EW, CONV ? kConvProducers : 1>::kT
     if (lane == 0 && leader) {
       // ------------------------------------------------------------ pair MMA issuer (leader)
       constexpr uint32_t idesc = make_idesc(A_MN, B_MN, PM, PN);
-      constexpr uint64_t kStageDesc = STAGE2 >> 4;   // one stage, in the descriptor's address field
+      constexpr uint64_t kStageDesc = STAGE2 >> 4;   // one slot, in the descriptor's address field
       const uint64_t a_desc0 = make_sdesc(smem_u32(smem), A_MN ? MN_CHUNK : 16, 1024);
       const uint64_t b_desc0 = make_sdesc(smem_u32(smem) + A_HALF, B_MN ? MN_CHUNK : 16, 1024);
       int s = 0;
@@ -228,30 +256,31 @@ __global__ void __launch_bounds__(PairCfg<TN, EW, CONV ? kConvProducers : 1>::kT
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + (uint32_t)(ab * PN);
         bool ok = true;
-        // full k-blocks, then (when this tile holds it) the group's partial last k-block
+        // stages of KS full k-blocks; the group's partial last k-block (the tile's last, when the
+        // tile holds it) takes only its steps that hold rows
         const LastKb lk = last_kb_of(p, w.g);
         const bool tail = lk.kb_last >= w.kb_lo && lk.kb_last < w.kb_hi;
-        const int kb_full = tail ? lk.kb_last : w.kb_hi;
-        int kb = w.kb_lo;
-        for (; kb < kb_full; ++kb) {
+        for (int kb = w.kb_lo; kb < w.kb_hi; kb += KS) {
+          const int nk = (KS == 1 || kb + 1 >= w.kb_hi) ? 1 : KS;
           if (!mbar_wait(smem_u32(&full_bar[s]), ph, abort_flag)) { ok = false; break; }
           tc_fence_after();
-          const uint64_t off = kStageDesc * (uint64_t)s;
-          mma_kblock_pair<A_MN, B_MN>(d_tmem, a_desc0 + off, b_desc0 + off, idesc, kb != w.kb_lo ? 1u : 0u);
-          umma_commit_pair(smem_u32(&empty_bar[s]));
-          if (++s == S2) { s = 0; ph ^= 1u; }
-        }
-        if (ok && tail) {
-          if (!mbar_wait(smem_u32(&full_bar[s]), ph, abort_flag)) {
-            ok = false;
+          const uint64_t off = kStageDesc * (uint64_t)(s * KS);
+          if (nk == KS && !(tail && kb + KS == w.kb_hi)) {
+            mma_kblock_pair<A_MN, B_MN>(d_tmem, a_desc0 + off, b_desc0 + off, idesc, kb != w.kb_lo ? 1u : 0u);
+            if (KS == 2) mma_kblock_pair<A_MN, B_MN>(d_tmem, a_desc0 + off + kStageDesc, b_desc0 + off + kStageDesc, idesc, 1u);
           } else {
-            tc_fence_after();
-            const uint64_t off = kStageDesc * (uint64_t)s;
-            mma_ksteps_pair<A_MN, B_MN>(d_tmem, a_desc0 + off, b_desc0 + off, idesc, kb != w.kb_lo ? 1u : 0u,
-                                        lk.steps);
-            umma_commit_pair(smem_u32(&empty_bar[s]));
-            if (++s == S2) { s = 0; ph ^= 1u; }
+            // the stage ends the tile: its k-blocks before the last are full, the last may be partial
+            if (KS == 2 && nk == 2)
+              mma_kblock_pair<A_MN, B_MN>(d_tmem, a_desc0 + off, b_desc0 + off, idesc, kb != w.kb_lo ? 1u : 0u);
+            const uint64_t o2 = off + kStageDesc * (uint64_t)(nk - 1);
+            const uint32_t acc = (kb + nk - 1) != w.kb_lo ? 1u : 0u;
+            if (tail)
+              mma_ksteps_pair<A_MN, B_MN>(d_tmem, a_desc0 + o2, b_desc0 + o2, idesc, acc, lk.steps);
+            else
+              mma_kblock_pair<A_MN, B_MN>(d_tmem, a_desc0 + o2, b_desc0 + o2, idesc, acc);
           }
+          umma_commit_pair(smem_u32(&empty_bar[s]));
+          if (++s == NB) { s = 0; ph ^= 1u; }
         }
         if (!ok) {
           record_error(p.st, kDevWaitTimeout, 13);
@@ -359,13 +388,13 @@ __global__ void __launch_bounds__(PairCfg<TN, EW, CONV ? kConvProducers : 1>::kT
   }
 }
 
-template <int EPI, bool A_MN, bool B_MN, bool CONV, int TN = 256, int EW = 4>
-cudaError_t launch_pair_variant(const TcGemmParams& p, int pairs_wanted, int num_sms, cudaStream_t s) {
+template <int EPI, bool A_MN, bool B_MN, bool CONV, int TN = 256, int EW = 4, int KS = 1>
+cudaError_t launch_pair_variant1(const TcGemmParams& p, int pairs_wanted, int num_sms, cudaStream_t s) {
   static bool configured = false;
   static int max_clusters = 0;
-  using Cfg = PairCfg<TN, EW, CONV ? kConvProducers : 1>;
+  using Cfg = PairCfg<TN, EW, CONV ? kConvProducers : 1, KS>;
   constexpr int kSmem2 = Cfg::kSmem2;
-  auto kern = tc_gemm_pair_kernel<EPI, A_MN, B_MN, CONV, TN, EW>;
+  auto kern = tc_gemm_pair_kernel<EPI, A_MN, B_MN, CONV, TN, EW, KS>;
   cudaLaunchConfig_t cfg = {};
   cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -401,6 +430,23 @@ cudaError_t launch_pair_variant(const TcGemmParams& p, int pairs_wanted, int num
   cudaError_t e = cudaLaunchKernelEx(&cfg, kern, p);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
+}
+
+// Two k-blocks per stage where a k-block's MMAs are shorter than a barrier round trip: the
+// 256 x 128 tiles, and every convolution product (whose producers also form box coordinates).
+// HS_KSTAGE=1 keeps one (the same MMAs in the same order: identical results).
+inline bool pair_two_kblocks(int tn, bool conv) {
+  const char* v = getenv("HS_KSTAGE");   // read per launch: a step replayed from a graph launches nothing
+  const int forced = v ? atoi(v) : 0;
+  if (forced == 1) return false;
+  if (forced == 2) return true;
+  return tn == 128 || conv;
+}
+
+template <int EPI, bool A_MN, bool B_MN, bool CONV, int TN = 256, int EW = 4>
+cudaError_t launch_pair_variant(const TcGemmParams& p, int pairs_wanted, int num_sms, cudaStream_t s) {
+  if (pair_two_kblocks(TN, CONV)) return launch_pair_variant1<EPI, A_MN, B_MN, CONV, TN, EW, 2>(p, pairs_wanted, num_sms, s);
+  return launch_pair_variant1<EPI, A_MN, B_MN, CONV, TN, EW, 1>(p, pairs_wanted, num_sms, s);
 }
 
 }  // namespace

@@ -131,6 +131,73 @@ __device__ __forceinline__ ConvColPart subpixel_col_part(const TcConvGeom& g, in
   const int th = t / nw, tw = t - th * nw;
   return {cb * 64, (pw && tw == 0) ? 1 : 0, (ph && th == 0) ? 1 : 0};
 }
+// The producers walk a tile's k-blocks in order, so instead of dividing per k-block (a long
+// dependent chain on the single issuing thread, slower than the k-block's MMAs) they step these
+// iterators: set up once per tile with divisions, then advanced by adds and compares.
+// Patch-column blocks of the A operand (K-major): forward (sub < 0) block = tap * cblocks + cb with
+// tap = 3 * kh + kw; sub-pixel class `sub` block = (th * nw + tw) * cblocks + cb.
+struct ConvColIter {
+  int cb, cblocks, a, na, b;   // forward: a = kw, b = kh (na = 3); sub-pixel: a = tw, b = th (na = nw)
+  int ph, pw;                  // sub-pixel class parities; -1 for the forward
+  __device__ __forceinline__ void init(const TcConvGeom& g, int sub, int kcol) {
+    const int blk = kcol >> 6;
+    cblocks = g.cblocks;
+    const int t = blk / cblocks;
+    cb = blk - t * cblocks;
+    if (sub < 0) {
+      ph = pw = -1;
+      na = 3;
+      b = t / 3;
+      a = t - 3 * b;
+    } else {
+      ph = sub >> 1;
+      pw = sub & 1;
+      na = pw ? 2 : 1;
+      b = t / na;
+      a = t - b * na;
+    }
+  }
+  __device__ __forceinline__ ConvColPart part() const {
+    if (ph < 0) return {cb * 64, a - 1, b - 1};
+    return {cb * 64, (pw && a == 0) ? 1 : 0, (ph && b == 0) ? 1 : 0};
+  }
+  __device__ __forceinline__ void next() {
+    if (++cb == cblocks) {
+      cb = 0;
+      if (++a == na) {
+        a = 0;
+        ++b;
+      }
+    }
+  }
+};
+// Output-pixel blocks of 64 rows of the implicit patch rows as the B operand (MN-major, K = pixels):
+// 64 / Wo output rows per block within an image, or 64 / hw whole images per block.
+struct ConvRowIter {
+  int img, ho, Ho, dho, dimg, stride;
+  __device__ __forceinline__ void init(const TcConvGeom& g, int row) {
+    img = row / g.hw;
+    ho = (row - img * g.hw) / g.Wo;
+    Ho = g.hw / g.Wo;
+    stride = g.stride;
+    if (g.hw >= 64) {
+      dho = 64 / g.Wo;
+      dimg = 0;
+    } else {
+      dho = 0;
+      dimg = 64 / g.hw;
+    }
+  }
+  __device__ __forceinline__ ConvRowPart part() const { return {img, stride * ho}; }
+  __device__ __forceinline__ void next() {
+    if (dimg) {
+      img += dimg;
+    } else if ((ho += dho) >= Ho) {
+      ho = 0;
+      ++img;
+    }
+  }
+};
 __device__ __forceinline__ void conv_coords(const ConvRowPart& r, const ConvColPart& k, int (&c)[4]) {
   c[0] = k.c0;
   c[1] = k.dw;

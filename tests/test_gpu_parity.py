@@ -10,6 +10,7 @@ For the bf16 path the oracle takes the ReLU' decisions in the kernel's precision
 every value it computes stays fp64 (a departure from taking them exactly, bounded separately in
 test_bf16_against_exact_decisions)."""
 import functools
+import types
 
 import numpy as np
 import pytest
@@ -333,3 +334,75 @@ def test_subpixel_input_gradient_matches_patch_space_gather(monkeypatch):
     assert np.allclose(sub[1], pat[1], rtol=1e-3, atol=0)
     assert rel(sub[0].numpy(), pat[0].numpy()) <= 1e-5
     assert pat[3] - sub[3] >= 0.9 * 4 * wl.global_batch * 256 * 576
+
+
+def _cnn_run_env(monkeypatch, env, wl, x, y, theta0, w, steps):
+    for k, v in env.items():
+        monkeypatch.setenv(k, v)
+    try:
+        return _cnn_run(monkeypatch, "1", wl, x, y, theta0, w, steps)
+    finally:
+        for k in env:
+            monkeypatch.delenv(k)
+
+
+@pytest.mark.parametrize("dims,N,M", [(None, None, None), ((3, 16, 16, 64, 128, 64, 7), 13, 3)])
+def test_conv_a_boxes_of_128_pixels_are_bit_identical(monkeypatch, dims, N, M):
+    """One 128-pixel 4-D box per 128 rows of the convolutions' A operands (forward patch rows,
+    shifted sub-pixel output gradient) lands in shared memory exactly as two 64-pixel boxes do, so
+    theta, losses and per-worker gradients agree bit for bit with HS_CONV_ABOX=64 (the CNN workload,
+    and 8x8 / 4x4 output grids where a box spans two or eight images, with a ragged last image)."""
+    if dims is None:
+        wl, x, y, theta0, w = _inputs(synth.CFG4)
+    else:
+        rng = np.random.default_rng(3)
+        x = rng.standard_normal((N,) + tuple(dims[:3]), dtype=np.float32)
+        y = rng.integers(0, dims[-1], N, dtype=np.int32)
+        theta0 = synth.he_normal_params(synth.CNN, dims, 5)
+        wl = types.SimpleNamespace(arch=synth.CNN, dims=dims, global_batch=N, workers=M, lr=0.05)
+        w = [1.0, 2.0, 3.5]
+    big = _cnn_run_env(monkeypatch, {}, wl, x, y, theta0, w, 3)
+    small = _cnn_run_env(monkeypatch, {"HS_CONV_ABOX": "64"}, wl, x, y, theta0, w, 3)
+    assert torch.equal(big[0], small[0])
+    assert big[1] == small[1]
+    assert torch.equal(big[2], small[2])
+
+
+def _env_run(monkeypatch, env, fn):
+    for k, v in env.items():
+        monkeypatch.setenv(k, v)
+    try:
+        return fn()
+    finally:
+        for k in env:
+            monkeypatch.delenv(k)
+
+
+@pytest.mark.parametrize("case", ["cnn", "mlp_ragged"])
+def test_two_kblocks_per_stage_are_bit_identical(monkeypatch, case):
+    """Two k-blocks per pipeline stage (one barrier round trip feeding two k-blocks of MMAs) issue the
+    same MMAs on the same operands in the same order as one, so every result is the same bit for
+    bit: the CNN workload (default: two for every convolution product and 256 x 128 tile, against
+    HS_KSTAGE=1), and an MLP with ragged worker segments whose grouped weight gradients end in
+    partial k-blocks and odd k-block counts (HS_KSTAGE=2 against 1)."""
+    if case == "cnn":
+        wl, x, y, theta0, w = _inputs(synth.CFG4)
+        args = (wl.arch, wl.dims, wl.workers, wl.global_batch, w, x, y, theta0, wl.lr, 3)
+        env_a, env_b = {}, {"HS_KSTAGE": "1"}
+    else:
+        dims, N, M, w = (256, 192, 136, 10), 333, 3, [1.0, 2.0, 3.5]
+        rng = np.random.default_rng(11)
+        x = rng.standard_normal((N, dims[0]), dtype=np.float32)
+        y = rng.integers(0, dims[-1], N, dtype=np.int32)
+        theta0 = synth.he_normal_params(synth.MLP, dims, 4)
+        args = (synth.MLP, dims, M, N, w, x, y, theta0, 0.05, 3)
+        env_a, env_b = {"HS_KSTAGE": "2"}, {"HS_KSTAGE": "1"}
+
+    def go():
+        return run_library(*args, hs.HS_BF16, hs.HS_SYNC_CP_WEIGHTED, keep_slabs=True)
+
+    a = _env_run(monkeypatch, env_a, go)
+    b = _env_run(monkeypatch, env_b, go)
+    assert np.array_equal(a["theta"], b["theta"])
+    assert a["losses"] == b["losses"]
+    assert np.array_equal(a["slabs_first"], b["slabs_first"])
