@@ -432,20 +432,22 @@ cudaError_t launch_pair_variant1(const TcGemmParams& p, int pairs_wanted, int nu
   return cudaGetLastError();
 }
 
-// Two k-blocks per stage where a k-block's MMAs are shorter than a barrier round trip: the
-// 256 x 128 tiles, and every convolution product (whose producers also form box coordinates).
-// HS_KSTAGE=1 keeps one (the same MMAs in the same order: identical results).
-inline bool pair_two_kblocks(int tn, bool conv) {
+// Two k-blocks per stage where a k-block's MMAs are shorter than, or about as long as, a barrier
+// round trip: the 256 x 128 tiles, every convolution product (whose producers also form box
+// coordinates) and the forward products (bias + ReLU, logits); measured, the 256 x 256 input- and
+// weight-gradient products gained nothing.  HS_KSTAGE=1 keeps one, HS_KSTAGE=2 takes two
+// everywhere (the same MMAs in the same order: identical results).
+inline bool pair_two_kblocks(int tn, bool conv, int epi) {
   const char* v = getenv("HS_KSTAGE");   // read per launch: a step replayed from a graph launches nothing
   const int forced = v ? atoi(v) : 0;
   if (forced == 1) return false;
   if (forced == 2) return true;
-  return tn == 128 || conv;
+  return tn == 128 || conv || epi == kTcEpiBiasReluBf16 || epi == kTcEpiBiasF32;
 }
 
 template <int EPI, bool A_MN, bool B_MN, bool CONV, int TN = 256, int EW = 4>
 cudaError_t launch_pair_variant(const TcGemmParams& p, int pairs_wanted, int num_sms, cudaStream_t s) {
-  if (pair_two_kblocks(TN, CONV)) return launch_pair_variant1<EPI, A_MN, B_MN, CONV, TN, EW, 2>(p, pairs_wanted, num_sms, s);
+  if (pair_two_kblocks(TN, CONV, EPI)) return launch_pair_variant1<EPI, A_MN, B_MN, CONV, TN, EW, 2>(p, pairs_wanted, num_sms, s);
   return launch_pair_variant1<EPI, A_MN, B_MN, CONV, TN, EW, 1>(p, pairs_wanted, num_sms, s);
 }
 
