@@ -733,6 +733,11 @@ hs_status cnn_build_static(hs_ctx* c) {
   }
   const int N = c->N;
   auto bf = [](void* p) { return reinterpret_cast<const __nv_bfloat16*>(p); };
+  c->conv_first_on = c->precision == HS_BF16 && conv_first_ok(c->convs[0]);
+  if (c->conv_first_on) {
+    hs_status st = conv_first_plan(c, &c->conv_first);
+    if (st != HS_OK) return st;
+  }
   c->tc_fwd.assign(4, TcGemmParams{});
   c->tc_dgrad.assign(4, TcGemmParams{});
   for (int k = 0; k < 3; ++k) {
@@ -793,6 +798,16 @@ hs_status cnn_step(hs_ctx* c, float* params, const float* x, const int32_t* y, c
     PhaseScope ph(c, HS_PHASE_FORWARD, s);
     for (int k = 0; k < 3; ++k) {
       const int64_t n_items = L[k].rows * L[k].cin;
+      if (k == 0 && c->conv_first_on && conv_first_bind_input(c, x)) {
+        // input boxes, patch rows, product, bias + ReLU in one kernel (the patch rows also written
+        // for the weight gradient)
+        ConvFirstParams& f = c->conv_first;
+        f.bias = params + L[0].b_off;
+        cudaError_t e = launch_conv_first(f, c->num_sms, s);
+        if (e != cudaSuccess) return cuda_fail(c, e, "first convolution launch");
+        ph.launched();
+        continue;
+      }
       if (k == 0) {
         if (bf16)
           launch_im2col_first(x, N, L[0], reinterpret_cast<__nv_bfloat16*>(c->d_col[0]), s);

@@ -27,6 +27,24 @@ struct ConvLayer {
 
 inline int64_t round_up(int64_t v, int64_t m) { return (v + m - 1) / m * m; }
 
+// The first convolution in one kernel (csrc/conv_first.cu): patch rows from the NCHW fp32 input in
+// shared memory (and written out for the weight gradient), the product with the resident bf16
+// weights, bias + ReLU into the NHWC bf16 activations.
+struct ConvFirstParams {
+  CUtensorMap tmW;            // bf16 weights [Cout][Kp], K-major, one box of 64 x npad
+  CUtensorMap tmX;            // the NCHW fp32 input in boxes of box_w x box_h x C (tc_make_nchw_box_map)
+  const float* x;             // NCHW fp32 input (the one tmX maps)
+  const float* bias;          // fp32 [Cout] (theta's bias of the layer, per launch)
+  __nv_bfloat16* col;         // patch rows out [rows][Kp] (tap-major, ones column at 9 * C)
+  __nv_bfloat16* out;         // activations [rows][Cout]
+  int64_t rows;               // N * Ho * Wo
+  int C, H, W, Ho, Wo, stride, Cout, Kp;
+  int npad, acc_cols;         // MMA width (Cout rounded up to 16), tensor-memory columns per accumulator
+  int R, tpi, tiles;          // output rows per tile (whole rows of one image), tiles per image, tiles
+  int box_w, box_h;           // input box: columns from -4, rows from stride * ho0 - 1
+  DevStatus* st;
+};
+
 // Per-layer bias-gradient chunk tables (worker, row begin, row end) for a given rows-per-sample.
 struct ChunkTable {
   int4* d_chunks = nullptr;
@@ -192,6 +210,8 @@ struct hs_ctx {
   hs::ChunkTable cnn_chunks[4];
   hs::CnnWgrad cnn_wgrad[4];
   bool cnn_fuse_update = true;        // HS_CNN_FUSED_UPDATE=0: split-K reductions, slab update and permutations apart
+  bool conv_first_on = false;         // bf16: the first convolution's forward in one kernel (conv_first_plan)
+  hs::ConvFirstParams conv_first{};
   const float* cnn_wcopy_src = nullptr;   // the params the bf16 weight copies (wperm, wsub) were last written from
 
   // tensor-core launch parameters (bf16 precision)
@@ -280,5 +300,12 @@ hs_status cnn_step(hs_ctx* c, float* params, const float* x, const int32_t* y, c
 bool cnn_fused_update(const hs_ctx* c);
 hs_status cnn_refresh_weights(hs_ctx* c, const float* params, cudaStream_t s);
 hs_status launch_cnn_update(hs_ctx* c, float* params, float lr, const float* lr_dev, cudaStream_t s);
+// The first convolution's forward in one kernel where its shape allows (HS_CONV_FIRST=0: never)
+bool conv_first_ok(const ConvLayer& L);
+hs_status conv_first_plan(hs_ctx* c, ConvFirstParams* p);
+// Points the input map at x (re-encoded only when x changes); false: x is not addressable by TMA
+// (the generic path runs instead)
+bool conv_first_bind_input(hs_ctx* c, const float* x);
+cudaError_t launch_conv_first(const ConvFirstParams& p, int num_sms, cudaStream_t s);
 
 }  // namespace hs

@@ -466,6 +466,28 @@ bool tc_make_grid_map(CUtensorMap* tm, const void* base, int C, int cols, int ro
   return true;
 }
 
+bool tc_make_nchw_box_map(CUtensorMap* tm, const float* x, int64_t images, int C, int H, int W, int box_w, int box_h,
+                          const char** why) {
+  if (!g_encode && !tc_init_driver(why)) return false;
+  if ((reinterpret_cast<uintptr_t>(x) & 15u) != 0 || (W * 4) % 16 || box_w % 4 || box_w > 256 || box_h > 256 ||
+      C > 256 || images < 1) {
+    *why = "NCHW input not addressable by TMA boxes";
+    return false;
+  }
+  cuuint64_t dims[4] = {(cuuint64_t)W, (cuuint64_t)H, (cuuint64_t)C, (cuuint64_t)images};
+  cuuint64_t strides[3] = {(cuuint64_t)W * 4, (cuuint64_t)H * W * 4, (cuuint64_t)C * H * W * 4};
+  cuuint32_t box[4] = {(cuuint32_t)box_w, (cuuint32_t)box_h, (cuuint32_t)C, 1};
+  cuuint32_t estr[4] = {1, 1, 1, 1};
+  CUresult r = g_encode(tm, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, const_cast<float*>(x), dims, strides, box, estr,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) {
+    *why = "cuTensorMapEncodeTiled rejected the NCHW input";
+    return false;
+  }
+  return true;
+}
+
 bool tc_make_store_map_parts(CUtensorMap* tm, float* base, int64_t rows, int64_t cols, int64_t ld, int64_t parts,
                              int64_t part_stride, const char** why) {
   if (!g_encode && !tc_init_driver(why)) return false;

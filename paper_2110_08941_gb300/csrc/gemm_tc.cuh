@@ -143,6 +143,11 @@ bool tc_make_store_map_bf16_32(CUtensorMap* tm, void* base, int64_t rows, int64_
 // box at byte 64 * r, fp32, or 32 * r, bf16, of the staging buffer).
 bool tc_make_store_map_16(CUtensorMap* tm, void* base, bool fp32, int64_t rows, int64_t cols, int64_t ld,
                           const char** why);
+// NCHW fp32 tensor [images][C][H][W] (W a multiple of 4, 16-byte aligned base) for TMA loads of
+// box_w columns x box_h rows x all C channels of one image, unswizzled (row r of channel c at float
+// (c * box_h + r) * box_w of the box); out-of-range coordinates read zeros.
+bool tc_make_nchw_box_map(CUtensorMap* tm, const float* x, int64_t images, int C, int H, int W, int box_w, int box_h,
+                          const char** why);
 // The same over `parts` such matrices `part_stride` elements apart (split-K partials, fp32).
 bool tc_make_store_map_parts(CUtensorMap* tm, float* base, int64_t rows, int64_t cols, int64_t ld, int64_t parts,
                              int64_t part_stride, const char** why);

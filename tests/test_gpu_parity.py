@@ -412,3 +412,29 @@ def test_two_kblocks_per_stage_are_bit_identical(monkeypatch, case):
     assert a["losses"] == b["losses"]
     if debug:
         assert np.array_equal(a["slabs_first"], b["slabs_first"])
+
+
+@pytest.mark.parametrize("dims,N,M,weights", [(None, None, None, None),
+                                              ((3, 9, 7, 8, 16, 24, 5), 7, 3, [1.0, 2.0, 4.0]),
+                                              ((2, 6, 6, 16, 8, 8, 3), 4, 4, None),
+                                              ((3, 16, 16, 32, 32, 64, 10), 33, 2, [1.0, 5.0])])
+def test_first_convolution_kernel_is_bit_identical(monkeypatch, dims, N, M, weights):
+    """The first convolution's forward as one kernel (patch rows built in shared memory from the NCHW
+    input and written out for the weight gradient, resident weights, bias + ReLU) against the
+    materialised patch rows and the tiled product (HS_CONV_FIRST=0): same bf16 operands and fp32
+    sums, so theta, losses and per-worker gradients agree bit for bit - on the CNN workload and on
+    8-, 16- and 32-channel first convolutions over odd grids with a ragged last tile."""
+    if dims is None:
+        wl, x, y, theta0, w = _inputs(synth.CFG4)
+    else:
+        rng = np.random.default_rng(N + dims[1])
+        x = rng.standard_normal((N,) + tuple(dims[:3]), dtype=np.float32)
+        y = rng.integers(0, dims[-1], N, dtype=np.int32)
+        theta0 = synth.he_normal_params(synth.CNN, dims, 5)
+        wl = types.SimpleNamespace(arch=synth.CNN, dims=dims, global_batch=N, workers=M, lr=0.05)
+        w = weights
+    one = _cnn_run_env(monkeypatch, {}, wl, x, y, theta0, w, 3)
+    two = _cnn_run_env(monkeypatch, {"HS_CONV_FIRST": "0"}, wl, x, y, theta0, w, 3)
+    assert torch.equal(one[0], two[0])
+    assert one[1] == two[1]
+    assert torch.equal(one[2], two[2])
