@@ -319,8 +319,18 @@ __global__ void permute_weights_kernel(const float* __restrict__ w, int cout, in
 // TcConvGeom): class (ph, pw) = 2 * ph + pw holds [taps x Cout][Cin], row t * Cout + co, where the
 // class's row taps are kh = 1 (ph = 0) or kh = 0, 2 (ph = 1) in that order, columns likewise, and
 // t = th * (number of column taps) + tw.  Classes hold 1, 2, 2, 4 taps and sit back to back.
+// comb: the combined layout of the one-product form instead: row T * Cout + co, column cls * Cin + ci,
+// T = 2 (1 - dh) + (1 - dw) the tap's shift (dh = ph && kh == 0, dw = pw && kw == 0); the other
+// blocks stay zero.
+__device__ __forceinline__ int subpixel_comb_index(int co, int ci, int kh, int kw, int cout, int cin) {
+  const int ph = kh != 1, pw = kw != 1;
+  const int dh = ph && kh == 0, dw = pw && kw == 0;
+  const int T = 2 * (1 - dh) + (1 - dw);
+  return ((T * cout + co) * 4 + 2 * ph + pw) * cin + ci;   // < 16 Cout Cin, well inside 32 bits
+}
+
 __global__ void permute_weights_subpixel_kernel(const float* __restrict__ w, int cout, int cin,
-                                                __nv_bfloat16* __restrict__ wc) {
+                                                __nv_bfloat16* __restrict__ wc, int comb) {
   pdl_wait();
   pdl_trigger();
   const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
@@ -329,6 +339,10 @@ __global__ void permute_weights_subpixel_kernel(const float* __restrict__ w, int
   const int ci = (int)((idx / 9) % cin);
   const int co = (int)(idx / (9 * (int64_t)cin));
   const int kh = tap / 3, kw = tap % 3;
+  if (comb) {
+    wc[subpixel_comb_index(co, ci, kh, kw, cout, cin)] = __float2bfloat16_rn(w[idx]);
+    return;
+  }
   const int ph = kh != 1, pw = kw != 1;
   const int th = (ph && kh == 2) ? 1 : 0, tw = (pw && kw == 2) ? 1 : 0;
   const int t = th * (pw ? 2 : 1) + tw;
@@ -388,7 +402,8 @@ struct CnnUpdLayer {
   int64_t w_off, b_off, first;   // theta offsets; first work item of the layer
   __nv_bfloat16* wperm;       // tap-major bf16 copy [rows][Kp] (convolutions)
   int Kp;
-  __nv_bfloat16* wsub;        // sub-pixel class copy (stride-2 convolutions whose input gradient is sub-pixel)
+  __nv_bfloat16* wsub;        // sub-pixel copy (stride-2 convolutions whose input gradient is sub-pixel): class
+                              // matrices, or the combined layout (kComb, subpixel_comb_index)
 };
 struct CnnUpdArgs {
   CnnUpdLayer layer[4];
@@ -403,7 +418,7 @@ struct CnnUpdArgs {
 // One layer's items for one block: the layer is the block's (blocks are assigned to layers in
 // order), read into registers through a switch so the kernel never indexes its parameter array
 // at run time.
-template <bool kRecipe>
+template <bool kRecipe, bool kComb>
 __device__ __forceinline__ void cnn_update_item(const CnnUpdLayer& L, int64_t it, float* __restrict__ theta, int M,
                                                 const float* __restrict__ w, float lr,
                                                 __nv_bfloat16* __restrict__ shadow, float* __restrict__ mbuf,
@@ -447,7 +462,9 @@ __device__ __forceinline__ void cnn_update_item(const CnnUpdLayer& L, int64_t it
   shadow[j] = tb;
   if (L.cin && pc < 9 * L.cin) {
     L.wperm[(int64_t)co * L.Kp + pc] = tb;
-    if (L.wsub) {
+    if (kComb && L.wsub) {
+      L.wsub[subpixel_comb_index(co, ci, tap / 3, tap % 3, L.rows, L.cin)] = tb;
+    } else if (L.wsub) {
       const int kh = tap / 3, kw = tap % 3;
       const int ph = kh != 1, pw = kw != 1;
       const int th = (ph && kh == 2) ? 1 : 0, tw = (pw && kw == 2) ? 1 : 0;
@@ -459,7 +476,9 @@ __device__ __forceinline__ void cnn_update_item(const CnnUpdLayer& L, int64_t it
   }
 }
 
-template <bool kRecipe>
+// kComb: the sub-pixel weight copies in the combined layout (a compile-time choice: the run-time branch
+// cost the kernel a third of its speed).
+template <bool kRecipe, bool kComb>
 __global__ void __launch_bounds__(256) cnn_update_kernel(const CnnUpdArgs a, float* __restrict__ theta, int M,
                                                          const float* __restrict__ w, float lr_arg,
                                                          const float* __restrict__ lr_dev,
@@ -489,7 +508,7 @@ __global__ void __launch_bounds__(256) cnn_update_kernel(const CnnUpdArgs a, flo
   else { L = a.layer[0]; base = 0; }
   const int64_t it = (int64_t)(b - base) * blockDim.x + threadIdx.x;
   if (it >= (int64_t)L.rows * L.cols) return;
-  cnn_update_item<kRecipe>(L, it, theta, M, w, lr, shadow, mbuf, mu, wd, first);
+  cnn_update_item<kRecipe, kComb>(L, it, theta, M, w, lr, shadow, mbuf, mu, wd, first);
 }
 
 inline int blocks_for(int64_t n, int threads) { return (int)((n + threads - 1) / threads); }
@@ -669,7 +688,10 @@ hs_status plan_dense(hs_ctx* c, TcGemmParams* p, int epi, const __nv_bfloat16* a
 // Input gradient of stride-2 convolution k as four grouped class products (see TcConvGeom):
 // A = dA_k [N][Ho][Wo][Cout] (64-pixel boxes), B = the class weights (MN-major), D = the class
 // pixels of dA_{k-1} [N][H][W][Cin] (32-pixel store boxes), ReLU' of h_{k-1} fused.
+hs_status plan_subpixel_dgrad_comb(hs_ctx* c, int k);
+
 hs_status plan_subpixel_dgrad(hs_ctx* c, int k) {
+  if (c->convs[k].comb) return plan_subpixel_dgrad_comb(c, k);
   const ConvLayer& L = c->convs[k];
   const char* why = nullptr;
   TcGemmParams& p = c->tc_dgrad[k];
@@ -715,6 +737,66 @@ hs_status plan_subpixel_dgrad(hs_ctx* c, int k) {
   p.ldd = L.cin;
   p.Z = reinterpret_cast<const __nv_bfloat16*>(c->d_cact[k - 1]);
   p.ldz = L.cin;
+  if (c->d_relu_bits.size() > (size_t)(k - 1) && c->d_relu_bits[k - 1]) {   // ReLU' of h_{k-1} as bits
+    p.relu_bits_in = c->d_relu_bits[k - 1];
+    p.bits_ld = c->convs[k - 1].rows;
+  }
+  p.st = c->d_status;
+  return HS_OK;
+}
+
+// The same input gradient as one product over all four classes (conv_d = 2): rows = the Ho x Wo grid,
+// K = the four shifts of A (the class-3 tap order (1,1), (1,0), (0,1), (0,0)) x Cout, columns = four
+// blocks of Cin (class c = 2 ph + pw), B = the combined weights [4 x Cout][4 x Cin] whose block (shift,
+// class) holds the class's tap with that shift, or zeros.  Each class sums the products of the
+// grouped form over its taps in the same order, with exact zeros between: the same bits.  A k-block
+// of A (one shift of the output gradient) now feeds the MMAs of every class that reads that shift
+// (four, two, two and one of them) in one 256-wide product instead of one 64- or 128-wide product
+// per class tap.
+hs_status plan_subpixel_dgrad_comb(hs_ctx* c, int k) {
+  const ConvLayer& L = c->convs[k];
+  const char* why = nullptr;
+  TcGemmParams& p = c->tc_dgrad[k];
+  std::memset(&p, 0, sizeof(p));
+  const int64_t hw = (int64_t)L.hout * L.wout;
+  auto* dprev = reinterpret_cast<__nv_bfloat16*>(c->d_dA[k - 1]);
+  const int abox = grid_a_box(L.hout, L.wout);
+  bool ok = tc_make_grid_map(&p.tmA[0], c->d_dA[k], L.cout, L.wout, L.hout, c->N, L.cout, (int64_t)L.wout * L.cout,
+                             hw * L.cout, abox, &why) &&
+            tc_make_mnmajor_map(&p.tmB[0], TcOperand{c->d_wsub[k], 4LL * L.cout, 4 * L.cin, 4LL * L.cin}, &why);
+  for (int g = 0; g < 4 && ok; ++g) {
+    const int ph = g >> 1, pw = g & 1;
+    ok = tc_make_grid_map(&p.tmD[g], dprev + ((int64_t)ph * L.win + pw) * L.cin, L.cin, L.wout, L.hout, c->N,
+                          2LL * L.cin, 2LL * L.win * L.cin, (int64_t)L.hin * L.win * L.cin, 32, &why);
+  }
+  if (!ok) return fail(c, HS_ERR_CUDA, why);
+  p.num_kb[0] = (int32_t)(4LL * L.cout / kTcBK);
+  p.groups = 1;
+  p.Mdim = (int32_t)L.rows;
+  p.Ndim = 4 * L.cin;
+  p.n_store = 4 * L.cin;
+  p.tiles_m = (p.Mdim + kTcBM - 1) / kTcBM;
+  p.tiles_n = (p.n_store + kTcBN - 1) / kTcBN;
+  p.epi = kTcEpiMaskBf16;
+  p.a_mn = 0;
+  p.b_mn = 1;
+  p.conv_a = 2;
+  p.conv_d = 2;
+  p.form = kTcFormPair;   // 256 x 256 SM-pair tiles
+  p.conv = tc_conv_geom(L.cout, L.hout, L.wout, L.stride);
+  p.conv.a_box = abox;
+  p.conv.a_cls = 3;
+  p.conv.cin_d = L.cin;
+  p.conv.H = L.hin;
+  p.conv.W = L.win;
+  p.D = dprev;
+  p.ldd = L.cin;
+  p.Z = reinterpret_cast<const __nv_bfloat16*>(c->d_cact[k - 1]);
+  p.ldz = L.cin;
+  if (c->d_relu_bits.size() > (size_t)(k - 1) && c->d_relu_bits[k - 1]) {   // ReLU' of h_{k-1} as bits
+    p.relu_bits_in = c->d_relu_bits[k - 1];
+    p.bits_ld = c->convs[k - 1].rows;
+  }
   p.st = c->d_status;
   return HS_OK;
 }
@@ -737,6 +819,10 @@ hs_status cnn_build_static(hs_ctx* c) {
   if (c->conv_first_on) {
     hs_status st = conv_first_plan(c, &c->conv_first);
     if (st != HS_OK) return st;
+    if (c->d_relu_bits.size() > 0 && c->d_relu_bits[0]) {
+      c->conv_first.bits = c->d_relu_bits[0];
+      c->conv_first.bits_ld = c->convs[0].rows;
+    }
   }
   c->tc_fwd.assign(4, TcGemmParams{});
   c->tc_dgrad.assign(4, TcGemmParams{});
@@ -749,6 +835,10 @@ hs_status cnn_build_static(hs_ctx* c) {
                               false, c->d_cact[k], false, (int)L.rows, L.cout, L.cout, L.cout, nullptr, 0,
                               L.implicit ? &L : nullptr, L.cout <= 128);
     if (st != HS_OK) return st;
+    if (c->d_relu_bits.size() > (size_t)k && c->d_relu_bits[k]) {   // ReLU' bits for the next input gradient
+      c->tc_fwd[k].relu_bits_out = c->d_relu_bits[k];
+      c->tc_fwd[k].bits_ld = L.rows;
+    }
   }
   // fully connected layer on the pooled features
   const int c3 = c->convs[2].cout;
@@ -1004,7 +1094,7 @@ hs_status cnn_refresh_weights(hs_ctx* c, const float* params, cudaStream_t s) {
     ph.launched();
     if (L.subpixel) {
       launch_pdl(permute_weights_subpixel_kernel, blocks_for(9LL * L.cout * L.cin, T), T, 0, s,
-          params + L.w_off, L.cout, L.cin, c->d_wsub[k]);
+          params + L.w_off, L.cout, L.cin, c->d_wsub[k], L.comb ? 1 : 0);
       ph.launched();
     }
   }
@@ -1046,13 +1136,16 @@ hs_status launch_cnn_update(hs_ctx* c, float* params, float lr, const float* lr_
   a.Ps = c->Ps;
   if (items + c->C != c->P) return fail(c, HS_ERR_CUDA, "fused CNN update does not cover the parameters");
   PhaseScope ph(c, HS_PHASE_UPDATE, s);
+  // the sub-pixel layers share the layout (a sub-pixel layer's input has a multiple of 64 channels)
+  const bool comb = c->convs[1].comb || c->convs[2].comb;
+  auto kern = c->opt_recipe ? (comb ? cnn_update_kernel<true, true> : cnn_update_kernel<true, false>)
+                            : (comb ? cnn_update_kernel<false, true> : cnn_update_kernel<false, false>);
   if (c->opt_recipe)
-    launch_pdl(cnn_update_kernel<true>, blocks, T, 0, s, a, params, c->M,
-               static_cast<const float*>(c->d_w), lr, lr_dev, c->d_shadow, c->d_mom, c->opt_momentum,
-               c->opt_weight_decay, c->mom_valid ? 0 : 1);
+    launch_pdl(kern, blocks, T, 0, s, a, params, c->M, static_cast<const float*>(c->d_w), lr, lr_dev, c->d_shadow,
+               c->d_mom, c->opt_momentum, c->opt_weight_decay, c->mom_valid ? 0 : 1);
   else
-    launch_pdl(cnn_update_kernel<false>, blocks, T, 0, s, a, params, c->M,
-               static_cast<const float*>(c->d_w), lr, lr_dev, c->d_shadow, static_cast<float*>(nullptr), 0.f, 0.f, 0);
+    launch_pdl(kern, blocks, T, 0, s, a, params, c->M, static_cast<const float*>(c->d_w), lr, lr_dev, c->d_shadow,
+               static_cast<float*>(nullptr), 0.f, 0.f, 0);
   ph.launched();
   HS_CUDA(c, cudaGetLastError());
   return HS_OK;

@@ -227,7 +227,9 @@ __global__ void __launch_bounds__(kCfThreads, 1) conv_first_fwd_kernel(const __g
       const bool live = r < p.R * p.Wo && ho0 + px.x < p.Ho;
       uint4* orow = reinterpret_cast<uint4*>(p.out + (((int64_t)n * p.Ho + ho0) * p.Wo + r) * p.Cout);
       const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(a * acc_cols);
-      // 32 columns per round: two loads issued, one wait
+      // 32 columns per round: two loads issued, one wait; with p.bits, the ReLU' of each 64 stored
+      // values as one word
+      uint64_t bits = 0;
       for (int cb = 0; cb < p.npad; cb += 32) {
         uint32_t v[2][16];
 #pragma unroll
@@ -248,6 +250,19 @@ __global__ void __launch_bounds__(kCfThreads, 1) conv_first_fwd_kernel(const __g
           if (live) {
             orow[c0 >> 3] = make_uint4(o[0], o[1], o[2], o[3]);
             if (c0 + 8 < p.Cout) orow[(c0 >> 3) + 1] = make_uint4(o[4], o[5], o[6], o[7]);
+          }
+          if (p.bits) {
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+              const __nv_bfloat162 pr = *reinterpret_cast<const __nv_bfloat162*>(&o[e]);
+              bits |= (uint64_t)(__low2float(pr) > 0.f) << ((c0 & 63) + 2 * e);
+              bits |= (uint64_t)(__high2float(pr) > 0.f) << ((c0 & 63) + 2 * e + 1);
+            }
+            if (((c0 + 16) & 63) == 0) {
+              if (live)
+                p.bits[(int64_t)(c0 >> 6) * p.bits_ld + ((int64_t)n * p.Ho + ho0) * p.Wo + r] = bits;
+              bits = 0;
+            }
           }
         }
       }

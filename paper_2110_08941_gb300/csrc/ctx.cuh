@@ -23,6 +23,9 @@ struct ConvLayer {
   int64_t rows;       // N * hout * wout
   bool implicit;      // bf16: the products read the patch rows straight from the input (no col buffer)
   bool subpixel;      // bf16: the input gradient is the grouped sub-pixel product (no patch-space buffer)
+  bool comb;          // ... as one product whose columns are the four classes' blocks (d_wsub holds
+                      // the combined weights [4 shifts x Cout][4 classes x Cin]; else [9 x Cout][Cin]
+                      // class matrices)
 };
 
 inline int64_t round_up(int64_t v, int64_t m) { return (v + m - 1) / m * m; }
@@ -40,6 +43,8 @@ struct ConvFirstParams {
   int64_t rows;               // N * Ho * Wo
   int C, H, W, Ho, Wo, stride, Cout, Kp;
   int npad, acc_cols;         // MMA width (Cout rounded up to 16), tensor-memory columns per accumulator
+  uint64_t* bits;             // non-null: ReLU' of the stored activations as bits, word [c / 64][row]
+  int64_t bits_ld;            // (rows); Cout a multiple of 64
   int R, tpi, tiles;          // output rows per tile (whole rows of one image), tiles per image, tiles
   int box_w, box_h;           // input box: columns from -4, rows from stride * ho0 - 1
   DevStatus* st;
@@ -211,6 +216,9 @@ struct hs_ctx {
   hs::CnnWgrad cnn_wgrad[4];
   bool cnn_fuse_update = true;        // HS_CNN_FUSED_UPDATE=0: split-K reductions, slab update and permutations apart
   bool conv_first_on = false;         // bf16: the first convolution's forward in one kernel (conv_first_plan)
+  bool subpixel_comb = true;          // sub-pixel input gradients as one product over all four classes
+                                      // (HS_SUBPIXEL=classes: one group per class); per layer where its
+                                      // input has a multiple of 64 channels (ConvLayer::comb)
   hs::ConvFirstParams conv_first{};
   const float* cnn_wcopy_src = nullptr;   // the params the bf16 weight copies (wperm, wsub) were last written from
 

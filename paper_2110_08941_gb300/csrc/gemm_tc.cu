@@ -118,7 +118,8 @@ __global__ void __launch_bounds__(threads_of<CONV>(), 1) tc_gemm_kernel(const __
         // patch-column blocks of A and pixel blocks of B, stepped once per k-block
         ConvColIter a_it;
         ConvRowIter b_it;
-        if (CONV && p.conv_a) a_it.init(p.conv, p.conv_a == 2 ? w.g : -1, w.kb_lo * BK);
+        if (CONV && p.conv_a)
+          a_it.init(p.conv, p.conv_a == 2 ? (p.conv.a_cls >= 0 ? p.conv.a_cls : w.g) : -1, w.kb_lo * BK);
         if (CONV && B_MN && p.conv_b) b_it.init(p.conv, w.kb_lo * BK);
         bool ok = true;
         for (int kb = w.kb_lo; kb < w.kb_hi; ++kb) {
@@ -398,6 +399,8 @@ TcConvGeom tc_conv_geom(int C, int Ho, int Wo, int stride) {
   g.stride = stride;
   g.ones_col = 9 * C;
   g.a_box = 64;
+  g.a_cls = -1;
+  g.cin_d = 0;
   return g;
 }
 

@@ -42,6 +42,9 @@ struct TcConvGeom {
   int32_t H, W;       // input grid (sub-pixel input gradient: where the ReLU' mask is read)
   int32_t a_box;      // output pixels per A box (conv_a): 64, or 128 (one box per 128 rows, whole
                       // output rows of one image or whole images; half the box issues per k-block)
+  int32_t a_cls;      // sub-pixel A (conv_a = 2): -1 = the group's class, else this class's taps for
+                      // every group (class 3: all four shifts (1,1), (1,0), (0,1), (0,0) in that order)
+  int32_t cin_d;      // conv_d = 2: input-gradient channels per class block of D's columns
 };
 
 // D[Mdim x n_store] (row-major, leading dimension ldd) = A[Mdim x K] * B[K x Ndim] + epilogue.
@@ -54,6 +57,10 @@ struct TcConvGeom {
 // conv_a = 2: A is the shifted output gradient of the sub-pixel input gradient (tc_make_grid_map,
 //             64-pixel boxes), class = group; conv_d = 1: D rows are that class's input pixels
 //             (tmD[g] from tc_make_grid_map with 32-pixel boxes) and the mask Z is read there.
+//             conv_d = 2: one product for all four classes: D's columns are four blocks of
+//             conv.cin_d channels, block c = class c (rows through tmD[c], mask at class c's pixels);
+//             A walks the four shifts (conv.a_cls = 3) and B holds, per shift, each class's tap
+//             with that shift or zeros.
 // conv_b: B (MN-major) is the implicit patch rows of the group's samples (tmB[g] a conv map over
 // them), and tmOnes supplies the ones column at conv.ones_col.
 struct TcGemmParams {

@@ -159,7 +159,8 @@ __global__ void __launch_bounds__(PairCfg<TN, EW, CONV ? kConvProducers : 1, KS>
         // patch-column blocks of A and pixel blocks of B, stepped once per k-block
         ConvColIter a_it;
         ConvRowIter b_it;
-        if (CONV && p.conv_a) a_it.init(p.conv, p.conv_a == 2 ? w.g : -1, w.kb_lo * BK);
+        if (CONV && p.conv_a)
+          a_it.init(p.conv, p.conv_a == 2 ? (p.conv.a_cls >= 0 ? p.conv.a_cls : w.g) : -1, w.kb_lo * BK);
         if (CONV && B_MN && p.conv_b) b_it.init(p.conv, w.kb_lo * BK);
         bool ok = true;
         for (int kb = w.kb_lo; kb < w.kb_hi; kb += KS) {

@@ -888,6 +888,8 @@ hs_status hs_init(const hs_model_desc* model, int32_t M, const double* compute_w
   // about 0.1 ms of host launches) keeps eager launches.  HS_STEP_GRAPH=0 / =1 force either.
   const char* cf = getenv("HS_CNN_FUSED_UPDATE");
   c->cnn_fuse_update = !(cf && !strcmp(cf, "0"));
+  const char* sp = getenv("HS_SUBPIXEL");
+  c->subpixel_comb = !(sp && !strcmp(sp, "classes"));
   const char* sg = getenv("HS_STEP_GRAPH");
   c->graph_on = !(sg && !strcmp(sg, "0"));
   c->graph_force = sg && !strcmp(sg, "1");
@@ -1017,9 +1019,24 @@ hs_status hs_init(const hs_model_desc* model, int32_t M, const double* compute_w
       for (int k = 0; k < 3; ++k)
         chk(dalloc(c, &c->d_wperm[k], sizeof(__nv_bfloat16) * (size_t)c->convs[k].cout * c->convs[k].Kp));
       chk(dalloc(c, &c->d_ones, sizeof(__nv_bfloat16) * 64 * 64));
-      for (int k = 1; k < 3; ++k)
-        if (c->convs[k].subpixel)
-          chk(dalloc(c, &c->d_wsub[k], sizeof(__nv_bfloat16) * 9 * (size_t)c->convs[k].cout * c->convs[k].cin));
+      // ReLU' of the first two convolutions' activations as bits, where the next convolution's input
+      // gradient is the sub-pixel product (it reads them at its class pixels; HS_RELU_BITS=0: the
+      // activations themselves)
+      const char* rb = getenv("HS_RELU_BITS");
+      c->d_relu_bits.assign(3, nullptr);
+      for (int k = 0; k < 2 && !(rb && !strcmp(rb, "0")); ++k)
+        if (c->convs[k].cout % 64 == 0 && c->convs[k + 1].subpixel)
+          chk(dalloc(c, &c->d_relu_bits[k], sizeof(uint64_t) * (size_t)c->convs[k].rows * (c->convs[k].cout / 64)));
+      for (int k = 1; k < 3; ++k) {
+        hs::ConvLayer& Lk = c->convs[k];
+        Lk.comb = Lk.subpixel && c->subpixel_comb && Lk.cin % 64 == 0;
+        if (!Lk.subpixel) continue;
+        // combined: 16 blocks of Cout x Cin per shift and class, 7 of them zero for good
+        const size_t n = (Lk.comb ? 16 : 9) * (size_t)Lk.cout * Lk.cin;
+        chk(dalloc(c, &c->d_wsub[k], sizeof(__nv_bfloat16) * n));
+        if (s2 == HS_OK && Lk.comb && cudaMemset(c->d_wsub[k], 0, sizeof(__nv_bfloat16) * n) != cudaSuccess)
+          chk(HS_ERR_CUDA);
+      }
     }
     delta_elems = N * (size_t)c->Cp;
     for (int k = 0; k < 4; ++k) {

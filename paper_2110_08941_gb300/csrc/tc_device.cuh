@@ -229,7 +229,13 @@ __device__ __forceinline__ void store_strip(const TcGemmParams& p, const CUtenso
     tma_store_3d(td, buf, n_base, row0, part);
   } else if (CONV && p.conv_d) {
     const int img = row0 / p.conv.hw;
-    const int c[4] = {n_base, 0, (row0 - img * p.conv.hw) / p.conv.Wo, img};
+    int col = n_base;
+    if (p.conv_d == 2) {   // column block = class: its own pixel grid
+      const int cls = n_base / p.conv.cin_d;
+      td = &p.tmD[cls];
+      col = n_base - cls * p.conv.cin_d;
+    }
+    const int c[4] = {col, 0, (row0 - img * p.conv.hw) / p.conv.Wo, img};
     tma_store_4d(td, buf, c);
   } else {
     tma_store_2d(td, buf, n_base, row0);
@@ -440,22 +446,27 @@ __device__ __forceinline__ void load_mask_unit(const TcGemmParams& p, int grp, i
 #pragma unroll
   for (int j = 0; j < 8; ++j) zq[j] = make_uint4(0u, 0u, 0u, 0u);
   if (row >= p.Mdim || n_base >= p.n_store) return;
-  if (!CONV && p.relu_bits_in) {
-    // the packed form of the same decisions, one 64-bit word per row and 64-column unit
-    const unsigned long long b =
-        __ldg(reinterpret_cast<const unsigned long long*>(p.relu_bits_in) + (int64_t)(n_base >> 6) * p.bits_ld + row);
-    zq[0].x = (uint32_t)b;
-    zq[0].y = (uint32_t)(b >> 32);
-    return;
-  }
   int64_t zrow = row;
+  int col = n_base;
   if (CONV && p.conv_d) {
+    if (p.conv_d == 2) {   // column block = class
+      grp = n_base / p.conv.cin_d;
+      col = n_base - grp * p.conv.cin_d;
+    }
     const int img = row / p.conv.hw;
     const int rem = row - img * p.conv.hw;
     const int a = rem / p.conv.Wo, b = rem - a * p.conv.Wo;
     zrow = ((int64_t)img * p.conv.H + 2 * a + (grp >> 1)) * p.conv.W + 2 * b + (grp & 1);
   }
-  const __nv_bfloat16* z = p.Z + zrow * p.ldz + n_base;
+  if (p.relu_bits_in) {
+    // the packed form of the same decisions, one 64-bit word per row of Z and 64-column unit
+    const unsigned long long b =
+        __ldg(reinterpret_cast<const unsigned long long*>(p.relu_bits_in) + (int64_t)(col >> 6) * p.bits_ld + zrow);
+    zq[0].x = (uint32_t)b;
+    zq[0].y = (uint32_t)(b >> 32);
+    return;
+  }
+  const __nv_bfloat16* z = p.Z + zrow * p.ldz + col;
   if (n_base + 64 <= p.n_store) {
     const uint4* z4 = reinterpret_cast<const uint4*>(z);
 #pragma unroll
@@ -515,7 +526,7 @@ __device__ __forceinline__ void epilogue_unit(const TcGemmParams& p, int grp, in
         for (int j = 0; j < 64; ++j)
           v[j] = fmaxf(v[j] + ((n_base + j < p.Ndim) ? __ldg(p.bias + n_base + j) : 0.f), 0.f);
       }
-    } else if (!CONV && p.relu_bits_in) {   // kTcEpiMaskBf16, ReLU' from the packed bits (in zq[0])
+    } else if (p.relu_bits_in) {   // kTcEpiMaskBf16, ReLU' from the packed bits (in zq[0])
       const uint64_t bits = (uint64_t)zq[0].x | ((uint64_t)zq[0].y << 32);
 #pragma unroll
       for (int k = 0; k < 64; ++k) v[k] = ((bits >> k) & 1ull) ? v[k] : 0.f;

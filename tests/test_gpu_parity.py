@@ -438,3 +438,54 @@ def test_first_convolution_kernel_is_bit_identical(monkeypatch, dims, N, M, weig
     assert torch.equal(one[0], two[0])
     assert one[1] == two[1]
     assert torch.equal(one[2], two[2])
+
+
+@pytest.mark.parametrize("dims,N,M,weights", [(None, None, None, None),
+                                              ((3, 16, 16, 64, 128, 64, 7), 13, 3, [1.0, 2.0, 3.5]),
+                                              ((3, 16, 32, 64, 64, 64, 5), 9, 2, [2.0, 1.0])])
+def test_subpixel_one_product_is_bit_identical(monkeypatch, dims, N, M, weights):
+    """The stride-2 convolutions' input gradients as one product over the four sub-pixel classes
+    (columns in four class blocks, the four shifts of the output gradient as K, zero weight blocks
+    where a class has no tap with that shift) against one grouped product per class
+    (HS_SUBPIXEL=classes): every class sums the same products in the same order with exact zeros
+    between, so theta, losses and per-worker gradients agree bit for bit - on the CNN workload, and on
+    8x8 / 4x4 and 8x16 / 4x8 output grids with 64- and 128-channel inputs."""
+    if dims is None:
+        wl, x, y, theta0, w = _inputs(synth.CFG4)
+    else:
+        rng = np.random.default_rng(N + dims[1])
+        x = rng.standard_normal((N,) + tuple(dims[:3]), dtype=np.float32)
+        y = rng.integers(0, dims[-1], N, dtype=np.int32)
+        theta0 = synth.he_normal_params(synth.CNN, dims, 5)
+        wl = types.SimpleNamespace(arch=synth.CNN, dims=dims, global_batch=N, workers=M, lr=0.05)
+        w = weights
+    one = _cnn_run_env(monkeypatch, {}, wl, x, y, theta0, w, 3)
+    grouped = _cnn_run_env(monkeypatch, {"HS_SUBPIXEL": "classes"}, wl, x, y, theta0, w, 3)
+    assert torch.equal(one[0], grouped[0])
+    assert one[1] == grouped[1]
+    assert torch.equal(one[2], grouped[2])
+
+
+@pytest.mark.parametrize("dims,N,M,weights", [(None, None, None, None),
+                                              ((3, 16, 16, 64, 128, 64, 7), 13, 3, [1.0, 2.0, 3.5])])
+@pytest.mark.parametrize("subpixel", ["", "classes"])
+def test_cnn_relu_bits_are_bit_identical(monkeypatch, dims, N, M, weights, subpixel):
+    """ReLU' of the first two convolutions' activations stored as bits by their forward epilogues and
+    read by the next convolution's sub-pixel input gradient at its class pixels, against reading the
+    bf16 activations themselves (HS_RELU_BITS=0): the same decisions, so the same bits everywhere,
+    for the one-product and the per-class sub-pixel forms."""
+    if dims is None:
+        wl, x, y, theta0, w = _inputs(synth.CFG4)
+    else:
+        rng = np.random.default_rng(N + dims[1])
+        x = rng.standard_normal((N,) + tuple(dims[:3]), dtype=np.float32)
+        y = rng.integers(0, dims[-1], N, dtype=np.int32)
+        theta0 = synth.he_normal_params(synth.CNN, dims, 5)
+        wl = types.SimpleNamespace(arch=synth.CNN, dims=dims, global_batch=N, workers=M, lr=0.05)
+        w = weights
+    env = {"HS_SUBPIXEL": subpixel} if subpixel else {}
+    bits = _cnn_run_env(monkeypatch, env, wl, x, y, theta0, w, 3)
+    acts = _cnn_run_env(monkeypatch, dict(env, HS_RELU_BITS="0"), wl, x, y, theta0, w, 3)
+    assert torch.equal(bits[0], acts[0])
+    assert bits[1] == acts[1]
+    assert torch.equal(bits[2], acts[2])
