@@ -121,11 +121,22 @@ __global__ void __launch_bounds__(threads_of<CONV>(), 1) tc_gemm_kernel(const __
         if (CONV && p.conv_a)
           a_it.init(p.conv, p.conv_a == 2 ? (p.conv.a_cls >= 0 ? p.conv.a_cls : w.g) : -1, w.kb_lo * BK);
         if (CONV && B_MN && p.conv_b) b_it.init(p.conv, w.kb_lo * BK);
+        // 64-wide MN-major boxes wholly past the product's rows (A) or columns (B) are not loaded:
+        // the tile's outputs in those rows and columns are never stored, and every stored output
+        // reads only its own row of A and column of B, so whatever the skipped slots hold is
+        // harmless (the one-SM tile is 128 x 256; the first convolution's weight gradient is 64 x 28)
+        int a_live = BM / 64, b_live = BN / 64;
+        if (A_MN) a_live = max(1, min(BM / 64, (p.Mdim - c.tm * BM + 63) / 64));
+        if (B_MN) {
+          const int ncols = (CONV && p.conv_b) ? p.conv.ones_col + 1 : p.Ndim;
+          b_live = max(1, min(BN / 64, (ncols - c.tn * BN + 63) / 64));
+        }
+        const uint32_t tx = (uint32_t)((A_MN ? a_live * MN_CHUNK : A_STAGE) + (B_MN ? b_live * MN_CHUNK : B_STAGE));
         bool ok = true;
         for (int kb = w.kb_lo; kb < w.kb_hi; ++kb) {
           if (!mbar_wait(smem_u32(&empty_bar[s]), ph ^ 1u, abort_flag)) { ok = false; break; }
           const uint32_t fb = smem_u32(&full_bar[s]);
-          if (prod == 0) mbar_expect_tx(fb, STAGE_TX);
+          if (prod == 0) mbar_expect_tx(fb, tx);
           const int k0 = kb * BK;
           const uint32_t a_dst = smem_u32(sA + s * A_STAGE);
           const uint32_t b_dst = smem_u32(sB + s * B_STAGE);
@@ -133,7 +144,7 @@ __global__ void __launch_bounds__(threads_of<CONV>(), 1) tc_gemm_kernel(const __
           if (A_MN) {
 #pragma unroll
             for (int j = 0; j < BM / 64; ++j)
-              if (box++ % NP == prod) tma_load_2d(a_dst + j * MN_CHUNK, ta, c.tm * BM + 64 * j, k0, fb);
+              if (j < a_live && box++ % NP == prod) tma_load_2d(a_dst + j * MN_CHUNK, ta, c.tm * BM + 64 * j, k0, fb);
           } else if (CONV && p.conv_a) {
             const ConvColPart kc = a_it.part();
             if (p.conv.a_box == BM) {
@@ -160,7 +171,7 @@ __global__ void __launch_bounds__(threads_of<CONV>(), 1) tc_gemm_kernel(const __
             if (CONV && p.conv_b) krow = b_it.part();
 #pragma unroll
             for (int j = 0; j < BN / 64; ++j) {
-              if (box++ % NP != prod) continue;
+              if (j >= b_live || box++ % NP != prod) continue;
               const int col = c.tn * BN + 64 * j;
               if (!CONV || !p.conv_b) {
                 tma_load_2d(b_dst + j * MN_CHUNK, tb, col, k0, fb);
