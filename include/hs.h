@@ -130,14 +130,24 @@ hs_status hs_param_count(const hs_model_desc* model, int64_t* P);
  *                        pair); =all: averaged in tensor memory on every layer
  *   HS_OVERLAP_UPDATE=0  slab-path updates on the step's stream, not beside the
  *                        remaining products
- *   HS_RELU_BITS=0       bf16 MLP: the input-gradient products read ReLU' from
- *                        the stored activations instead of packed bits
+ *   HS_RELU_BITS=0       bf16: the input-gradient products (MLP; the CNN's
+ *                        sub-pixel ones) read ReLU' from the stored activations
+ *                        instead of packed bits
  *   HS_CONV_IMPLICIT=0|fwd  bf16 CNN: materialised patch rows everywhere, or
  *                        for the input gradients only
  *   HS_TC_FORM=single    one-SM tensor-core tiles instead of SM pairs (read
  *                        when the library loads)
  *   HS_NARROW_EW=4       256 x 128 SM-pair tiles with four epilogue warps instead
  *                        of two groups of four on alternate tiles
+ *   HS_CONV_FIRST=0      bf16 CNN: the first convolution as patch rows plus the
+ *                        tiled product instead of its one kernel
+ *   HS_SUBPIXEL=classes  bf16 CNN: the stride-2 input gradients as one grouped
+ *                        product per sub-pixel class instead of one product
+ *                        over the four classes
+ *   HS_CONV_ABOX=64      bf16 CNN: 64-pixel A boxes instead of 128-pixel ones
+ *   HS_KSTAGE=1|2        one k-block per pipeline stage everywhere, or two
+ *                        everywhere (read per launch; default: two for the
+ *                        forward products, 256 x 128 tiles and convolutions)
  *   HS_CNN_FUSED_UPDATE=0  bf16 CNN: per-worker split-K reductions into the slabs,
  *                        the slab update and the weight permutations as separate
  *                        launches instead of one update kernel (debug read-back
