@@ -144,6 +144,9 @@ hs_status hs_param_count(const hs_model_desc* model, int64_t* P);
  *   HS_SUBPIXEL=classes  bf16 CNN: the stride-2 input gradients as one grouped
  *                        product per sub-pixel class instead of one product
  *                        over the four classes
+ *   HS_SUBPIXEL_EW=4|8   bf16 CNN: four or eight epilogue warps on every
+ *                        one-product sub-pixel input gradient (default: eight
+ *                        where the input has <= 64 channels, else four)
  *   HS_CONV_ABOX=64      bf16 CNN: 64-pixel A boxes instead of 128-pixel ones
  *   HS_KSTAGE=1|2        one k-block per pipeline stage everywhere, or two
  *                        everywhere (read per launch; default: two for the

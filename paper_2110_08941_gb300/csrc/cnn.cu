@@ -783,6 +783,10 @@ hs_status plan_subpixel_dgrad_comb(hs_ctx* c, int k) {
   p.conv_a = 2;
   p.conv_d = 2;
   p.form = kTcFormPair;   // 256 x 256 SM-pair tiles
+  // eight epilogue warps (two groups of four on alternate tiles) where the epilogue bounds it:
+  // 64 channels per class block, four class blocks per tile (HS_SUBPIXEL_EW=4 or 8 forces either)
+  const char* ew = getenv("HS_SUBPIXEL_EW");
+  p.ew = (ew && !strcmp(ew, "8")) ? 8 : (ew && !strcmp(ew, "4")) ? 4 : (L.cin <= 64 ? 8 : 4);
   p.conv = tc_conv_geom(L.cout, L.hout, L.wout, L.stride);
   p.conv.a_box = abox;
   p.conv.a_cls = 3;

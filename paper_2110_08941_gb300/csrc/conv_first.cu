@@ -252,12 +252,15 @@ __global__ void __launch_bounds__(kCfThreads, 1) conv_first_fwd_kernel(const __g
             if (c0 + 8 < p.Cout) orow[(c0 >> 3) + 1] = make_uint4(o[4], o[5], o[6], o[7]);
           }
           if (p.bits) {
+            // bf16 h > 0 exactly when 1 <= h <= 0x7fff as an unsigned half-word (sign clear, not
+            // zero): the same decision as comparing the stored value, in integer operations
+            uint32_t b16 = 0;
 #pragma unroll
             for (int e = 0; e < 8; ++e) {
-              const __nv_bfloat162 pr = *reinterpret_cast<const __nv_bfloat162*>(&o[e]);
-              bits |= (uint64_t)(__low2float(pr) > 0.f) << ((c0 & 63) + 2 * e);
-              bits |= (uint64_t)(__high2float(pr) > 0.f) << ((c0 & 63) + 2 * e + 1);
+              b16 |= (uint32_t)((o[e] & 0xffffu) - 1u < 0x7fffu) << (2 * e);
+              b16 |= (uint32_t)((o[e] >> 16) - 1u < 0x7fffu) << (2 * e + 1);
             }
+            bits |= (uint64_t)b16 << (c0 & 63);
             if (((c0 + 16) & 63) == 0) {
               if (live)
                 p.bits[(int64_t)(c0 >> 6) * p.bits_ld + ((int64_t)n * p.Ho + ho0) * p.Wo + r] = bits;

@@ -479,6 +479,8 @@ cudaError_t launch_tc_gemm_pair(const TcGemmParams& p, int num_sms, cudaStream_t
   }
   // implicit convolution operands (forward, weight gradient, sub-pixel input gradient)
   if (p.conv_a || p.conv_b || p.conv_d) {
+    if (p.ew == 8 && p.epi == kTcEpiMaskBf16 && !p.a_mn && p.b_mn)   // the one-product sub-pixel input gradient
+      return launch_pair_variant<kTcEpiMaskBf16, false, true, true, 256, 8>(p, pairs, grid, s);
     if (p.epi == kTcEpiBiasReluBf16 && !p.a_mn && !p.b_mn) return launch_pair_variant<kTcEpiBiasReluBf16, false, false, true>(p, pairs, grid, s);
     if (p.epi == kTcEpiStoreF32 && p.a_mn && p.b_mn) return launch_pair_variant<kTcEpiStoreF32, true, true, true>(p, pairs, grid, s);
     if (p.epi == kTcEpiMaskBf16 && !p.a_mn && p.b_mn) return launch_pair_variant<kTcEpiMaskBf16, false, true, true>(p, pairs, grid, s);
