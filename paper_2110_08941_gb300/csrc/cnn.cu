@@ -227,31 +227,81 @@ __global__ void gap_forward_kernel(const T* __restrict__ h, int N, int HW, int C
   pooled[idx] = from_f<T>(acc / (float)HW);
 }
 
-// dA[n][p][c] = dpooled[n][c] / HW * 1[h[n][p][c] > 0] (pooling backward with ReLU').
-// The same for bf16 activations, eight channels per thread (16-byte loads and stores; C % 8 == 0).
-__global__ void gap_backward_vec8_kernel(const float* __restrict__ dpooled, const __nv_bfloat16* __restrict__ h,
-                                         int N, int HW, int C, __nv_bfloat16* __restrict__ dA) {
+constexpr int kGapThreads = 256;   // block of the bf16 pooling kernels: C / 8 channel groups x G pixel groups
+
+// The same for bf16 activations (C % 8 == 0, C / 8 <= the block): one block per sample; thread
+// (pixel group g, eight channels c8) sums pixels g, g + G, ... of its channels in fp32 from 16-byte
+// loads, and each channel's G partial sums are then added in group order.  The activations come
+// straight from the last convolution's epilogue (L2-resident); the loads of one thread are
+// independent, so a sample's 64 pixels take one round of loads instead of 64.
+__global__ void gap_forward_vec8_kernel(const __nv_bfloat16* __restrict__ h, int HW, int C,
+                                        __nv_bfloat16* __restrict__ pooled) {
+  extern __shared__ float gap_part[];   // [G][C]
   pdl_wait();
   pdl_trigger();
   const int C8 = C >> 3;
-  const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (idx >= (int64_t)N * HW * C8) return;
-  const int c8 = (int)(idx % C8);
-  const int64_t n = idx / ((int64_t)HW * C8);
-  const float4 g0 = __ldg(reinterpret_cast<const float4*>(dpooled + n * C + c8 * 8));
-  const float4 g1 = __ldg(reinterpret_cast<const float4*>(dpooled + n * C + c8 * 8 + 4));
-  const float g[8] = {g0.x, g0.y, g0.z, g0.w, g1.x, g1.y, g1.z, g1.w};
-  const uint4 hv = __ldg(reinterpret_cast<const uint4*>(h) + idx);
-  const uint32_t hw4[4] = {hv.x, hv.y, hv.z, hv.w};
-  uint32_t o[4];
+  const int G = (int)blockDim.x / C8;
+  const int n = blockIdx.x;
+  const int c8 = (int)threadIdx.x % C8, g = (int)threadIdx.x / C8;
+  if (g < G) {
+    float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+    const uint4* src = reinterpret_cast<const uint4*>(h + (int64_t)n * HW * C) + c8;
+#pragma unroll 8
+    for (int p = g; p < HW; p += G) {
+      const uint4 v = __ldg(src + (int64_t)p * C8);
+      const uint32_t w[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
-  for (int j = 0; j < 4; ++j) {
-    const __nv_bfloat162 pr = *reinterpret_cast<const __nv_bfloat162*>(&hw4[j]);
-    __nv_bfloat162 q = __floats2bfloat162_rn(__low2float(pr) > 0.f ? g[2 * j] / (float)HW : 0.f,
-                                             __high2float(pr) > 0.f ? g[2 * j + 1] / (float)HW : 0.f);
-    o[j] = *reinterpret_cast<uint32_t*>(&q);
+      for (int j = 0; j < 4; ++j) {
+        const __nv_bfloat162 pr = *reinterpret_cast<const __nv_bfloat162*>(&w[j]);
+        acc[2 * j] += __low2float(pr);
+        acc[2 * j + 1] += __high2float(pr);
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < 8; ++j) gap_part[g * C + c8 * 8 + j] = acc[j];
   }
-  reinterpret_cast<uint4*>(dA)[idx] = make_uint4(o[0], o[1], o[2], o[3]);
+  __syncthreads();
+  for (int c = threadIdx.x; c < C; c += blockDim.x) {
+    float sum = 0.f;
+    for (int gg = 0; gg < G; ++gg) sum += gap_part[gg * C + c];
+    pooled[(int64_t)n * C + c] = __float2bfloat16_rn(sum / (float)HW);
+  }
+}
+
+// dA[n][p][c] = dpooled[n][c] / HW * 1[h[n][p][c] > 0] (pooling backward with ReLU').
+// The same for bf16 activations, eight channels per thread (16-byte loads and stores; C % 8 == 0,
+// C / 8 <= the block): one block per sample, thread (pixel group g, channels c8) writing pixels
+// g, g + G, ... from one load of its eight dpooled / HW.
+__global__ void gap_backward_vec8_kernel(const float* __restrict__ dpooled, const __nv_bfloat16* __restrict__ h,
+                                         int HW, int C, __nv_bfloat16* __restrict__ dA) {
+  pdl_wait();
+  pdl_trigger();
+  const int C8 = C >> 3;
+  const int G = (int)blockDim.x / C8;
+  const int n = blockIdx.x;
+  const int c8 = (int)threadIdx.x % C8, g = (int)threadIdx.x / C8;
+  if (g >= G) return;
+  const float4 g0 = __ldg(reinterpret_cast<const float4*>(dpooled + (int64_t)n * C + c8 * 8));
+  const float4 g1 = __ldg(reinterpret_cast<const float4*>(dpooled + (int64_t)n * C + c8 * 8 + 4));
+  const float inv[8] = {g0.x / (float)HW, g0.y / (float)HW, g0.z / (float)HW, g0.w / (float)HW,
+                        g1.x / (float)HW, g1.y / (float)HW, g1.z / (float)HW, g1.w / (float)HW};
+  const int64_t base = (int64_t)n * HW * C8 + c8;
+  const uint4* hs = reinterpret_cast<const uint4*>(h) + base;
+  uint4* ds = reinterpret_cast<uint4*>(dA) + base;
+#pragma unroll 8
+  for (int p = g; p < HW; p += G) {
+    const uint4 hv = __ldg(hs + (int64_t)p * C8);
+    const uint32_t hw4[4] = {hv.x, hv.y, hv.z, hv.w};
+    uint32_t o[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const __nv_bfloat162 pr = *reinterpret_cast<const __nv_bfloat162*>(&hw4[j]);
+      __nv_bfloat162 q = __floats2bfloat162_rn(__low2float(pr) > 0.f ? inv[2 * j] : 0.f,
+                                               __high2float(pr) > 0.f ? inv[2 * j + 1] : 0.f);
+      o[j] = *reinterpret_cast<uint32_t*>(&q);
+    }
+    ds[(int64_t)p * C8] = make_uint4(o[0], o[1], o[2], o[3]);
+  }
 }
 
 template <typename T>
@@ -938,7 +988,10 @@ hs_status cnn_step(hs_ctx* c, float* params, const float* x, const int32_t* y, c
       }
       ph.launched();
     }
-    if (bf16)
+    if (bf16 && c3 % 8 == 0 && c3 / 8 <= kGapThreads)
+      launch_pdl(gap_forward_vec8_kernel, N, kGapThreads, (size_t)(kGapThreads / (c3 / 8)) * c3 * sizeof(float), s,
+          reinterpret_cast<const __nv_bfloat16*>(c->d_cact[2]), hw3, c3, reinterpret_cast<__nv_bfloat16*>(c->d_pooled));
+    else if (bf16)
       launch_pdl(gap_forward_kernel<__nv_bfloat16>, blocks_for((int64_t)N * c3, T), T, 0, s,
           reinterpret_cast<const __nv_bfloat16*>(c->d_cact[2]), N, hw3, c3, reinterpret_cast<__nv_bfloat16*>(c->d_pooled));
     else
@@ -1037,8 +1090,12 @@ hs_status cnn_step(hs_ctx* c, float* params, const float* x, const int32_t* y, c
         d.Mdim = N; d.Ndim = c3; d.Kdim = c->C; d.epi = kEpiStore;
         launch_gemm_f32(d, s);
       }
-      if (bf16)
-        launch_pdl(gap_backward_vec8_kernel, blocks_for((int64_t)N * hw3 * (c3 / 8), T), T, 0, s,
+      if (bf16 && c3 % 8 == 0 && c3 / 8 <= kGapThreads)
+        launch_pdl(gap_backward_vec8_kernel, N, kGapThreads, 0, s,
+            c->d_dpooled, reinterpret_cast<const __nv_bfloat16*>(c->d_cact[2]), hw3, c3,
+            reinterpret_cast<__nv_bfloat16*>(c->d_dA[2]));
+      else if (bf16)
+        launch_pdl(gap_backward_kernel<__nv_bfloat16>, blocks_for((int64_t)N * hw3 * c3, T), T, 0, s,
             c->d_dpooled, reinterpret_cast<const __nv_bfloat16*>(c->d_cact[2]), N, hw3, c3,
             reinterpret_cast<__nv_bfloat16*>(c->d_dA[2]));
       else

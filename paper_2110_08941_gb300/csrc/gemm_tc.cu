@@ -202,7 +202,7 @@ __global__ void __launch_bounds__(threads_of<CONV>(), 1) tc_gemm_kernel(const __
   } else if (warp == 1) {
     if (lane == 0) {
       // ------------------------------------------------------------ MMA issuer
-      constexpr uint32_t idesc = make_idesc(A_MN, B_MN, BM, BN);
+      constexpr uint32_t idesc_full = make_idesc(A_MN, B_MN, BM, BN);
       const uint64_t a_desc0 = make_sdesc(smem_u32(sA), A_MN ? MN_CHUNK : 16, 1024);
       const uint64_t b_desc0 = make_sdesc(smem_u32(sB), B_MN ? MN_CHUNK : 16, 1024);
       int s = 0;
@@ -218,6 +218,14 @@ __global__ void __launch_bounds__(threads_of<CONV>(), 1) tc_gemm_kernel(const __
         }
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + (uint32_t)(ab * BN);
+        // an MN-major B tile with 64-wide boxes past the product's columns runs narrower MMAs
+        // (N = 64 x the live boxes): the stored columns get the same sums, the rest are never stored
+        uint32_t idesc = idesc_full;
+        if (B_MN) {
+          const int ncols = (CONV && p.conv_b) ? p.conv.ones_col + 1 : p.Ndim;
+          const int b_live = max(1, min(BN / 64, (ncols - w.c.tn * BN + 63) / 64));
+          idesc = make_idesc(A_MN, B_MN, BM, 64 * b_live);
+        }
         bool ok = true;
         const LastKb lk = last_kb_of(p, w.g);
         for (int kb = w.kb_lo; kb < w.kb_hi; ++kb) {
