@@ -1018,7 +1018,12 @@ hs_status cnn_step(hs_ctx* c, float* params, const float* x, const int32_t* y, c
     PhaseScope ph(c, HS_PHASE_LOSS, s);
     launch_softmax_xent(c->d_logits, c->Cp, y, c->d_scale, N, c->C, c->d_delta[0], c->Cp, bf16, c->d_ce, c->d_status,
                         s);
-    launch_loss_reduce(c->d_ce, c->d_offsets, c->M, c->d_w, c->d_lm, c->d_status, c->d_ticket, s);
+    if (bf16 && c->C <= loss_bias_max_width())   // the fc bias gradients in the same launch
+      launch_loss_bias_reduce(c->d_ce, c->d_offsets, c->M, c->d_w, c->d_lm, c->d_status, c->d_ticket,
+                              reinterpret_cast<const __nv_bfloat16*>(c->d_delta[0]), c->Cp, c->C, c->d_slabs, c->Ps,
+                              c->fc_b_off, s);
+    else
+      launch_loss_reduce(c->d_ce, c->d_offsets, c->M, c->d_w, c->d_lm, c->d_status, c->d_ticket, s);
     ph.launched(2);
   }
   // ---- backward: layer index 3 = fc, 2..0 = conv3..conv1
@@ -1065,6 +1070,8 @@ hs_status cnn_step(hs_ctx* c, float* params, const float* x, const int32_t* y, c
       PhaseScope ph(c, HS_PHASE_BIASGRAD, s);
       if (bf16 && !fc) {
         // the convolutions' bias gradients came out of the weight-gradient product (ones column)
+      } else if (bf16 && c->C <= loss_bias_max_width()) {
+        // the fc bias gradients came out of the loss reduction
       } else if (bf16) {
         const ChunkTable& ct = c->cnn_chunks[k];
         launch_bias_grad_bf16(reinterpret_cast<const __nv_bfloat16*>(delta), ld_delta, width, ct.d_chunks, ct.n,

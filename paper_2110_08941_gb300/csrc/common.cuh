@@ -64,6 +64,12 @@ void launch_softmax_xent(const float* logits, int ldl, const int32_t* y, const f
                          cudaStream_t s);
 void launch_loss_reduce(const float* ce, const int32_t* d_offsets, int M, const float* d_w,
                         float* lm, DevStatus* st, unsigned int* ticket, cudaStream_t s);
+// The same, and in the same launch the last layer's per-worker bias gradients from its bf16 delta
+// (width <= loss_bias_max_width()): slabs[m*Ps + b_off + j] = sum_{i in seg_m} delta[i*ld + j].
+int loss_bias_max_width();
+void launch_loss_bias_reduce(const float* ce, const int32_t* d_offsets, int M, const float* d_w, float* lm,
+                             DevStatus* st, unsigned int* ticket, const __nv_bfloat16* delta, int ld, int width,
+                             float* slabs, int64_t Ps, int64_t b_off, cudaStream_t s);
 // slabs[m*Ps + b_off + j] = sum_{i in seg_m} delta[i*ld + j], j < width
 void launch_bias_grad(const void* delta, bool delta_bf16, int ld, int width, const int32_t* d_offsets,
                       int M, float* slabs, int64_t Ps, int64_t b_off, cudaStream_t s);

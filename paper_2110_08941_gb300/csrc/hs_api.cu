@@ -451,6 +451,7 @@ hs_status mlp_step_fp32(hs_ctx* c, float* params, const float* x, const int32_t*
       ph.launched();
     }
   }
+  const bool loss_bias = !c->fused_sync && c->C <= hs::loss_bias_max_width();
   {
     PhaseScope ph(c, HS_PHASE_LOSS, s);
     hs::launch_softmax_xent(c->d_logits, c->Cp, y, c->fused_sync ? c->d_scale_fused : c->d_scale, c->N, c->C,
@@ -549,12 +550,18 @@ hs_status mlp_step_bf16(hs_ctx* c, float* params, const float* x, const int32_t*
       ph.launched();
     }
   }
+  const bool loss_bias = !c->fused_sync && c->C <= hs::loss_bias_max_width();
   {
     PhaseScope ph(c, HS_PHASE_LOSS, s);
     hs::launch_softmax_xent(c->d_logits, c->Cp, y, c->fused_sync ? c->d_scale_fused : c->d_scale, c->N, c->C,
                             c->delta_buf(L - 1), c->Cp, true,
                             c->d_ce, c->d_status, s);
-    hs::launch_loss_reduce(c->d_ce, c->d_offsets, c->M, c->d_w, c->d_lm, c->d_status, c->d_ticket, s);
+    if (loss_bias)   // the output layer's bias gradients in the same launch
+      hs::launch_loss_bias_reduce(c->d_ce, c->d_offsets, c->M, c->d_w, c->d_lm, c->d_status, c->d_ticket,
+                                  reinterpret_cast<const __nv_bfloat16*>(c->delta_buf(L - 1)), c->delta_ld(L - 1),
+                                  c->C, c->d_slabs, c->Ps, c->layers[L - 1].b_off, s);
+    else
+      hs::launch_loss_reduce(c->d_ce, c->d_offsets, c->M, c->d_w, c->d_lm, c->d_status, c->d_ticket, s);
     ph.launched(2);
   }
   // Per-worker weight gradients averaged tile by tile in tensor memory, the update fused in: the
@@ -593,7 +600,7 @@ hs_status mlp_step_bf16(hs_ctx* c, float* params, const float* x, const int32_t*
         }
       }
     }
-    {
+    if (!(loss_bias && l == L - 1)) {
       PhaseScope ph(c, HS_PHASE_BIASGRAD, s);
       const int out_cols = (l == L - 1) ? c->C : ly.out;
       const hs::ChunkTable* ct = nullptr;

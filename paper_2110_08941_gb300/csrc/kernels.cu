@@ -223,21 +223,43 @@ void launch_softmax_xent(const float* logits, int ldl, const int32_t* y, const f
 }
 
 // ------------------------------------------------------------------ per-worker loss reduction
-// L_m = (1/n_m) sum_{i in seg_m} ce_i (Eq. 1); loss = sum_m w_m L_m.  One block, fixed order.
+// L_m = (1/n_m) sum_{i in seg_m} ce_i (Eq. 1); loss = sum_m w_m L_m.
 // One block per worker: L_m = mean of its per-sample losses (strided partial sums, then a tree, in
 // a fixed order); the last block to finish forms sum_m w_m L_m in worker order and resets the
-// ticket for the next step.
-__global__ void loss_reduce_kernel(const float* __restrict__ ce, const int32_t* __restrict__ offsets,
-                                   int M, const float* __restrict__ w, float* __restrict__ lm,
-                                   DevStatus* st, unsigned int* ticket) {
+// ticket for the next step.  With `delta`, the block also forms its worker's bias gradient of the
+// output layer (width <= 32 columns, one lane per column): warp v sums rows b + v, b + v + 32, ...
+// in row order, and the 32 warps' sums are added in warp order (deterministic); the two launches
+// of the chunked bias-gradient reduction are then not needed for that layer.
+constexpr int kLossThreads = 1024;
+
+__global__ void __launch_bounds__(kLossThreads) loss_reduce_kernel(
+    const float* __restrict__ ce, const int32_t* __restrict__ offsets, int M, const float* __restrict__ w,
+    float* __restrict__ lm, DevStatus* st, unsigned int* ticket, const __nv_bfloat16* __restrict__ delta, int ld,
+    int width, float* __restrict__ slabs, int64_t Ps, int64_t b_off) {
   pdl_wait();
   pdl_trigger();
-  __shared__ float red[1024];
+  __shared__ float red[kLossThreads];
   __shared__ bool last;
   const int m = blockIdx.x;
   const int b = offsets[m], e = offsets[m + 1];
   float acc = 0.f;
   for (int i = b + threadIdx.x; i < e; i += blockDim.x) acc += ce[i];
+  float bacc = 0.f;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (delta && lane < width) {
+    int i = b + warp;
+    for (; i + 96 < e; i += 128) {   // four rows in flight, added in row order
+      const float v0 = __bfloat162float(delta[(int64_t)i * ld + lane]);
+      const float v1 = __bfloat162float(delta[(int64_t)(i + 32) * ld + lane]);
+      const float v2 = __bfloat162float(delta[(int64_t)(i + 64) * ld + lane]);
+      const float v3 = __bfloat162float(delta[(int64_t)(i + 96) * ld + lane]);
+      bacc += v0;
+      bacc += v1;
+      bacc += v2;
+      bacc += v3;
+    }
+    for (; i < e; i += 32) bacc += __bfloat162float(delta[(int64_t)i * ld + lane]);
+  }
   red[threadIdx.x] = acc;
   __syncthreads();
   for (int h = blockDim.x >> 1; h > 0; h >>= 1) {
@@ -250,6 +272,15 @@ __global__ void loss_reduce_kernel(const float* __restrict__ ce, const int32_t* 
     last = (atomicAdd(ticket, 1u) == (unsigned int)(M - 1));
   }
   __syncthreads();
+  if (delta) {
+    red[threadIdx.x] = bacc;   // [warp][lane]
+    __syncthreads();
+    if (threadIdx.x < width) {
+      float t = 0.f;
+      for (int v = 0; v < kLossThreads / 32; ++v) t += red[v * 32 + threadIdx.x];
+      slabs[(int64_t)m * Ps + b_off + threadIdx.x] = t;
+    }
+  }
   if (last && threadIdx.x == 0) {
     __threadfence();
     const volatile float* lmv = lm;
@@ -262,7 +293,17 @@ __global__ void loss_reduce_kernel(const float* __restrict__ ce, const int32_t* 
 
 void launch_loss_reduce(const float* ce, const int32_t* d_offsets, int M, const float* d_w,
                         float* lm, DevStatus* st, unsigned int* ticket, cudaStream_t s) {
-  launch_pdl(loss_reduce_kernel, M, 1024, 0, s, ce, d_offsets, M, d_w, lm, st, ticket);
+  launch_pdl(loss_reduce_kernel, M, kLossThreads, 0, s, ce, d_offsets, M, d_w, lm, st, ticket,
+             (const __nv_bfloat16*)nullptr, 0, 0, (float*)nullptr, (int64_t)0, (int64_t)0);
+}
+
+int loss_bias_max_width() { return 32; }
+
+void launch_loss_bias_reduce(const float* ce, const int32_t* d_offsets, int M, const float* d_w, float* lm,
+                             DevStatus* st, unsigned int* ticket, const __nv_bfloat16* delta, int ld, int width,
+                             float* slabs, int64_t Ps, int64_t b_off, cudaStream_t s) {
+  launch_pdl(loss_reduce_kernel, M, kLossThreads, 0, s, ce, d_offsets, M, d_w, lm, st, ticket, delta, ld, width,
+             slabs, Ps, b_off);
 }
 
 // ------------------------------------------------------------------ per-worker bias gradient
