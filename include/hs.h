@@ -155,6 +155,9 @@ hs_status hs_param_count(const hs_model_desc* model, int64_t* P);
  *                        the slab update and the weight permutations as separate
  *                        launches instead of one update kernel (debug read-back
  *                        always takes the separate launches)
+ *   HS_CNN_FC_POOL=0     bf16 CNN: the fc layer's logits and input gradient as
+ *                        two tensor-core products instead of inside the pooling
+ *                        kernels (at most 32 classes)
  *   HS_STEP_GRAPH=0      every hs_step enqueues its kernels one by one (no
  *                        replay of a captured step, see hs_step); =1 replays
  *                        captured steps also above 1e11 parameter-samples */

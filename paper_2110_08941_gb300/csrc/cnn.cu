@@ -234,9 +234,15 @@ constexpr int kGapThreads = 256;   // block of the bf16 pooling kernels: C / 8 c
 // loads, and each channel's G partial sums are then added in group order.  The activations come
 // straight from the last convolution's epilogue (L2-resident); the loads of one thread are
 // independent, so a sample's 64 pixels take one round of loads instead of 64.
+// kFc: the fc layer in the same block (ncls <= 32 classes): logits[n][j] = sum_c p[c] W[j][c] + b[j]
+// with p the stored (bf16) pooled row, W the fc weights' bf16 copy [ncls][C]; one warp per class,
+// lanes on channels, an xor-shuffle tree, fp32.
+template <bool kFc>
 __global__ void gap_forward_vec8_kernel(const __nv_bfloat16* __restrict__ h, int HW, int C,
-                                        __nv_bfloat16* __restrict__ pooled) {
-  extern __shared__ float gap_part[];   // [G][C]
+                                        __nv_bfloat16* __restrict__ pooled, const __nv_bfloat16* __restrict__ W,
+                                        const float* __restrict__ bias, int ncls, float* __restrict__ logits,
+                                        int ldl) {
+  extern __shared__ float gap_part[];   // [G][C], then (kFc) the pooled row [C]
   pdl_wait();
   pdl_trigger();
   const int C8 = C >> 3;
@@ -261,10 +267,25 @@ __global__ void gap_forward_vec8_kernel(const __nv_bfloat16* __restrict__ h, int
     for (int j = 0; j < 8; ++j) gap_part[g * C + c8 * 8 + j] = acc[j];
   }
   __syncthreads();
+  float* row = gap_part + G * C;
   for (int c = threadIdx.x; c < C; c += blockDim.x) {
     float sum = 0.f;
     for (int gg = 0; gg < G; ++gg) sum += gap_part[gg * C + c];
-    pooled[(int64_t)n * C + c] = __float2bfloat16_rn(sum / (float)HW);
+    const __nv_bfloat16 pb = __float2bfloat16_rn(sum / (float)HW);
+    pooled[(int64_t)n * C + c] = pb;
+    if (kFc) row[c] = __bfloat162float(pb);
+  }
+  if (kFc) {
+    __syncthreads();
+    const int warp = (int)threadIdx.x >> 5, lane = (int)threadIdx.x & 31;
+    for (int j = warp; j < ncls; j += (int)blockDim.x >> 5) {
+      const __nv_bfloat16* wj = W + (int64_t)j * C;
+      float acc = 0.f;
+      for (int c = lane; c < C; c += 32) acc = fmaf(row[c], __bfloat162float(wj[c]), acc);
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+      if (lane == 0) logits[(int64_t)n * ldl + j] = acc + bias[j];
+    }
   }
 }
 
@@ -272,17 +293,34 @@ __global__ void gap_forward_vec8_kernel(const __nv_bfloat16* __restrict__ h, int
 // The same for bf16 activations, eight channels per thread (16-byte loads and stores; C % 8 == 0,
 // C / 8 <= the block): one block per sample, thread (pixel group g, channels c8) writing pixels
 // g, g + G, ... from one load of its eight dpooled / HW.
+// kFc: dpooled formed in the block from the fc layer's delta (bf16 [N][ldd], ncls classes) and
+// weights (bf16 [ncls][C]): dpooled[c] = sum_j delta[n][j] W[j][c] in class order, fp32.
+template <bool kFc>
 __global__ void gap_backward_vec8_kernel(const float* __restrict__ dpooled, const __nv_bfloat16* __restrict__ h,
-                                         int HW, int C, __nv_bfloat16* __restrict__ dA) {
+                                         int HW, int C, __nv_bfloat16* __restrict__ dA,
+                                         const __nv_bfloat16* __restrict__ delta, int ldd,
+                                         const __nv_bfloat16* __restrict__ W, int ncls) {
+  extern __shared__ float gap_dp[];   // kFc: dpooled of the block's sample [C]
   pdl_wait();
   pdl_trigger();
   const int C8 = C >> 3;
   const int G = (int)blockDim.x / C8;
   const int n = blockIdx.x;
   const int c8 = (int)threadIdx.x % C8, g = (int)threadIdx.x / C8;
+  const float* dp = dpooled + (int64_t)n * C;
+  if (kFc) {
+    const __nv_bfloat16* dn = delta + (int64_t)n * ldd;
+    for (int c = threadIdx.x; c < C; c += blockDim.x) {
+      float acc = 0.f;
+      for (int j = 0; j < ncls; ++j) acc = fmaf(__bfloat162float(dn[j]), __bfloat162float(W[(int64_t)j * C + c]), acc);
+      gap_dp[c] = acc;
+    }
+    __syncthreads();
+    dp = gap_dp;
+  }
   if (g >= G) return;
-  const float4 g0 = __ldg(reinterpret_cast<const float4*>(dpooled + (int64_t)n * C + c8 * 8));
-  const float4 g1 = __ldg(reinterpret_cast<const float4*>(dpooled + (int64_t)n * C + c8 * 8 + 4));
+  const float4 g0 = *reinterpret_cast<const float4*>(dp + c8 * 8);
+  const float4 g1 = *reinterpret_cast<const float4*>(dp + c8 * 8 + 4);
   const float inv[8] = {g0.x / (float)HW, g0.y / (float)HW, g0.z / (float)HW, g0.w / (float)HW,
                         g1.x / (float)HW, g1.y / (float)HW, g1.z / (float)HW, g1.w / (float)HW};
   const int64_t base = (int64_t)n * HW * C8 + c8;
@@ -562,6 +600,14 @@ __global__ void __launch_bounds__(256) cnn_update_kernel(const CnnUpdArgs a, flo
 }
 
 inline int blocks_for(int64_t n, int threads) { return (int)((n + threads - 1) / threads); }
+
+// bf16 step whose fc layer (at most 32 classes) runs inside the pooling kernels: the logits in the
+// pooling forward's block of each sample, the fc input gradient in the pooling backward's
+// (HS_CNN_FC_POOL=0 keeps the two tensor-core products).
+inline bool cnn_fc_in_pooling(const hs_ctx* c) {
+  const int c3 = c->convs[2].cout;
+  return c->precision == HS_BF16 && c->cnn_fc_pool && c3 % 8 == 0 && c3 / 8 <= kGapThreads && c->C <= 32;
+}
 
 // bf16 patch rows of the first convolution: one thread per row where the row is short, else the
 // per-channel kernel.
@@ -988,21 +1034,34 @@ hs_status cnn_step(hs_ctx* c, float* params, const float* x, const int32_t* y, c
       }
       ph.launched();
     }
-    if (bf16 && c3 % 8 == 0 && c3 / 8 <= kGapThreads)
-      launch_pdl(gap_forward_vec8_kernel, N, kGapThreads, (size_t)(kGapThreads / (c3 / 8)) * c3 * sizeof(float), s,
-          reinterpret_cast<const __nv_bfloat16*>(c->d_cact[2]), hw3, c3, reinterpret_cast<__nv_bfloat16*>(c->d_pooled));
-    else if (bf16)
+    const bool fc_pool = cnn_fc_in_pooling(c);
+    const __nv_bfloat16* w_fc = c->d_shadow + c->fc_w_off;
+    if (bf16 && c3 % 8 == 0 && c3 / 8 <= kGapThreads) {
+      const size_t smem = ((size_t)(kGapThreads / (c3 / 8)) * c3 + (fc_pool ? c3 : 0)) * sizeof(float);
+      if (fc_pool)   // the fc layer's logits in the same block
+        launch_pdl(gap_forward_vec8_kernel<true>, N, kGapThreads, smem, s,
+            reinterpret_cast<const __nv_bfloat16*>(c->d_cact[2]), hw3, c3, reinterpret_cast<__nv_bfloat16*>(c->d_pooled),
+            w_fc, params + c->fc_b_off, c->C, c->d_logits, c->Cp);
+      else
+        launch_pdl(gap_forward_vec8_kernel<false>, N, kGapThreads, smem, s,
+            reinterpret_cast<const __nv_bfloat16*>(c->d_cact[2]), hw3, c3, reinterpret_cast<__nv_bfloat16*>(c->d_pooled),
+            (const __nv_bfloat16*)nullptr, (const float*)nullptr, 0, (float*)nullptr, 0);
+    } else if (bf16) {
       launch_pdl(gap_forward_kernel<__nv_bfloat16>, blocks_for((int64_t)N * c3, T), T, 0, s,
           reinterpret_cast<const __nv_bfloat16*>(c->d_cact[2]), N, hw3, c3, reinterpret_cast<__nv_bfloat16*>(c->d_pooled));
-    else
+    } else {
       launch_pdl(gap_forward_kernel<float>, blocks_for((int64_t)N * c3, T), T, 0, s,
           reinterpret_cast<const float*>(c->d_cact[2]), N, hw3, c3, reinterpret_cast<float*>(c->d_pooled));
+    }
     ph.launched();
-    if (bf16) {
+    if (fc_pool) {
+      // the logits came out of the pooling kernel
+    } else if (bf16) {
       TcGemmParams& f = c->tc_fwd[3];
       f.bias = params + c->fc_b_off;
       cudaError_t e = launch_tc_gemm(f, c->num_sms, s);
       if (e != cudaSuccess) return cuda_fail(c, e, "fc forward GEMM launch");
+      ph.launched();
     } else {
       GemmF32Args g{};
       g.A = reinterpret_cast<const float*>(c->d_pooled); g.a_sm = c3; g.a_sk = 1;
@@ -1011,8 +1070,8 @@ hs_status cnn_step(hs_ctx* c, float* params, const float* x, const int32_t* y, c
       g.Mdim = N; g.Ndim = c->C; g.Kdim = c3;
       g.epi = kEpiBias; g.bias = params + c->fc_b_off;
       launch_gemm_f32(g, s);
+      ph.launched();
     }
-    ph.launched();
   }
   {
     PhaseScope ph(c, HS_PHASE_LOSS, s);
@@ -1086,9 +1145,13 @@ hs_status cnn_step(hs_ctx* c, float* params, const float* x, const int32_t* y, c
     PhaseScope ph(c, HS_PHASE_DGRAD, s);
     if (fc) {
       // dpooled = delta W_fc, then pooling backward with ReLU' into conv3's output gradient
-      if (bf16) {
+      const bool fc_pool = cnn_fc_in_pooling(c);
+      if (fc_pool) {
+        // dpooled is formed inside the pooling backward
+      } else if (bf16) {
         cudaError_t e = launch_tc_gemm(c->tc_dgrad[3], c->num_sms, s);
         if (e != cudaSuccess) return cuda_fail(c, e, "fc input-gradient GEMM launch");
+        ph.launched();
       } else {
         GemmF32Args d{};
         d.A = reinterpret_cast<const float*>(c->d_delta[0]); d.a_sm = c->Cp; d.a_sk = 1;
@@ -1096,11 +1159,18 @@ hs_status cnn_step(hs_ctx* c, float* params, const float* x, const int32_t* y, c
         d.C = c->d_dpooled; d.ldc = c3;
         d.Mdim = N; d.Ndim = c3; d.Kdim = c->C; d.epi = kEpiStore;
         launch_gemm_f32(d, s);
+        ph.launched();
       }
-      if (bf16 && c3 % 8 == 0 && c3 / 8 <= kGapThreads)
-        launch_pdl(gap_backward_vec8_kernel, N, kGapThreads, 0, s,
+      if (fc_pool)
+        launch_pdl(gap_backward_vec8_kernel<true>, N, kGapThreads, c3 * sizeof(float), s,
+            (const float*)nullptr, reinterpret_cast<const __nv_bfloat16*>(c->d_cact[2]), hw3, c3,
+            reinterpret_cast<__nv_bfloat16*>(c->d_dA[2]), reinterpret_cast<const __nv_bfloat16*>(c->d_delta[0]), c->Cp,
+            c->d_shadow + c->fc_w_off, c->C);
+      else if (bf16 && c3 % 8 == 0 && c3 / 8 <= kGapThreads)
+        launch_pdl(gap_backward_vec8_kernel<false>, N, kGapThreads, 0, s,
             c->d_dpooled, reinterpret_cast<const __nv_bfloat16*>(c->d_cact[2]), hw3, c3,
-            reinterpret_cast<__nv_bfloat16*>(c->d_dA[2]));
+            reinterpret_cast<__nv_bfloat16*>(c->d_dA[2]), (const __nv_bfloat16*)nullptr, 0,
+            (const __nv_bfloat16*)nullptr, 0);
       else if (bf16)
         launch_pdl(gap_backward_kernel<__nv_bfloat16>, blocks_for((int64_t)N * hw3 * c3, T), T, 0, s,
             c->d_dpooled, reinterpret_cast<const __nv_bfloat16*>(c->d_cact[2]), N, hw3, c3,
@@ -1108,7 +1178,7 @@ hs_status cnn_step(hs_ctx* c, float* params, const float* x, const int32_t* y, c
       else
         launch_pdl(gap_backward_kernel<float>, blocks_for((int64_t)N * hw3 * c3, T), T, 0, s,
             c->d_dpooled, reinterpret_cast<const float*>(c->d_cact[2]), N, hw3, c3, reinterpret_cast<float*>(c->d_dA[2]));
-      ph.launched(2);
+      ph.launched();
     } else {
       if (L[k].subpixel) {
         // the four class products write dA_{k-1} directly (ReLU' of h_{k-1} fused)

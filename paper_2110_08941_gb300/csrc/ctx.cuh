@@ -217,6 +217,7 @@ struct hs_ctx {
   bool cnn_fuse_update = true;        // HS_CNN_FUSED_UPDATE=0: split-K reductions, slab update and permutations apart
   bool conv_first_on = false;         // bf16: the first convolution's forward in one kernel (conv_first_plan)
   bool subpixel_comb = true;          // sub-pixel input gradients as one product over all four classes
+  bool cnn_fc_pool = true;            // bf16 CNN: the fc layer's forward and input gradient inside the pooling kernels
                                       // (HS_SUBPIXEL=classes: one group per class); per layer where its
                                       // input has a multiple of 64 channels (ConvLayer::comb)
   hs::ConvFirstParams conv_first{};

@@ -897,6 +897,8 @@ hs_status hs_init(const hs_model_desc* model, int32_t M, const double* compute_w
   c->cnn_fuse_update = !(cf && !strcmp(cf, "0"));
   const char* sp = getenv("HS_SUBPIXEL");
   c->subpixel_comb = !(sp && !strcmp(sp, "classes"));
+  const char* fp = getenv("HS_CNN_FC_POOL");
+  c->cnn_fc_pool = !(fp && !strcmp(fp, "0"));
   const char* sg = getenv("HS_STEP_GRAPH");
   c->graph_on = !(sg && !strcmp(sg, "0"));
   c->graph_force = sg && !strcmp(sg, "1");
