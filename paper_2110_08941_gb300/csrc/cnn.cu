@@ -1075,15 +1075,23 @@ hs_status cnn_step(hs_ctx* c, float* params, const float* x, const int32_t* y, c
   }
   {
     PhaseScope ph(c, HS_PHASE_LOSS, s);
-    launch_softmax_xent(c->d_logits, c->Cp, y, c->d_scale, N, c->C, c->d_delta[0], c->Cp, bf16, c->d_ce, c->d_status,
-                        s);
-    if (bf16 && c->C <= loss_bias_max_width())   // the fc bias gradients in the same launch
-      launch_loss_bias_reduce(c->d_ce, c->d_offsets, c->M, c->d_w, c->d_lm, c->d_status, c->d_ticket,
-                              reinterpret_cast<const __nv_bfloat16*>(c->d_delta[0]), c->Cp, c->C, c->d_slabs, c->Ps,
-                              c->fc_b_off, s);
-    else
-      launch_loss_reduce(c->d_ce, c->d_offsets, c->M, c->d_w, c->d_lm, c->d_status, c->d_ticket, s);
-    ph.launched(2);
+    if (bf16 && softmax_loss_bias_ok(c->C, c->Cp, c->Cp)) {
+      // softmax, loss reduction and the fc bias gradients in one launch
+      launch_softmax_loss_bias(c->d_logits, c->Cp, y, c->d_scale, c->C, reinterpret_cast<__nv_bfloat16*>(c->d_delta[0]),
+                               c->Cp, c->d_ce, c->d_offsets, c->M, c->d_w, c->d_lm, c->d_status, c->d_ticket,
+                               c->d_slabs, c->Ps, c->fc_b_off, s);
+      ph.launched();
+    } else {
+      launch_softmax_xent(c->d_logits, c->Cp, y, c->d_scale, N, c->C, c->d_delta[0], c->Cp, bf16, c->d_ce,
+                          c->d_status, s);
+      if (bf16 && c->C <= loss_bias_max_width())   // the fc bias gradients in the same launch
+        launch_loss_bias_reduce(c->d_ce, c->d_offsets, c->M, c->d_w, c->d_lm, c->d_status, c->d_ticket,
+                                reinterpret_cast<const __nv_bfloat16*>(c->d_delta[0]), c->Cp, c->C, c->d_slabs, c->Ps,
+                                c->fc_b_off, s);
+      else
+        launch_loss_reduce(c->d_ce, c->d_offsets, c->M, c->d_w, c->d_lm, c->d_status, c->d_ticket, s);
+      ph.launched(2);
+    }
   }
   // ---- backward: layer index 3 = fc, 2..0 = conv3..conv1
   for (int k = 3; k >= 0; --k) {

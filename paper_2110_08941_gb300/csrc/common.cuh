@@ -67,6 +67,13 @@ void launch_loss_reduce(const float* ce, const int32_t* d_offsets, int M, const 
 // The same, and in the same launch the last layer's per-worker bias gradients from its bf16 delta
 // (width <= loss_bias_max_width()): slabs[m*Ps + b_off + j] = sum_{i in seg_m} delta[i*ld + j].
 int loss_bias_max_width();
+// softmax_xent + launch_loss_bias_reduce in one launch (bf16 delta; at most 16 classes, ldd % 8 == 0,
+// ldd <= 16, ldl % 4 == 0): softmax_loss_bias_ok says whether the shapes allow it.
+bool softmax_loss_bias_ok(int C, int ldl, int ldd);
+void launch_softmax_loss_bias(const float* logits, int ldl, const int32_t* y, const float* scale, int C,
+                              __nv_bfloat16* delta, int ldd, float* ce, const int32_t* d_offsets, int M,
+                              const float* d_w, float* lm, DevStatus* st, unsigned int* ticket, float* slabs,
+                              int64_t Ps, int64_t b_off, cudaStream_t s);
 void launch_loss_bias_reduce(const float* ce, const int32_t* d_offsets, int M, const float* d_w, float* lm,
                              DevStatus* st, unsigned int* ticket, const __nv_bfloat16* delta, int ld, int width,
                              float* slabs, int64_t Ps, int64_t b_off, cudaStream_t s);

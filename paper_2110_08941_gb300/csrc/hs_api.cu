@@ -553,16 +553,24 @@ hs_status mlp_step_bf16(hs_ctx* c, float* params, const float* x, const int32_t*
   const bool loss_bias = !c->fused_sync && c->C <= hs::loss_bias_max_width();
   {
     PhaseScope ph(c, HS_PHASE_LOSS, s);
-    hs::launch_softmax_xent(c->d_logits, c->Cp, y, c->fused_sync ? c->d_scale_fused : c->d_scale, c->N, c->C,
-                            c->delta_buf(L - 1), c->Cp, true,
-                            c->d_ce, c->d_status, s);
-    if (loss_bias)   // the output layer's bias gradients in the same launch
-      hs::launch_loss_bias_reduce(c->d_ce, c->d_offsets, c->M, c->d_w, c->d_lm, c->d_status, c->d_ticket,
-                                  reinterpret_cast<const __nv_bfloat16*>(c->delta_buf(L - 1)), c->delta_ld(L - 1),
-                                  c->C, c->d_slabs, c->Ps, c->layers[L - 1].b_off, s);
-    else
-      hs::launch_loss_reduce(c->d_ce, c->d_offsets, c->M, c->d_w, c->d_lm, c->d_status, c->d_ticket, s);
-    ph.launched(2);
+    __nv_bfloat16* delta_out = reinterpret_cast<__nv_bfloat16*>(c->delta_buf(L - 1));
+    if (loss_bias && hs::softmax_loss_bias_ok(c->C, c->Cp, c->delta_ld(L - 1))) {
+      // softmax, loss reduction and the output layer's bias gradients in one launch
+      hs::launch_softmax_loss_bias(c->d_logits, c->Cp, y, c->d_scale, c->C, delta_out, c->delta_ld(L - 1), c->d_ce,
+                                   c->d_offsets, c->M, c->d_w, c->d_lm, c->d_status, c->d_ticket, c->d_slabs, c->Ps,
+                                   c->layers[L - 1].b_off, s);
+      ph.launched();
+    } else {
+      hs::launch_softmax_xent(c->d_logits, c->Cp, y, c->fused_sync ? c->d_scale_fused : c->d_scale, c->N, c->C,
+                              c->delta_buf(L - 1), c->Cp, true,
+                              c->d_ce, c->d_status, s);
+      if (loss_bias)   // the output layer's bias gradients in the same launch
+        hs::launch_loss_bias_reduce(c->d_ce, c->d_offsets, c->M, c->d_w, c->d_lm, c->d_status, c->d_ticket,
+                                    delta_out, c->delta_ld(L - 1), c->C, c->d_slabs, c->Ps, c->layers[L - 1].b_off, s);
+      else
+        hs::launch_loss_reduce(c->d_ce, c->d_offsets, c->M, c->d_w, c->d_lm, c->d_status, c->d_ticket, s);
+      ph.launched(2);
+    }
   }
   // Per-worker weight gradients averaged tile by tile in tensor memory, the update fused in: the
   // default where the layer's operands allow it; debug read-back, the slab-free formulation and

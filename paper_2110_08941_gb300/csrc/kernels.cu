@@ -306,6 +306,125 @@ void launch_loss_bias_reduce(const float* ce, const int32_t* d_offsets, int M, c
              slabs, Ps, b_off);
 }
 
+// Softmax cross-entropy, per-worker loss and the output layer's per-worker bias gradient in one
+// launch, for at most 16 classes with bf16 delta (ldl % 4 == 0, ldd % 8 == 0, ldd <= 16): one block
+// per worker, one thread per row of it (rows b + t, b + t + blockDim, ...).  Each row takes the
+// arithmetic of softmax_xent (max, exp once per entry, ce = lse - z_y, delta_j = (e_j / se - [j = y])
+// * scale_i, columns C..ldd-1 zero); then L_m = mean of the block's ce (per-thread sums, a tree) and
+// the bias sums of the stored bf16 delta per class (each thread's rows in order, a warp xor tree,
+// the warps' sums in warp order), deterministic; the last block forms sum_m w_m L_m as
+// loss_reduce does.
+constexpr int kSlbThreads = 512;
+constexpr int kSlbMaxC = 16;
+
+__global__ void __launch_bounds__(kSlbThreads) softmax_loss_bias_kernel(
+    const float* __restrict__ logits, int ldl, const int32_t* __restrict__ y, const float* __restrict__ scale, int C,
+    __nv_bfloat16* __restrict__ delta, int ldd, float* __restrict__ ce, const int32_t* __restrict__ offsets, int M,
+    const float* __restrict__ w, float* __restrict__ lm, DevStatus* st, unsigned int* ticket,
+    float* __restrict__ slabs, int64_t Ps, int64_t b_off) {
+  pdl_wait();
+  pdl_trigger();
+  __shared__ float red[kSlbThreads];
+  __shared__ float bred[kSlbThreads / 32][kSlbMaxC];
+  __shared__ bool last;
+  const int m = blockIdx.x;
+  const int b = offsets[m], e = offsets[m + 1];
+  float lacc = 0.f;
+  float bsum[kSlbMaxC];
+#pragma unroll
+  for (int j = 0; j < kSlbMaxC; ++j) bsum[j] = 0.f;
+  for (int i = b + (int)threadIdx.x; i < e; i += blockDim.x) {
+    const float* zr = logits + (int64_t)i * ldl;
+    float z[kSlbMaxC];
+#pragma unroll
+    for (int q = 0; q < kSlbMaxC / 4; ++q) {
+      float4 v = make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY);
+      if (4 * q < C) v = __ldg(reinterpret_cast<const float4*>(zr + 4 * q));
+      z[4 * q] = v.x;
+      z[4 * q + 1] = (4 * q + 1 < C) ? v.y : -INFINITY;
+      z[4 * q + 2] = (4 * q + 2 < C) ? v.z : -INFINITY;
+      z[4 * q + 3] = (4 * q + 3 < C) ? v.w : -INFINITY;
+    }
+    int label = y[i];
+    if (label < 0 || label >= C) {
+      record_error(st, kDevBadLabel, i);
+      label = label < 0 ? 0 : C - 1;
+    }
+    float mx = -INFINITY;
+#pragma unroll
+    for (int j = 0; j < kSlbMaxC; ++j) mx = fmaxf(mx, z[j]);
+    float se = 0.f;
+#pragma unroll
+    for (int j = 0; j < kSlbMaxC; ++j) {
+      z[j] = (j < C) ? expf(z[j] - mx) : 0.f;
+      se += z[j];
+    }
+    const float cei = mx + logf(se) - __ldg(zr + label);
+    ce[i] = cei;
+    lacc += cei;
+    const float inv = 1.0f / se;
+    const float sc = scale[i];
+    uint32_t pk[kSlbMaxC / 2];
+#pragma unroll
+    for (int j = 0; j < kSlbMaxC; j += 2) {
+      const float d0 = (j < C) ? (z[j] * inv - (j == label ? 1.f : 0.f)) * sc : 0.f;
+      const float d1 = (j + 1 < C) ? (z[j + 1] * inv - (j + 1 == label ? 1.f : 0.f)) * sc : 0.f;
+      const __nv_bfloat162 q = __floats2bfloat162_rn(d0, d1);
+      bsum[j] += __low2float(q);
+      bsum[j + 1] += __high2float(q);
+      pk[j / 2] = *reinterpret_cast<const uint32_t*>(&q);
+    }
+    uint4* drow = reinterpret_cast<uint4*>(delta + (int64_t)i * ldd);
+    drow[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+    if (ldd > 8) drow[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+  }
+  red[threadIdx.x] = lacc;
+  __syncthreads();
+  for (int h = blockDim.x >> 1; h > 0; h >>= 1) {
+    if (threadIdx.x < h) red[threadIdx.x] += red[threadIdx.x + h];
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) {
+    lm[m] = red[0] / (float)(e - b);
+    __threadfence();
+    last = (atomicAdd(ticket, 1u) == (unsigned int)(M - 1));
+  }
+  const int warp = (int)threadIdx.x >> 5, lane = (int)threadIdx.x & 31;
+#pragma unroll
+  for (int j = 0; j < kSlbMaxC; ++j) {
+    float v = bsum[j];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    if (lane == 0) bred[warp][j] = v;
+  }
+  __syncthreads();
+  if ((int)threadIdx.x < C) {
+    float t = 0.f;
+    for (int v = 0; v < kSlbThreads / 32; ++v) t += bred[v][threadIdx.x];
+    slabs[(int64_t)m * Ps + b_off + threadIdx.x] = t;
+  }
+  if (last && threadIdx.x == 0) {
+    __threadfence();
+    const volatile float* lmv = lm;
+    float loss = 0.f;
+    for (int k = 0; k < M; ++k) loss += w[k] * lmv[k];
+    st->loss = loss;
+    *ticket = 0u;
+  }
+}
+
+bool softmax_loss_bias_ok(int C, int ldl, int ldd) {
+  return C <= kSlbMaxC && ldd <= kSlbMaxC && ldd % 8 == 0 && ldl % 4 == 0 && C <= ldd && C <= ldl;
+}
+
+void launch_softmax_loss_bias(const float* logits, int ldl, const int32_t* y, const float* scale, int C,
+                              __nv_bfloat16* delta, int ldd, float* ce, const int32_t* d_offsets, int M,
+                              const float* d_w, float* lm, DevStatus* st, unsigned int* ticket, float* slabs,
+                              int64_t Ps, int64_t b_off, cudaStream_t s) {
+  launch_pdl(softmax_loss_bias_kernel, M, kSlbThreads, 0, s, logits, ldl, y, scale, C, delta, ldd, ce, d_offsets, M,
+             d_w, lm, st, ticket, slabs, Ps, b_off);
+}
+
 // ------------------------------------------------------------------ per-worker bias gradient
 // G_m[b_l][j] = sum_{i in seg_m} delta_l[i][j]: one thread per column, rows in order.
 template <bool kBf16>
