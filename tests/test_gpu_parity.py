@@ -125,6 +125,10 @@ EDGE = [
     ((136, 264, 136, 1000), 517, 7, [0.3, 2.0, 1.0, 1.0, 0.7, 4.0, 0.01]),
     ((32, 8), 130, 1, None),
     ((40, 48, 56, 9), 257, 40, None),
+    # 16 classes (the widest output whose softmax, loss and bias gradient run in one launch), a
+    # worker of more than 512 rows; 23 classes (the loss reduction with the bias gradient)
+    ((40, 24, 16), 1100, 2, [1.0, 3.0]),
+    ((40, 24, 23), 300, 3, None),
 ]
 
 
